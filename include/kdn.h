@@ -1,0 +1,170 @@
+/*
+ * kdn.h -- C ABI of the GB300 (sm_103a) Kalman Delta Network token-mixer
+ * library (libkdn.so).
+ *
+ * Operations (all from "Kalman Delta Networks"):
+ *   kdn_diag_fwd / kdn_iso_fwd
+ *       Chunked prefill / training forward of the Diagonal KDN (Prop. 3) and
+ *       the Isotropic KDN (Prop. 5; App. E): the Moebius uncertainty scan
+ *       (eq. kla-box-mobius, eq. iso-kla-box-mobius), the Kalman gain emitted
+ *       from the pre-write predictive variance (eq. kla-box-gain,
+ *       eq. iso-kla-box-gain, App. F.1 eq. chunk-gain-emission) and the
+ *       asymmetric delta-rule memory scan in compact-WY form (App. F.2,
+ *       eq. chunk-memory-wy and eq. chunk-memory-output-state).
+ *   kdn_diag_bwd / kdn_iso_bwd
+ *       Gradients of the forward.  The paper gives no backward; these are
+ *       the exact adjoints of the forward recurrence.
+ *   kdn_diag_decode_step / kdn_iso_decode_step
+ *       One token of the recurrence (the boxed update of Prop. 3 / Prop. 5)
+ *       applied in place to a batch of states.
+ *
+ * Per token t and head h the layer computes, with alpha_t = exp(g_t):
+ *   Diagonal:  phat = alpha^2 p + omega;  kappa = phat k / (r + sum phat k^2)
+ *              u = mu k^2 / r;            p' = phat / (1 + u phat)
+ *   Isotropic: a = mean_i alpha_i^2 (alpha^2 for scalar decay);
+ *              bhat = a b + omega;  beta = bhat / (r + bhat |k|^2); kappa = beta k
+ *              u = mu |k|^2 / (d_k r); b' = bhat / (1 + u bhat)
+ *   Memory:    S' = (I - kappa k^T) diag(alpha) S + kappa v^T;  o = scale * S'^T q
+ *
+ * Conventions
+ *   Ownership  The caller owns every buffer, device and host.  Entry points
+ *              allocate no memory (scratch lives in the caller's workspace),
+ *              keep no global state between calls and are reentrant.
+ *   Pointers   Device pointers unless stated otherwise, 16-byte aligned.
+ *   Streams    `stream` is a cudaStream_t passed as void* (NULL = the legacy
+ *              default stream).  Every call is asynchronous on that stream.
+ *   Errors     Argument errors are detected before anything is launched and
+ *              leave all outputs untouched.  A failed launch returns
+ *              KDN_ERR_CUDA.
+ *   Inputs     q, k, v, g, omega, r are post-activation values: g = log(alpha)
+ *              <= 0 (alpha = sigmoid(.) in the paper), omega > 0, r > 0.  The
+ *              library does not normalise q or k and applies no gate
+ *              activation.
+ *   Layouts    (row-major, last index fastest)
+ *              q, k            [B, T, H, dk]        v, o, dO      [B, T, H, dv]
+ *              r               [B, T, H]
+ *              diag: g, omega  [B, T, H, dk]
+ *              iso:  omega     [B, T, H];  g [B, T, H, dk] (decay_per_channel=1)
+ *                                           or [B, T, H]     (decay_per_channel=0)
+ *              S0, ST, dST, dS0 (float32)   [B, H, dk, dv]
+ *              p0, pT, dpT, dp0 (float32)   diag [B, H, dk];  iso [B, H]
+ *              Gradients have the layout of the input they belong to.
+ *   Dtypes     q, k, v, g, omega, r, o, dO and the input gradients share
+ *              desc->dtype (float32 or bfloat16).  State is always float32;
+ *              all arithmetic is float32.
+ *   Sizes      dk, dv in {32, 64, 128}; T >= 0 (any length; a ragged last
+ *              chunk is padded with identity tokens); B, H >= 0.
+ */
+#ifndef KDN_H
+#define KDN_H
+
+#include <stddef.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  KDN_OK = 0,
+  KDN_ERR_INVALID_ARG = 1, /* null / misaligned pointer, bad size or field */
+  KDN_ERR_UNSUPPORTED = 2, /* valid but not built (e.g. dk = 96) */
+  KDN_ERR_WORKSPACE = 3,   /* workspace missing or smaller than required */
+  KDN_ERR_CUDA = 4,        /* a CUDA launch or runtime call failed */
+  KDN_ERR_TIMEOUT = 5      /* a bounded device-side wait gave up */
+} kdn_status_t;
+
+typedef enum { KDN_F32 = 0, KDN_BF16 = 1 } kdn_dtype_t;
+
+typedef struct {
+  int B, T, H;           /* batch, tokens, heads */
+  int dk, dv;            /* key and value head dimensions */
+  int chunk;             /* memory-chunk length C_m of App. F.2: 0 (= 64), 32 or 64;
+                            a tuning choice, results agree to rounding */
+  int dtype;             /* kdn_dtype_t of activations and their gradients */
+  float mu;              /* information scale of eq. diag-cov-update; <= 0 -> dk */
+  float scale;           /* query scale tau of App. F.2; NaN -> 1/sqrt(dk) */
+  int decay_per_channel; /* isotropic only: 1 -> g is [B,T,H,dk], 0 -> [B,T,H].
+                            Ignored by the diagonal variant (always per channel). */
+  int out_dtype;         /* kdn_dtype_t of o and of dq, dk, dv, dg, domega, dr.
+                            0 (KDN_F32, the zero-initialised default) keeps the
+                            float32 accumulators; KDN_BF16 rounds them once on
+                            store. */
+} kdn_desc_t;
+
+/* Library version as major*10000 + minor*100 + patch. */
+int kdn_version(void);
+
+/* Human-readable name of a status code (static string, never NULL). */
+const char *kdn_status_string(kdn_status_t status);
+
+/* Workspace (device scratch) bytes that kdn_*_fwd / kdn_*_bwd need for this
+   descriptor; variant 0 = diagonal, 1 = isotropic.  Returns 0 for an invalid
+   descriptor.  The workspace must be 256-byte aligned; its contents need no
+   initialisation and are clobbered by every call. */
+size_t kdn_fwd_workspace_bytes(const kdn_desc_t *desc, int variant);
+size_t kdn_bwd_workspace_bytes(const kdn_desc_t *desc, int variant);
+
+/* Forward over T tokens (Prop. 3, App. F).
+   S0 NULL -> zero initial memory; p0 NULL -> unit initial uncertainty
+   (z_0 = [p_0, 1] of eq. chunk-gain-carry with p_0 = 1).
+   ST / pT NULL -> final state not written.  o is always written. */
+kdn_status_t kdn_diag_fwd(const kdn_desc_t *desc, const void *q, const void *k,
+                          const void *v, const void *g, const void *omega,
+                          const void *r, const float *S0, const float *p0,
+                          void *o, float *ST, float *pT, void *workspace,
+                          size_t workspace_bytes, void *stream);
+
+/* Forward of the Isotropic KDN (Prop. 5, App. E); p0 / pT are b_0 / b_T [B,H]. */
+kdn_status_t kdn_iso_fwd(const kdn_desc_t *desc, const void *q, const void *k,
+                         const void *v, const void *g, const void *omega,
+                         const void *r, const float *S0, const float *p0,
+                         void *o, float *ST, float *pT, void *workspace,
+                         size_t workspace_bytes, void *stream);
+
+/* Backward: gradients of <dO, o> + <dST, ST> + <dpT, pT> with respect to every
+   forward input.  It recomputes the forward from the inputs (no saved
+   context).  dST / dpT NULL -> zero cotangent.  dS0 / dp0 NULL -> not written;
+   all other gradient pointers are required. */
+kdn_status_t kdn_diag_bwd(const kdn_desc_t *desc, const void *q, const void *k,
+                          const void *v, const void *g, const void *omega,
+                          const void *r, const float *S0, const float *p0,
+                          const void *dO, const float *dST, const float *dpT,
+                          void *dq, void *dk, void *dv, void *dg, void *domega,
+                          void *dr, float *dS0, float *dp0, void *workspace,
+                          size_t workspace_bytes, void *stream);
+
+kdn_status_t kdn_iso_bwd(const kdn_desc_t *desc, const void *q, const void *k,
+                         const void *v, const void *g, const void *omega,
+                         const void *r, const float *S0, const float *p0,
+                         const void *dO, const float *dST, const float *dpT,
+                         void *dq, void *dk, void *dv, void *dg, void *domega,
+                         void *dr, float *dS0, float *dp0, void *workspace,
+                         size_t workspace_bytes, void *stream);
+
+/* One decode token for all B*H heads (the update of Prop. 3), in place:
+   S [B,H,dk,dv] and p [B,H,dk] are read and overwritten; o [B,H,dv] is
+   written.  Per-step inputs drop the T axis: q, k [B,H,dk], v [B,H,dv],
+   g, omega [B,H,dk], r [B,H].  desc->T is ignored.  Needs no workspace. */
+kdn_status_t kdn_diag_decode_step(const kdn_desc_t *desc, const void *q,
+                                  const void *k, const void *v, const void *g,
+                                  const void *omega, const void *r, float *S,
+                                  float *p, void *o, void *stream);
+
+/* Isotropic decode step (Prop. 5): p is b [B,H]; omega [B,H];
+   g [B,H,dk] or [B,H] per desc->decay_per_channel. */
+kdn_status_t kdn_iso_decode_step(const kdn_desc_t *desc, const void *q,
+                                 const void *k, const void *v, const void *g,
+                                 const void *omega, const void *r, float *S,
+                                 float *p, void *o, void *stream);
+
+/* Synchronises `stream`, then returns and clears the device status word kept
+   in the first bytes of `workspace`: KDN_OK, or KDN_ERR_TIMEOUT when a bounded
+   device-side wait of the most recent kdn_*_fwd / kdn_*_bwd call on that
+   workspace gave up.  Each of those calls clears the word before it starts. */
+kdn_status_t kdn_get_device_status(void *workspace, void *stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* KDN_H */

@@ -1,0 +1,243 @@
+"""GB300 (sm_103a) Kalman Delta Network token mixers.
+
+Thin Python binding of ``libkdn.so`` (C ABI in ``include/kdn.h``).  The
+functions below carry the C entry points' names and only marshal arguments:
+they allocate outputs and the scratch workspace with PyTorch (device memory is
+PyTorch's job here), pass raw pointers and the current CUDA stream, and raise
+on any non-OK status.  Every step of the computation runs in the library's
+CUDA kernels; there is no CPU or PyTorch fallback, and importing a function
+whose library is missing raises.
+
+Layouts follow the C ABI: q, k [B,T,H,dk]; v [B,T,H,dv]; r [B,T,H];
+diag g, omega [B,T,H,dk]; iso omega [B,T,H], g [B,T,H,dk] or [B,T,H];
+S0 [B,H,dk,dv] float32; p0 diag [B,H,dk], iso [B,H] float32.
+"""
+from __future__ import annotations
+
+import ctypes
+import math
+import os
+import threading
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libkdn.so")
+
+KDN_OK, KDN_ERR_INVALID_ARG, KDN_ERR_UNSUPPORTED, KDN_ERR_WORKSPACE, KDN_ERR_CUDA, \
+    KDN_ERR_TIMEOUT = range(6)
+KDN_F32, KDN_BF16 = 0, 1
+
+_DTYPES = {torch.float32: KDN_F32, torch.bfloat16: KDN_BF16}
+
+
+class kdn_desc_t(ctypes.Structure):
+    _fields_ = [("B", ctypes.c_int), ("T", ctypes.c_int), ("H", ctypes.c_int),
+                ("dk", ctypes.c_int), ("dv", ctypes.c_int), ("chunk", ctypes.c_int),
+                ("dtype", ctypes.c_int), ("mu", ctypes.c_float), ("scale", ctypes.c_float),
+                ("decay_per_channel", ctypes.c_int), ("out_dtype", ctypes.c_int)]
+
+
+class KdnError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__(f"{where}: {status_string(status)}")
+
+
+_lib = None
+_lock = threading.Lock()
+
+_P = ctypes.c_void_p
+_SIG = {
+    "kdn_version": ([], ctypes.c_int),
+    "kdn_status_string": ([ctypes.c_int], ctypes.c_char_p),
+    "kdn_fwd_workspace_bytes": ([ctypes.POINTER(kdn_desc_t), ctypes.c_int], ctypes.c_size_t),
+    "kdn_bwd_workspace_bytes": ([ctypes.POINTER(kdn_desc_t), ctypes.c_int], ctypes.c_size_t),
+    "kdn_diag_fwd": ([ctypes.POINTER(kdn_desc_t)] + [_P] * 12 + [ctypes.c_size_t, _P], ctypes.c_int),
+    "kdn_iso_fwd": ([ctypes.POINTER(kdn_desc_t)] + [_P] * 12 + [ctypes.c_size_t, _P], ctypes.c_int),
+    "kdn_diag_bwd": ([ctypes.POINTER(kdn_desc_t)] + [_P] * 20 + [ctypes.c_size_t, _P], ctypes.c_int),
+    "kdn_iso_bwd": ([ctypes.POINTER(kdn_desc_t)] + [_P] * 20 + [ctypes.c_size_t, _P], ctypes.c_int),
+    "kdn_diag_decode_step": ([ctypes.POINTER(kdn_desc_t)] + [_P] * 10, ctypes.c_int),
+    "kdn_iso_decode_step": ([ctypes.POINTER(kdn_desc_t)] + [_P] * 10, ctypes.c_int),
+    "kdn_get_device_status": ([_P, _P], ctypes.c_int),
+}
+EXPORTED = tuple(_SIG)
+
+
+def lib():
+    """The loaded ``libkdn.so`` (ctypes), built beforehand by ``build.build()``."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            if not os.path.exists(LIB_PATH):
+                raise RuntimeError(f"{LIB_PATH} is missing: run paper_2609_07816_gb300.build."
+                                   "build() first (there is no fallback implementation)")
+            L = ctypes.CDLL(LIB_PATH)
+            for name, (args, res) in _SIG.items():
+                fn = getattr(L, name)
+                fn.argtypes = args
+                fn.restype = res
+            _lib = L
+    return _lib
+
+
+def status_string(status: int) -> str:
+    return lib().kdn_status_string(int(status)).decode()
+
+
+def _check(status: int, where: str):
+    if status != KDN_OK:
+        raise KdnError(status, where)
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    s = torch.cuda.current_stream() if stream is None else stream
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _code(dtype):
+    return _DTYPES[dtype] if isinstance(dtype, torch.dtype) else int(dtype)
+
+
+def make_desc(B, T, H, dk, dv, dtype, *, chunk=0, mu=None, scale=None,
+              decay_per_channel=1, out_dtype=KDN_F32) -> kdn_desc_t:
+    return kdn_desc_t(B, T, H, dk, dv, chunk, _code(dtype), 0.0 if mu is None else float(mu),
+                      math.nan if scale is None else float(scale), int(decay_per_channel),
+                      _code(out_dtype))
+
+
+def _desc_from(variant, q, v, g, *, chunk, mu, scale, out_dtype):
+    B, T, H, dk = q.shape
+    dv = v.shape[-1]
+    pcd = 1 if variant == 0 else int(g.dim() == 4)
+    return make_desc(B, T, H, dk, dv, q.dtype, chunk=chunk, mu=mu, scale=scale,
+                     decay_per_channel=pcd, out_dtype=out_dtype)
+
+
+def workspace_bytes(desc: kdn_desc_t, variant: int, backward: bool = False) -> int:
+    fn = lib().kdn_bwd_workspace_bytes if backward else lib().kdn_fwd_workspace_bytes
+    return int(fn(ctypes.byref(desc), int(variant)))
+
+
+def alloc_workspace(desc, variant, backward=False, device=None):
+    n = workspace_bytes(desc, variant, backward)
+    return torch.empty(max(n, 256), dtype=torch.uint8, device=device or "cuda")
+
+
+def _fwd(name, variant, q, k, v, g, omega, r, S0, p0, *, chunk, mu, scale, o, ST, pT,
+         want_state, workspace, stream, out_dtype):
+    desc = _desc_from(variant, q, v, g, chunk=chunk, mu=mu, scale=scale, out_dtype=out_dtype)
+    B, T, H, dk = q.shape
+    dv = v.shape[-1]
+    dev = q.device
+    if o is None:
+        o = torch.empty(B, T, H, dv, dtype=out_dtype, device=dev)
+    if want_state and ST is None:
+        ST = torch.empty(B, H, dk, dv, dtype=torch.float32, device=dev)
+    if want_state and pT is None:
+        pT = torch.empty((B, H, dk) if variant == 0 else (B, H), dtype=torch.float32, device=dev)
+    if workspace is None:
+        workspace = alloc_workspace(desc, variant, False, dev)
+    st = getattr(lib(), name)(ctypes.byref(desc), _ptr(q), _ptr(k), _ptr(v), _ptr(g),
+                              _ptr(omega), _ptr(r), _ptr(S0), _ptr(p0), _ptr(o), _ptr(ST),
+                              _ptr(pT), _ptr(workspace), workspace.numel(), _stream(stream))
+    _check(st, name)
+    return o, ST, pT
+
+
+def kdn_diag_fwd(q, k, v, g, omega, r, S0=None, p0=None, *, chunk=0, mu=None, scale=None,
+                 o=None, ST=None, pT=None, want_state=True, workspace=None, stream=None,
+                 out_dtype=torch.float32):
+    """Diagonal KDN forward (Prop. 3).  Returns (o, ST, pT)."""
+    return _fwd("kdn_diag_fwd", 0, q, k, v, g, omega, r, S0, p0, chunk=chunk, mu=mu,
+                scale=scale, o=o, ST=ST, pT=pT, want_state=want_state, workspace=workspace,
+                stream=stream, out_dtype=out_dtype)
+
+
+def kdn_iso_fwd(q, k, v, g, omega, r, S0=None, p0=None, *, chunk=0, mu=None, scale=None,
+                o=None, ST=None, pT=None, want_state=True, workspace=None, stream=None,
+                 out_dtype=torch.float32):
+    """Isotropic KDN forward (Prop. 5).  g [B,T,H,dk] = per-channel decay, [B,T,H] = scalar."""
+    return _fwd("kdn_iso_fwd", 1, q, k, v, g, omega, r, S0, p0, chunk=chunk, mu=mu,
+                scale=scale, o=o, ST=ST, pT=pT, want_state=want_state, workspace=workspace,
+                stream=stream, out_dtype=out_dtype)
+
+
+def _bwd(name, variant, q, k, v, g, omega, r, S0, p0, dO, dST, dpT, *, chunk, mu, scale,
+         grads, want_state_grads, workspace, stream, out_dtype):
+    desc = _desc_from(variant, q, v, g, chunk=chunk, mu=mu, scale=scale, out_dtype=out_dtype)
+    B, T, H, dk = q.shape
+    dv = v.shape[-1]
+    dev = q.device
+    if grads is None:
+        grads = {n: torch.empty(x.shape, dtype=out_dtype, device=dev) for n, x in
+                 (("dq", q), ("dk", k), ("dv", v), ("dg", g), ("domega", omega), ("dr", r))}
+        if want_state_grads:
+            grads["dS0"] = torch.empty(B, H, dk, dv, dtype=torch.float32, device=dev)
+            grads["dp0"] = torch.empty((B, H, dk) if variant == 0 else (B, H),
+                                       dtype=torch.float32, device=dev)
+    if workspace is None:
+        workspace = alloc_workspace(desc, variant, True, dev)
+    G = grads
+    st = getattr(lib(), name)(ctypes.byref(desc), _ptr(q), _ptr(k), _ptr(v), _ptr(g),
+                              _ptr(omega), _ptr(r), _ptr(S0), _ptr(p0), _ptr(dO), _ptr(dST),
+                              _ptr(dpT), _ptr(G["dq"]), _ptr(G["dk"]), _ptr(G["dv"]),
+                              _ptr(G["dg"]), _ptr(G["domega"]), _ptr(G["dr"]),
+                              _ptr(G.get("dS0")), _ptr(G.get("dp0")), _ptr(workspace),
+                              workspace.numel(), _stream(stream))
+    _check(st, name)
+    return grads
+
+
+def kdn_diag_bwd(q, k, v, g, omega, r, S0, p0, dO, dST=None, dpT=None, *, chunk=0, mu=None,
+                 scale=None, grads=None, want_state_grads=True, workspace=None, stream=None,
+                 out_dtype=torch.float32):
+    """Gradients of the Diagonal KDN forward.  Returns a dict dq, dk, dv, dg, domega, dr, dS0, dp0."""
+    return _bwd("kdn_diag_bwd", 0, q, k, v, g, omega, r, S0, p0, dO, dST, dpT, chunk=chunk,
+                mu=mu, scale=scale, grads=grads, want_state_grads=want_state_grads,
+                workspace=workspace, stream=stream, out_dtype=out_dtype)
+
+
+def kdn_iso_bwd(q, k, v, g, omega, r, S0, p0, dO, dST=None, dpT=None, *, chunk=0, mu=None,
+                scale=None, grads=None, want_state_grads=True, workspace=None, stream=None,
+                 out_dtype=torch.float32):
+    """Gradients of the Isotropic KDN forward."""
+    return _bwd("kdn_iso_bwd", 1, q, k, v, g, omega, r, S0, p0, dO, dST, dpT, chunk=chunk,
+                mu=mu, scale=scale, grads=grads, want_state_grads=want_state_grads,
+                workspace=workspace, stream=stream, out_dtype=out_dtype)
+
+
+def _decode(name, variant, q, k, v, g, omega, r, S, p, *, mu, scale, o, stream, out_dtype):
+    B, H, dk = q.shape
+    dv = v.shape[-1]
+    pcd = 1 if variant == 0 else int(g.dim() == 3)
+    desc = make_desc(B, 1, H, dk, dv, q.dtype, mu=mu, scale=scale, decay_per_channel=pcd,
+                     out_dtype=out_dtype)
+    if o is None:
+        o = torch.empty(B, H, dv, dtype=out_dtype, device=q.device)
+    st = getattr(lib(), name)(ctypes.byref(desc), _ptr(q), _ptr(k), _ptr(v), _ptr(g),
+                              _ptr(omega), _ptr(r), _ptr(S), _ptr(p), _ptr(o), _stream(stream))
+    _check(st, name)
+    return o
+
+
+def kdn_diag_decode_step(q, k, v, g, omega, r, S, p, *, mu=None, scale=None, o=None,
+                         stream=None, out_dtype=torch.float32):
+    """One Diagonal KDN token for every head, S [B,H,dk,dv] and p [B,H,dk] updated in place."""
+    return _decode("kdn_diag_decode_step", 0, q, k, v, g, omega, r, S, p, mu=mu, scale=scale,
+                   o=o, stream=stream, out_dtype=out_dtype)
+
+
+def kdn_iso_decode_step(q, k, v, g, omega, r, S, p, *, mu=None, scale=None, o=None,
+                        stream=None, out_dtype=torch.float32):
+    """One Isotropic KDN token for every head; g [B,H,dk] or [B,H]; p [B,H] in place."""
+    return _decode("kdn_iso_decode_step", 1, q, k, v, g, omega, r, S, p, mu=mu, scale=scale,
+                   o=o, stream=stream, out_dtype=out_dtype)
+
+
+def kdn_get_device_status(workspace, stream=None) -> int:
+    return int(lib().kdn_get_device_status(_ptr(workspace), _stream(stream)))

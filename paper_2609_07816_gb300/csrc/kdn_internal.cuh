@@ -1,0 +1,99 @@
+// kdn_internal.cuh -- internal types and device helpers shared by the CUDA
+// translation units of libkdn.so.  Not part of the public ABI (include/kdn.h).
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/kdn.h"
+
+namespace kdn {
+
+// ---------------------------------------------------------------------------
+// dtype helpers: activations are float32 or bfloat16, arithmetic is float32.
+
+template <typename DT> __device__ __forceinline__ float ld(const void *p, size_t i);
+template <> __device__ __forceinline__ float ld<float>(const void *p, size_t i) {
+  return static_cast<const float *>(p)[i];
+}
+template <> __device__ __forceinline__ float ld<__nv_bfloat16>(const void *p, size_t i) {
+  return __bfloat162float(static_cast<const __nv_bfloat16 *>(p)[i]);
+}
+template <typename DT> __device__ __forceinline__ void st(void *p, size_t i, float x);
+template <> __device__ __forceinline__ void st<float>(void *p, size_t i, float x) {
+  static_cast<float *>(p)[i] = x;
+}
+template <> __device__ __forceinline__ void st<__nv_bfloat16>(void *p, size_t i, float x) {
+  static_cast<__nv_bfloat16 *>(p)[i] = __float2bfloat16_rn(x);
+}
+
+// Output store in the caller's output dtype (a uniform runtime choice).
+__device__ __forceinline__ void sto(int odt, void *p, size_t i, float x) {
+  if (odt == KDN_BF16) static_cast<__nv_bfloat16 *>(p)[i] = __float2bfloat16_rn(x);
+  else static_cast<float *>(p)[i] = x;
+}
+
+__device__ __forceinline__ float warp_sum(float x) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+  return x;
+}
+
+// ---------------------------------------------------------------------------
+// Internal argument bundle: everything an entry point received, plus derived
+// sizes and the carve-up of the caller's workspace.
+
+struct Args {
+  int variant;  // 0 diagonal, 1 isotropic
+  int B, T, H, dk, dv;
+  int C;        // memory chunk length used by the kernels
+  int NC, Tp;   // number of chunks, padded length NC*C
+  int P;        // uncertainty entries per head: dk (diag) or 1 (iso)
+  int pcd;      // decay has a channel axis (g is [..,dk])
+  int dtype;
+  int odt;      // dtype of o and of the input gradients
+  float mu, tau;
+  // forward inputs / outputs
+  const void *q, *k, *v, *g, *omega, *r;
+  const float *S0, *p0;
+  void *o;
+  float *ST, *pT;
+  // backward inputs / outputs
+  const void *dO;
+  const float *dST, *dpT;
+  void *dq, *dk_, *dv_, *dg, *domega, *dr;
+  float *dS0, *dp0;
+  // workspace regions (float32 unless noted)
+  unsigned *status;
+  float *phat;    // [BH][Tp][P]   predictive variance phat_t (pre-write)
+  float *isotok;  // [BH][Tp][2]   isotropic: a_t, |k_t|^2
+  float *W, *U;   // [BH][NC][C][dk], [BH][NC][C][dv]
+  float *Qb;      // [BH][NC][C][dk]
+  float *Aqk;     // [BH][NC][C][C]
+  float *Kt;      // [BH][NC][C][dk]
+  float *gC;      // [BH][NC][dk]   gamma_C
+  float *Sin;     // [BH][NC][dk][dv] chunk-entry memory (backward)
+  float *dSout;   // [BH][NC][dk][dv] cotangent of the chunk-exit memory
+  float *dR;      // [BH][NC][C][dv]
+  float *dkpart;  // [BH][Tp][dk]
+  float *dgpart;  // [BH][Tp][dk]
+  float *dphloc;  // [BH][Tp][P]
+  float *drpart;  // [BH][Tp]
+  float *drw;     // [BH][Tp][4]
+  float *isoadj;  // [BH][Tp][2]
+};
+
+__host__ __device__ inline size_t tok_index(const Args &a, int b, int t, int h) {
+  return ((size_t)b * a.T + t) * a.H + h;
+}
+
+// Workspace carve-up; returns total bytes.  `bwd` adds the backward regions.
+size_t workspace_layout(Args *a, char *base, bool bwd);
+
+// Launchers (each returns KDN_OK or KDN_ERR_CUDA).
+kdn_status_t launch_chunked_fwd(const Args &a, cudaStream_t s, bool save_states);
+kdn_status_t launch_chunked_bwd(const Args &a, cudaStream_t s);
+kdn_status_t launch_decode(const Args &a, float *S, float *p, cudaStream_t s);
+
+}  // namespace kdn

@@ -1,0 +1,137 @@
+"""C ABI checks that need no GPU: the library builds and loads, exports every
+entry point that include/kdn.h declares, sizes workspaces, and rejects bad
+arguments before any CUDA call is made."""
+import ctypes
+import math
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def kdn():
+    from paper_2609_07816_gb300 import build
+    build.build()
+    import paper_2609_07816_gb300 as m
+    return m
+
+
+def _header_functions():
+    text = open(os.path.join(ROOT, "include", "kdn.h")).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(kdn_[a-z_0-9]+)\s*\(", text)))
+
+
+def test_exports_every_declared_symbol(kdn):
+    names = _header_functions()
+    assert len(names) >= 11
+    L = ctypes.CDLL(kdn.LIB_PATH)
+    for n in names:
+        assert hasattr(L, n), n
+    assert set(names) == set(kdn.EXPORTED)
+
+
+def test_version_and_status_strings(kdn):
+    assert kdn.lib().kdn_version() >= 100
+    for code, name in enumerate(["KDN_OK", "KDN_ERR_INVALID_ARG", "KDN_ERR_UNSUPPORTED",
+                                 "KDN_ERR_WORKSPACE", "KDN_ERR_CUDA", "KDN_ERR_TIMEOUT"]):
+        assert kdn.status_string(code) == name
+    assert kdn.status_string(99) == "KDN_ERR_UNKNOWN"
+
+
+def test_workspace_sizes(kdn):
+    d = kdn.make_desc(2, 100, 3, 64, 32, kdn.KDN_BF16)
+    f0, b0 = kdn.workspace_bytes(d, 0), kdn.workspace_bytes(d, 0, True)
+    f1 = kdn.workspace_bytes(d, 1)
+    assert 0 < f0 < b0 and f1 > 0
+    assert f0 % 256 == 0 and b0 % 256 == 0
+    bad = kdn.make_desc(2, 100, 3, 96, 32, kdn.KDN_BF16)
+    assert kdn.workspace_bytes(bad, 0) == 0
+    # workspace grows linearly in T (per-chunk intermediates)
+    d2 = kdn.make_desc(2, 200, 3, 64, 32, kdn.KDN_BF16)
+    assert kdn.workspace_bytes(d2, 0) > f0
+
+
+FAKE = ctypes.c_void_p(1 << 20)          # 16-byte aligned, never dereferenced
+MIS = ctypes.c_void_p((1 << 20) + 4)     # misaligned
+
+
+def _fwd(kdn, desc, ptrs=None, ws=FAKE, ws_bytes=1 << 40):
+    p = ptrs or [FAKE] * 11
+    return kdn.lib().kdn_diag_fwd(ctypes.byref(desc), *p, ws, ws_bytes, None)
+
+
+def test_rejects_bad_descriptors_before_launch(kdn):
+    L = kdn.lib()
+    assert L.kdn_diag_fwd(None, *([FAKE] * 11), FAKE, 1 << 40, None) == kdn.KDN_ERR_INVALID_ARG
+    cases = [
+        (dict(dk=96), kdn.KDN_ERR_UNSUPPORTED),
+        (dict(dv=48), kdn.KDN_ERR_UNSUPPORTED),
+        (dict(dk=0), kdn.KDN_ERR_INVALID_ARG),
+        (dict(T=-1), kdn.KDN_ERR_INVALID_ARG),
+        (dict(B=-2), kdn.KDN_ERR_INVALID_ARG),
+        (dict(chunk=48), kdn.KDN_ERR_INVALID_ARG),
+        (dict(dtype=7), kdn.KDN_ERR_INVALID_ARG),
+        (dict(out_dtype=3), kdn.KDN_ERR_INVALID_ARG),
+        (dict(mu=math.nan), kdn.KDN_ERR_INVALID_ARG),
+        (dict(scale=math.inf), kdn.KDN_ERR_INVALID_ARG),
+    ]
+    for over, want in cases:
+        kw = dict(B=1, T=10, H=1, dk=32, dv=32, dtype=kdn.KDN_F32)
+        kw.update(over)
+        d = kdn.make_desc(kw["B"], kw["T"], kw["H"], kw["dk"], kw["dv"], kw["dtype"],
+                          chunk=kw.get("chunk", 0), mu=kw.get("mu"), scale=kw.get("scale"),
+                          out_dtype=kw.get("out_dtype", 0))
+        assert _fwd(kdn, d) == want, over
+
+
+def test_rejects_null_and_misaligned_pointers(kdn):
+    d = kdn.make_desc(1, 10, 1, 32, 32, kdn.KDN_F32)
+    for i in range(7):  # q, k, v, g, omega, r are required; S0, p0 optional; o required
+        idx = i if i < 6 else 8
+        p = [FAKE] * 11
+        p[idx] = None
+        assert _fwd(kdn, d, p) == kdn.KDN_ERR_INVALID_ARG, idx
+        p[idx] = MIS
+        assert _fwd(kdn, d, p) == kdn.KDN_ERR_INVALID_ARG, idx
+    p = [FAKE] * 11
+    p[6] = MIS  # optional S0 must still be aligned
+    assert _fwd(kdn, d, p) == kdn.KDN_ERR_INVALID_ARG
+
+
+def test_rejects_small_or_misaligned_workspace(kdn):
+    d = kdn.make_desc(1, 10, 1, 32, 32, kdn.KDN_F32)
+    need = kdn.workspace_bytes(d, 0)
+    assert _fwd(kdn, d, ws_bytes=need - 1) == kdn.KDN_ERR_WORKSPACE
+    assert _fwd(kdn, d, ws=None, ws_bytes=need) == kdn.KDN_ERR_WORKSPACE
+    assert _fwd(kdn, d, ws=ctypes.c_void_p((1 << 20) + 16), ws_bytes=need) == \
+        kdn.KDN_ERR_WORKSPACE
+
+
+def test_backward_and_decode_validate(kdn):
+    L = kdn.lib()
+    d = kdn.make_desc(1, 10, 1, 32, 32, kdn.KDN_BF16)
+    p = [FAKE] * 19
+    p[15] = None  # domega is required
+    assert L.kdn_iso_bwd(ctypes.byref(d), *p, FAKE, 1 << 40, None) == kdn.KDN_ERR_INVALID_ARG
+    q = [FAKE] * 9
+    q[7] = None  # p (state) is required
+    assert L.kdn_diag_decode_step(ctypes.byref(d), *q, None) == kdn.KDN_ERR_INVALID_ARG
+    bad = kdn.make_desc(1, 1, 1, 32, 40, kdn.KDN_BF16)
+    assert L.kdn_iso_decode_step(ctypes.byref(bad), *([FAKE] * 9), None) == \
+        kdn.KDN_ERR_UNSUPPORTED
+    iso = kdn.make_desc(1, 10, 1, 32, 32, kdn.KDN_BF16, decay_per_channel=3)
+    assert L.kdn_iso_fwd(ctypes.byref(iso), *([FAKE] * 11), FAKE, 1 << 40, None) == \
+        kdn.KDN_ERR_INVALID_ARG
+
+
+def test_product_package_does_not_import_oracle():
+    pkg = os.path.join(ROOT, "paper_2609_07816_gb300")
+    for dirpath, _, files in os.walk(pkg):
+        for f in files:
+            if f.endswith((".py", ".cu", ".cuh", ".h")):
+                text = open(os.path.join(dirpath, f)).read()
+                assert "oracle" not in text.lower().replace("oracle-free", ""), f

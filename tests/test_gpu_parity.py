@@ -1,0 +1,215 @@
+"""GPU parity: the CUDA path (through the C ABI) against the fp64 oracle on the
+same seeded inputs, element by element, for the forward, the backward and the
+decode step, at sizes that span several chunks and a ragged tail, plus the
+edge cases (T = 0, T = 1, zero keys, alpha = 1, state hand-off)."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from kdn_inputs import make_decode_inputs, make_inputs
+from kdn_gpu_util import check, check_stored_bf16, head_slice, to_dev, to_np
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def kdn():
+    from paper_2609_07816_gb300 import build
+    build.build()
+    import paper_2609_07816_gb300 as m
+    torch.cuda.init()
+    return m
+
+
+def _gpu_fwd(kdn, variant, d, **kw):
+    fn = kdn.kdn_diag_fwd if variant == "diag" else kdn.kdn_iso_fwd
+    return fn(d["q"], d["k"], d["v"], d["g"], d["omega"], d["r"], d["S0"], d["p0"], **kw)
+
+
+def _oracle_fwd(variant, ins, **kw):
+    return oracle.fwd(variant, *[ins[n] for n in ("q", "k", "v", "g", "omega", "r")],
+                      ins["S0"], ins["p0"], **kw)
+
+
+FWD_CASES = [
+    # variant, per-channel decay, dtype, B, T, H, dk, dv, s0_std, p0_range
+    ("diag", True, "f32", 1, 256, 2, 32, 32, 0.0, None),       # 1 GB300 parity workload (fp32)
+    ("diag", True, "f32", 2, 70, 3, 64, 32, 0.3, (0.5, 2.0)),
+    ("diag", True, "f32", 1, 100, 2, 128, 128, 0.02, (0.5, 2.0)),
+    ("diag", True, "bf16", 2, 200, 2, 128, 128, 0.0, None),
+    ("diag", True, "bf16", 1, 97, 3, 64, 128, 0.02, (0.1, 2.0)),
+    ("iso", False, "f32", 2, 90, 2, 128, 64, 0.0, None),
+    ("iso", False, "bf16", 2, 150, 3, 128, 128, 0.02, (0.5, 2.0)),
+    ("iso", True, "f32", 1, 65, 2, 32, 128, 0.1, (0.5, 2.0)),
+    ("iso", True, "bf16", 2, 129, 2, 128, 128, 0.0, None),
+]
+
+
+@pytest.mark.parametrize("case", FWD_CASES, ids=lambda c: "-".join(map(str, c[:8])))
+def test_forward_parity(kdn, case):
+    variant, pc, dt, B, T, H, dk, dv, s0, p0r = case
+    ins = make_inputs(variant, B, T, H, dk, dv, dtype=dt, seed=T + dk, s0_std=s0,
+                      p0_range=p0r, per_channel_decay=pc)
+    ref = _oracle_fwd(variant, ins)
+    o, ST, pT = _gpu_fwd(kdn, variant, to_dev(ins))
+    torch.cuda.synchronize()
+    check("o", o, ref["o"], dt)
+    check("ST", ST, ref["ST"], dt)
+    check("pT", pT, ref["pT"], dt)
+
+
+@pytest.mark.parametrize("chunk", [0, 32, 64])
+def test_forward_chunk_argument_is_tuning_only(kdn, chunk):
+    ins = make_inputs("diag", 1, 130, 2, 64, 64, dtype="f32", seed=3)
+    ref = _oracle_fwd("diag", ins)
+    o, ST, pT = _gpu_fwd(kdn, "diag", to_dev(ins), chunk=chunk)
+    check("o", o, ref["o"], "f32")
+    check("ST", ST, ref["ST"], "f32")
+
+
+BWD_CASES = [
+    ("diag", True, "f32", 1, 75, 2, 32, 32),
+    ("diag", True, "f32", 2, 64, 1, 128, 128),
+    ("diag", True, "bf16", 1, 140, 2, 128, 128),
+    ("iso", False, "f32", 2, 50, 2, 64, 32),
+    ("iso", False, "bf16", 1, 100, 2, 128, 128),
+    ("iso", True, "f32", 1, 45, 2, 32, 64),
+    ("iso", True, "bf16", 1, 96, 2, 128, 128),
+]
+
+
+@pytest.mark.parametrize("case", BWD_CASES, ids=lambda c: "-".join(map(str, c)))
+def test_backward_parity(kdn, case):
+    variant, pc, dt, B, T, H, dk, dv = case
+    ins = make_inputs(variant, B, T, H, dk, dv, dtype=dt, seed=7 * T + dk, s0_std=0.1,
+                      p0_range=(0.5, 2.0), per_channel_decay=pc, with_grad=True)
+    rng = np.random.default_rng(T)
+    dST = rng.standard_normal((B, H, dk, dv)).astype(np.float32).astype(np.float64)
+    dpT = rng.standard_normal(ins["p0"].shape).astype(np.float32).astype(np.float64)
+    ref = oracle.bwd(variant, *[ins[n] for n in ("q", "k", "v", "g", "omega", "r")], ins["S0"],
+                     ins["p0"], ins["dO"], dST, dpT)
+    d = to_dev(ins)
+    fn = kdn.kdn_diag_bwd if variant == "diag" else kdn.kdn_iso_bwd
+    gr = fn(d["q"], d["k"], d["v"], d["g"], d["omega"], d["r"], d["S0"], d["p0"], d["dO"],
+            torch.tensor(dST, dtype=torch.float32, device="cuda"),
+            torch.tensor(dpT, dtype=torch.float32, device="cuda"))
+    torch.cuda.synchronize()
+    for n in ("dq", "dk", "dv", "dg", "domega", "dr", "dS0", "dp0"):
+        check(n, gr[n], ref[n], dt)
+
+
+def test_backward_without_state_cotangents(kdn):
+    ins = make_inputs("diag", 1, 40, 1, 32, 32, dtype="f32", seed=5, with_grad=True)
+    ref = oracle.bwd("diag", *[ins[n] for n in ("q", "k", "v", "g", "omega", "r")], None, None,
+                     ins["dO"])
+    d = to_dev(ins)
+    gr = kdn.kdn_diag_bwd(d["q"], d["k"], d["v"], d["g"], d["omega"], d["r"], None, None,
+                          d["dO"])
+    for n in ("dq", "dk", "dv", "dg", "domega", "dr", "dS0", "dp0"):
+        check(n, gr[n], ref[n], "f32")
+
+
+DEC_CASES = [
+    ("diag", True, "f32", 3, 2, 128, 128),
+    ("diag", True, "bf16", 4, 3, 64, 32),
+    ("diag", True, "bf16", 2, 2, 32, 128),
+    ("iso", False, "f32", 3, 2, 128, 64),
+    ("iso", False, "bf16", 2, 4, 128, 128),
+    ("iso", True, "bf16", 2, 2, 64, 64),
+]
+
+
+@pytest.mark.parametrize("case", DEC_CASES, ids=lambda c: "-".join(map(str, c)))
+def test_decode_parity(kdn, case):
+    variant, pc, dt, B, H, dk, dv = case
+    steps = 5
+    ins = make_decode_inputs(variant, B, H, dk, dv, steps, dtype=dt, seed=B * H + dk,
+                             per_channel_decay=pc)
+    tdt = torch.float32 if dt == "f32" else torch.bfloat16
+    S = torch.tensor(ins["S"], dtype=torch.float32, device="cuda")
+    p = torch.tensor(ins["p"], dtype=torch.float32, device="cuda")
+    S_ref, p_ref = ins["S"].copy(), ins["p"].copy()
+    fn = kdn.kdn_diag_decode_step if variant == "diag" else kdn.kdn_iso_decode_step
+    for s in range(steps):
+        x = {n: torch.tensor(ins[n][s], dtype=tdt, device="cuda")
+             for n in ("q", "k", "v", "g", "omega", "r")}
+        o = fn(x["q"], x["k"], x["v"], x["g"], x["omega"], x["r"], S, p)
+        o_ref, S_ref, p_ref = oracle.decode_step(variant, *[ins[n][s] for n in
+                                                 ("q", "k", "v", "g", "omega", "r")], S_ref, p_ref)
+        check(f"o[{s}]", o, o_ref, dt)
+    check("S", S, S_ref, dt)
+    check("p", p, p_ref, dt)
+
+
+@pytest.mark.parametrize("variant", ["diag", "iso"])
+def test_prefill_then_decode_equals_longer_prefill(kdn, variant):
+    T = 77
+    ins = make_inputs(variant, 2, T + 1, 2, 128, 128, dtype="f32", seed=11, s0_std=0.05)
+    d = to_dev(ins)
+    fwd = kdn.kdn_diag_fwd if variant == "diag" else kdn.kdn_iso_fwd
+    dec = kdn.kdn_diag_decode_step if variant == "diag" else kdn.kdn_iso_decode_step
+    sl = lambda x: x[:, :T].contiguous()
+    o1, ST, pT = fwd(*[sl(d[n]) for n in ("q", "k", "v", "g", "omega", "r")], d["S0"], d["p0"])
+    last = {n: d[n][:, T].contiguous() for n in ("q", "k", "v", "g", "omega", "r")}
+    o_last = dec(last["q"], last["k"], last["v"], last["g"], last["omega"], last["r"], ST, pT)
+    o_full, ST_full, pT_full = fwd(*[d[n] for n in ("q", "k", "v", "g", "omega", "r")],
+                                   d["S0"], d["p0"])
+    ref = _oracle_fwd(variant, ins)
+    check("o_last", o_last, ref["o"][:, T], "f32")
+    check("ST", ST, ref["ST"], "f32")
+    check("ST_full", ST_full, ref["ST"], "f32")
+    assert torch.allclose(o_last, o_full[:, T], rtol=1e-4, atol=1e-5)
+
+
+@pytest.mark.parametrize("variant", ["diag", "iso"])
+def test_empty_and_single_token(kdn, variant):
+    ins = make_inputs(variant, 2, 1, 3, 32, 32, dtype="f32", seed=1, s0_std=0.3,
+                      p0_range=(0.5, 2.0))
+    d = to_dev(ins)
+    fwd = kdn.kdn_diag_fwd if variant == "diag" else kdn.kdn_iso_fwd
+    o, ST, pT = fwd(d["q"], d["k"], d["v"], d["g"], d["omega"], d["r"], d["S0"], d["p0"])
+    ref = _oracle_fwd(variant, ins)
+    check("o", o, ref["o"], "f32")
+    check("ST", ST, ref["ST"], "f32")
+    check("pT", pT, ref["pT"], "f32")
+    e = {n: d[n][:, :0].contiguous() for n in ("q", "k", "v", "g", "omega", "r")}
+    o0, ST0, pT0 = fwd(e["q"], e["k"], e["v"], e["g"], e["omega"], e["r"], d["S0"], d["p0"])
+    assert o0.numel() == 0
+    assert torch.equal(ST0, d["S0"]) and torch.equal(pT0, d["p0"])
+    o0, ST0, pT0 = fwd(e["q"], e["k"], e["v"], e["g"], e["omega"], e["r"])
+    assert torch.count_nonzero(ST0) == 0 and torch.all(pT0 == 1)
+
+
+def test_degenerate_inputs(kdn):
+    """Zero keys (kappa = 0, memory only decays) and alpha = 1 with tiny omega."""
+    ins = make_inputs("diag", 1, 70, 2, 64, 64, dtype="f32", seed=2, s0_std=0.5)
+    ins["k"][:, 10:30] = 0.0
+    ins["g"][:, 40:] = 0.0
+    ins["omega"][:, 40:] = 1e-6
+    ref = _oracle_fwd("diag", ins)
+    o, ST, pT = _gpu_fwd(kdn, "diag", to_dev(ins))
+    check("o", o, ref["o"], "f32")
+    check("ST", ST, ref["ST"], "f32")
+    check("pT", pT, ref["pT"], "f32")
+
+
+@pytest.mark.parametrize("variant", ["diag", "iso"])
+def test_bf16_stored_outputs(kdn, variant):
+    """o and the input gradients stored as bfloat16 (out_dtype = KDN_BF16)."""
+    ins = make_inputs(variant, 1, 97, 3, 64, 128, dtype="bf16", seed=161, s0_std=0.02,
+                      p0_range=(0.1, 2.0), with_grad=True)
+    d = to_dev(ins)
+    names = ("q", "k", "v", "g", "omega", "r")
+    fwd = kdn.kdn_diag_fwd if variant == "diag" else kdn.kdn_iso_fwd
+    bwd = kdn.kdn_diag_bwd if variant == "diag" else kdn.kdn_iso_bwd
+    o, ST, pT = fwd(*[d[n] for n in names], d["S0"], d["p0"], out_dtype=torch.bfloat16)
+    assert o.dtype == torch.bfloat16
+    ref = _oracle_fwd(variant, ins)
+    check_stored_bf16("o", o, ref["o"])
+    check("ST", ST, ref["ST"], "bf16")
+    gr = bwd(*[d[n] for n in names], d["S0"], d["p0"], d["dO"], out_dtype=torch.bfloat16)
+    rg = oracle.bwd(variant, *[ins[n] for n in names], ins["S0"], ins["p0"], ins["dO"])
+    for n in ("dq", "dk", "dv", "dg", "domega", "dr"):
+        assert gr[n].dtype == torch.bfloat16
+        check_stored_bf16(n, gr[n], rg[n])
