@@ -1,0 +1,463 @@
+"""Benchmark of the KDN token-mixer hot path on GB300.
+
+One step = one Diagonal-KDN forward + backward (all steps of the chunked
+forward, its adjoint) over one synthetic batch shaped like a 1.3B-model layer:
+B=8, H=16, T=4096, d_k=d_v=128, bfloat16 activations, float32 state and
+outputs.  `value` is layer tokens/s (B*T per step, summed over ranks).  The
+same JSON line also carries the decode step (B=256, H=16, d=128, 1024
+consecutive tokens in one CUDA graph) in steps/s, the forward kernel's
+roofline, an end-to-end number through host buffers, and the oracle's CPU
+throughput on a bounded sample.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+
+With --impl reference the fp64 CPU oracle is timed on a bounded sample of the
+same workload on the host cores (rank 0 only).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "KDN layer fwd+bwd tokens/s at 1 GB300 and % of roofline; decode steps/s"
+B, T, H, DK, DV = 8, 4096, 16, 128, 128
+DEC_B, DEC_H, DEC_STEPS = 256, 16, 1024
+NAMES = ("q", "k", "v", "g", "omega", "r")
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), float(p["bf16_tflops"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return 6800.0, 1900.0, "fallback"
+
+
+# ---------------------------------------------------------------------------
+# algorithmic work (bytes that must cross HBM once; no intermediates)
+
+def fwd_bytes(b, t, h, dk, dv, in_bytes=2, out_bytes=4, with_state=True):
+    # per token-head: q, k, g, omega (dk each) + v (dv) + r read; o (dv) written
+    per_tok = (4 * dk + dv + 1) * in_bytes + dv * out_bytes
+    per_seq = (dk * dv * 4 + dk * 4) if with_state else 0   # S_T, p_T written
+    return b * t * h * per_tok + b * h * per_seq
+
+
+def bwd_bytes(b, t, h, dk, dv, in_bytes=2, out_bytes=4):
+    reads = (2 * dk + dv + 2 * dk + 1 + dv) * in_bytes          # q k v g omega r dO
+    writes = (2 * dk + dv + 2 * dk + 1) * out_bytes              # dq dk dv dg domega dr
+    per_seq = dk * dv * 4 + dk * 4                               # dS0, dp0
+    return b * t * h * (reads + writes) + b * h * per_seq
+
+
+def decode_bytes(b, h, dk, dv, in_bytes=2, out_bytes=4):
+    state = 2 * (dk * dv * 4 + dk * 4)
+    ins = (2 * dk + dv + 2 * dk + 1) * in_bytes
+    return b * h * (state + ins + dv * out_bytes)
+
+
+def chunk_flops(dk, dv, C=64):
+    # App. F chunked form per token-head: two C x C products, three C x C by
+    # C x d products and three d x d products (dense-counted).
+    return 10 * C * max(dk, dv) + 6 * dk * dv
+
+
+# ---------------------------------------------------------------------------
+# clock sampling during the timed region
+
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+            time.sleep(0.25)
+        except OSError:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 7:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx.append(float(parts[1]))
+            except ValueError:
+                continue
+            for n, val in zip(names, parts[3:7]):
+                if val.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx),
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------
+# distributed plumbing (one process per GPU; replicas, no data exchange)
+
+def dist_setup(n):
+    import torch
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world != n:
+        raise SystemExit(f"--gpus {n} but WORLD_SIZE={world}")
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    else:
+        torch.cuda.set_device(0)
+    return rank, local, world
+
+
+def barrier(world):
+    import torch
+    torch.cuda.synchronize()
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+    torch.cuda.synchronize()
+
+
+def reduce_max(x, world):
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ---------------------------------------------------------------------------
+# synthetic inputs on the device (same recipe as kdn_inputs, drawn with torch)
+
+def device_inputs(variant, b, t, h, dk, dv, seed, dtype, per_channel=True, with_grad=True):
+    import torch
+    gen = torch.Generator(device="cuda")
+    gen.manual_seed(seed)
+    f = dict(device="cuda", generator=gen, dtype=torch.float32)
+    q = torch.randn(b, t, h, dk, **f)
+    q = q / q.norm(dim=-1, keepdim=True)
+    k = torch.randn(b, t, h, dk, **f)
+    k = k / k.norm(dim=-1, keepdim=True)
+    v = torch.randn(b, t, h, dv, **f)
+    gshape = (b, t, h, dk) if per_channel else (b, t, h)
+    g = torch.nn.functional.logsigmoid(torch.randn(gshape, **f) + 2.0)
+    wshape = (b, t, h, dk) if variant == "diag" else (b, t, h)
+    om = torch.nn.functional.softplus(torch.randn(wshape, **f))
+    r = torch.nn.functional.softplus(torch.randn(b, t, h, **f))
+    out = {n: x.to(dtype) for n, x in zip(NAMES, (q, k, v, g, om, r))}
+    if with_grad:
+        out["dO"] = torch.randn(b, t, h, dv, **f).to(dtype)
+    return out
+
+
+# ---------------------------------------------------------------------------
+
+def run_gpu(args):
+    import torch
+    import paper_2609_07816_gb300 as kdn
+    from paper_2609_07816_gb300 import build as kbuild
+
+    kbuild.build()
+    rank, local, world = dist_setup(args.gpus)
+    hbm, tf, peak_kind = peaks()
+    global B
+    B = args.batch
+    dt = torch.bfloat16
+    ins = device_inputs("diag", B, T, H, DK, DV, seed=1000 + rank, dtype=dt)
+    x = [ins[n] for n in NAMES]
+    desc = kdn.make_desc(B, T, H, DK, DV, dt)
+    ws_f = kdn.alloc_workspace(desc, 0, False)
+    ws_b = kdn.alloc_workspace(desc, 0, True)
+    o = torch.empty(B, T, H, DV, dtype=torch.float32, device="cuda")
+    ST = torch.empty(B, H, DK, DV, dtype=torch.float32, device="cuda")
+    pT = torch.empty(B, H, DK, dtype=torch.float32, device="cuda")
+    grads = {n: torch.empty(ins[m].shape, dtype=torch.float32, device="cuda") for n, m in
+             (("dq", "q"), ("dk", "k"), ("dv", "v"), ("dg", "g"), ("domega", "omega"),
+              ("dr", "r"))}
+    grads["dS0"] = torch.empty(B, H, DK, DV, dtype=torch.float32, device="cuda")
+    grads["dp0"] = torch.empty(B, H, DK, dtype=torch.float32, device="cuda")
+    stream = torch.cuda.current_stream()
+
+    def step(ev=None):
+        if ev is not None:
+            ev[0].record(stream)
+        kdn.kdn_diag_fwd(*x, o=o, ST=ST, pT=pT, workspace=ws_f)
+        if ev is not None:
+            ev[1].record(stream)
+        kdn.kdn_diag_bwd(*x, None, None, ins["dO"], grads=grads, workspace=ws_b)
+        if ev is not None:
+            ev[2].record(stream)
+
+    for _ in range(args.warmup):
+        step()
+    launches_per_step = kdn.kdn_kernel_launches(desc, 0, 0) + kdn.kdn_kernel_launches(desc, 0, 1)
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier(world)
+    with ClockSampler(local) as clk:
+        start.record(stream)
+        for i in range(args.steps):
+            step(evs[i])
+        stop.record(stream)
+        torch.cuda.synchronize()
+    barrier(world)
+    total_ms = reduce_max(start.elapsed_time(stop), world)
+    fwd_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in evs)
+    bwd_ms = statistics.mean(e[1].elapsed_time(e[2]) for e in evs)
+    ms_step = total_ms / args.steps
+    tokens = B * T * world
+    value = tokens / (ms_step / 1e3)
+
+    fb = fwd_bytes(B, T, H, DK, DV)
+    bb = bwd_bytes(B, T, H, DK, DV)
+    roof = {"bound": "hbm", "kernel": "kdn_diag_fwd (forward entry point)",
+            "achieved": fb / (fwd_ms / 1e3) / 1e9, "peak": hbm, "unit": "GB/s",
+            "peak_kind": peak_kind, "traffic": None, "algorithmic_bytes": fb}
+    roof["frac"] = roof["achieved"] / roof["peak"]
+    bwd_roof = {"bound": "hbm", "achieved": bb / (bwd_ms / 1e3) / 1e9, "peak": hbm,
+                "unit": "GB/s", "algorithmic_bytes": bb}
+    bwd_roof["frac"] = bwd_roof["achieved"] / hbm
+    # the paper-style roofline: max(FLOPs / 2.25 PF, bytes / 8 TB/s)
+    spec_time = max(B * T * H * chunk_flops(DK, DV) * 3.5 / 2.25e15, (fb + bb) / 8e12)
+
+    dec = run_decode(kdn, torch, hbm) if rank == 0 and not args.no_decode else None
+    e2e = run_e2e(kdn, torch, x, ins, args) if rank == 0 and not args.no_e2e else None
+    out = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "data": "synthetic",
+        "config": {"workload": "Diagonal KDN fwd+bwd, 1.3B-layer shape", "B": B, "T": T, "H": H,
+                   "dk": DK, "dv": DV, "activations": "bf16", "outputs": "f32",
+                   "state": "f32", "parallelism": f"replicas x{world}",
+                   "l2": "inputs larger than L2 (each activation tensor 134 MB)"},
+        "fwd_ms": fwd_ms, "bwd_ms": bwd_ms,
+        "roofline": roof, "bwd_roofline": bwd_roof,
+        "spec_roofline_frac": spec_time / (ms_step / 1e3) if ms_step > 0 else None,
+        "gpu_launches": launches_per_step * args.steps,
+        "clocks": clk.summary(),
+        "decode": dec, "e2e": e2e,
+    }
+    if rank == 0 and not args.no_cpu_baseline:
+        out["cpu_baseline"] = cpu_baseline(sample_heads=args.cpu_heads)
+    if rank == 0:
+        print(json.dumps(out))
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+def run_decode(kdn, torch, hbm):
+    """1024 consecutive decode tokens for B=256, H=16 in one CUDA graph, both variants."""
+    res = {}
+    for variant in ("diag", "iso"):
+        gen = torch.Generator(device="cuda")
+        gen.manual_seed(7)
+        f = dict(device="cuda", generator=gen, dtype=torch.float32)
+        S = torch.randn(DEC_B, DEC_H, DK, DV, **f) * 0.02
+        p = (torch.rand((DEC_B, DEC_H, DK) if variant == "diag" else (DEC_B, DEC_H), **f)
+             * 1.9 + 0.1)
+        shape = (DEC_STEPS, DEC_B, DEC_H)
+        q = torch.randn(*shape, DK, **f)
+        q = (q / q.norm(dim=-1, keepdim=True)).bfloat16()
+        k = torch.randn(*shape, DK, **f)
+        k = (k / k.norm(dim=-1, keepdim=True)).bfloat16()
+        v = torch.randn(*shape, DV, **f).bfloat16()
+        g = torch.nn.functional.logsigmoid(
+            torch.randn(*shape, DK, **f) + 2.0 if variant == "diag" else torch.randn(*shape, **f) + 2.0
+        ).bfloat16()
+        om = torch.nn.functional.softplus(
+            torch.randn(*shape, DK, **f) if variant == "diag" else torch.randn(*shape, **f)).bfloat16()
+        r = torch.nn.functional.softplus(torch.randn(*shape, **f)).bfloat16()
+        o = torch.empty(DEC_B, DEC_H, DV, dtype=torch.float32, device="cuda")
+        fn = kdn.kdn_diag_decode_step if variant == "diag" else kdn.kdn_iso_decode_step
+        s = torch.cuda.Stream()
+        s.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(s):
+            for i in range(3):
+                fn(q[i], k[i], v[i], g[i], om[i], r[i], S, p, o=o, stream=s)
+        torch.cuda.current_stream().wait_stream(s)
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph):
+            st = torch.cuda.current_stream()
+            for i in range(DEC_STEPS):
+                fn(q[i], k[i], v[i], g[i], om[i], r[i], S, p, o=o, stream=st)
+        graph.replay()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        graph.replay()
+        e1.record()
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1)
+        per = ms / DEC_STEPS
+        by = decode_bytes(DEC_B, DEC_H, DK, DV)
+        res[variant] = {"steps_per_s": DEC_STEPS / (ms / 1e3), "us_per_step": per * 1e3,
+                        "achieved_GBs": by / (per / 1e3) / 1e9, "frac_hbm": by / (per / 1e3) / 1e9 / hbm,
+                        "gpu_launches": DEC_STEPS}
+        del graph
+    return {"metric": "decode steps/s (B=256, H=16, d=128, 1024 steps, CUDA graph)",
+            "value": res["diag"]["steps_per_s"], "unit": "steps/s", **res}
+
+
+def run_e2e(kdn, torch, x, ins, args):
+    """Same step through the public API with host buffers: pinned host -> device
+    copies of the step's inputs, forward + backward, device -> host copies of the
+    outputs and gradients, all inside the timed region."""
+    host_in = {n: ins[n].cpu().pin_memory() for n in NAMES + ("dO",)}
+    dev_in = {n: torch.empty_like(ins[n]) for n in NAMES + ("dO",)}
+    outs_host = {}
+    stream = torch.cuda.current_stream()
+
+    def step():
+        for n in NAMES + ("dO",):
+            dev_in[n].copy_(host_in[n], non_blocking=True)
+        xx = [dev_in[n] for n in NAMES]
+        o, _, _ = kdn.kdn_diag_fwd(*xx, want_state=False)
+        gr = kdn.kdn_diag_bwd(*xx, None, None, dev_in["dO"], want_state_grads=False)
+        res = {"o": o, **gr}
+        for n, t in res.items():
+            if n not in outs_host:
+                outs_host[n] = torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
+            outs_host[n].copy_(t, non_blocking=True)
+        return res
+
+    for _ in range(max(1, args.warmup)):
+        step()
+    torch.cuda.synchronize()
+    n = max(1, min(args.steps, 3))
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(n):
+        res = step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / n
+    h2d = sum(host_in[k].numel() * host_in[k].element_size() for k in host_in)
+    d2h = sum(t.numel() * t.element_size() for t in res.values())
+    return {"value": B * T / (ms / 1e3), "unit": "tokens/s", "ms_per_step": ms,
+            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle timing (bounded sample of the same workload)
+
+def cpu_baseline(sample_heads=None):
+    import numpy as np
+
+    import oracle
+    from kdn_inputs import make_inputs
+    oracle.build()
+    cores = os.cpu_count() or 1
+    n = sample_heads or min(2 * cores, B * H)
+    ins = make_inputs("diag", 1, T, n, DK, DV, dtype="bf16", seed=0, with_grad=True)
+    args = [ins[k] for k in NAMES]
+    t0 = time.perf_counter()
+    r1 = oracle.fwd("diag", *args, None, None, threads=cores)
+    r2 = oracle.bwd("diag", *args, None, None, ins["dO"], threads=cores)
+    wall = time.perf_counter() - t0
+    token_heads = n * T
+    return {"value": token_heads / H / wall, "unit": "tokens/s", "cores": int(r2["threads"]),
+            "kind": "oracle", "wall_s": wall,
+            "sample": f"fwd+bwd of {n} (batch, head) sequences of T={T}, d=128 "
+                      f"(= {token_heads / H:.0f} layer tokens of H={H})"}
+
+
+def run_reference(args):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    import oracle
+    oracle.build()
+    cores = os.cpu_count() or 1
+    n = min(2 * cores, B * H)
+    samples = []
+    for i in range(args.warmup + args.steps):
+        cb = cpu_baseline(sample_heads=n)
+        if i >= args.warmup:
+            samples.append(cb)
+    val = statistics.mean(s["value"] for s in samples)
+    ms = statistics.mean(s["wall_s"] for s in samples) * 1e3
+    out = {"impl": "reference", "metric": METRIC, "value": val, "unit": "tokens/s",
+           "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+           "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+           "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+           "config": {"workload": "Diagonal KDN fwd+bwd, 1.3B-layer shape", "B": B, "T": T,
+                      "H": H, "dk": DK, "dv": DV, "activations": "bf16",
+                      "sample": samples[0]["sample"]},
+           "cpu_baseline": {"value": val, "unit": "tokens/s", "cores": samples[0]["cores"],
+                            "kind": "oracle", "sample": samples[0]["sample"]},
+           "e2e": {"value": val, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                   "d2h_bytes_per_step": 0}}
+    print(json.dumps(out))
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="kdn", choices=["kdn", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-decode", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--batch", type=int, default=B, help="batch size (profiling runs only)")
+    ap.add_argument("--cpu-heads", type=int, default=None)
+    args = ap.parse_args()
+    if args.warmup < 3 and args.impl != "reference":
+        raise SystemExit("--warmup must be >= 3")
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_gpu(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -157,6 +157,12 @@ kdn_status_t kdn_iso_decode_step(const kdn_desc_t *desc, const void *q,
                                  const void *omega, const void *r, float *S,
                                  float *p, void *o, void *stream);
 
+/* Number of CUDA kernels one call of an entry point launches for this
+   descriptor when T > 0 (op 0 = kdn_*_fwd, 1 = kdn_*_bwd, 2 = kdn_*_decode_step;
+   variant 0 = diagonal, 1 = isotropic).  -1 for an invalid descriptor or op.
+   Calls with T = 0 launch at most one small fill kernel. */
+int kdn_kernel_launches(const kdn_desc_t *desc, int variant, int op);
+
 /* Synchronises `stream`, then returns and clears the device status word kept
    in the first bytes of `workspace`: KDN_OK, or KDN_ERR_TIMEOUT when a bounded
    device-side wait of the most recent kdn_*_fwd / kdn_*_bwd call on that

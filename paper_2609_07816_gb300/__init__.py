@@ -59,6 +59,7 @@ _SIG = {
     "kdn_iso_bwd": ([ctypes.POINTER(kdn_desc_t)] + [_P] * 20 + [ctypes.c_size_t, _P], ctypes.c_int),
     "kdn_diag_decode_step": ([ctypes.POINTER(kdn_desc_t)] + [_P] * 10, ctypes.c_int),
     "kdn_iso_decode_step": ([ctypes.POINTER(kdn_desc_t)] + [_P] * 10, ctypes.c_int),
+    "kdn_kernel_launches": ([ctypes.POINTER(kdn_desc_t), ctypes.c_int, ctypes.c_int], ctypes.c_int),
     "kdn_get_device_status": ([_P, _P], ctypes.c_int),
 }
 EXPORTED = tuple(_SIG)
@@ -237,6 +238,11 @@ def kdn_iso_decode_step(q, k, v, g, omega, r, S, p, *, mu=None, scale=None, o=No
     """One Isotropic KDN token for every head; g [B,H,dk] or [B,H]; p [B,H] in place."""
     return _decode("kdn_iso_decode_step", 1, q, k, v, g, omega, r, S, p, mu=mu, scale=scale,
                    o=o, stream=stream, out_dtype=out_dtype)
+
+
+def kdn_kernel_launches(desc: kdn_desc_t, variant: int, op: int) -> int:
+    """Kernels one call launches (op 0 fwd, 1 bwd, 2 decode step)."""
+    return int(lib().kdn_kernel_launches(ctypes.byref(desc), int(variant), int(op)))
 
 
 def kdn_get_device_status(workspace, stream=None) -> int:

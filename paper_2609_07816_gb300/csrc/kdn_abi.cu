@@ -281,6 +281,17 @@ kdn_status_t kdn_iso_decode_step(const kdn_desc_t *desc, const void *q, const vo
   return decode_entry(1, desc, q, k, v, g, omega, r, S, p, o, stream);
 }
 
+int kdn_kernel_launches(const kdn_desc_t *desc, int variant, int op) {
+  Args a;
+  if (fill_sizes(desc, variant, op == 2, &a) != KDN_OK) return -1;
+  switch (op) {
+    case 0: return chunked_fwd_launches(a);
+    case 1: return chunked_bwd_launches(a);
+    case 2: return 1;
+  }
+  return -1;
+}
+
 kdn_status_t kdn_get_device_status(void *workspace, void *stream) {
   if (!workspace || ((uintptr_t)workspace % kAlign)) return KDN_ERR_INVALID_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);

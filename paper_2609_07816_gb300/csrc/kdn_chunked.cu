@@ -832,6 +832,9 @@ kdn_status_t bwd_dk(const Args &a, cudaStream_t s) {
 
 int chunked_chunk_len() { return CC; }
 
+int chunked_fwd_launches(const Args &) { return 3; }
+int chunked_bwd_launches(const Args &a) { return chunked_fwd_launches(a) + 4; }
+
 kdn_status_t launch_chunked_fwd(const Args &a, cudaStream_t s, bool save_states) {
   if (a.variant == 0)
     return a.dtype == KDN_BF16 ? fwd_dk<0, __nv_bfloat16>(a, s, save_states)

@@ -96,4 +96,8 @@ kdn_status_t launch_chunked_fwd(const Args &a, cudaStream_t s, bool save_states)
 kdn_status_t launch_chunked_bwd(const Args &a, cudaStream_t s);
 kdn_status_t launch_decode(const Args &a, float *S, float *p, cudaStream_t s);
 
+// Kernels launched by launch_chunked_fwd / launch_chunked_bwd for these sizes.
+int chunked_fwd_launches(const Args &a);
+int chunked_bwd_launches(const Args &a);
+
 }  // namespace kdn

@@ -135,3 +135,12 @@ def test_product_package_does_not_import_oracle():
             if f.endswith((".py", ".cu", ".cuh", ".h")):
                 text = open(os.path.join(dirpath, f)).read()
                 assert "oracle" not in text.lower().replace("oracle-free", ""), f
+
+
+def test_kernel_launch_query(kdn):
+    d = kdn.make_desc(2, 100, 3, 64, 32, kdn.KDN_BF16)
+    f, b, dec = (kdn.kdn_kernel_launches(d, 0, op) for op in (0, 1, 2))
+    assert f >= 1 and b > f and dec == 1
+    assert kdn.kdn_kernel_launches(d, 1, 0) >= 1
+    assert kdn.kdn_kernel_launches(d, 0, 7) == -1
+    assert kdn.kdn_kernel_launches(kdn.make_desc(1, 4, 1, 96, 32, 0), 0, 0) == -1
