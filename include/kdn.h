@@ -157,6 +157,29 @@ kdn_status_t kdn_iso_decode_step(const kdn_desc_t *desc, const void *q,
                                  const void *omega, const void *r, float *S,
                                  float *p, void *o, void *stream);
 
+/* Size of the library-owned scratch array used by kdn_diag_fwd_noalloc. */
+#define KDN_NOALLOC_SCRATCH_BYTES ((size_t)32 << 20)
+
+/* Diagonal-KDN forward that allocates nothing and takes no workspace.  The
+   paper has no counterpart: this exists for callers that are handed only
+   input and output buffers and may not call cudaMalloc (e.g. a latency-
+   critical thread where cudaMalloc can stall on a device synchronisation, or
+   a framework that forbids allocation outside its own allocator).  Arguments
+   and results are those of kdn_diag_fwd without the workspace pair.
+   Scratch is a fixed array of KDN_NOALLOC_SCRATCH_BYTES in the library's
+   device memory, held by every GPU that loads the library until exit; a
+   problem whose kdn_fwd_workspace_bytes() exceeds it is rejected with
+   KDN_ERR_WORKSPACE before anything runs.  The first call on a device looks
+   up the array's device address (cudaGetSymbolAddress, with that device
+   current); make it before any stream capture.  All calls on a device share
+   the array, so calls that overlap on the GPU race and must be serialised by
+   the caller. */
+kdn_status_t kdn_diag_fwd_noalloc(const kdn_desc_t *desc, const void *q,
+                                  const void *k, const void *v, const void *g,
+                                  const void *omega, const void *r,
+                                  const float *S0, const float *p0, void *o,
+                                  float *ST, float *pT, void *stream);
+
 /* Number of CUDA kernels one call of an entry point launches for this
    descriptor when T > 0 (op 0 = kdn_*_fwd, 1 = kdn_*_bwd, 2 = kdn_*_decode_step;
    variant 0 = diagonal, 1 = isotropic).  -1 for an invalid descriptor or op.

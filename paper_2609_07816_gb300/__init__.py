@@ -59,6 +59,7 @@ _SIG = {
     "kdn_iso_bwd": ([ctypes.POINTER(kdn_desc_t)] + [_P] * 20 + [ctypes.c_size_t, _P], ctypes.c_int),
     "kdn_diag_decode_step": ([ctypes.POINTER(kdn_desc_t)] + [_P] * 10, ctypes.c_int),
     "kdn_iso_decode_step": ([ctypes.POINTER(kdn_desc_t)] + [_P] * 10, ctypes.c_int),
+    "kdn_diag_fwd_noalloc": ([ctypes.POINTER(kdn_desc_t)] + [_P] * 12, ctypes.c_int),
     "kdn_kernel_launches": ([ctypes.POINTER(kdn_desc_t), ctypes.c_int, ctypes.c_int], ctypes.c_int),
     "kdn_get_device_status": ([_P, _P], ctypes.c_int),
 }
@@ -238,6 +239,20 @@ def kdn_iso_decode_step(q, k, v, g, omega, r, S, p, *, mu=None, scale=None, o=No
     """One Isotropic KDN token for every head; g [B,H,dk] or [B,H]; p [B,H] in place."""
     return _decode("kdn_iso_decode_step", 1, q, k, v, g, omega, r, S, p, mu=mu, scale=scale,
                    o=o, stream=stream, out_dtype=out_dtype)
+
+
+def kdn_diag_fwd_noalloc(q, k, v, g, omega, r, S0=None, p0=None, *, o, ST=None, pT=None,
+                         mu=None, scale=None, stream=None):
+    """Diagonal KDN forward into caller-provided outputs, using the library's own
+    fixed scratch array instead of a workspace, for callers that may not
+    allocate device memory.  Problems needing more than
+    KDN_NOALLOC_SCRATCH_BYTES of scratch are rejected.  Returns o."""
+    desc = _desc_from(0, q, v, g, chunk=0, mu=mu, scale=scale, out_dtype=o.dtype)
+    st = lib().kdn_diag_fwd_noalloc(ctypes.byref(desc), _ptr(q), _ptr(k), _ptr(v), _ptr(g),
+                                    _ptr(omega), _ptr(r), _ptr(S0), _ptr(p0), _ptr(o), _ptr(ST),
+                                    _ptr(pT), _stream(stream))
+    _check(st, "kdn_diag_fwd_noalloc")
+    return o
 
 
 def kdn_kernel_launches(desc: kdn_desc_t, variant: int, op: int) -> int:

@@ -1,0 +1,70 @@
+// kdn_noalloc.cu -- a Diagonal-KDN forward for callers that cannot allocate.
+//
+// kdn_diag_fwd needs a scratch workspace that the caller allocates.  Some
+// callers cannot do that: their interface hands them only input and output
+// buffers, and they may not call cudaMalloc themselves -- for instance a
+// latency-critical serving thread, where cudaMalloc can stall on an implicit
+// device synchronisation, or a host framework that forbids any allocation
+// outside its own allocator once it is running.  kdn_diag_fwd_noalloc serves
+// them: its scratch is a fixed array in the library's own device memory, so
+// the call itself allocates nothing.
+//
+// The array is a file-scope __device__ variable of KDN_NOALLOC_SCRATCH_BYTES.
+// Every GPU that loads this library holds that memory until the process
+// exits.  Host code cannot use the array's name as a device address, so the
+// first call on each device looks the address up with cudaGetSymbolAddress
+// (with that device current) and caches it; make that first call before any
+// stream capture.  All calls on a device share the one array and it keeps the
+// previous call's contents; nothing in it needs to start at zero (the forward
+// writes every scratch element before reading it, and clears its status word
+// itself), but calls whose executions overlap on the GPU -- on different
+// streams, or from different host threads -- race on it and must be
+// serialised by the caller.
+#include <mutex>
+
+#include "../../include/kdn.h"
+#include <cuda_runtime.h>
+
+namespace {
+
+constexpr size_t kScratchBytes = KDN_NOALLOC_SCRATCH_BYTES;
+constexpr int kMaxDevices = 64;
+
+static __device__ __align__(256) unsigned char kdn_noalloc_scratch[kScratchBytes];
+
+std::mutex g_mutex;
+void *g_scratch[kMaxDevices] = {};
+
+// Device address of the scratch array on the current device (set-up on first use).
+kdn_status_t scratch_address(void **out) {
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return KDN_ERR_CUDA;
+  std::lock_guard<std::mutex> lock(g_mutex);
+  if (!g_scratch[dev]) {
+    void *p = nullptr;
+    if (cudaGetSymbolAddress(&p, kdn_noalloc_scratch) != cudaSuccess || !p) return KDN_ERR_CUDA;
+    g_scratch[dev] = p;
+  }
+  *out = g_scratch[dev];
+  return KDN_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+kdn_status_t kdn_diag_fwd_noalloc(const kdn_desc_t *desc, const void *q, const void *k,
+                                  const void *v, const void *g, const void *omega,
+                                  const void *r, const float *S0, const float *p0, void *o,
+                                  float *ST, float *pT, void *stream) {
+  const size_t need = kdn_fwd_workspace_bytes(desc, 0);
+  if (need == 0)  // invalid descriptor: let the regular entry point name the error
+    return kdn_diag_fwd(desc, q, k, v, g, omega, r, S0, p0, o, ST, pT, nullptr, 0, stream);
+  if (need > kScratchBytes) return KDN_ERR_WORKSPACE;  // problem too large for the array
+  void *ws = nullptr;
+  kdn_status_t st = scratch_address(&ws);
+  if (st != KDN_OK) return st;
+  return kdn_diag_fwd(desc, q, k, v, g, omega, r, S0, p0, o, ST, pT, ws, kScratchBytes, stream);
+}
+
+}  // extern "C"
