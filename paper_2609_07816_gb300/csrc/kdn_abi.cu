@@ -51,10 +51,15 @@ kdn_status_t fill_sizes(const kdn_desc_t *d, int variant, bool decode, Args *a) 
   a->pcd = variant == 0 ? 1 : d->decay_per_channel;
   a->dtype = d->dtype;
   a->odt = d->out_dtype;
+  a->chunk = d->chunk;
   a->mu = d->mu > 0.f ? d->mu : (float)d->dk;
   a->tau = isnan(d->scale) ? 1.0f / sqrtf((float)d->dk) : d->scale;
   return KDN_OK;
 }
+
+// The fused forward serves bf16 activations with dk = dv = 128 and the default
+// (or 64-token) chunk; everything else runs the general chunked kernels.
+bool use_fused(const Args &a) { return a.chunk != 32 && fused_fwd_supported(a); }
 
 bool ptrs_ok(std::initializer_list<const void *> required,
              std::initializer_list<const void *> optional) {
@@ -124,6 +129,7 @@ kdn_status_t fwd_entry(int variant, const kdn_desc_t *d, const void *q, const vo
   if (cudaMemsetAsync(a.status, 0, sizeof(unsigned), s) != cudaSuccess) return KDN_ERR_CUDA;
   if ((size_t)a.B * a.H == 0) return KDN_OK;
   if (a.T == 0) return empty_fwd(a, s);
+  if (use_fused(a)) return launch_fused_fwd(a, s);
   return launch_chunked_fwd(a, s, false);
 }
 
@@ -179,6 +185,7 @@ size_t workspace_layout(Args *a, char *base, bool bwd) {
     return p;
   };
   a->status = reinterpret_cast<unsigned *>(take(kAlign / sizeof(float)));
+  if (!bwd && use_fused(*a)) return off;
   a->phat = take(BH * Tp * P);
   a->isotok = a->variant == 1 ? take(BH * Tp * 2) : nullptr;
   a->W = take(BH * NC * C * dk);
@@ -285,7 +292,7 @@ int kdn_kernel_launches(const kdn_desc_t *desc, int variant, int op) {
   Args a;
   if (fill_sizes(desc, variant, op == 2, &a) != KDN_OK) return -1;
   switch (op) {
-    case 0: return chunked_fwd_launches(a);
+    case 0: return use_fused(a) ? 1 : chunked_fwd_launches(a);
     case 1: return chunked_bwd_launches(a);
     case 2: return 1;
   }

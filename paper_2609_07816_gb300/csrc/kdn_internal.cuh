@@ -3,6 +3,7 @@
 #pragma once
 
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -53,6 +54,7 @@ struct Args {
   int pcd;      // decay has a channel axis (g is [..,dk])
   int dtype;
   int odt;      // dtype of o and of the input gradients
+  int chunk;    // chunk length requested in the descriptor (0, 32 or 64)
   float mu, tau;
   // forward inputs / outputs
   const void *q, *k, *v, *g, *omega, *r;
@@ -89,7 +91,12 @@ __host__ __device__ inline size_t tok_index(const Args &a, int b, int t, int h) 
 }
 
 // Workspace carve-up; returns total bytes.  `bwd` adds the backward regions.
+// A forward that runs the fused kernel only needs the status word.
 size_t workspace_layout(Args *a, char *base, bool bwd);
+
+// Fused tcgen05 forward (bf16, dk = dv = 128, 64-token chunks).
+bool fused_fwd_supported(const Args &a);
+kdn_status_t launch_fused_fwd(const Args &a, cudaStream_t s);
 
 // Launchers (each returns KDN_OK or KDN_ERR_CUDA).
 kdn_status_t launch_chunked_fwd(const Args &a, cudaStream_t s, bool save_states);
