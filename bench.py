@@ -230,13 +230,15 @@ def run_gpu(args):
         kdn.kdn_diag_fwd(*x, o=o, ST=ST, pT=pT, workspace=ws_f)
         if ev is not None:
             ev[1].record(stream)
-        kdn.kdn_diag_bwd(*x, None, None, ins["dO"], grads=grads, workspace=ws_b)
+        if not args.fwd_only:
+            kdn.kdn_diag_bwd(*x, None, None, ins["dO"], grads=grads, workspace=ws_b)
         if ev is not None:
             ev[2].record(stream)
 
     for _ in range(args.warmup):
         step()
-    launches_per_step = kdn.kdn_kernel_launches(desc, 0, 0) + kdn.kdn_kernel_launches(desc, 0, 1)
+    launches_per_step = kdn.kdn_kernel_launches(desc, 0, 0) + (
+        0 if args.fwd_only else kdn.kdn_kernel_launches(desc, 0, 1))
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
     start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     barrier(world)
@@ -448,6 +450,7 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-decode", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--fwd-only", action="store_true", help="profiling runs: forward only")
     ap.add_argument("--batch", type=int, default=B, help="batch size (profiling runs only)")
     ap.add_argument("--cpu-heads", type=int, default=None)
     args = ap.parse_args()

@@ -65,7 +65,7 @@ constexpr int OFF_B3 = OFF_A2 + 16384;    // S_in fp16 (MN-major)               
 constexpr int OFF_F = OFF_B3 + 32768;     // fp32 scratch: Y [64][128] / T, A [64][65] + X
 constexpr int F_BYTES = 2 * 64 * 65 * 4 + 3 * 256 * 4;  // 36352 >= 32768
 constexpr int OFF_SM = OFF_F + F_BYTES;                  // small arrays
-constexpr int SMALL_FLOATS = 64 * 6 + 128 * 2;
+constexpr int SMALL_FLOATS = 64 * 7 + 128 * 3;
 constexpr int OFF_BAR = OFF_SM + SMALL_FLOATS * 4;
 constexpr int SMEM_BYTES = OFF_BAR + 64 + 1024;  // + alignment slack
 
@@ -80,35 +80,54 @@ __device__ __forceinline__ float bf(const unsigned char *base, int slab_bytes, i
   return __bfloat162float(
       *reinterpret_cast<const __nv_bfloat16 *>(base + s * slab_bytes + sw128_off(row, col & 63)));
 }
-__device__ __forceinline__ void bfw(unsigned char *base, int slab_bytes, int row, int col, float x) {
-  const int s = col >> 6;
-  *reinterpret_cast<__nv_bfloat16 *>(base + s * slab_bytes + sw128_off(row, col & 63)) =
-      __float2bfloat16_rn(x);
+// 16-byte chunk `cc` (8 consecutive 2-byte elements) of row `row` in a
+// 128-byte-swizzled slab.
+__device__ __forceinline__ uint32_t chunk_off(int row, int cc) {
+  return (uint32_t)row * 128u + ((uint32_t)(cc ^ (row & 7)) << 4);
 }
-
-__device__ __forceinline__ void hw(unsigned char *base, int slab_bytes, int row, int col, float x) {
-  const int s = col >> 6;
-  *reinterpret_cast<__half *>(base + s * slab_bytes + sw128_off(row, col & 63)) = __float2half_rn(x);
+__device__ __forceinline__ void unpack_bf8(uint4 u, float *v) {
+  const __nv_bfloat162 *h = reinterpret_cast<const __nv_bfloat162 *>(&u);
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    const float2 f = __bfloat1622float2(h[j]);
+    v[2 * j] = f.x;
+    v[2 * j + 1] = f.y;
+  }
 }
-// x ~ hi + lo with both parts in bf16 (about 16 significant bits together)
-__device__ __forceinline__ void bfw2(unsigned char *hi, unsigned char *lo, int slab_bytes, int row,
-                                     int col, float x) {
-  const __nv_bfloat16 h = __float2bfloat16_rn(x);
-  const int s = col >> 6;
-  const uint32_t off = s * slab_bytes + sw128_off(row, col & 63);
-  *reinterpret_cast<__nv_bfloat16 *>(hi + off) = h;
-  *reinterpret_cast<__nv_bfloat16 *>(lo + off) = __float2bfloat16_rn(x - __bfloat162float(h));
+__device__ __forceinline__ uint4 pack_bf8(const float *v) {
+  uint4 u;
+  __nv_bfloat162 *h = reinterpret_cast<__nv_bfloat162 *>(&u);
+#pragma unroll
+  for (int j = 0; j < 4; ++j) h[j] = __floats2bfloat162_rn(v[2 * j], v[2 * j + 1]);
+  return u;
 }
-__device__ __forceinline__ float bf2(const unsigned char *hi, const unsigned char *lo,
-                                     int slab_bytes, int row, int col) {
-  return bf(hi, slab_bytes, row, col) + bf(lo, slab_bytes, row, col);
+__device__ __forceinline__ uint4 pack_h8(const float *v) {
+  uint4 u;
+  __half2 *h = reinterpret_cast<__half2 *>(&u);
+#pragma unroll
+  for (int j = 0; j < 4; ++j) h[j] = __floats2half2_rn(v[2 * j], v[2 * j + 1]);
+  return u;
+}
+// x ~ hi + lo, both bf16: returns hi, writes the lo chunk
+__device__ __forceinline__ uint4 split_bf8(const float *x, uint4 *lo) {
+  float h[8], l[8];
+  const uint4 hi = pack_bf8(x);
+  unpack_bf8(hi, h);
+#pragma unroll
+  for (int j = 0; j < 8; ++j) l[j] = x[j] - h[j];
+  *lo = pack_bf8(l);
+  return hi;
+}
+__device__ __forceinline__ uint4 &sm16(unsigned char *base, uint32_t off) {
+  return *reinterpret_cast<uint4 *>(base + off);
 }
 
 template <int V>
 __global__ void __launch_bounds__(FT, 1)
     k_fused_fwd(const __grid_constant__ CUtensorMap mq, const __grid_constant__ CUtensorMap mk,
                 const __grid_constant__ CUtensorMap mv, const __grid_constant__ CUtensorMap mg,
-                const __grid_constant__ CUtensorMap mw, const FusedParams P) {
+                const __grid_constant__ CUtensorMap mw, const __grid_constant__ CUtensorMap mo,
+                const FusedParams P) {
   const Args &a = P.a;
   extern __shared__ unsigned char smraw[];
   unsigned char *sm =
@@ -124,8 +143,10 @@ __global__ void __launch_bounds__(FT, 1)
   float *s_a = s_n2 + 64;    // [64] a_t (iso)
   float *s_om = s_a + 64;    // [64] omega_t (iso)
   float *s_gs = s_om + 64;   // [64] scalar g_t (iso, scalar decay)
-  float *s_gC = s_gs + 64;   // [128] gamma_C
+  float *s_ri = s_gs + 64;   // [64] 1 / r_t
+  float *s_gC = s_ri + 64;   // [128] gamma_C
   float *s_b = s_gC + 128;   // [1] isotropic carry b
+  float *s_p = s_b + 128;    // [128] diagonal carry p (per channel)
   uint64_t *bars = reinterpret_cast<uint64_t *>(sm + OFF_BAR);
   uint64_t *bar_raw = bars, *bar_v = bars + 1, *bar_mma = bars + 2;
   uint32_t *s_tbase = reinterpret_cast<uint32_t *>(bars + 4);
@@ -206,9 +227,8 @@ __global__ void __launch_bounds__(FT, 1)
     }
     tmem_st_wait();
   }
-  // uncertainty carry (diag: one channel per thread of warps 0-3)
-  float pcarry = 1.f;
-  if (V == 0 && tid < D && a.p0) pcarry = a.p0[(size_t)bh * D + tid];
+  // uncertainty carry (diag: one value per channel)
+  if (V == 0 && tid < D) s_p[tid] = a.p0 ? a.p0[(size_t)bh * D + tid] : 1.f;
   // per-token scalars of the next chunk, prefetched into registers
   float nr = 1.f, nom = 0.f, ng = 0.f;
   auto load_scalars = [&](int c) {
@@ -243,59 +263,103 @@ __global__ void __launch_bounds__(FT, 1)
     // ---- [1] raw tiles and per-token scalars of this chunk
     if (tid < CM) {
       s_r[tid] = nr;
+      s_ri[tid] = 1.f / nr;
       s_om[tid] = nom;
       s_gs[tid] = ng;
     }
+    if (tid == 0) bulk_wait_read();  // O staging (fs) of the previous chunk has been read
     ok = __syncthreads_and(mbar_wait(bar_raw, c & 1, kWaitIters));
     if (!ok) break;
     load_scalars(c + 1);
 
-    // ---- [2] gain, decay and the scaled operand tiles (hi/lo bf16 pairs)
+    // ---- [2] the sequential recursions of this chunk: per channel (diag) the
+    //          uncertainty chain and the cumulative decay, per head (iso) the
+    //          scalar chain; results go to fp32 scratch (b3 and fs are free here)
+    float *Pb = reinterpret_cast<float *>(b3);  // [64][128] phat_t
+    float *Eb = fs;                             // [64][128] gamma_t
     if (V == 0) {
-      if (tid < D) {
-        // warps 0-3: uncertainty recursion of channel i (eq. prefix-diag-uncertainty);
-        // Kbar overwrites raw k, the unscaled gain X = phat k / gamma overwrites raw omega
-        const int i = tid;
-        float p = pcarry, e = 1.f;
-        for (int t = 0; t < CM; ++t) {
-          const float gg = bf(rg, 8192, t, i), w = bf(rw, 8192, t, i), kk = bf(kq, 16384, t, i);
-          const float al = __expf(gg);
-          e *= al;
-          const float ph = al * al * p + w;  // eq. diag-covariance-prediction
-          fs[t * D + i] = ph * kk * kk;      // summand of s_t
-          bfw2(rw, b1l, 8192, t, i, __fdividef(ph * kk, e));
-          bfw2(kq, a1l, 16384, t, i, e * kk);
-          const float u = a.mu * kk * kk / s_r[t];
-          p = __fdividef(ph, 1.f + u * ph);
+      // Warps 0-3 run tokens 0..31 of channel i from the carry.  Warps 4-7 first
+      // form the Moebius product M_31 ... M_0 (eq. chunk-gain-summary; it does not
+      // depend on the carry), apply it to z_in = [p_in, 1] (eq. chunk-gain-carry)
+      // and run tokens 32..63 (eq. chunk-gain-local-prefix, -emission).
+      const int i = tid & (D - 1);
+      const bool second = tid >= D;
+      const float p_in = s_p[i];
+      float p = p_in, e = 1.f;
+      if (second) {
+        float m00 = 1.f, m01 = 0.f, m10 = 0.f, m11 = 1.f;
+        for (int t0 = 0; t0 < 32; t0 += 8) {
+          float al[8], w[8], uk[8];
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const float kk = bf(kq, 16384, t0 + j, i);
+            al[j] = __expf(bf(rg, 8192, t0 + j, i));
+            w[j] = bf(rw, 8192, t0 + j, i);
+            uk[j] = a.mu * kk * kk * s_ri[t0 + j];
+          }
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const float a2 = al[j] * al[j], ua2 = uk[j] * a2, d1 = 1.f + uk[j] * w[j];
+            const float n00 = a2 * m00 + w[j] * m10, n01 = a2 * m01 + w[j] * m11;
+            const float n10 = ua2 * m00 + d1 * m10, n11 = ua2 * m01 + d1 * m11;
+            m00 = n00; m01 = n01; m10 = n10; m11 = n11;
+            e *= al[j];
+          }
+          // renormalise by the largest magnitude (the ratio n/d is scale free)
+          const float mx = fmaxf(fmaxf(fabsf(m00), fabsf(m01)), fmaxf(fabsf(m10), fabsf(m11)));
+          const float sc = 1.f / mx;
+          m00 *= sc; m01 *= sc; m10 *= sc; m11 *= sc;
         }
-        pcarry = p;
-      } else {
-        // warps 4-7: cumulative decay and Qbar of channel i (overwrites raw q)
-        const int i = tid - D;
-        float e = 1.f;
-        for (int t = 0; t < CM; ++t) {
-          e *= __expf(bf(rg, 8192, t, i));
-          bfw2(kq, a1l, 16384, 64 + t, i, a.tau * e * bf(kq, 16384, 64 + t, i));
+        p = __fdividef(m00 * p_in + m01, m10 * p_in + m11);
+      }
+      const int tb = second ? 32 : 0;
+      for (int t0 = tb; t0 < tb + 32; t0 += 8) {
+        float al[8], w[8], uk[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const float kk = bf(kq, 16384, t0 + j, i);
+          al[j] = __expf(bf(rg, 8192, t0 + j, i));
+          w[j] = bf(rw, 8192, t0 + j, i);
+          uk[j] = a.mu * kk * kk * s_ri[t0 + j];
         }
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          e *= al[j];
+          const float ph = al[j] * al[j] * p + w[j];  // eq. diag-covariance-prediction
+          Pb[(t0 + j) * D + i] = ph;
+          Eb[(t0 + j) * D + i] = e;
+          p = __fdividef(ph, 1.f + uk[j] * ph);     // eq. prefix-diag-uncertainty
+        }
+      }
+      __syncthreads();  // every thread has read s_p
+      if (second) {
+        s_p[i] = p;
         s_gC[i] = e;
       }
     } else {
-      // isotropic: per-token reductions a_t and |k_t|^2
-      for (int t = warp * 8; t < warp * 8 + 8; ++t) {
+      // per-token reductions a_t and |k_t|^2, one half-warp per token
+      for (int m = 0; m < 4; ++m) {
+        const int t = 16 * m + 2 * warp + (lane >> 4), c8 = lane & 15, sl = c8 >> 3, cc = c8 & 7;
+        float kv[8];
+        unpack_bf8(sm16(kq, sl * 16384 + chunk_off(t, cc)), kv);
         float n2 = 0.f, sa = 0.f;
 #pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          const int i = lane + 32 * j;
-          const float kk = bf(kq, 16384, t, i);
-          n2 += kk * kk;
-          if (pcd) {
-            const float al = __expf(bf(rg, 8192, t, i));
+        for (int j = 0; j < 8; ++j) n2 += kv[j] * kv[j];
+        if (pcd) {
+          float gv[8];
+          unpack_bf8(sm16(rg, sl * 8192 + chunk_off(t, cc)), gv);
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const float al = __expf(gv[j]);
             sa += al * al;
           }
         }
-        n2 = warp_sum(n2);
-        sa = warp_sum(sa);
-        if (lane == 0) {
+#pragma unroll
+        for (int o = 8; o > 0; o >>= 1) {
+          n2 += __shfl_xor_sync(0xffffffffu, n2, o);
+          sa += __shfl_xor_sync(0xffffffffu, sa, o);
+        }
+        if (c8 == 0) {
           s_n2[t] = n2;
           const float al = __expf(s_gs[t]);
           s_a[t] = pcd ? sa / D : al * al;
@@ -305,13 +369,10 @@ __global__ void __launch_bounds__(FT, 1)
       if (tid < D) {
         const int i = tid;
         float e = 1.f;
+#pragma unroll 8
         for (int t = 0; t < CM; ++t) {
-          const float gg = pcd ? bf(rg, 8192, t, i) : s_gs[t];
-          e *= __expf(gg);
-          const float kk = bf(kq, 16384, t, i);
-          bfw2(rw, b1l, 8192, t, i, __fdividef(kk, e));
-          bfw2(kq, a1l, 16384, t, i, e * kk);
-          bfw2(kq, a1l, 16384, 64 + t, i, a.tau * e * bf(kq, 16384, 64 + t, i));
+          e *= __expf(pcd ? bf(rg, 8192, t, i) : s_gs[t]);
+          Eb[t * D + i] = e;
         }
         s_gC[i] = e;
       } else if (tid == D) {
@@ -319,32 +380,60 @@ __global__ void __launch_bounds__(FT, 1)
         float bb = s_b[0];
         for (int t = 0; t < CM; ++t) {
           const float bhat = s_a[t] * bb + s_om[t];
-          const float rr = s_r[t];
-          s_x[t] = __fdividef(bhat, rr + bhat * s_n2[t]);
-          const float u = a.mu * s_n2[t] / (D * rr);
-          bb = __fdividef(bhat, 1.f + u * bhat);
+          s_x[t] = __fdividef(bhat, s_r[t] + bhat * s_n2[t]);
+          bb = __fdividef(bhat, 1.f + a.mu * s_n2[t] * s_ri[t] * (1.f / D) * bhat);
         }
         s_b[0] = bb;
       }
     }
     __syncthreads();
     if (tid == 0 && c + 1 < NC) issue_raw_g(c + 1);  // the decay tile is no longer read
-    // ---- [3] Kk = X / s_t (diag) or beta_t X (iso), kept as a hi/lo pair
-    for (int t = warp * 8; t < warp * 8 + 8; ++t) {
-      float sc;
+    // ---- [3] operand tiles, 16-byte chunks (t, 8 channels), one half-warp per token:
+    //   Kk = phat k / (s_t gamma) (diag, s_t = r_t + sum phat k^2) or beta_t k / gamma (iso)
+    //   Kbar = gamma k, Qbar = tau gamma q; each as a hi/lo bf16 pair, written over
+    //   the raw tiles (hi) and into the lo buffers
+    for (int m = 0; m < 4; ++m) {
+      const int t = 16 * m + 2 * warp + (lane >> 4), c8 = lane & 15, sl = c8 >> 3, cc = c8 & 7;
+      const uint32_t ok16 = sl * 16384 + chunk_off(t, cc), oq16 = ok16 + 8192;
+      const uint32_t o8 = sl * 8192 + chunk_off(t, cc);
+      float kv[8], qv[8], ev[8], xv[8];
+      unpack_bf8(sm16(kq, ok16), kv);
+      unpack_bf8(sm16(kq, oq16), qv);
+      {
+        const float4 *ep = reinterpret_cast<const float4 *>(Eb + t * D + 8 * c8);
+        const float4 e0 = ep[0], e1 = ep[1];
+        ev[0] = e0.x; ev[1] = e0.y; ev[2] = e0.z; ev[3] = e0.w;
+        ev[4] = e1.x; ev[5] = e1.y; ev[6] = e1.z; ev[7] = e1.w;
+      }
       if (V == 0) {
-        float part = 0.f;
+        const float4 *pp = reinterpret_cast<const float4 *>(Pb + t * D + 8 * c8);
+        const float4 p0 = pp[0], p1 = pp[1];
+        const float ph[8] = {p0.x, p0.y, p0.z, p0.w, p1.x, p1.y, p1.z, p1.w};
+        float y = 0.f;
 #pragma unroll
-        for (int j = 0; j < 4; ++j) part += fs[t * D + lane + 32 * j];
-        sc = 1.f / (s_r[t] + warp_sum(part));
+        for (int j = 0; j < 8; ++j) y += ph[j] * kv[j] * kv[j];
+#pragma unroll
+        for (int o = 8; o > 0; o >>= 1) y += __shfl_xor_sync(0xffffffffu, y, o);
+        const float sc = 1.f / (s_r[t] + y);  // eq. kla-box-gain
+#pragma unroll
+        for (int j = 0; j < 8; ++j) xv[j] = __fdividef(ph[j] * kv[j] * sc, ev[j]);
       } else {
-        sc = s_x[t];
-      }
+        const float beta = s_x[t];
 #pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        const int i = lane + 32 * j;
-        bfw2(rw, b1l, 8192, t, i, sc * bf2(rw, b1l, 8192, t, i));
+        for (int j = 0; j < 8; ++j) xv[j] = __fdividef(beta * kv[j], ev[j]);
       }
+      uint4 lo;
+      sm16(rw, o8) = split_bf8(xv, &lo);
+      sm16(b1l, o8) = lo;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        xv[j] = ev[j] * kv[j];
+        qv[j] = a.tau * ev[j] * qv[j];
+      }
+      sm16(kq, ok16) = split_bf8(xv, &lo);
+      sm16(a1l, ok16) = lo;
+      sm16(kq, oq16) = split_bf8(qv, &lo);
+      sm16(a1l, oq16) = lo;
     }
     fence_proxy_async();
     tc_fence_before();
@@ -364,7 +453,9 @@ __global__ void __launch_bounds__(FT, 1)
     }
     if (!(ok = mma_wait())) break;
     tc_fence_after();
-    // ---- [5] T -> fp32 smem, A = (I + T)^-1
+    // ---- [5] T -> fp32 smem, A = (I + T)^-1 by 16x16 blocks:
+    //   diagonal blocks D_I = (I + T_II)^-1 by forward substitution (a column per lane),
+    //   then A_IJ = -D_I sum_{K=J}^{I-1} T_IK A_KJ level by level (I - J = 1, 2, 3)
     float *sT = fs, *sA = fs + 64 * 65, *sX = fs + 2 * 64 * 65;
     if (wq < 2) {
       const int r = 32 * wq + lane;
@@ -377,40 +468,59 @@ __global__ void __launch_bounds__(FT, 1)
       }
     }
     __syncthreads();
-    if (tid < 64) {
-      const int bI = tid >> 4, j = tid & 15, o0 = bI * 16;
+    if (warp < 4 && lane < 16) {
+      const int o0 = 16 * warp, l = lane;
+      float av[16];
+#pragma unroll
       for (int r = 0; r < 16; ++r) {
-        float acc = (r == j) ? 1.f : 0.f;
-        for (int s = j; s < r; ++s) acc -= sT[(o0 + r) * 65 + o0 + s] * sA[(o0 + s) * 65 + o0 + j];
-        sA[(o0 + r) * 65 + o0 + j] = (r >= j) ? acc : 0.f;
+        float acc0 = (r == l) ? 1.f : 0.f, acc1 = 0.f;
+#pragma unroll
+        for (int q2 = 0; q2 < r; q2 += 2) {
+          acc0 -= sT[(o0 + r) * 65 + o0 + q2] * av[q2];
+          if (q2 + 1 < r) acc1 -= sT[(o0 + r) * 65 + o0 + q2 + 1] * av[q2 + 1];
+        }
+        av[r] = acc0 + acc1;
       }
+#pragma unroll
+      for (int r = 0; r < 16; ++r) sA[(o0 + r) * 65 + o0 + l] = av[r];
     }
     __syncthreads();
     for (int L = 1; L < 4; ++L) {
       const int nb = 4 - L;
       for (int e = tid; e < nb * 256; e += FT) {
         const int J = e >> 8, rr = (e >> 4) & 15, cc = e & 15, I = J + L;
-        float acc = 0.f;
-        for (int K = J; K < I; ++K)
+        float acc[4] = {0.f, 0.f, 0.f, 0.f};
+        for (int K = J; K < I; ++K) {
+          const float *tr = sT + (16 * I + rr) * 65 + 16 * K;
+          const float *ac = sA + (16 * K) * 65 + 16 * J + cc;
 #pragma unroll
-          for (int m = 0; m < 16; ++m)
-            acc += sT[(16 * I + rr) * 65 + 16 * K + m] * sA[(16 * K + m) * 65 + 16 * J + cc];
-        sX[J * 256 + rr * 16 + cc] = acc;
+          for (int m = 0; m < 16; ++m) acc[m & 3] += tr[m] * ac[m * 65];
+        }
+        sX[J * 256 + rr * 16 + cc] = (acc[0] + acc[1]) + (acc[2] + acc[3]);
       }
       __syncthreads();
       for (int e = tid; e < nb * 256; e += FT) {
         const int J = e >> 8, rr = (e >> 4) & 15, cc = e & 15, I = J + L;
-        float acc = 0.f;
-        for (int m = 0; m <= rr; ++m) acc += sA[(16 * I + rr) * 65 + 16 * I + m] * sX[J * 256 + m * 16 + cc];
-        sA[(16 * I + rr) * 65 + 16 * J + cc] = -acc;
+        const float *dr = sA + (16 * I + rr) * 65 + 16 * I;
+        const float *xc = sX + J * 256 + cc;
+        float acc[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int m = 0; m < 16; ++m)
+          if (m <= rr) acc[m & 3] += dr[m] * xc[m * 16];
+        sA[(16 * I + rr) * 65 + 16 * J + cc] = -((acc[0] + acc[1]) + (acc[2] + acc[3]));
       }
       __syncthreads();
     }
-    // [A; 0] -> a2 (bf16, K-major, K = 64 source tokens)
-    for (int e = tid; e < 128 * 64; e += FT) {
-      const int r = e >> 6, s = e & 63;
-      const float val = (r < 64 && s <= r) ? sA[r * 65 + s] : 0.f;
-      *reinterpret_cast<__nv_bfloat16 *>(a2 + sw128_off(r, s)) = __float2bfloat16_rn(val);
+    // [A; 0] -> a2 (bf16, K-major, K = 64 source tokens), 16-byte chunks
+    for (int e = tid; e < 128 * 8; e += FT) {
+      const int r = e >> 3, cc = e & 7;
+      float v[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const int sidx = 8 * cc + j;
+        v[j] = (r < 64 && sidx <= r) ? sA[r * 65 + sidx] : 0.f;
+      }
+      sm16(a2, chunk_off(r, cc)) = pack_bf8(v);
     }
     fence_proxy_async();
     ok = __syncthreads_and(mbar_wait(bar_v, c & 1, kWaitIters));
@@ -437,13 +547,14 @@ __global__ void __launch_bounds__(FT, 1)
       const int r = 32 * wq + lane;
       for (int c0 = 0; c0 < 64; c0 += 16) {
         float v[16];
-        const int j0 = 64 * wh + c0;
+        const int j0 = 64 * wh + c0, sl = j0 >> 6, cc0 = (j0 & 63) >> 3;
         tmem_ld16(TW + lane_base + j0, v);
 #pragma unroll
-        for (int u = 0; u < 16; ++u) hw(a1l, 16384, r, j0 + u, -v[u]);
+        for (int u = 0; u < 16; ++u) v[u] = -v[u];
+        sm16(a1l, sl * 16384 + chunk_off(r, cc0)) = pack_h8(v);
+        sm16(a1l, sl * 16384 + chunk_off(r, cc0 + 1)) = pack_h8(v + 8);
       }
-      for (int s = 32 * wh; s < 32 * wh + 32; ++s)
-        *reinterpret_cast<__half *>(a2 + sw128_off(r, s)) = __float2half_rn(0.f);
+      for (int cc = 4 * wh; cc < 4 * wh + 4; ++cc) sm16(a2, chunk_off(r, cc)) = make_uint4(0, 0, 0, 0);
     } else {
       const int r = 32 * wq + lane - 64;
       for (int c0 = 0; c0 < 32; c0 += 16) {
@@ -452,8 +563,9 @@ __global__ void __launch_bounds__(FT, 1)
         tmem_ld16(TD1 + lane_base + s0, v);
 #pragma unroll
         for (int u = 0; u < 16; ++u)
-          *reinterpret_cast<__half *>(a2 + sw128_off(64 + r, s0 + u)) =
-              __float2half_rn(s0 + u <= r ? v[u] : 0.f);
+          if (s0 + u > r) v[u] = 0.f;
+        sm16(a2, chunk_off(64 + r, s0 >> 3)) = pack_h8(v);
+        sm16(a2, chunk_off(64 + r, (s0 >> 3) + 1)) = pack_h8(v + 8);
       }
     }
     {
@@ -461,20 +573,29 @@ __global__ void __launch_bounds__(FT, 1)
       const float gC = s_gC[i];
       for (int c0 = 0; c0 < 64; c0 += 16) {
         float v[16];
-        const int j0 = 64 * wh + c0;
+        const int j0 = 64 * wh + c0, sl = j0 >> 6, cc0 = (j0 & 63) >> 3;
         tmem_ld16(TS + lane_base + j0, v);
+        sm16(b3, sl * 16384 + chunk_off(i, cc0)) = pack_h8(v);
+        sm16(b3, sl * 16384 + chunk_off(i, cc0 + 1)) = pack_h8(v + 8);
 #pragma unroll
-        for (int u = 0; u < 16; ++u) {
-          hw(b3, 16384, i, j0 + u, v[u]);
-          v[u] *= gC;
-        }
+        for (int u = 0; u < 16; ++u) v[u] *= gC;
         tmem_st16(TS + lane_base + j0, v);
       }
     }
-    for (int e = tid; e < CM * D; e += FT) {
-      const int t = e >> 7, i = e & 127;
-      hw(a1l, 16384, 64 + t, i, bf2(kq, a1l, 16384, 64 + t, i));
-      hw(b1l, 8192, t, i, s_gC[i] * bf2(rw, b1l, 8192, t, i));
+    for (int m = 0; m < 4; ++m) {
+      const int t = 16 * m + 2 * warp + (lane >> 4), c8 = lane & 15, sl = c8 >> 3, cc = c8 & 7;
+      const uint32_t oq16 = sl * 16384 + 8192 + chunk_off(t, cc), o8 = sl * 8192 + chunk_off(t, cc);
+      float hv[8], lv[8];
+      unpack_bf8(sm16(kq, oq16), hv);
+      unpack_bf8(sm16(a1l, oq16), lv);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) hv[j] += lv[j];
+      sm16(a1l, oq16) = pack_h8(hv);
+      unpack_bf8(sm16(rw, o8), hv);
+      unpack_bf8(sm16(b1l, o8), lv);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) hv[j] = s_gC[8 * c8 + j] * (hv[j] + lv[j]);
+      sm16(b1l, o8) = pack_h8(hv);
     }
     tmem_st_wait();
     fence_proxy_async();
@@ -497,10 +618,10 @@ __global__ void __launch_bounds__(FT, 1)
       const int t = 32 * wq + lane;
       for (int c0 = 0; c0 < 64; c0 += 16) {
         float v[16];
-        const int j0 = 64 * wh + c0;
+        const int j0 = 64 * wh + c0, sl = j0 >> 6, cc0 = (j0 & 63) >> 3;
         tmem_ld16(TU + lane_base + j0, v);
-#pragma unroll
-        for (int u = 0; u < 16; ++u) hw(vr, 8192, t, j0 + u, v[u]);
+        sm16(vr, sl * 8192 + chunk_off(t, cc0)) = pack_h8(v);
+        sm16(vr, sl * 8192 + chunk_off(t, cc0 + 1)) = pack_h8(v + 8);
       }
     }
     fence_proxy_async();
@@ -520,26 +641,38 @@ __global__ void __launch_bounds__(FT, 1)
     if (!(ok = mma_wait())) break;
     tc_fence_after();
     if (tid == 0 && c + 1 < NC) issue_v(c + 1);  // R in vr has been consumed
-    // ---- [11] O (rows 64..127 of TU) -> global
+    // ---- [11] O (rows 64..127 of TU) -> 128-byte-swizzled staging tiles in fs
+    //           -> TMA bulk tensor stores (rows past T are not written)
     if (wq >= 2) {
-      const int t = 32 * wq + lane - 64, tt = c * CM + t;
+      const int t = 32 * wq + lane - 64;
+      unsigned char *stg = reinterpret_cast<unsigned char *>(fs);
       for (int c0 = 0; c0 < 64; c0 += 16) {
         float v[16];
         const int j0 = 64 * wh + c0;
         tmem_ld16(TU + lane_base + j0, v);
-        if (tt < a.T) {
-          const size_t o = tok_index(a, b, tt, h) * D + j0;
-          if (a.odt == KDN_BF16) {
-            __nv_bfloat162 *dst = reinterpret_cast<__nv_bfloat162 *>(static_cast<__nv_bfloat16 *>(a.o) + o);
+        if (a.odt == KDN_BF16) {
+          // box = 64 bf16 columns: box j0 / 64, chunks (j0 % 64) / 8 + {0, 1}
+          const int bx = j0 >> 6, cc = (j0 & 63) >> 3;
+          sm16(stg, bx * 8192 + chunk_off(t, cc)) = pack_bf8(v);
+          sm16(stg, bx * 8192 + chunk_off(t, cc + 1)) = pack_bf8(v + 8);
+        } else {
+          // box = 32 fp32 columns: box j0 / 32, chunks (j0 % 32) / 4 + {0..3}
+          const int bx = j0 >> 5, cc = (j0 & 31) >> 2;
 #pragma unroll
-            for (int u = 0; u < 8; ++u) dst[u] = __floats2bfloat162_rn(v[2 * u], v[2 * u + 1]);
-          } else {
-            float4 *dst = reinterpret_cast<float4 *>(static_cast<float *>(a.o) + o);
-#pragma unroll
-            for (int u = 0; u < 4; ++u) dst[u] = make_float4(v[4 * u], v[4 * u + 1], v[4 * u + 2], v[4 * u + 3]);
-          }
+          for (int m = 0; m < 4; ++m)
+            sm16(stg, bx * 8192 + chunk_off(t, cc + m)) =
+                make_uint4(__float_as_uint(v[4 * m]), __float_as_uint(v[4 * m + 1]),
+                           __float_as_uint(v[4 * m + 2]), __float_as_uint(v[4 * m + 3]));
         }
       }
+    }
+    fence_proxy_async();
+    __syncthreads();
+    if (tid == 0) {
+      const unsigned char *stg = reinterpret_cast<const unsigned char *>(fs);
+      const int nbox = a.odt == KDN_BF16 ? 2 : 4, bw = a.odt == KDN_BF16 ? 64 : 32;
+      for (int bx = 0; bx < nbox; ++bx) tma_store_4d(&mo, stg + bx * 8192, bx * bw, h, c * CM, b);
+      bulk_commit();
     }
     tc_fence_before();
     __syncthreads();
@@ -560,7 +693,7 @@ __global__ void __launch_bounds__(FT, 1)
       }
     }
     if (a.pT) {
-      if (V == 0 && tid < D) a.pT[(size_t)bh * D + tid] = pcarry;
+      if (V == 0 && tid < D) a.pT[(size_t)bh * D + tid] = s_p[tid];
       if (V == 1 && tid == 0) a.pT[bh] = s_b[0];
     }
   } else {
@@ -573,6 +706,7 @@ __global__ void __launch_bounds__(FT, 1)
       mbar_wait(bar_v, 1, kWaitIters);
     }
   }
+  if (tid == 0) bulk_wait_all();
   tc_fence_before();
   __syncthreads();
   if (warp == 0) tmem_dealloc(tb, 512);
@@ -595,18 +729,21 @@ PFN_cuTensorMapEncodeTiled_v12000 encoder() {
   return fn;
 }
 
-// [B, T, H, 128] bf16 tensor, box = 64 channels x 1 head x 64 tokens x 1 batch
-bool make_map(CUtensorMap *m, const void *ptr, const Args &a) {
+// [B, T, H, 128] tensor of 2- or 4-byte elements; box = 128 bytes of channels
+// x 1 head x 64 tokens x 1 batch, 128-byte swizzle.
+bool make_map(CUtensorMap *m, const void *ptr, const Args &a, bool fp32 = false) {
   auto enc = encoder();
   if (!enc) return false;
+  const cuuint64_t es_bytes = fp32 ? 4 : 2;
   cuuint64_t dims[4] = {(cuuint64_t)D, (cuuint64_t)a.H, (cuuint64_t)a.T, (cuuint64_t)a.B};
-  cuuint64_t strides[3] = {(cuuint64_t)D * 2, (cuuint64_t)a.H * D * 2,
-                           (cuuint64_t)a.T * a.H * D * 2};
-  cuuint32_t box[4] = {64, 1, 64, 1};
+  cuuint64_t strides[3] = {(cuuint64_t)D * es_bytes, (cuuint64_t)a.H * D * es_bytes,
+                           (cuuint64_t)a.T * a.H * D * es_bytes};
+  cuuint32_t box[4] = {fp32 ? 32u : 64u, 1, 64, 1};
   cuuint32_t es[4] = {1, 1, 1, 1};
-  return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void *>(ptr), dims, strides, box,
-             es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+  return enc(m, fp32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4,
+             const_cast<void *>(ptr), dims, strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
+             CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 }  // namespace
@@ -622,8 +759,9 @@ kdn_status_t launch_fused_fwd(const Args &a, cudaStream_t s) {
   P.a = a;
   P.has_g_map = (a.variant == 0 || a.pcd) ? 1 : 0;
   P.has_w_map = a.variant == 0 ? 1 : 0;
-  CUtensorMap mq, mk, mv, mg, mw;
-  if (!make_map(&mq, a.q, a) || !make_map(&mk, a.k, a) || !make_map(&mv, a.v, a))
+  CUtensorMap mq, mk, mv, mg, mw, mo;
+  if (!make_map(&mq, a.q, a) || !make_map(&mk, a.k, a) || !make_map(&mv, a.v, a) ||
+      !make_map(&mo, a.o, a, a.odt != KDN_BF16))
     return KDN_ERR_CUDA;
   mg = mq;
   mw = mq;
@@ -634,12 +772,12 @@ kdn_status_t launch_fused_fwd(const Args &a, cudaStream_t s) {
     if (cudaFuncSetAttribute(k_fused_fwd<0>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              SMEM_BYTES) != cudaSuccess)
       return KDN_ERR_CUDA;
-    k_fused_fwd<0><<<BH, FT, SMEM_BYTES, s>>>(mq, mk, mv, mg, mw, P);
+    k_fused_fwd<0><<<BH, FT, SMEM_BYTES, s>>>(mq, mk, mv, mg, mw, mo, P);
   } else {
     if (cudaFuncSetAttribute(k_fused_fwd<1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              SMEM_BYTES) != cudaSuccess)
       return KDN_ERR_CUDA;
-    k_fused_fwd<1><<<BH, FT, SMEM_BYTES, s>>>(mq, mk, mv, mg, mw, P);
+    k_fused_fwd<1><<<BH, FT, SMEM_BYTES, s>>>(mq, mk, mv, mg, mw, mo, P);
   }
   return cudaGetLastError() == cudaSuccess ? KDN_OK : KDN_ERR_CUDA;
 }
