@@ -37,6 +37,11 @@ constexpr int LC = CC + 1;
 // ---------------------------------------------------------------------------
 // Uncertainty recursion over time.
 
+// Tokens are processed in blocks of GU; the inputs of block n+1 are loaded
+// into registers before block n is computed, so the loads never sit on the
+// loop-carried dependence of the recursion.
+constexpr int GU = 16;
+
 template <typename DT>
 __global__ void __launch_bounds__(32) k_gain_scan_diag(Args a) {
   const int bh = blockIdx.x, b = bh / a.H, h = bh % a.H;
@@ -44,17 +49,37 @@ __global__ void __launch_bounds__(32) k_gain_scan_diag(Args a) {
   const int dk = a.dk;
   float p = a.p0 ? a.p0[(size_t)bh * dk + i] : 1.f;
   float *out = a.phat + (size_t)bh * a.Tp * dk + i;
-  for (int t = 0; t < a.T; ++t) {
-    const size_t th = tok_index(a, b, t, h);
-    const float gg = ld<DT>(a.g, th * dk + i);
-    const float w = ld<DT>(a.omega, th * dk + i);
-    const float kk = ld<DT>(a.k, th * dk + i);
-    const float rr = ld<DT>(a.r, th);
-    const float al2 = expf(2.f * gg);
-    const float ph = al2 * p + w;  // eq. diag-covariance-prediction
-    out[(size_t)t * dk] = ph;
-    const float u = a.mu * kk * kk / rr;  // eq. diag-cov-update
-    p = ph / (1.f + u * ph);
+  float cg[GU], cw[GU], ck[GU], cr[GU];
+  auto load = [&](int t0, float *g_, float *w_, float *k_, float *r_) {
+#pragma unroll
+    for (int j = 0; j < GU; ++j) {
+      const int t = t0 + j;
+      g_[j] = 0.f; w_[j] = 0.f; k_[j] = 0.f; r_[j] = 1.f;
+      if (t < a.T) {
+        const size_t th = tok_index(a, b, t, h);
+        g_[j] = ld<DT>(a.g, th * dk + i);
+        w_[j] = ld<DT>(a.omega, th * dk + i);
+        k_[j] = ld<DT>(a.k, th * dk + i);
+        r_[j] = ld<DT>(a.r, th);
+      }
+    }
+  };
+  load(0, cg, cw, ck, cr);
+  for (int t0 = 0; t0 < a.T; t0 += GU) {
+    float ng[GU], nw[GU], nk[GU], nr[GU];
+    load(t0 + GU, ng, nw, nk, nr);
+#pragma unroll
+    for (int j = 0; j < GU; ++j) {
+      if (t0 + j < a.T) {
+        const float al2 = expf(2.f * cg[j]);
+        const float ph = al2 * p + cw[j];  // eq. diag-covariance-prediction
+        out[(size_t)(t0 + j) * dk] = ph;
+        const float u = a.mu * ck[j] * ck[j] / cr[j];  // eq. diag-cov-update
+        p = ph / (1.f + u * ph);
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < GU; ++j) { cg[j] = ng[j]; cw[j] = nw[j]; ck[j] = nk[j]; cr[j] = nr[j]; }
   }
   for (int t = a.T; t < a.Tp; ++t) out[(size_t)t * dk] = 0.f;
   if (a.pT) a.pT[(size_t)bh * dk + i] = p;
@@ -64,34 +89,36 @@ template <typename DT>
 __global__ void __launch_bounds__(32) k_gain_scan_iso(Args a) {
   const int bh = blockIdx.x, b = bh / a.H, h = bh % a.H;
   const int lane = threadIdx.x, dk = a.dk;
-  __shared__ float s_a[32], s_n2[32];
+  __shared__ float s_a[32], s_n2[32], s_w[32], s_r[32];
   float bst = a.p0 ? a.p0[bh] : 1.f;
   for (int t0 = 0; t0 < a.T; t0 += 32) {
     const int t = t0 + lane;
-    float aa = 1.f, n2 = 0.f;
+    float aa = 1.f, n2 = 0.f, w = 0.f, rr = 1.f;
     if (t < a.T) {
       const size_t th = tok_index(a, b, t, h);
       float sa = 0.f;
+#pragma unroll 8
       for (int i = 0; i < dk; ++i) {
         const float kk = ld<DT>(a.k, th * dk + i);
         n2 += kk * kk;
         if (a.pcd) sa += expf(2.f * ld<DT>(a.g, th * dk + i));
       }
       aa = a.pcd ? sa / dk : expf(2.f * ld<DT>(a.g, th));
+      w = ld<DT>(a.omega, th);
+      rr = ld<DT>(a.r, th);
       a.isotok[((size_t)bh * a.Tp + t) * 2 + 0] = aa;
       a.isotok[((size_t)bh * a.Tp + t) * 2 + 1] = n2;
     }
     s_a[lane] = aa;
     s_n2[lane] = n2;
+    s_w[lane] = w;
+    s_r[lane] = rr;
     __syncwarp();
     if (lane == 0) {
       for (int j = 0; j < 32 && t0 + j < a.T; ++j) {
-        const size_t th = tok_index(a, b, t0 + j, h);
-        const float w = ld<DT>(a.omega, th);
-        const float rr = ld<DT>(a.r, th);
-        const float bhat = s_a[j] * bst + w;  // eq. iso-kla-box-cov-update
+        const float bhat = s_a[j] * bst + s_w[j];  // eq. iso-kla-box-cov-update
         a.phat[(size_t)bh * a.Tp + t0 + j] = bhat;
-        const float u = a.mu * s_n2[j] / (dk * rr);
+        const float u = a.mu * s_n2[j] / (dk * s_r[j]);
         bst = bhat / (1.f + u * bhat);
       }
     }
@@ -249,36 +276,88 @@ __global__ void __launch_bounds__(NT) k_chunk_prep(Args a) {
 }
 
 // ---------------------------------------------------------------------------
-// Inter-chunk state pass (forward).
+// Inter-chunk state passes.  The per-chunk factors (W, Qbar, K_tail, A_qk,
+// gamma_C and the chunk's U or dO slice) are double-buffered in shared memory
+// with cp.async, so chunk c+1 streams in while chunk c is computed.
+
+__device__ __forceinline__ uint32_t smem_addr(const void *p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+// 16-byte global -> shared copy; zero-filled when `valid` is false
+__device__ __forceinline__ void cp16(void *dst, const void *src, bool valid = true) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_addr(dst)), "l"(src),
+               "r"(valid ? 16 : 0)
+               : "memory");
+}
+__device__ __forceinline__ void cp_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
+template <int DK>
+struct StateBuf {
+  static constexpr int LD = DK + 4;  // 16-byte aligned rows
+  static constexpr int LA = CC + 4;
+  static constexpr int LS = CW + 4;
+  // floats per buffer: W, Qbar, K_tail, A_qk, gamma_C, and a [C][CW] slice (U or raw dO)
+  static constexpr int FLOATS = 3 * CC * LD + CC * LA + DK + CC * LS;
+};
+
+// Issues the cp.async copies of chunk c's factors into buffer `buf`.
+// `slice` is U (forward, fp32) or dO (backward, bytes of the activation dtype).
+template <int DK>
+__device__ void issue_chunk_factors(const Args &a, int bh, int c, float *buf, int j0,
+                                    bool backward) {
+  using SB = StateBuf<DK>;
+  float *sW = buf, *sQ = sW + CC * SB::LD, *sKt = sQ + CC * SB::LD, *sAqk = sKt + CC * SB::LD;
+  float *sgC = sAqk + CC * SB::LA, *sSl = sgC + DK;
+  const size_t base = (size_t)bh * a.NC + c;
+  constexpr int RC = DK / 4;  // 16-byte chunks per factor row
+  for (int e = KDN_TID; e < CC * RC; e += NT) {
+    const int r = e / RC, q = e % RC;
+    const size_t o = (base * CC + r) * DK + 4 * q;
+    cp16(sW + r * SB::LD + 4 * q, a.W + o);
+    cp16(sQ + r * SB::LD + 4 * q, a.Qb + o);
+    cp16(sKt + r * SB::LD + 4 * q, a.Kt + o);
+  }
+  for (int e = KDN_TID; e < CC * (CC / 4); e += NT) {
+    const int r = e / (CC / 4), q = e % (CC / 4);
+    cp16(sAqk + r * SB::LA + 4 * q, a.Aqk + base * CC * CC + r * CC + 4 * q);
+  }
+  for (int e = KDN_TID; e < DK / 4; e += NT) cp16(sgC + 4 * e, a.gC + base * DK + 4 * e);
+  if (!backward) {
+    for (int e = KDN_TID; e < CC * (CW / 4); e += NT) {
+      const int r = e / (CW / 4), q = e % (CW / 4);
+      cp16(sSl + r * SB::LS + 4 * q, a.U + (base * CC + r) * a.dv + j0 + 4 * q);
+    }
+  } else {
+    // raw dO rows of this slice: CW elements of the activation dtype
+    const int es = a.dtype == KDN_BF16 ? 2 : 4;
+    const int rc = CW * es / 16;
+    const int b = bh / a.H, h = bh % a.H;
+    for (int e = KDN_TID; e < CC * rc; e += NT) {
+      const int r = e / rc, q = e % rc, tt = c * CC + r;
+      const bool valid = tt < a.T;
+      const char *src = static_cast<const char *>(a.dO) +
+                        ((valid ? tok_index(a, b, tt, h) : 0) * a.dv + j0) * es + 16 * q;
+      cp16(reinterpret_cast<char *>(sSl + r * SB::LS) + 16 * q, src, valid);
+    }
+  }
+}
 
 template <int DK>
 constexpr size_t state_smem_bytes() {
-  return sizeof(float) * (DK * (CW + 1) + 3 * CC * (DK + 1) + CC * LC + 2 * CC * (CW + 1) + DK);
-}
-
-// Loads W, Qbar, K_tail, A_qk and gamma_C of one chunk into shared memory.
-template <int DK>
-__device__ void load_chunk_factors(const Args &a, size_t base, float *sW, float *sQ, float *sKt,
-                                   float *sAqk, float *s_gC) {
-  constexpr int LD = DK + 1;
-  for (int idx = KDN_TID; idx < CC * DK; idx += NT) {
-    const int r = idx / DK, i = idx % DK;
-    const size_t o = (base * CC + r) * DK + i;
-    sW[r * LD + i] = a.W[o];
-    sQ[r * LD + i] = a.Qb[o];
-    sKt[r * LD + i] = a.Kt[o];
-  }
-  for (int idx = KDN_TID; idx < CC * CC; idx += NT)
-    sAqk[(idx / CC) * LC + idx % CC] = a.Aqk[base * CC * CC + idx];
-  if (KDN_TID < DK) s_gC[KDN_TID] = a.gC[base * DK + KDN_TID];
+  using SB = StateBuf<DK>;
+  return sizeof(float) * (2 * SB::FLOATS + DK * SB::LS + CC * SB::LS);
 }
 
 template <typename DT, int DK>
 __global__ void __launch_bounds__(NT) k_state_fwd(Args a, int save_states) {
-  constexpr int LD = DK + 1, LS = CW + 1;
-  extern __shared__ float sm[];
-  float *sS = sm, *sW = sS + DK * LS, *sQ = sW + CC * LD, *sKt = sQ + CC * LD;
-  float *sAqk = sKt + CC * LD, *sR = sAqk + CC * LC, *sO = sR + CC * LS, *s_gC = sO + CC * LS;
+  using SB = StateBuf<DK>;
+  constexpr int LD = SB::LD, LA = SB::LA, LS = SB::LS;
+  extern __shared__ __align__(16) float sm[];
+  float *bufs = sm, *sS = bufs + 2 * SB::FLOATS, *sR = sS + DK * LS;
   const int bh = blockIdx.x, j0 = blockIdx.y * CW, tid = KDN_TID;
   const int b = bh / a.H, h = bh % a.H, dv = a.dv;
   const size_t sbase = (size_t)bh * DK * dv;
@@ -286,51 +365,63 @@ __global__ void __launch_bounds__(NT) k_state_fwd(Args a, int save_states) {
     const int i = idx / CW, j = idx % CW;
     sS[i * LS + j] = a.S0 ? a.S0[sbase + (size_t)i * dv + j0 + j] : 0.f;
   }
+  issue_chunk_factors<DK>(a, bh, 0, bufs, j0, false);
+  cp_commit();
   for (int c = 0; c < a.NC; ++c) {
-    const size_t base = (size_t)bh * a.NC + c;
+    float *buf = bufs + (c & 1) * SB::FLOATS;
+    if (c + 1 < a.NC) issue_chunk_factors<DK>(a, bh, c + 1, bufs + ((c + 1) & 1) * SB::FLOATS, j0, false);
+    cp_commit();
+    cp_wait<1>();
     __syncthreads();
+    float *sW = buf, *sQ = sW + CC * LD, *sKt = sQ + CC * LD, *sAqk = sKt + CC * LD;
+    float *sgC = sAqk + CC * LA, *sU = sgC + DK;
+    const size_t base = (size_t)bh * a.NC + c;
     if (save_states) {
       for (int idx = tid; idx < DK * CW; idx += NT) {
         const int i = idx / CW, j = idx % CW;
         a.Sin[(base * DK + i) * dv + j0 + j] = sS[i * LS + j];
       }
     }
-    load_chunk_factors<DK>(a, base, sW, sQ, sKt, sAqk, s_gC);
-    for (int idx = tid; idx < CC * CW; idx += NT) {
-      const int r = idx / CW, j = idx % CW;
-      sR[r * LS + j] = a.U[(base * CC + r) * dv + j0 + j];
-    }
-    __syncthreads();
     // R = U - W S_in
     for (int idx = tid; idx < CC * CW; idx += NT) {
       const int r = idx / CW, j = idx % CW;
-      float acc = 0.f;
+      float acc0 = 0.f, acc1 = 0.f;
 #pragma unroll 8
-      for (int i = 0; i < DK; ++i) acc += sW[r * LD + i] * sS[i * LS + j];
-      sR[r * LS + j] -= acc;
+      for (int i = 0; i < DK; i += 2) {
+        acc0 += sW[r * LD + i] * sS[i * LS + j];
+        acc1 += sW[r * LD + i + 1] * sS[(i + 1) * LS + j];
+      }
+      sR[r * LS + j] = sU[r * LS + j] - (acc0 + acc1);
     }
     __syncthreads();
     // O = Qbar S_in + A_qk R
     for (int idx = tid; idx < CC * CW; idx += NT) {
       const int r = idx / CW, j = idx % CW;
-      float acc = 0.f;
+      float acc0 = 0.f, acc1 = 0.f;
 #pragma unroll 8
-      for (int i = 0; i < DK; ++i) acc += sQ[r * LD + i] * sS[i * LS + j];
-      for (int s = 0; s <= r; ++s) acc += sAqk[r * LC + s] * sR[s * LS + j];
+      for (int i = 0; i < DK; i += 2) {
+        acc0 += sQ[r * LD + i] * sS[i * LS + j];
+        acc1 += sQ[r * LD + i + 1] * sS[(i + 1) * LS + j];
+      }
+      for (int s2 = 0; s2 <= r; ++s2) acc0 += sAqk[r * LA + s2] * sR[s2 * LS + j];
       const int tt = c * CC + r;
-      if (a.o && tt < a.T) sto(a.odt, a.o, tok_index(a, b, tt, h) * dv + j0 + j, acc);
+      if (a.o && tt < a.T) sto(a.odt, a.o, tok_index(a, b, tt, h) * dv + j0 + j, acc0 + acc1);
     }
     __syncthreads();
     // S_out = diag(gamma_C) S_in + K_tail^T R
     for (int idx = tid; idx < DK * CW; idx += NT) {
       const int i = idx / CW, j = idx % CW;
-      float acc = s_gC[i] * sS[i * LS + j];
+      float acc0 = sgC[i] * sS[i * LS + j], acc1 = 0.f;
 #pragma unroll 8
-      for (int s = 0; s < CC; ++s) acc += sKt[s * LD + i] * sR[s * LS + j];
-      sS[i * LS + j] = acc;
+      for (int s2 = 0; s2 < CC; s2 += 2) {
+        acc0 += sKt[s2 * LD + i] * sR[s2 * LS + j];
+        acc1 += sKt[(s2 + 1) * LD + i] * sR[(s2 + 1) * LS + j];
+      }
+      sS[i * LS + j] = acc0 + acc1;
     }
+    __syncthreads();
   }
-  __syncthreads();
+  cp_wait<0>();
   if (a.ST) {
     for (int idx = tid; idx < DK * CW; idx += NT) {
       const int i = idx / CW, j = idx % CW;
@@ -339,56 +430,67 @@ __global__ void __launch_bounds__(NT) k_state_fwd(Args a, int save_states) {
   }
 }
 
-// ---------------------------------------------------------------------------
-// Inter-chunk state pass (backward): dR = A_qk^T dO + K_tail dS_out,
-// dS_in = Qbar^T dO + diag(gamma_C) dS_out - W^T dR.
-
+// dR = A_qk^T dO + K_tail dS_out,  dS_in = Qbar^T dO + diag(gamma_C) dS_out - W^T dR
 template <typename DT, int DK>
 __global__ void __launch_bounds__(NT) k_state_bwd(Args a) {
-  constexpr int LD = DK + 1, LS = CW + 1;
-  extern __shared__ float sm[];
-  float *sS = sm, *sW = sS + DK * LS, *sQ = sW + CC * LD, *sKt = sQ + CC * LD;
-  float *sAqk = sKt + CC * LD, *sdR = sAqk + CC * LC, *sdO = sdR + CC * LS, *s_gC = sdO + CC * LS;
+  using SB = StateBuf<DK>;
+  constexpr int LD = SB::LD, LA = SB::LA, LS = SB::LS;
+  extern __shared__ __align__(16) float sm[];
+  float *bufs = sm, *sS = bufs + 2 * SB::FLOATS, *sdR = sS + DK * LS;
   const int bh = blockIdx.x, j0 = blockIdx.y * CW, tid = KDN_TID;
-  const int b = bh / a.H, h = bh % a.H, dv = a.dv;
+  const int dv = a.dv;
   const size_t sbase = (size_t)bh * DK * dv;
   for (int idx = tid; idx < DK * CW; idx += NT) {
     const int i = idx / CW, j = idx % CW;
     sS[i * LS + j] = a.dST ? a.dST[sbase + (size_t)i * dv + j0 + j] : 0.f;
   }
+  if (a.NC > 0) issue_chunk_factors<DK>(a, bh, a.NC - 1, bufs + ((a.NC - 1) & 1) * SB::FLOATS, j0, true);
+  cp_commit();
   for (int c = a.NC - 1; c >= 0; --c) {
-    const size_t base = (size_t)bh * a.NC + c;
+    float *buf = bufs + (c & 1) * SB::FLOATS;
+    if (c > 0) issue_chunk_factors<DK>(a, bh, c - 1, bufs + ((c - 1) & 1) * SB::FLOATS, j0, true);
+    cp_commit();
+    cp_wait<1>();
     __syncthreads();
+    float *sW = buf, *sQ = sW + CC * LD, *sKt = sQ + CC * LD, *sAqk = sKt + CC * LD;
+    float *sgC = sAqk + CC * LA;
+    const DT *sdO = reinterpret_cast<const DT *>(sgC + DK);
+    const size_t base = (size_t)bh * a.NC + c;
     for (int idx = tid; idx < DK * CW; idx += NT) {
       const int i = idx / CW, j = idx % CW;
       a.dSout[(base * DK + i) * dv + j0 + j] = sS[i * LS + j];
     }
-    load_chunk_factors<DK>(a, base, sW, sQ, sKt, sAqk, s_gC);
-    for (int idx = tid; idx < CC * CW; idx += NT) {
-      const int r = idx / CW, j = idx % CW, tt = c * CC + r;
-      sdO[r * LS + j] = tt < a.T ? ld<DT>(a.dO, tok_index(a, b, tt, h) * dv + j0 + j) : 0.f;
-    }
-    __syncthreads();
+    // dO row r of the slice starts LS floats apart (raw activation dtype)
+    auto dO = [&](int r, int j) -> float {
+      const DT *row = reinterpret_cast<const DT *>(reinterpret_cast<const float *>(sdO) + r * LS);
+      return ld<DT>(row, j);
+    };
     for (int idx = tid; idx < CC * CW; idx += NT) {
       const int r = idx / CW, j = idx % CW;
-      float acc = 0.f;
-      for (int s = r; s < CC; ++s) acc += sAqk[s * LC + r] * sdO[s * LS + j];
+      float acc0 = 0.f, acc1 = 0.f;
+      for (int s2 = r; s2 < CC; ++s2) acc0 += sAqk[s2 * LA + r] * dO(s2, j);
 #pragma unroll 8
-      for (int i = 0; i < DK; ++i) acc += sKt[r * LD + i] * sS[i * LS + j];
-      sdR[r * LS + j] = acc;
-      a.dR[(base * CC + r) * dv + j0 + j] = acc;
+      for (int i = 0; i < DK; i += 2) {
+        acc0 += sKt[r * LD + i] * sS[i * LS + j];
+        acc1 += sKt[r * LD + i + 1] * sS[(i + 1) * LS + j];
+      }
+      sdR[r * LS + j] = acc0 + acc1;
+      a.dR[(base * CC + r) * dv + j0 + j] = acc0 + acc1;
     }
     __syncthreads();
     for (int idx = tid; idx < DK * CW; idx += NT) {
       const int i = idx / CW, j = idx % CW;
-      float acc = s_gC[i] * sS[i * LS + j];
+      float acc0 = sgC[i] * sS[i * LS + j], acc1 = 0.f;
 #pragma unroll 8
-      for (int r = 0; r < CC; ++r)
-        acc += sQ[r * LD + i] * sdO[r * LS + j] - sW[r * LD + i] * sdR[r * LS + j];
-      sS[i * LS + j] = acc;
+      for (int r = 0; r < CC; r += 2) {
+        acc0 += sQ[r * LD + i] * dO(r, j) - sW[r * LD + i] * sdR[r * LS + j];
+        acc1 += sQ[(r + 1) * LD + i] * dO(r + 1, j) - sW[(r + 1) * LD + i] * sdR[(r + 1) * LS + j];
+      }
+      sS[i * LS + j] = acc0 + acc1;
     }
+    __syncthreads();
   }
-  __syncthreads();
+  cp_wait<0>();
   if (a.dS0) {
     for (int idx = tid; idx < DK * CW; idx += NT) {
       const int i = idx / CW, j = idx % CW;
@@ -650,38 +752,72 @@ __global__ void __launch_bounds__(32) k_gain_bwd_diag(Args a) {
   const int lane = threadIdx.x, i = blockIdx.y * 32 + lane, dk = a.dk;
   float dp = a.dpT ? a.dpT[(size_t)bh * dk + i] : 0.f;
   const size_t hrow = (size_t)bh * a.Tp;
-  // state before token T-1 is needed first: walk backwards, recomputing
-  // p_{t-1} from phat_{t-1} and u_{t-1}
-  for (int t = a.T - 1; t >= 0; --t) {
-    const size_t th = tok_index(a, b, t, h);
-    const size_t row = hrow + t;
-    const float ph = a.phat[row * dk + i];
-    const float kk = ld<DT>(a.k, th * dk + i);
-    const float rr = ld<DT>(a.r, th);
-    const float gg = ld<DT>(a.g, th * dk + i);
-    const float u = a.mu * kk * kk / rr;
-    const float den = 1.f + u * ph;
-    const float pt = ph / den;
-    const float dph = dp / (den * den) + a.dphloc[row * dk + i];
-    const float du = -dp * pt * pt;
-    const float dkk = a.dkpart[row * dk + i] + du * 2.f * a.mu * kk / rr;
-    const float drp = warp_sum(-du * u / rr);
-    if (lane == 0) a.drw[row * 4 + blockIdx.y] = drp;
-    float pprev;
-    if (t > 0) {
-      const size_t th1 = tok_index(a, b, t - 1, h);
-      const float k1 = ld<DT>(a.k, th1 * dk + i);
-      const float r1 = ld<DT>(a.r, th1);
-      const float ph1 = a.phat[(row - 1) * dk + i];
-      pprev = ph1 / (1.f + a.mu * k1 * k1 / r1 * ph1);
-    } else {
-      pprev = a.p0 ? a.p0[(size_t)bh * dk + i] : 1.f;
+  const float p_init = a.p0 ? a.p0[(size_t)bh * dk + i] : 1.f;
+  // per token: phat, k, r, g, local dphat, dk and dg partials; blocks of GU
+  // tokens walk backwards with the next (earlier) block prefetched
+  float cph[GU], ck[GU], cr[GU], cg[GU], cdl[GU], cdk[GU], cdg[GU];
+  auto load = [&](int t0, float *ph_, float *k_, float *r_, float *g_, float *dl_, float *dk_,
+                  float *dg_) {
+#pragma unroll
+    for (int j = 0; j < GU; ++j) {
+      const int t = t0 + j;
+      ph_[j] = 0.f; k_[j] = 0.f; r_[j] = 1.f; g_[j] = 0.f; dl_[j] = 0.f; dk_[j] = 0.f; dg_[j] = 0.f;
+      if (t >= 0 && t < a.T) {
+        const size_t th = tok_index(a, b, t, h), row = hrow + t;
+        ph_[j] = a.phat[row * dk + i];
+        k_[j] = ld<DT>(a.k, th * dk + i);
+        r_[j] = ld<DT>(a.r, th);
+        g_[j] = ld<DT>(a.g, th * dk + i);
+        dl_[j] = a.dphloc[row * dk + i];
+        dk_[j] = a.dkpart[row * dk + i];
+        dg_[j] = a.dgpart[row * dk + i];
+      }
     }
-    const float al2 = expf(2.f * gg);
-    sto(a.odt, a.domega, th * dk + i, dph);
-    sto(a.odt, a.dg, th * dk + i, a.dgpart[row * dk + i] + 2.f * al2 * pprev * dph);
-    sto(a.odt, a.dk_, th * dk + i, dkk);
-    dp = al2 * dph;
+  };
+  const int nblk = (a.T + GU - 1) / GU;
+  int t0 = (nblk - 1) * GU;
+  load(t0, cph, ck, cr, cg, cdl, cdk, cdg);
+  for (; t0 >= 0; t0 -= GU) {
+    float nph[GU], nk[GU], nr[GU], ng[GU], ndl[GU], ndk[GU], ndg[GU];
+    load(t0 - GU, nph, nk, nr, ng, ndl, ndk, ndg);
+    // posterior variance before the block: p_{t0-1}
+    float pprev_block = p_init;
+    if (t0 > 0) {
+      const float u1 = a.mu * nk[GU - 1] * nk[GU - 1] / nr[GU - 1];
+      pprev_block = nph[GU - 1] / (1.f + u1 * nph[GU - 1]);
+    }
+    // p_t for every token of the block (from phat_t and u_t)
+    float pt[GU];
+#pragma unroll
+    for (int j = 0; j < GU; ++j) {
+      const float u = a.mu * ck[j] * ck[j] / cr[j];
+      pt[j] = cph[j] / (1.f + u * cph[j]);
+    }
+#pragma unroll
+    for (int j = GU - 1; j >= 0; --j) {
+      const int t = t0 + j;
+      if (t < a.T) {
+        const size_t th = tok_index(a, b, t, h), row = hrow + t;
+        const float u = a.mu * ck[j] * ck[j] / cr[j];
+        const float den = 1.f + u * cph[j];
+        const float dph = dp / (den * den) + cdl[j];
+        const float du = -dp * pt[j] * pt[j];
+        const float dkk = cdk[j] + du * 2.f * a.mu * ck[j] / cr[j];
+        const float drp = warp_sum(-du * u / cr[j]);
+        if (lane == 0) a.drw[row * 4 + blockIdx.y] = drp;
+        const float pprev = j > 0 ? pt[j - 1] : pprev_block;
+        const float al2 = expf(2.f * cg[j]);
+        sto(a.odt, a.domega, th * dk + i, dph);
+        sto(a.odt, a.dg, th * dk + i, cdg[j] + 2.f * al2 * pprev * dph);
+        sto(a.odt, a.dk_, th * dk + i, dkk);
+        dp = al2 * dph;
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < GU; ++j) {
+      cph[j] = nph[j]; ck[j] = nk[j]; cr[j] = nr[j]; cg[j] = ng[j];
+      cdl[j] = ndl[j]; cdk[j] = ndk[j]; cdg[j] = ndg[j];
+    }
   }
   if (a.dp0) a.dp0[(size_t)bh * dk + i] = dp;
 }
@@ -703,34 +839,70 @@ __global__ void k_finalize_dr_diag(Args a) {
 template <typename DT>
 __global__ void __launch_bounds__(32) k_gain_bwd_iso(Args a) {
   const int bh = blockIdx.x, b = bh / a.H, h = bh % a.H;
-  if (threadIdx.x != 0) return;
+  const int lane = threadIdx.x;
+  __shared__ float s_ph[33], s_a[33], s_n2[33], s_r[33], s_dl[32], s_dr[32], s_o1[32], s_o2[32], s_dw[32];
   float db = a.dpT ? a.dpT[bh] : 0.f;
   const size_t hrow = (size_t)bh * a.Tp;
-  for (int t = a.T - 1; t >= 0; --t) {
-    const size_t th = tok_index(a, b, t, h), row = hrow + t;
-    const float bhat = a.phat[row];
-    const float aa = a.isotok[row * 2 + 0], n2 = a.isotok[row * 2 + 1];
-    const float rr = ld<DT>(a.r, th);
-    const float u = a.mu * n2 / (a.dk * rr);
-    const float den = 1.f + u * bhat;
-    const float bt = bhat / den;
-    const float dbh = db / (den * den) + a.dphloc[row];
-    const float du = -db * bt * bt;
-    a.drpart[row] += -du * u / rr;
-    float bprev;
-    if (t > 0) {
-      const float bh1 = a.phat[row - 1];
-      const float u1 = a.mu * a.isotok[(row - 1) * 2 + 1] / (a.dk * ld<DT>(a.r, tok_index(a, b, t - 1, h)));
-      bprev = bh1 / (1.f + u1 * bh1);
-    } else {
-      bprev = a.p0 ? a.p0[bh] : 1.f;
+  const int nblk = (a.T + 31) / 32;
+  for (int blk = nblk - 1; blk >= 0; --blk) {
+    const int t0 = blk * 32;
+    // lane j stages token t0 + j; slot 32 holds token t0 - 1
+    for (int j = lane; j < 33; j += 32) {
+      const int t = j < 32 ? t0 + j : t0 - 1;
+      float ph = 0.f, aa = 1.f, n2 = 0.f, rr = 1.f;
+      if (t >= 0 && t < a.T) {
+        const size_t row = hrow + t;
+        ph = a.phat[row];
+        aa = a.isotok[row * 2 + 0];
+        n2 = a.isotok[row * 2 + 1];
+        rr = ld<DT>(a.r, tok_index(a, b, t, h));
+        if (j < 32) {
+          s_dl[j] = a.dphloc[row];
+          s_dr[j] = a.drpart[row];
+        }
+      }
+      s_ph[j] = ph; s_a[j] = aa; s_n2[j] = n2; s_r[j] = rr;
     }
-    a.isoadj[row * 2 + 0] = du * a.mu / (a.dk * rr);  // d|k|^2 through u
-    a.isoadj[row * 2 + 1] = bprev * dbh;               // d a_t
-    sto(a.odt, a.domega, th, dbh);
-    db = aa * dbh;
+    __syncwarp();
+    if (lane == 0) {
+      for (int j = 31; j >= 0; --j) {
+        const int t = t0 + j;
+        if (t >= a.T) continue;
+        const float bhat = s_ph[j], rr = s_r[j];
+        const float u = a.mu * s_n2[j] / (a.dk * rr);
+        const float den = 1.f + u * bhat;
+        const float bt = bhat / den;
+        const float dbh = db / (den * den) + s_dl[j];
+        const float du = -db * bt * bt;
+        s_dr[j] += -du * u / rr;
+        float bprev;
+        if (j > 0 || t > 0) {
+          const int jj = j > 0 ? j - 1 : 32;
+          const float u1 = a.mu * s_n2[jj] / (a.dk * s_r[jj]);
+          bprev = s_ph[jj] / (1.f + u1 * s_ph[jj]);
+        } else {
+          bprev = a.p0 ? a.p0[bh] : 1.f;
+        }
+        s_o1[j] = du * a.mu / (a.dk * rr);  // d|k|^2 through u
+        s_o2[j] = bprev * dbh;              // d a_t
+        s_dw[j] = dbh;
+        db = s_a[j] * dbh;
+      }
+    }
+    __syncwarp();
+    {
+      const int t = t0 + lane;
+      if (t < a.T) {
+        const size_t row = hrow + t;
+        a.drpart[row] = s_dr[lane];
+        a.isoadj[row * 2 + 0] = s_o1[lane];
+        a.isoadj[row * 2 + 1] = s_o2[lane];
+        sto(a.odt, a.domega, tok_index(a, b, t, h), s_dw[lane]);
+      }
+    }
+    __syncwarp();
   }
-  if (a.dp0) a.dp0[bh] = db;
+  if (lane == 0 && a.dp0) a.dp0[bh] = db;
 }
 
 // per token: dk += 2 k d|k|^2, dg += d a_t * d a_t / d g, dr -> output dtype
