@@ -44,7 +44,7 @@ namespace {
 
 using namespace sm103;
 
-constexpr int FT = 256;   // threads
+constexpr int FT = 512;   // threads (16 warps)
 constexpr int CM = 64;    // chunk length
 constexpr int D = 128;    // head dim (dk = dv)
 constexpr uint32_t kWaitIters = 1u << 25;
@@ -62,8 +62,9 @@ constexpr int OFF_B1L = OFF_A1L + 32768;  // lo part of Kk -> K_tail fp16       
 constexpr int OFF_VR = OFF_B1L + 16384;   // V tile (TMA), later R in fp16        16 KB
 constexpr int OFF_A2 = OFF_VR + 16384;    // [A; 0] bf16 -> [0; A_qk] fp16        16 KB
 constexpr int OFF_B3 = OFF_A2 + 16384;    // S_in fp16 (MN-major)                 32 KB
-constexpr int OFF_F = OFF_B3 + 32768;     // fp32 scratch: Y [64][128] / T, A [64][65] + X
-constexpr int F_BYTES = 2 * 64 * 65 * 4 + 3 * 256 * 4;  // 36352 >= 32768
+constexpr int OFF_F = OFF_B3 + 32768;     // fp32 scratch: gamma [64][128] / T, A [64][LT] + X
+constexpr int LT = 68;                    // row stride of T and A (16-byte rows, conflict-free)
+constexpr int F_BYTES = 2 * 64 * LT * 4 + 3 * 256 * 4;  // 37888 >= 32768
 constexpr int OFF_SM = OFF_F + F_BYTES;                  // small arrays
 constexpr int SMALL_FLOATS = 64 * 7 + 128 * 3;
 constexpr int OFF_BAR = OFF_SM + SMALL_FLOATS * 4;
@@ -152,7 +153,7 @@ __global__ void __launch_bounds__(FT, 1)
   uint32_t *s_tbase = reinterpret_cast<uint32_t *>(bars + 4);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int wq = warp & 3, wh = warp >> 2;
+  const int wq = warp & 3, wg = warp >> 2;  // TMEM lane quarter, column group
   const int bh = blockIdx.x, b = bh / a.H, h = bh % a.H;
   const int NC = (a.T + CM - 1) / CM;
   const bool pcd = (V == 0) || a.pcd;
@@ -209,9 +210,9 @@ __global__ void __launch_bounds__(FT, 1)
   // initial memory S_0 -> TMEM (row = key channel i, column = value j)
   {
     const int i = 32 * wq + lane;
-    for (int c0 = 0; c0 < 64; c0 += 16) {
+    for (int c0 = 0; c0 < 32; c0 += 16) {
       float v[16];
-      const int j0 = 64 * wh + c0;
+      const int j0 = 32 * wg + c0;
       if (a.S0) {
         const float4 *src = reinterpret_cast<const float4 *>(a.S0 + ((size_t)bh * D + i) * D + j0);
 #pragma unroll
@@ -272,118 +273,150 @@ __global__ void __launch_bounds__(FT, 1)
     if (!ok) break;
     load_scalars(c + 1);
 
-    // ---- [2] the sequential recursions of this chunk: per channel (diag) the
-    //          uncertainty chain and the cumulative decay, per head (iso) the
-    //          scalar chain; results go to fp32 scratch (b3 and fs are free here)
+    // ---- [2] the sequential recursions of this chunk, split into four quarters
+    //          of 16 tokens: each quarter first forms the Moebius product of its
+    //          tokens (independent of the carry; eq. chunk-gain-summary), the
+    //          products are combined into the state entering each quarter
+    //          (eq. chunk-gain-carry), then every quarter runs its own 16 steps
+    //          (eq. chunk-gain-local-prefix, -emission).  Results go to fp32
+    //          scratch: phat to b3, gamma to fs (both free here).
     float *Pb = reinterpret_cast<float *>(b3);  // [64][128] phat_t
     float *Eb = fs;                             // [64][128] gamma_t
-    if (V == 0) {
-      // Warps 0-3 run tokens 0..31 of channel i from the carry.  Warps 4-7 first
-      // form the Moebius product M_31 ... M_0 (eq. chunk-gain-summary; it does not
-      // depend on the carry), apply it to z_in = [p_in, 1] (eq. chunk-gain-carry)
-      // and run tokens 32..63 (eq. chunk-gain-local-prefix, -emission).
-      const int i = tid & (D - 1);
-      const bool second = tid >= D;
-      const float p_in = s_p[i];
-      float p = p_in, e = 1.f;
-      if (second) {
-        float m00 = 1.f, m01 = 0.f, m10 = 0.f, m11 = 1.f;
-        for (int t0 = 0; t0 < 32; t0 += 8) {
-          float al[8], w[8], uk[8];
+    float *sQ = reinterpret_cast<float *>(a2);  // [4][128][5] per-quarter summaries (a2 is free)
+    float carry_out = 0.f, gc_out = 0.f;        // written after the closing barrier
+    {
+      const int i = tid & (D - 1), qq = tid >> 7, t0 = 16 * qq;
+      if (V == 0) {
+        float al[16], w[16], uk[16];
 #pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            const float kk = bf(kq, 16384, t0 + j, i);
-            al[j] = __expf(bf(rg, 8192, t0 + j, i));
-            w[j] = bf(rw, 8192, t0 + j, i);
-            uk[j] = a.mu * kk * kk * s_ri[t0 + j];
-          }
-#pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            const float a2 = al[j] * al[j], ua2 = uk[j] * a2, d1 = 1.f + uk[j] * w[j];
-            const float n00 = a2 * m00 + w[j] * m10, n01 = a2 * m01 + w[j] * m11;
-            const float n10 = ua2 * m00 + d1 * m10, n11 = ua2 * m01 + d1 * m11;
-            m00 = n00; m01 = n01; m10 = n10; m11 = n11;
-            e *= al[j];
-          }
-          // renormalise by the largest magnitude (the ratio n/d is scale free)
-          const float mx = fmaxf(fmaxf(fabsf(m00), fabsf(m01)), fmaxf(fabsf(m10), fabsf(m11)));
-          const float sc = 1.f / mx;
-          m00 *= sc; m01 *= sc; m10 *= sc; m11 *= sc;
-        }
-        p = __fdividef(m00 * p_in + m01, m10 * p_in + m11);
-      }
-      const int tb = second ? 32 : 0;
-      for (int t0 = tb; t0 < tb + 32; t0 += 8) {
-        float al[8], w[8], uk[8];
-#pragma unroll
-        for (int j = 0; j < 8; ++j) {
+        for (int j = 0; j < 16; ++j) {
           const float kk = bf(kq, 16384, t0 + j, i);
           al[j] = __expf(bf(rg, 8192, t0 + j, i));
           w[j] = bf(rw, 8192, t0 + j, i);
           uk[j] = a.mu * kk * kk * s_ri[t0 + j];
         }
+        float m00 = 1.f, m01 = 0.f, m10 = 0.f, m11 = 1.f, eq = 1.f;
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
+        for (int j = 0; j < 16; ++j) {
+          const float a2_ = al[j] * al[j], ua2 = uk[j] * a2_, d1 = 1.f + uk[j] * w[j];
+          const float n00 = a2_ * m00 + w[j] * m10, n01 = a2_ * m01 + w[j] * m11;
+          const float n10 = ua2 * m00 + d1 * m10, n11 = ua2 * m01 + d1 * m11;
+          m00 = n00; m01 = n01; m10 = n10; m11 = n11;
+          eq *= al[j];
+          if ((j & 7) == 7) {  // renormalise by the largest magnitude (n/d is scale free)
+            const float sc = __frcp_rn(fmaxf(fmaxf(fabsf(m00), fabsf(m01)), fmaxf(fabsf(m10), fabsf(m11))));
+            m00 *= sc; m01 *= sc; m10 *= sc; m11 *= sc;
+          }
+        }
+        float *mine = sQ + (qq * D + i) * 5;
+        mine[0] = m00; mine[1] = m01; mine[2] = m10; mine[3] = m11; mine[4] = eq;
+        __syncthreads();
+        float n = s_p[i], d = 1.f, e = 1.f;
+        for (int q2 = 0; q2 < qq; ++q2) {
+          const float *o = sQ + (q2 * D + i) * 5;
+          const float nn = o[0] * n + o[1] * d, dd = o[2] * n + o[3] * d;
+          const float sc = __frcp_rn(fmaxf(fabsf(nn), fabsf(dd)));
+          n = nn * sc;
+          d = dd * sc;
+          e *= o[4];
+        }
+        float p = __fdividef(n, d);
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
           e *= al[j];
           const float ph = al[j] * al[j] * p + w[j];  // eq. diag-covariance-prediction
           Pb[(t0 + j) * D + i] = ph;
           Eb[(t0 + j) * D + i] = e;
           p = __fdividef(ph, 1.f + uk[j] * ph);     // eq. prefix-diag-uncertainty
         }
-      }
-      __syncthreads();  // every thread has read s_p
-      if (second) {
-        s_p[i] = p;
-        s_gC[i] = e;
-      }
-    } else {
-      // per-token reductions a_t and |k_t|^2, one half-warp per token
-      for (int m = 0; m < 4; ++m) {
-        const int t = 16 * m + 2 * warp + (lane >> 4), c8 = lane & 15, sl = c8 >> 3, cc = c8 & 7;
-        float kv[8];
-        unpack_bf8(sm16(kq, sl * 16384 + chunk_off(t, cc)), kv);
-        float n2 = 0.f, sa = 0.f;
+        carry_out = p;
+        gc_out = e;
+      } else {
+        // per-token reductions a_t and |k_t|^2, one half-warp per token
+        for (int m = 0; m < 2; ++m) {
+          const int t = 32 * m + 2 * warp + (lane >> 4), c8 = lane & 15, sl = c8 >> 3, cc = c8 & 7;
+          float kv[8];
+          unpack_bf8(sm16(kq, sl * 16384 + chunk_off(t, cc)), kv);
+          float n2 = 0.f, sa = 0.f;
 #pragma unroll
-        for (int j = 0; j < 8; ++j) n2 += kv[j] * kv[j];
-        if (pcd) {
-          float gv[8];
-          unpack_bf8(sm16(rg, sl * 8192 + chunk_off(t, cc)), gv);
+          for (int j = 0; j < 8; ++j) n2 += kv[j] * kv[j];
+          if (pcd) {
+            float gv[8];
+            unpack_bf8(sm16(rg, sl * 8192 + chunk_off(t, cc)), gv);
 #pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            const float al = __expf(gv[j]);
-            sa += al * al;
+            for (int j = 0; j < 8; ++j) {
+              const float al = __expf(gv[j]);
+              sa += al * al;
+            }
+          }
+#pragma unroll
+          for (int o = 8; o > 0; o >>= 1) {
+            n2 += __shfl_xor_sync(0xffffffffu, n2, o);
+            sa += __shfl_xor_sync(0xffffffffu, sa, o);
+          }
+          if (c8 == 0) {
+            s_n2[t] = n2;
+            const float al = __expf(s_gs[t]);
+            s_a[t] = pcd ? sa / D : al * al;
           }
         }
+        __syncthreads();
+        // cumulative decay of channel i within this quarter
+        float el[16], eq = 1.f;
 #pragma unroll
-        for (int o = 8; o > 0; o >>= 1) {
-          n2 += __shfl_xor_sync(0xffffffffu, n2, o);
-          sa += __shfl_xor_sync(0xffffffffu, sa, o);
+        for (int j = 0; j < 16; ++j) {
+          eq *= __expf(pcd ? bf(rg, 8192, t0 + j, i) : s_gs[t0 + j]);
+          el[j] = eq;
         }
-        if (c8 == 0) {
-          s_n2[t] = n2;
-          const float al = __expf(s_gs[t]);
-          s_a[t] = pcd ? sa / D : al * al;
+        sQ[(qq * D + i) * 5 + 4] = eq;
+        // scalar Moebius product of this quarter (Prop. 5, eq. iso-kla-box-mobius)
+        if (i == 0) {
+          float m00 = 1.f, m01 = 0.f, m10 = 0.f, m11 = 1.f;
+          for (int j = 0; j < 16; ++j) {
+            const int t = t0 + j;
+            const float at = s_a[t], wt = s_om[t], ut = a.mu * s_n2[t] * s_ri[t] * (1.f / D);
+            const float n00 = at * m00 + wt * m10, n01 = at * m01 + wt * m11;
+            const float n10 = ut * at * m00 + (1.f + ut * wt) * m10;
+            const float n11 = ut * at * m01 + (1.f + ut * wt) * m11;
+            m00 = n00; m01 = n01; m10 = n10; m11 = n11;
+            if ((j & 7) == 7) {
+              const float sc = __frcp_rn(fmaxf(fmaxf(fabsf(m00), fabsf(m01)), fmaxf(fabsf(m10), fabsf(m11))));
+              m00 *= sc; m01 *= sc; m10 *= sc; m11 *= sc;
+            }
+          }
+          float *mine = sQ + (qq * D) * 5;
+          mine[0] = m00; mine[1] = m01; mine[2] = m10; mine[3] = m11;
+        }
+        __syncthreads();
+        float pre = 1.f;
+        for (int q2 = 0; q2 < qq; ++q2) pre *= sQ[(q2 * D + i) * 5 + 4];
+#pragma unroll
+        for (int j = 0; j < 16; ++j) Eb[(t0 + j) * D + i] = pre * el[j];
+        gc_out = pre * eq;
+        if (i == 0) {
+          float n = s_b[0], d = 1.f;
+          for (int q2 = 0; q2 < qq; ++q2) {
+            const float *o = sQ + (q2 * D) * 5;
+            const float nn = o[0] * n + o[1] * d, dd = o[2] * n + o[3] * d;
+            const float sc = __frcp_rn(fmaxf(fabsf(nn), fabsf(dd)));
+            n = nn * sc;
+            d = dd * sc;
+          }
+          float bb = __fdividef(n, d);
+          for (int j = 0; j < 16; ++j) {
+            const int t = t0 + j;
+            const float bhat = s_a[t] * bb + s_om[t];          // eq. iso-kla-box-cov-update
+            s_x[t] = __fdividef(bhat, s_r[t] + bhat * s_n2[t]);  // beta_t, eq. iso-kla-box-gain
+            bb = __fdividef(bhat, 1.f + a.mu * s_n2[t] * s_ri[t] * (1.f / D) * bhat);
+          }
+          carry_out = bb;
         }
       }
       __syncthreads();
-      if (tid < D) {
-        const int i = tid;
-        float e = 1.f;
-#pragma unroll 8
-        for (int t = 0; t < CM; ++t) {
-          e *= __expf(pcd ? bf(rg, 8192, t, i) : s_gs[t]);
-          Eb[t * D + i] = e;
-        }
-        s_gC[i] = e;
-      } else if (tid == D) {
-        // scalar recursion of Prop. 5 (eq. iso-kla-box-cov-update, -gain)
-        float bb = s_b[0];
-        for (int t = 0; t < CM; ++t) {
-          const float bhat = s_a[t] * bb + s_om[t];
-          s_x[t] = __fdividef(bhat, s_r[t] + bhat * s_n2[t]);
-          bb = __fdividef(bhat, 1.f + a.mu * s_n2[t] * s_ri[t] * (1.f / D) * bhat);
-        }
-        s_b[0] = bb;
+      if (qq == 3) {
+        s_gC[i] = gc_out;
+        if (V == 0) s_p[i] = carry_out;
+        else if (i == 0) s_b[0] = carry_out;
       }
     }
     __syncthreads();
@@ -392,8 +425,8 @@ __global__ void __launch_bounds__(FT, 1)
     //   Kk = phat k / (s_t gamma) (diag, s_t = r_t + sum phat k^2) or beta_t k / gamma (iso)
     //   Kbar = gamma k, Qbar = tau gamma q; each as a hi/lo bf16 pair, written over
     //   the raw tiles (hi) and into the lo buffers
-    for (int m = 0; m < 4; ++m) {
-      const int t = 16 * m + 2 * warp + (lane >> 4), c8 = lane & 15, sl = c8 >> 3, cc = c8 & 7;
+    for (int m = 0; m < 2; ++m) {
+      const int t = 32 * m + 2 * warp + (lane >> 4), c8 = lane & 15, sl = c8 >> 3, cc = c8 & 7;
       const uint32_t ok16 = sl * 16384 + chunk_off(t, cc), oq16 = ok16 + 8192;
       const uint32_t o8 = sl * 8192 + chunk_off(t, cc);
       float kv[8], qv[8], ev[8], xv[8];
@@ -454,60 +487,89 @@ __global__ void __launch_bounds__(FT, 1)
     if (!(ok = mma_wait())) break;
     tc_fence_after();
     // ---- [5] T -> fp32 smem, A = (I + T)^-1 by 16x16 blocks:
-    //   diagonal blocks D_I = (I + T_II)^-1 by forward substitution (a column per lane),
+    //   diagonal blocks D_I = (I + T_II)^-1 by column substitution (rows across a half-warp),
     //   then A_IJ = -D_I sum_{K=J}^{I-1} T_IK A_KJ level by level (I - J = 1, 2, 3)
-    float *sT = fs, *sA = fs + 64 * 65, *sX = fs + 2 * 64 * 65;
+    float *sT = fs, *sA = fs + 64 * LT, *sX = fs + 2 * 64 * LT;
     if (wq < 2) {
-      const int r = 32 * wq + lane;
-      for (int c0 = 0; c0 < 32; c0 += 16) {
-        float v[16];
-        const int s0 = 32 * wh + c0;
-        tmem_ld16(TD1 + lane_base + s0, v);
+      const int r = 32 * wq + lane, s0 = 16 * wg;
+      float v[16];
+      tmem_ld16(TD1 + lane_base + s0, v);
 #pragma unroll
-        for (int u = 0; u < 16; ++u) sT[r * 65 + s0 + u] = (s0 + u < r) ? v[u] : 0.f;
-      }
+      for (int u = 0; u < 16; ++u)
+        if (s0 + u >= r) v[u] = 0.f;
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+        *reinterpret_cast<float4 *>(sT + r * LT + s0 + 4 * u) = make_float4(v[4 * u], v[4 * u + 1], v[4 * u + 2], v[4 * u + 3]);
     }
     __syncthreads();
-    if (warp < 4 && lane < 16) {
-      const int o0 = 16 * warp, l = lane;
-      float av[16];
+    {
+      // diagonal block I = warp / 4, columns c, c + 1 (c = 4 (warp % 4) + 2 (lane / 16));
+      // lane % 16 is the row.  Column substitution: once x_s is final it is broadcast
+      // along the half-warp and every lower row subtracts T_rs x_s.
+      const int o0 = 16 * (warp >> 2), rr = lane & 15, cl = 4 * (warp & 3) + 2 * (lane >> 4);
+      float trow[16];
 #pragma unroll
-      for (int r = 0; r < 16; ++r) {
-        float acc0 = (r == l) ? 1.f : 0.f, acc1 = 0.f;
-#pragma unroll
-        for (int q2 = 0; q2 < r; q2 += 2) {
-          acc0 -= sT[(o0 + r) * 65 + o0 + q2] * av[q2];
-          if (q2 + 1 < r) acc1 -= sT[(o0 + r) * 65 + o0 + q2 + 1] * av[q2 + 1];
-        }
-        av[r] = acc0 + acc1;
+      for (int u = 0; u < 4; ++u) {  // 0 for columns >= rr
+        const float4 t4 = *reinterpret_cast<const float4 *>(sT + (o0 + rr) * LT + o0 + 4 * u);
+        trow[4 * u] = t4.x; trow[4 * u + 1] = t4.y; trow[4 * u + 2] = t4.z; trow[4 * u + 3] = t4.w;
       }
+      float x0 = (rr == cl) ? 1.f : 0.f, x1 = (rr == cl + 1) ? 1.f : 0.f;
 #pragma unroll
-      for (int r = 0; r < 16; ++r) sA[(o0 + r) * 65 + o0 + l] = av[r];
+      for (int s2 = 0; s2 < 15; ++s2) {
+        const float y0 = __shfl_sync(0xffffffffu, x0, s2, 16);
+        const float y1 = __shfl_sync(0xffffffffu, x1, s2, 16);
+        x0 -= trow[s2] * y0;
+        x1 -= trow[s2] * y1;
+      }
+      sA[(o0 + rr) * LT + o0 + cl] = x0;  // zero above the diagonal
+      sA[(o0 + rr) * LT + o0 + cl + 1] = x1;
     }
     __syncthreads();
+    // off-diagonal levels: one thread per (block J, row, 4 columns), float4 operands
     for (int L = 1; L < 4; ++L) {
       const int nb = 4 - L;
-      for (int e = tid; e < nb * 256; e += FT) {
-        const int J = e >> 8, rr = (e >> 4) & 15, cc = e & 15, I = J + L;
-        float acc[4] = {0.f, 0.f, 0.f, 0.f};
+      const int J = tid >> 6, rr = (tid >> 2) & 15, cg = tid & 3, I = J + L;
+      if (J < nb) {
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
         for (int K = J; K < I; ++K) {
-          const float *tr = sT + (16 * I + rr) * 65 + 16 * K;
-          const float *ac = sA + (16 * K) * 65 + 16 * J + cc;
+          const float *tr = sT + (16 * I + rr) * LT + 16 * K;
+          const float *ac = sA + (16 * K) * LT + 16 * J + 4 * cg;
 #pragma unroll
-          for (int m = 0; m < 16; ++m) acc[m & 3] += tr[m] * ac[m * 65];
+          for (int m4 = 0; m4 < 4; ++m4) {
+            const float4 t4 = *reinterpret_cast<const float4 *>(tr + 4 * m4);
+            const float tv[4] = {t4.x, t4.y, t4.z, t4.w};
+#pragma unroll
+            for (int mm = 0; mm < 4; ++mm) {
+              const float4 a4 = *reinterpret_cast<const float4 *>(ac + (4 * m4 + mm) * LT);
+              acc.x += tv[mm] * a4.x;
+              acc.y += tv[mm] * a4.y;
+              acc.z += tv[mm] * a4.z;
+              acc.w += tv[mm] * a4.w;
+            }
+          }
         }
-        sX[J * 256 + rr * 16 + cc] = (acc[0] + acc[1]) + (acc[2] + acc[3]);
+        *reinterpret_cast<float4 *>(sX + J * 256 + rr * 16 + 4 * cg) = acc;
       }
       __syncthreads();
-      for (int e = tid; e < nb * 256; e += FT) {
-        const int J = e >> 8, rr = (e >> 4) & 15, cc = e & 15, I = J + L;
-        const float *dr = sA + (16 * I + rr) * 65 + 16 * I;
-        const float *xc = sX + J * 256 + cc;
-        float acc[4] = {0.f, 0.f, 0.f, 0.f};
+      if (J < nb) {
+        const float *dr = sA + (16 * I + rr) * LT + 16 * I;
+        const float *xc = sX + J * 256 + 4 * cg;
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
-        for (int m = 0; m < 16; ++m)
-          if (m <= rr) acc[m & 3] += dr[m] * xc[m * 16];
-        sA[(16 * I + rr) * 65 + 16 * J + cc] = -((acc[0] + acc[1]) + (acc[2] + acc[3]));
+        for (int m4 = 0; m4 < 4; ++m4) {
+          const float4 d4 = *reinterpret_cast<const float4 *>(dr + 4 * m4);
+          const float dv[4] = {d4.x, d4.y, d4.z, d4.w};
+#pragma unroll
+          for (int mm = 0; mm < 4; ++mm) {
+            const float4 x4 = *reinterpret_cast<const float4 *>(xc + (4 * m4 + mm) * 16);
+            acc.x += dv[mm] * x4.x;
+            acc.y += dv[mm] * x4.y;
+            acc.z += dv[mm] * x4.z;
+            acc.w += dv[mm] * x4.w;
+          }
+        }
+        *reinterpret_cast<float4 *>(sA + (16 * I + rr) * LT + 16 * J + 4 * cg) =
+            make_float4(-acc.x, -acc.y, -acc.z, -acc.w);
       }
       __syncthreads();
     }
@@ -518,7 +580,7 @@ __global__ void __launch_bounds__(FT, 1)
 #pragma unroll
       for (int j = 0; j < 8; ++j) {
         const int sidx = 8 * cc + j;
-        v[j] = (r < 64 && sidx <= r) ? sA[r * 65 + sidx] : 0.f;
+        v[j] = (r < 64 && sidx <= r) ? sA[r * LT + sidx] : 0.f;
       }
       sm16(a2, chunk_off(r, cc)) = pack_bf8(v);
     }
@@ -545,35 +607,32 @@ __global__ void __launch_bounds__(FT, 1)
     //   b3 <- S_in (and diag(gamma_C) S_in back to TMEM);  b1l <- K_tail
     if (wq < 2) {
       const int r = 32 * wq + lane;
-      for (int c0 = 0; c0 < 64; c0 += 16) {
+      for (int c0 = 0; c0 < 32; c0 += 16) {
         float v[16];
-        const int j0 = 64 * wh + c0, sl = j0 >> 6, cc0 = (j0 & 63) >> 3;
+        const int j0 = 32 * wg + c0, sl = j0 >> 6, cc0 = (j0 & 63) >> 3;
         tmem_ld16(TW + lane_base + j0, v);
 #pragma unroll
         for (int u = 0; u < 16; ++u) v[u] = -v[u];
         sm16(a1l, sl * 16384 + chunk_off(r, cc0)) = pack_h8(v);
         sm16(a1l, sl * 16384 + chunk_off(r, cc0 + 1)) = pack_h8(v + 8);
       }
-      for (int cc = 4 * wh; cc < 4 * wh + 4; ++cc) sm16(a2, chunk_off(r, cc)) = make_uint4(0, 0, 0, 0);
+      for (int cc = 2 * wg; cc < 2 * wg + 2; ++cc) sm16(a2, chunk_off(r, cc)) = make_uint4(0, 0, 0, 0);
     } else {
-      const int r = 32 * wq + lane - 64;
-      for (int c0 = 0; c0 < 32; c0 += 16) {
-        float v[16];
-        const int s0 = 32 * wh + c0;
-        tmem_ld16(TD1 + lane_base + s0, v);
+      const int r = 32 * wq + lane - 64, s0 = 16 * wg;
+      float v[16];
+      tmem_ld16(TD1 + lane_base + s0, v);
 #pragma unroll
-        for (int u = 0; u < 16; ++u)
-          if (s0 + u > r) v[u] = 0.f;
-        sm16(a2, chunk_off(64 + r, s0 >> 3)) = pack_h8(v);
-        sm16(a2, chunk_off(64 + r, (s0 >> 3) + 1)) = pack_h8(v + 8);
-      }
+      for (int u = 0; u < 16; ++u)
+        if (s0 + u > r) v[u] = 0.f;
+      sm16(a2, chunk_off(64 + r, s0 >> 3)) = pack_h8(v);
+      sm16(a2, chunk_off(64 + r, (s0 >> 3) + 1)) = pack_h8(v + 8);
     }
     {
       const int i = 32 * wq + lane;
       const float gC = s_gC[i];
-      for (int c0 = 0; c0 < 64; c0 += 16) {
+      for (int c0 = 0; c0 < 32; c0 += 16) {
         float v[16];
-        const int j0 = 64 * wh + c0, sl = j0 >> 6, cc0 = (j0 & 63) >> 3;
+        const int j0 = 32 * wg + c0, sl = j0 >> 6, cc0 = (j0 & 63) >> 3;
         tmem_ld16(TS + lane_base + j0, v);
         sm16(b3, sl * 16384 + chunk_off(i, cc0)) = pack_h8(v);
         sm16(b3, sl * 16384 + chunk_off(i, cc0 + 1)) = pack_h8(v + 8);
@@ -582,8 +641,8 @@ __global__ void __launch_bounds__(FT, 1)
         tmem_st16(TS + lane_base + j0, v);
       }
     }
-    for (int m = 0; m < 4; ++m) {
-      const int t = 16 * m + 2 * warp + (lane >> 4), c8 = lane & 15, sl = c8 >> 3, cc = c8 & 7;
+    for (int m = 0; m < 2; ++m) {
+      const int t = 32 * m + 2 * warp + (lane >> 4), c8 = lane & 15, sl = c8 >> 3, cc = c8 & 7;
       const uint32_t oq16 = sl * 16384 + 8192 + chunk_off(t, cc), o8 = sl * 8192 + chunk_off(t, cc);
       float hv[8], lv[8];
       unpack_bf8(sm16(kq, oq16), hv);
@@ -616,9 +675,9 @@ __global__ void __launch_bounds__(FT, 1)
     // ---- [9] R -> fp16 vr (MN-major [64 tok][128 dv])
     if (wq < 2) {
       const int t = 32 * wq + lane;
-      for (int c0 = 0; c0 < 64; c0 += 16) {
+      for (int c0 = 0; c0 < 32; c0 += 16) {
         float v[16];
-        const int j0 = 64 * wh + c0, sl = j0 >> 6, cc0 = (j0 & 63) >> 3;
+        const int j0 = 32 * wg + c0, sl = j0 >> 6, cc0 = (j0 & 63) >> 3;
         tmem_ld16(TU + lane_base + j0, v);
         sm16(vr, sl * 8192 + chunk_off(t, cc0)) = pack_h8(v);
         sm16(vr, sl * 8192 + chunk_off(t, cc0 + 1)) = pack_h8(v + 8);
@@ -646,9 +705,9 @@ __global__ void __launch_bounds__(FT, 1)
     if (wq >= 2) {
       const int t = 32 * wq + lane - 64;
       unsigned char *stg = reinterpret_cast<unsigned char *>(fs);
-      for (int c0 = 0; c0 < 64; c0 += 16) {
+      for (int c0 = 0; c0 < 32; c0 += 16) {
         float v[16];
-        const int j0 = 64 * wh + c0;
+        const int j0 = 32 * wg + c0;
         tmem_ld16(TU + lane_base + j0, v);
         if (a.odt == KDN_BF16) {
           // box = 64 bf16 columns: box j0 / 64, chunks (j0 % 64) / 8 + {0, 1}
@@ -683,9 +742,9 @@ __global__ void __launch_bounds__(FT, 1)
     // final state
     if (a.ST) {
       const int i = 32 * wq + lane;
-      for (int c0 = 0; c0 < 64; c0 += 16) {
+      for (int c0 = 0; c0 < 32; c0 += 16) {
         float v[16];
-        const int j0 = 64 * wh + c0;
+        const int j0 = 32 * wg + c0;
         tmem_ld16(TS + lane_base + j0, v);
         float4 *dst = reinterpret_cast<float4 *>(a.ST + ((size_t)bh * D + i) * D + j0);
 #pragma unroll
