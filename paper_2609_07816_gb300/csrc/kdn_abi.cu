@@ -60,6 +60,7 @@ kdn_status_t fill_sizes(const kdn_desc_t *d, int variant, bool decode, Args *a) 
 // The fused forward serves bf16 activations with dk = dv = 128 and the default
 // (or 64-token) chunk; everything else runs the general chunked kernels.
 bool use_fused(const Args &a) { return a.chunk != 32 && fused_fwd_supported(a); }
+bool use_fused_bwd(const Args &a) { return fused_bwd_supported(a); }
 
 bool ptrs_ok(std::initializer_list<const void *> required,
              std::initializer_list<const void *> optional) {
@@ -158,6 +159,7 @@ kdn_status_t bwd_entry(int variant, const kdn_desc_t *d, const void *q, const vo
   if (cudaMemsetAsync(a.status, 0, sizeof(unsigned), s) != cudaSuccess) return KDN_ERR_CUDA;
   if ((size_t)a.B * a.H == 0) return KDN_OK;
   if (a.T == 0) return empty_bwd(a, s);
+  if (use_fused_bwd(a)) return launch_fused_bwd(a, s);
   return launch_chunked_bwd(a, s);
 }
 
@@ -186,6 +188,12 @@ size_t workspace_layout(Args *a, char *base, bool bwd) {
   };
   a->status = reinterpret_cast<unsigned *>(take(kAlign / sizeof(float)));
   if (!bwd && use_fused(*a)) return off;
+  if (bwd && a->T > 0 && use_fused_bwd(*a)) {
+    const size_t NC64 = (a->T + 63) / 64;  // the fused kernels use 64-token chunks
+    a->fSin = reinterpret_cast<unsigned char *>(take(BH * NC64 * 32768 / sizeof(float)));
+    a->fpin = take(BH * NC64 * dk);
+    return off;
+  }
   a->phat = take(BH * Tp * P);
   a->isotok = a->variant == 1 ? take(BH * Tp * 2) : nullptr;
   a->W = take(BH * NC * C * dk);
@@ -293,7 +301,7 @@ int kdn_kernel_launches(const kdn_desc_t *desc, int variant, int op) {
   if (fill_sizes(desc, variant, op == 2, &a) != KDN_OK) return -1;
   switch (op) {
     case 0: return use_fused(a) ? 1 : chunked_fwd_launches(a);
-    case 1: return chunked_bwd_launches(a);
+    case 1: return (a.T > 0 && use_fused_bwd(a)) ? 2 : chunked_bwd_launches(a);
     case 2: return 1;
   }
   return -1;

@@ -1,0 +1,995 @@
+// kdn_fused_bwd.cu -- fused chunked backward of the Diagonal KDN for bfloat16
+// activations with d_k = d_v = 128 and 64-token chunks (App. F), on the
+// tcgen05 tensor cores of sm_103a.
+//
+// Two launches:
+//  1. the fused forward in its state-saving mode stores, per chunk, the fp16
+//     image of the entry memory S_in (the tile MMA-S1 consumes) and the
+//     uncertainty p entering the chunk;
+//  2. k_fused_bwd: one CTA per (batch, head) walks the chunks backwards.  The
+//     memory cotangent dS (128 x 128 fp32) stays in tensor memory for the whole
+//     sweep; the uncertainty cotangent dp (one value per channel) is carried in
+//     shared memory.
+// Per chunk (notation of App. F.2: Kbar = Gamma.K, Kk = Kbar^kappa, Qbar = tau
+// Gamma.Q, A = (I + T)^-1, W = A Kbar, U = A V, R = U - W S_in, K_tail =
+// gamma_C.Kk) the kernel recomputes the forward factors and forms the adjoint of
+// O = Qbar S_in + A_qk R,  S_out = diag(gamma_C) S_in + K_tail^T R:
+//   dR     = A_qk^T dO + K_tail dS                      (B1)
+//   dS_in  = diag(gamma_C) dS + Qbar^T dO - W^T dR      (B2)
+//   dA_qk  = lower(dO R^T),  dK_tail = R dS^T           (B3, B4)
+//   dW     = -dR S_in^T,     dV = A^T dR                (B5, B7)
+//   dQbar  = dO S_in^T + dA_qk Kk                       (B8)
+//   dA     = dR V^T + dW Kbar^T,  dT = strict_lower(-A^T dA A^T)   (B6, X, Y)
+//   dKk    = dA_qk^T Qbar + gamma_C.dK_tail + dT^T Kbar (B9)
+//   dKbar  = A^T dW + dT Kk                             (B10)
+//   dgamma_C = colsum(dK_tail.Kk) + rowsum(dS.S_in)
+// and then, per channel on CUDA cores, the adjoint of the scaling by Gamma and
+// of the gain emission (eq. chunk-gain-emission, eq. kla-box-gain) and of the
+// uncertainty recursion (eq. diag-covariance-prediction, eq. prefix-diag-
+// uncertainty) backwards over the chunk's tokens.
+//
+// Every product runs as a cta_group::1, M = 128 MMA.  Products whose natural
+// row count is 64 read 64 further rows of whatever follows the operand in
+// shared memory; those accumulator rows are never read.  The matrices with
+// 128 rows (channels) are computed transposed, so that channel i is TMEM lane i
+// and the per-channel recursions read their operands straight from TMEM.
+//
+// Precision: the Gamma-scaled operands Kbar, Qbar, Kk and dA_qk (exp(+-G)
+// factors) are split into hi + lo bf16 pairs where they meet one another;
+// everything else is fp16 (10-bit mantissa).  The cotangents are scaled by a
+// power of two lambda (from max|dO| and max|dS_T| of the head) before they
+// enter fp16, and every gradient is scaled back by 1/lambda, so the fp16 range
+// holds for any magnitude of the incoming cotangents.
+//
+// Every wait on an mbarrier is bounded; on timeout the kernel records
+// KDN_ERR_TIMEOUT in the workspace status word and returns.
+#include "kdn_internal.cuh"
+#include "kdn_sm103.cuh"
+#include "kdn_fused_common.cuh"
+
+namespace kdn {
+namespace {
+
+using namespace sm103;
+using namespace fused;
+
+constexpr int BT = 512;  // threads (16 warps)
+constexpr int CM = 64;   // chunk length
+constexpr int D = 128;   // head dim (dk = dv)
+constexpr uint32_t kWaitIters = 1u << 25;
+constexpr int KB = 1024;
+
+// Shared-memory map (bytes from the 1024-aligned base).  Regions are reused
+// across the stages of a chunk; the comments give the sequence of tenants.
+constexpr int O_RKQ = 0;         // raw k | q, interleaved per 64-channel slab (whole chunk)
+constexpr int O_SIN = 32 * KB;   // S_in fp16 [i][j]  -> [Kbar; Qbar] hi (second operand set)
+constexpr int O_RV = 64 * KB;    // raw v  -> v fp16
+constexpr int O_RDO = 80 * KB;   // raw dO -> lambda dO fp16 -> Qbar lo (second set)
+constexpr int O_RG = 96 * KB;    // raw g  -> Kk lo (first set) -> T fp32 -> A bf16 | A fp16
+constexpr int O_RW = 112 * KB;   // raw omega -> Kk hi (first set) -> (T) | A_qk fp16 -> dT bf16
+constexpr int O_KQH = 128 * KB;  // [Kbar; Qbar] hi (first) -> -W fp16 | K_tail -> Kk hi | dR^T
+constexpr int O_KQL = 160 * KB;  // [Kbar; Qbar] lo (first) -> A fp32 -> dS fp16 -> dA_qk^T | Qbar
+                                 //   fp16 -> dW^T | Kk lo -> dA^T | X
+constexpr int O_RH = 192 * KB;   // R fp16 (16 KB; the next 8 KB are read as padding rows)
+                                 //   -> lo part of dR^T fp16 -> per-channel scratch
+constexpr int BUF_END = 216 * KB;
+// derived tenants
+constexpr int O_AB = O_RG, O_AH = O_RG + 8 * KB, O_AQ = O_RW + 8 * KB, O_DT = O_RW;
+constexpr int O_WN = O_KQH, O_KT = O_KQH + 16 * KB, O_DRT = O_KQH + 16 * KB;
+constexpr int O_KKH2 = O_KQH, O_DSH = O_KQL, O_DAQ = O_KQL, O_QH = O_KQL + 16 * KB;
+constexpr int O_KKL2 = O_KQL + 16 * KB, O_DWT = O_KQL, O_DAT = O_KQL + 16 * KB;
+constexpr int O_XT = O_KQL + 24 * KB, O_KQH2 = O_SIN, O_QL2 = O_RDO, O_DRTL = O_RH;
+// small arrays
+constexpr int OFF_SM = BUF_END;
+constexpr int SMALL_FLOATS = 64 * 3 + 256 * 2 + 128 * 2 + 16;
+constexpr int OFF_BAR = OFF_SM + SMALL_FLOATS * 4;
+constexpr int SMEM_BYTES = OFF_BAR + 64 + 1024;  // + alignment slack
+static_assert(SMEM_BYTES <= 232448, "shared memory");
+static_assert(O_AQ + 8 * KB <= O_KQH && O_DAT + 16 * KB <= O_RH, "map");
+
+struct BwdParams {
+  Args a;
+};
+
+__device__ __forceinline__ uint64_t kdesc(const unsigned char *p) {
+  return sw128_desc(smem_u32(p), 16, 1024);
+}
+__device__ __forceinline__ uint64_t mdesc(const unsigned char *p, uint32_t lbo) {
+  return sw128_desc(smem_u32(p), lbo, 1024);
+}
+// byte offset of element (row, col) of a [rows][128] 16-bit tile stored as two
+// 64-column slabs `slab` bytes apart
+__device__ __forceinline__ uint32_t el_off(int row, int col, int slab) {
+  return (uint32_t)(col >> 6) * slab + sw128_off(row, col & 63);
+}
+__device__ __forceinline__ void st_bf(unsigned char *base, uint32_t off, float x) {
+  *reinterpret_cast<__nv_bfloat16 *>(base + off) = __float2bfloat16_rn(x);
+}
+__device__ __forceinline__ void st_h(unsigned char *base, uint32_t off, float x) {
+  *reinterpret_cast<__half *>(base + off) = __float2half_rn(x);
+}
+// x = hi + lo with both parts bf16
+__device__ __forceinline__ void st_split(unsigned char *hi, unsigned char *lo, uint32_t off, float x) {
+  const __nv_bfloat16 h = __float2bfloat16_rn(x);
+  *reinterpret_cast<__nv_bfloat16 *>(hi + off) = h;
+  *reinterpret_cast<__nv_bfloat16 *>(lo + off) = __float2bfloat16_rn(x - __bfloat162float(h));
+}
+
+// x ~ hi + lo, both fp16: returns hi, writes the lo chunk
+__device__ __forceinline__ uint4 split_h8(const float *x, uint4 *lo) {
+  float h[8], l[8];
+  const uint4 hi = pack_h8(x);
+  unpack_h8(hi, h);
+#pragma unroll
+  for (int j = 0; j < 8; ++j) l[j] = x[j] - h[j];
+  *lo = pack_h8(l);
+  return hi;
+}
+
+// Reduce-scatter of 16 per-lane values over a warp: returns, in lanes 2j and
+// 2j + 1, the warp-wide sum of v[j].
+__device__ __forceinline__ float rs16(const float *v, int lane) {
+  float w8[8], w4[4], w2[2];
+  const bool b4 = lane & 16, b3 = lane & 8, b2 = lane & 4, b1 = lane & 2;
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    const float keep = b4 ? v[8 + j] : v[j], send = b4 ? v[j] : v[8 + j];
+    w8[j] = keep + __shfl_xor_sync(0xffffffffu, send, 16);
+  }
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    const float keep = b3 ? w8[4 + j] : w8[j], send = b3 ? w8[j] : w8[4 + j];
+    w4[j] = keep + __shfl_xor_sync(0xffffffffu, send, 8);
+  }
+#pragma unroll
+  for (int j = 0; j < 2; ++j) {
+    const float keep = b2 ? w4[2 + j] : w4[j], send = b2 ? w4[j] : w4[2 + j];
+    w2[j] = keep + __shfl_xor_sync(0xffffffffu, send, 4);
+  }
+  const float keep = b1 ? w2[1] : w2[0], send = b1 ? w2[0] : w2[1];
+  const float w1 = keep + __shfl_xor_sync(0xffffffffu, send, 2);
+  return w1 + __shfl_xor_sync(0xffffffffu, w1, 1);
+}
+
+__global__ void __launch_bounds__(BT, 1)
+    k_fused_bwd(const __grid_constant__ CUtensorMap mq, const __grid_constant__ CUtensorMap mk,
+                const __grid_constant__ CUtensorMap mv, const __grid_constant__ CUtensorMap mg,
+                const __grid_constant__ CUtensorMap mw, const __grid_constant__ CUtensorMap mdo,
+                const BwdParams P) {
+  const Args &a = P.a;
+  extern __shared__ unsigned char smraw[];
+  unsigned char *sm =
+      reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(smraw) + 1023) & ~uintptr_t(1023));
+  unsigned char *rkq = sm + O_RKQ, *sin = sm + O_SIN, *rv = sm + O_RV, *rdo = sm + O_RDO;
+  unsigned char *rg = sm + O_RG, *rw = sm + O_RW, *bkqh = sm + O_KQH, *bkql = sm + O_KQL;
+  float *s_r = reinterpret_cast<float *>(sm + OFF_SM);  // [64] r_t
+  float *s_ri = s_r + 64;     // [64] 1 / r_t
+  float *s_s = s_ri + 64;     // [64] s_t = r_t + sum_i phat k^2
+  float *s_red = s_s + 64;    // [4][64] per-warp partial sums over channels (ds_t)
+  float *s_red2 = s_red + 256;  // [4][64] (dr_t)
+  float *s_gC = s_red2 + 256;   // [128] gamma_C
+  float *s_dp = s_gC + 128;     // [128] uncertainty cotangent carried between chunks
+  float *s_misc = s_dp + 128;   // [0] lambda, [1..] scratch
+  uint64_t *bars = reinterpret_cast<uint64_t *>(sm + OFF_BAR);
+  uint64_t *bar_a = bars, *bar_b = bars + 1, *bar_mma = bars + 2;
+  uint32_t *s_tbase = reinterpret_cast<uint32_t *>(bars + 4);
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int wq = warp & 3, wg = warp >> 2;  // TMEM lane quarter, column group
+  const int ci = tid & (D - 1), qq = tid >> 7, t0 = 16 * qq;  // channel view: channel, token quarter
+  const int bh = blockIdx.x, b = bh / a.H, h = bh % a.H;
+  const int NC = (a.T + CM - 1) / CM;
+  const float tau = a.tau, mu = a.mu;
+
+  if (tid == 0) {
+    mbar_init(bar_a, 1);
+    mbar_init(bar_b, 1);
+    mbar_init(bar_mma, 1);
+    fence_mbar_init();
+    prefetch_tmap(&mq);
+    prefetch_tmap(&mk);
+    prefetch_tmap(&mv);
+    prefetch_tmap(&mg);
+    prefetch_tmap(&mw);
+    prefetch_tmap(&mdo);
+  }
+  if (warp == 0) {
+    tmem_alloc(s_tbase, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tb = *s_tbase;
+  const uint32_t TS = tb, TPH = tb + 128, TGM = tb + 192;
+  const uint32_t X0 = tb + 256, X1 = tb + 320, X2 = tb + 384, X3 = tb + 448;
+  const uint32_t lane_base = (uint32_t)(32 * wq) << 16;
+
+  // loads of chunk c: bar_a <- g, omega, S_in (issued when their buffers free up)
+  // and k, q (issued last; the one expect_tx covers both groups); bar_b <- dO, v
+  constexpr uint32_t kBytesA = 6 * 16384;
+  auto issue_a_gws = [&](int c) {
+    mbar_expect_tx(bar_a, kBytesA);
+    for (int s = 0; s < 2; ++s) {
+      tma_load_4d(rg + s * 8192, &mg, bar_a, 64 * s, h, c * CM, b);
+      tma_load_4d(rw + s * 8192, &mw, bar_a, 64 * s, h, c * CM, b);
+    }
+    bulk_g2s(sin, a.fSin + ((size_t)bh * NC + c) * 32768, 32768, bar_a);
+  };
+  auto issue_a_kq = [&](int c) {
+    for (int s = 0; s < 2; ++s) {
+      tma_load_4d(rkq + s * 16384, &mk, bar_a, 64 * s, h, c * CM, b);
+      tma_load_4d(rkq + s * 16384 + 8192, &mq, bar_a, 64 * s, h, c * CM, b);
+    }
+  };
+  auto issue_b_do = [&](int c) {
+    mbar_expect_tx(bar_b, 32768);
+    for (int s = 0; s < 2; ++s) tma_load_4d(rdo + s * 8192, &mdo, bar_b, 64 * s, h, c * CM, b);
+  };
+  auto issue_b_v = [&](int c) {
+    for (int s = 0; s < 2; ++s) tma_load_4d(rv + s * 8192, &mv, bar_b, 64 * s, h, c * CM, b);
+  };
+  if (tid == 0) {
+    issue_a_gws(NC - 1);
+    issue_a_kq(NC - 1);
+    issue_b_do(NC - 1);
+    issue_b_v(NC - 1);
+  }
+
+  // ---- cotangent scale lambda = 2^-e with max(|dO|, |dS_T|) * lambda in [1, 2)
+  {
+    float m = 0.f;
+    const unsigned char *dO = static_cast<const unsigned char *>(a.dO);
+    for (int e = tid; e < a.T * 16; e += BT) {
+      const int t = e >> 4, c16 = e & 15;
+      const uint4 u = *reinterpret_cast<const uint4 *>(dO + (tok_index(a, b, t, h) * D) * 2 + c16 * 16);
+      float v[8];
+      unpack_bf8(u, v);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) m = fmaxf(m, fabsf(v[j]));
+    }
+    if (a.dST) {
+      const float4 *src = reinterpret_cast<const float4 *>(a.dST + (size_t)bh * D * D);
+      for (int e = tid; e < D * D / 4; e += BT) {
+        const float4 x = src[e];
+        m = fmaxf(fmaxf(m, fmaxf(fabsf(x.x), fabsf(x.y))), fmaxf(fabsf(x.z), fabsf(x.w)));
+      }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+    if (lane == 0) s_red[warp] = m;
+    __syncthreads();
+    if (tid == 0) {
+      float mm = 0.f;
+      for (int w = 0; w < BT / 32; ++w) mm = fmaxf(mm, s_red[w]);
+      float lam = 1.f;
+      if (mm > 0.f && isfinite(mm)) {
+        int e;
+        frexpf(mm, &e);  // mm = f 2^e, f in [0.5, 1)
+        e = max(e, -100);
+        lam = ldexpf(1.f, 1 - e);
+      }
+      s_misc[0] = lam;
+    }
+    __syncthreads();
+  }
+  const float lam = s_misc[0], invl = 1.f / lam;
+
+  // dS = lambda dS_T -> TMEM (row = key channel i, column = value j); dp = lambda dp_T
+  {
+    const int i = 32 * wq + lane;
+    for (int c0 = 0; c0 < 32; c0 += 16) {
+      float v[16];
+      const int j0 = 32 * wg + c0;
+      if (a.dST) {
+        const float4 *src = reinterpret_cast<const float4 *>(a.dST + ((size_t)bh * D + i) * D + j0);
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const float4 x = src[u];
+          v[4 * u] = lam * x.x; v[4 * u + 1] = lam * x.y; v[4 * u + 2] = lam * x.z; v[4 * u + 3] = lam * x.w;
+        }
+      } else {
+#pragma unroll
+        for (int u = 0; u < 16; ++u) v[u] = 0.f;
+      }
+      tmem_st16(TS + lane_base + j0, v);
+    }
+    tmem_st_wait();
+  }
+  if (tid < D) s_dp[tid] = a.dpT ? lam * a.dpT[(size_t)bh * D + tid] : 0.f;
+
+  // per-token r of the next chunk, prefetched into registers
+  float nr = 1.f;
+  auto load_r = [&](int c) {
+    nr = 1.f;
+    if (tid < CM && c >= 0) {
+      const int t = c * CM + tid;
+      if (t < a.T) nr = ld<__nv_bfloat16>(a.r, tok_index(a, b, t, h));
+    }
+  };
+  load_r(NC - 1);
+
+  uint32_t mma_phase = 0;
+  bool ok = true;
+  const uint32_t id_T = idesc_bf16(128, 64, 0, 0);
+  const uint32_t id_WU = idesc_bf16(128, 128, 0, 1), id_U = idesc_f16(128, 128, 0, 1);
+  auto mma_wait = [&]() -> bool {
+    bool r = mbar_wait(bar_mma, mma_phase & 1, kWaitIters);
+    ++mma_phase;
+    return __syncthreads_and(r);
+  };
+  // the thread's tokens t0..t0+15: phat, gamma from TMEM, k from the raw tile
+  auto load_ph_ga = [&](float *ph, float *ga) {
+    tmem_ld16(TPH + lane_base + t0, ph);
+    tmem_ld16(TGM + lane_base + t0, ga);
+  };
+  auto raw_k = [&](int t) { return bf(rkq, 16384, t, ci); };
+  auto raw_q = [&](int t) { return bf(rkq + 8192, 16384, t, ci); };
+
+  for (int it = 0; it < NC && ok; ++it) {
+    const int c = NC - 1 - it;
+    // ---- [1] per-token scalars; raw tiles of this chunk
+    if (tid < CM) {
+      s_r[tid] = nr;
+      s_ri[tid] = 1.f / nr;
+    }
+    ok = __syncthreads_and(mbar_wait(bar_a, it & 1, kWaitIters));
+    if (!ok) break;
+    load_r(c - 1);
+
+    // ---- [2] gain recursion of this chunk from the saved entry uncertainty (as in
+    //          the forward: four quarters of 16 tokens, Moebius products combined
+    //          into each quarter's entry value); phat, gamma -> TMEM (lane = channel)
+    float dgc = 0.f;  // this thread's part of dgamma_C for channel ci
+    {
+      float *sQ = reinterpret_cast<float *>(bkqh);  // [4][128][5] quarter summaries
+      float al[16], w[16], uk[16];
+#pragma unroll
+      for (int j = 0; j < 16; ++j) {
+        const float kk = raw_k(t0 + j);
+        al[j] = __expf(bf(rg, 8192, t0 + j, ci));
+        w[j] = bf(rw, 8192, t0 + j, ci);
+        uk[j] = mu * kk * kk * s_ri[t0 + j];
+      }
+      float m00 = 1.f, m01 = 0.f, m10 = 0.f, m11 = 1.f, eq = 1.f;
+#pragma unroll
+      for (int j = 0; j < 16; ++j) {
+        const float a2_ = al[j] * al[j], ua2 = uk[j] * a2_, d1 = 1.f + uk[j] * w[j];
+        const float n00 = a2_ * m00 + w[j] * m10, n01 = a2_ * m01 + w[j] * m11;
+        const float n10 = ua2 * m00 + d1 * m10, n11 = ua2 * m01 + d1 * m11;
+        m00 = n00; m01 = n01; m10 = n10; m11 = n11;
+        eq *= al[j];
+        if ((j & 7) == 7) {
+          const float sc = __frcp_rn(fmaxf(fmaxf(fabsf(m00), fabsf(m01)), fmaxf(fabsf(m10), fabsf(m11))));
+          m00 *= sc; m01 *= sc; m10 *= sc; m11 *= sc;
+        }
+      }
+      float *mine = sQ + (qq * D + ci) * 5;
+      mine[0] = m00; mine[1] = m01; mine[2] = m10; mine[3] = m11; mine[4] = eq;
+      __syncthreads();
+      float n = a.fpin[((size_t)bh * NC + c) * D + ci], d = 1.f, e = 1.f;
+      for (int q2 = 0; q2 < qq; ++q2) {
+        const float *o = sQ + (q2 * D + ci) * 5;
+        const float nn = o[0] * n + o[1] * d, dd = o[2] * n + o[3] * d;
+        const float sc = __frcp_rn(fmaxf(fabsf(nn), fabsf(dd)));
+        n = nn * sc;
+        d = dd * sc;
+        e *= o[4];
+      }
+      float p = __fdividef(n, d);
+      float ph16[16], e16[16], y[16];
+#pragma unroll
+      for (int j = 0; j < 16; ++j) {
+        e *= al[j];
+        const float ph = al[j] * al[j] * p + w[j];  // eq. diag-covariance-prediction
+        ph16[j] = ph;
+        e16[j] = e;
+        p = __fdividef(ph, 1.f + uk[j] * ph);  // eq. prefix-diag-uncertainty
+      }
+      tmem_st16(TPH + lane_base + t0, ph16);
+      tmem_st16(TGM + lane_base + t0, e16);
+      if (qq == 3) s_gC[ci] = e;
+#pragma unroll
+      for (int j = 0; j < 16; ++j) {
+        const float kk = raw_k(t0 + j);
+        y[j] = ph16[j] * kk * kk;
+      }
+      const float ys = rs16(y, lane);
+      if ((lane & 1) == 0) s_red[wq * 64 + t0 + (lane >> 1)] = ys;
+      tmem_st_wait();
+      __syncthreads();
+      if (tid < CM) s_s[tid] = s_r[tid] + ((s_red[tid] + s_red[64 + tid]) + (s_red[128 + tid] + s_red[192 + tid]));
+      __syncthreads();
+      // ---- [3] first operand set: [Kbar; Qbar] hi / lo (interleaved slabs), Kk hi / lo
+#pragma unroll
+      for (int j = 0; j < 16; ++j) {
+        const int t = t0 + j;
+        const float kk = raw_k(t), qv = raw_q(t), ga = e16[j];
+        const uint32_t o16 = el_off(t, ci, 16384), o8 = el_off(t, ci, 8192);
+        st_split(bkqh, bkql, o16, ga * kk);
+        st_split(bkqh, bkql, o16 + 8192, tau * ga * qv);
+        st_split(rw, rg, o8, __fdividef(ph16[j] * kk, s_s[t] * ga));  // eq. kla-box-gain / gamma
+      }
+    }
+    fence_proxy_async();
+    tc_fence_before();
+    __syncthreads();
+    // ---- [4] MMA-T: X0 = [Kbar; Qbar] Kk^T  (hi.hi + lo.hi + hi.lo)
+    if (tid == 0) {
+      tc_fence_after();
+      for (int kk = 0; kk < 8; ++kk) {
+        const uint32_t ao = (kk >> 2) * 16384 + (kk & 3) * 32, bo = (kk >> 2) * 8192 + (kk & 3) * 32;
+        const uint64_t ah = kdesc(bkqh + ao), bhd = kdesc(rw + bo);
+        umma_bf16(X0, ah, bhd, id_T, kk > 0);
+        umma_bf16(X0, kdesc(bkql + ao), bhd, id_T, 1);
+        umma_bf16(X0, ah, kdesc(rg + bo), id_T, 1);
+      }
+      umma_commit(bar_mma);
+    }
+    if (!(ok = mma_wait())) break;
+    tc_fence_after();
+    // ---- [5] T -> fp32 (strict lower), A_qk -> fp16 [t][s] (lower); A = (I + T)^-1
+    float *sT = reinterpret_cast<float *>(rg), *sA = reinterpret_cast<float *>(bkql);
+    float *sX = sA + 64 * LT;
+    {
+      const int s0 = 16 * wg;
+      float v[16];
+      tmem_ld16(X0 + lane_base + s0, v);
+      if (wq < 2) {
+        const int r = 32 * wq + lane;
+#pragma unroll
+        for (int u = 0; u < 16; ++u)
+          if (s0 + u >= r) v[u] = 0.f;
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+          *reinterpret_cast<float4 *>(sT + r * LT + s0 + 4 * u) =
+              make_float4(v[4 * u], v[4 * u + 1], v[4 * u + 2], v[4 * u + 3]);
+      } else {
+        const int r = 32 * wq + lane - 64;
+#pragma unroll
+        for (int u = 0; u < 16; ++u)
+          if (s0 + u > r) v[u] = 0.f;
+        sm16(sm + O_AQ, chunk_off(r, s0 >> 3)) = pack_h8(v);
+        sm16(sm + O_AQ, chunk_off(r, (s0 >> 3) + 1)) = pack_h8(v + 8);
+      }
+    }
+    __syncthreads();
+    tri_inverse64(sT, sA, sX);
+    // A -> bf16 and fp16 [t][s] tiles (zero above the diagonal)
+    for (int e = tid; e < 64 * 8; e += BT) {
+      const int r = e >> 3, cc = e & 7;
+      float v[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) v[j] = (8 * cc + j <= r) ? sA[r * LT + 8 * cc + j] : 0.f;
+      sm16(sm + O_AB, chunk_off(r, cc)) = pack_bf8(v);
+      sm16(sm + O_AH, chunk_off(r, cc)) = pack_h8(v);
+    }
+    ok = __syncthreads_and(mbar_wait(bar_b, it & 1, kWaitIters));
+    if (!ok) break;
+    // lambda dO and v -> fp16 in place
+    for (int e = tid; e < 64 * 16; e += BT) {
+      const int row = e >> 4, c16 = e & 15;
+      const uint32_t off = (c16 >> 3) * 8192 + chunk_off(row, c16 & 7);
+      float v[8];
+      unpack_bf8(sm16(rdo, off), v);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) v[j] *= lam;
+      sm16(rdo, off) = pack_h8(v);
+      unpack_bf8(sm16(rv, off), v);
+      sm16(rv, off) = pack_h8(v);
+    }
+    fence_proxy_async();
+    tc_fence_before();
+    __syncthreads();
+    // ---- [6] MMA-W (bf16): X2 = A Kbar;  MMA-U (fp16): X0 = A V
+    if (tid == 0) {
+      tc_fence_after();
+      for (int kk = 0; kk < 4; ++kk) {
+        umma_bf16(X2, kdesc(sm + O_AB + kk * 32), mdesc(bkqh + kk * 2048, 16384), id_WU, kk > 0);
+        umma_bf16(X0, kdesc(sm + O_AH + kk * 32), mdesc(rv + kk * 2048, 8192), id_U, kk > 0);
+      }
+      umma_commit(bar_mma);
+    }
+    if (!(ok = mma_wait())) break;
+    tc_fence_after();
+    // ---- [7] fp16 operands: -W [t][i]; dS -> fp16 [i][j] and dS <- gamma_C dS in TMEM;
+    //          K_tail [s][i]
+    if (wq < 2) {
+      const int r = 32 * wq + lane;
+      for (int c0 = 0; c0 < 32; c0 += 16) {
+        float v[16];
+        const int j0 = 32 * wg + c0, sl = j0 >> 6, cc0 = (j0 & 63) >> 3;
+        tmem_ld16(X2 + lane_base + j0, v);
+#pragma unroll
+        for (int u = 0; u < 16; ++u) v[u] = -v[u];
+        sm16(sm + O_WN, sl * 8192 + chunk_off(r, cc0)) = pack_h8(v);
+        sm16(sm + O_WN, sl * 8192 + chunk_off(r, cc0 + 1)) = pack_h8(v + 8);
+      }
+    }
+    {
+      const int i = 32 * wq + lane;
+      const float gC = s_gC[i];
+      for (int c0 = 0; c0 < 32; c0 += 16) {
+        float v[16], sv[16];
+        const int j0 = 32 * wg + c0, sl = j0 >> 6, cc0 = (j0 & 63) >> 3;
+        const uint32_t o0 = sl * 16384 + chunk_off(i, cc0), o1 = sl * 16384 + chunk_off(i, cc0 + 1);
+        tmem_ld16(TS + lane_base + j0, v);
+        sm16(sm + O_DSH, o0) = pack_h8(v);
+        sm16(sm + O_DSH, o1) = pack_h8(v + 8);
+        unpack_h8(sm16(sin, o0), sv);
+        unpack_h8(sm16(sin, o1), sv + 8);
+#pragma unroll
+        for (int u = 0; u < 16; ++u) {
+          dgc += v[u] * sv[u];
+          v[u] *= gC;
+        }
+        tmem_st16(TS + lane_base + j0, v);
+      }
+    }
+    {
+      float ph[16], ga[16];
+      load_ph_ga(ph, ga);
+      const float gC = s_gC[ci];
+#pragma unroll
+      for (int j = 0; j < 16; ++j) {
+        const int t = t0 + j;
+        st_h(sm + O_KT, el_off(t, ci, 8192), gC * __fdividef(ph[j] * raw_k(t), s_s[t] * ga[j]));
+      }
+    }
+    tmem_st_wait();
+    fence_proxy_async();
+    tc_fence_before();
+    __syncthreads();
+    // ---- [8] MMA-S1 (fp16): X0 += -W S_in  -> rows 0..63 hold R
+    if (tid == 0) {
+      tc_fence_after();
+      const uint32_t id = idesc_f16(128, 128, 0, 1);
+      for (int kk = 0; kk < 8; ++kk)
+        umma_bf16(X0, kdesc(sm + O_WN + (kk >> 2) * 8192 + (kk & 3) * 32),
+                  mdesc(sin + kk * 2048, 16384), id, 1);
+      umma_commit(bar_mma);
+    }
+    if (!(ok = mma_wait())) break;
+    tc_fence_after();
+    // ---- [9] R -> fp16 [s][j]
+    if (wq < 2) {
+      const int t = 32 * wq + lane;
+      for (int c0 = 0; c0 < 32; c0 += 16) {
+        float v[16];
+        const int j0 = 32 * wg + c0, sl = j0 >> 6, cc0 = (j0 & 63) >> 3;
+        tmem_ld16(X0 + lane_base + j0, v);
+        sm16(sm + O_RH, sl * 8192 + chunk_off(t, cc0)) = pack_h8(v);
+        sm16(sm + O_RH, sl * 8192 + chunk_off(t, cc0 + 1)) = pack_h8(v + 8);
+      }
+    }
+    fence_proxy_async();
+    tc_fence_before();
+    __syncthreads();
+    // ---- [10] B1: X2 = dR^T;  B3: X3 = dA_qk^T (before masking);  B4: X0 = dK_tail^T
+    if (tid == 0) {
+      tc_fence_after();
+      const uint32_t id11 = idesc_f16(128, 64, 1, 1), id10 = idesc_f16(128, 64, 1, 0);
+      const uint32_t id00 = idesc_f16(128, 64, 0, 0);
+      for (int kk = 0; kk < 4; ++kk)
+        umma_bf16(X2, mdesc(rdo + kk * 2048, 8192), mdesc(sm + O_AQ + kk * 2048, 8192), id11, kk > 0);
+      for (int kk = 0; kk < 8; ++kk)
+        umma_bf16(X2, mdesc(sm + O_DSH + kk * 2048, 16384),
+                  kdesc(sm + O_KT + (kk >> 2) * 8192 + (kk & 3) * 32), id10, 1);
+      for (int kk = 0; kk < 8; ++kk) {
+        const uint32_t o8 = (kk >> 2) * 8192 + (kk & 3) * 32;
+        umma_bf16(X3, kdesc(sm + O_RH + o8), kdesc(rdo + o8), id00, kk > 0);
+        umma_bf16(X0, kdesc(sm + O_DSH + (kk >> 2) * 16384 + (kk & 3) * 32), kdesc(sm + O_RH + o8),
+                  id00, kk > 0);
+      }
+      umma_commit(bar_mma);
+    }
+    if (!(ok = mma_wait())) break;
+    tc_fence_after();
+    // ---- [11] dR^T -> fp16 [j][t] (and its fp16 remainder); dA_qk^T (masked to s <= t) -> hi/lo bf16 [s][t];
+    //           X0 <- gamma_C dK_tail^T (start of dKk^T) and its dgamma_C part; Qbar fp16
+    {
+      const int j = 32 * wq + lane, tc0 = 16 * wg;
+      float v[16];
+      tmem_ld16(X2 + lane_base + tc0, v);
+      uint4 l0, l1;
+      sm16(sm + O_DRT, chunk_off(j, tc0 >> 3)) = split_h8(v, &l0);
+      sm16(sm + O_DRT, chunk_off(j, (tc0 >> 3) + 1)) = split_h8(v + 8, &l1);
+      sm16(sm + O_DRTL, chunk_off(j, tc0 >> 3)) = l0;
+      sm16(sm + O_DRTL, chunk_off(j, (tc0 >> 3) + 1)) = l1;
+      if (wq < 2) {
+        tmem_ld16(X3 + lane_base + tc0, v);
+#pragma unroll
+        for (int u = 0; u < 16; ++u)
+          if (tc0 + u < j) v[u] = 0.f;
+        uint4 lo0, lo1;
+        sm16(sm + O_DAQ, chunk_off(j, tc0 >> 3)) = split_bf8(v, &lo0);
+        sm16(sm + O_DAQ, chunk_off(j, (tc0 >> 3) + 1)) = split_bf8(v + 8, &lo1);
+        sm16(sm + O_DAQ + 8192, chunk_off(j, tc0 >> 3)) = lo0;
+        sm16(sm + O_DAQ + 8192, chunk_off(j, (tc0 >> 3) + 1)) = lo1;
+      }
+    }
+    {
+      float ph[16], ga[16], x[16];
+      load_ph_ga(ph, ga);
+      tmem_ld16(X0 + lane_base + t0, x);
+      const float gC = s_gC[ci];
+#pragma unroll
+      for (int j = 0; j < 16; ++j) {
+        const int t = t0 + j;
+        const float kk = raw_k(t);
+        dgc += x[j] * __fdividef(ph[j] * kk, s_s[t] * ga[j]);
+        x[j] *= gC;
+        st_h(sm + O_QH, el_off(t, ci, 8192), tau * ga[j] * raw_q(t));
+      }
+      tmem_st16(X0 + lane_base + t0, x);
+    }
+    tmem_st_wait();
+    fence_proxy_async();
+    tc_fence_before();
+    __syncthreads();
+    // ---- [12] B2: TS += Qbar^T dO - W^T dR;  B5: X1 = -dW^T;  B7: X2 = dV^T (dR as hi + lo fp16);
+    //           B8a: X3 = (dO S_in^T)^T
+    if (tid == 0) {
+      tc_fence_after();
+      const uint32_t idS11 = idesc_f16(128, 128, 1, 1), idS10 = idesc_f16(128, 128, 1, 0);
+      const uint32_t id01 = idesc_f16(128, 64, 0, 1), id00 = idesc_f16(128, 64, 0, 0);
+      for (int kk = 0; kk < 4; ++kk) {
+        umma_bf16(TS, mdesc(sm + O_QH + kk * 2048, 8192), mdesc(rdo + kk * 2048, 8192), idS11, 1);
+        umma_bf16(TS, mdesc(sm + O_WN + kk * 2048, 8192), kdesc(sm + O_DRT + kk * 32), idS10, 1);
+        const uint64_t ah = mdesc(sm + O_AH + kk * 2048, 8192);
+        umma_bf16(X2, kdesc(sm + O_DRT + kk * 32), ah, id01, kk > 0);
+        umma_bf16(X2, kdesc(sm + O_DRTL + kk * 32), ah, id01, 1);
+      }
+      for (int kk = 0; kk < 8; ++kk) {
+        const uint64_t as = kdesc(sin + (kk >> 2) * 16384 + (kk & 3) * 32);
+        umma_bf16(X1, as, mdesc(sm + O_DRT + kk * 2048, 8192), id01, kk > 0);
+        umma_bf16(X3, as, kdesc(rdo + (kk >> 2) * 8192 + (kk & 3) * 32), id00, kk > 0);
+      }
+      umma_commit(bar_mma);
+    }
+    if (!(ok = mma_wait())) break;
+    tc_fence_after();
+    // ---- [13] second operand set: [Kbar; Qbar] hi (interleaved), Qbar lo, Kk hi / lo;
+    //           B8b: X3 += (dA_qk Kk)^T;  B9a: X0 += (dA_qk^T Qbar)^T
+    {
+      float ph[16], ga[16];
+      load_ph_ga(ph, ga);
+#pragma unroll
+      for (int j = 0; j < 16; ++j) {
+        const int t = t0 + j;
+        const float kk = raw_k(t);
+        const uint32_t o16 = el_off(t, ci, 16384), o8 = el_off(t, ci, 8192);
+        st_bf(sm + O_KQH2, o16, ga[j] * kk);
+        const float qb = tau * ga[j] * raw_q(t);
+        const __nv_bfloat16 qh = __float2bfloat16_rn(qb);
+        *reinterpret_cast<__nv_bfloat16 *>(sm + O_KQH2 + 8192 + o16) = qh;
+        st_bf(sm + O_QL2, o8, qb - __bfloat162float(qh));
+        st_split(sm + O_KKH2, sm + O_KKL2, o8, __fdividef(ph[j] * kk, s_s[t] * ga[j]));
+      }
+    }
+    fence_proxy_async();
+    tc_fence_before();
+    __syncthreads();
+    if (tid == 0) {
+      tc_fence_after();
+      const uint32_t id11 = idesc_bf16(128, 64, 1, 1), id10 = idesc_bf16(128, 64, 1, 0);
+      for (int kk = 0; kk < 4; ++kk) {
+        const uint64_t kh = mdesc(sm + O_KKH2 + kk * 2048, 8192), kl = mdesc(sm + O_KKL2 + kk * 2048, 8192);
+        const uint64_t dh = mdesc(sm + O_DAQ + kk * 2048, 8192), dl = mdesc(sm + O_DAQ + 8192 + kk * 2048, 8192);
+        umma_bf16(X3, kh, dh, id11, 1);
+        umma_bf16(X3, kl, dh, id11, 1);
+        umma_bf16(X3, kh, dl, id11, 1);
+        const uint64_t qh = mdesc(sm + O_KQH2 + 8192 + kk * 2048, 16384), ql = mdesc(sm + O_QL2 + kk * 2048, 8192);
+        const uint64_t eh = kdesc(sm + O_DAQ + kk * 32), el = kdesc(sm + O_DAQ + 8192 + kk * 32);
+        umma_bf16(X0, qh, eh, id10, 1);
+        umma_bf16(X0, ql, eh, id10, 1);
+        umma_bf16(X0, qh, el, id10, 1);
+      }
+      umma_commit(bar_mma);
+    }
+    if (!(ok = mma_wait())) break;
+    tc_fence_after();
+    if (tid == 0 && c > 0) issue_b_do(c - 1);  // dO / Qbar lo buffer is free
+    // ---- [14] dW^T -> bf16 [i][t];  dV^T -> dv
+    {
+      const int j = 32 * wq + lane, tc0 = 16 * wg;
+      float v[16];
+      tmem_ld16(X1 + lane_base + tc0, v);
+#pragma unroll
+      for (int u = 0; u < 16; ++u) v[u] = -v[u];
+      sm16(sm + O_DWT, chunk_off(j, tc0 >> 3)) = pack_bf8(v);
+      sm16(sm + O_DWT, chunk_off(j, (tc0 >> 3) + 1)) = pack_bf8(v + 8);
+      tmem_ld16(X2 + lane_base + tc0, v);
+#pragma unroll
+      for (int u = 0; u < 16; ++u) {
+        const int t = c * CM + tc0 + u;
+        if (t < a.T) sto(a.odt, a.dv_, tok_index(a, b, t, h) * D + j, v[u] * invl);
+      }
+    }
+    fence_proxy_async();
+    tc_fence_before();
+    __syncthreads();
+    // ---- [15] B6: X1 = dA^T = (dR V^T + dW Kbar^T)^T;  B10a: X2 = (A^T dW)^T
+    if (tid == 0) {
+      tc_fence_after();
+      const uint32_t ih01 = idesc_f16(128, 64, 0, 1), ib01 = idesc_bf16(128, 64, 0, 1);
+      for (int kk = 0; kk < 8; ++kk) {
+        umma_bf16(X1, kdesc(rv + (kk >> 2) * 8192 + (kk & 3) * 32), mdesc(sm + O_DRT + kk * 2048, 8192),
+                  ih01, kk > 0);
+        umma_bf16(X1, kdesc(sm + O_KQH2 + (kk >> 2) * 16384 + (kk & 3) * 32),
+                  mdesc(sm + O_DWT + kk * 2048, 8192), ib01, 1);
+      }
+      for (int kk = 0; kk < 4; ++kk)
+        umma_bf16(X2, kdesc(sm + O_DWT + kk * 32), mdesc(sm + O_AB + kk * 2048, 8192), ib01, kk > 0);
+      umma_commit(bar_mma);
+    }
+    if (!(ok = mma_wait())) break;
+    tc_fence_after();
+    if (tid == 0 && c > 0) issue_b_v(c - 1);  // v buffer is free
+    // ---- [16] dT = strict_lower(-A^T dA A^T): X = A^T dA, Y = X A^T (fp16)
+    if (wq < 2) {
+      const int s = 32 * wq + lane, tc0 = 16 * wg;
+      float v[16];
+      tmem_ld16(X1 + lane_base + tc0, v);
+      sm16(sm + O_DAT, chunk_off(s, tc0 >> 3)) = pack_h8(v);
+      sm16(sm + O_DAT, chunk_off(s, (tc0 >> 3) + 1)) = pack_h8(v + 8);
+    }
+    fence_proxy_async();
+    tc_fence_before();
+    __syncthreads();
+    if (tid == 0) {
+      tc_fence_after();
+      const uint32_t id = idesc_f16(128, 64, 1, 0);
+      for (int kk = 0; kk < 4; ++kk)
+        umma_bf16(X1, mdesc(sm + O_AH + kk * 2048, 8192), kdesc(sm + O_DAT + kk * 32), id, kk > 0);
+      umma_commit(bar_mma);
+    }
+    if (!(ok = mma_wait())) break;
+    tc_fence_after();
+    if (wq < 2) {
+      const int r = 32 * wq + lane, tc0 = 16 * wg;
+      float v[16];
+      tmem_ld16(X1 + lane_base + tc0, v);
+      sm16(sm + O_XT, chunk_off(r, tc0 >> 3)) = pack_h8(v);
+      sm16(sm + O_XT, chunk_off(r, (tc0 >> 3) + 1)) = pack_h8(v + 8);
+    }
+    fence_proxy_async();
+    tc_fence_before();
+    __syncthreads();
+    if (tid == 0) {
+      tc_fence_after();
+      const uint32_t id = idesc_f16(128, 64, 0, 0);
+      for (int kk = 0; kk < 4; ++kk)
+        umma_bf16(X1, kdesc(sm + O_XT + kk * 32), kdesc(sm + O_AH + kk * 32), id, kk > 0);
+      umma_commit(bar_mma);
+    }
+    if (!(ok = mma_wait())) break;
+    tc_fence_after();
+    if (wq < 2) {
+      const int r = 32 * wq + lane, tc0 = 16 * wg;
+      float v[16];
+      tmem_ld16(X1 + lane_base + tc0, v);
+#pragma unroll
+      for (int u = 0; u < 16; ++u) v[u] = (tc0 + u < r) ? -v[u] : 0.f;
+      sm16(sm + O_DT, chunk_off(r, tc0 >> 3)) = pack_bf8(v);
+      sm16(sm + O_DT, chunk_off(r, (tc0 >> 3) + 1)) = pack_bf8(v + 8);
+    }
+    fence_proxy_async();
+    tc_fence_before();
+    __syncthreads();
+    // ---- [17] B9b: X0 += (dT^T Kbar)^T;  B10b: X2 += (dT Kk)^T
+    if (tid == 0) {
+      tc_fence_after();
+      const uint32_t id11 = idesc_bf16(128, 64, 1, 1), id10 = idesc_bf16(128, 64, 1, 0);
+      for (int kk = 0; kk < 4; ++kk) {
+        umma_bf16(X0, mdesc(sm + O_KQH2 + kk * 2048, 16384), mdesc(sm + O_DT + kk * 2048, 8192), id11, 1);
+        umma_bf16(X2, mdesc(sm + O_KKH2 + kk * 2048, 8192), kdesc(sm + O_DT + kk * 32), id10, 1);
+      }
+      umma_commit(bar_mma);
+    }
+    if (!(ok = mma_wait())) break;
+    tc_fence_after();
+    if (tid == 0 && c > 0) issue_a_gws(c - 1);  // g, omega, S_in buffers are free
+    // ---- [18] per channel (lane ci, tokens t0..t0+15): back through Gamma and the
+    //           gain emission, then the uncertainty recursion backwards in time
+    {
+      float *sdg = reinterpret_cast<float *>(bkql);  // [16][512] dG -> reverse cumsum
+      float *s_tot = reinterpret_cast<float *>(sm + O_RH);  // [4][128] quarter sums of dG
+      float *s_dgc = s_tot + 512;                           // [4][128] dgamma_C parts
+      float *s_aff = s_dgc + 512;                           // [4][128][2] affine summaries
+      float part[16];
+#pragma unroll
+      for (int h8 = 0; h8 < 2; ++h8) {
+        float xq[8], xk[8], xb[8], ph[8], ga[8];
+        tmem_ld8(X3 + lane_base + t0 + 8 * h8, xq);
+        tmem_ld8(X0 + lane_base + t0 + 8 * h8, xk);
+        tmem_ld8(X2 + lane_base + t0 + 8 * h8, xb);
+        tmem_ld8(TPH + lane_base + t0 + 8 * h8, ph);
+        tmem_ld8(TGM + lane_base + t0 + 8 * h8, ga);
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          const int j = 8 * h8 + u, t = t0 + j;
+          const float kk = raw_k(t), qv = raw_q(t);
+          const float kap = __fdividef(ph[u] * kk, s_s[t]);
+          const float Kk = __fdividef(kap, ga[u]);
+          sdg[j * BT + tid] = xb[u] * ga[u] * kk - xk[u] * Kk + xq[u] * tau * ga[u] * qv;
+          part[j] = __fdividef(xk[u], ga[u]) * kap;  // dkappa . kappa
+          const int tt = c * CM + t;
+          if (tt < a.T) sto(a.odt, a.dq, tok_index(a, b, tt, h) * D + ci, tau * ga[u] * xq[u] * invl);
+        }
+      }
+      s_dgc[qq * D + ci] = dgc;
+      const float rsum = rs16(part, lane);
+      if ((lane & 1) == 0) s_red[wq * 64 + t0 + (lane >> 1)] = rsum;
+      __syncthreads();
+      if (qq == 3) {
+        const float dgC = (s_dgc[ci] + s_dgc[D + ci]) + (s_dgc[2 * D + ci] + s_dgc[3 * D + ci]);
+        sdg[15 * BT + tid] += dgC * s_gC[ci];
+      }
+      float tot = 0.f;
+#pragma unroll
+      for (int j = 0; j < 16; ++j) tot += sdg[j * BT + tid];
+      s_tot[qq * D + ci] = tot;
+      __syncthreads();
+      {
+        float run = 0.f;
+        for (int q2 = qq + 1; q2 < 4; ++q2) run += s_tot[q2 * D + ci];
+#pragma unroll
+        for (int j = 15; j >= 0; --j) {
+          run += sdg[j * BT + tid];
+          sdg[j * BT + tid] = run;
+        }
+      }
+      // per-token values of the recursion
+      float ph[16], ga[16];
+      load_ph_ga(ph, ga);
+      float ga_prev = 1.f, p_prev;
+      if (qq > 0) {
+        float t8[8], g8[8];
+        tmem_ld8(TPH + lane_base + t0 - 8, t8);
+        tmem_ld8(TGM + lane_base + t0 - 8, g8);
+        const float kk = raw_k(t0 - 1);
+        ga_prev = g8[7];
+        p_prev = __fdividef(t8[7], 1.f + mu * kk * kk * s_ri[t0 - 1] * t8[7]);
+      } else {
+        p_prev = a.fpin[((size_t)bh * NC + c) * D + ci];
+      }
+      auto ds_of = [&](int t) {
+        return -((s_red[t] + s_red[64 + t]) + (s_red[128 + t] + s_red[192 + t])) / s_s[t];
+      };
+      // affine summary of this quarter: dp_before = A dp_after + B
+      {
+        float A = 1.f, Bv = 0.f;
+        float xk[16];
+        tmem_ld16(X0 + lane_base + t0, xk);
+#pragma unroll
+        for (int j = 15; j >= 0; --j) {
+          const int t = t0 + j;
+          const float kk = raw_k(t), sinv = 1.f / s_s[t];
+          const float gp = j > 0 ? ga[j - 1] : ga_prev;
+          const float al = __fdividef(ga[j], gp), al2 = al * al;
+          const float den = 1.f + mu * kk * kk * s_ri[t] * ph[j];
+          const float dphl = __fdividef(xk[j], ga[j]) * kk * sinv + ds_of(t) * kk * kk;
+          const float aj = __fdividef(al2, den * den);
+          Bv = aj * Bv + al2 * dphl;
+          A = aj * A;
+        }
+        s_aff[(qq * D + ci) * 2] = A;
+        s_aff[(qq * D + ci) * 2 + 1] = Bv;
+      }
+      __syncthreads();
+      float dp = s_dp[ci];
+      for (int q2 = 3; q2 > qq; --q2) dp = s_aff[(q2 * D + ci) * 2] * dp + s_aff[(q2 * D + ci) * 2 + 1];
+      float drp[16];
+      {
+        float xk[16], xb[16];
+        tmem_ld16(X0 + lane_base + t0, xk);
+        tmem_ld16(X2 + lane_base + t0, xb);
+#pragma unroll
+        for (int j = 15; j >= 0; --j) {
+          const int t = t0 + j, tt = c * CM + t;
+          const float kk = raw_k(t), sinv = 1.f / s_s[t], ds = ds_of(t);
+          const float gp = j > 0 ? ga[j - 1] : ga_prev;
+          const float al = __fdividef(ga[j], gp), al2 = al * al;
+          const float u = mu * kk * kk * s_ri[t];
+          const float den = 1.f + u * ph[j], pt = __fdividef(ph[j], den);
+          float pprev;
+          if (j > 0) {
+            const float kp = raw_k(t - 1);
+            pprev = __fdividef(ph[j - 1], 1.f + mu * kp * kp * s_ri[t - 1] * ph[j - 1]);
+          } else {
+            pprev = p_prev;
+          }
+          const float dkap = __fdividef(xk[j], ga[j]);
+          const float dphl = dkap * kk * sinv + ds * kk * kk;
+          const float dph = __fdividef(dp, den * den) + dphl;
+          const float du = -dp * pt * pt;
+          const float dkt = xb[j] * ga[j] + dkap * ph[j] * sinv + 2.f * ds * ph[j] * kk +
+                            du * 2.f * mu * kk * s_ri[t];
+          drp[j] = -du * u * s_ri[t];
+          const float dgt = sdg[j * BT + tid] + 2.f * al2 * pprev * dph;
+          if (tt < a.T) {
+            const size_t idx = tok_index(a, b, tt, h) * D + ci;
+            sto(a.odt, a.dk_, idx, dkt * invl);
+            sto(a.odt, a.domega, idx, dph * invl);
+            sto(a.odt, a.dg, idx, dgt * invl);
+          }
+          dp = al2 * dph;
+        }
+      }
+      const float rs2 = rs16(drp, lane);
+      if ((lane & 1) == 0) s_red2[wq * 64 + t0 + (lane >> 1)] = rs2;
+      __syncthreads();
+      if (qq == 0) s_dp[ci] = dp;
+      if (tid < CM) {
+        const int tt = c * CM + tid;
+        if (tt < a.T) {
+          const float dr = ds_of(tid) + ((s_red2[tid] + s_red2[64 + tid]) + (s_red2[128 + tid] + s_red2[192 + tid]));
+          sto(a.odt, a.dr, tok_index(a, b, tt, h), dr * invl);
+        }
+      }
+    }
+    fence_proxy_async();
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (tid == 0 && c > 0) issue_a_kq(c - 1);  // raw k, q have been read
+  }
+
+  if (ok) {
+    if (a.dS0) {
+      const int i = 32 * wq + lane;
+      for (int c0 = 0; c0 < 32; c0 += 16) {
+        float v[16];
+        const int j0 = 32 * wg + c0;
+        tmem_ld16(TS + lane_base + j0, v);
+        float4 *dst = reinterpret_cast<float4 *>(a.dS0 + ((size_t)bh * D + i) * D + j0);
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+          dst[u] = make_float4(v[4 * u] * invl, v[4 * u + 1] * invl, v[4 * u + 2] * invl, v[4 * u + 3] * invl);
+      }
+    }
+    if (a.dp0 && tid < D) a.dp0[(size_t)bh * D + tid] = s_dp[tid] * invl;
+  } else {
+    if (tid == 0) atomicExch(a.status, (unsigned)KDN_ERR_TIMEOUT);
+    // let copies already in flight land before the CTA's shared memory goes away
+    if (tid == 0) {
+      mbar_wait(bar_a, 0, kWaitIters);
+      mbar_wait(bar_a, 1, kWaitIters);
+      mbar_wait(bar_b, 0, kWaitIters);
+      mbar_wait(bar_b, 1, kWaitIters);
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) tmem_dealloc(tb, 512);
+}
+
+}  // namespace
+
+bool fused_bwd_supported(const Args &a) {
+  return a.variant == 0 && a.chunk != 32 && fused_fwd_supported(a);
+}
+
+kdn_status_t launch_fused_bwd(const Args &a, cudaStream_t s) {
+  // state-saving forward pass
+  Args f = a;
+  f.o = nullptr;
+  f.ST = nullptr;
+  f.pT = nullptr;
+  kdn_status_t st = launch_fused_fwd(f, s, a.fSin, a.fpin);
+  if (st != KDN_OK) return st;
+  BwdParams P;
+  P.a = a;
+  CUtensorMap mq, mk, mv, mg, mw, mdo;
+  if (!make_map(&mq, a.q, a) || !make_map(&mk, a.k, a) || !make_map(&mv, a.v, a) ||
+      !make_map(&mg, a.g, a) || !make_map(&mw, a.omega, a) || !make_map(&mdo, a.dO, a))
+    return KDN_ERR_CUDA;
+  if (cudaFuncSetAttribute(k_fused_bwd, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES) !=
+      cudaSuccess)
+    return KDN_ERR_CUDA;
+  k_fused_bwd<<<a.B * a.H, BT, SMEM_BYTES, s>>>(mq, mk, mv, mg, mw, mdo, P);
+  return cudaGetLastError() == cudaSuccess ? KDN_OK : KDN_ERR_CUDA;
+}
+
+}  // namespace kdn

@@ -32,17 +32,15 @@
 // fp32; with alpha = sigmoid(x) that needs an average alpha > 0.29 over a
 // 64-token chunk).  Every wait on an mbarrier is bounded; on timeout the
 // kernel records KDN_ERR_TIMEOUT in the workspace status word and returns.
-#include <cudaTypedefs.h>
-
-#include <mutex>
-
 #include "kdn_internal.cuh"
 #include "kdn_sm103.cuh"
+#include "kdn_fused_common.cuh"
 
 namespace kdn {
 namespace {
 
 using namespace sm103;
+using namespace fused;
 
 constexpr int FT = 512;   // threads (16 warps)
 constexpr int CM = 64;    // chunk length
@@ -63,7 +61,6 @@ constexpr int OFF_VR = OFF_B1L + 16384;   // V tile (TMA), later R in fp16      
 constexpr int OFF_A2 = OFF_VR + 16384;    // [A; 0] bf16 -> [0; A_qk] fp16        16 KB
 constexpr int OFF_B3 = OFF_A2 + 16384;    // S_in fp16 (MN-major)                 32 KB
 constexpr int OFF_F = OFF_B3 + 32768;     // fp32 scratch: gamma [64][128] / T, A [64][LT] + X
-constexpr int LT = 68;                    // row stride of T and A (16-byte rows, conflict-free)
 constexpr int F_BYTES = 2 * 64 * LT * 4 + 3 * 256 * 4;  // 37888 >= 32768
 constexpr int OFF_SM = OFF_F + F_BYTES;                  // small arrays
 constexpr int SMALL_FLOATS = 64 * 7 + 128 * 3;
@@ -74,54 +71,10 @@ struct FusedParams {
   Args a;
   int has_g_map;  // per-channel decay tile through TMA
   int has_w_map;  // per-channel omega tile through TMA (diag)
+  int write_o;    // 0: the outputs o are not written (state-saving pass of the backward)
+  unsigned char *save_S;  // optional [BH][NC] 32 KB images of S_in (fp16 tile of MMA-S1)
+  float *save_p;          // optional [BH][NC][128] uncertainty carry entering each chunk
 };
-
-__device__ __forceinline__ float bf(const unsigned char *base, int slab_bytes, int row, int col) {
-  const int s = col >> 6;
-  return __bfloat162float(
-      *reinterpret_cast<const __nv_bfloat16 *>(base + s * slab_bytes + sw128_off(row, col & 63)));
-}
-// 16-byte chunk `cc` (8 consecutive 2-byte elements) of row `row` in a
-// 128-byte-swizzled slab.
-__device__ __forceinline__ uint32_t chunk_off(int row, int cc) {
-  return (uint32_t)row * 128u + ((uint32_t)(cc ^ (row & 7)) << 4);
-}
-__device__ __forceinline__ void unpack_bf8(uint4 u, float *v) {
-  const __nv_bfloat162 *h = reinterpret_cast<const __nv_bfloat162 *>(&u);
-#pragma unroll
-  for (int j = 0; j < 4; ++j) {
-    const float2 f = __bfloat1622float2(h[j]);
-    v[2 * j] = f.x;
-    v[2 * j + 1] = f.y;
-  }
-}
-__device__ __forceinline__ uint4 pack_bf8(const float *v) {
-  uint4 u;
-  __nv_bfloat162 *h = reinterpret_cast<__nv_bfloat162 *>(&u);
-#pragma unroll
-  for (int j = 0; j < 4; ++j) h[j] = __floats2bfloat162_rn(v[2 * j], v[2 * j + 1]);
-  return u;
-}
-__device__ __forceinline__ uint4 pack_h8(const float *v) {
-  uint4 u;
-  __half2 *h = reinterpret_cast<__half2 *>(&u);
-#pragma unroll
-  for (int j = 0; j < 4; ++j) h[j] = __floats2half2_rn(v[2 * j], v[2 * j + 1]);
-  return u;
-}
-// x ~ hi + lo, both bf16: returns hi, writes the lo chunk
-__device__ __forceinline__ uint4 split_bf8(const float *x, uint4 *lo) {
-  float h[8], l[8];
-  const uint4 hi = pack_bf8(x);
-  unpack_bf8(hi, h);
-#pragma unroll
-  for (int j = 0; j < 8; ++j) l[j] = x[j] - h[j];
-  *lo = pack_bf8(l);
-  return hi;
-}
-__device__ __forceinline__ uint4 &sm16(unsigned char *base, uint32_t off) {
-  return *reinterpret_cast<uint4 *>(base + off);
-}
 
 template <int V>
 __global__ void __launch_bounds__(FT, 1)
@@ -268,7 +221,9 @@ __global__ void __launch_bounds__(FT, 1)
       s_om[tid] = nom;
       s_gs[tid] = ng;
     }
-    if (tid == 0) bulk_wait_read();  // O staging (fs) of the previous chunk has been read
+    if (tid == 0) bulk_wait_read();  // O staging and the saved S image have been read
+    if (P.save_p && tid < D)
+      P.save_p[((size_t)bh * NC + c) * D + tid] = (V == 0) ? s_p[tid] : s_b[0];
     ok = __syncthreads_and(mbar_wait(bar_raw, c & 1, kWaitIters));
     if (!ok) break;
     load_scalars(c + 1);
@@ -502,77 +457,7 @@ __global__ void __launch_bounds__(FT, 1)
         *reinterpret_cast<float4 *>(sT + r * LT + s0 + 4 * u) = make_float4(v[4 * u], v[4 * u + 1], v[4 * u + 2], v[4 * u + 3]);
     }
     __syncthreads();
-    {
-      // diagonal block I = warp / 4, columns c, c + 1 (c = 4 (warp % 4) + 2 (lane / 16));
-      // lane % 16 is the row.  Column substitution: once x_s is final it is broadcast
-      // along the half-warp and every lower row subtracts T_rs x_s.
-      const int o0 = 16 * (warp >> 2), rr = lane & 15, cl = 4 * (warp & 3) + 2 * (lane >> 4);
-      float trow[16];
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {  // 0 for columns >= rr
-        const float4 t4 = *reinterpret_cast<const float4 *>(sT + (o0 + rr) * LT + o0 + 4 * u);
-        trow[4 * u] = t4.x; trow[4 * u + 1] = t4.y; trow[4 * u + 2] = t4.z; trow[4 * u + 3] = t4.w;
-      }
-      float x0 = (rr == cl) ? 1.f : 0.f, x1 = (rr == cl + 1) ? 1.f : 0.f;
-#pragma unroll
-      for (int s2 = 0; s2 < 15; ++s2) {
-        const float y0 = __shfl_sync(0xffffffffu, x0, s2, 16);
-        const float y1 = __shfl_sync(0xffffffffu, x1, s2, 16);
-        x0 -= trow[s2] * y0;
-        x1 -= trow[s2] * y1;
-      }
-      sA[(o0 + rr) * LT + o0 + cl] = x0;  // zero above the diagonal
-      sA[(o0 + rr) * LT + o0 + cl + 1] = x1;
-    }
-    __syncthreads();
-    // off-diagonal levels: one thread per (block J, row, 4 columns), float4 operands
-    for (int L = 1; L < 4; ++L) {
-      const int nb = 4 - L;
-      const int J = tid >> 6, rr = (tid >> 2) & 15, cg = tid & 3, I = J + L;
-      if (J < nb) {
-        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-        for (int K = J; K < I; ++K) {
-          const float *tr = sT + (16 * I + rr) * LT + 16 * K;
-          const float *ac = sA + (16 * K) * LT + 16 * J + 4 * cg;
-#pragma unroll
-          for (int m4 = 0; m4 < 4; ++m4) {
-            const float4 t4 = *reinterpret_cast<const float4 *>(tr + 4 * m4);
-            const float tv[4] = {t4.x, t4.y, t4.z, t4.w};
-#pragma unroll
-            for (int mm = 0; mm < 4; ++mm) {
-              const float4 a4 = *reinterpret_cast<const float4 *>(ac + (4 * m4 + mm) * LT);
-              acc.x += tv[mm] * a4.x;
-              acc.y += tv[mm] * a4.y;
-              acc.z += tv[mm] * a4.z;
-              acc.w += tv[mm] * a4.w;
-            }
-          }
-        }
-        *reinterpret_cast<float4 *>(sX + J * 256 + rr * 16 + 4 * cg) = acc;
-      }
-      __syncthreads();
-      if (J < nb) {
-        const float *dr = sA + (16 * I + rr) * LT + 16 * I;
-        const float *xc = sX + J * 256 + 4 * cg;
-        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-        for (int m4 = 0; m4 < 4; ++m4) {
-          const float4 d4 = *reinterpret_cast<const float4 *>(dr + 4 * m4);
-          const float dv[4] = {d4.x, d4.y, d4.z, d4.w};
-#pragma unroll
-          for (int mm = 0; mm < 4; ++mm) {
-            const float4 x4 = *reinterpret_cast<const float4 *>(xc + (4 * m4 + mm) * 16);
-            acc.x += dv[mm] * x4.x;
-            acc.y += dv[mm] * x4.y;
-            acc.z += dv[mm] * x4.z;
-            acc.w += dv[mm] * x4.w;
-          }
-        }
-        *reinterpret_cast<float4 *>(sA + (16 * I + rr) * LT + 16 * J + 4 * cg) =
-            make_float4(-acc.x, -acc.y, -acc.z, -acc.w);
-      }
-      __syncthreads();
-    }
+    tri_inverse64(sT, sA, sX);
     // [A; 0] -> a2 (bf16, K-major, K = 64 source tokens), 16-byte chunks
     for (int e = tid; e < 128 * 8; e += FT) {
       const int r = e >> 3, cc = e & 7;
@@ -661,6 +546,10 @@ __global__ void __launch_bounds__(FT, 1)
     tc_fence_before();
     __syncthreads();
     if (tid == 0 && c + 1 < NC) issue_raw_kqw(c + 1);  // raw k, q, omega buffers are free
+    if (tid == 0 && P.save_S) {
+      bulk_s2g(P.save_S + ((size_t)bh * NC + c) * 32768, b3, 32768);
+      bulk_commit();
+    }
     // ---- [8] MMA-S1 (fp16): [U; 0] += [-W; Qbar] S_in
     if (tid == 0) {
       tc_fence_after();
@@ -702,7 +591,7 @@ __global__ void __launch_bounds__(FT, 1)
     if (tid == 0 && c + 1 < NC) issue_v(c + 1);  // R in vr has been consumed
     // ---- [11] O (rows 64..127 of TU) -> 128-byte-swizzled staging tiles in fs
     //           -> TMA bulk tensor stores (rows past T are not written)
-    if (wq >= 2) {
+    if (wq >= 2 && P.write_o) {
       const int t = 32 * wq + lane - 64;
       unsigned char *stg = reinterpret_cast<unsigned char *>(fs);
       for (int c0 = 0; c0 < 32; c0 += 16) {
@@ -727,7 +616,7 @@ __global__ void __launch_bounds__(FT, 1)
     }
     fence_proxy_async();
     __syncthreads();
-    if (tid == 0) {
+    if (tid == 0 && P.write_o) {
       const unsigned char *stg = reinterpret_cast<const unsigned char *>(fs);
       const int nbox = a.odt == KDN_BF16 ? 2 : 4, bw = a.odt == KDN_BF16 ? 64 : 32;
       for (int bx = 0; bx < nbox; ++bx) tma_store_4d(&mo, stg + bx * 8192, bx * bw, h, c * CM, b);
@@ -774,37 +663,6 @@ __global__ void __launch_bounds__(FT, 1)
 // ---------------------------------------------------------------------------
 // host side
 
-PFN_cuTensorMapEncodeTiled_v12000 encoder() {
-  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-  static std::once_flag once;
-  std::call_once(once, [] {
-    cudaDriverEntryPointQueryResult q;
-    void *p = nullptr;
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
-                                         &q) == cudaSuccess &&
-        q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
-  });
-  return fn;
-}
-
-// [B, T, H, 128] tensor of 2- or 4-byte elements; box = 128 bytes of channels
-// x 1 head x 64 tokens x 1 batch, 128-byte swizzle.
-bool make_map(CUtensorMap *m, const void *ptr, const Args &a, bool fp32 = false) {
-  auto enc = encoder();
-  if (!enc) return false;
-  const cuuint64_t es_bytes = fp32 ? 4 : 2;
-  cuuint64_t dims[4] = {(cuuint64_t)D, (cuuint64_t)a.H, (cuuint64_t)a.T, (cuuint64_t)a.B};
-  cuuint64_t strides[3] = {(cuuint64_t)D * es_bytes, (cuuint64_t)a.H * D * es_bytes,
-                           (cuuint64_t)a.T * a.H * D * es_bytes};
-  cuuint32_t box[4] = {fp32 ? 32u : 64u, 1, 64, 1};
-  cuuint32_t es[4] = {1, 1, 1, 1};
-  return enc(m, fp32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4,
-             const_cast<void *>(ptr), dims, strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
-             CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
 }  // namespace
 
 bool fused_fwd_supported(const Args &a) {
@@ -813,14 +671,19 @@ bool fused_fwd_supported(const Args &a) {
 
 int fused_fwd_smem_bytes() { return SMEM_BYTES; }
 
-kdn_status_t launch_fused_fwd(const Args &a, cudaStream_t s) {
+kdn_status_t launch_fused_fwd(const Args &a, cudaStream_t s, unsigned char *save_S,
+                              float *save_p) {
   FusedParams P;
   P.a = a;
   P.has_g_map = (a.variant == 0 || a.pcd) ? 1 : 0;
   P.has_w_map = a.variant == 0 ? 1 : 0;
+  P.write_o = save_S ? 0 : 1;
+  P.save_S = save_S;
+  P.save_p = save_p;
   CUtensorMap mq, mk, mv, mg, mw, mo;
-  if (!make_map(&mq, a.q, a) || !make_map(&mk, a.k, a) || !make_map(&mv, a.v, a) ||
-      !make_map(&mo, a.o, a, a.odt != KDN_BF16))
+  if (!make_map(&mq, a.q, a) || !make_map(&mk, a.k, a) || !make_map(&mv, a.v, a))
+    return KDN_ERR_CUDA;
+  if (P.write_o ? !make_map(&mo, a.o, a, a.odt != KDN_BF16) : !make_map(&mo, a.q, a))
     return KDN_ERR_CUDA;
   mg = mq;
   mw = mq;

@@ -84,6 +84,8 @@ struct Args {
   float *drpart;  // [BH][Tp]
   float *drw;     // [BH][Tp][4]
   float *isoadj;  // [BH][Tp][2]
+  unsigned char *fSin;  // fused backward: [BH][NC] 32 KB fp16 images of S_in
+  float *fpin;          // fused backward: [BH][NC][dk] uncertainty entering each chunk
 };
 
 __host__ __device__ inline size_t tok_index(const Args &a, int b, int t, int h) {
@@ -94,9 +96,17 @@ __host__ __device__ inline size_t tok_index(const Args &a, int b, int t, int h) 
 // A forward that runs the fused kernel only needs the status word.
 size_t workspace_layout(Args *a, char *base, bool bwd);
 
-// Fused tcgen05 forward (bf16, dk = dv = 128, 64-token chunks).
+// Fused tcgen05 forward (bf16, dk = dv = 128, 64-token chunks).  With
+// `save_S` / `save_p` it is the state-saving pass of the fused backward: o is
+// not written; the fp16 image of every chunk's entry memory (32 KB) and the
+// uncertainty carry entering every chunk (128 floats) are stored instead.
 bool fused_fwd_supported(const Args &a);
-kdn_status_t launch_fused_fwd(const Args &a, cudaStream_t s);
+kdn_status_t launch_fused_fwd(const Args &a, cudaStream_t s, unsigned char *save_S = nullptr,
+                              float *save_p = nullptr);
+// Fused tcgen05 backward (Diagonal KDN, bf16, dk = dv = 128, 64-token chunks):
+// a state-saving forward pass, then one reverse sweep per (batch, head).
+bool fused_bwd_supported(const Args &a);
+kdn_status_t launch_fused_bwd(const Args &a, cudaStream_t s);
 
 // Launchers (each returns KDN_OK or KDN_ERR_CUDA).
 kdn_status_t launch_chunked_fwd(const Args &a, cudaStream_t s, bool save_states);

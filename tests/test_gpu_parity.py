@@ -71,7 +71,10 @@ def test_forward_chunk_argument_is_tuning_only(kdn, chunk):
 BWD_CASES = [
     ("diag", True, "f32", 1, 75, 2, 32, 32),
     ("diag", True, "f32", 2, 64, 1, 128, 128),
-    ("diag", True, "bf16", 1, 140, 2, 128, 128),
+    ("diag", True, "bf16", 1, 140, 2, 128, 128),   # fused tcgen05 backward from here
+    ("diag", True, "bf16", 2, 200, 3, 128, 128),
+    ("diag", True, "bf16", 1, 64, 1, 128, 128),
+    ("diag", True, "bf16", 1, 1, 2, 128, 128),
     ("iso", False, "f32", 2, 50, 2, 64, 32),
     ("iso", False, "bf16", 1, 100, 2, 128, 128),
     ("iso", True, "f32", 1, 45, 2, 32, 64),
@@ -210,6 +213,71 @@ def test_bf16_stored_outputs(kdn, variant):
     check("ST", ST, ref["ST"], "bf16")
     gr = bwd(*[d[n] for n in names], d["S0"], d["p0"], d["dO"], out_dtype=torch.bfloat16)
     rg = oracle.bwd(variant, *[ins[n] for n in names], ins["S0"], ins["p0"], ins["dO"])
+    for n in ("dq", "dk", "dv", "dg", "domega", "dr"):
+        assert gr[n].dtype == torch.bfloat16
+        check_stored_bf16(n, gr[n], rg[n])
+
+
+def _diag_bwd_inputs(B, T, H, seed):
+    ins = make_inputs("diag", B, T, H, 128, 128, dtype="bf16", seed=seed, s0_std=0.1,
+                      p0_range=(0.5, 2.0), with_grad=True)
+    rng = np.random.default_rng(seed)
+    ins["dST"] = rng.standard_normal((B, H, 128, 128)).astype(np.float32).astype(np.float64)
+    ins["dpT"] = rng.standard_normal((B, H, 128)).astype(np.float32).astype(np.float64)
+    return ins
+
+
+def _run_diag_bwd(kdn, ins, scale=1.0, **kw):
+    d = to_dev(ins)
+    f32 = lambda x: torch.tensor(x * scale, dtype=torch.float32, device="cuda")
+    dO = (d["dO"].float() * scale).to(torch.bfloat16)
+    return kdn.kdn_diag_bwd(*[d[n] for n in ("q", "k", "v", "g", "omega", "r")], d["S0"], d["p0"],
+                            dO, f32(ins["dST"]), f32(ins["dpT"]), **kw)
+
+
+def test_fused_backward_cotangent_scale(kdn):
+    """The backward is linear in (dO, dS_T, dp_T).  The fused kernel normalises
+    the cotangents by a power of two before they enter fp16 operands, so a
+    power-of-two scale of the cotangents scales every gradient exactly, and tiny
+    cotangents (1e-6, below fp16's normal range) keep full accuracy."""
+    ins = _diag_bwd_inputs(1, 150, 2, 31)
+    g1 = _run_diag_bwd(kdn, ins)
+    g2 = _run_diag_bwd(kdn, ins, scale=2.0 ** -20)
+    torch.cuda.synchronize()
+    for n in ("dq", "dk", "dv", "dg", "domega", "dr", "dS0", "dp0"):
+        assert torch.equal(g2[n], g1[n] * 2.0 ** -20), n
+    small = dict(ins)
+    small["dO"] = ins["dO"] * 1e-6
+    small["dST"] = ins["dST"] * 1e-6
+    small["dpT"] = ins["dpT"] * 1e-6
+    small["dO"] = np.asarray(torch.tensor(small["dO"]).to(torch.bfloat16).double())
+    ref = oracle.bwd("diag", *[small[n] for n in ("q", "k", "v", "g", "omega", "r")], small["S0"],
+                     small["p0"], small["dO"], small["dST"], small["dpT"])
+    g3 = _run_diag_bwd(kdn, small)
+    torch.cuda.synchronize()
+    for n in ("dq", "dk", "dv", "dg", "domega", "dr", "dS0", "dp0"):
+        check(n, g3[n], ref[n], "bf16")
+
+
+def test_backward_chunk_argument_is_tuning_only(kdn):
+    """chunk = 32 selects the general CUDA-core kernels, the default the fused
+    tcgen05 backward; both match the oracle on the same inputs."""
+    ins = _diag_bwd_inputs(1, 100, 2, 41)
+    ref = oracle.bwd("diag", *[ins[n] for n in ("q", "k", "v", "g", "omega", "r")], ins["S0"],
+                     ins["p0"], ins["dO"], ins["dST"], ins["dpT"])
+    for chunk in (0, 32):
+        gr = _run_diag_bwd(kdn, ins, chunk=chunk)
+        torch.cuda.synchronize()
+        for n in ("dq", "dk", "dv", "dg", "domega", "dr", "dS0", "dp0"):
+            check(f"{n}[chunk={chunk}]", gr[n], ref[n], "bf16")
+
+
+def test_fused_backward_bf16_stored_gradients(kdn):
+    ins = _diag_bwd_inputs(2, 90, 2, 43)
+    rg = oracle.bwd("diag", *[ins[n] for n in ("q", "k", "v", "g", "omega", "r")], ins["S0"],
+                    ins["p0"], ins["dO"], ins["dST"], ins["dpT"])
+    gr = _run_diag_bwd(kdn, ins, out_dtype=torch.bfloat16)
+    torch.cuda.synchronize()
     for n in ("dq", "dk", "dv", "dg", "domega", "dr"):
         assert gr[n].dtype == torch.bfloat16
         check_stored_bf16(n, gr[n], rg[n])
