@@ -81,7 +81,7 @@ constexpr int O_KKL2 = O_KQL + 16 * KB, O_DWT = O_KQL, O_DAT = O_KQL + 16 * KB;
 constexpr int O_XT = O_KQL + 24 * KB, O_KQH2 = O_SIN, O_QL2 = O_RDO, O_DRTL = O_RH;
 // small arrays
 constexpr int OFF_SM = BUF_END;
-constexpr int SMALL_FLOATS = 64 * 3 + 256 * 2 + 128 * 2 + 16;
+constexpr int SMALL_FLOATS = 64 * 5 + 256 * 2 + 128 * 2 + 16;
 constexpr int OFF_BAR = OFF_SM + SMALL_FLOATS * 4;
 constexpr int SMEM_BYTES = OFF_BAR + 64 + 1024;  // + alignment slack
 static_assert(SMEM_BYTES <= 232448, "shared memory");
@@ -97,24 +97,6 @@ __device__ __forceinline__ uint64_t kdesc(const unsigned char *p) {
 __device__ __forceinline__ uint64_t mdesc(const unsigned char *p, uint32_t lbo) {
   return sw128_desc(smem_u32(p), lbo, 1024);
 }
-// byte offset of element (row, col) of a [rows][128] 16-bit tile stored as two
-// 64-column slabs `slab` bytes apart
-__device__ __forceinline__ uint32_t el_off(int row, int col, int slab) {
-  return (uint32_t)(col >> 6) * slab + sw128_off(row, col & 63);
-}
-__device__ __forceinline__ void st_bf(unsigned char *base, uint32_t off, float x) {
-  *reinterpret_cast<__nv_bfloat16 *>(base + off) = __float2bfloat16_rn(x);
-}
-__device__ __forceinline__ void st_h(unsigned char *base, uint32_t off, float x) {
-  *reinterpret_cast<__half *>(base + off) = __float2half_rn(x);
-}
-// x = hi + lo with both parts bf16
-__device__ __forceinline__ void st_split(unsigned char *hi, unsigned char *lo, uint32_t off, float x) {
-  const __nv_bfloat16 h = __float2bfloat16_rn(x);
-  *reinterpret_cast<__nv_bfloat16 *>(hi + off) = h;
-  *reinterpret_cast<__nv_bfloat16 *>(lo + off) = __float2bfloat16_rn(x - __bfloat162float(h));
-}
-
 // x ~ hi + lo, both fp16: returns hi, writes the lo chunk
 __device__ __forceinline__ uint4 split_h8(const float *x, uint4 *lo) {
   float h[8], l[8];
@@ -124,6 +106,25 @@ __device__ __forceinline__ uint4 split_h8(const float *x, uint4 *lo) {
   for (int j = 0; j < 8; ++j) l[j] = x[j] - h[j];
   *lo = pack_h8(l);
   return hi;
+}
+
+// Row `row` of a [128][64] 16-bit tile (one 128-byte-swizzled slab), tokens
+// 16 q .. 16 q + 15: two 16-byte chunks.
+__device__ __forceinline__ void st_row16_bf(unsigned char *tile, int row, int q, const float *v) {
+  sm16(tile, chunk_off(row, 2 * q)) = pack_bf8(v);
+  sm16(tile, chunk_off(row, 2 * q + 1)) = pack_bf8(v + 8);
+}
+__device__ __forceinline__ void st_row16_h(unsigned char *tile, int row, int q, const float *v) {
+  sm16(tile, chunk_off(row, 2 * q)) = pack_h8(v);
+  sm16(tile, chunk_off(row, 2 * q + 1)) = pack_h8(v + 8);
+}
+__device__ __forceinline__ void st_row16_split(unsigned char *hi, unsigned char *lo, int row, int q,
+                                               const float *v) {
+  uint4 l0, l1;
+  sm16(hi, chunk_off(row, 2 * q)) = split_bf8(v, &l0);
+  sm16(hi, chunk_off(row, 2 * q + 1)) = split_bf8(v + 8, &l1);
+  sm16(lo, chunk_off(row, 2 * q)) = l0;
+  sm16(lo, chunk_off(row, 2 * q + 1)) = l1;
 }
 
 // Reduce-scatter of 16 per-lane values over a warp: returns, in lanes 2j and
@@ -169,7 +170,9 @@ __global__ void __launch_bounds__(BT, 1)
   float *s_red2 = s_red + 256;  // [4][64] (dr_t)
   float *s_gC = s_red2 + 256;   // [128] gamma_C
   float *s_dp = s_gC + 128;     // [128] uncertainty cotangent carried between chunks
-  float *s_misc = s_dp + 128;   // [0] lambda, [1..] scratch
+  float *s_si = s_dp + 128;     // [64] 1 / s_t
+  float *s_ds = s_si + 64;      // [64] ds_t (cotangent of s_t)
+  float *s_misc = s_ds + 64;    // [0] lambda, [1..] scratch
   uint64_t *bars = reinterpret_cast<uint64_t *>(sm + OFF_BAR);
   uint64_t *bar_a = bars, *bar_b = bars + 1, *bar_mma = bars + 2;
   uint32_t *s_tbase = reinterpret_cast<uint32_t *>(bars + 4);
@@ -311,8 +314,8 @@ __global__ void __launch_bounds__(BT, 1)
 
   uint32_t mma_phase = 0;
   bool ok = true;
-  const uint32_t id_T = idesc_bf16(128, 64, 0, 0);
-  const uint32_t id_WU = idesc_bf16(128, 128, 0, 1), id_U = idesc_f16(128, 128, 0, 1);
+  const uint32_t id_T = idesc_bf16(128, 64, 1, 1);
+  const uint32_t id_W = idesc_bf16(128, 128, 0, 0), id_U = idesc_f16(128, 128, 0, 1);
   auto mma_wait = [&]() -> bool {
     bool r = mbar_wait(bar_mma, mma_phase & 1, kWaitIters);
     ++mma_phase;
@@ -398,31 +401,39 @@ __global__ void __launch_bounds__(BT, 1)
       if ((lane & 1) == 0) s_red[wq * 64 + t0 + (lane >> 1)] = ys;
       tmem_st_wait();
       __syncthreads();
-      if (tid < CM) s_s[tid] = s_r[tid] + ((s_red[tid] + s_red[64 + tid]) + (s_red[128 + tid] + s_red[192 + tid]));
+      if (tid < CM) {
+        const float st = s_r[tid] + ((s_red[tid] + s_red[64 + tid]) + (s_red[128 + tid] + s_red[192 + tid]));
+        s_s[tid] = st;
+        s_si[tid] = 1.f / st;
+      }
       __syncthreads();
-      // ---- [3] first operand set: [Kbar; Qbar] hi / lo (interleaved slabs), Kk hi / lo
+      // ---- [3] first operand set, stored transposed ([channel][token] tiles): Kbar, Qbar,
+      //          Kk as hi / lo bf16 pairs
+      {
+        float v[16];
 #pragma unroll
-      for (int j = 0; j < 16; ++j) {
-        const int t = t0 + j;
-        const float kk = raw_k(t), qv = raw_q(t), ga = e16[j];
-        const uint32_t o16 = el_off(t, ci, 16384), o8 = el_off(t, ci, 8192);
-        st_split(bkqh, bkql, o16, ga * kk);
-        st_split(bkqh, bkql, o16 + 8192, tau * ga * qv);
-        st_split(rw, rg, o8, __fdividef(ph16[j] * kk, s_s[t] * ga));  // eq. kla-box-gain / gamma
+        for (int j = 0; j < 16; ++j) v[j] = e16[j] * raw_k(t0 + j);
+        st_row16_split(bkqh, bkql, ci, qq, v);
+#pragma unroll
+        for (int j = 0; j < 16; ++j) v[j] = tau * e16[j] * raw_q(t0 + j);
+        st_row16_split(bkqh + 16384, bkql + 16384, ci, qq, v);
+#pragma unroll
+        for (int j = 0; j < 16; ++j)  // eq. kla-box-gain, divided by gamma
+          v[j] = __fdividef(ph16[j] * raw_k(t0 + j) * s_si[t0 + j], e16[j]);
+        st_row16_split(rw, rg, ci, qq, v);
       }
     }
     fence_proxy_async();
     tc_fence_before();
     __syncthreads();
-    // ---- [4] MMA-T: X0 = [Kbar; Qbar] Kk^T  (hi.hi + lo.hi + hi.lo)
+    // ---- [4] MMA-T: X0 = [Kbar; Qbar] Kk^T  (hi.hi + lo.hi + hi.lo; both operands MN-major)
     if (tid == 0) {
       tc_fence_after();
       for (int kk = 0; kk < 8; ++kk) {
-        const uint32_t ao = (kk >> 2) * 16384 + (kk & 3) * 32, bo = (kk >> 2) * 8192 + (kk & 3) * 32;
-        const uint64_t ah = kdesc(bkqh + ao), bhd = kdesc(rw + bo);
+        const uint64_t ah = mdesc(bkqh + kk * 2048, 16384), bhd = mdesc(rw + kk * 2048, 8192);
         umma_bf16(X0, ah, bhd, id_T, kk > 0);
-        umma_bf16(X0, kdesc(bkql + ao), bhd, id_T, 1);
-        umma_bf16(X0, ah, kdesc(rg + bo), id_T, 1);
+        umma_bf16(X0, mdesc(bkql + kk * 2048, 16384), bhd, id_T, 1);
+        umma_bf16(X0, ah, mdesc(rg + kk * 2048, 8192), id_T, 1);
       }
       umma_commit(bar_mma);
     }
@@ -485,7 +496,7 @@ __global__ void __launch_bounds__(BT, 1)
     if (tid == 0) {
       tc_fence_after();
       for (int kk = 0; kk < 4; ++kk) {
-        umma_bf16(X2, kdesc(sm + O_AB + kk * 32), mdesc(bkqh + kk * 2048, 16384), id_WU, kk > 0);
+        umma_bf16(X2, kdesc(sm + O_AB + kk * 32), kdesc(bkqh + kk * 32), id_W, kk > 0);
         umma_bf16(X0, kdesc(sm + O_AH + kk * 32), mdesc(rv + kk * 2048, 8192), id_U, kk > 0);
       }
       umma_commit(bar_mma);
@@ -531,10 +542,8 @@ __global__ void __launch_bounds__(BT, 1)
       load_ph_ga(ph, ga);
       const float gC = s_gC[ci];
 #pragma unroll
-      for (int j = 0; j < 16; ++j) {
-        const int t = t0 + j;
-        st_h(sm + O_KT, el_off(t, ci, 8192), gC * __fdividef(ph[j] * raw_k(t), s_s[t] * ga[j]));
-      }
+      for (int j = 0; j < 16; ++j) ph[j] = gC * __fdividef(ph[j] * raw_k(t0 + j) * s_si[t0 + j], ga[j]);
+      st_row16_h(sm + O_KT, ci, qq, ph);  // K_tail^T [i][s]
     }
     tmem_st_wait();
     fence_proxy_async();
@@ -568,13 +577,11 @@ __global__ void __launch_bounds__(BT, 1)
     // ---- [10] B1: X2 = dR^T;  B3: X3 = dA_qk^T (before masking);  B4: X0 = dK_tail^T
     if (tid == 0) {
       tc_fence_after();
-      const uint32_t id11 = idesc_f16(128, 64, 1, 1), id10 = idesc_f16(128, 64, 1, 0);
-      const uint32_t id00 = idesc_f16(128, 64, 0, 0);
+      const uint32_t id11 = idesc_f16(128, 64, 1, 1), id00 = idesc_f16(128, 64, 0, 0);
       for (int kk = 0; kk < 4; ++kk)
         umma_bf16(X2, mdesc(rdo + kk * 2048, 8192), mdesc(sm + O_AQ + kk * 2048, 8192), id11, kk > 0);
       for (int kk = 0; kk < 8; ++kk)
-        umma_bf16(X2, mdesc(sm + O_DSH + kk * 2048, 16384),
-                  kdesc(sm + O_KT + (kk >> 2) * 8192 + (kk & 3) * 32), id10, 1);
+        umma_bf16(X2, mdesc(sm + O_DSH + kk * 2048, 16384), mdesc(sm + O_KT + kk * 2048, 8192), id11, 1);
       for (int kk = 0; kk < 8; ++kk) {
         const uint32_t o8 = (kk >> 2) * 8192 + (kk & 3) * 32;
         umma_bf16(X3, kdesc(sm + O_RH + o8), kdesc(rdo + o8), id00, kk > 0);
@@ -616,12 +623,12 @@ __global__ void __launch_bounds__(BT, 1)
 #pragma unroll
       for (int j = 0; j < 16; ++j) {
         const int t = t0 + j;
-        const float kk = raw_k(t);
-        dgc += x[j] * __fdividef(ph[j] * kk, s_s[t] * ga[j]);
+        dgc += x[j] * __fdividef(ph[j] * raw_k(t) * s_si[t], ga[j]);
         x[j] *= gC;
-        st_h(sm + O_QH, el_off(t, ci, 8192), tau * ga[j] * raw_q(t));
+        ph[j] = tau * ga[j] * raw_q(t);
       }
       tmem_st16(X0 + lane_base + t0, x);
+      st_row16_h(sm + O_QH, ci, qq, ph);  // Qbar^T [i][t]
     }
     tmem_st_wait();
     fence_proxy_async();
@@ -631,10 +638,10 @@ __global__ void __launch_bounds__(BT, 1)
     //           B8a: X3 = (dO S_in^T)^T
     if (tid == 0) {
       tc_fence_after();
-      const uint32_t idS11 = idesc_f16(128, 128, 1, 1), idS10 = idesc_f16(128, 128, 1, 0);
+      const uint32_t idS01 = idesc_f16(128, 128, 0, 1), idS10 = idesc_f16(128, 128, 1, 0);
       const uint32_t id01 = idesc_f16(128, 64, 0, 1), id00 = idesc_f16(128, 64, 0, 0);
       for (int kk = 0; kk < 4; ++kk) {
-        umma_bf16(TS, mdesc(sm + O_QH + kk * 2048, 8192), mdesc(rdo + kk * 2048, 8192), idS11, 1);
+        umma_bf16(TS, kdesc(sm + O_QH + kk * 32), mdesc(rdo + kk * 2048, 8192), idS01, 1);
         umma_bf16(TS, mdesc(sm + O_WN + kk * 2048, 8192), kdesc(sm + O_DRT + kk * 32), idS10, 1);
         const uint64_t ah = mdesc(sm + O_AH + kk * 2048, 8192);
         umma_bf16(X2, kdesc(sm + O_DRT + kk * 32), ah, id01, kk > 0);
@@ -652,38 +659,35 @@ __global__ void __launch_bounds__(BT, 1)
     // ---- [13] second operand set: [Kbar; Qbar] hi (interleaved), Qbar lo, Kk hi / lo;
     //           B8b: X3 += (dA_qk Kk)^T;  B9a: X0 += (dA_qk^T Qbar)^T
     {
-      float ph[16], ga[16];
+      float ph[16], ga[16], v[16];
       load_ph_ga(ph, ga);
 #pragma unroll
-      for (int j = 0; j < 16; ++j) {
-        const int t = t0 + j;
-        const float kk = raw_k(t);
-        const uint32_t o16 = el_off(t, ci, 16384), o8 = el_off(t, ci, 8192);
-        st_bf(sm + O_KQH2, o16, ga[j] * kk);
-        const float qb = tau * ga[j] * raw_q(t);
-        const __nv_bfloat16 qh = __float2bfloat16_rn(qb);
-        *reinterpret_cast<__nv_bfloat16 *>(sm + O_KQH2 + 8192 + o16) = qh;
-        st_bf(sm + O_QL2, o8, qb - __bfloat162float(qh));
-        st_split(sm + O_KKH2, sm + O_KKL2, o8, __fdividef(ph[j] * kk, s_s[t] * ga[j]));
-      }
+      for (int j = 0; j < 16; ++j) v[j] = ga[j] * raw_k(t0 + j);
+      st_row16_bf(sm + O_KQH2, ci, qq, v);  // Kbar^T hi
+#pragma unroll
+      for (int j = 0; j < 16; ++j) v[j] = tau * ga[j] * raw_q(t0 + j);
+      st_row16_split(sm + O_KQH2 + 16384, sm + O_QL2, ci, qq, v);  // Qbar^T hi / lo
+#pragma unroll
+      for (int j = 0; j < 16; ++j) v[j] = __fdividef(ph[j] * raw_k(t0 + j) * s_si[t0 + j], ga[j]);
+      st_row16_split(sm + O_KKH2, sm + O_KKL2, ci, qq, v);  // Kk^T hi / lo
     }
     fence_proxy_async();
     tc_fence_before();
     __syncthreads();
     if (tid == 0) {
       tc_fence_after();
-      const uint32_t id11 = idesc_bf16(128, 64, 1, 1), id10 = idesc_bf16(128, 64, 1, 0);
+      const uint32_t id01 = idesc_bf16(128, 64, 0, 1), id00 = idesc_bf16(128, 64, 0, 0);
       for (int kk = 0; kk < 4; ++kk) {
-        const uint64_t kh = mdesc(sm + O_KKH2 + kk * 2048, 8192), kl = mdesc(sm + O_KKL2 + kk * 2048, 8192);
+        const uint64_t kh = kdesc(sm + O_KKH2 + kk * 32), kl = kdesc(sm + O_KKL2 + kk * 32);
         const uint64_t dh = mdesc(sm + O_DAQ + kk * 2048, 8192), dl = mdesc(sm + O_DAQ + 8192 + kk * 2048, 8192);
-        umma_bf16(X3, kh, dh, id11, 1);
-        umma_bf16(X3, kl, dh, id11, 1);
-        umma_bf16(X3, kh, dl, id11, 1);
-        const uint64_t qh = mdesc(sm + O_KQH2 + 8192 + kk * 2048, 16384), ql = mdesc(sm + O_QL2 + kk * 2048, 8192);
+        umma_bf16(X3, kh, dh, id01, 1);
+        umma_bf16(X3, kl, dh, id01, 1);
+        umma_bf16(X3, kh, dl, id01, 1);
+        const uint64_t qh = kdesc(sm + O_KQH2 + 16384 + kk * 32), ql = kdesc(sm + O_QL2 + kk * 32);
         const uint64_t eh = kdesc(sm + O_DAQ + kk * 32), el = kdesc(sm + O_DAQ + 8192 + kk * 32);
-        umma_bf16(X0, qh, eh, id10, 1);
-        umma_bf16(X0, ql, eh, id10, 1);
-        umma_bf16(X0, qh, el, id10, 1);
+        umma_bf16(X0, qh, eh, id00, 1);
+        umma_bf16(X0, ql, eh, id00, 1);
+        umma_bf16(X0, qh, el, id00, 1);
       }
       umma_commit(bar_mma);
     }
@@ -713,11 +717,12 @@ __global__ void __launch_bounds__(BT, 1)
     if (tid == 0) {
       tc_fence_after();
       const uint32_t ih01 = idesc_f16(128, 64, 0, 1), ib01 = idesc_bf16(128, 64, 0, 1);
+      const uint32_t ib11 = idesc_bf16(128, 64, 1, 1);
       for (int kk = 0; kk < 8; ++kk) {
         umma_bf16(X1, kdesc(rv + (kk >> 2) * 8192 + (kk & 3) * 32), mdesc(sm + O_DRT + kk * 2048, 8192),
                   ih01, kk > 0);
-        umma_bf16(X1, kdesc(sm + O_KQH2 + (kk >> 2) * 16384 + (kk & 3) * 32),
-                  mdesc(sm + O_DWT + kk * 2048, 8192), ib01, 1);
+        umma_bf16(X1, mdesc(sm + O_KQH2 + kk * 2048, 16384), mdesc(sm + O_DWT + kk * 2048, 8192), ib11,
+                  1);
       }
       for (int kk = 0; kk < 4; ++kk)
         umma_bf16(X2, kdesc(sm + O_DWT + kk * 32), mdesc(sm + O_AB + kk * 2048, 8192), ib01, kk > 0);
@@ -780,10 +785,10 @@ __global__ void __launch_bounds__(BT, 1)
     // ---- [17] B9b: X0 += (dT^T Kbar)^T;  B10b: X2 += (dT Kk)^T
     if (tid == 0) {
       tc_fence_after();
-      const uint32_t id11 = idesc_bf16(128, 64, 1, 1), id10 = idesc_bf16(128, 64, 1, 0);
+      const uint32_t id01 = idesc_bf16(128, 64, 0, 1), id00 = idesc_bf16(128, 64, 0, 0);
       for (int kk = 0; kk < 4; ++kk) {
-        umma_bf16(X0, mdesc(sm + O_KQH2 + kk * 2048, 16384), mdesc(sm + O_DT + kk * 2048, 8192), id11, 1);
-        umma_bf16(X2, mdesc(sm + O_KKH2 + kk * 2048, 8192), kdesc(sm + O_DT + kk * 32), id10, 1);
+        umma_bf16(X0, kdesc(sm + O_KQH2 + kk * 32), mdesc(sm + O_DT + kk * 2048, 8192), id01, 1);
+        umma_bf16(X2, kdesc(sm + O_KKH2 + kk * 32), kdesc(sm + O_DT + kk * 32), id00, 1);
       }
       umma_commit(bar_mma);
     }
@@ -791,141 +796,152 @@ __global__ void __launch_bounds__(BT, 1)
     tc_fence_after();
     if (tid == 0 && c > 0) issue_a_gws(c - 1);  // g, omega, S_in buffers are free
     // ---- [18] per channel (lane ci, tokens t0..t0+15): back through Gamma and the
-    //           gain emission, then the uncertainty recursion backwards in time
+    //           gain emission, then the uncertainty recursion backwards in time.
+    //           Free TMEM columns hold per-(channel, token) intermediates between passes:
+    //           X2 <- dphat (gain part), X1 <- dk (memory + gain part), X0 <- alpha^2,
+    //           X3 <- 1 / (1 + u phat).
     {
-      float *sdg = reinterpret_cast<float *>(bkql);  // [16][512] dG -> reverse cumsum
+      float *sdg = reinterpret_cast<float *>(bkql);  // [16][512] dG_t
       float *s_tot = reinterpret_cast<float *>(sm + O_RH);  // [4][128] quarter sums of dG
       float *s_dgc = s_tot + 512;                           // [4][128] dgamma_C parts
       float *s_aff = s_dgc + 512;                           // [4][128][2] affine summaries
-      float part[16];
-#pragma unroll
-      for (int h8 = 0; h8 < 2; ++h8) {
-        float xq[8], xk[8], xb[8], ph[8], ga[8];
-        tmem_ld8(X3 + lane_base + t0 + 8 * h8, xq);
-        tmem_ld8(X0 + lane_base + t0 + 8 * h8, xk);
-        tmem_ld8(X2 + lane_base + t0 + 8 * h8, xb);
-        tmem_ld8(TPH + lane_base + t0 + 8 * h8, ph);
-        tmem_ld8(TGM + lane_base + t0 + 8 * h8, ga);
-#pragma unroll
-        for (int u = 0; u < 8; ++u) {
-          const int j = 8 * h8 + u, t = t0 + j;
-          const float kk = raw_k(t), qv = raw_q(t);
-          const float kap = __fdividef(ph[u] * kk, s_s[t]);
-          const float Kk = __fdividef(kap, ga[u]);
-          sdg[j * BT + tid] = xb[u] * ga[u] * kk - xk[u] * Kk + xq[u] * tau * ga[u] * qv;
-          part[j] = __fdividef(xk[u], ga[u]) * kap;  // dkappa . kappa
-          const int tt = c * CM + t;
-          if (tt < a.T) sto(a.odt, a.dq, tok_index(a, b, tt, h) * D + ci, tau * ga[u] * xq[u] * invl);
-        }
-      }
-      s_dgc[qq * D + ci] = dgc;
-      const float rsum = rs16(part, lane);
-      if ((lane & 1) == 0) s_red[wq * 64 + t0 + (lane >> 1)] = rsum;
-      __syncthreads();
-      if (qq == 3) {
-        const float dgC = (s_dgc[ci] + s_dgc[D + ci]) + (s_dgc[2 * D + ci] + s_dgc[3 * D + ci]);
-        sdg[15 * BT + tid] += dgC * s_gC[ci];
-      }
-      float tot = 0.f;
-#pragma unroll
-      for (int j = 0; j < 16; ++j) tot += sdg[j * BT + tid];
-      s_tot[qq * D + ci] = tot;
-      __syncthreads();
-      {
-        float run = 0.f;
-        for (int q2 = qq + 1; q2 < 4; ++q2) run += s_tot[q2 * D + ci];
-#pragma unroll
-        for (int j = 15; j >= 0; --j) {
-          run += sdg[j * BT + tid];
-          sdg[j * BT + tid] = run;
-        }
-      }
-      // per-token values of the recursion
-      float ph[16], ga[16];
+      float ph[16], ga[16], k16[16];
       load_ph_ga(ph, ga);
+#pragma unroll
+      for (int j = 0; j < 16; ++j) k16[j] = raw_k(t0 + j);
+      // outputs of token t0 + j live at obase + j * ostride; nval tokens of the quarter are real
+      const size_t ostride = (size_t)a.H * D;
+      const size_t obase = tok_index(a, b, c * CM + t0, h) * D + ci;
+      const int nval = min(16, a.T - (c * CM + t0));
+      const bool obf = a.odt == KDN_BF16;
+      auto out = [&](void *p, int j, float x) {
+        const size_t idx = obase + (size_t)j * ostride;
+        if (obf) static_cast<__nv_bfloat16 *>(p)[idx] = __float2bfloat16_rn(x);
+        else static_cast<float *>(p)[idx] = x;
+      };
+      // pass A: dq, dG, the ds_t partial sums and the ds-free parts of dphat and dk
+      {
+        float part[16], tot = 0.f;
+#pragma unroll
+        for (int h8 = 0; h8 < 2; ++h8) {
+          float xq[8], xk[8], xb[8], c1[8], c2[8];
+          tmem_ld8(X3 + lane_base + t0 + 8 * h8, xq);
+          tmem_ld8(X0 + lane_base + t0 + 8 * h8, xk);
+          tmem_ld8(X2 + lane_base + t0 + 8 * h8, xb);
+#pragma unroll
+          for (int u = 0; u < 8; ++u) {
+            const int j = 8 * h8 + u, t = t0 + j;
+            const float kk = k16[j], qv = raw_q(t), si = s_si[t], g_ = ga[j], ig = __fdividef(1.f, g_);
+            const float kap = ph[j] * kk * si;  // kappa_t (eq. kla-box-gain)
+            const float dG = xb[u] * g_ * kk - xk[u] * kap * ig + xq[u] * tau * g_ * qv;
+            sdg[j * BT + tid] = dG;
+            tot += dG;
+            const float dkap = xk[u] * ig;
+            part[j] = dkap * kap;
+            c1[u] = dkap * kk * si;
+            c2[u] = xb[u] * g_ + dkap * ph[j] * si;
+            if (j < nval) out(a.dq, j, tau * g_ * xq[u] * invl);
+          }
+          tmem_st8(X2 + lane_base + t0 + 8 * h8, c1);
+          tmem_st8(X1 + lane_base + t0 + 8 * h8, c2);
+        }
+        s_dgc[qq * D + ci] = dgc;
+        s_tot[qq * D + ci] = tot;
+        const float rsum = rs16(part, lane);
+        if ((lane & 1) == 0) s_red[wq * 64 + t0 + (lane >> 1)] = rsum;
+      }
+      tmem_st_wait();
+      __syncthreads();
+      if (tid < CM) s_ds[tid] = -((s_red[tid] + s_red[64 + tid]) + (s_red[128 + tid] + s_red[192 + tid])) * s_si[tid];
+      __syncthreads();
+      // entry values of this quarter: gamma_{t0-1}, p_{t0-1}
       float ga_prev = 1.f, p_prev;
       if (qq > 0) {
         float t8[8], g8[8];
         tmem_ld8(TPH + lane_base + t0 - 8, t8);
         tmem_ld8(TGM + lane_base + t0 - 8, g8);
         const float kk = raw_k(t0 - 1);
-        ga_prev = g8[7];
+        ga_prev = g8[7];  // gamma_{t0-1}
         p_prev = __fdividef(t8[7], 1.f + mu * kk * kk * s_ri[t0 - 1] * t8[7]);
       } else {
         p_prev = a.fpin[((size_t)bh * NC + c) * D + ci];
       }
-      auto ds_of = [&](int t) {
-        return -((s_red[t] + s_red[64 + t]) + (s_red[128 + t] + s_red[192 + t])) / s_s[t];
-      };
-      // affine summary of this quarter: dp_before = A dp_after + B
+      // pass B: per-token coefficients of dp_{t-1} = a_t dp_t + b_t and the quarter's
+      //         composition dp_before = A dp_after + B
       {
         float A = 1.f, Bv = 0.f;
-        float xk[16];
-        tmem_ld16(X0 + lane_base + t0, xk);
 #pragma unroll
-        for (int j = 15; j >= 0; --j) {
-          const int t = t0 + j;
-          const float kk = raw_k(t), sinv = 1.f / s_s[t];
-          const float gp = j > 0 ? ga[j - 1] : ga_prev;
-          const float al = __fdividef(ga[j], gp), al2 = al * al;
-          const float den = 1.f + mu * kk * kk * s_ri[t] * ph[j];
-          const float dphl = __fdividef(xk[j], ga[j]) * kk * sinv + ds_of(t) * kk * kk;
-          const float aj = __fdividef(al2, den * den);
-          Bv = aj * Bv + al2 * dphl;
-          A = aj * A;
+        for (int h8 = 1; h8 >= 0; --h8) {
+          float c1[8], a2v[8], rdv[8];
+          tmem_ld8(X2 + lane_base + t0 + 8 * h8, c1);
+#pragma unroll
+          for (int u = 7; u >= 0; --u) {
+            const int j = 8 * h8 + u, t = t0 + j;
+            const float kk = k16[j];
+            const float al = __fdividef(ga[j], j > 0 ? ga[j - 1] : ga_prev), al2 = al * al;
+            const float rd = __fdividef(1.f, 1.f + mu * kk * kk * s_ri[t] * ph[j]);
+            const float dphl = c1[u] + s_ds[t] * kk * kk;
+            const float aj = al2 * rd * rd;
+            Bv = aj * Bv + al2 * dphl;
+            A = aj * A;
+            a2v[u] = al2;
+            rdv[u] = rd;
+            c1[u] = dphl;
+          }
+          tmem_st8(X0 + lane_base + t0 + 8 * h8, a2v);
+          tmem_st8(X3 + lane_base + t0 + 8 * h8, rdv);
+          tmem_st8(X2 + lane_base + t0 + 8 * h8, c1);
         }
         s_aff[(qq * D + ci) * 2] = A;
         s_aff[(qq * D + ci) * 2 + 1] = Bv;
       }
+      tmem_st_wait();
       __syncthreads();
-      float dp = s_dp[ci];
-      for (int q2 = 3; q2 > qq; --q2) dp = s_aff[(q2 * D + ci) * 2] * dp + s_aff[(q2 * D + ci) * 2 + 1];
-      float drp[16];
+      // pass C: the recursion backwards through this quarter's tokens
       {
-        float xk[16], xb[16];
-        tmem_ld16(X0 + lane_base + t0, xk);
-        tmem_ld16(X2 + lane_base + t0, xb);
+        float dp = s_dp[ci];
+        for (int q2 = 3; q2 > qq; --q2) dp = s_aff[(q2 * D + ci) * 2] * dp + s_aff[(q2 * D + ci) * 2 + 1];
+        const float dgC = (s_dgc[ci] + s_dgc[D + ci]) + (s_dgc[2 * D + ci] + s_dgc[3 * D + ci]);
+        float run = dgC * s_gC[ci];  // dG_63 gains dgamma_C gamma_C; it lies in every suffix
+        for (int q2 = qq + 1; q2 < 4; ++q2) run += s_tot[q2 * D + ci];
+        float rd16[16], drp[16];
+        tmem_ld16(X3 + lane_base + t0, rd16);
 #pragma unroll
-        for (int j = 15; j >= 0; --j) {
-          const int t = t0 + j, tt = c * CM + t;
-          const float kk = raw_k(t), sinv = 1.f / s_s[t], ds = ds_of(t);
-          const float gp = j > 0 ? ga[j - 1] : ga_prev;
-          const float al = __fdividef(ga[j], gp), al2 = al * al;
-          const float u = mu * kk * kk * s_ri[t];
-          const float den = 1.f + u * ph[j], pt = __fdividef(ph[j], den);
-          float pprev;
-          if (j > 0) {
-            const float kp = raw_k(t - 1);
-            pprev = __fdividef(ph[j - 1], 1.f + mu * kp * kp * s_ri[t - 1] * ph[j - 1]);
-          } else {
-            pprev = p_prev;
+        for (int h8 = 1; h8 >= 0; --h8) {
+          float a2v[8], dphl[8], c2[8];
+          tmem_ld8(X0 + lane_base + t0 + 8 * h8, a2v);
+          tmem_ld8(X2 + lane_base + t0 + 8 * h8, dphl);
+          tmem_ld8(X1 + lane_base + t0 + 8 * h8, c2);
+#pragma unroll
+          for (int u = 7; u >= 0; --u) {
+            const int j = 8 * h8 + u, t = t0 + j;
+            const float kk = k16[j], ds = s_ds[t], ri = s_ri[t];
+            const float pt = ph[j] * rd16[j];
+            const float pprev = j > 0 ? ph[j - 1] * rd16[j - 1] : p_prev;
+            const float dph = dp * rd16[j] * rd16[j] + dphl[u];
+            const float du = -dp * pt * pt;
+            const float dkt = c2[u] + 2.f * ds * ph[j] * kk + du * 2.f * mu * kk * ri;
+            drp[j] = -du * mu * kk * kk * ri * ri;
+            run += sdg[j * BT + tid];
+            const float dgt = run + 2.f * a2v[u] * pprev * dph;
+            if (j < nval) {
+              out(a.dk_, j, dkt * invl);
+              out(a.domega, j, dph * invl);
+              out(a.dg, j, dgt * invl);
+            }
+            dp = a2v[u] * dph;
           }
-          const float dkap = __fdividef(xk[j], ga[j]);
-          const float dphl = dkap * kk * sinv + ds * kk * kk;
-          const float dph = __fdividef(dp, den * den) + dphl;
-          const float du = -dp * pt * pt;
-          const float dkt = xb[j] * ga[j] + dkap * ph[j] * sinv + 2.f * ds * ph[j] * kk +
-                            du * 2.f * mu * kk * s_ri[t];
-          drp[j] = -du * u * s_ri[t];
-          const float dgt = sdg[j * BT + tid] + 2.f * al2 * pprev * dph;
-          if (tt < a.T) {
-            const size_t idx = tok_index(a, b, tt, h) * D + ci;
-            sto(a.odt, a.dk_, idx, dkt * invl);
-            sto(a.odt, a.domega, idx, dph * invl);
-            sto(a.odt, a.dg, idx, dgt * invl);
-          }
-          dp = al2 * dph;
         }
-      }
-      const float rs2 = rs16(drp, lane);
-      if ((lane & 1) == 0) s_red2[wq * 64 + t0 + (lane >> 1)] = rs2;
-      __syncthreads();
-      if (qq == 0) s_dp[ci] = dp;
-      if (tid < CM) {
-        const int tt = c * CM + tid;
-        if (tt < a.T) {
-          const float dr = ds_of(tid) + ((s_red2[tid] + s_red2[64 + tid]) + (s_red2[128 + tid] + s_red2[192 + tid]));
-          sto(a.odt, a.dr, tok_index(a, b, tt, h), dr * invl);
+        const float rs2 = rs16(drp, lane);
+        if ((lane & 1) == 0) s_red2[wq * 64 + t0 + (lane >> 1)] = rs2;
+        __syncthreads();
+        if (qq == 0) s_dp[ci] = dp;
+        if (tid < CM) {
+          const int tt = c * CM + tid;
+          if (tt < a.T) {
+            const float dr = s_ds[tid] + ((s_red2[tid] + s_red2[64 + tid]) + (s_red2[128 + tid] + s_red2[192 + tid]));
+            sto(a.odt, a.dr, tok_index(a, b, tt, h), dr * invl);
+          }
         }
       }
     }
