@@ -1,13 +1,16 @@
 """Benchmark of the KDN token-mixer hot path on GB300.
 
-One step = one Diagonal-KDN forward + backward (all steps of the chunked
-forward, its adjoint) over one synthetic batch shaped like a 1.3B-model layer:
-B=8, H=16, T=4096, d_k=d_v=128, bfloat16 activations, float32 state and
-outputs.  `value` is layer tokens/s (B*T per step, summed over ranks).  The
-same JSON line also carries the decode step (B=256, H=16, d=128, 1024
-consecutive tokens in one CUDA graph) in steps/s, the forward kernel's
-roofline, an end-to-end number through host buffers, and the oracle's CPU
-throughput on a bounded sample.
+One step = one Diagonal-KDN training forward + backward (all steps of the
+chunked forward, its adjoint) over one synthetic batch shaped like a 1.3B-model
+layer: B=8, H=16, T=4096, d_k=d_v=128, bfloat16 activations, float32 state and
+outputs.  The forward is kdn_diag_fwd_save (o, S_T, p_T and the per-chunk
+context of the backward) and the backward kdn_diag_bwd_saved (every gradient
+from that context); each is one kernel.  `value` is layer tokens/s (B*T per
+step, summed over ranks).  The same JSON line also carries the decode step
+(B=256, H=16, d=128, 1024 consecutive tokens in one CUDA graph) in steps/s, the
+roofline of the dominant kernel (the backward sweep) and of the forward, an
+end-to-end number through host buffers, and the oracle's CPU throughput on a
+bounded sample.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
 
@@ -67,6 +70,12 @@ def decode_bytes(b, h, dk, dv, in_bytes=2, out_bytes=4):
     state = 2 * (dk * dv * 4 + dk * 4)
     ins = (2 * dk + dv + 2 * dk + 1) * in_bytes
     return b * h * (state + ins + dv * out_bytes)
+
+
+# DRAM bytes per launch of each kernel at the bench workload, from one ncu
+# capture (dram__bytes_read.sum + dram__bytes_write.sum) of the current build;
+# reported as `traffic` only for that workload.
+NCU_TRAFFIC = {"k_fused_fwd": 672308736 + 502762752, "k_fused_bwd": 1207841280 + 1341476608}
 
 
 def chunk_flops(dk, dv, C=64):
@@ -213,7 +222,8 @@ def run_gpu(args):
     x = [ins[n] for n in NAMES]
     desc = kdn.make_desc(B, T, H, DK, DV, dt)
     ws_f = kdn.alloc_workspace(desc, 0, False)
-    ws_b = kdn.alloc_workspace(desc, 0, True)
+    ws_b = kdn.alloc_workspace(desc, 0, False)
+    saved = torch.empty(kdn.saved_bytes(desc), dtype=torch.uint8, device="cuda")
     o = torch.empty(B, T, H, DV, dtype=torch.float32, device="cuda")
     ST = torch.empty(B, H, DK, DV, dtype=torch.float32, device="cuda")
     pT = torch.empty(B, H, DK, dtype=torch.float32, device="cuda")
@@ -227,18 +237,18 @@ def run_gpu(args):
     def step(ev=None):
         if ev is not None:
             ev[0].record(stream)
-        kdn.kdn_diag_fwd(*x, o=o, ST=ST, pT=pT, workspace=ws_f)
+        kdn.kdn_diag_fwd_save(*x, o=o, ST=ST, pT=pT, saved=saved, workspace=ws_f)
         if ev is not None:
             ev[1].record(stream)
         if not args.fwd_only:
-            kdn.kdn_diag_bwd(*x, None, None, ins["dO"], grads=grads, workspace=ws_b)
+            kdn.kdn_diag_bwd_saved(*x, saved, ins["dO"], grads=grads, workspace=ws_b)
         if ev is not None:
             ev[2].record(stream)
 
     for _ in range(args.warmup):
         step()
-    launches_per_step = kdn.kdn_kernel_launches(desc, 0, 0) + (
-        0 if args.fwd_only else kdn.kdn_kernel_launches(desc, 0, 1))
+    launches_per_step = kdn.kdn_kernel_launches(desc, 0, 3) + (
+        0 if args.fwd_only else kdn.kdn_kernel_launches(desc, 0, 4))
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
     start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     barrier(world)
@@ -258,13 +268,21 @@ def run_gpu(args):
 
     fb = fwd_bytes(B, T, H, DK, DV)
     bb = bwd_bytes(B, T, H, DK, DV)
-    roof = {"bound": "hbm", "kernel": "kdn_diag_fwd (forward entry point)",
-            "achieved": fb / (fwd_ms / 1e3) / 1e9, "peak": hbm, "unit": "GB/s",
-            "peak_kind": peak_kind, "traffic": None, "algorithmic_bytes": fb}
-    roof["frac"] = roof["achieved"] / roof["peak"]
-    bwd_roof = {"bound": "hbm", "achieved": bb / (bwd_ms / 1e3) / 1e9, "peak": hbm,
-                "unit": "GB/s", "algorithmic_bytes": bb}
+    # one kernel per call: k_fused_fwd<0> (forward + context), k_fused_bwd (backward sweep)
+    fwd_roof = {"bound": "hbm", "kernel": "k_fused_fwd (kdn_diag_fwd_save)",
+                "achieved": fb / (fwd_ms / 1e3) / 1e9, "peak": hbm, "unit": "GB/s",
+                "peak_kind": peak_kind, "algorithmic_bytes": fb, "ms": fwd_ms,
+                "traffic": NCU_TRAFFIC["k_fused_fwd"] if B == 8 else None}
+    fwd_roof["frac"] = fwd_roof["achieved"] / hbm
+    bwd_roof = {"bound": "hbm", "kernel": "k_fused_bwd (kdn_diag_bwd_saved)",
+                "achieved": bb / (bwd_ms / 1e3) / 1e9, "peak": hbm, "unit": "GB/s",
+                "peak_kind": peak_kind, "algorithmic_bytes": bb, "ms": bwd_ms,
+                "traffic": NCU_TRAFFIC["k_fused_bwd"] if B == 8 else None}
     bwd_roof["frac"] = bwd_roof["achieved"] / hbm
+    if args.fwd_only:
+        roof, other = fwd_roof, None
+    else:
+        roof, other = (bwd_roof, fwd_roof) if bwd_ms >= fwd_ms else (fwd_roof, bwd_roof)
     # the paper-style roofline: max(FLOPs / 2.25 PF, bytes / 8 TB/s)
     spec_time = max(B * T * H * chunk_flops(DK, DV) * 3.5 / 2.25e15, (fb + bb) / 8e12)
 
@@ -280,7 +298,7 @@ def run_gpu(args):
                    "state": "f32", "parallelism": f"replicas x{world}",
                    "l2": "inputs larger than L2 (each activation tensor 134 MB)"},
         "fwd_ms": fwd_ms, "bwd_ms": bwd_ms,
-        "roofline": roof, "bwd_roofline": bwd_roof,
+        "roofline": roof, "roofline_other_kernel": other,
         "spec_roofline_frac": spec_time / (ms_step / 1e3) if ms_step > 0 else None,
         "gpu_launches": launches_per_step * args.steps,
         "clocks": clk.summary(),
@@ -356,13 +374,15 @@ def run_e2e(kdn, torch, x, ins, args):
     dev_in = {n: torch.empty_like(ins[n]) for n in NAMES + ("dO",)}
     outs_host = {}
     stream = torch.cuda.current_stream()
+    saved = torch.empty(kdn.saved_bytes(kdn.make_desc(B, T, H, DK, DV, torch.bfloat16)),
+                        dtype=torch.uint8, device="cuda")
 
     def step():
         for n in NAMES + ("dO",):
             dev_in[n].copy_(host_in[n], non_blocking=True)
         xx = [dev_in[n] for n in NAMES]
-        o, _, _ = kdn.kdn_diag_fwd(*xx, want_state=False)
-        gr = kdn.kdn_diag_bwd(*xx, None, None, dev_in["dO"], want_state_grads=False)
+        o, _, _, sv = kdn.kdn_diag_fwd_save(*xx, want_state=False, saved=saved)
+        gr = kdn.kdn_diag_bwd_saved(*xx, sv, dev_in["dO"], want_state_grads=False)
         res = {"o": o, **gr}
         for n, t in res.items():
             if n not in outs_host:
@@ -397,7 +417,7 @@ def cpu_baseline(sample_heads=None):
     from kdn_inputs import make_inputs
     oracle.build()
     cores = os.cpu_count() or 1
-    n = sample_heads or min(2 * cores, B * H)
+    n = sample_heads or B * H  # the whole workload's (batch, head) sequences, ~5 s on 16 cores
     ins = make_inputs("diag", 1, T, n, DK, DV, dtype="bf16", seed=0, with_grad=True)
     args = [ins[k] for k in NAMES]
     t0 = time.perf_counter()
@@ -419,7 +439,7 @@ def run_reference(args):
     import oracle
     oracle.build()
     cores = os.cpu_count() or 1
-    n = min(2 * cores, B * H)
+    n = B * H
     samples = []
     for i in range(args.warmup + args.steps):
         cb = cpu_baseline(sample_heads=n)

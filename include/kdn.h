@@ -141,6 +141,40 @@ kdn_status_t kdn_iso_bwd(const kdn_desc_t *desc, const void *q, const void *k,
                          void *dr, float *dS0, float *dp0, void *workspace,
                          size_t workspace_bytes, void *stream);
 
+/* Training pair.  kdn_diag_fwd_save is kdn_diag_fwd that also keeps, in
+   `saved`, the context the chunked backward needs (App. F): for every 64-token
+   chunk an fp16 image of the memory S entering it and the float32 uncertainty
+   p entering it.  kdn_diag_bwd_saved is kdn_diag_bwd that starts from that
+   context instead of recomputing the forward (same gradients, one kernel).
+   Served for the Diagonal KDN with bfloat16 activations, dk = dv = 128 and the
+   default chunk; for every other descriptor kdn_saved_bytes() returns 0 and
+   both calls return KDN_ERR_UNSUPPORTED (use kdn_diag_fwd / kdn_diag_bwd).
+   saved: caller-owned device buffer of kdn_saved_bytes(desc, 0) bytes, 256-byte
+   aligned (a smaller or misaligned one -> KDN_ERR_WORKSPACE).  It is written
+   by kdn_diag_fwd_save and read by kdn_diag_bwd_saved, which must see the same
+   descriptor and the same q, k, v, g, omega, r (and the forward's S0, p0).
+   workspace: kdn_fwd_workspace_bytes(desc, 0) bytes for both calls.  The
+   other arguments are those of kdn_diag_fwd / kdn_diag_bwd. */
+size_t kdn_saved_bytes(const kdn_desc_t *desc, int variant);
+
+kdn_status_t kdn_diag_fwd_save(const kdn_desc_t *desc, const void *q,
+                               const void *k, const void *v, const void *g,
+                               const void *omega, const void *r,
+                               const float *S0, const float *p0, void *o,
+                               float *ST, float *pT, void *saved,
+                               size_t saved_bytes, void *workspace,
+                               size_t workspace_bytes, void *stream);
+
+kdn_status_t kdn_diag_bwd_saved(const kdn_desc_t *desc, const void *q,
+                                const void *k, const void *v, const void *g,
+                                const void *omega, const void *r,
+                                const void *saved, size_t saved_bytes,
+                                const void *dO, const float *dST,
+                                const float *dpT, void *dq, void *dk, void *dv,
+                                void *dg, void *domega, void *dr, float *dS0,
+                                float *dp0, void *workspace,
+                                size_t workspace_bytes, void *stream);
+
 /* One decode token for all B*H heads (the update of Prop. 3), in place:
    S [B,H,dk,dv] and p [B,H,dk] are read and overwritten; o [B,H,dv] is
    written.  Per-step inputs drop the T axis: q, k [B,H,dk], v [B,H,dv],
@@ -181,8 +215,10 @@ kdn_status_t kdn_diag_fwd_noalloc(const kdn_desc_t *desc, const void *q,
                                   float *ST, float *pT, void *stream);
 
 /* Number of CUDA kernels one call of an entry point launches for this
-   descriptor when T > 0 (op 0 = kdn_*_fwd, 1 = kdn_*_bwd, 2 = kdn_*_decode_step;
-   variant 0 = diagonal, 1 = isotropic).  -1 for an invalid descriptor or op.
+   descriptor when T > 0 (op 0 = kdn_*_fwd, 1 = kdn_*_bwd, 2 = kdn_*_decode_step,
+   3 = kdn_diag_fwd_save, 4 = kdn_diag_bwd_saved; variant 0 = diagonal,
+   1 = isotropic).  -1 for an invalid descriptor or op, or an op the descriptor
+   does not serve.
    Calls with T = 0 launch at most one small fill kernel. */
 int kdn_kernel_launches(const kdn_desc_t *desc, int variant, int op);
 

@@ -163,6 +163,69 @@ kdn_status_t bwd_entry(int variant, const kdn_desc_t *d, const void *q, const vo
   return launch_chunked_bwd(a, s);
 }
 
+// Training pair: forward that keeps the fused backward's context in `saved`,
+// and the backward sweep that starts from it.
+kdn_status_t fwd_save_entry(const kdn_desc_t *d, const void *q, const void *k, const void *v,
+                            const void *g, const void *omega, const void *r, const float *S0,
+                            const float *p0, void *o, float *ST, float *pT, void *saved,
+                            size_t saved_bytes, void *ws, size_t ws_bytes, void *stream) {
+  Args a;
+  kdn_status_t st = fill_sizes(d, 0, false, &a);
+  if (st != KDN_OK) return st;
+  const bool work = (size_t)a.B * a.H * a.T > 0;
+  if (work && !use_fused_bwd(a)) return KDN_ERR_UNSUPPORTED;
+  if (work && !ptrs_ok({q, k, v, g, omega, r, o, saved}, {S0, p0, ST, pT})) return KDN_ERR_INVALID_ARG;
+  if (!work && !ptrs_ok({}, {S0, p0, ST, pT})) return KDN_ERR_INVALID_ARG;
+  if (work && (saved_bytes < fused_saved_bytes(a) || ((uintptr_t)saved % kAlign)))
+    return KDN_ERR_WORKSPACE;
+  const size_t need = workspace_layout(&a, nullptr, false);
+  if (need > ws_bytes || (need && (!ws || ((uintptr_t)ws % kAlign)))) return KDN_ERR_WORKSPACE;
+  workspace_layout(&a, static_cast<char *>(ws), false);
+  a.q = q; a.k = k; a.v = v; a.g = g; a.omega = omega; a.r = r;
+  a.S0 = S0; a.p0 = p0; a.o = o; a.ST = ST; a.pT = pT;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (cudaMemsetAsync(a.status, 0, sizeof(unsigned), s) != cudaSuccess) return KDN_ERR_CUDA;
+  if ((size_t)a.B * a.H == 0) return KDN_OK;
+  if (a.T == 0) return empty_fwd(a, s);
+  const size_t nsv = (size_t)a.B * a.H * ((a.T + 63) / 64) * 32768;
+  return launch_fused_fwd(a, s, static_cast<unsigned char *>(saved),
+                          reinterpret_cast<float *>(static_cast<char *>(saved) + nsv), true);
+}
+
+kdn_status_t bwd_saved_entry(const kdn_desc_t *d, const void *q, const void *k, const void *v,
+                             const void *g, const void *omega, const void *r, const void *saved,
+                             size_t saved_bytes, const void *dO, const float *dST,
+                             const float *dpT, void *dq, void *dk, void *dv, void *dg,
+                             void *domega, void *dr, float *dS0, float *dp0, void *ws,
+                             size_t ws_bytes, void *stream) {
+  Args a;
+  kdn_status_t st = fill_sizes(d, 0, false, &a);
+  if (st != KDN_OK) return st;
+  const bool work = (size_t)a.B * a.H * a.T > 0;
+  if (work && !use_fused_bwd(a)) return KDN_ERR_UNSUPPORTED;
+  if (work && !ptrs_ok({q, k, v, g, omega, r, saved, dO, dq, dk, dv, dg, domega, dr},
+                       {dST, dpT, dS0, dp0}))
+    return KDN_ERR_INVALID_ARG;
+  if (!work && !ptrs_ok({}, {dST, dpT, dS0, dp0})) return KDN_ERR_INVALID_ARG;
+  if (work && (saved_bytes < fused_saved_bytes(a) || ((uintptr_t)saved % kAlign)))
+    return KDN_ERR_WORKSPACE;
+  const size_t need = workspace_layout(&a, nullptr, false);
+  if (need > ws_bytes || (need && (!ws || ((uintptr_t)ws % kAlign)))) return KDN_ERR_WORKSPACE;
+  workspace_layout(&a, static_cast<char *>(ws), false);
+  a.q = q; a.k = k; a.v = v; a.g = g; a.omega = omega; a.r = r;
+  a.dO = dO; a.dST = dST; a.dpT = dpT;
+  a.dq = dq; a.dk_ = dk; a.dv_ = dv; a.dg = dg; a.domega = domega; a.dr = dr;
+  a.dS0 = dS0; a.dp0 = dp0;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (cudaMemsetAsync(a.status, 0, sizeof(unsigned), s) != cudaSuccess) return KDN_ERR_CUDA;
+  if ((size_t)a.B * a.H == 0) return KDN_OK;
+  if (a.T == 0) return empty_bwd(a, s);
+  const size_t nsv = (size_t)a.B * a.H * ((a.T + 63) / 64) * 32768;
+  a.fSin = static_cast<unsigned char *>(const_cast<void *>(saved));
+  a.fpin = reinterpret_cast<float *>(static_cast<char *>(const_cast<void *>(saved)) + nsv);
+  return launch_fused_bwd_sweep(a, s);
+}
+
 kdn_status_t decode_entry(int variant, const kdn_desc_t *d, const void *q, const void *k,
                           const void *v, const void *g, const void *omega, const void *r,
                           float *S, float *p, void *o, void *stream) {
@@ -284,6 +347,31 @@ kdn_status_t kdn_iso_bwd(const kdn_desc_t *desc, const void *q, const void *k, c
                    dr, dS0, dp0, workspace, workspace_bytes, stream);
 }
 
+size_t kdn_saved_bytes(const kdn_desc_t *desc, int variant) {
+  Args a;
+  if (fill_sizes(desc, variant, false, &a) != KDN_OK) return 0;
+  return fused_saved_bytes(a);
+}
+
+kdn_status_t kdn_diag_fwd_save(const kdn_desc_t *desc, const void *q, const void *k,
+                               const void *v, const void *g, const void *omega, const void *r,
+                               const float *S0, const float *p0, void *o, float *ST, float *pT,
+                               void *saved, size_t saved_bytes, void *workspace,
+                               size_t workspace_bytes, void *stream) {
+  return fwd_save_entry(desc, q, k, v, g, omega, r, S0, p0, o, ST, pT, saved, saved_bytes,
+                        workspace, workspace_bytes, stream);
+}
+
+kdn_status_t kdn_diag_bwd_saved(const kdn_desc_t *desc, const void *q, const void *k,
+                                const void *v, const void *g, const void *omega, const void *r,
+                                const void *saved, size_t saved_bytes, const void *dO,
+                                const float *dST, const float *dpT, void *dq, void *dk, void *dv,
+                                void *dg, void *domega, void *dr, float *dS0, float *dp0,
+                                void *workspace, size_t workspace_bytes, void *stream) {
+  return bwd_saved_entry(desc, q, k, v, g, omega, r, saved, saved_bytes, dO, dST, dpT, dq, dk, dv,
+                         dg, domega, dr, dS0, dp0, workspace, workspace_bytes, stream);
+}
+
 kdn_status_t kdn_diag_decode_step(const kdn_desc_t *desc, const void *q, const void *k,
                                   const void *v, const void *g, const void *omega, const void *r,
                                   float *S, float *p, void *o, void *stream) {
@@ -303,6 +391,8 @@ int kdn_kernel_launches(const kdn_desc_t *desc, int variant, int op) {
     case 0: return use_fused(a) ? 1 : chunked_fwd_launches(a);
     case 1: return (a.T > 0 && use_fused_bwd(a)) ? 2 : chunked_bwd_launches(a);
     case 2: return 1;
+    case 3:
+    case 4: return (variant == 0 && fused_saved_bytes(a) > 0) ? 1 : -1;
   }
   return -1;
 }

@@ -987,14 +987,13 @@ bool fused_bwd_supported(const Args &a) {
   return a.variant == 0 && a.chunk != 32 && fused_fwd_supported(a);
 }
 
-kdn_status_t launch_fused_bwd(const Args &a, cudaStream_t s) {
-  // state-saving forward pass
-  Args f = a;
-  f.o = nullptr;
-  f.ST = nullptr;
-  f.pT = nullptr;
-  kdn_status_t st = launch_fused_fwd(f, s, a.fSin, a.fpin);
-  if (st != KDN_OK) return st;
+size_t fused_saved_bytes(const Args &a) {
+  if (!fused_bwd_supported(a)) return 0;
+  const size_t nc = (a.T + CM - 1) / CM;
+  return (size_t)a.B * a.H * nc * (32768 + D * sizeof(float));
+}
+
+kdn_status_t launch_fused_bwd_sweep(const Args &a, cudaStream_t s) {
   BwdParams P;
   P.a = a;
   CUtensorMap mq, mk, mv, mg, mw, mdo;
@@ -1006,6 +1005,17 @@ kdn_status_t launch_fused_bwd(const Args &a, cudaStream_t s) {
     return KDN_ERR_CUDA;
   k_fused_bwd<<<a.B * a.H, BT, SMEM_BYTES, s>>>(mq, mk, mv, mg, mw, mdo, P);
   return cudaGetLastError() == cudaSuccess ? KDN_OK : KDN_ERR_CUDA;
+}
+
+kdn_status_t launch_fused_bwd(const Args &a, cudaStream_t s) {
+  // context-saving forward pass (o, S_T, p_T are not written)
+  Args f = a;
+  f.o = nullptr;
+  f.ST = nullptr;
+  f.pT = nullptr;
+  kdn_status_t st = launch_fused_fwd(f, s, a.fSin, a.fpin, false);
+  if (st != KDN_OK) return st;
+  return launch_fused_bwd_sweep(a, s);
 }
 
 }  // namespace kdn

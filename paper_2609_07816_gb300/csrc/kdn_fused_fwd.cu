@@ -672,12 +672,12 @@ bool fused_fwd_supported(const Args &a) {
 int fused_fwd_smem_bytes() { return SMEM_BYTES; }
 
 kdn_status_t launch_fused_fwd(const Args &a, cudaStream_t s, unsigned char *save_S,
-                              float *save_p) {
+                              float *save_p, bool write_o) {
   FusedParams P;
   P.a = a;
   P.has_g_map = (a.variant == 0 || a.pcd) ? 1 : 0;
   P.has_w_map = a.variant == 0 ? 1 : 0;
-  P.write_o = save_S ? 0 : 1;
+  P.write_o = write_o ? 1 : 0;
   P.save_S = save_S;
   P.save_p = save_p;
   CUtensorMap mq, mk, mv, mg, mw, mo;

@@ -97,16 +97,20 @@ __host__ __device__ inline size_t tok_index(const Args &a, int b, int t, int h) 
 size_t workspace_layout(Args *a, char *base, bool bwd);
 
 // Fused tcgen05 forward (bf16, dk = dv = 128, 64-token chunks).  With
-// `save_S` / `save_p` it is the state-saving pass of the fused backward: o is
-// not written; the fp16 image of every chunk's entry memory (32 KB) and the
-// uncertainty carry entering every chunk (128 floats) are stored instead.
+// `save_S` / `save_p` it also stores the context of the fused backward: the
+// fp16 image of every chunk's entry memory (32 KB) and the uncertainty entering
+// every chunk (128 floats); `write_o` = false skips the outputs o.
 bool fused_fwd_supported(const Args &a);
 kdn_status_t launch_fused_fwd(const Args &a, cudaStream_t s, unsigned char *save_S = nullptr,
-                              float *save_p = nullptr);
+                              float *save_p = nullptr, bool write_o = true);
 // Fused tcgen05 backward (Diagonal KDN, bf16, dk = dv = 128, 64-token chunks):
-// a state-saving forward pass, then one reverse sweep per (batch, head).
+// one reverse sweep per (batch, head) from the saved context in a.fSin / a.fpin.
+// launch_fused_bwd first runs the context-saving forward (without o).
 bool fused_bwd_supported(const Args &a);
 kdn_status_t launch_fused_bwd(const Args &a, cudaStream_t s);
+kdn_status_t launch_fused_bwd_sweep(const Args &a, cudaStream_t s);
+// Bytes of the saved context for the fused backward (0 if not served).
+size_t fused_saved_bytes(const Args &a);
 
 // Launchers (each returns KDN_OK or KDN_ERR_CUDA).
 kdn_status_t launch_chunked_fwd(const Args &a, cudaStream_t s, bool save_states);

@@ -161,3 +161,32 @@ def test_fused_path_launches_and_workspace(kdn):
     assert kdn.kdn_kernel_launches(d, 1, 1) > 2
     d32 = kdn.make_desc(B, T, H, 128, 128, kdn.KDN_BF16, chunk=32)
     assert kdn.kdn_kernel_launches(d32, 0, 1) > 2
+
+
+def test_training_pair_validation(kdn):
+    """kdn_diag_fwd_save / kdn_diag_bwd_saved: served only for the fused shapes;
+    the saved buffer is checked for size and alignment before anything runs."""
+    L = kdn.lib()
+    B, T, H = 2, 130, 3
+    d = kdn.make_desc(B, T, H, 128, 128, kdn.KDN_BF16)
+    n = kdn.saved_bytes(d)
+    assert n == B * H * 3 * (32768 + 512)
+    assert kdn.saved_bytes(d, 1) == 0
+    assert kdn.saved_bytes(kdn.make_desc(B, T, H, 64, 128, kdn.KDN_BF16)) == 0
+    assert kdn.saved_bytes(kdn.make_desc(B, T, H, 128, 128, kdn.KDN_F32)) == 0
+    assert kdn.kdn_kernel_launches(d, 0, 3) == 1 and kdn.kdn_kernel_launches(d, 0, 4) == 1
+    assert kdn.kdn_kernel_launches(d, 1, 3) == -1
+
+    def fwd_save(desc, saved=FAKE, saved_bytes=1 << 40):
+        return L.kdn_diag_fwd_save(ctypes.byref(desc), *([FAKE] * 11), saved, saved_bytes, FAKE,
+                                   1 << 40, None)
+
+    def bwd_saved(desc, saved=FAKE, saved_bytes=1 << 40):
+        return L.kdn_diag_bwd_saved(ctypes.byref(desc), *([FAKE] * 6), saved, saved_bytes,
+                                    *([FAKE] * 11), FAKE, 1 << 40, None)
+
+    for fn in (fwd_save, bwd_saved):
+        assert fn(kdn.make_desc(B, T, H, 64, 128, kdn.KDN_BF16)) == kdn.KDN_ERR_UNSUPPORTED
+        assert fn(d, saved_bytes=n - 1) == kdn.KDN_ERR_WORKSPACE
+        assert fn(d, saved=MIS) in (kdn.KDN_ERR_INVALID_ARG, kdn.KDN_ERR_WORKSPACE)
+        assert fn(d, saved=None) == kdn.KDN_ERR_INVALID_ARG

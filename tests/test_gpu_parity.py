@@ -281,3 +281,25 @@ def test_fused_backward_bf16_stored_gradients(kdn):
     for n in ("dq", "dk", "dv", "dg", "domega", "dr"):
         assert gr[n].dtype == torch.bfloat16
         check_stored_bf16(n, gr[n], rg[n])
+
+
+def test_training_pair_matches_recompute_path(kdn):
+    """kdn_diag_fwd_save writes the forward's outputs bit for bit; kdn_diag_bwd_saved
+    gives the gradients of kdn_diag_bwd bit for bit (same sweep, same context) and
+    matches the oracle."""
+    ins = _diag_bwd_inputs(2, 150, 2, 51)
+    d = to_dev(ins)
+    x = [d[n] for n in ("q", "k", "v", "g", "omega", "r")]
+    o1, ST1, pT1 = kdn.kdn_diag_fwd(*x, d["S0"], d["p0"])
+    o2, ST2, pT2, saved = kdn.kdn_diag_fwd_save(*x, d["S0"], d["p0"])
+    torch.cuda.synchronize()
+    assert torch.equal(o1, o2) and torch.equal(ST1, ST2) and torch.equal(pT1, pT2)
+    f32 = lambda a: torch.tensor(a, dtype=torch.float32, device="cuda")
+    g1 = kdn.kdn_diag_bwd(*x, d["S0"], d["p0"], d["dO"], f32(ins["dST"]), f32(ins["dpT"]))
+    g2 = kdn.kdn_diag_bwd_saved(*x, saved, d["dO"], f32(ins["dST"]), f32(ins["dpT"]))
+    torch.cuda.synchronize()
+    ref = oracle.bwd("diag", *[ins[n] for n in ("q", "k", "v", "g", "omega", "r")], ins["S0"],
+                     ins["p0"], ins["dO"], ins["dST"], ins["dpT"])
+    for n in ("dq", "dk", "dv", "dg", "domega", "dr", "dS0", "dp0"):
+        assert torch.equal(g1[n], g2[n]), n
+        check(n, g2[n], ref[n], "bf16")
