@@ -349,7 +349,7 @@ kdn_status_t kdn_iso_bwd(const kdn_desc_t *desc, const void *q, const void *k, c
 
 size_t kdn_saved_bytes(const kdn_desc_t *desc, int variant) {
   Args a;
-  if (fill_sizes(desc, variant, false, &a) != KDN_OK) return 0;
+  if (variant != 0 || fill_sizes(desc, variant, false, &a) != KDN_OK) return 0;
   return fused_saved_bytes(a);
 }
 

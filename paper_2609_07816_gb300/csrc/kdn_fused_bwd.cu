@@ -1,6 +1,6 @@
-// kdn_fused_bwd.cu -- fused chunked backward of the Diagonal KDN for bfloat16
-// activations with d_k = d_v = 128 and 64-token chunks (App. F), on the
-// tcgen05 tensor cores of sm_103a.
+// kdn_fused_bwd.cu -- fused chunked backward of the Diagonal and Isotropic KDN
+// for bfloat16 activations with d_k = d_v = 128 and 64-token chunks (App. F),
+// on the tcgen05 tensor cores of sm_103a.
 //
 // Two launches:
 //  1. the fused forward in its state-saving mode stores, per chunk, the fp16
@@ -24,9 +24,11 @@
 //   dKbar  = A^T dW + dT Kk                             (B10)
 //   dgamma_C = colsum(dK_tail.Kk) + rowsum(dS.S_in)
 // and then, per channel on CUDA cores, the adjoint of the scaling by Gamma and
-// of the gain emission (eq. chunk-gain-emission, eq. kla-box-gain) and of the
-// uncertainty recursion (eq. diag-covariance-prediction, eq. prefix-diag-
-// uncertainty) backwards over the chunk's tokens.
+// of the gain emission (eq. chunk-gain-emission, eq. kla-box-gain /
+// iso-kla-box-gain) and of the uncertainty recursion backwards over the chunk's
+// tokens: per channel for the Diagonal KDN (eq. diag-covariance-prediction,
+// eq. prefix-diag-uncertainty), one scalar per head for the Isotropic KDN
+// (eq. iso-kla-box-cov-update, Prop. 5).
 //
 // Every product runs as a cta_group::1, M = 128 MMA.  Products whose natural
 // row count is 64 read 64 further rows of whatever follows the operand in
@@ -81,7 +83,7 @@ constexpr int O_KKL2 = O_KQL + 16 * KB, O_DWT = O_KQL, O_DAT = O_KQL + 16 * KB;
 constexpr int O_XT = O_KQL + 24 * KB, O_KQH2 = O_SIN, O_QL2 = O_RDO, O_DRTL = O_RH;
 // small arrays
 constexpr int OFF_SM = BUF_END;
-constexpr int SMALL_FLOATS = 64 * 5 + 256 * 2 + 128 * 2 + 16;
+constexpr int SMALL_FLOATS = 64 * 14 + 256 * 2 + 128 * 2 + 16;
 constexpr int OFF_BAR = OFF_SM + SMALL_FLOATS * 4;
 constexpr int SMEM_BYTES = OFF_BAR + 64 + 1024;  // + alignment slack
 static_assert(SMEM_BYTES <= 232448, "shared memory");
@@ -89,6 +91,8 @@ static_assert(O_AQ + 8 * KB <= O_KQH && O_DAT + 16 * KB <= O_RH, "map");
 
 struct BwdParams {
   Args a;
+  int has_g_map;  // per-channel decay tile through TMA
+  int has_w_map;  // per-channel omega tile through TMA (diag)
 };
 
 __device__ __forceinline__ uint64_t kdesc(const unsigned char *p) {
@@ -152,6 +156,7 @@ __device__ __forceinline__ float rs16(const float *v, int lane) {
   return w1 + __shfl_xor_sync(0xffffffffu, w1, 1);
 }
 
+template <int V>
 __global__ void __launch_bounds__(BT, 1)
     k_fused_bwd(const __grid_constant__ CUtensorMap mq, const __grid_constant__ CUtensorMap mk,
                 const __grid_constant__ CUtensorMap mv, const __grid_constant__ CUtensorMap mg,
@@ -172,7 +177,16 @@ __global__ void __launch_bounds__(BT, 1)
   float *s_dp = s_gC + 128;     // [128] uncertainty cotangent carried between chunks
   float *s_si = s_dp + 128;     // [64] 1 / s_t
   float *s_ds = s_si + 64;      // [64] ds_t (cotangent of s_t)
-  float *s_misc = s_ds + 64;    // [0] lambda, [1..] scratch
+  float *s_om = s_ds + 64;      // [64] omega_t (iso)
+  float *s_gs = s_om + 64;      // [64] scalar log-decay g_t (iso, one decay per head)
+  float *s_n2 = s_gs + 64;      // [64] |k_t|^2 (iso)
+  float *s_a = s_n2 + 64;       // [64] a_t = mean alpha^2 (iso)
+  float *s_bh = s_a + 64;       // [64] bhat_t (iso)
+  float *s_bp = s_bh + 64;      // [64] b_{t-1} (iso)
+  float *s_x = s_bp + 64;       // [64] beta_t (iso)
+  float *s_dn2 = s_x + 64;      // [64] cotangent of |k_t|^2 (iso)
+  float *s_da = s_dn2 + 64;     // [64] cotangent of a_t (iso)
+  float *s_misc = s_da + 64;    // [0] lambda, [1..] scratch
   uint64_t *bars = reinterpret_cast<uint64_t *>(sm + OFF_BAR);
   uint64_t *bar_a = bars, *bar_b = bars + 1, *bar_mma = bars + 2;
   uint32_t *s_tbase = reinterpret_cast<uint32_t *>(bars + 4);
@@ -183,6 +197,7 @@ __global__ void __launch_bounds__(BT, 1)
   const int bh = blockIdx.x, b = bh / a.H, h = bh % a.H;
   const int NC = (a.T + CM - 1) / CM;
   const float tau = a.tau, mu = a.mu;
+  const bool pcd = (V == 0) || a.pcd;
 
   if (tid == 0) {
     mbar_init(bar_a, 1);
@@ -192,8 +207,8 @@ __global__ void __launch_bounds__(BT, 1)
     prefetch_tmap(&mq);
     prefetch_tmap(&mk);
     prefetch_tmap(&mv);
-    prefetch_tmap(&mg);
-    prefetch_tmap(&mw);
+    if (P.has_g_map) prefetch_tmap(&mg);
+    if (P.has_w_map) prefetch_tmap(&mw);
     prefetch_tmap(&mdo);
   }
   if (warp == 0) {
@@ -210,12 +225,12 @@ __global__ void __launch_bounds__(BT, 1)
 
   // loads of chunk c: bar_a <- g, omega, S_in (issued when their buffers free up)
   // and k, q (issued last; the one expect_tx covers both groups); bar_b <- dO, v
-  constexpr uint32_t kBytesA = 6 * 16384;
+  const uint32_t kBytesA = 16384u * (4 + (P.has_g_map ? 1 : 0) + (P.has_w_map ? 1 : 0));
   auto issue_a_gws = [&](int c) {
     mbar_expect_tx(bar_a, kBytesA);
     for (int s = 0; s < 2; ++s) {
-      tma_load_4d(rg + s * 8192, &mg, bar_a, 64 * s, h, c * CM, b);
-      tma_load_4d(rw + s * 8192, &mw, bar_a, 64 * s, h, c * CM, b);
+      if (P.has_g_map) tma_load_4d(rg + s * 8192, &mg, bar_a, 64 * s, h, c * CM, b);
+      if (P.has_w_map) tma_load_4d(rw + s * 8192, &mw, bar_a, 64 * s, h, c * CM, b);
     }
     bulk_g2s(sin, a.fSin + ((size_t)bh * NC + c) * 32768, 32768, bar_a);
   };
@@ -299,15 +314,28 @@ __global__ void __launch_bounds__(BT, 1)
     }
     tmem_st_wait();
   }
-  if (tid < D) s_dp[tid] = a.dpT ? lam * a.dpT[(size_t)bh * D + tid] : 0.f;
+  if (tid < D) {
+    const size_t pi = V == 0 ? (size_t)bh * D + tid : (size_t)bh;
+    s_dp[tid] = a.dpT ? lam * a.dpT[pi] : 0.f;
+  }
 
-  // per-token r of the next chunk, prefetched into registers
-  float nr = 1.f;
+  // per-token scalars of the next chunk (r; omega and a scalar decay for the
+  // isotropic KDN), prefetched into registers
+  float nr = 1.f, nom = 0.f, ng = 0.f;
   auto load_r = [&](int c) {
     nr = 1.f;
+    nom = 0.f;
+    ng = 0.f;
     if (tid < CM && c >= 0) {
       const int t = c * CM + tid;
-      if (t < a.T) nr = ld<__nv_bfloat16>(a.r, tok_index(a, b, t, h));
+      if (t < a.T) {
+        const size_t th = tok_index(a, b, t, h);
+        nr = ld<__nv_bfloat16>(a.r, th);
+        if (V == 1) {
+          nom = ld<__nv_bfloat16>(a.omega, th);
+          if (!a.pcd) ng = ld<__nv_bfloat16>(a.g, th);
+        }
+      }
     }
   };
   load_r(NC - 1);
@@ -326,6 +354,18 @@ __global__ void __launch_bounds__(BT, 1)
     tmem_ld16(TPH + lane_base + t0, ph);
     tmem_ld16(TGM + lane_base + t0, ga);
   };
+  // gamma and the gain factor f_t with kappa = f_t k (diag: phat / s_t; iso: beta_t)
+  auto load_gain = [&](float *gf, float *ga) {
+    tmem_ld16(TGM + lane_base + t0, ga);
+    if (V == 0) {
+      tmem_ld16(TPH + lane_base + t0, gf);
+#pragma unroll
+      for (int j = 0; j < 16; ++j) gf[j] *= s_si[t0 + j];
+    } else {
+#pragma unroll
+      for (int j = 0; j < 16; ++j) gf[j] = s_x[t0 + j];
+    }
+  };
   auto raw_k = [&](int t) { return bf(rkq, 16384, t, ci); };
   auto raw_q = [&](int t) { return bf(rkq + 8192, 16384, t, ci); };
 
@@ -335,6 +375,8 @@ __global__ void __launch_bounds__(BT, 1)
     if (tid < CM) {
       s_r[tid] = nr;
       s_ri[tid] = 1.f / nr;
+      s_om[tid] = nom;
+      s_gs[tid] = ng;
     }
     ok = __syncthreads_and(mbar_wait(bar_a, it & 1, kWaitIters));
     if (!ok) break;
@@ -346,6 +388,8 @@ __global__ void __launch_bounds__(BT, 1)
     float dgc = 0.f;  // this thread's part of dgamma_C for channel ci
     {
       float *sQ = reinterpret_cast<float *>(bkqh);  // [4][128][5] quarter summaries
+      float ph16[16], e16[16];
+      if (V == 0) {
       float al[16], w[16], uk[16];
 #pragma unroll
       for (int j = 0; j < 16; ++j) {
@@ -380,7 +424,7 @@ __global__ void __launch_bounds__(BT, 1)
         e *= o[4];
       }
       float p = __fdividef(n, d);
-      float ph16[16], e16[16], y[16];
+      float y[16];
 #pragma unroll
       for (int j = 0; j < 16; ++j) {
         e *= al[j];
@@ -407,6 +451,91 @@ __global__ void __launch_bounds__(BT, 1)
         s_si[tid] = 1.f / st;
       }
       __syncthreads();
+      } else {
+        // per-token |k_t|^2 and a_t = mean_i alpha_ti^2 (or alpha_t^2), one half-warp per token
+        for (int m = 0; m < 2; ++m) {
+          const int t = 32 * m + 2 * warp + (lane >> 4), c8 = lane & 15, sl = c8 >> 3, cc = c8 & 7;
+          float kv[8];
+          unpack_bf8(sm16(rkq, sl * 16384 + chunk_off(t, cc)), kv);
+          float n2 = 0.f, sa = 0.f;
+#pragma unroll
+          for (int j = 0; j < 8; ++j) n2 += kv[j] * kv[j];
+          if (pcd) {
+            float gv[8];
+            unpack_bf8(sm16(rg, sl * 8192 + chunk_off(t, cc)), gv);
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+              const float al = __expf(gv[j]);
+              sa += al * al;
+            }
+          }
+#pragma unroll
+          for (int o = 8; o > 0; o >>= 1) {
+            n2 += __shfl_xor_sync(0xffffffffu, n2, o);
+            sa += __shfl_xor_sync(0xffffffffu, sa, o);
+          }
+          if (c8 == 0) {
+            s_n2[t] = n2;
+            const float al = __expf(s_gs[t]);
+            s_a[t] = pcd ? sa * (1.f / D) : al * al;
+          }
+        }
+        __syncthreads();
+        // cumulative decay of channel ci within this quarter
+        float eq = 1.f;
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+          eq *= __expf(pcd ? bf(rg, 8192, t0 + j, ci) : s_gs[t0 + j]);
+          e16[j] = eq;
+        }
+        sQ[(qq * D + ci) * 5 + 4] = eq;
+        // scalar Moebius product of this quarter (Prop. 5, eq. iso-kla-box-mobius)
+        if (ci == 0) {
+          float m00 = 1.f, m01 = 0.f, m10 = 0.f, m11 = 1.f;
+          for (int j = 0; j < 16; ++j) {
+            const int t = t0 + j;
+            const float at = s_a[t], wt = s_om[t], ut = mu * s_n2[t] * s_ri[t] * (1.f / D);
+            const float n00 = at * m00 + wt * m10, n01 = at * m01 + wt * m11;
+            const float n10 = ut * at * m00 + (1.f + ut * wt) * m10;
+            const float n11 = ut * at * m01 + (1.f + ut * wt) * m11;
+            m00 = n00; m01 = n01; m10 = n10; m11 = n11;
+            if ((j & 7) == 7) {
+              const float sc = __frcp_rn(fmaxf(fmaxf(fabsf(m00), fabsf(m01)), fmaxf(fabsf(m10), fabsf(m11))));
+              m00 *= sc; m01 *= sc; m10 *= sc; m11 *= sc;
+            }
+          }
+          float *mine = sQ + (qq * D) * 5;
+          mine[0] = m00; mine[1] = m01; mine[2] = m10; mine[3] = m11;
+        }
+        __syncthreads();
+        float pre = 1.f;
+        for (int q2 = 0; q2 < qq; ++q2) pre *= sQ[(q2 * D + ci) * 5 + 4];
+#pragma unroll
+        for (int j = 0; j < 16; ++j) e16[j] *= pre;
+        tmem_st16(TGM + lane_base + t0, e16);
+        if (qq == 3) s_gC[ci] = e16[15];
+        if (ci == 0) {
+          float n = a.fpin[((size_t)bh * NC + c) * D], d = 1.f;
+          for (int q2 = 0; q2 < qq; ++q2) {
+            const float *o = sQ + (q2 * D) * 5;
+            const float nn = o[0] * n + o[1] * d, dd = o[2] * n + o[3] * d;
+            const float sc = __frcp_rn(fmaxf(fabsf(nn), fabsf(dd)));
+            n = nn * sc;
+            d = dd * sc;
+          }
+          float bb = __fdividef(n, d);
+          for (int j = 0; j < 16; ++j) {
+            const int t = t0 + j;
+            const float bhat = s_a[t] * bb + s_om[t];  // eq. iso-kla-box-cov-update
+            s_bp[t] = bb;
+            s_bh[t] = bhat;
+            s_x[t] = __fdividef(bhat, s_r[t] + bhat * s_n2[t]);  // beta_t, eq. iso-kla-box-gain
+            bb = __fdividef(bhat, 1.f + mu * s_n2[t] * s_ri[t] * (1.f / D) * bhat);
+          }
+        }
+        tmem_st_wait();
+        __syncthreads();
+      }
       // ---- [3] first operand set, stored transposed ([channel][token] tiles): Kbar, Qbar,
       //          Kk as hi / lo bf16 pairs
       {
@@ -418,8 +547,8 @@ __global__ void __launch_bounds__(BT, 1)
         for (int j = 0; j < 16; ++j) v[j] = tau * e16[j] * raw_q(t0 + j);
         st_row16_split(bkqh + 16384, bkql + 16384, ci, qq, v);
 #pragma unroll
-        for (int j = 0; j < 16; ++j)  // eq. kla-box-gain, divided by gamma
-          v[j] = __fdividef(ph16[j] * raw_k(t0 + j) * s_si[t0 + j], e16[j]);
+        for (int j = 0; j < 16; ++j)  // eq. kla-box-gain / iso-kla-box-gain, divided by gamma
+          v[j] = __fdividef((V == 0 ? ph16[j] * s_si[t0 + j] : s_x[t0 + j]) * raw_k(t0 + j), e16[j]);
         st_row16_split(rw, rg, ci, qq, v);
       }
     }
@@ -538,12 +667,12 @@ __global__ void __launch_bounds__(BT, 1)
       }
     }
     {
-      float ph[16], ga[16];
-      load_ph_ga(ph, ga);
+      float gf[16], ga[16];
+      load_gain(gf, ga);
       const float gC = s_gC[ci];
 #pragma unroll
-      for (int j = 0; j < 16; ++j) ph[j] = gC * __fdividef(ph[j] * raw_k(t0 + j) * s_si[t0 + j], ga[j]);
-      st_row16_h(sm + O_KT, ci, qq, ph);  // K_tail^T [i][s]
+      for (int j = 0; j < 16; ++j) gf[j] = gC * __fdividef(gf[j] * raw_k(t0 + j), ga[j]);
+      st_row16_h(sm + O_KT, ci, qq, gf);  // K_tail^T [i][s]
     }
     tmem_st_wait();
     fence_proxy_async();
@@ -616,19 +745,19 @@ __global__ void __launch_bounds__(BT, 1)
       }
     }
     {
-      float ph[16], ga[16], x[16];
-      load_ph_ga(ph, ga);
+      float gf[16], ga[16], x[16];
+      load_gain(gf, ga);
       tmem_ld16(X0 + lane_base + t0, x);
       const float gC = s_gC[ci];
 #pragma unroll
       for (int j = 0; j < 16; ++j) {
         const int t = t0 + j;
-        dgc += x[j] * __fdividef(ph[j] * raw_k(t) * s_si[t], ga[j]);
+        dgc += x[j] * __fdividef(gf[j] * raw_k(t), ga[j]);
         x[j] *= gC;
-        ph[j] = tau * ga[j] * raw_q(t);
+        gf[j] = tau * ga[j] * raw_q(t);
       }
       tmem_st16(X0 + lane_base + t0, x);
-      st_row16_h(sm + O_QH, ci, qq, ph);  // Qbar^T [i][t]
+      st_row16_h(sm + O_QH, ci, qq, gf);  // Qbar^T [i][t]
     }
     tmem_st_wait();
     fence_proxy_async();
@@ -659,8 +788,8 @@ __global__ void __launch_bounds__(BT, 1)
     // ---- [13] second operand set: [Kbar; Qbar] hi (interleaved), Qbar lo, Kk hi / lo;
     //           B8b: X3 += (dA_qk Kk)^T;  B9a: X0 += (dA_qk^T Qbar)^T
     {
-      float ph[16], ga[16], v[16];
-      load_ph_ga(ph, ga);
+      float gf[16], ga[16], v[16];
+      load_gain(gf, ga);
 #pragma unroll
       for (int j = 0; j < 16; ++j) v[j] = ga[j] * raw_k(t0 + j);
       st_row16_bf(sm + O_KQH2, ci, qq, v);  // Kbar^T hi
@@ -668,7 +797,7 @@ __global__ void __launch_bounds__(BT, 1)
       for (int j = 0; j < 16; ++j) v[j] = tau * ga[j] * raw_q(t0 + j);
       st_row16_split(sm + O_KQH2 + 16384, sm + O_QL2, ci, qq, v);  // Qbar^T hi / lo
 #pragma unroll
-      for (int j = 0; j < 16; ++j) v[j] = __fdividef(ph[j] * raw_k(t0 + j) * s_si[t0 + j], ga[j]);
+      for (int j = 0; j < 16; ++j) v[j] = __fdividef(gf[j] * raw_k(t0 + j), ga[j]);
       st_row16_split(sm + O_KKH2, sm + O_KKL2, ci, qq, v);  // Kk^T hi / lo
     }
     fence_proxy_async();
@@ -800,6 +929,7 @@ __global__ void __launch_bounds__(BT, 1)
     //           Free TMEM columns hold per-(channel, token) intermediates between passes:
     //           X2 <- dphat (gain part), X1 <- dk (memory + gain part), X0 <- alpha^2,
     //           X3 <- 1 / (1 + u phat).
+    if (V == 0)
     {
       float *sdg = reinterpret_cast<float *>(bkql);  // [16][512] dG_t
       float *s_tot = reinterpret_cast<float *>(sm + O_RH);  // [4][128] quarter sums of dG
@@ -945,6 +1075,139 @@ __global__ void __launch_bounds__(BT, 1)
         }
       }
     }
+    else {
+      // Isotropic KDN: kappa_t = beta_t k_t with one uncertainty b per head.
+      float *sdg = reinterpret_cast<float *>(bkql);  // [16][512] dG_t
+      float *s_tot = reinterpret_cast<float *>(sm + O_RH);  // [4][128] quarter sums of dG
+      float *s_dgc = s_tot + 512;                           // [4][128] dgamma_C parts
+      float *s_aff = s_dgc + 512;                           // [4][2] affine summaries
+      float ga[16], k16[16];
+      tmem_ld16(TGM + lane_base + t0, ga);
+#pragma unroll
+      for (int j = 0; j < 16; ++j) k16[j] = raw_k(t0 + j);
+      const size_t ostride = (size_t)a.H * D;
+      const size_t obase = tok_index(a, b, c * CM + t0, h) * D + ci;
+      const int nval = min(16, a.T - (c * CM + t0));
+      const bool obf = a.odt == KDN_BF16;
+      auto out = [&](void *p, int j, float x) {
+        const size_t idx = obase + (size_t)j * ostride;
+        if (obf) static_cast<__nv_bfloat16 *>(p)[idx] = __float2bfloat16_rn(x);
+        else static_cast<float *>(p)[idx] = x;
+      };
+      // pass A: dq, dG, the dbeta_t partial sums and dk from the memory path and kappa
+      {
+        float part[16], tot = 0.f;
+#pragma unroll
+        for (int h8 = 0; h8 < 2; ++h8) {
+          float xq[8], xk[8], xb[8], c2[8];
+          tmem_ld8(X3 + lane_base + t0 + 8 * h8, xq);
+          tmem_ld8(X0 + lane_base + t0 + 8 * h8, xk);
+          tmem_ld8(X2 + lane_base + t0 + 8 * h8, xb);
+#pragma unroll
+          for (int u = 0; u < 8; ++u) {
+            const int j = 8 * h8 + u, t = t0 + j;
+            const float kk = k16[j], qv = raw_q(t), g_ = ga[j], ig = __fdividef(1.f, g_);
+            const float beta = s_x[t], kap = beta * kk;
+            const float dG = xb[u] * g_ * kk - xk[u] * kap * ig + xq[u] * tau * g_ * qv;
+            sdg[j * BT + tid] = dG;
+            tot += dG;
+            const float dkap = xk[u] * ig;
+            part[j] = dkap * kk;
+            c2[u] = xb[u] * g_ + beta * dkap;
+            if (j < nval) out(a.dq, j, tau * g_ * xq[u] * invl);
+          }
+          tmem_st8(X1 + lane_base + t0 + 8 * h8, c2);
+        }
+        s_dgc[qq * D + ci] = dgc;
+        s_tot[qq * D + ci] = tot;
+        const float rsum = rs16(part, lane);
+        if ((lane & 1) == 0) s_red[wq * 64 + t0 + (lane >> 1)] = rsum;
+      }
+      tmem_st_wait();
+      __syncthreads();
+      if (tid < CM) s_ds[tid] = (s_red[tid] + s_red[64 + tid]) + (s_red[128 + tid] + s_red[192 + tid]);
+      __syncthreads();
+      // the scalar recursion: db_{t-1} = a_t (db_t / den_t^2 + dbeta_t r_t / dd_t^2), one
+      // thread per quarter composes its 16 maps, then runs its tokens
+      if (ci == 0) {
+        float A = 1.f, Bv = 0.f;
+        for (int j = 15; j >= 0; --j) {
+          const int t = t0 + j;
+          const float bhat = s_bh[t], u = mu * s_n2[t] * s_ri[t] * (1.f / D);
+          const float rden = __fdividef(1.f, 1.f + u * bhat), dd = s_r[t] + bhat * s_n2[t];
+          const float aj = s_a[t] * rden * rden;
+          Bv = aj * Bv + s_a[t] * __fdividef(s_ds[t] * s_r[t], dd * dd);
+          A = aj * A;
+        }
+        s_aff[qq * 2] = A;
+        s_aff[qq * 2 + 1] = Bv;
+      }
+      __syncthreads();
+      float db = 0.f;
+      if (ci == 0) {
+        db = s_dp[0];
+        for (int q2 = 3; q2 > qq; --q2) db = s_aff[q2 * 2] * db + s_aff[q2 * 2 + 1];
+        for (int j = 15; j >= 0; --j) {
+          const int t = t0 + j, tt = c * CM + t;
+          const float bhat = s_bh[t], beta = s_x[t], n2 = s_n2[t], r = s_r[t], ri = s_ri[t];
+          const float u = mu * n2 * ri * (1.f / D);
+          const float rden = __fdividef(1.f, 1.f + u * bhat), bt = bhat * rden;
+          const float dd = r + bhat * n2, dbeta = s_ds[t];
+          const float dbhat = db * rden * rden + __fdividef(dbeta * r, dd * dd);
+          const float du = -db * bt * bt;
+          s_dn2[t] = -dbeta * beta * beta + du * mu * ri * (1.f / D);
+          s_da[t] = s_bp[t] * dbhat;
+          if (tt < a.T) {
+            const size_t th = tok_index(a, b, tt, h);
+            sto(a.odt, a.domega, th, dbhat * invl);
+            sto(a.odt, a.dr, th, (-__fdividef(dbeta * beta, dd) - du * u * ri) * invl);
+          }
+          db = s_a[t] * dbhat;
+        }
+      }
+      __syncthreads();
+      if (tid == 0) s_dp[0] = db;
+      // per element: dk and dg
+      {
+        const float dgC = (s_dgc[ci] + s_dgc[D + ci]) + (s_dgc[2 * D + ci] + s_dgc[3 * D + ci]);
+        float run = dgC * s_gC[ci];  // dG_63 gains dgamma_C gamma_C; it lies in every suffix
+        for (int q2 = qq + 1; q2 < 4; ++q2) run += s_tot[q2 * D + ci];
+        float ga_prev = 1.f;
+        if (qq > 0) {
+          float g8[8];
+          tmem_ld8(TGM + lane_base + t0 - 8, g8);
+          ga_prev = g8[7];
+        }
+        float c2[16], dgp[16];
+        tmem_ld16(X1 + lane_base + t0, c2);
+#pragma unroll
+        for (int j = 15; j >= 0; --j) {
+          const int t = t0 + j;
+          run += sdg[j * BT + tid];
+          if (j < nval) out(a.dk_, j, (c2[j] + 2.f * k16[j] * s_dn2[t]) * invl);
+          if (pcd) {
+            const float al = __fdividef(ga[j], j > 0 ? ga[j - 1] : ga_prev);
+            if (j < nval) out(a.dg, j, (run + s_da[t] * 2.f * al * al * (1.f / D)) * invl);
+          } else {
+            dgp[j] = run;
+          }
+        }
+        if (!pcd) {  // one decay per head: dg_t = sum_i dG-suffix + 2 alpha_t^2 da_t
+          const float rs2 = rs16(dgp, lane);
+          if ((lane & 1) == 0) s_red2[wq * 64 + t0 + (lane >> 1)] = rs2;
+          __syncthreads();
+          if (tid < CM) {
+            const int tt = c * CM + tid;
+            if (tt < a.T) {
+              const float al = __expf(s_gs[tid]);
+              const float dg = (s_red2[tid] + s_red2[64 + tid]) + (s_red2[128 + tid] + s_red2[192 + tid]) +
+                               2.f * al * al * s_da[tid];
+              sto(a.odt, a.dg, tok_index(a, b, tt, h), dg * invl);
+            }
+          }
+        }
+      }
+    }
     fence_proxy_async();
     tc_fence_before();
     __syncthreads();
@@ -965,7 +1228,10 @@ __global__ void __launch_bounds__(BT, 1)
           dst[u] = make_float4(v[4 * u] * invl, v[4 * u + 1] * invl, v[4 * u + 2] * invl, v[4 * u + 3] * invl);
       }
     }
-    if (a.dp0 && tid < D) a.dp0[(size_t)bh * D + tid] = s_dp[tid] * invl;
+    if (a.dp0 && tid < D) {
+      if (V == 0) a.dp0[(size_t)bh * D + tid] = s_dp[tid] * invl;
+      else if (tid == 0) a.dp0[bh] = s_dp[0] * invl;
+    }
   } else {
     if (tid == 0) atomicExch(a.status, (unsigned)KDN_ERR_TIMEOUT);
     // let copies already in flight land before the CTA's shared memory goes away
@@ -983,9 +1249,7 @@ __global__ void __launch_bounds__(BT, 1)
 
 }  // namespace
 
-bool fused_bwd_supported(const Args &a) {
-  return a.variant == 0 && a.chunk != 32 && fused_fwd_supported(a);
-}
+bool fused_bwd_supported(const Args &a) { return a.chunk != 32 && fused_fwd_supported(a); }
 
 size_t fused_saved_bytes(const Args &a) {
   if (!fused_bwd_supported(a)) return 0;
@@ -996,14 +1260,21 @@ size_t fused_saved_bytes(const Args &a) {
 kdn_status_t launch_fused_bwd_sweep(const Args &a, cudaStream_t s) {
   BwdParams P;
   P.a = a;
+  P.has_g_map = (a.variant == 0 || a.pcd) ? 1 : 0;
+  P.has_w_map = a.variant == 0 ? 1 : 0;
   CUtensorMap mq, mk, mv, mg, mw, mdo;
   if (!make_map(&mq, a.q, a) || !make_map(&mk, a.k, a) || !make_map(&mv, a.v, a) ||
-      !make_map(&mg, a.g, a) || !make_map(&mw, a.omega, a) || !make_map(&mdo, a.dO, a))
+      !make_map(&mdo, a.dO, a))
     return KDN_ERR_CUDA;
-  if (cudaFuncSetAttribute(k_fused_bwd, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES) !=
+  mg = mq;
+  mw = mq;
+  if (P.has_g_map && !make_map(&mg, a.g, a)) return KDN_ERR_CUDA;
+  if (P.has_w_map && !make_map(&mw, a.omega, a)) return KDN_ERR_CUDA;
+  auto kern = a.variant == 0 ? k_fused_bwd<0> : k_fused_bwd<1>;
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES) !=
       cudaSuccess)
     return KDN_ERR_CUDA;
-  k_fused_bwd<<<a.B * a.H, BT, SMEM_BYTES, s>>>(mq, mk, mv, mg, mw, mdo, P);
+  kern<<<a.B * a.H, BT, SMEM_BYTES, s>>>(mq, mk, mv, mg, mw, mdo, P);
   return cudaGetLastError() == cudaSuccess ? KDN_OK : KDN_ERR_CUDA;
 }
 

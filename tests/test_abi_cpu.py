@@ -147,9 +147,10 @@ def test_kernel_launch_query(kdn):
 
 
 def test_fused_path_launches_and_workspace(kdn):
-    """bf16, dk = dv = 128: the fused forward is one launch; the fused Diagonal
-    backward is two (state-saving forward + reverse sweep) and its workspace
-    holds a 32 KB fp16 image of S_in and 128 floats of uncertainty per chunk."""
+    """bf16, dk = dv = 128: the fused forward is one launch; the fused backward
+    (both variants) is two (state-saving forward + reverse sweep) and its
+    workspace holds a 32 KB fp16 image of S_in and 128 floats of uncertainty per
+    chunk."""
     B, T, H = 2, 130, 3
     d = kdn.make_desc(B, T, H, 128, 128, kdn.KDN_BF16)
     assert kdn.kdn_kernel_launches(d, 0, 0) == 1
@@ -157,8 +158,9 @@ def test_fused_path_launches_and_workspace(kdn):
     NC = (T + 63) // 64
     need = 256 + B * H * NC * 32768 + B * H * NC * 128 * 4
     assert kdn.workspace_bytes(d, 0, True) == need
-    # the isotropic backward and the 32-token chunk keep the general kernels
-    assert kdn.kdn_kernel_launches(d, 1, 1) > 2
+    # the isotropic backward is fused too; the 32-token chunk keeps the general kernels
+    assert kdn.kdn_kernel_launches(d, 1, 1) == 2
+    assert kdn.workspace_bytes(d, 1, True) == need
     d32 = kdn.make_desc(B, T, H, 128, 128, kdn.KDN_BF16, chunk=32)
     assert kdn.kdn_kernel_launches(d32, 0, 1) > 2
 

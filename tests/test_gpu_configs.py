@@ -44,6 +44,22 @@ def test_iso_750m_layer_shape(kdn):
     _sampled_fwd_check(kdn, "iso", ins, [(0, 0), (3, 7), (7, 11)])
 
 
+def test_iso_750m_layer_shape_backward(kdn):
+    """Isotropic KDN backward, B=8 H=12 T=2048 d=128, scalar decay, dO ~ N(0,1)."""
+    ins = make_inputs("iso", 8, 2048, 12, 128, 128, dtype="bf16", seed=0,
+                      per_channel_decay=False, with_grad=True)
+    d = to_dev(ins)
+    gr = kdn.kdn_iso_bwd(*[d[n] for n in NAMES], None, None, d["dO"])
+    torch.cuda.synchronize()
+    for b, h in [(0, 0), (7, 11)]:
+        sl = head_slice(ins, b, h)
+        ref = oracle.bwd("iso", *[sl[n] for n in NAMES], None, None, sl["dO"])
+        for n in ("dq", "dk", "dv", "dg", "domega", "dr"):
+            check(f"{n}[{b},{h}]", gr[n][b:b + 1, :, h:h + 1], ref[n], "bf16")
+        check(f"dS0[{b},{h}]", gr["dS0"][b:b + 1, h:h + 1], ref["dS0"], "bf16")
+        check(f"dp0[{b},{h}]", gr["dp0"][b:b + 1, h:h + 1], ref["dp0"], "bf16")
+
+
 def test_diag_1p3b_layer_shape_forward(kdn):
     """Diagonal KDN forward, B=8 H=16 T=4096 d=128."""
     ins = make_inputs("diag", 8, 4096, 16, 128, 128, dtype="bf16", seed=0)

@@ -76,9 +76,12 @@ BWD_CASES = [
     ("diag", True, "bf16", 1, 64, 1, 128, 128),
     ("diag", True, "bf16", 1, 1, 2, 128, 128),
     ("iso", False, "f32", 2, 50, 2, 64, 32),
-    ("iso", False, "bf16", 1, 100, 2, 128, 128),
+    ("iso", False, "bf16", 1, 100, 2, 128, 128),   # fused
+    ("iso", False, "bf16", 2, 200, 3, 128, 128),
     ("iso", True, "f32", 1, 45, 2, 32, 64),
-    ("iso", True, "bf16", 1, 96, 2, 128, 128),
+    ("iso", True, "bf16", 1, 96, 2, 128, 128),     # fused
+    ("iso", True, "bf16", 2, 150, 2, 128, 128),
+    ("iso", True, "bf16", 1, 1, 1, 128, 128),
 ]
 
 
