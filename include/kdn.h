@@ -143,8 +143,9 @@ kdn_status_t kdn_iso_bwd(const kdn_desc_t *desc, const void *q, const void *k,
 
 /* Training pair.  kdn_diag_fwd_save is kdn_diag_fwd that also keeps, in
    `saved`, the context the chunked backward needs (App. F): for every 64-token
-   chunk an fp16 image of the memory S entering it and the float32 uncertainty
-   p entering it.  kdn_diag_bwd_saved is kdn_diag_bwd that starts from that
+   chunk the memory S entering it, its R = U - W S_in, -W, A_qk and
+   A = (I + T)^-1 as fp16 tiles (80 KB) and the float32 uncertainty p entering
+   it.  kdn_diag_bwd_saved is kdn_diag_bwd that starts from that
    context instead of recomputing the forward (same gradients, one kernel).
    Served for the Diagonal KDN with bfloat16 activations, dk = dv = 128 and the
    default chunk; for every other descriptor kdn_saved_bytes() returns 0 and

@@ -187,7 +187,7 @@ kdn_status_t fwd_save_entry(const kdn_desc_t *d, const void *q, const void *k, c
   if (cudaMemsetAsync(a.status, 0, sizeof(unsigned), s) != cudaSuccess) return KDN_ERR_CUDA;
   if ((size_t)a.B * a.H == 0) return KDN_OK;
   if (a.T == 0) return empty_fwd(a, s);
-  const size_t nsv = (size_t)a.B * a.H * ((a.T + 63) / 64) * 32768;
+  const size_t nsv = (size_t)a.B * a.H * ((a.T + 63) / 64) * fused_ctx_record_bytes();
   return launch_fused_fwd(a, s, static_cast<unsigned char *>(saved),
                           reinterpret_cast<float *>(static_cast<char *>(saved) + nsv), true);
 }
@@ -220,7 +220,7 @@ kdn_status_t bwd_saved_entry(const kdn_desc_t *d, const void *q, const void *k, 
   if (cudaMemsetAsync(a.status, 0, sizeof(unsigned), s) != cudaSuccess) return KDN_ERR_CUDA;
   if ((size_t)a.B * a.H == 0) return KDN_OK;
   if (a.T == 0) return empty_bwd(a, s);
-  const size_t nsv = (size_t)a.B * a.H * ((a.T + 63) / 64) * 32768;
+  const size_t nsv = (size_t)a.B * a.H * ((a.T + 63) / 64) * fused_ctx_record_bytes();
   a.fSin = static_cast<unsigned char *>(const_cast<void *>(saved));
   a.fpin = reinterpret_cast<float *>(static_cast<char *>(const_cast<void *>(saved)) + nsv);
   return launch_fused_bwd_sweep(a, s);
@@ -253,7 +253,7 @@ size_t workspace_layout(Args *a, char *base, bool bwd) {
   if (!bwd && use_fused(*a)) return off;
   if (bwd && a->T > 0 && use_fused_bwd(*a)) {
     const size_t NC64 = (a->T + 63) / 64;  // the fused kernels use 64-token chunks
-    a->fSin = reinterpret_cast<unsigned char *>(take(BH * NC64 * 32768 / sizeof(float)));
+    a->fSin = reinterpret_cast<unsigned char *>(take(BH * NC64 * fused_ctx_record_bytes() / sizeof(float)));
     a->fpin = take(BH * NC64 * dk);
     return off;
   }

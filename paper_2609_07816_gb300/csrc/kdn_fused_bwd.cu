@@ -64,30 +64,32 @@ constexpr int KB = 1024;
 // Shared-memory map (bytes from the 1024-aligned base).  Regions are reused
 // across the stages of a chunk; the comments give the sequence of tenants.
 constexpr int O_RKQ = 0;         // raw k | q, interleaved per 64-channel slab (whole chunk)
-constexpr int O_SIN = 32 * KB;   // S_in fp16 [i][j]  -> [Kbar; Qbar] hi (second operand set)
+constexpr int O_SIN = 32 * KB;   // S_in fp16 [i][j] (context)  -> Kbar^T hi | Qbar^T hi (second set)
 constexpr int O_RV = 64 * KB;    // raw v  -> v fp16
-constexpr int O_RDO = 80 * KB;   // raw dO -> lambda dO fp16 -> Qbar lo (second set)
-constexpr int O_RG = 96 * KB;    // raw g  -> Kk lo (first set) -> T fp32 -> A bf16 | A fp16
-constexpr int O_RW = 112 * KB;   // raw omega -> Kk hi (first set) -> (T) | A_qk fp16 -> dT bf16
-constexpr int O_KQH = 128 * KB;  // [Kbar; Qbar] hi (first) -> -W fp16 | K_tail -> Kk hi | dR^T
-constexpr int O_KQL = 160 * KB;  // [Kbar; Qbar] lo (first) -> A fp32 -> dS fp16 -> dA_qk^T | Qbar
-                                 //   fp16 -> dW^T | Kk lo -> dA^T | X
-constexpr int O_RH = 192 * KB;   // R fp16 (16 KB; the next 8 KB are read as padding rows)
-                                 //   -> lo part of dR^T fp16 -> per-channel scratch
+constexpr int O_RDO = 80 * KB;   // raw dO -> lambda dO fp16 -> Qbar^T lo
+constexpr int O_AH = 96 * KB;    // A fp16 [t][s] (context)
+constexpr int O_SQ = 104 * KB;   // gain quarter summaries (10 KB)  -> A bf16 [t][s]
+constexpr int O_DT = 112 * KB;   // dT bf16  -> per-channel scratch of the final stage
+constexpr int O_AQ = 120 * KB;   // A_qk fp16 [t][s] (context)
+constexpr int O_WN = 128 * KB;   // -W fp16 [t][i] (context)  -> Kk^T hi
+constexpr int O_KT = 144 * KB;   // K_tail^T fp16  -> dR^T fp16
+constexpr int O_G = 160 * KB;    // raw g | raw omega  -> dS fp16  -> dA_qk^T | Qbar^T fp16
+                                 //   -> dW^T | Kk^T lo -> dA^T | X  -> dG of the final stage
+constexpr int O_RH = 192 * KB;   // R fp16 (context; the next 8 KB are read as padding rows)
+                                 //   -> lo part of dR^T fp16
 constexpr int BUF_END = 216 * KB;
 // derived tenants
-constexpr int O_AB = O_RG, O_AH = O_RG + 8 * KB, O_AQ = O_RW + 8 * KB, O_DT = O_RW;
-constexpr int O_WN = O_KQH, O_KT = O_KQH + 16 * KB, O_DRT = O_KQH + 16 * KB;
-constexpr int O_KKH2 = O_KQH, O_DSH = O_KQL, O_DAQ = O_KQL, O_QH = O_KQL + 16 * KB;
-constexpr int O_KKL2 = O_KQL + 16 * KB, O_DWT = O_KQL, O_DAT = O_KQL + 16 * KB;
-constexpr int O_XT = O_KQL + 24 * KB, O_KQH2 = O_SIN, O_QL2 = O_RDO, O_DRTL = O_RH;
+constexpr int O_W = O_G + 16 * KB, O_AB = O_SQ, O_DRT = O_KT, O_KKH2 = O_WN;
+constexpr int O_DSH = O_G, O_DAQ = O_G, O_QH = O_G + 16 * KB, O_KKL2 = O_G + 16 * KB;
+constexpr int O_DWT = O_G, O_DAT = O_G + 16 * KB, O_XT = O_G + 24 * KB, O_KQH2 = O_SIN;
+constexpr int O_QL2 = O_RDO, O_DRTL = O_RH;
 // small arrays
 constexpr int OFF_SM = BUF_END;
 constexpr int SMALL_FLOATS = 64 * 14 + 256 * 2 + 128 * 2 + 16;
 constexpr int OFF_BAR = OFF_SM + SMALL_FLOATS * 4;
 constexpr int SMEM_BYTES = OFF_BAR + 64 + 1024;  // + alignment slack
 static_assert(SMEM_BYTES <= 232448, "shared memory");
-static_assert(O_AQ + 8 * KB <= O_KQH && O_DAT + 16 * KB <= O_RH, "map");
+static_assert(O_AQ + 8 * KB <= O_WN && O_XT + 8 * KB <= O_RH, "map");
 
 struct BwdParams {
   Args a;
@@ -167,7 +169,7 @@ __global__ void __launch_bounds__(BT, 1)
   unsigned char *sm =
       reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(smraw) + 1023) & ~uintptr_t(1023));
   unsigned char *rkq = sm + O_RKQ, *sin = sm + O_SIN, *rv = sm + O_RV, *rdo = sm + O_RDO;
-  unsigned char *rg = sm + O_RG, *rw = sm + O_RW, *bkqh = sm + O_KQH, *bkql = sm + O_KQL;
+  unsigned char *rg = sm + O_G, *rw = sm + O_W;
   float *s_r = reinterpret_cast<float *>(sm + OFF_SM);  // [64] r_t
   float *s_ri = s_r + 64;     // [64] 1 / r_t
   float *s_s = s_ri + 64;     // [64] s_t = r_t + sum_i phat k^2
@@ -223,21 +225,25 @@ __global__ void __launch_bounds__(BT, 1)
   const uint32_t X0 = tb + 256, X1 = tb + 320, X2 = tb + 384, X3 = tb + 448;
   const uint32_t lane_base = (uint32_t)(32 * wq) << 16;
 
-  // loads of chunk c: bar_a <- g, omega, S_in (issued when their buffers free up)
-  // and k, q (issued last; the one expect_tx covers both groups); bar_b <- dO, v
-  const uint32_t kBytesA = 16384u * (4 + (P.has_g_map ? 1 : 0) + (P.has_w_map ? 1 : 0));
-  auto issue_a_gws = [&](int c) {
+  // loads of chunk c on bar_a: the context record (S_in, R, -W, A_qk, A; issued as
+  // soon as their buffers free up) and the raw k, q, g, omega tiles (issued once the
+  // previous chunk is done; the one expect_tx covers both groups); bar_b <- dO, v
+  const uint32_t kBytesA = 81920u + 16384u * (2 + (P.has_g_map ? 1 : 0) + (P.has_w_map ? 1 : 0));
+  auto issue_a_ctx = [&](int c) {
+    const unsigned char *rec = a.fSin + ((size_t)bh * NC + c) * kCtxBytes;
     mbar_expect_tx(bar_a, kBytesA);
-    for (int s = 0; s < 2; ++s) {
-      if (P.has_g_map) tma_load_4d(rg + s * 8192, &mg, bar_a, 64 * s, h, c * CM, b);
-      if (P.has_w_map) tma_load_4d(rw + s * 8192, &mw, bar_a, 64 * s, h, c * CM, b);
-    }
-    bulk_g2s(sin, a.fSin + ((size_t)bh * NC + c) * 32768, 32768, bar_a);
+    bulk_g2s(sin, rec + kCtxS, 32768, bar_a);
+    bulk_g2s(sm + O_RH, rec + kCtxR, 16384, bar_a);
+    bulk_g2s(sm + O_WN, rec + kCtxW, 16384, bar_a);
+    bulk_g2s(sm + O_AQ, rec + kCtxAqk, 8192, bar_a);
+    bulk_g2s(sm + O_AH, rec + kCtxA, 8192, bar_a);
   };
-  auto issue_a_kq = [&](int c) {
+  auto issue_a_raw = [&](int c) {
     for (int s = 0; s < 2; ++s) {
       tma_load_4d(rkq + s * 16384, &mk, bar_a, 64 * s, h, c * CM, b);
       tma_load_4d(rkq + s * 16384 + 8192, &mq, bar_a, 64 * s, h, c * CM, b);
+      if (P.has_g_map) tma_load_4d(rg + s * 8192, &mg, bar_a, 64 * s, h, c * CM, b);
+      if (P.has_w_map) tma_load_4d(rw + s * 8192, &mw, bar_a, 64 * s, h, c * CM, b);
     }
   };
   auto issue_b_do = [&](int c) {
@@ -248,8 +254,8 @@ __global__ void __launch_bounds__(BT, 1)
     for (int s = 0; s < 2; ++s) tma_load_4d(rv + s * 8192, &mv, bar_b, 64 * s, h, c * CM, b);
   };
   if (tid == 0) {
-    issue_a_gws(NC - 1);
-    issue_a_kq(NC - 1);
+    issue_a_ctx(NC - 1);
+    issue_a_raw(NC - 1);
     issue_b_do(NC - 1);
     issue_b_v(NC - 1);
   }
@@ -342,10 +348,11 @@ __global__ void __launch_bounds__(BT, 1)
 
   uint32_t mma_phase = 0;
   bool ok = true;
-  const uint32_t id_T = idesc_bf16(128, 64, 1, 1);
-  const uint32_t id_W = idesc_bf16(128, 128, 0, 0), id_U = idesc_f16(128, 128, 0, 1);
+  // One thread polls the MMA-completion barrier; the CTA barrier then orders every
+  // thread's TMEM reads after it (each caller issues tcgen05.fence::after_thread_sync).
   auto mma_wait = [&]() -> bool {
-    bool r = mbar_wait(bar_mma, mma_phase & 1, kWaitIters);
+    bool r = true;
+    if (tid == 0) r = mbar_wait(bar_mma, mma_phase & 1, kWaitIters);
     ++mma_phase;
     return __syncthreads_and(r);
   };
@@ -387,7 +394,7 @@ __global__ void __launch_bounds__(BT, 1)
     //          into each quarter's entry value); phat, gamma -> TMEM (lane = channel)
     float dgc = 0.f;  // this thread's part of dgamma_C for channel ci
     {
-      float *sQ = reinterpret_cast<float *>(bkqh);  // [4][128][5] quarter summaries
+      float *sQ = reinterpret_cast<float *>(sm + O_SQ);  // [4][128][5] quarter summaries
       float ph16[16], e16[16];
       if (V == 0) {
       float al[16], w[16], uk[16];
@@ -536,115 +543,15 @@ __global__ void __launch_bounds__(BT, 1)
         tmem_st_wait();
         __syncthreads();
       }
-      // ---- [3] first operand set, stored transposed ([channel][token] tiles): Kbar, Qbar,
-      //          Kk as hi / lo bf16 pairs
-      {
-        float v[16];
-#pragma unroll
-        for (int j = 0; j < 16; ++j) v[j] = e16[j] * raw_k(t0 + j);
-        st_row16_split(bkqh, bkql, ci, qq, v);
-#pragma unroll
-        for (int j = 0; j < 16; ++j) v[j] = tau * e16[j] * raw_q(t0 + j);
-        st_row16_split(bkqh + 16384, bkql + 16384, ci, qq, v);
-#pragma unroll
-        for (int j = 0; j < 16; ++j)  // eq. kla-box-gain / iso-kla-box-gain, divided by gamma
-          v[j] = __fdividef((V == 0 ? ph16[j] * s_si[t0 + j] : s_x[t0 + j]) * raw_k(t0 + j), e16[j]);
-        st_row16_split(rw, rg, ci, qq, v);
-      }
     }
-    fence_proxy_async();
-    tc_fence_before();
-    __syncthreads();
-    // ---- [4] MMA-T: X0 = [Kbar; Qbar] Kk^T  (hi.hi + lo.hi + hi.lo; both operands MN-major)
-    if (tid == 0) {
-      tc_fence_after();
-      for (int kk = 0; kk < 8; ++kk) {
-        const uint64_t ah = mdesc(bkqh + kk * 2048, 16384), bhd = mdesc(rw + kk * 2048, 8192);
-        umma_bf16(X0, ah, bhd, id_T, kk > 0);
-        umma_bf16(X0, mdesc(bkql + kk * 2048, 16384), bhd, id_T, 1);
-        umma_bf16(X0, ah, mdesc(rg + kk * 2048, 8192), id_T, 1);
-      }
-      umma_commit(bar_mma);
-    }
-    if (!(ok = mma_wait())) break;
-    tc_fence_after();
-    // ---- [5] T -> fp32 (strict lower), A_qk -> fp16 [t][s] (lower); A = (I + T)^-1
-    float *sT = reinterpret_cast<float *>(rg), *sA = reinterpret_cast<float *>(bkql);
-    float *sX = sA + 64 * LT;
+    // ---- [3] operands of the chunk adjoint from the context and the gains:
+    //          A bf16 (from the saved fp16 A); dS -> fp16 [i][j] and dS <- gamma_C dS in
+    //          TMEM; K_tail^T [i][s]; lambda dO and v to fp16 in place
     {
-      const int s0 = 16 * wg;
-      float v[16];
-      tmem_ld16(X0 + lane_base + s0, v);
-      if (wq < 2) {
-        const int r = 32 * wq + lane;
-#pragma unroll
-        for (int u = 0; u < 16; ++u)
-          if (s0 + u >= r) v[u] = 0.f;
-#pragma unroll
-        for (int u = 0; u < 4; ++u)
-          *reinterpret_cast<float4 *>(sT + r * LT + s0 + 4 * u) =
-              make_float4(v[4 * u], v[4 * u + 1], v[4 * u + 2], v[4 * u + 3]);
-      } else {
-        const int r = 32 * wq + lane - 64;
-#pragma unroll
-        for (int u = 0; u < 16; ++u)
-          if (s0 + u > r) v[u] = 0.f;
-        sm16(sm + O_AQ, chunk_off(r, s0 >> 3)) = pack_h8(v);
-        sm16(sm + O_AQ, chunk_off(r, (s0 >> 3) + 1)) = pack_h8(v + 8);
-      }
-    }
-    __syncthreads();
-    tri_inverse64(sT, sA, sX);
-    // A -> bf16 and fp16 [t][s] tiles (zero above the diagonal)
-    for (int e = tid; e < 64 * 8; e += BT) {
-      const int r = e >> 3, cc = e & 7;
+      const uint4 ah = sm16(sm + O_AH, tid * 16);  // 512 chunks of 8: the whole 8 KB tile
       float v[8];
-#pragma unroll
-      for (int j = 0; j < 8; ++j) v[j] = (8 * cc + j <= r) ? sA[r * LT + 8 * cc + j] : 0.f;
-      sm16(sm + O_AB, chunk_off(r, cc)) = pack_bf8(v);
-      sm16(sm + O_AH, chunk_off(r, cc)) = pack_h8(v);
-    }
-    ok = __syncthreads_and(mbar_wait(bar_b, it & 1, kWaitIters));
-    if (!ok) break;
-    // lambda dO and v -> fp16 in place
-    for (int e = tid; e < 64 * 16; e += BT) {
-      const int row = e >> 4, c16 = e & 15;
-      const uint32_t off = (c16 >> 3) * 8192 + chunk_off(row, c16 & 7);
-      float v[8];
-      unpack_bf8(sm16(rdo, off), v);
-#pragma unroll
-      for (int j = 0; j < 8; ++j) v[j] *= lam;
-      sm16(rdo, off) = pack_h8(v);
-      unpack_bf8(sm16(rv, off), v);
-      sm16(rv, off) = pack_h8(v);
-    }
-    fence_proxy_async();
-    tc_fence_before();
-    __syncthreads();
-    // ---- [6] MMA-W (bf16): X2 = A Kbar;  MMA-U (fp16): X0 = A V
-    if (tid == 0) {
-      tc_fence_after();
-      for (int kk = 0; kk < 4; ++kk) {
-        umma_bf16(X2, kdesc(sm + O_AB + kk * 32), kdesc(bkqh + kk * 32), id_W, kk > 0);
-        umma_bf16(X0, kdesc(sm + O_AH + kk * 32), mdesc(rv + kk * 2048, 8192), id_U, kk > 0);
-      }
-      umma_commit(bar_mma);
-    }
-    if (!(ok = mma_wait())) break;
-    tc_fence_after();
-    // ---- [7] fp16 operands: -W [t][i]; dS -> fp16 [i][j] and dS <- gamma_C dS in TMEM;
-    //          K_tail [s][i]
-    if (wq < 2) {
-      const int r = 32 * wq + lane;
-      for (int c0 = 0; c0 < 32; c0 += 16) {
-        float v[16];
-        const int j0 = 32 * wg + c0, sl = j0 >> 6, cc0 = (j0 & 63) >> 3;
-        tmem_ld16(X2 + lane_base + j0, v);
-#pragma unroll
-        for (int u = 0; u < 16; ++u) v[u] = -v[u];
-        sm16(sm + O_WN, sl * 8192 + chunk_off(r, cc0)) = pack_h8(v);
-        sm16(sm + O_WN, sl * 8192 + chunk_off(r, cc0 + 1)) = pack_h8(v + 8);
-      }
+      unpack_h8(ah, v);
+      sm16(sm + O_AB, tid * 16) = pack_bf8(v);
     }
     {
       const int i = 32 * wq + lane;
@@ -674,32 +581,20 @@ __global__ void __launch_bounds__(BT, 1)
       for (int j = 0; j < 16; ++j) gf[j] = gC * __fdividef(gf[j] * raw_k(t0 + j), ga[j]);
       st_row16_h(sm + O_KT, ci, qq, gf);  // K_tail^T [i][s]
     }
+    ok = __syncthreads_and(mbar_wait(bar_b, it & 1, kWaitIters));
+    if (!ok) break;
+    for (int e = tid; e < 64 * 16; e += BT) {
+      const int row = e >> 4, c16 = e & 15;
+      const uint32_t off = (c16 >> 3) * 8192 + chunk_off(row, c16 & 7);
+      float v[8];
+      unpack_bf8(sm16(rdo, off), v);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) v[j] *= lam;
+      sm16(rdo, off) = pack_h8(v);
+      unpack_bf8(sm16(rv, off), v);
+      sm16(rv, off) = pack_h8(v);
+    }
     tmem_st_wait();
-    fence_proxy_async();
-    tc_fence_before();
-    __syncthreads();
-    // ---- [8] MMA-S1 (fp16): X0 += -W S_in  -> rows 0..63 hold R
-    if (tid == 0) {
-      tc_fence_after();
-      const uint32_t id = idesc_f16(128, 128, 0, 1);
-      for (int kk = 0; kk < 8; ++kk)
-        umma_bf16(X0, kdesc(sm + O_WN + (kk >> 2) * 8192 + (kk & 3) * 32),
-                  mdesc(sin + kk * 2048, 16384), id, 1);
-      umma_commit(bar_mma);
-    }
-    if (!(ok = mma_wait())) break;
-    tc_fence_after();
-    // ---- [9] R -> fp16 [s][j]
-    if (wq < 2) {
-      const int t = 32 * wq + lane;
-      for (int c0 = 0; c0 < 32; c0 += 16) {
-        float v[16];
-        const int j0 = 32 * wg + c0, sl = j0 >> 6, cc0 = (j0 & 63) >> 3;
-        tmem_ld16(X0 + lane_base + j0, v);
-        sm16(sm + O_RH, sl * 8192 + chunk_off(t, cc0)) = pack_h8(v);
-        sm16(sm + O_RH, sl * 8192 + chunk_off(t, cc0 + 1)) = pack_h8(v + 8);
-      }
-    }
     fence_proxy_async();
     tc_fence_before();
     __syncthreads();
@@ -923,7 +818,7 @@ __global__ void __launch_bounds__(BT, 1)
     }
     if (!(ok = mma_wait())) break;
     tc_fence_after();
-    if (tid == 0 && c > 0) issue_a_gws(c - 1);  // g, omega, S_in buffers are free
+    if (tid == 0 && c > 0) issue_a_ctx(c - 1);  // the context buffers are free
     // ---- [18] per channel (lane ci, tokens t0..t0+15): back through Gamma and the
     //           gain emission, then the uncertainty recursion backwards in time.
     //           Free TMEM columns hold per-(channel, token) intermediates between passes:
@@ -931,8 +826,8 @@ __global__ void __launch_bounds__(BT, 1)
     //           X3 <- 1 / (1 + u phat).
     if (V == 0)
     {
-      float *sdg = reinterpret_cast<float *>(bkql);  // [16][512] dG_t
-      float *s_tot = reinterpret_cast<float *>(sm + O_RH);  // [4][128] quarter sums of dG
+      float *sdg = reinterpret_cast<float *>(sm + O_G);  // [16][512] dG_t
+      float *s_tot = reinterpret_cast<float *>(sm + O_DT);  // [4][128] quarter sums of dG
       float *s_dgc = s_tot + 512;                           // [4][128] dgamma_C parts
       float *s_aff = s_dgc + 512;                           // [4][128][2] affine summaries
       float ph[16], ga[16], k16[16];
@@ -1077,8 +972,8 @@ __global__ void __launch_bounds__(BT, 1)
     }
     else {
       // Isotropic KDN: kappa_t = beta_t k_t with one uncertainty b per head.
-      float *sdg = reinterpret_cast<float *>(bkql);  // [16][512] dG_t
-      float *s_tot = reinterpret_cast<float *>(sm + O_RH);  // [4][128] quarter sums of dG
+      float *sdg = reinterpret_cast<float *>(sm + O_G);  // [16][512] dG_t
+      float *s_tot = reinterpret_cast<float *>(sm + O_DT);  // [4][128] quarter sums of dG
       float *s_dgc = s_tot + 512;                           // [4][128] dgamma_C parts
       float *s_aff = s_dgc + 512;                           // [4][2] affine summaries
       float ga[16], k16[16];
@@ -1212,7 +1107,7 @@ __global__ void __launch_bounds__(BT, 1)
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    if (tid == 0 && c > 0) issue_a_kq(c - 1);  // raw k, q have been read
+    if (tid == 0 && c > 0) issue_a_raw(c - 1);  // raw k, q, g, omega buffers are free
   }
 
   if (ok) {
@@ -1254,8 +1149,10 @@ bool fused_bwd_supported(const Args &a) { return a.chunk != 32 && fused_fwd_supp
 size_t fused_saved_bytes(const Args &a) {
   if (!fused_bwd_supported(a)) return 0;
   const size_t nc = (a.T + CM - 1) / CM;
-  return (size_t)a.B * a.H * nc * (32768 + D * sizeof(float));
+  return (size_t)a.B * a.H * nc * (kCtxBytes + D * sizeof(float));
 }
+
+size_t fused_ctx_record_bytes() { return kCtxBytes; }
 
 kdn_status_t launch_fused_bwd_sweep(const Args &a, cudaStream_t s) {
   BwdParams P;

@@ -72,6 +72,17 @@ __device__ __forceinline__ void unpack_h8(uint4 u, float *v) {
   }
 }
 
+// Per-chunk record of the backward context written by the fused forward in
+// its saving mode (byte offsets; every tile is the 128-byte-swizzled 16-bit
+// image the kernels use in shared memory):
+//   S_in  fp16 [128 i][128 j] as two 64-column slabs          32 KB
+//   R     fp16 [64 s][128 j] as two slabs                      16 KB
+//   -W    fp16 [64 t][128 i] as two slabs                      16 KB
+//   A_qk  fp16 [64 t][64 s] (lower triangle)                    8 KB
+//   A     fp16 [64 t][64 s] (lower triangle)                    8 KB
+constexpr int kCtxS = 0, kCtxR = 32768, kCtxW = 49152, kCtxAqk = 65536, kCtxA = 73728;
+constexpr int kCtxBytes = 81920;
+
 // Row stride (floats) of the fp32 T and A tiles: 16-byte rows, conflict-free.
 constexpr int LT = 68;
 

@@ -72,7 +72,7 @@ struct FusedParams {
   int has_g_map;  // per-channel decay tile through TMA
   int has_w_map;  // per-channel omega tile through TMA (diag)
   int write_o;    // 0: the outputs o are not written (state-saving pass of the backward)
-  unsigned char *save_S;  // optional [BH][NC] 32 KB images of S_in (fp16 tile of MMA-S1)
+  unsigned char *save_S;  // optional [BH][NC] context records of the backward (kCtxBytes each)
   float *save_p;          // optional [BH][NC][128] uncertainty carry entering each chunk
 };
 
@@ -204,11 +204,14 @@ __global__ void __launch_bounds__(FT, 1)
   uint32_t mma_phase = 0;
   bool ok = true;
   const uint32_t id_T = idesc_bf16(128, 64, 0, 0);
-  const uint32_t id_WU = idesc_bf16(128, 128, 0, 1);
+  const uint32_t id_WU = idesc_bf16(128, 128, 0, 1), id_U = idesc_f16(128, 128, 0, 1);
   const uint32_t ih_S1 = idesc_f16(128, 128, 0, 1);
   const uint32_t ih_S2 = idesc_f16(128, 128, 1, 1);
+  // One thread polls the MMA-completion barrier; the CTA barrier then orders every
+  // thread's TMEM reads after it (each caller issues tcgen05.fence::after_thread_sync).
   auto mma_wait = [&]() -> bool {
-    bool r = mbar_wait(bar_mma, mma_phase & 1, kWaitIters);
+    bool r = true;
+    if (tid == 0) r = mbar_wait(bar_mma, mma_phase & 1, kWaitIters);
     ++mma_phase;
     return __syncthreads_and(r);
   };
@@ -224,6 +227,7 @@ __global__ void __launch_bounds__(FT, 1)
     if (tid == 0) bulk_wait_read();  // O staging and the saved S image have been read
     if (P.save_p && tid < D)
       P.save_p[((size_t)bh * NC + c) * D + tid] = (V == 0) ? s_p[tid] : s_b[0];
+    unsigned char *ctx = P.save_S ? P.save_S + ((size_t)bh * NC + c) * kCtxBytes : nullptr;
     ok = __syncthreads_and(mbar_wait(bar_raw, c & 1, kWaitIters));
     if (!ok) break;
     load_scalars(c + 1);
@@ -445,6 +449,7 @@ __global__ void __launch_bounds__(FT, 1)
     //   diagonal blocks D_I = (I + T_II)^-1 by column substitution (rows across a half-warp),
     //   then A_IJ = -D_I sum_{K=J}^{I-1} T_IK A_KJ level by level (I - J = 1, 2, 3)
     float *sT = fs, *sA = fs + 64 * LT, *sX = fs + 2 * 64 * LT;
+    unsigned char *af = reinterpret_cast<unsigned char *>(fs);  // [A; 0] fp16, 16 KB over T
     if (wq < 2) {
       const int r = 32 * wq + lane, s0 = 16 * wg;
       float v[16];
@@ -468,25 +473,37 @@ __global__ void __launch_bounds__(FT, 1)
         v[j] = (r < 64 && sidx <= r) ? sA[r * LT + sidx] : 0.f;
       }
       sm16(a2, chunk_off(r, cc)) = pack_bf8(v);
+      sm16(af, chunk_off(r, cc)) = pack_h8(v);  // [A; 0] fp16 for MMA-U (over the dead T tile)
     }
-    fence_proxy_async();
     ok = __syncthreads_and(mbar_wait(bar_v, c & 1, kWaitIters));
     if (!ok) break;
+    for (int e = tid; e < 64 * 16; e += FT) {  // V -> fp16 in place
+      const uint32_t off = (e >> 9) * 8192 + chunk_off((e >> 3) & 63, e & 7);  // slab, row, chunk
+      float v[8];
+      unpack_bf8(sm16(vr, off), v);
+      sm16(vr, off) = pack_h8(v);
+    }
+    fence_proxy_async();
     tc_fence_before();
     __syncthreads();
-    // ---- [6] MMA-W, MMA-U (bf16; Kbar enters as its hi part)
+    // ---- [6] MMA-W (bf16; Kbar enters as its hi part), MMA-U (fp16)
     if (tid == 0) {
       tc_fence_after();
-      const uint32_t A2 = smem_u32(a2), KQ = smem_u32(kq), VR = smem_u32(vr);
+      const uint32_t A2 = smem_u32(a2), AF = smem_u32(af), KQ = smem_u32(kq), VR = smem_u32(vr);
       for (int kk = 0; kk < 4; ++kk) {
-        const uint64_t ad = sw128_desc(A2 + kk * 32, 16, 1024);
-        umma_bf16(TW, ad, sw128_desc(KQ + kk * 2048, 16384, 1024), id_WU, kk > 0);
-        umma_bf16(TU, ad, sw128_desc(VR + kk * 2048, 8192, 1024), id_WU, kk > 0);
+        umma_bf16(TW, sw128_desc(A2 + kk * 32, 16, 1024), sw128_desc(KQ + kk * 2048, 16384, 1024), id_WU,
+                  kk > 0);
+        umma_bf16(TU, sw128_desc(AF + kk * 32, 16, 1024), sw128_desc(VR + kk * 2048, 8192, 1024), id_U,
+                  kk > 0);
       }
       umma_commit(bar_mma);
     }
     if (!(ok = mma_wait())) break;
     tc_fence_after();
+    if (tid == 0 && P.save_S) {  // A fp16 [t][s] into the backward context
+      bulk_s2g(ctx + kCtxA, af, 8192);
+      bulk_commit();
+    }
     // ---- [7] fp16 operands of the state products:
     //   a1l rows 0..63 <- -W, rows 64..127 <- Qbar;  a2 <- [0; A_qk];
     //   b3 <- S_in (and diag(gamma_C) S_in back to TMEM);  b1l <- K_tail
@@ -546,8 +563,11 @@ __global__ void __launch_bounds__(FT, 1)
     tc_fence_before();
     __syncthreads();
     if (tid == 0 && c + 1 < NC) issue_raw_kqw(c + 1);  // raw k, q, omega buffers are free
-    if (tid == 0 && P.save_S) {
-      bulk_s2g(P.save_S + ((size_t)bh * NC + c) * 32768, b3, 32768);
+    if (tid == 0 && P.save_S) {  // S_in, -W and A_qk into the backward context
+      bulk_s2g(ctx + kCtxS, b3, 32768);
+      bulk_s2g(ctx + kCtxW, a1l, 8192);
+      bulk_s2g(ctx + kCtxW + 8192, a1l + 16384, 8192);
+      bulk_s2g(ctx + kCtxAqk, a2 + 8192, 8192);
       bulk_commit();
     }
     // ---- [8] MMA-S1 (fp16): [U; 0] += [-W; Qbar] S_in
@@ -575,6 +595,10 @@ __global__ void __launch_bounds__(FT, 1)
     fence_proxy_async();
     tc_fence_before();
     __syncthreads();
+    if (tid == 0 && P.save_S) {  // R into the backward context
+      bulk_s2g(ctx + kCtxR, vr, 16384);
+      bulk_commit();
+    }
     // ---- [10] MMA-O and MMA-S2 (fp16)
     if (tid == 0) {
       tc_fence_after();
@@ -586,6 +610,7 @@ __global__ void __launch_bounds__(FT, 1)
       }
       umma_commit(bar_mma);
     }
+    if (tid == 0 && P.save_S) bulk_wait_read();  // the saved R and A have left vr and fs
     if (!(ok = mma_wait())) break;
     tc_fence_after();
     if (tid == 0 && c + 1 < NC) issue_v(c + 1);  // R in vr has been consumed

@@ -84,7 +84,7 @@ struct Args {
   float *drpart;  // [BH][Tp]
   float *drw;     // [BH][Tp][4]
   float *isoadj;  // [BH][Tp][2]
-  unsigned char *fSin;  // fused backward: [BH][NC] 32 KB fp16 images of S_in
+  unsigned char *fSin;  // fused backward: [BH][NC] context records (S_in, R, -W, A_qk, A)
   float *fpin;          // fused backward: [BH][NC][dk] uncertainty entering each chunk
 };
 
@@ -109,8 +109,11 @@ kdn_status_t launch_fused_fwd(const Args &a, cudaStream_t s, unsigned char *save
 bool fused_bwd_supported(const Args &a);
 kdn_status_t launch_fused_bwd(const Args &a, cudaStream_t s);
 kdn_status_t launch_fused_bwd_sweep(const Args &a, cudaStream_t s);
-// Bytes of the saved context for the fused backward (0 if not served).
+// Bytes of the saved context for the fused backward (0 if not served): per
+// (batch, head) and 64-token chunk one record of fused_ctx_record_bytes(), then
+// per chunk the 128 float32 uncertainties entering it.
 size_t fused_saved_bytes(const Args &a);
+size_t fused_ctx_record_bytes();
 
 // Launchers (each returns KDN_OK or KDN_ERR_CUDA).
 kdn_status_t launch_chunked_fwd(const Args &a, cudaStream_t s, bool save_states);
