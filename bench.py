@@ -146,39 +146,50 @@ class ClockSampler:
 # ---------------------------------------------------------------------------
 # distributed plumbing (one process per GPU; replicas, no data exchange)
 
-def dist_setup(n):
+def dist_setup(n, backend="nccl"):
+    """One process per GPU (replicas): rank / local rank / world from the launcher's env."""
     import torch
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
     if world != n:
         raise SystemExit(f"--gpus {n} but WORLD_SIZE={world}")
+    cuda = backend == "nccl"
     if world > 1:
         import torch.distributed as dist
-        torch.cuda.set_device(local)
-        dist.init_process_group("nccl")
-    else:
+        if cuda:
+            torch.cuda.set_device(local)
+        dist.init_process_group(backend)
+    elif cuda:
         torch.cuda.set_device(0)
     return rank, local, world
 
 
-def barrier(world):
+def barrier(world, cuda=True):
     import torch
-    torch.cuda.synchronize()
+    if cuda:
+        torch.cuda.synchronize()
     if world > 1:
         import torch.distributed as dist
         dist.barrier()
-    torch.cuda.synchronize()
+    if cuda:
+        torch.cuda.synchronize()
 
 
-def reduce_max(x, world):
+def reduce_max(x, world, device="cuda"):
+    """Max of a per-rank float over all ranks (the job's time is its slowest rank's)."""
     if world == 1:
         return x
     import torch
     import torch.distributed as dist
-    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    t = torch.tensor([x], dtype=torch.float64, device=device)
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
+
+
+def job_throughput(tokens_per_rank, world, ms_per_step):
+    """Whole-job tokens/s: every rank's tokens over the max-over-ranks step time."""
+    return tokens_per_rank * world / (ms_per_step / 1e3)
 
 
 # ---------------------------------------------------------------------------
@@ -263,8 +274,7 @@ def run_gpu(args):
     fwd_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in evs)
     bwd_ms = statistics.mean(e[1].elapsed_time(e[2]) for e in evs)
     ms_step = total_ms / args.steps
-    tokens = B * T * world
-    value = tokens / (ms_step / 1e3)
+    value = job_throughput(B * T, world, ms_step)
 
     fb = fwd_bytes(B, T, H, DK, DV)
     bb = bwd_bytes(B, T, H, DK, DV)
