@@ -70,7 +70,11 @@ typedef enum {
   KDN_ERR_UNSUPPORTED = 2, /* valid but not built (e.g. dk = 96) */
   KDN_ERR_WORKSPACE = 3,   /* workspace missing or smaller than required */
   KDN_ERR_CUDA = 4,        /* a CUDA launch or runtime call failed */
-  KDN_ERR_TIMEOUT = 5      /* a bounded device-side wait gave up */
+  KDN_ERR_TIMEOUT = 5,     /* a bounded device-side wait gave up */
+  KDN_ERR_RANGE = 6        /* device status only: a 64-token chunk's cumulative decay
+                              exp(G_C) fell below 1e-36 in some channel, outside the fused
+                              kernels' range (results of that call are invalid); the
+                              general kernels (desc->chunk = 32) halve the exposure */
 } kdn_status_t;
 
 typedef enum { KDN_F32 = 0, KDN_BF16 = 1 } kdn_dtype_t;
@@ -224,7 +228,8 @@ kdn_status_t kdn_diag_fwd_noalloc(const kdn_desc_t *desc, const void *q,
 int kdn_kernel_launches(const kdn_desc_t *desc, int variant, int op);
 
 /* Synchronises `stream`, then returns and clears the device status word kept
-   in the first bytes of `workspace`: KDN_OK, or KDN_ERR_TIMEOUT when a bounded
+   in the first bytes of `workspace`: KDN_OK; KDN_ERR_RANGE when a fused kernel
+   met a chunk whose cumulative decay left its range; or KDN_ERR_TIMEOUT when a bounded
    device-side wait of the most recent kdn_*_fwd / kdn_*_bwd call on that
    workspace gave up.  Each of those calls clears the word before it starts. */
 kdn_status_t kdn_get_device_status(void *workspace, void *stream);

@@ -25,7 +25,7 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libkdn.so")
 
 KDN_OK, KDN_ERR_INVALID_ARG, KDN_ERR_UNSUPPORTED, KDN_ERR_WORKSPACE, KDN_ERR_CUDA, \
-    KDN_ERR_TIMEOUT = range(6)
+    KDN_ERR_TIMEOUT, KDN_ERR_RANGE = range(7)
 KDN_F32, KDN_BF16 = 0, 1
 
 _DTYPES = {torch.float32: KDN_F32, torch.bfloat16: KDN_BF16}

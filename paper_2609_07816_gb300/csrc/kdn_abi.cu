@@ -295,6 +295,7 @@ const char *kdn_status_string(kdn_status_t s) {
     case KDN_ERR_WORKSPACE: return "KDN_ERR_WORKSPACE";
     case KDN_ERR_CUDA: return "KDN_ERR_CUDA";
     case KDN_ERR_TIMEOUT: return "KDN_ERR_TIMEOUT";
+    case KDN_ERR_RANGE: return "KDN_ERR_RANGE";
   }
   return "KDN_ERR_UNKNOWN";
 }
@@ -407,7 +408,7 @@ kdn_status_t kdn_get_device_status(void *workspace, void *stream) {
   if (word != 0) {
     if (cudaMemsetAsync(workspace, 0, sizeof word, s) != cudaSuccess) return KDN_ERR_CUDA;
     if (cudaStreamSynchronize(s) != cudaSuccess) return KDN_ERR_CUDA;
-    return word == KDN_ERR_TIMEOUT ? KDN_ERR_TIMEOUT : static_cast<kdn_status_t>(word);
+    return static_cast<kdn_status_t>(word);
   }
   return KDN_OK;
 }

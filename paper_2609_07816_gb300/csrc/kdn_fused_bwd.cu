@@ -442,7 +442,10 @@ __global__ void __launch_bounds__(BT, 1)
       }
       tmem_st16(TPH + lane_base + t0, ph16);
       tmem_st16(TGM + lane_base + t0, e16);
-      if (qq == 3) s_gC[ci] = e;
+      if (qq == 3) {
+        s_gC[ci] = e;
+        check_gamma_range(e, a.status);
+      }
 #pragma unroll
       for (int j = 0; j < 16; ++j) {
         const float kk = raw_k(t0 + j);
@@ -520,7 +523,10 @@ __global__ void __launch_bounds__(BT, 1)
 #pragma unroll
         for (int j = 0; j < 16; ++j) e16[j] *= pre;
         tmem_st16(TGM + lane_base + t0, e16);
-        if (qq == 3) s_gC[ci] = e16[15];
+        if (qq == 3) {
+          s_gC[ci] = e16[15];
+          check_gamma_range(e16[15], a.status);
+        }
         if (ci == 0) {
           float n = a.fpin[((size_t)bh * NC + c) * D], d = 1.f;
           for (int q2 = 0; q2 < qq; ++q2) {

@@ -83,6 +83,14 @@ __device__ __forceinline__ void unpack_h8(uint4 u, float *v) {
 constexpr int kCtxS = 0, kCtxR = 32768, kCtxW = 49152, kCtxAqk = 65536, kCtxA = 73728;
 constexpr int kCtxBytes = 81920;
 
+// Smallest cumulative decay gamma_C = exp(G_C) of a chunk the fused kernels
+// accept: they divide by gamma (Kk = kappa / gamma), which must stay a normal
+// fp32 number.  Below it a kernel records KDN_ERR_RANGE in the status word.
+constexpr float kMinGammaC = 1e-36f;
+__device__ __forceinline__ void check_gamma_range(float gC, unsigned *status) {
+  if (!(gC >= kMinGammaC)) atomicCAS(status, 0u, (unsigned)KDN_ERR_RANGE);
+}
+
 // Row stride (floats) of the fp32 T and A tiles: 16-byte rows, conflict-free.
 constexpr int LT = 68;
 

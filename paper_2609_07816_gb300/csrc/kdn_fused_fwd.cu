@@ -374,6 +374,7 @@ __global__ void __launch_bounds__(FT, 1)
       __syncthreads();
       if (qq == 3) {
         s_gC[i] = gc_out;
+        check_gamma_range(gc_out, a.status);
         if (V == 0) s_p[i] = carry_out;
         else if (i == 0) s_b[0] = carry_out;
       }

@@ -37,7 +37,8 @@ def test_exports_every_declared_symbol(kdn):
 def test_version_and_status_strings(kdn):
     assert kdn.lib().kdn_version() >= 100
     for code, name in enumerate(["KDN_OK", "KDN_ERR_INVALID_ARG", "KDN_ERR_UNSUPPORTED",
-                                 "KDN_ERR_WORKSPACE", "KDN_ERR_CUDA", "KDN_ERR_TIMEOUT"]):
+                                 "KDN_ERR_WORKSPACE", "KDN_ERR_CUDA", "KDN_ERR_TIMEOUT",
+                                 "KDN_ERR_RANGE"]):
         assert kdn.status_string(code) == name
     assert kdn.status_string(99) == "KDN_ERR_UNKNOWN"
 

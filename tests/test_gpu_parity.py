@@ -306,3 +306,33 @@ def test_training_pair_matches_recompute_path(kdn):
     for n in ("dq", "dk", "dv", "dg", "domega", "dr", "dS0", "dp0"):
         assert torch.equal(g1[n], g2[n]), n
         check(n, g2[n], ref[n], "bf16")
+
+
+@pytest.mark.parametrize("variant", ["diag", "iso"])
+def test_fused_decay_range_is_reported(kdn, variant):
+    """alpha = e^-2 for 64 tokens puts exp(G_C) at e^-128, below the fused kernels'
+    range: the call records KDN_ERR_RANGE in the workspace status word (no fault);
+    the general kernels (32-token chunks, exp(G_C) >= e^-64) match the oracle."""
+    ins = make_inputs(variant, 1, 100, 2, 128, 128, dtype="bf16", seed=3, with_grad=True)
+    ins["g"][...] = -2.0
+    d = to_dev(ins)
+    x = [d[n] for n in ("q", "k", "v", "g", "omega", "r")]
+    fwd = kdn.kdn_diag_fwd if variant == "diag" else kdn.kdn_iso_fwd
+    desc = kdn.make_desc(1, 100, 2, 128, 128, torch.bfloat16,
+                         decay_per_channel=int(d["g"].dim() == 4))
+    ws = kdn.alloc_workspace(desc, 0 if variant == "diag" else 1, True)
+    fwd(*x, workspace=ws)
+    assert kdn.kdn_get_device_status(ws) == kdn.KDN_ERR_RANGE
+    fwd(*x, workspace=ws)  # the word is cleared by the query and set again by the call
+    assert kdn.kdn_get_device_status(ws) == kdn.KDN_ERR_RANGE
+    bwd = kdn.kdn_diag_bwd if variant == "diag" else kdn.kdn_iso_bwd
+    bwd(*x, None, None, d["dO"], workspace=ws)
+    assert kdn.kdn_get_device_status(ws) == kdn.KDN_ERR_RANGE
+    desc32 = kdn.make_desc(1, 100, 2, 128, 128, torch.bfloat16, chunk=32,
+                           decay_per_channel=int(d["g"].dim() == 4))
+    ws32 = kdn.alloc_workspace(desc32, 0 if variant == "diag" else 1, False)
+    o, ST, pT = fwd(*x, chunk=32, workspace=ws32)
+    torch.cuda.synchronize()
+    assert kdn.kdn_get_device_status(ws32) == kdn.KDN_OK
+    ref = _oracle_fwd(variant, ins)
+    check("o", o, ref["o"], "bf16")
