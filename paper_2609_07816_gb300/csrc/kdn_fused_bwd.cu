@@ -68,18 +68,18 @@ constexpr int O_SIN = 32 * KB;   // S_in fp16 [i][j] (context)  -> Kbar^T hi | Q
 constexpr int O_RV = 64 * KB;    // raw v  -> v fp16
 constexpr int O_RDO = 80 * KB;   // raw dO -> lambda dO fp16 -> Qbar^T lo
 constexpr int O_AH = 96 * KB;    // A fp16 [t][s] (context)
-constexpr int O_SQ = 104 * KB;   // gain quarter summaries (10 KB)  -> A bf16 [t][s]
+constexpr int O_AB = 104 * KB;   // A bf16 [t][s] (from the saved fp16 A)
 constexpr int O_DT = 112 * KB;   // dT bf16  -> per-channel scratch of the final stage
 constexpr int O_AQ = 120 * KB;   // A_qk fp16 [t][s] (context)
 constexpr int O_WN = 128 * KB;   // -W fp16 [t][i] (context)  -> Kk^T hi
 constexpr int O_KT = 144 * KB;   // K_tail^T fp16  -> dR^T fp16
-constexpr int O_G = 160 * KB;    // raw g | raw omega  -> dS fp16  -> dA_qk^T | Qbar^T fp16
-                                 //   -> dW^T | Kk^T lo -> dA^T | X  -> dG of the final stage
+constexpr int O_G = 160 * KB;    // dS fp16  -> dA_qk^T | Qbar^T fp16  -> dW^T | Kk^T lo
+                                 //   -> dA^T | X  -> dG of the final stage
 constexpr int O_RH = 192 * KB;   // R fp16 (context; the next 8 KB are read as padding rows)
                                  //   -> lo part of dR^T fp16
 constexpr int BUF_END = 216 * KB;
 // derived tenants
-constexpr int O_W = O_G + 16 * KB, O_AB = O_SQ, O_DRT = O_KT, O_KKH2 = O_WN;
+constexpr int O_DRT = O_KT, O_KKH2 = O_WN;
 constexpr int O_DSH = O_G, O_DAQ = O_G, O_QH = O_G + 16 * KB, O_KKL2 = O_G + 16 * KB;
 constexpr int O_DWT = O_G, O_DAT = O_G + 16 * KB, O_XT = O_G + 24 * KB, O_KQH2 = O_SIN;
 constexpr int O_QL2 = O_RDO, O_DRTL = O_RH;
@@ -93,8 +93,6 @@ static_assert(O_AQ + 8 * KB <= O_WN && O_XT + 8 * KB <= O_RH, "map");
 
 struct BwdParams {
   Args a;
-  int has_g_map;  // per-channel decay tile through TMA
-  int has_w_map;  // per-channel omega tile through TMA (diag)
 };
 
 __device__ __forceinline__ uint64_t kdesc(const unsigned char *p) {
@@ -161,15 +159,13 @@ __device__ __forceinline__ float rs16(const float *v, int lane) {
 template <int V>
 __global__ void __launch_bounds__(BT, 1)
     k_fused_bwd(const __grid_constant__ CUtensorMap mq, const __grid_constant__ CUtensorMap mk,
-                const __grid_constant__ CUtensorMap mv, const __grid_constant__ CUtensorMap mg,
-                const __grid_constant__ CUtensorMap mw, const __grid_constant__ CUtensorMap mdo,
+                const __grid_constant__ CUtensorMap mv, const __grid_constant__ CUtensorMap mdo,
                 const BwdParams P) {
   const Args &a = P.a;
   extern __shared__ unsigned char smraw[];
   unsigned char *sm =
       reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(smraw) + 1023) & ~uintptr_t(1023));
   unsigned char *rkq = sm + O_RKQ, *sin = sm + O_SIN, *rv = sm + O_RV, *rdo = sm + O_RDO;
-  unsigned char *rg = sm + O_G, *rw = sm + O_W;
   float *s_r = reinterpret_cast<float *>(sm + OFF_SM);  // [64] r_t
   float *s_ri = s_r + 64;     // [64] 1 / r_t
   float *s_s = s_ri + 64;     // [64] s_t = r_t + sum_i phat k^2
@@ -209,8 +205,6 @@ __global__ void __launch_bounds__(BT, 1)
     prefetch_tmap(&mq);
     prefetch_tmap(&mk);
     prefetch_tmap(&mv);
-    if (P.has_g_map) prefetch_tmap(&mg);
-    if (P.has_w_map) prefetch_tmap(&mw);
     prefetch_tmap(&mdo);
   }
   if (warp == 0) {
@@ -228,7 +222,7 @@ __global__ void __launch_bounds__(BT, 1)
   // loads of chunk c on bar_a: the context record (S_in, R, -W, A_qk, A; issued as
   // soon as their buffers free up) and the raw k, q, g, omega tiles (issued once the
   // previous chunk is done; the one expect_tx covers both groups); bar_b <- dO, v
-  const uint32_t kBytesA = 81920u + 16384u * (2 + (P.has_g_map ? 1 : 0) + (P.has_w_map ? 1 : 0));
+  const uint32_t kBytesA = 81920u + 16384u * 2;
   auto issue_a_ctx = [&](int c) {
     const unsigned char *rec = a.fSin + ((size_t)bh * NC + c) * kCtxBytes;
     mbar_expect_tx(bar_a, kBytesA);
@@ -242,8 +236,6 @@ __global__ void __launch_bounds__(BT, 1)
     for (int s = 0; s < 2; ++s) {
       tma_load_4d(rkq + s * 16384, &mk, bar_a, 64 * s, h, c * CM, b);
       tma_load_4d(rkq + s * 16384 + 8192, &mq, bar_a, 64 * s, h, c * CM, b);
-      if (P.has_g_map) tma_load_4d(rg + s * 8192, &mg, bar_a, 64 * s, h, c * CM, b);
-      if (P.has_w_map) tma_load_4d(rw + s * 8192, &mw, bar_a, 64 * s, h, c * CM, b);
     }
   };
   auto issue_b_do = [&](int c) {
@@ -325,22 +317,18 @@ __global__ void __launch_bounds__(BT, 1)
     s_dp[tid] = a.dpT ? lam * a.dpT[pi] : 0.f;
   }
 
-  // per-token scalars of the next chunk (r; omega and a scalar decay for the
-  // isotropic KDN), prefetched into registers
-  float nr = 1.f, nom = 0.f, ng = 0.f;
+  // per-token scalars of the next chunk (r; the scalar decay of the isotropic KDN),
+  // prefetched into registers
+  float nr = 1.f, ng = 0.f;
   auto load_r = [&](int c) {
     nr = 1.f;
-    nom = 0.f;
     ng = 0.f;
     if (tid < CM && c >= 0) {
       const int t = c * CM + tid;
       if (t < a.T) {
         const size_t th = tok_index(a, b, t, h);
         nr = ld<__nv_bfloat16>(a.r, th);
-        if (V == 1) {
-          nom = ld<__nv_bfloat16>(a.omega, th);
-          if (!a.pcd) ng = ld<__nv_bfloat16>(a.g, th);
-        }
+        if (V == 1 && !a.pcd) ng = ld<__nv_bfloat16>(a.g, th);
       }
     }
   };
@@ -378,177 +366,59 @@ __global__ void __launch_bounds__(BT, 1)
 
   for (int it = 0; it < NC && ok; ++it) {
     const int c = NC - 1 - it;
-    // ---- [1] per-token scalars; raw tiles of this chunk
+    // ---- [1] per-token scalars; the chunk's gains from the context the forward saved
+    //          (global loads issued before the wait for the tiles); raw tiles
     if (tid < CM) {
       s_r[tid] = nr;
       s_ri[tid] = 1.f / nr;
-      s_om[tid] = nom;
       s_gs[tid] = ng;
+    }
+    const unsigned char *rec = a.fSin + ((size_t)bh * NC + c) * kCtxBytes;
+    float e16[16], ph16[16], tk[5];
+    {
+      const float *cga = reinterpret_cast<const float *>(rec + kCtxGa) + t0 * D + ci;
+      const float *cph = reinterpret_cast<const float *>(rec + kCtxPh) + t0 * D + ci;
+      const float *tok = reinterpret_cast<const float *>(rec + kCtxTok);
+#pragma unroll
+      for (int j = 0; j < 16; ++j) e16[j] = cga[j * D];
+      if (V == 0) {
+#pragma unroll
+        for (int j = 0; j < 16; ++j) ph16[j] = cph[j * D];
+      }
+      if (tid < CM) {
+#pragma unroll
+        for (int m = 0; m < (V == 0 ? 1 : 5); ++m) tk[m] = tok[64 * m + tid];
+      }
     }
     ok = __syncthreads_and(mbar_wait(bar_a, it & 1, kWaitIters));
     if (!ok) break;
     load_r(c - 1);
 
-    // ---- [2] gain recursion of this chunk from the saved entry uncertainty (as in
-    //          the forward: four quarters of 16 tokens, Moebius products combined
-    //          into each quarter's entry value); phat, gamma -> TMEM (lane = channel)
+    // ---- [2] the chunk's gains from the context the forward saved: phat (diag) and
+    //          gamma -> TMEM (lane = channel), per-token s_t (diag) or beta_t, |k_t|^2,
+    //          a_t, bhat_t, b_{t-1} (iso)
     float dgc = 0.f;  // this thread's part of dgamma_C for channel ci
     {
-      float *sQ = reinterpret_cast<float *>(sm + O_SQ);  // [4][128][5] quarter summaries
-      float ph16[16], e16[16];
-      if (V == 0) {
-      float al[16], w[16], uk[16];
-#pragma unroll
-      for (int j = 0; j < 16; ++j) {
-        const float kk = raw_k(t0 + j);
-        al[j] = __expf(bf(rg, 8192, t0 + j, ci));
-        w[j] = bf(rw, 8192, t0 + j, ci);
-        uk[j] = mu * kk * kk * s_ri[t0 + j];
-      }
-      float m00 = 1.f, m01 = 0.f, m10 = 0.f, m11 = 1.f, eq = 1.f;
-#pragma unroll
-      for (int j = 0; j < 16; ++j) {
-        const float a2_ = al[j] * al[j], ua2 = uk[j] * a2_, d1 = 1.f + uk[j] * w[j];
-        const float n00 = a2_ * m00 + w[j] * m10, n01 = a2_ * m01 + w[j] * m11;
-        const float n10 = ua2 * m00 + d1 * m10, n11 = ua2 * m01 + d1 * m11;
-        m00 = n00; m01 = n01; m10 = n10; m11 = n11;
-        eq *= al[j];
-        if ((j & 7) == 7) {
-          const float sc = __frcp_rn(fmaxf(fmaxf(fabsf(m00), fabsf(m01)), fmaxf(fabsf(m10), fabsf(m11))));
-          m00 *= sc; m01 *= sc; m10 *= sc; m11 *= sc;
-        }
-      }
-      float *mine = sQ + (qq * D + ci) * 5;
-      mine[0] = m00; mine[1] = m01; mine[2] = m10; mine[3] = m11; mine[4] = eq;
-      __syncthreads();
-      float n = a.fpin[((size_t)bh * NC + c) * D + ci], d = 1.f, e = 1.f;
-      for (int q2 = 0; q2 < qq; ++q2) {
-        const float *o = sQ + (q2 * D + ci) * 5;
-        const float nn = o[0] * n + o[1] * d, dd = o[2] * n + o[3] * d;
-        const float sc = __frcp_rn(fmaxf(fabsf(nn), fabsf(dd)));
-        n = nn * sc;
-        d = dd * sc;
-        e *= o[4];
-      }
-      float p = __fdividef(n, d);
-      float y[16];
-#pragma unroll
-      for (int j = 0; j < 16; ++j) {
-        e *= al[j];
-        const float ph = al[j] * al[j] * p + w[j];  // eq. diag-covariance-prediction
-        ph16[j] = ph;
-        e16[j] = e;
-        p = __fdividef(ph, 1.f + uk[j] * ph);  // eq. prefix-diag-uncertainty
-      }
-      tmem_st16(TPH + lane_base + t0, ph16);
+      if (V == 0) tmem_st16(TPH + lane_base + t0, ph16);
       tmem_st16(TGM + lane_base + t0, e16);
       if (qq == 3) {
-        s_gC[ci] = e;
-        check_gamma_range(e, a.status);
+        s_gC[ci] = e16[15];
+        check_gamma_range(e16[15], a.status);
       }
-#pragma unroll
-      for (int j = 0; j < 16; ++j) {
-        const float kk = raw_k(t0 + j);
-        y[j] = ph16[j] * kk * kk;
+      if (tid < CM) {
+        if (V == 0) {
+          s_s[tid] = tk[0];
+          s_si[tid] = 1.f / tk[0];
+        } else {
+          s_x[tid] = tk[0];
+          s_n2[tid] = tk[1];
+          s_a[tid] = tk[2];
+          s_bh[tid] = tk[3];
+          s_bp[tid] = tk[4];
+        }
       }
-      const float ys = rs16(y, lane);
-      if ((lane & 1) == 0) s_red[wq * 64 + t0 + (lane >> 1)] = ys;
       tmem_st_wait();
       __syncthreads();
-      if (tid < CM) {
-        const float st = s_r[tid] + ((s_red[tid] + s_red[64 + tid]) + (s_red[128 + tid] + s_red[192 + tid]));
-        s_s[tid] = st;
-        s_si[tid] = 1.f / st;
-      }
-      __syncthreads();
-      } else {
-        // per-token |k_t|^2 and a_t = mean_i alpha_ti^2 (or alpha_t^2), one half-warp per token
-        for (int m = 0; m < 2; ++m) {
-          const int t = 32 * m + 2 * warp + (lane >> 4), c8 = lane & 15, sl = c8 >> 3, cc = c8 & 7;
-          float kv[8];
-          unpack_bf8(sm16(rkq, sl * 16384 + chunk_off(t, cc)), kv);
-          float n2 = 0.f, sa = 0.f;
-#pragma unroll
-          for (int j = 0; j < 8; ++j) n2 += kv[j] * kv[j];
-          if (pcd) {
-            float gv[8];
-            unpack_bf8(sm16(rg, sl * 8192 + chunk_off(t, cc)), gv);
-#pragma unroll
-            for (int j = 0; j < 8; ++j) {
-              const float al = __expf(gv[j]);
-              sa += al * al;
-            }
-          }
-#pragma unroll
-          for (int o = 8; o > 0; o >>= 1) {
-            n2 += __shfl_xor_sync(0xffffffffu, n2, o);
-            sa += __shfl_xor_sync(0xffffffffu, sa, o);
-          }
-          if (c8 == 0) {
-            s_n2[t] = n2;
-            const float al = __expf(s_gs[t]);
-            s_a[t] = pcd ? sa * (1.f / D) : al * al;
-          }
-        }
-        __syncthreads();
-        // cumulative decay of channel ci within this quarter
-        float eq = 1.f;
-#pragma unroll
-        for (int j = 0; j < 16; ++j) {
-          eq *= __expf(pcd ? bf(rg, 8192, t0 + j, ci) : s_gs[t0 + j]);
-          e16[j] = eq;
-        }
-        sQ[(qq * D + ci) * 5 + 4] = eq;
-        // scalar Moebius product of this quarter (Prop. 5, eq. iso-kla-box-mobius)
-        if (ci == 0) {
-          float m00 = 1.f, m01 = 0.f, m10 = 0.f, m11 = 1.f;
-          for (int j = 0; j < 16; ++j) {
-            const int t = t0 + j;
-            const float at = s_a[t], wt = s_om[t], ut = mu * s_n2[t] * s_ri[t] * (1.f / D);
-            const float n00 = at * m00 + wt * m10, n01 = at * m01 + wt * m11;
-            const float n10 = ut * at * m00 + (1.f + ut * wt) * m10;
-            const float n11 = ut * at * m01 + (1.f + ut * wt) * m11;
-            m00 = n00; m01 = n01; m10 = n10; m11 = n11;
-            if ((j & 7) == 7) {
-              const float sc = __frcp_rn(fmaxf(fmaxf(fabsf(m00), fabsf(m01)), fmaxf(fabsf(m10), fabsf(m11))));
-              m00 *= sc; m01 *= sc; m10 *= sc; m11 *= sc;
-            }
-          }
-          float *mine = sQ + (qq * D) * 5;
-          mine[0] = m00; mine[1] = m01; mine[2] = m10; mine[3] = m11;
-        }
-        __syncthreads();
-        float pre = 1.f;
-        for (int q2 = 0; q2 < qq; ++q2) pre *= sQ[(q2 * D + ci) * 5 + 4];
-#pragma unroll
-        for (int j = 0; j < 16; ++j) e16[j] *= pre;
-        tmem_st16(TGM + lane_base + t0, e16);
-        if (qq == 3) {
-          s_gC[ci] = e16[15];
-          check_gamma_range(e16[15], a.status);
-        }
-        if (ci == 0) {
-          float n = a.fpin[((size_t)bh * NC + c) * D], d = 1.f;
-          for (int q2 = 0; q2 < qq; ++q2) {
-            const float *o = sQ + (q2 * D) * 5;
-            const float nn = o[0] * n + o[1] * d, dd = o[2] * n + o[3] * d;
-            const float sc = __frcp_rn(fmaxf(fabsf(nn), fabsf(dd)));
-            n = nn * sc;
-            d = dd * sc;
-          }
-          float bb = __fdividef(n, d);
-          for (int j = 0; j < 16; ++j) {
-            const int t = t0 + j;
-            const float bhat = s_a[t] * bb + s_om[t];  // eq. iso-kla-box-cov-update
-            s_bp[t] = bb;
-            s_bh[t] = bhat;
-            s_x[t] = __fdividef(bhat, s_r[t] + bhat * s_n2[t]);  // beta_t, eq. iso-kla-box-gain
-            bb = __fdividef(bhat, 1.f + mu * s_n2[t] * s_ri[t] * (1.f / D) * bhat);
-          }
-        }
-        tmem_st_wait();
-        __syncthreads();
-      }
     }
     // ---- [3] operands of the chunk adjoint from the context and the gains:
     //          A bf16 (from the saved fp16 A); dS -> fp16 [i][j] and dS <- gamma_C dS in
@@ -836,10 +706,17 @@ __global__ void __launch_bounds__(BT, 1)
       float *s_tot = reinterpret_cast<float *>(sm + O_DT);  // [4][128] quarter sums of dG
       float *s_dgc = s_tot + 512;                           // [4][128] dgamma_C parts
       float *s_aff = s_dgc + 512;                           // [4][128][2] affine summaries
-      float ph[16], ga[16], k16[16];
+      float ph[16], ga[16], k16[16], q16[16];
       load_ph_ga(ph, ga);
 #pragma unroll
-      for (int j = 0; j < 16; ++j) k16[j] = raw_k(t0 + j);
+      for (int j = 0; j < 16; ++j) {
+        k16[j] = raw_k(t0 + j);
+        q16[j] = raw_q(t0 + j);
+      }
+      const float kprev = qq > 0 ? raw_k(t0 - 1) : 0.f;
+      fence_proxy_async();
+      __syncthreads();  // raw k, q are in registers: the next chunk's tiles may land
+      if (tid == 0 && c > 0) issue_a_raw(c - 1);
       // outputs of token t0 + j live at obase + j * ostride; nval tokens of the quarter are real
       const size_t ostride = (size_t)a.H * D;
       const size_t obase = tok_index(a, b, c * CM + t0, h) * D + ci;
@@ -862,7 +739,7 @@ __global__ void __launch_bounds__(BT, 1)
 #pragma unroll
           for (int u = 0; u < 8; ++u) {
             const int j = 8 * h8 + u, t = t0 + j;
-            const float kk = k16[j], qv = raw_q(t), si = s_si[t], g_ = ga[j], ig = __fdividef(1.f, g_);
+            const float kk = k16[j], qv = q16[j], si = s_si[t], g_ = ga[j], ig = __fdividef(1.f, g_);
             const float kap = ph[j] * kk * si;  // kappa_t (eq. kla-box-gain)
             const float dG = xb[u] * g_ * kk - xk[u] * kap * ig + xq[u] * tau * g_ * qv;
             sdg[j * BT + tid] = dG;
@@ -891,7 +768,7 @@ __global__ void __launch_bounds__(BT, 1)
         float t8[8], g8[8];
         tmem_ld8(TPH + lane_base + t0 - 8, t8);
         tmem_ld8(TGM + lane_base + t0 - 8, g8);
-        const float kk = raw_k(t0 - 1);
+        const float kk = kprev;
         ga_prev = g8[7];  // gamma_{t0-1}
         p_prev = __fdividef(t8[7], 1.f + mu * kk * kk * s_ri[t0 - 1] * t8[7]);
       } else {
@@ -982,10 +859,16 @@ __global__ void __launch_bounds__(BT, 1)
       float *s_tot = reinterpret_cast<float *>(sm + O_DT);  // [4][128] quarter sums of dG
       float *s_dgc = s_tot + 512;                           // [4][128] dgamma_C parts
       float *s_aff = s_dgc + 512;                           // [4][2] affine summaries
-      float ga[16], k16[16];
+      float ga[16], k16[16], q16[16];
       tmem_ld16(TGM + lane_base + t0, ga);
 #pragma unroll
-      for (int j = 0; j < 16; ++j) k16[j] = raw_k(t0 + j);
+      for (int j = 0; j < 16; ++j) {
+        k16[j] = raw_k(t0 + j);
+        q16[j] = raw_q(t0 + j);
+      }
+      fence_proxy_async();
+      __syncthreads();  // raw k, q are in registers: the next chunk's tiles may land
+      if (tid == 0 && c > 0) issue_a_raw(c - 1);
       const size_t ostride = (size_t)a.H * D;
       const size_t obase = tok_index(a, b, c * CM + t0, h) * D + ci;
       const int nval = min(16, a.T - (c * CM + t0));
@@ -1007,7 +890,7 @@ __global__ void __launch_bounds__(BT, 1)
 #pragma unroll
           for (int u = 0; u < 8; ++u) {
             const int j = 8 * h8 + u, t = t0 + j;
-            const float kk = k16[j], qv = raw_q(t), g_ = ga[j], ig = __fdividef(1.f, g_);
+            const float kk = k16[j], qv = q16[j], g_ = ga[j], ig = __fdividef(1.f, g_);
             const float beta = s_x[t], kap = beta * kk;
             const float dG = xb[u] * g_ * kk - xk[u] * kap * ig + xq[u] * tau * g_ * qv;
             sdg[j * BT + tid] = dG;
@@ -1109,11 +992,9 @@ __global__ void __launch_bounds__(BT, 1)
         }
       }
     }
-    fence_proxy_async();
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    if (tid == 0 && c > 0) issue_a_raw(c - 1);  // raw k, q, g, omega buffers are free
   }
 
   if (ok) {
@@ -1163,21 +1044,15 @@ size_t fused_ctx_record_bytes() { return kCtxBytes; }
 kdn_status_t launch_fused_bwd_sweep(const Args &a, cudaStream_t s) {
   BwdParams P;
   P.a = a;
-  P.has_g_map = (a.variant == 0 || a.pcd) ? 1 : 0;
-  P.has_w_map = a.variant == 0 ? 1 : 0;
-  CUtensorMap mq, mk, mv, mg, mw, mdo;
+  CUtensorMap mq, mk, mv, mdo;
   if (!make_map(&mq, a.q, a) || !make_map(&mk, a.k, a) || !make_map(&mv, a.v, a) ||
       !make_map(&mdo, a.dO, a))
     return KDN_ERR_CUDA;
-  mg = mq;
-  mw = mq;
-  if (P.has_g_map && !make_map(&mg, a.g, a)) return KDN_ERR_CUDA;
-  if (P.has_w_map && !make_map(&mw, a.omega, a)) return KDN_ERR_CUDA;
   auto kern = a.variant == 0 ? k_fused_bwd<0> : k_fused_bwd<1>;
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES) !=
       cudaSuccess)
     return KDN_ERR_CUDA;
-  kern<<<a.B * a.H, BT, SMEM_BYTES, s>>>(mq, mk, mv, mg, mw, mdo, P);
+  kern<<<a.B * a.H, BT, SMEM_BYTES, s>>>(mq, mk, mv, mdo, P);
   return cudaGetLastError() == cudaSuccess ? KDN_OK : KDN_ERR_CUDA;
 }
 

@@ -80,8 +80,13 @@ __device__ __forceinline__ void unpack_h8(uint4 u, float *v) {
 //   -W    fp16 [64 t][128 i] as two slabs                      16 KB
 //   A_qk  fp16 [64 t][64 s] (lower triangle)                    8 KB
 //   A     fp16 [64 t][64 s] (lower triangle)                    8 KB
+//   phat  fp32 [64 t][128 i] (diag; pre-write variance)        32 KB
+//   gamma fp32 [64 t][128 i] (cumulative decay in the chunk)   32 KB
+//   per-token fp32 [5][64]: s_t (diag) or beta_t, then |k_t|^2, a_t, bhat_t,
+//         b_{t-1} (iso)                                          2 KB
 constexpr int kCtxS = 0, kCtxR = 32768, kCtxW = 49152, kCtxAqk = 65536, kCtxA = 73728;
-constexpr int kCtxBytes = 81920;
+constexpr int kCtxPh = 81920, kCtxGa = 114688, kCtxTok = 147456;
+constexpr int kCtxBytes = 149504;
 
 // Smallest cumulative decay gamma_C = exp(G_C) of a chunk the fused kernels
 // accept: they divide by gamma (Kk = kappa / gamma), which must stay a normal

@@ -63,7 +63,7 @@ constexpr int OFF_B3 = OFF_A2 + 16384;    // S_in fp16 (MN-major)               
 constexpr int OFF_F = OFF_B3 + 32768;     // fp32 scratch: gamma [64][128] / T, A [64][LT] + X
 constexpr int F_BYTES = 2 * 64 * LT * 4 + 3 * 256 * 4;  // 37888 >= 32768
 constexpr int OFF_SM = OFF_F + F_BYTES;                  // small arrays
-constexpr int SMALL_FLOATS = 64 * 7 + 128 * 3;
+constexpr int SMALL_FLOATS = 64 * 9 + 128 * 3;
 constexpr int OFF_BAR = OFF_SM + SMALL_FLOATS * 4;
 constexpr int SMEM_BYTES = OFF_BAR + 64 + 1024;  // + alignment slack
 
@@ -95,7 +95,9 @@ __global__ void __launch_bounds__(FT, 1)
   float *s_x = s_r + 64;     // [64] s_t (diag) / beta_t (iso)
   float *s_n2 = s_x + 64;    // [64] |k|^2 (iso)
   float *s_a = s_n2 + 64;    // [64] a_t (iso)
-  float *s_om = s_a + 64;    // [64] omega_t (iso)
+  float *s_bh = s_a + 64;    // [64] bhat_t (iso)
+  float *s_bp = s_bh + 64;   // [64] b_{t-1} (iso)
+  float *s_om = s_bp + 64;   // [64] omega_t (iso)
   float *s_gs = s_om + 64;   // [64] scalar g_t (iso, scalar decay)
   float *s_ri = s_gs + 64;   // [64] 1 / r_t
   float *s_gC = s_ri + 64;   // [128] gamma_C
@@ -365,6 +367,8 @@ __global__ void __launch_bounds__(FT, 1)
           for (int j = 0; j < 16; ++j) {
             const int t = t0 + j;
             const float bhat = s_a[t] * bb + s_om[t];          // eq. iso-kla-box-cov-update
+            s_bp[t] = bb;
+            s_bh[t] = bhat;
             s_x[t] = __fdividef(bhat, s_r[t] + bhat * s_n2[t]);  // beta_t, eq. iso-kla-box-gain
             bb = __fdividef(bhat, 1.f + a.mu * s_n2[t] * s_ri[t] * (1.f / D) * bhat);
           }
@@ -379,8 +383,14 @@ __global__ void __launch_bounds__(FT, 1)
         else if (i == 0) s_b[0] = carry_out;
       }
     }
+    fence_proxy_async();  // phat / gamma are read by the bulk copies below
     __syncthreads();
     if (tid == 0 && c + 1 < NC) issue_raw_g(c + 1);  // the decay tile is no longer read
+    if (tid == 0 && P.save_S) {  // phat and gamma into the backward context
+      if (V == 0) bulk_s2g(ctx + kCtxPh, Pb, 32768);
+      bulk_s2g(ctx + kCtxGa, Eb, 32768);
+      bulk_commit();
+    }
     // ---- [3] operand tiles, 16-byte chunks (t, 8 channels), one half-warp per token:
     //   Kk = phat k / (s_t gamma) (diag, s_t = r_t + sum phat k^2) or beta_t k / gamma (iso)
     //   Kbar = gamma k, Qbar = tau gamma q; each as a hi/lo bf16 pair, written over
@@ -407,7 +417,8 @@ __global__ void __launch_bounds__(FT, 1)
         for (int j = 0; j < 8; ++j) y += ph[j] * kv[j] * kv[j];
 #pragma unroll
         for (int o = 8; o > 0; o >>= 1) y += __shfl_xor_sync(0xffffffffu, y, o);
-        const float sc = 1.f / (s_r[t] + y);  // eq. kla-box-gain
+        const float st = s_r[t] + y, sc = 1.f / st;  // eq. kla-box-gain
+        if (c8 == 0) s_x[t] = st;
 #pragma unroll
         for (int j = 0; j < 8; ++j) xv[j] = __fdividef(ph[j] * kv[j] * sc, ev[j]);
       } else {
@@ -431,6 +442,10 @@ __global__ void __launch_bounds__(FT, 1)
     fence_proxy_async();
     tc_fence_before();
     __syncthreads();
+    if (tid == 0 && P.save_S) {  // per-token scalars of the gain into the backward context
+      bulk_s2g(ctx + kCtxTok, s_x, 5 * 64 * 4);
+      bulk_commit();
+    }
     // ---- [4] MMA-T: D1 = [Kbar; Qbar] Kk^T, hi.hi + lo.hi + hi.lo
     if (tid == 0) {
       tc_fence_after();
@@ -444,6 +459,7 @@ __global__ void __launch_bounds__(FT, 1)
       }
       umma_commit(bar_mma);
     }
+    if (tid == 0 && P.save_S) bulk_wait_read();  // phat / gamma have left b3 / fs
     if (!(ok = mma_wait())) break;
     tc_fence_after();
     // ---- [5] T -> fp32 smem, A = (I + T)^-1 by 16x16 blocks:

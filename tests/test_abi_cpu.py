@@ -157,7 +157,7 @@ def test_fused_path_launches_and_workspace(kdn):
     assert kdn.kdn_kernel_launches(d, 0, 0) == 1
     assert kdn.kdn_kernel_launches(d, 0, 1) == 2
     NC = (T + 63) // 64
-    need = 256 + B * H * NC * 81920 + B * H * NC * 128 * 4
+    need = 256 + B * H * NC * 149504 + B * H * NC * 128 * 4
     assert kdn.workspace_bytes(d, 0, True) == need
     # the isotropic backward is fused too; the 32-token chunk keeps the general kernels
     assert kdn.kdn_kernel_launches(d, 1, 1) == 2
@@ -173,7 +173,7 @@ def test_training_pair_validation(kdn):
     B, T, H = 2, 130, 3
     d = kdn.make_desc(B, T, H, 128, 128, kdn.KDN_BF16)
     n = kdn.saved_bytes(d)
-    assert n == B * H * 3 * (81920 + 512)
+    assert n == B * H * 3 * (149504 + 512)
     assert kdn.saved_bytes(d, 1) == 0
     assert kdn.saved_bytes(kdn.make_desc(B, T, H, 64, 128, kdn.KDN_BF16)) == 0
     assert kdn.saved_bytes(kdn.make_desc(B, T, H, 128, 128, kdn.KDN_F32)) == 0
