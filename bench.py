@@ -297,6 +297,7 @@ def run_gpu(args):
     spec_time = max(B * T * H * chunk_flops(DK, DV) * 3.5 / 2.25e15, (fb + bb) / 8e12)
 
     dec = run_decode(kdn, torch, hbm) if rank == 0 and not args.no_decode else None
+    iso = run_iso_step(kdn, torch, args) if rank == 0 and not args.no_decode else None
     e2e = run_e2e(kdn, torch, x, ins, args) if rank == 0 and not args.no_e2e else None
     out = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
@@ -312,7 +313,7 @@ def run_gpu(args):
         "spec_roofline_frac": spec_time / (ms_step / 1e3) if ms_step > 0 else None,
         "gpu_launches": launches_per_step * args.steps,
         "clocks": clk.summary(),
-        "decode": dec, "e2e": e2e,
+        "decode": dec, "iso_step": iso, "e2e": e2e,
     }
     if rank == 0 and not args.no_cpu_baseline:
         out["cpu_baseline"] = cpu_baseline(sample_heads=args.cpu_heads)
@@ -321,6 +322,35 @@ def run_gpu(args):
     if world > 1:
         import torch.distributed as dist
         dist.destroy_process_group()
+
+
+def run_iso_step(kdn, torch, args):
+    """The Isotropic KDN training step on its 750M-layer shape (B=8, H=12, T=2048,
+    d=128, one decay per head): kdn_iso_fwd_save + kdn_iso_bwd_saved, tokens/s."""
+    b, t, h = 8, 2048, 12
+    ins = device_inputs("iso", b, t, h, DK, DV, seed=7, dtype=torch.bfloat16, per_channel=False)
+    x = [ins[n] for n in NAMES]
+    desc = kdn.make_desc(b, t, h, DK, DV, torch.bfloat16, decay_per_channel=0)
+    saved = torch.empty(kdn.saved_bytes(desc, 1), dtype=torch.uint8, device="cuda")
+    ws = kdn.alloc_workspace(desc, 1, False)
+
+    def step():
+        kdn.kdn_iso_fwd_save(*x, saved=saved, want_state=False, workspace=ws)
+        kdn.kdn_iso_bwd_saved(*x, saved, ins["dO"], want_state_grads=False, workspace=ws)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(args.steps):
+        step()
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / args.steps
+    return {"workload": f"Isotropic KDN fwd+bwd, B={b} H={h} T={t} d=128, one decay per head",
+            "value": b * t / (ms / 1e3), "unit": "tokens/s", "ms_per_step": ms,
+            "gpu_launches": 2 * args.steps}
 
 
 def run_decode(kdn, torch, hbm):

@@ -151,15 +151,16 @@ kdn_status_t kdn_iso_bwd(const kdn_desc_t *desc, const void *q, const void *k,
    A = (I + T)^-1 as fp16 tiles (80 KB) and the float32 uncertainty p entering
    it.  kdn_diag_bwd_saved is kdn_diag_bwd that starts from that
    context instead of recomputing the forward (same gradients, one kernel).
-   Served for the Diagonal KDN with bfloat16 activations, dk = dv = 128 and the
-   default chunk; for every other descriptor kdn_saved_bytes() returns 0 and
-   both calls return KDN_ERR_UNSUPPORTED (use kdn_diag_fwd / kdn_diag_bwd).
-   saved: caller-owned device buffer of kdn_saved_bytes(desc, 0) bytes, 256-byte
+   kdn_iso_fwd_save / kdn_iso_bwd_saved are the same for the Isotropic KDN.
+   Served for bfloat16 activations, dk = dv = 128 and the default chunk; for
+   every other descriptor kdn_saved_bytes() returns 0 and the calls return
+   KDN_ERR_UNSUPPORTED (use kdn_*_fwd / kdn_*_bwd).
+   saved: caller-owned device buffer of kdn_saved_bytes(desc, variant) bytes, 256-byte
    aligned (a smaller or misaligned one -> KDN_ERR_WORKSPACE).  It is written
    by kdn_diag_fwd_save and read by kdn_diag_bwd_saved, which must see the same
    descriptor and the same q, k, v, g, omega, r (and the forward's S0, p0).
-   workspace: kdn_fwd_workspace_bytes(desc, 0) bytes for both calls.  The
-   other arguments are those of kdn_diag_fwd / kdn_diag_bwd. */
+   workspace: kdn_fwd_workspace_bytes(desc, variant) bytes for both calls.  The
+   other arguments are those of kdn_*_fwd / kdn_*_bwd. */
 size_t kdn_saved_bytes(const kdn_desc_t *desc, int variant);
 
 kdn_status_t kdn_diag_fwd_save(const kdn_desc_t *desc, const void *q,
@@ -179,6 +180,24 @@ kdn_status_t kdn_diag_bwd_saved(const kdn_desc_t *desc, const void *q,
                                 void *dg, void *domega, void *dr, float *dS0,
                                 float *dp0, void *workspace,
                                 size_t workspace_bytes, void *stream);
+
+kdn_status_t kdn_iso_fwd_save(const kdn_desc_t *desc, const void *q,
+                              const void *k, const void *v, const void *g,
+                              const void *omega, const void *r,
+                              const float *S0, const float *p0, void *o,
+                              float *ST, float *pT, void *saved,
+                              size_t saved_bytes, void *workspace,
+                              size_t workspace_bytes, void *stream);
+
+kdn_status_t kdn_iso_bwd_saved(const kdn_desc_t *desc, const void *q,
+                               const void *k, const void *v, const void *g,
+                               const void *omega, const void *r,
+                               const void *saved, size_t saved_bytes,
+                               const void *dO, const float *dST,
+                               const float *dpT, void *dq, void *dk, void *dv,
+                               void *dg, void *domega, void *dr, float *dS0,
+                               float *dp0, void *workspace,
+                               size_t workspace_bytes, void *stream);
 
 /* One decode token for all B*H heads (the update of Prop. 3), in place:
    S [B,H,dk,dv] and p [B,H,dk] are read and overwritten; o [B,H,dv] is
@@ -221,7 +240,7 @@ kdn_status_t kdn_diag_fwd_noalloc(const kdn_desc_t *desc, const void *q,
 
 /* Number of CUDA kernels one call of an entry point launches for this
    descriptor when T > 0 (op 0 = kdn_*_fwd, 1 = kdn_*_bwd, 2 = kdn_*_decode_step,
-   3 = kdn_diag_fwd_save, 4 = kdn_diag_bwd_saved; variant 0 = diagonal,
+   3 = kdn_*_fwd_save, 4 = kdn_*_bwd_saved; variant 0 = diagonal,
    1 = isotropic).  -1 for an invalid descriptor or op, or an op the descriptor
    does not serve.
    Calls with T = 0 launch at most one small fill kernel. */

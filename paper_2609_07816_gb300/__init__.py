@@ -65,6 +65,10 @@ _SIG = {
                                                                    ctypes.c_size_t, _P], ctypes.c_int),
     "kdn_diag_bwd_saved": ([ctypes.POINTER(kdn_desc_t)] + [_P] * 7 + [ctypes.c_size_t] + [_P] * 12
                            + [ctypes.c_size_t, _P], ctypes.c_int),
+    "kdn_iso_fwd_save": ([ctypes.POINTER(kdn_desc_t)] + [_P] * 12 + [ctypes.c_size_t, _P,
+                                                                  ctypes.c_size_t, _P], ctypes.c_int),
+    "kdn_iso_bwd_saved": ([ctypes.POINTER(kdn_desc_t)] + [_P] * 7 + [ctypes.c_size_t] + [_P] * 12
+                          + [ctypes.c_size_t, _P], ctypes.c_int),
     "kdn_kernel_launches": ([ctypes.POINTER(kdn_desc_t), ctypes.c_int, ctypes.c_int], ctypes.c_int),
     "kdn_get_device_status": ([_P, _P], ctypes.c_int),
 }
@@ -223,12 +227,9 @@ def saved_bytes(desc: kdn_desc_t, variant: int = 0) -> int:
     return int(lib().kdn_saved_bytes(ctypes.byref(desc), int(variant)))
 
 
-def kdn_diag_fwd_save(q, k, v, g, omega, r, S0=None, p0=None, *, mu=None, scale=None, o=None,
-                      ST=None, pT=None, saved=None, want_state=True, workspace=None, stream=None,
-                      out_dtype=torch.float32):
-    """Diagonal KDN forward that also keeps the chunked backward's context.
-    Returns (o, ST, pT, saved); pass `saved` to kdn_diag_bwd_saved."""
-    desc = _desc_from(0, q, v, g, chunk=0, mu=mu, scale=scale, out_dtype=out_dtype)
+def _fwd_save(name, variant, q, k, v, g, omega, r, S0, p0, *, mu, scale, o, ST, pT, saved,
+              want_state, workspace, stream, out_dtype):
+    desc = _desc_from(variant, q, v, g, chunk=0, mu=mu, scale=scale, out_dtype=out_dtype)
     B, T, H, dk = q.shape
     dv = v.shape[-1]
     dev = q.device
@@ -237,24 +238,41 @@ def kdn_diag_fwd_save(q, k, v, g, omega, r, S0=None, p0=None, *, mu=None, scale=
     if want_state and ST is None:
         ST = torch.empty(B, H, dk, dv, dtype=torch.float32, device=dev)
     if want_state and pT is None:
-        pT = torch.empty(B, H, dk, dtype=torch.float32, device=dev)
+        pT = torch.empty((B, H, dk) if variant == 0 else (B, H), dtype=torch.float32, device=dev)
     if saved is None:
-        saved = torch.empty(max(saved_bytes(desc), 256), dtype=torch.uint8, device=dev)
+        saved = torch.empty(max(saved_bytes(desc, variant), 256), dtype=torch.uint8, device=dev)
     if workspace is None:
-        workspace = alloc_workspace(desc, 0, False, dev)
-    st = lib().kdn_diag_fwd_save(ctypes.byref(desc), _ptr(q), _ptr(k), _ptr(v), _ptr(g),
-                                 _ptr(omega), _ptr(r), _ptr(S0), _ptr(p0), _ptr(o), _ptr(ST),
-                                 _ptr(pT), _ptr(saved), saved.numel(), _ptr(workspace),
-                                 workspace.numel(), _stream(stream))
-    _check(st, "kdn_diag_fwd_save")
+        workspace = alloc_workspace(desc, variant, False, dev)
+    st = getattr(lib(), name)(ctypes.byref(desc), _ptr(q), _ptr(k), _ptr(v), _ptr(g),
+                              _ptr(omega), _ptr(r), _ptr(S0), _ptr(p0), _ptr(o), _ptr(ST),
+                              _ptr(pT), _ptr(saved), saved.numel(), _ptr(workspace),
+                              workspace.numel(), _stream(stream))
+    _check(st, name)
     return o, ST, pT, saved
 
 
-def kdn_diag_bwd_saved(q, k, v, g, omega, r, saved, dO, dST=None, dpT=None, *, mu=None,
-                       scale=None, grads=None, want_state_grads=True, workspace=None, stream=None,
-                       out_dtype=torch.float32):
-    """Gradients of the Diagonal KDN forward from the context kept by kdn_diag_fwd_save."""
-    desc = _desc_from(0, q, v, g, chunk=0, mu=mu, scale=scale, out_dtype=out_dtype)
+def kdn_diag_fwd_save(q, k, v, g, omega, r, S0=None, p0=None, *, mu=None, scale=None, o=None,
+                      ST=None, pT=None, saved=None, want_state=True, workspace=None, stream=None,
+                      out_dtype=torch.float32):
+    """Diagonal KDN forward that also keeps the chunked backward's context.
+    Returns (o, ST, pT, saved); pass `saved` to kdn_diag_bwd_saved."""
+    return _fwd_save("kdn_diag_fwd_save", 0, q, k, v, g, omega, r, S0, p0, mu=mu, scale=scale,
+                     o=o, ST=ST, pT=pT, saved=saved, want_state=want_state, workspace=workspace,
+                     stream=stream, out_dtype=out_dtype)
+
+
+def kdn_iso_fwd_save(q, k, v, g, omega, r, S0=None, p0=None, *, mu=None, scale=None, o=None,
+                     ST=None, pT=None, saved=None, want_state=True, workspace=None, stream=None,
+                     out_dtype=torch.float32):
+    """Isotropic KDN forward that also keeps the chunked backward's context."""
+    return _fwd_save("kdn_iso_fwd_save", 1, q, k, v, g, omega, r, S0, p0, mu=mu, scale=scale,
+                     o=o, ST=ST, pT=pT, saved=saved, want_state=want_state, workspace=workspace,
+                     stream=stream, out_dtype=out_dtype)
+
+
+def _bwd_saved(name, variant, q, k, v, g, omega, r, saved, dO, dST, dpT, *, mu, scale, grads,
+               want_state_grads, workspace, stream, out_dtype):
+    desc = _desc_from(variant, q, v, g, chunk=0, mu=mu, scale=scale, out_dtype=out_dtype)
     B, T, H, dk = q.shape
     dv = v.shape[-1]
     dev = q.device
@@ -263,18 +281,37 @@ def kdn_diag_bwd_saved(q, k, v, g, omega, r, saved, dO, dST=None, dpT=None, *, m
                  (("dq", q), ("dk", k), ("dv", v), ("dg", g), ("domega", omega), ("dr", r))}
         if want_state_grads:
             grads["dS0"] = torch.empty(B, H, dk, dv, dtype=torch.float32, device=dev)
-            grads["dp0"] = torch.empty(B, H, dk, dtype=torch.float32, device=dev)
+            grads["dp0"] = torch.empty((B, H, dk) if variant == 0 else (B, H),
+                                       dtype=torch.float32, device=dev)
     if workspace is None:
-        workspace = alloc_workspace(desc, 0, False, dev)
+        workspace = alloc_workspace(desc, variant, False, dev)
     G = grads
-    st = lib().kdn_diag_bwd_saved(ctypes.byref(desc), _ptr(q), _ptr(k), _ptr(v), _ptr(g),
-                                  _ptr(omega), _ptr(r), _ptr(saved), saved.numel(), _ptr(dO),
-                                  _ptr(dST), _ptr(dpT), _ptr(G["dq"]), _ptr(G["dk"]),
-                                  _ptr(G["dv"]), _ptr(G["dg"]), _ptr(G["domega"]), _ptr(G["dr"]),
-                                  _ptr(G.get("dS0")), _ptr(G.get("dp0")), _ptr(workspace),
-                                  workspace.numel(), _stream(stream))
-    _check(st, "kdn_diag_bwd_saved")
+    st = getattr(lib(), name)(ctypes.byref(desc), _ptr(q), _ptr(k), _ptr(v), _ptr(g),
+                              _ptr(omega), _ptr(r), _ptr(saved), saved.numel(), _ptr(dO),
+                              _ptr(dST), _ptr(dpT), _ptr(G["dq"]), _ptr(G["dk"]),
+                              _ptr(G["dv"]), _ptr(G["dg"]), _ptr(G["domega"]), _ptr(G["dr"]),
+                              _ptr(G.get("dS0")), _ptr(G.get("dp0")), _ptr(workspace),
+                              workspace.numel(), _stream(stream))
+    _check(st, name)
     return grads
+
+
+def kdn_diag_bwd_saved(q, k, v, g, omega, r, saved, dO, dST=None, dpT=None, *, mu=None,
+                       scale=None, grads=None, want_state_grads=True, workspace=None, stream=None,
+                       out_dtype=torch.float32):
+    """Gradients of the Diagonal KDN forward from the context kept by kdn_diag_fwd_save."""
+    return _bwd_saved("kdn_diag_bwd_saved", 0, q, k, v, g, omega, r, saved, dO, dST, dpT, mu=mu,
+                      scale=scale, grads=grads, want_state_grads=want_state_grads,
+                      workspace=workspace, stream=stream, out_dtype=out_dtype)
+
+
+def kdn_iso_bwd_saved(q, k, v, g, omega, r, saved, dO, dST=None, dpT=None, *, mu=None,
+                      scale=None, grads=None, want_state_grads=True, workspace=None, stream=None,
+                      out_dtype=torch.float32):
+    """Gradients of the Isotropic KDN forward from the context kept by kdn_iso_fwd_save."""
+    return _bwd_saved("kdn_iso_bwd_saved", 1, q, k, v, g, omega, r, saved, dO, dST, dpT, mu=mu,
+                      scale=scale, grads=grads, want_state_grads=want_state_grads,
+                      workspace=workspace, stream=stream, out_dtype=out_dtype)
 
 
 def _decode(name, variant, q, k, v, g, omega, r, S, p, *, mu, scale, o, stream, out_dtype):

@@ -165,12 +165,12 @@ kdn_status_t bwd_entry(int variant, const kdn_desc_t *d, const void *q, const vo
 
 // Training pair: forward that keeps the fused backward's context in `saved`,
 // and the backward sweep that starts from it.
-kdn_status_t fwd_save_entry(const kdn_desc_t *d, const void *q, const void *k, const void *v,
+kdn_status_t fwd_save_entry(int variant, const kdn_desc_t *d, const void *q, const void *k, const void *v,
                             const void *g, const void *omega, const void *r, const float *S0,
                             const float *p0, void *o, float *ST, float *pT, void *saved,
                             size_t saved_bytes, void *ws, size_t ws_bytes, void *stream) {
   Args a;
-  kdn_status_t st = fill_sizes(d, 0, false, &a);
+  kdn_status_t st = fill_sizes(d, variant, false, &a);
   if (st != KDN_OK) return st;
   const bool work = (size_t)a.B * a.H * a.T > 0;
   if (work && !use_fused_bwd(a)) return KDN_ERR_UNSUPPORTED;
@@ -192,14 +192,14 @@ kdn_status_t fwd_save_entry(const kdn_desc_t *d, const void *q, const void *k, c
                           reinterpret_cast<float *>(static_cast<char *>(saved) + nsv), true);
 }
 
-kdn_status_t bwd_saved_entry(const kdn_desc_t *d, const void *q, const void *k, const void *v,
+kdn_status_t bwd_saved_entry(int variant, const kdn_desc_t *d, const void *q, const void *k, const void *v,
                              const void *g, const void *omega, const void *r, const void *saved,
                              size_t saved_bytes, const void *dO, const float *dST,
                              const float *dpT, void *dq, void *dk, void *dv, void *dg,
                              void *domega, void *dr, float *dS0, float *dp0, void *ws,
                              size_t ws_bytes, void *stream) {
   Args a;
-  kdn_status_t st = fill_sizes(d, 0, false, &a);
+  kdn_status_t st = fill_sizes(d, variant, false, &a);
   if (st != KDN_OK) return st;
   const bool work = (size_t)a.B * a.H * a.T > 0;
   if (work && !use_fused_bwd(a)) return KDN_ERR_UNSUPPORTED;
@@ -350,7 +350,7 @@ kdn_status_t kdn_iso_bwd(const kdn_desc_t *desc, const void *q, const void *k, c
 
 size_t kdn_saved_bytes(const kdn_desc_t *desc, int variant) {
   Args a;
-  if (variant != 0 || fill_sizes(desc, variant, false, &a) != KDN_OK) return 0;
+  if (fill_sizes(desc, variant, false, &a) != KDN_OK) return 0;
   return fused_saved_bytes(a);
 }
 
@@ -359,7 +359,7 @@ kdn_status_t kdn_diag_fwd_save(const kdn_desc_t *desc, const void *q, const void
                                const float *S0, const float *p0, void *o, float *ST, float *pT,
                                void *saved, size_t saved_bytes, void *workspace,
                                size_t workspace_bytes, void *stream) {
-  return fwd_save_entry(desc, q, k, v, g, omega, r, S0, p0, o, ST, pT, saved, saved_bytes,
+  return fwd_save_entry(0, desc, q, k, v, g, omega, r, S0, p0, o, ST, pT, saved, saved_bytes,
                         workspace, workspace_bytes, stream);
 }
 
@@ -369,7 +369,26 @@ kdn_status_t kdn_diag_bwd_saved(const kdn_desc_t *desc, const void *q, const voi
                                 const float *dST, const float *dpT, void *dq, void *dk, void *dv,
                                 void *dg, void *domega, void *dr, float *dS0, float *dp0,
                                 void *workspace, size_t workspace_bytes, void *stream) {
-  return bwd_saved_entry(desc, q, k, v, g, omega, r, saved, saved_bytes, dO, dST, dpT, dq, dk, dv,
+  return bwd_saved_entry(0, desc, q, k, v, g, omega, r, saved, saved_bytes, dO, dST, dpT, dq, dk, dv,
+                         dg, domega, dr, dS0, dp0, workspace, workspace_bytes, stream);
+}
+
+kdn_status_t kdn_iso_fwd_save(const kdn_desc_t *desc, const void *q, const void *k,
+                              const void *v, const void *g, const void *omega, const void *r,
+                              const float *S0, const float *p0, void *o, float *ST, float *pT,
+                              void *saved, size_t saved_bytes, void *workspace,
+                              size_t workspace_bytes, void *stream) {
+  return fwd_save_entry(1, desc, q, k, v, g, omega, r, S0, p0, o, ST, pT, saved, saved_bytes,
+                        workspace, workspace_bytes, stream);
+}
+
+kdn_status_t kdn_iso_bwd_saved(const kdn_desc_t *desc, const void *q, const void *k,
+                               const void *v, const void *g, const void *omega, const void *r,
+                               const void *saved, size_t saved_bytes, const void *dO,
+                               const float *dST, const float *dpT, void *dq, void *dk, void *dv,
+                               void *dg, void *domega, void *dr, float *dS0, float *dp0,
+                               void *workspace, size_t workspace_bytes, void *stream) {
+  return bwd_saved_entry(1, desc, q, k, v, g, omega, r, saved, saved_bytes, dO, dST, dpT, dq, dk, dv,
                          dg, domega, dr, dS0, dp0, workspace, workspace_bytes, stream);
 }
 
@@ -393,7 +412,7 @@ int kdn_kernel_launches(const kdn_desc_t *desc, int variant, int op) {
     case 1: return (a.T > 0 && use_fused_bwd(a)) ? 2 : chunked_bwd_launches(a);
     case 2: return 1;
     case 3:
-    case 4: return (variant == 0 && fused_saved_bytes(a) > 0) ? 1 : -1;
+    case 4: return fused_saved_bytes(a) > 0 ? 1 : -1;
   }
   return -1;
 }

@@ -174,11 +174,12 @@ def test_training_pair_validation(kdn):
     d = kdn.make_desc(B, T, H, 128, 128, kdn.KDN_BF16)
     n = kdn.saved_bytes(d)
     assert n == B * H * 3 * (149504 + 512)
-    assert kdn.saved_bytes(d, 1) == 0
+    assert kdn.saved_bytes(d, 1) == n
     assert kdn.saved_bytes(kdn.make_desc(B, T, H, 64, 128, kdn.KDN_BF16)) == 0
     assert kdn.saved_bytes(kdn.make_desc(B, T, H, 128, 128, kdn.KDN_F32)) == 0
     assert kdn.kdn_kernel_launches(d, 0, 3) == 1 and kdn.kdn_kernel_launches(d, 0, 4) == 1
-    assert kdn.kdn_kernel_launches(d, 1, 3) == -1
+    assert kdn.kdn_kernel_launches(d, 1, 3) == 1 and kdn.kdn_kernel_launches(d, 1, 4) == 1
+    assert kdn.kdn_kernel_launches(kdn.make_desc(B, T, H, 64, 128, kdn.KDN_BF16), 1, 3) == -1
 
     def fwd_save(desc, saved=FAKE, saved_bytes=1 << 40):
         return L.kdn_diag_fwd_save(ctypes.byref(desc), *([FAKE] * 11), saved, saved_bytes, FAKE,

@@ -336,3 +336,24 @@ def test_fused_decay_range_is_reported(kdn, variant):
     assert kdn.kdn_get_device_status(ws32) == kdn.KDN_OK
     ref = _oracle_fwd(variant, ins)
     check("o", o, ref["o"], "bf16")
+
+
+def test_isotropic_training_pair_matches_recompute_path(kdn):
+    """kdn_iso_fwd_save / kdn_iso_bwd_saved (scalar decay per head) against
+    kdn_iso_fwd / kdn_iso_bwd bit for bit, and against the oracle."""
+    ins = make_inputs("iso", 2, 150, 2, 128, 128, dtype="bf16", seed=53, s0_std=0.1,
+                      p0_range=(0.5, 2.0), per_channel_decay=False, with_grad=True)
+    d = to_dev(ins)
+    x = [d[n] for n in ("q", "k", "v", "g", "omega", "r")]
+    o1, ST1, pT1 = kdn.kdn_iso_fwd(*x, d["S0"], d["p0"])
+    o2, ST2, pT2, saved = kdn.kdn_iso_fwd_save(*x, d["S0"], d["p0"])
+    torch.cuda.synchronize()
+    assert torch.equal(o1, o2) and torch.equal(ST1, ST2) and torch.equal(pT1, pT2)
+    g1 = kdn.kdn_iso_bwd(*x, d["S0"], d["p0"], d["dO"])
+    g2 = kdn.kdn_iso_bwd_saved(*x, saved, d["dO"])
+    torch.cuda.synchronize()
+    ref = oracle.bwd("iso", *[ins[n] for n in ("q", "k", "v", "g", "omega", "r")], ins["S0"],
+                     ins["p0"], ins["dO"])
+    for n in ("dq", "dk", "dv", "dg", "domega", "dr", "dS0", "dp0"):
+        assert torch.equal(g1[n], g2[n]), n
+        check(n, g2[n], ref[n], "bf16")
