@@ -156,7 +156,14 @@ __device__ __forceinline__ float rs16(const float *v, int lane) {
   return w1 + __shfl_xor_sync(0xffffffffu, w1, 1);
 }
 
-template <int V>
+// Output store in the gradient dtype (OBF: bfloat16, else float32).
+template <int OBF>
+__device__ __forceinline__ void st_grad(void *p, size_t i, float x) {
+  if (OBF) static_cast<__nv_bfloat16 *>(p)[i] = __float2bfloat16_rn(x);
+  else static_cast<float *>(p)[i] = x;
+}
+
+template <int V, int OBF>
 __global__ void __launch_bounds__(BT, 1)
     k_fused_bwd(const __grid_constant__ CUtensorMap mq, const __grid_constant__ CUtensorMap mk,
                 const __grid_constant__ CUtensorMap mv, const __grid_constant__ CUtensorMap mdo,
@@ -607,7 +614,7 @@ __global__ void __launch_bounds__(BT, 1)
 #pragma unroll
       for (int u = 0; u < 16; ++u) {
         const int t = c * CM + tc0 + u;
-        if (t < a.T) sto(a.odt, a.dv_, tok_index(a, b, t, h) * D + j, v[u] * invl);
+        if (t < a.T) st_grad<OBF>(a.dv_, tok_index(a, b, t, h) * D + j, v[u] * invl);
       }
     }
     fence_proxy_async();
@@ -721,12 +728,7 @@ __global__ void __launch_bounds__(BT, 1)
       const size_t ostride = (size_t)a.H * D;
       const size_t obase = tok_index(a, b, c * CM + t0, h) * D + ci;
       const int nval = min(16, a.T - (c * CM + t0));
-      const bool obf = a.odt == KDN_BF16;
-      auto out = [&](void *p, int j, float x) {
-        const size_t idx = obase + (size_t)j * ostride;
-        if (obf) static_cast<__nv_bfloat16 *>(p)[idx] = __float2bfloat16_rn(x);
-        else static_cast<float *>(p)[idx] = x;
-      };
+      auto out = [&](void *p, int j, float x) { st_grad<OBF>(p, obase + (size_t)j * ostride, x); };
       // pass A: dq, dG, the ds_t partial sums and the ds-free parts of dphat and dk
       {
         float part[16], tot = 0.f;
@@ -848,7 +850,7 @@ __global__ void __launch_bounds__(BT, 1)
           const int tt = c * CM + tid;
           if (tt < a.T) {
             const float dr = s_ds[tid] + ((s_red2[tid] + s_red2[64 + tid]) + (s_red2[128 + tid] + s_red2[192 + tid]));
-            sto(a.odt, a.dr, tok_index(a, b, tt, h), dr * invl);
+            st_grad<OBF>(a.dr, tok_index(a, b, tt, h), dr * invl);
           }
         }
       }
@@ -872,12 +874,7 @@ __global__ void __launch_bounds__(BT, 1)
       const size_t ostride = (size_t)a.H * D;
       const size_t obase = tok_index(a, b, c * CM + t0, h) * D + ci;
       const int nval = min(16, a.T - (c * CM + t0));
-      const bool obf = a.odt == KDN_BF16;
-      auto out = [&](void *p, int j, float x) {
-        const size_t idx = obase + (size_t)j * ostride;
-        if (obf) static_cast<__nv_bfloat16 *>(p)[idx] = __float2bfloat16_rn(x);
-        else static_cast<float *>(p)[idx] = x;
-      };
+      auto out = [&](void *p, int j, float x) { st_grad<OBF>(p, obase + (size_t)j * ostride, x); };
       // pass A: dq, dG, the dbeta_t partial sums and dk from the memory path and kappa
       {
         float part[16], tot = 0.f;
@@ -943,8 +940,8 @@ __global__ void __launch_bounds__(BT, 1)
           s_da[t] = s_bp[t] * dbhat;
           if (tt < a.T) {
             const size_t th = tok_index(a, b, tt, h);
-            sto(a.odt, a.domega, th, dbhat * invl);
-            sto(a.odt, a.dr, th, (-__fdividef(dbeta * beta, dd) - du * u * ri) * invl);
+            st_grad<OBF>(a.domega, th, dbhat * invl);
+            st_grad<OBF>(a.dr, th, (-__fdividef(dbeta * beta, dd) - du * u * ri) * invl);
           }
           db = s_a[t] * dbhat;
         }
@@ -986,7 +983,7 @@ __global__ void __launch_bounds__(BT, 1)
               const float al = __expf(s_gs[tid]);
               const float dg = (s_red2[tid] + s_red2[64 + tid]) + (s_red2[128 + tid] + s_red2[192 + tid]) +
                                2.f * al * al * s_da[tid];
-              sto(a.odt, a.dg, tok_index(a, b, tt, h), dg * invl);
+              st_grad<OBF>(a.dg, tok_index(a, b, tt, h), dg * invl);
             }
           }
         }
@@ -1048,7 +1045,9 @@ kdn_status_t launch_fused_bwd_sweep(const Args &a, cudaStream_t s) {
   if (!make_map(&mq, a.q, a) || !make_map(&mk, a.k, a) || !make_map(&mv, a.v, a) ||
       !make_map(&mdo, a.dO, a))
     return KDN_ERR_CUDA;
-  auto kern = a.variant == 0 ? k_fused_bwd<0> : k_fused_bwd<1>;
+  const bool obf = a.odt == KDN_BF16;
+  auto kern = a.variant == 0 ? (obf ? k_fused_bwd<0, 1> : k_fused_bwd<0, 0>)
+                             : (obf ? k_fused_bwd<1, 1> : k_fused_bwd<1, 0>);
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES) !=
       cudaSuccess)
     return KDN_ERR_CUDA;
