@@ -299,6 +299,7 @@ def run_gpu(args):
     dec = run_decode(kdn, torch, hbm) if rank == 0 and not args.no_decode else None
     iso = run_iso_step(kdn, torch, args) if rank == 0 and not args.no_decode else None
     e2e = run_e2e(kdn, torch, x, ins, args) if rank == 0 and not args.no_e2e else None
+    lng = run_long_context(kdn, torch, args, hbm) if rank == 0 and not args.no_long else None
     out = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
@@ -313,7 +314,7 @@ def run_gpu(args):
         "spec_roofline_frac": spec_time / (ms_step / 1e3) if ms_step > 0 else None,
         "gpu_launches": launches_per_step * args.steps,
         "clocks": clk.summary(),
-        "decode": dec, "iso_step": iso, "e2e": e2e,
+        "decode": dec, "iso_step": iso, "e2e": e2e, "long_context": lng,
     }
     if rank == 0 and not args.no_cpu_baseline:
         out["cpu_baseline"] = cpu_baseline(sample_heads=args.cpu_heads)
@@ -351,6 +352,62 @@ def run_iso_step(kdn, torch, args):
     return {"workload": f"Isotropic KDN fwd+bwd, B={b} H={h} T={t} d=128, one decay per head",
             "value": b * t / (ms / 1e3), "unit": "tokens/s", "ms_per_step": ms,
             "gpu_launches": 2 * args.steps}
+
+
+def run_long_context(kdn, torch, args, hbm):
+    """Long-context forward, B=1 H=16 T=65536 d=128 (S_0 ~ N(0, 0.02^2), p_0 ~
+    U(0.5, 2)), both variants (iso: one decay per head): kdn_*_fwd with o, S_T
+    and p_T, tokens/s and the HBM roofline of the whole call.  With B*H = 16 the
+    call runs sequence-parallel (8 segments of 128 chunks)."""
+    b, t, h = 1, 65536, 16
+    res = {}
+    for variant in ("diag", "iso"):
+        pc = variant == "diag"
+        ins = device_inputs(variant, b, t, h, DK, DV, seed=11, dtype=torch.bfloat16,
+                            per_channel=pc, with_grad=False)
+        x = [ins[n] for n in NAMES]
+        gen = torch.Generator(device="cuda")
+        gen.manual_seed(12)
+        S0 = 0.02 * torch.randn(b, h, DK, DV, device="cuda", generator=gen)
+        pshape = (b, h, DK) if pc else (b, h)
+        p0 = 0.5 + 1.5 * torch.rand(pshape, device="cuda", generator=gen)
+        desc = kdn.make_desc(b, t, h, DK, DV, torch.bfloat16, decay_per_channel=int(pc))
+        vi = 0 if pc else 1
+        ws = kdn.alloc_workspace(desc, vi)
+        o = torch.empty(b, t, h, DV, dtype=torch.float32, device="cuda")
+        ST = torch.empty(b, h, DK, DV, dtype=torch.float32, device="cuda")
+        pT = torch.empty(pshape, dtype=torch.float32, device="cuda")
+        fn = kdn.kdn_diag_fwd if pc else kdn.kdn_iso_fwd
+
+        def call():
+            fn(*x, S0, p0, o=o, ST=ST, pT=pT, workspace=ws)
+
+        for _ in range(max(3, args.warmup)):
+            call()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        n = max(3, args.steps)
+        e0.record()
+        for _ in range(n):
+            call()
+        e1.record()
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1) / n
+        nb = fwd_bytes(b, t, h, DK, DV, with_state=True)
+        if not pc:  # one decay and one noise value per token-head
+            nb -= b * t * h * 2 * DK * 2 - b * t * h * 2 * 2
+        res[variant] = {
+            "workload": f"{'Diagonal' if pc else 'Isotropic'} KDN forward, B={b} H={h} T={t} "
+                        f"d=128, bf16 in, f32 o / state",
+            "value": b * t / (ms / 1e3), "unit": "tokens/s", "ms": ms,
+            "sequence_parallel": kdn.kdn_kernel_launches(desc, vi, 0) == 6,
+            "gpu_launches": kdn.kdn_kernel_launches(desc, vi, 0),
+            "roofline": {"bound": "hbm", "achieved": nb / (ms / 1e3) / 1e9, "peak": hbm,
+                         "unit": "GB/s", "frac": nb / (ms / 1e3) / 1e9 / hbm,
+                         "algorithmic_bytes": nb},
+        }
+        del ins, x, o, ws
+    return res
 
 
 def run_decode(kdn, torch, hbm):
@@ -535,6 +592,7 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-decode", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-long", action="store_true", help="skip the long-context forward")
     ap.add_argument("--fwd-only", action="store_true", help="profiling runs: forward only")
     ap.add_argument("--batch", type=int, default=B, help="batch size (profiling runs only)")
     ap.add_argument("--cpu-heads", type=int, default=None)

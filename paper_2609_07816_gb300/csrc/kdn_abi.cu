@@ -121,7 +121,9 @@ kdn_status_t fwd_entry(int variant, const kdn_desc_t *d, const void *q, const vo
   const bool work = (size_t)a.B * a.H * a.T > 0;
   if (work && !ptrs_ok({q, k, v, g, omega, r, o}, {S0, p0, ST, pT})) return KDN_ERR_INVALID_ARG;
   if (!work && !ptrs_ok({}, {S0, p0, ST, pT})) return KDN_ERR_INVALID_ARG;
-  const size_t need = workspace_layout(&a, nullptr, false);
+  const size_t base = workspace_layout(&a, nullptr, false);
+  const int nseg = seg_count(a);
+  const size_t need = base + (nseg > 1 ? seg_workspace_bytes(a, nseg) : 0);
   if (need > ws_bytes || (need && (!ws || ((uintptr_t)ws % kAlign)))) return KDN_ERR_WORKSPACE;
   workspace_layout(&a, static_cast<char *>(ws), false);
   a.q = q; a.k = k; a.v = v; a.g = g; a.omega = omega; a.r = r;
@@ -130,6 +132,7 @@ kdn_status_t fwd_entry(int variant, const kdn_desc_t *d, const void *q, const vo
   if (cudaMemsetAsync(a.status, 0, sizeof(unsigned), s) != cudaSuccess) return KDN_ERR_CUDA;
   if ((size_t)a.B * a.H == 0) return KDN_OK;
   if (a.T == 0) return empty_fwd(a, s);
+  if (nseg > 1) return launch_seg_fwd(a, nseg, static_cast<char *>(ws) + base, s);
   if (use_fused(a)) return launch_fused_fwd(a, s);
   return launch_chunked_fwd(a, s, false);
 }
@@ -303,7 +306,8 @@ const char *kdn_status_string(kdn_status_t s) {
 size_t kdn_fwd_workspace_bytes(const kdn_desc_t *desc, int variant) {
   Args a;
   if (fill_sizes(desc, variant, false, &a) != KDN_OK) return 0;
-  return workspace_layout(&a, nullptr, false);
+  const int nseg = seg_count(a);
+  return workspace_layout(&a, nullptr, false) + (nseg > 1 ? seg_workspace_bytes(a, nseg) : 0);
 }
 
 size_t kdn_bwd_workspace_bytes(const kdn_desc_t *desc, int variant) {
@@ -408,7 +412,7 @@ int kdn_kernel_launches(const kdn_desc_t *desc, int variant, int op) {
   Args a;
   if (fill_sizes(desc, variant, op == 2, &a) != KDN_OK) return -1;
   switch (op) {
-    case 0: return use_fused(a) ? 1 : chunked_fwd_launches(a);
+    case 0: return seg_count(a) > 1 ? 6 : use_fused(a) ? 1 : chunked_fwd_launches(a);
     case 1: return (a.T > 0 && use_fused_bwd(a)) ? 2 : chunked_bwd_launches(a);
     case 2: return 1;
     case 3:

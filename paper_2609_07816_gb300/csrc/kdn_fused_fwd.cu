@@ -72,6 +72,7 @@ struct FusedParams {
   int has_g_map;  // per-channel decay tile through TMA
   int has_w_map;  // per-channel omega tile through TMA (diag)
   int write_o;    // 0: the outputs o are not written (state-saving pass of the backward)
+  int s0_eye;     // 1: the initial memory is the identity (dk = dv); S0 is ignored
   unsigned char *save_S;  // optional [BH][NC] context records of the backward (kCtxBytes each)
   float *save_p;          // optional [BH][NC][128] uncertainty carry entering each chunk
 };
@@ -177,7 +178,7 @@ __global__ void __launch_bounds__(FT, 1)
         }
       } else {
 #pragma unroll
-        for (int u = 0; u < 16; ++u) v[u] = 0.f;
+        for (int u = 0; u < 16; ++u) v[u] = (P.s0_eye && i == j0 + u) ? 1.f : 0.f;
       }
       tmem_st16(TS + lane_base + j0, v);
     }
@@ -714,17 +715,27 @@ bool fused_fwd_supported(const Args &a) {
 int fused_fwd_smem_bytes() { return SMEM_BYTES; }
 
 kdn_status_t launch_fused_fwd(const Args &a, cudaStream_t s, unsigned char *save_S,
-                              float *save_p, bool write_o) {
+                              float *save_p, bool write_o, bool s0_eye, const void *v_zero) {
   FusedParams P;
   P.a = a;
   P.has_g_map = (a.variant == 0 || a.pcd) ? 1 : 0;
   P.has_w_map = a.variant == 0 ? 1 : 0;
   P.write_o = write_o ? 1 : 0;
+  P.s0_eye = s0_eye ? 1 : 0;
   P.save_S = save_S;
   P.save_p = save_p;
   CUtensorMap mq, mk, mv, mg, mw, mo;
-  if (!make_map(&mq, a.q, a) || !make_map(&mk, a.k, a) || !make_map(&mv, a.v, a))
+  if (!make_map(&mq, a.q, a) || !make_map(&mk, a.k, a)) return KDN_ERR_CUDA;
+  if (v_zero) {
+    // v = 0: a map over one zeroed 64-token block of a single sequence; every
+    // other chunk lies outside it and the TMA fills the tile with zeros.
+    Args az = a;
+    az.B = 1;
+    az.T = 64;
+    if (!make_map(&mv, v_zero, az)) return KDN_ERR_CUDA;
+  } else if (!make_map(&mv, a.v, a)) {
     return KDN_ERR_CUDA;
+  }
   if (P.write_o ? !make_map(&mo, a.o, a, a.odt != KDN_BF16) : !make_map(&mo, a.q, a))
     return KDN_ERR_CUDA;
   mg = mq;

@@ -100,9 +100,12 @@ size_t workspace_layout(Args *a, char *base, bool bwd);
 // `save_S` / `save_p` it also stores the context of the fused backward: the
 // fp16 image of every chunk's entry memory (32 KB) and the uncertainty entering
 // every chunk (128 floats); `write_o` = false skips the outputs o.
+// `s0_eye` starts every sequence from S = I (dk = dv) instead of a.S0; `v_zero`
+// (a zeroed device buffer of 64 * H * 128 bf16) replaces v by zeros.
 bool fused_fwd_supported(const Args &a);
 kdn_status_t launch_fused_fwd(const Args &a, cudaStream_t s, unsigned char *save_S = nullptr,
-                              float *save_p = nullptr, bool write_o = true);
+                              float *save_p = nullptr, bool write_o = true, bool s0_eye = false,
+                              const void *v_zero = nullptr);
 // Fused tcgen05 backward (Diagonal KDN, bf16, dk = dv = 128, 64-token chunks):
 // one reverse sweep per (batch, head) from the saved context in a.fSin / a.fpin.
 // launch_fused_bwd first runs the context-saving forward (without o).
@@ -114,6 +117,14 @@ kdn_status_t launch_fused_bwd_sweep(const Args &a, cudaStream_t s);
 // per chunk the 128 float32 uncertainties entering it.
 size_t fused_saved_bytes(const Args &a);
 size_t fused_ctx_record_bytes();
+
+// Sequence-parallel forward (kdn_segmented.cu): the number of segments P each
+// sequence is cut into (1: not used), the workspace it needs after the common
+// layout, and the launcher (gain summaries, scan, two fused runs per segment,
+// the state join and the final fused run).
+int seg_count(const Args &a);
+size_t seg_workspace_bytes(const Args &a, int P);
+kdn_status_t launch_seg_fwd(const Args &a, int P, char *ws, cudaStream_t s);
 
 // Launchers (each returns KDN_OK or KDN_ERR_CUDA).
 kdn_status_t launch_chunked_fwd(const Args &a, cudaStream_t s, bool save_states);

@@ -166,6 +166,42 @@ def test_fused_path_launches_and_workspace(kdn):
     assert kdn.kdn_kernel_launches(d32, 0, 1) > 2
 
 
+def _seg_bytes(B, T, H, P, variant):
+    r = lambda x: (x + 255) // 256 * 256
+    Pn = 128 if variant == 0 else 1
+    BH, NC = B * H, T // 64
+    return (r(BH * NC * Pn * 16) + 2 * r(BH * P * Pn * 4) + 3 * r(BH * P * 128 * 128 * 4)
+            + r(64 * H * 128 * 2))
+
+
+@pytest.mark.parametrize("B,T,H,P", [
+    (1, 65536, 16, 8),    # long context: 1024 chunks cut into 8 segments of 128
+    (1, 2048, 2, 4),      # 32 chunks: 4 segments of 8
+    (2, 2560, 1, 5),      # 40 chunks: 5 segments of 8
+    (1, 2304, 2, 4),      # 36 chunks: 4 segments of 9
+    (2, 4096, 1, 8),
+    (8, 4096, 16, 1),     # B*H = 128: already one CTA per SM, no segments
+    (1, 2047, 2, 1),      # T not a multiple of 64
+    (1, 1536, 2, 1),      # 24 chunks: too short for 4 segments of 8
+])
+def test_sequence_parallel_forward_selection(kdn, B, T, H, P):
+    """The plain bf16 d = 128 forward of few long sequences is cut into P
+    segments (the largest divisor of the chunk count with B*H*P <= 152 and
+    segments of at least 8 chunks, P >= 4): six launches and the segment
+    buffers after the status word; otherwise one fused launch."""
+    for variant in (0, 1):
+        d = kdn.make_desc(B, T, H, 128, 128, kdn.KDN_BF16)
+        if P > 1:
+            assert kdn.kdn_kernel_launches(d, variant, 0) == 6
+            assert kdn.workspace_bytes(d, variant) == 256 + _seg_bytes(B, T, H, P, variant)
+        else:
+            assert kdn.kdn_kernel_launches(d, variant, 0) == 1
+            assert kdn.workspace_bytes(d, variant) == 256
+        # the 32-token chunk keeps the general kernels
+        d32 = kdn.make_desc(B, T, H, 128, 128, kdn.KDN_BF16, chunk=32)
+        assert kdn.kdn_kernel_launches(d32, variant, 0) not in (1, 6)
+
+
 def test_training_pair_validation(kdn):
     """kdn_diag_fwd_save / kdn_diag_bwd_saved: served only for the fused shapes;
     the saved buffer is checked for size and alignment before anything runs."""

@@ -59,6 +59,50 @@ def test_forward_parity(kdn, case):
     check("pT", pT, ref["pT"], dt)
 
 
+SEG_CASES = [
+    # variant, per-channel decay, B, T, H, s0_std, p0_range, segments
+    ("diag", True, 1, 2048, 2, 0.02, (0.5, 2.0), 4),
+    ("diag", True, 2, 4096, 1, 0.0, None, 8),
+    ("diag", True, 1, 2304, 2, 0.3, (0.1, 2.0), 4),     # 9 chunks per segment
+    ("iso", False, 1, 2048, 2, 0.02, (0.5, 2.0), 4),
+    ("iso", True, 2, 2560, 1, 0.1, (0.1, 2.0), 5),
+]
+
+
+@pytest.mark.parametrize("case", SEG_CASES, ids=lambda c: "-".join(map(str, c[:5])))
+def test_sequence_parallel_forward_parity(kdn, case):
+    """Few long sequences: the forward cut into segments (gain summaries and
+    scan, a run from S = 0, a run from S = I with v = 0, the state join, the
+    final run) matches the token-by-token oracle on o, S_T and p_T."""
+    variant, pc, B, T, H, s0, p0r, nseg = case
+    ins = make_inputs(variant, B, T, H, 128, 128, dtype="bf16", seed=T + B, s0_std=s0,
+                      p0_range=p0r, per_channel_decay=pc)
+    d = kdn.make_desc(B, T, H, 128, 128, kdn.KDN_BF16, decay_per_channel=int(pc))
+    assert kdn.kdn_kernel_launches(d, 0 if variant == "diag" else 1, 0) == 6
+    ref = _oracle_fwd(variant, ins)
+    o, ST, pT = _gpu_fwd(kdn, variant, to_dev(ins))
+    torch.cuda.synchronize()
+    check("o", o, ref["o"], "bf16")
+    check("ST", ST, ref["ST"], "bf16")
+    check("pT", pT, ref["pT"], "bf16")
+    # the state hand-off at every segment boundary: o right after each boundary
+    step = T // nseg
+    for j in range(1, nseg):
+        t = j * step
+        check(f"o[t={t}]", o[:, t:t + 2], ref["o"][:, t:t + 2], "bf16")
+
+
+def test_sequence_parallel_forward_without_state_outputs(kdn):
+    """The segmented forward with ST / pT not requested writes the same o."""
+    ins = make_inputs("diag", 1, 2048, 2, 128, 128, dtype="bf16", seed=5, s0_std=0.02)
+    dev = to_dev(ins)
+    o1, _, _ = _gpu_fwd(kdn, "diag", dev)
+    o2, ST2, pT2 = _gpu_fwd(kdn, "diag", dev, want_state=False)
+    torch.cuda.synchronize()
+    assert ST2 is None and pT2 is None
+    assert torch.equal(o1, o2)
+
+
 @pytest.mark.parametrize("chunk", [0, 32, 64])
 def test_forward_chunk_argument_is_tuning_only(kdn, chunk):
     ins = make_inputs("diag", 1, 130, 2, 64, 64, dtype="f32", seed=3)
