@@ -104,7 +104,16 @@ const char *kdn_status_string(kdn_status_t status);
 /* Workspace (device scratch) bytes that kdn_*_fwd / kdn_*_bwd need for this
    descriptor; variant 0 = diagonal, 1 = isotropic.  Returns 0 for an invalid
    descriptor.  The workspace must be 256-byte aligned; its contents need no
-   initialisation and are clobbered by every call. */
+   initialisation and are clobbered by every call.
+   For bf16 inputs with d_k = d_v = 128 and few long sequences (B*H*P <= 152
+   for some P >= 4 that divides the T/64 chunks into segments of >= 8 chunks,
+   T a multiple of 64) the forward runs sequence-parallel: it cuts each
+   sequence into P segments, joined exactly (uncertainty by a scan of per-chunk
+   Moebius summaries, memory by the linearity of the chunk recurrence in
+   (S_in, v)), and kdn_fwd_workspace_bytes includes its segment buffers
+   (3 x 64 KB per (batch, head, segment) and 2 KB per (batch, head, chunk)).
+   A smaller workspace that still holds the single-pass layout (256 bytes)
+   runs the single pass. */
 size_t kdn_fwd_workspace_bytes(const kdn_desc_t *desc, int variant);
 size_t kdn_bwd_workspace_bytes(const kdn_desc_t *desc, int variant);
 
@@ -226,8 +235,9 @@ kdn_status_t kdn_iso_decode_step(const kdn_desc_t *desc, const void *q,
    and results are those of kdn_diag_fwd without the workspace pair.
    Scratch is a fixed array of KDN_NOALLOC_SCRATCH_BYTES in the library's
    device memory, held by every GPU that loads the library until exit; a
-   problem whose kdn_fwd_workspace_bytes() exceeds it is rejected with
-   KDN_ERR_WORKSPACE before anything runs.  The first call on a device looks
+   problem whose single-pass workspace exceeds it is rejected with
+   KDN_ERR_WORKSPACE before anything runs (the sequence-parallel forward is
+   used when its larger workspace fits the array, else the single pass).  The first call on a device looks
    up the array's device address (cudaGetSymbolAddress, with that device
    current); make it before any stream capture.  All calls on a device share
    the array, so calls that overlap on the GPU race and must be serialised by

@@ -122,7 +122,9 @@ kdn_status_t fwd_entry(int variant, const kdn_desc_t *d, const void *q, const vo
   if (work && !ptrs_ok({q, k, v, g, omega, r, o}, {S0, p0, ST, pT})) return KDN_ERR_INVALID_ARG;
   if (!work && !ptrs_ok({}, {S0, p0, ST, pT})) return KDN_ERR_INVALID_ARG;
   const size_t base = workspace_layout(&a, nullptr, false);
-  const int nseg = seg_count(a);
+  int nseg = seg_count(a);
+  // a workspace without room for the segment buffers runs the single pass
+  if (nseg > 1 && base + seg_workspace_bytes(a, nseg) > ws_bytes) nseg = 1;
   const size_t need = base + (nseg > 1 ? seg_workspace_bytes(a, nseg) : 0);
   if (need > ws_bytes || (need && (!ws || ((uintptr_t)ws % kAlign)))) return KDN_ERR_WORKSPACE;
   workspace_layout(&a, static_cast<char *>(ws), false);
@@ -242,6 +244,12 @@ kdn_status_t decode_entry(int variant, const kdn_desc_t *d, const void *q, const
 }
 
 }  // namespace
+
+size_t fwd_min_workspace_bytes(const kdn_desc_t *desc, int variant) {
+  Args a;
+  if (fill_sizes(desc, variant, false, &a) != KDN_OK) return 0;
+  return workspace_layout(&a, nullptr, false);
+}
 
 size_t workspace_layout(Args *a, char *base, bool bwd) {
   const size_t BH = (size_t)a->B * a->H, Tp = a->Tp, NC = a->NC, C = a->C;

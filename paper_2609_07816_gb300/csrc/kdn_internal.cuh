@@ -123,6 +123,9 @@ size_t fused_ctx_record_bytes();
 // layout, and the launcher (gain summaries, scan, two fused runs per segment,
 // the state join and the final fused run).
 int seg_count(const Args &a);
+// Smallest forward workspace for a descriptor (the single-pass layout; 0 for an
+// invalid descriptor); kdn_fwd_workspace_bytes adds the segment buffers.
+size_t fwd_min_workspace_bytes(const kdn_desc_t *desc, int variant);
 size_t seg_workspace_bytes(const Args &a, int P);
 kdn_status_t launch_seg_fwd(const Args &a, int P, char *ws, cudaStream_t s);
 

@@ -22,8 +22,7 @@
 // serialised by the caller.
 #include <mutex>
 
-#include "../../include/kdn.h"
-#include <cuda_runtime.h>
+#include "kdn_internal.cuh"
 
 namespace {
 
@@ -57,7 +56,9 @@ kdn_status_t kdn_diag_fwd_noalloc(const kdn_desc_t *desc, const void *q, const v
                                   const void *v, const void *g, const void *omega,
                                   const void *r, const float *S0, const float *p0, void *o,
                                   float *ST, float *pT, void *stream) {
-  const size_t need = kdn_fwd_workspace_bytes(desc, 0);
+  // the single-pass layout must fit; the sequence-parallel buffers are used
+  // when they fit as well (the regular entry point decides)
+  const size_t need = kdn::fwd_min_workspace_bytes(desc, 0);
   if (need == 0)  // invalid descriptor: let the regular entry point name the error
     return kdn_diag_fwd(desc, q, k, v, g, omega, r, S0, p0, o, ST, pT, nullptr, 0, stream);
   if (need > kScratchBytes) return KDN_ERR_WORKSPACE;  // problem too large for the array

@@ -46,7 +46,8 @@ def _noalloc(kdn, d, o, ST, pT):
 
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
 def test_noalloc_matches_workspace_entry_point_twice(kdn, dtype):
-    shapes = [(2, 150, 2, 128, 128, 3), (1, 97, 3, 64, 32, 4)]  # two different problems
+    # two different problems, then (bf16) one served by the sequence-parallel forward
+    shapes = [(2, 150, 2, 128, 128, 3), (1, 97, 3, 64, 32, 4), (1, 2048, 2, 128, 128, 5)]
     for B, T, H, dk, dv, seed in shapes:
         ins = make_inputs("diag", B, T, H, dk, dv, dtype=dtype, seed=seed, s0_std=0.05,
                           p0_range=(0.5, 2.0))
