@@ -296,7 +296,8 @@ def run_gpu(args):
     # the paper-style roofline: max(FLOPs / 2.25 PF, bytes / 8 TB/s)
     spec_time = max(B * T * H * chunk_flops(DK, DV) * 3.5 / 2.25e15, (fb + bb) / 8e12)
 
-    dec = run_decode(kdn, torch, hbm) if rank == 0 and not args.no_decode else None
+    dec = (run_decode(kdn, torch, hbm, args.decode_steps)
+           if rank == 0 and not args.no_decode else None)
     iso = run_iso_step(kdn, torch, args) if rank == 0 and not args.no_decode else None
     e2e = run_e2e(kdn, torch, x, ins, args) if rank == 0 and not args.no_e2e else None
     lng = run_long_context(kdn, torch, args, hbm) if rank == 0 and not args.no_long else None
@@ -410,8 +411,10 @@ def run_long_context(kdn, torch, args, hbm):
     return res
 
 
-def run_decode(kdn, torch, hbm):
-    """1024 consecutive decode tokens for B=256, H=16 in one CUDA graph, both variants."""
+def run_decode(kdn, torch, hbm, steps=DEC_STEPS):
+    """1024 consecutive decode tokens for B=256, H=16 in one CUDA graph, both variants
+    (`steps` fewer for profiling runs)."""
+    DEC_STEPS = steps
     res = {}
     for variant in ("diag", "iso"):
         gen = torch.Generator(device="cuda")
@@ -459,7 +462,7 @@ def run_decode(kdn, torch, hbm):
                         "achieved_GBs": by / (per / 1e3) / 1e9, "frac_hbm": by / (per / 1e3) / 1e9 / hbm,
                         "gpu_launches": DEC_STEPS}
         del graph
-    return {"metric": "decode steps/s (B=256, H=16, d=128, 1024 steps, CUDA graph)",
+    return {"metric": f"decode steps/s (B=256, H=16, d=128, {DEC_STEPS} steps, CUDA graph)",
             "value": res["diag"]["steps_per_s"], "unit": "steps/s", **res}
 
 
@@ -593,6 +596,8 @@ def main():
     ap.add_argument("--no-decode", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-long", action="store_true", help="skip the long-context forward")
+    ap.add_argument("--decode-steps", type=int, default=DEC_STEPS,
+                    help="decode tokens per graph (profiling runs only)")
     ap.add_argument("--fwd-only", action="store_true", help="profiling runs: forward only")
     ap.add_argument("--batch", type=int, default=B, help="batch size (profiling runs only)")
     ap.add_argument("--cpu-heads", type=int, default=None)
