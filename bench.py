@@ -298,7 +298,7 @@ def run_gpu(args):
 
     dec = (run_decode(kdn, torch, hbm, args.decode_steps)
            if rank == 0 and not args.no_decode else None)
-    iso = run_iso_step(kdn, torch, args) if rank == 0 and not args.no_decode else None
+    iso = run_iso_step(kdn, torch, args, hbm) if rank == 0 and not args.no_decode else None
     e2e = run_e2e(kdn, torch, x, ins, args) if rank == 0 and not args.no_e2e else None
     lng = run_long_context(kdn, torch, args, hbm) if rank == 0 and not args.no_long else None
     out = {
@@ -326,9 +326,10 @@ def run_gpu(args):
         dist.destroy_process_group()
 
 
-def run_iso_step(kdn, torch, args):
-    """The Isotropic KDN training step on its 750M-layer shape (B=8, H=12, T=2048,
-    d=128, one decay per head): kdn_iso_fwd_save + kdn_iso_bwd_saved, tokens/s."""
+def run_iso_step(kdn, torch, args, hbm):
+    """The Isotropic KDN on its 750M-layer shape (B=8, H=12, T=2048, d=128, one
+    decay per head): the training step kdn_iso_fwd_save + kdn_iso_bwd_saved, and
+    the inference forward kdn_iso_fwd alone, tokens/s."""
     b, t, h = 8, 2048, 12
     ins = device_inputs("iso", b, t, h, DK, DV, seed=7, dtype=torch.bfloat16, per_channel=False)
     x = [ins[n] for n in NAMES]
@@ -350,9 +351,32 @@ def run_iso_step(kdn, torch, args):
     e1.record()
     torch.cuda.synchronize()
     ms = e0.elapsed_time(e1) / args.steps
+    # the inference forward alone (o, S_T, b_T) through kdn_iso_fwd
+    o = torch.empty(b, t, h, DV, dtype=torch.float32, device="cuda")
+    ST = torch.empty(b, h, DK, DV, dtype=torch.float32, device="cuda")
+    bT = torch.empty(b, h, dtype=torch.float32, device="cuda")
+
+    def fwd():
+        kdn.kdn_iso_fwd(*x, o=o, ST=ST, pT=bT, workspace=ws)
+
+    for _ in range(args.warmup):
+        fwd()
+    torch.cuda.synchronize()
+    e0.record()
+    for _ in range(args.steps):
+        fwd()
+    e1.record()
+    torch.cuda.synchronize()
+    fms = e0.elapsed_time(e1) / args.steps
+    nb = fwd_bytes(b, t, h, DK, DV) - b * t * h * (2 * DK * 2 - 2 * 2)  # one g, omega per token
     return {"workload": f"Isotropic KDN fwd+bwd, B={b} H={h} T={t} d=128, one decay per head",
             "value": b * t / (ms / 1e3), "unit": "tokens/s", "ms_per_step": ms,
-            "gpu_launches": 2 * args.steps}
+            "gpu_launches": 2 * args.steps,
+            "forward": {"value": b * t / (fms / 1e3), "unit": "tokens/s", "ms": fms,
+                        "roofline": {"bound": "hbm", "achieved": nb / (fms / 1e3) / 1e9,
+                                     "peak": hbm, "unit": "GB/s",
+                                     "frac": nb / (fms / 1e3) / 1e9 / hbm,
+                                     "algorithmic_bytes": nb}}}
 
 
 def run_long_context(kdn, torch, args, hbm):
