@@ -99,6 +99,60 @@ __device__ __forceinline__ void check_gamma_range(float gC, unsigned *status) {
 // Row stride (floats) of the fp32 T and A tiles: 16-byte rows, conflict-free.
 constexpr int LT = 68;
 
+// Level L (= I - J) of the blocked inverse below: one thread per (block J, row,
+// 4 columns), float4 operands; X_IJ = sum_{K=J}^{I-1} T_IK A_KJ, then A_IJ = -D_I X_IJ.
+template <int L>
+__device__ __forceinline__ void tri_inverse_level(const float *sT, float *sA, float *sX) {
+  constexpr int nb = 4 - L;
+  const int tid = threadIdx.x;
+  const int J = tid >> 6, rr = (tid >> 2) & 15, cg = tid & 3, I = J + L;
+  if (J < nb) {
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int k = 0; k < L; ++k) {
+      const int K = J + k;
+      const float *tr = sT + (16 * I + rr) * LT + 16 * K;
+      const float *ac = sA + (16 * K) * LT + 16 * J + 4 * cg;
+#pragma unroll
+      for (int m4 = 0; m4 < 4; ++m4) {
+        const float4 t4 = *reinterpret_cast<const float4 *>(tr + 4 * m4);
+        const float tv[4] = {t4.x, t4.y, t4.z, t4.w};
+#pragma unroll
+        for (int mm = 0; mm < 4; ++mm) {
+          const float4 a4 = *reinterpret_cast<const float4 *>(ac + (4 * m4 + mm) * LT);
+          acc.x += tv[mm] * a4.x;
+          acc.y += tv[mm] * a4.y;
+          acc.z += tv[mm] * a4.z;
+          acc.w += tv[mm] * a4.w;
+        }
+      }
+    }
+    *reinterpret_cast<float4 *>(sX + J * 256 + rr * 16 + 4 * cg) = acc;
+  }
+  __syncthreads();
+  if (J < nb) {
+    const float *dr = sA + (16 * I + rr) * LT + 16 * I;
+    const float *xc = sX + J * 256 + 4 * cg;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int m4 = 0; m4 < 4; ++m4) {
+      const float4 d4 = *reinterpret_cast<const float4 *>(dr + 4 * m4);
+      const float dv[4] = {d4.x, d4.y, d4.z, d4.w};
+#pragma unroll
+      for (int mm = 0; mm < 4; ++mm) {
+        const float4 x4 = *reinterpret_cast<const float4 *>(xc + (4 * m4 + mm) * 16);
+        acc.x += dv[mm] * x4.x;
+        acc.y += dv[mm] * x4.y;
+        acc.z += dv[mm] * x4.z;
+        acc.w += dv[mm] * x4.w;
+      }
+    }
+    *reinterpret_cast<float4 *>(sA + (16 * I + rr) * LT + 16 * J + 4 * cg) =
+        make_float4(-acc.x, -acc.y, -acc.z, -acc.w);
+  }
+  __syncthreads();
+}
+
 // A = (I + T)^-1 for a strictly lower triangular 64 x 64 fp32 T (row stride
 // LT, zero on and above the diagonal), by 16 x 16 blocks, with 512 threads:
 // diagonal blocks D_I = (I + T_II)^-1 by column substitution (rows across a
@@ -131,56 +185,11 @@ __device__ __forceinline__ void tri_inverse64(const float *sT, float *sA, float 
     sA[(o0 + rr) * LT + o0 + cl + 1] = x1;
   }
   __syncthreads();
-  // off-diagonal levels: one thread per (block J, row, 4 columns), float4 operands
-  for (int L = 1; L < 4; ++L) {
-    const int nb = 4 - L;
-    const int J = tid >> 6, rr = (tid >> 2) & 15, cg = tid & 3, I = J + L;
-    if (J < nb) {
-      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-      for (int K = J; K < I; ++K) {
-        const float *tr = sT + (16 * I + rr) * LT + 16 * K;
-        const float *ac = sA + (16 * K) * LT + 16 * J + 4 * cg;
-#pragma unroll
-        for (int m4 = 0; m4 < 4; ++m4) {
-          const float4 t4 = *reinterpret_cast<const float4 *>(tr + 4 * m4);
-          const float tv[4] = {t4.x, t4.y, t4.z, t4.w};
-#pragma unroll
-          for (int mm = 0; mm < 4; ++mm) {
-            const float4 a4 = *reinterpret_cast<const float4 *>(ac + (4 * m4 + mm) * LT);
-            acc.x += tv[mm] * a4.x;
-            acc.y += tv[mm] * a4.y;
-            acc.z += tv[mm] * a4.z;
-            acc.w += tv[mm] * a4.w;
-          }
-        }
-      }
-      *reinterpret_cast<float4 *>(sX + J * 256 + rr * 16 + 4 * cg) = acc;
-    }
-    __syncthreads();
-    if (J < nb) {
-      const float *dr = sA + (16 * I + rr) * LT + 16 * I;
-      const float *xc = sX + J * 256 + 4 * cg;
-      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-      for (int m4 = 0; m4 < 4; ++m4) {
-        const float4 d4 = *reinterpret_cast<const float4 *>(dr + 4 * m4);
-        const float dv[4] = {d4.x, d4.y, d4.z, d4.w};
-#pragma unroll
-        for (int mm = 0; mm < 4; ++mm) {
-          const float4 x4 = *reinterpret_cast<const float4 *>(xc + (4 * m4 + mm) * 16);
-          acc.x += dv[mm] * x4.x;
-          acc.y += dv[mm] * x4.y;
-          acc.z += dv[mm] * x4.z;
-          acc.w += dv[mm] * x4.w;
-        }
-      }
-      *reinterpret_cast<float4 *>(sA + (16 * I + rr) * LT + 16 * J + 4 * cg) =
-          make_float4(-acc.x, -acc.y, -acc.z, -acc.w);
-    }
-    __syncthreads();
-  }
+  // off-diagonal levels, each with its K sum fully unrolled
+  tri_inverse_level<1>(sT, sA, sX);
+  tri_inverse_level<2>(sT, sA, sX);
+  tri_inverse_level<3>(sT, sA, sX);
 }
-
 
 inline PFN_cuTensorMapEncodeTiled_v12000 encoder() {
   static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
