@@ -460,8 +460,20 @@ __global__ void __launch_bounds__(FT, 1)
       }
       umma_commit(bar_mma);
     }
+    // V -> fp16 in place while MMA-T runs (the tile arrived during the previous chunk);
+    // on a timeout the MMA is still waited for before leaving
+    const bool v_ok = __syncthreads_and(mbar_wait(bar_v, c & 1, kWaitIters));
+    if (v_ok) {
+      for (int e = tid; e < 64 * 16; e += FT) {
+        const uint32_t off = (e >> 9) * 8192 + chunk_off((e >> 3) & 63, e & 7);  // slab, row, chunk
+        float v[8];
+        unpack_bf8(sm16(vr, off), v);
+        sm16(vr, off) = pack_h8(v);
+      }
+    }
     if (tid == 0 && P.save_S) bulk_wait_read();  // phat / gamma have left b3 / fs
-    if (!(ok = mma_wait())) break;
+    ok = mma_wait() && v_ok;
+    if (!ok) break;
     tc_fence_after();
     // ---- [5] T -> fp32 smem, A = (I + T)^-1 by 16x16 blocks:
     //   diagonal blocks D_I = (I + T_II)^-1 by column substitution (rows across a half-warp),
@@ -493,14 +505,6 @@ __global__ void __launch_bounds__(FT, 1)
       sm16(a2, chunk_off(r, cc)) = pack_bf8(v);
       sm16(af, chunk_off(r, cc)) = pack_h8(v);  // [A; 0] fp16 for MMA-U (over the dead T tile)
     }
-    ok = __syncthreads_and(mbar_wait(bar_v, c & 1, kWaitIters));
-    if (!ok) break;
-    for (int e = tid; e < 64 * 16; e += FT) {  // V -> fp16 in place
-      const uint32_t off = (e >> 9) * 8192 + chunk_off((e >> 3) & 63, e & 7);  // slab, row, chunk
-      float v[8];
-      unpack_bf8(sm16(vr, off), v);
-      sm16(vr, off) = pack_h8(v);
-    }
     fence_proxy_async();
     tc_fence_before();
     __syncthreads();
@@ -516,37 +520,11 @@ __global__ void __launch_bounds__(FT, 1)
       }
       umma_commit(bar_mma);
     }
-    if (!(ok = mma_wait())) break;
     tc_fence_after();
-    if (tid == 0 && P.save_S) {  // A fp16 [t][s] into the backward context
-      bulk_s2g(ctx + kCtxA, af, 8192);
-      bulk_commit();
-    }
-    // ---- [7] fp16 operands of the state products:
-    //   a1l rows 0..63 <- -W, rows 64..127 <- Qbar;  a2 <- [0; A_qk];
-    //   b3 <- S_in (and diag(gamma_C) S_in back to TMEM);  b1l <- K_tail
-    if (wq < 2) {
-      const int r = 32 * wq + lane;
-      for (int c0 = 0; c0 < 32; c0 += 16) {
-        float v[16];
-        const int j0 = 32 * wg + c0, sl = j0 >> 6, cc0 = (j0 & 63) >> 3;
-        tmem_ld16(TW + lane_base + j0, v);
-#pragma unroll
-        for (int u = 0; u < 16; ++u) v[u] = -v[u];
-        sm16(a1l, sl * 16384 + chunk_off(r, cc0)) = pack_h8(v);
-        sm16(a1l, sl * 16384 + chunk_off(r, cc0 + 1)) = pack_h8(v + 8);
-      }
-      for (int cc = 2 * wg; cc < 2 * wg + 2; ++cc) sm16(a2, chunk_off(r, cc)) = make_uint4(0, 0, 0, 0);
-    } else {
-      const int r = 32 * wq + lane - 64, s0 = 16 * wg;
-      float v[16];
-      tmem_ld16(TD1 + lane_base + s0, v);
-#pragma unroll
-      for (int u = 0; u < 16; ++u)
-        if (s0 + u > r) v[u] = 0.f;
-      sm16(a2, chunk_off(64 + r, s0 >> 3)) = pack_h8(v);
-      sm16(a2, chunk_off(64 + r, (s0 >> 3) + 1)) = pack_h8(v + 8);
-    }
+    // While MMA-W/U run, the state operands that depend on neither W nor U
+    // (MMA-T has finished reading their buffers; MMA-W/U read a2, kq rows 0..63,
+    // af and vr):  b3 <- S_in fp16 and diag(gamma_C) S_in back to TMEM;
+    // a1l rows 64..127 <- Qbar fp16;  b1l <- K_tail fp16
     {
       const int i = 32 * wq + lane;
       const float gC = s_gC[i];
@@ -577,6 +555,36 @@ __global__ void __launch_bounds__(FT, 1)
       sm16(b1l, o8) = pack_h8(hv);
     }
     tmem_st_wait();
+    if (!(ok = mma_wait())) break;
+    tc_fence_after();
+    if (tid == 0 && P.save_S) {  // A fp16 [t][s] into the backward context
+      bulk_s2g(ctx + kCtxA, af, 8192);
+      bulk_commit();
+    }
+    // ---- [7] the remaining fp16 operands of the state products:
+    //   a1l rows 0..63 <- -W;  a2 <- [0; A_qk]  (a2 held [A; 0] for MMA-W)
+    if (wq < 2) {
+      const int r = 32 * wq + lane;
+      for (int c0 = 0; c0 < 32; c0 += 16) {
+        float v[16];
+        const int j0 = 32 * wg + c0, sl = j0 >> 6, cc0 = (j0 & 63) >> 3;
+        tmem_ld16(TW + lane_base + j0, v);
+#pragma unroll
+        for (int u = 0; u < 16; ++u) v[u] = -v[u];
+        sm16(a1l, sl * 16384 + chunk_off(r, cc0)) = pack_h8(v);
+        sm16(a1l, sl * 16384 + chunk_off(r, cc0 + 1)) = pack_h8(v + 8);
+      }
+      for (int cc = 2 * wg; cc < 2 * wg + 2; ++cc) sm16(a2, chunk_off(r, cc)) = make_uint4(0, 0, 0, 0);
+    } else {
+      const int r = 32 * wq + lane - 64, s0 = 16 * wg;
+      float v[16];
+      tmem_ld16(TD1 + lane_base + s0, v);
+#pragma unroll
+      for (int u = 0; u < 16; ++u)
+        if (s0 + u > r) v[u] = 0.f;
+      sm16(a2, chunk_off(64 + r, s0 >> 3)) = pack_h8(v);
+      sm16(a2, chunk_off(64 + r, (s0 >> 3) + 1)) = pack_h8(v + 8);
+    }
     fence_proxy_async();
     tc_fence_before();
     __syncthreads();
