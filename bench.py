@@ -75,7 +75,7 @@ def decode_bytes(b, h, dk, dv, in_bytes=2, out_bytes=4):
 # DRAM bytes per launch of each kernel at the bench workload, from one ncu
 # capture (dram__bytes_read.sum + dram__bytes_write.sum) of the current build;
 # reported as `traffic` only for that workload.
-NCU_TRAFFIC = {"k_fused_fwd": None, "k_fused_bwd": 1883722496 + 1344765952}
+NCU_TRAFFIC = {"k_fused_fwd": 672730624 + 1443745536, "k_fused_bwd": 1883973632 + 1345471232}
 
 
 def chunk_flops(dk, dv, C=64):
