@@ -301,6 +301,8 @@ def run_gpu(args):
     iso = run_iso_step(kdn, torch, args, hbm) if rank == 0 and not args.no_decode else None
     e2e = run_e2e(kdn, torch, x, ins, args) if rank == 0 and not args.no_e2e else None
     lng = run_long_context(kdn, torch, args, hbm) if rank == 0 and not args.no_long else None
+    lgt = (run_logit_step(kdn, torch, args, x, o, saved, grads, ws_f, ws_b, ins["dO"])
+           if rank == 0 and not args.no_decode else None)
     out = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
@@ -315,7 +317,7 @@ def run_gpu(args):
         "spec_roofline_frac": spec_time / (ms_step / 1e3) if ms_step > 0 else None,
         "gpu_launches": launches_per_step * args.steps,
         "clocks": clk.summary(),
-        "decode": dec, "iso_step": iso, "e2e": e2e, "long_context": lng,
+        "decode": dec, "iso_step": iso, "e2e": e2e, "long_context": lng, "logit_gates": lgt,
     }
     if rank == 0 and not args.no_cpu_baseline:
         out["cpu_baseline"] = cpu_baseline(sample_heads=args.cpu_heads)
@@ -329,7 +331,8 @@ def run_gpu(args):
 def run_iso_step(kdn, torch, args, hbm):
     """The Isotropic KDN on its 750M-layer shape (B=8, H=12, T=2048, d=128, one
     decay per head): the training step kdn_iso_fwd_save + kdn_iso_bwd_saved, and
-    the inference forward kdn_iso_fwd alone, tokens/s."""
+    the inference forward kdn_iso_fwd alone, tokens/s; then both again with one
+    decay per channel (the paper's layer)."""
     b, t, h = 8, 2048, 12
     ins = device_inputs("iso", b, t, h, DK, DV, seed=7, dtype=torch.bfloat16, per_channel=False)
     x = [ins[n] for n in NAMES]
@@ -369,6 +372,32 @@ def run_iso_step(kdn, torch, args, hbm):
     torch.cuda.synchronize()
     fms = e0.elapsed_time(e1) / args.steps
     nb = fwd_bytes(b, t, h, DK, DV) - b * t * h * (2 * DK * 2 - 2 * 2)  # one g, omega per token
+    # the paper's layer: one decay per channel (alpha_t in R^dk), same shape, both calls
+    pins = device_inputs("iso", b, t, h, DK, DV, seed=8, dtype=torch.bfloat16, per_channel=True)
+    px = [pins[n] for n in NAMES]
+    pdesc = kdn.make_desc(b, t, h, DK, DV, torch.bfloat16, decay_per_channel=1)
+    psaved = torch.empty(kdn.saved_bytes(pdesc, 1), dtype=torch.uint8, device="cuda")
+
+    def pstep():
+        kdn.kdn_iso_fwd_save(*px, saved=psaved, want_state=False, workspace=ws)
+        kdn.kdn_iso_bwd_saved(*px, psaved, pins["dO"], want_state_grads=False, workspace=ws)
+
+    def pfwd():
+        kdn.kdn_iso_fwd(*px, o=o, ST=ST, pT=bT, workspace=ws)
+
+    res_pc = {}
+    for name, fn in (("step", pstep), ("forward", pfwd)):
+        for _ in range(args.warmup):
+            fn()
+        torch.cuda.synchronize()
+        e0.record()
+        for _ in range(args.steps):
+            fn()
+        e1.record()
+        torch.cuda.synchronize()
+        res_pc[name + "_ms"] = e0.elapsed_time(e1) / args.steps
+    nb_pc = fwd_bytes(b, t, h, DK, DV) - b * t * h * (DK * 2 - 2)  # g per channel, one omega
+    del pins, px, psaved
     return {"workload": f"Isotropic KDN fwd+bwd, B={b} H={h} T={t} d=128, one decay per head",
             "value": b * t / (ms / 1e3), "unit": "tokens/s", "ms_per_step": ms,
             "gpu_launches": 2 * args.steps,
@@ -376,7 +405,44 @@ def run_iso_step(kdn, torch, args, hbm):
                         "roofline": {"bound": "hbm", "achieved": nb / (fms / 1e3) / 1e9,
                                      "peak": hbm, "unit": "GB/s",
                                      "frac": nb / (fms / 1e3) / 1e9 / hbm,
-                                     "algorithmic_bytes": nb}}}
+                                     "algorithmic_bytes": nb}},
+            "per_channel_decay": {
+                "workload": f"Isotropic KDN, B={b} H={h} T={t} d=128, one decay per channel",
+                "step_value": b * t / (res_pc["step_ms"] / 1e3), "step_ms": res_pc["step_ms"],
+                "forward_value": b * t / (res_pc["forward_ms"] / 1e3),
+                "forward_ms": res_pc["forward_ms"], "unit": "tokens/s",
+                "forward_roofline_frac": nb_pc / (res_pc["forward_ms"] / 1e3) / 1e9 / hbm}}
+
+
+def run_logit_step(kdn, torch, args, x, o, saved, grads, ws_f, ws_b, dO):
+    """The bench step with the gates given as logits (KDN_GATES_LOGITS: sigmoid,
+    softplus and r_min + softplus applied inside the kernels, logit gradients out):
+    same shape, x ~ N(2, 1), y, z ~ N(0, 1)."""
+    gen = torch.Generator(device="cuda")
+    gen.manual_seed(5)
+    lg = [t for t in x]
+    for idx, mean in ((3, 2.0), (4, 0.0), (5, 0.0)):
+        lg[idx] = (torch.randn(x[idx].shape, device="cuda", generator=gen) + mean).to(x[idx].dtype)
+    kw = dict(gates=kdn.KDN_GATES_LOGITS, r_min=0.01)
+
+    def step():
+        kdn.kdn_diag_fwd_save(*lg, o=o, want_state=False, saved=saved, workspace=ws_f, **kw)
+        kdn.kdn_diag_bwd_saved(*lg, saved, dO, grads=grads, want_state_grads=False,
+                               workspace=ws_b, **kw)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(args.steps):
+        step()
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / args.steps
+    return {"workload": f"Diagonal KDN fwd+bwd with logit gates, B={B} H={H} T={T} d=128",
+            "value": B * T / (ms / 1e3), "unit": "tokens/s", "ms_per_step": ms,
+            "gpu_launches": 2 * args.steps}
 
 
 def run_long_context(kdn, torch, args, hbm):

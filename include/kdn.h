@@ -93,7 +93,18 @@ typedef struct {
                             0 (KDN_F32, the zero-initialised default) keeps the
                             float32 accumulators; KDN_BF16 rounds them once on
                             store. */
+  int gates;             /* kdn_gates_t: what g, omega and r hold (below) */
+  float r_min;           /* observation-noise floor of KDN_GATES_LOGITS (>= 0) */
 } kdn_desc_t;
+
+/* The gate inputs.  KDN_GATES_POST (0, the zero-initialised default): g = log
+   alpha <= 0, omega > 0 and r > 0 as the recurrence uses them.  KDN_GATES_LOGITS:
+   g, omega and r are the pre-activation values x, y, z of the layer's
+   parameterisation (eq. kla-box-parameterization; r_min of Sec. 5):
+   alpha = sigmoid(x), omega = softplus(y), r = r_min + softplus(z), applied
+   in float32 inside the kernels.  The backward then returns the gradients with
+   respect to x, y and z (in dg, domega, dr). */
+typedef enum { KDN_GATES_POST = 0, KDN_GATES_LOGITS = 1 } kdn_gates_t;
 
 /* Library version as major*10000 + minor*100 + patch. */
 int kdn_version(void);

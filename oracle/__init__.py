@@ -83,14 +83,39 @@ def _variant(name):
     raise ValueError(f"unknown variant {name!r}")
 
 
+def _softplus(x):
+    return np.logaddexp(0.0, x)
+
+
+def _sigmoid(x):
+    return np.exp(-np.logaddexp(0.0, -x))
+
+
+def gates_from_logits(x, y, z, r_min):
+    """The layer's gate parameterisation (eq. kla-box-parameterization, r_min of
+    Sec. 5): alpha = sigmoid(x), omega = softplus(y), r = r_min + softplus(z).
+    Returns (g = log alpha, omega, r) in float64."""
+    x, y, z = map(_f64, (x, y, z))
+    return -_softplus(-x), _softplus(y), r_min + _softplus(z)
+
+
+def _check_gates(gates):
+    if gates not in ("post", "logits"):
+        raise ValueError(gates)
+
+
 def fwd(variant, q, k, v, g, omega, r, S0=None, p0=None, *, mu=None, scale=None,
-        bhat=None, trace=False, threads=0):
+        bhat=None, trace=False, threads=0, gates="post", r_min=0.01):
     """Forward over all tokens.  Returns dict(o, ST, pT[, kappa, phat, p], threads).
 
     ``bhat`` (isotropic only) switches to the surrogate mode of
     eq. fixed-gain-approx: the predicted variance is taken from ``bhat`` [B,T,H]
-    instead of being tracked.
+    instead of being tracked.  ``gates="logits"``: g, omega, r are the logits of
+    the layer's parameterisation (``gates_from_logits``).
     """
+    _check_gates(gates)
+    if gates == "logits":
+        g, omega, r = gates_from_logits(g, omega, r, r_min)
     lib = _load()
     vid = _variant(variant)
     q, k, v, g, omega, r = map(_f64, (q, k, v, g, omega, r))
@@ -120,8 +145,23 @@ def fwd(variant, q, k, v, g, omega, r, S0=None, p0=None, *, mu=None, scale=None,
 
 
 def bwd(variant, q, k, v, g, omega, r, S0, p0, dO, dST=None, dpT=None, *, mu=None,
-        scale=None, bhat=None, threads=0):
-    """Gradients of <dO, o> + <dST, ST> + <dpT, pT> with respect to every input."""
+        scale=None, bhat=None, threads=0, gates="post", r_min=0.01):
+    """Gradients of <dO, o> + <dST, ST> + <dpT, pT> with respect to every input.
+
+    ``gates="logits"``: g, omega, r are logits, and dg, domega, dr are the
+    gradients with respect to them (chain rule through ``gates_from_logits``:
+    d log alpha / dx = sigmoid(-x), d omega / dy = sigmoid(y), d r / dz = sigmoid(z)).
+    """
+    _check_gates(gates)
+    if gates == "logits":
+        x, y, z = map(_f64, (g, omega, r))
+        g, omega, r = gates_from_logits(x, y, z, r_min)
+        out = bwd(variant, q, k, v, g, omega, r, S0, p0, dO, dST, dpT, mu=mu, scale=scale,
+                  bhat=bhat, threads=threads)
+        out["dg"] = out["dg"] * _sigmoid(-x)
+        out["domega"] = out["domega"] * _sigmoid(y)
+        out["dr"] = out["dr"] * _sigmoid(z)
+        return out
     lib = _load()
     vid = _variant(variant)
     q, k, v, g, omega, r, dO = map(_f64, (q, k, v, g, omega, r, dO))
@@ -146,7 +186,8 @@ def bwd(variant, q, k, v, g, omega, r, S0, p0, dO, dST=None, dpT=None, *, mu=Non
     return out
 
 
-def decode_step(variant, q, k, v, g, omega, r, S, p, *, mu=None, scale=None):
+def decode_step(variant, q, k, v, g, omega, r, S, p, *, mu=None, scale=None, gates="post",
+                r_min=0.01):
     """One token of the recurrence on a given state (T = 1 of ``fwd``).
 
     Inputs are per-step arrays without the T axis: q, k [B,H,dk], v [B,H,dv],
@@ -154,5 +195,5 @@ def decode_step(variant, q, k, v, g, omega, r, S, p, *, mu=None, scale=None):
     """
     ins = [None if a is None else np.asarray(a, dtype=np.float64)[:, None]
            for a in (q, k, v, g, omega, r)]
-    res = fwd(variant, *ins, S0=S, p0=p, mu=mu, scale=scale)
+    res = fwd(variant, *ins, S0=S, p0=p, mu=mu, scale=scale, gates=gates, r_min=r_min)
     return res["o"][:, 0], res["ST"], res["pT"]

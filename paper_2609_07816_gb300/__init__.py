@@ -27,6 +27,8 @@ LIB_PATH = os.path.join(_HERE, "libkdn.so")
 KDN_OK, KDN_ERR_INVALID_ARG, KDN_ERR_UNSUPPORTED, KDN_ERR_WORKSPACE, KDN_ERR_CUDA, \
     KDN_ERR_TIMEOUT, KDN_ERR_RANGE = range(7)
 KDN_F32, KDN_BF16 = 0, 1
+KDN_GATES_POST, KDN_GATES_LOGITS = 0, 1
+R_MIN_DEFAULT = 0.01  # the layer's observation-noise floor
 
 _DTYPES = {torch.float32: KDN_F32, torch.bfloat16: KDN_BF16}
 
@@ -35,7 +37,8 @@ class kdn_desc_t(ctypes.Structure):
     _fields_ = [("B", ctypes.c_int), ("T", ctypes.c_int), ("H", ctypes.c_int),
                 ("dk", ctypes.c_int), ("dv", ctypes.c_int), ("chunk", ctypes.c_int),
                 ("dtype", ctypes.c_int), ("mu", ctypes.c_float), ("scale", ctypes.c_float),
-                ("decay_per_channel", ctypes.c_int), ("out_dtype", ctypes.c_int)]
+                ("decay_per_channel", ctypes.c_int), ("out_dtype", ctypes.c_int),
+                ("gates", ctypes.c_int), ("r_min", ctypes.c_float)]
 
 
 class KdnError(RuntimeError):
@@ -115,18 +118,23 @@ def _code(dtype):
 
 
 def make_desc(B, T, H, dk, dv, dtype, *, chunk=0, mu=None, scale=None,
-              decay_per_channel=1, out_dtype=KDN_F32) -> kdn_desc_t:
+              decay_per_channel=1, out_dtype=KDN_F32, gates=KDN_GATES_POST,
+              r_min=R_MIN_DEFAULT) -> kdn_desc_t:
+    """``gates``: KDN_GATES_POST (g = log alpha, omega, r) or KDN_GATES_LOGITS
+    (g, omega, r are the logits of sigmoid / softplus / r_min + softplus)."""
     return kdn_desc_t(B, T, H, dk, dv, chunk, _code(dtype), 0.0 if mu is None else float(mu),
                       math.nan if scale is None else float(scale), int(decay_per_channel),
-                      _code(out_dtype))
+                      _code(out_dtype), int(gates), float(r_min))
 
 
-def _desc_from(variant, q, v, g, *, chunk, mu, scale, out_dtype):
+def _desc_from(variant, q, v, g, *, chunk, mu, scale, out_dtype, gates=KDN_GATES_POST,
+               r_min=R_MIN_DEFAULT):
     B, T, H, dk = q.shape
     dv = v.shape[-1]
     pcd = 1 if variant == 0 else int(g.dim() == 4)
     return make_desc(B, T, H, dk, dv, q.dtype, chunk=chunk, mu=mu, scale=scale,
-                     decay_per_channel=pcd, out_dtype=out_dtype)
+                     decay_per_channel=pcd, out_dtype=out_dtype,
+        gates=gates, r_min=r_min)
 
 
 def workspace_bytes(desc: kdn_desc_t, variant: int, backward: bool = False) -> int:
@@ -140,8 +148,10 @@ def alloc_workspace(desc, variant, backward=False, device=None):
 
 
 def _fwd(name, variant, q, k, v, g, omega, r, S0, p0, *, chunk, mu, scale, o, ST, pT,
-         want_state, workspace, stream, out_dtype):
-    desc = _desc_from(variant, q, v, g, chunk=chunk, mu=mu, scale=scale, out_dtype=out_dtype)
+         want_state, workspace, stream, out_dtype,
+         gates=KDN_GATES_POST, r_min=R_MIN_DEFAULT):
+    desc = _desc_from(variant, q, v, g, chunk=chunk, mu=mu, scale=scale, out_dtype=out_dtype,
+                      gates=gates, r_min=r_min)
     B, T, H, dk = q.shape
     dv = v.shape[-1]
     dev = q.device
@@ -162,25 +172,31 @@ def _fwd(name, variant, q, k, v, g, omega, r, S0, p0, *, chunk, mu, scale, o, ST
 
 def kdn_diag_fwd(q, k, v, g, omega, r, S0=None, p0=None, *, chunk=0, mu=None, scale=None,
                  o=None, ST=None, pT=None, want_state=True, workspace=None, stream=None,
-                 out_dtype=torch.float32):
+                 out_dtype=torch.float32, gates=KDN_GATES_POST,
+                 r_min=R_MIN_DEFAULT):
     """Diagonal KDN forward (Prop. 3).  Returns (o, ST, pT)."""
     return _fwd("kdn_diag_fwd", 0, q, k, v, g, omega, r, S0, p0, chunk=chunk, mu=mu,
                 scale=scale, o=o, ST=ST, pT=pT, want_state=want_state, workspace=workspace,
-                stream=stream, out_dtype=out_dtype)
+                stream=stream, out_dtype=out_dtype,
+        gates=gates, r_min=r_min)
 
 
 def kdn_iso_fwd(q, k, v, g, omega, r, S0=None, p0=None, *, chunk=0, mu=None, scale=None,
                 o=None, ST=None, pT=None, want_state=True, workspace=None, stream=None,
-                 out_dtype=torch.float32):
+                 out_dtype=torch.float32, gates=KDN_GATES_POST,
+                 r_min=R_MIN_DEFAULT):
     """Isotropic KDN forward (Prop. 5).  g [B,T,H,dk] = per-channel decay, [B,T,H] = scalar."""
     return _fwd("kdn_iso_fwd", 1, q, k, v, g, omega, r, S0, p0, chunk=chunk, mu=mu,
                 scale=scale, o=o, ST=ST, pT=pT, want_state=want_state, workspace=workspace,
-                stream=stream, out_dtype=out_dtype)
+                stream=stream, out_dtype=out_dtype,
+        gates=gates, r_min=r_min)
 
 
 def _bwd(name, variant, q, k, v, g, omega, r, S0, p0, dO, dST, dpT, *, chunk, mu, scale,
-         grads, want_state_grads, workspace, stream, out_dtype):
-    desc = _desc_from(variant, q, v, g, chunk=chunk, mu=mu, scale=scale, out_dtype=out_dtype)
+         grads, want_state_grads, workspace, stream, out_dtype,
+         gates=KDN_GATES_POST, r_min=R_MIN_DEFAULT):
+    desc = _desc_from(variant, q, v, g, chunk=chunk, mu=mu, scale=scale, out_dtype=out_dtype,
+                      gates=gates, r_min=r_min)
     B, T, H, dk = q.shape
     dv = v.shape[-1]
     dev = q.device
@@ -206,20 +222,24 @@ def _bwd(name, variant, q, k, v, g, omega, r, S0, p0, dO, dST, dpT, *, chunk, mu
 
 def kdn_diag_bwd(q, k, v, g, omega, r, S0, p0, dO, dST=None, dpT=None, *, chunk=0, mu=None,
                  scale=None, grads=None, want_state_grads=True, workspace=None, stream=None,
-                 out_dtype=torch.float32):
+                 out_dtype=torch.float32, gates=KDN_GATES_POST,
+                 r_min=R_MIN_DEFAULT):
     """Gradients of the Diagonal KDN forward.  Returns a dict dq, dk, dv, dg, domega, dr, dS0, dp0."""
     return _bwd("kdn_diag_bwd", 0, q, k, v, g, omega, r, S0, p0, dO, dST, dpT, chunk=chunk,
                 mu=mu, scale=scale, grads=grads, want_state_grads=want_state_grads,
-                workspace=workspace, stream=stream, out_dtype=out_dtype)
+                workspace=workspace, stream=stream, out_dtype=out_dtype,
+        gates=gates, r_min=r_min)
 
 
 def kdn_iso_bwd(q, k, v, g, omega, r, S0, p0, dO, dST=None, dpT=None, *, chunk=0, mu=None,
                 scale=None, grads=None, want_state_grads=True, workspace=None, stream=None,
-                 out_dtype=torch.float32):
+                 out_dtype=torch.float32, gates=KDN_GATES_POST,
+                 r_min=R_MIN_DEFAULT):
     """Gradients of the Isotropic KDN forward."""
     return _bwd("kdn_iso_bwd", 1, q, k, v, g, omega, r, S0, p0, dO, dST, dpT, chunk=chunk,
                 mu=mu, scale=scale, grads=grads, want_state_grads=want_state_grads,
-                workspace=workspace, stream=stream, out_dtype=out_dtype)
+                workspace=workspace, stream=stream, out_dtype=out_dtype,
+        gates=gates, r_min=r_min)
 
 
 def saved_bytes(desc: kdn_desc_t, variant: int = 0) -> int:
@@ -228,8 +248,10 @@ def saved_bytes(desc: kdn_desc_t, variant: int = 0) -> int:
 
 
 def _fwd_save(name, variant, q, k, v, g, omega, r, S0, p0, *, mu, scale, o, ST, pT, saved,
-              want_state, workspace, stream, out_dtype):
-    desc = _desc_from(variant, q, v, g, chunk=0, mu=mu, scale=scale, out_dtype=out_dtype)
+              want_state, workspace, stream, out_dtype,
+              gates=KDN_GATES_POST, r_min=R_MIN_DEFAULT):
+    desc = _desc_from(variant, q, v, g, chunk=0, mu=mu, scale=scale, out_dtype=out_dtype,
+                      gates=gates, r_min=r_min)
     B, T, H, dk = q.shape
     dv = v.shape[-1]
     dev = q.device
@@ -253,26 +275,32 @@ def _fwd_save(name, variant, q, k, v, g, omega, r, S0, p0, *, mu, scale, o, ST, 
 
 def kdn_diag_fwd_save(q, k, v, g, omega, r, S0=None, p0=None, *, mu=None, scale=None, o=None,
                       ST=None, pT=None, saved=None, want_state=True, workspace=None, stream=None,
-                      out_dtype=torch.float32):
+                      out_dtype=torch.float32, gates=KDN_GATES_POST,
+                 r_min=R_MIN_DEFAULT):
     """Diagonal KDN forward that also keeps the chunked backward's context.
     Returns (o, ST, pT, saved); pass `saved` to kdn_diag_bwd_saved."""
     return _fwd_save("kdn_diag_fwd_save", 0, q, k, v, g, omega, r, S0, p0, mu=mu, scale=scale,
                      o=o, ST=ST, pT=pT, saved=saved, want_state=want_state, workspace=workspace,
-                     stream=stream, out_dtype=out_dtype)
+                     stream=stream, out_dtype=out_dtype,
+        gates=gates, r_min=r_min)
 
 
 def kdn_iso_fwd_save(q, k, v, g, omega, r, S0=None, p0=None, *, mu=None, scale=None, o=None,
                      ST=None, pT=None, saved=None, want_state=True, workspace=None, stream=None,
-                     out_dtype=torch.float32):
+                     out_dtype=torch.float32, gates=KDN_GATES_POST,
+                 r_min=R_MIN_DEFAULT):
     """Isotropic KDN forward that also keeps the chunked backward's context."""
     return _fwd_save("kdn_iso_fwd_save", 1, q, k, v, g, omega, r, S0, p0, mu=mu, scale=scale,
                      o=o, ST=ST, pT=pT, saved=saved, want_state=want_state, workspace=workspace,
-                     stream=stream, out_dtype=out_dtype)
+                     stream=stream, out_dtype=out_dtype,
+        gates=gates, r_min=r_min)
 
 
 def _bwd_saved(name, variant, q, k, v, g, omega, r, saved, dO, dST, dpT, *, mu, scale, grads,
-               want_state_grads, workspace, stream, out_dtype):
-    desc = _desc_from(variant, q, v, g, chunk=0, mu=mu, scale=scale, out_dtype=out_dtype)
+               want_state_grads, workspace, stream, out_dtype,
+               gates=KDN_GATES_POST, r_min=R_MIN_DEFAULT):
+    desc = _desc_from(variant, q, v, g, chunk=0, mu=mu, scale=scale, out_dtype=out_dtype,
+                      gates=gates, r_min=r_min)
     B, T, H, dk = q.shape
     dv = v.shape[-1]
     dev = q.device
@@ -298,28 +326,34 @@ def _bwd_saved(name, variant, q, k, v, g, omega, r, saved, dO, dST, dpT, *, mu, 
 
 def kdn_diag_bwd_saved(q, k, v, g, omega, r, saved, dO, dST=None, dpT=None, *, mu=None,
                        scale=None, grads=None, want_state_grads=True, workspace=None, stream=None,
-                       out_dtype=torch.float32):
+                       out_dtype=torch.float32, gates=KDN_GATES_POST,
+                 r_min=R_MIN_DEFAULT):
     """Gradients of the Diagonal KDN forward from the context kept by kdn_diag_fwd_save."""
     return _bwd_saved("kdn_diag_bwd_saved", 0, q, k, v, g, omega, r, saved, dO, dST, dpT, mu=mu,
                       scale=scale, grads=grads, want_state_grads=want_state_grads,
-                      workspace=workspace, stream=stream, out_dtype=out_dtype)
+                      workspace=workspace, stream=stream, out_dtype=out_dtype,
+        gates=gates, r_min=r_min)
 
 
 def kdn_iso_bwd_saved(q, k, v, g, omega, r, saved, dO, dST=None, dpT=None, *, mu=None,
                       scale=None, grads=None, want_state_grads=True, workspace=None, stream=None,
-                      out_dtype=torch.float32):
+                      out_dtype=torch.float32, gates=KDN_GATES_POST,
+                 r_min=R_MIN_DEFAULT):
     """Gradients of the Isotropic KDN forward from the context kept by kdn_iso_fwd_save."""
     return _bwd_saved("kdn_iso_bwd_saved", 1, q, k, v, g, omega, r, saved, dO, dST, dpT, mu=mu,
                       scale=scale, grads=grads, want_state_grads=want_state_grads,
-                      workspace=workspace, stream=stream, out_dtype=out_dtype)
+                      workspace=workspace, stream=stream, out_dtype=out_dtype,
+        gates=gates, r_min=r_min)
 
 
-def _decode(name, variant, q, k, v, g, omega, r, S, p, *, mu, scale, o, stream, out_dtype):
+def _decode(name, variant, q, k, v, g, omega, r, S, p, *, mu, scale, o, stream, out_dtype,
+            gates=KDN_GATES_POST, r_min=R_MIN_DEFAULT):
     B, H, dk = q.shape
     dv = v.shape[-1]
     pcd = 1 if variant == 0 else int(g.dim() == 3)
     desc = make_desc(B, 1, H, dk, dv, q.dtype, mu=mu, scale=scale, decay_per_channel=pcd,
-                     out_dtype=out_dtype)
+                     out_dtype=out_dtype,
+        gates=gates, r_min=r_min)
     if o is None:
         o = torch.empty(B, H, dv, dtype=out_dtype, device=q.device)
     st = getattr(lib(), name)(ctypes.byref(desc), _ptr(q), _ptr(k), _ptr(v), _ptr(g),
@@ -329,26 +363,32 @@ def _decode(name, variant, q, k, v, g, omega, r, S, p, *, mu, scale, o, stream, 
 
 
 def kdn_diag_decode_step(q, k, v, g, omega, r, S, p, *, mu=None, scale=None, o=None,
-                         stream=None, out_dtype=torch.float32):
+                         stream=None, out_dtype=torch.float32, gates=KDN_GATES_POST,
+                 r_min=R_MIN_DEFAULT):
     """One Diagonal KDN token for every head, S [B,H,dk,dv] and p [B,H,dk] updated in place."""
     return _decode("kdn_diag_decode_step", 0, q, k, v, g, omega, r, S, p, mu=mu, scale=scale,
-                   o=o, stream=stream, out_dtype=out_dtype)
+                   o=o, stream=stream, out_dtype=out_dtype,
+        gates=gates, r_min=r_min)
 
 
 def kdn_iso_decode_step(q, k, v, g, omega, r, S, p, *, mu=None, scale=None, o=None,
-                        stream=None, out_dtype=torch.float32):
+                        stream=None, out_dtype=torch.float32, gates=KDN_GATES_POST,
+                 r_min=R_MIN_DEFAULT):
     """One Isotropic KDN token for every head; g [B,H,dk] or [B,H]; p [B,H] in place."""
     return _decode("kdn_iso_decode_step", 1, q, k, v, g, omega, r, S, p, mu=mu, scale=scale,
-                   o=o, stream=stream, out_dtype=out_dtype)
+                   o=o, stream=stream, out_dtype=out_dtype,
+        gates=gates, r_min=r_min)
 
 
 def kdn_diag_fwd_noalloc(q, k, v, g, omega, r, S0=None, p0=None, *, o, ST=None, pT=None,
-                         mu=None, scale=None, stream=None):
+                         mu=None, scale=None, stream=None, gates=KDN_GATES_POST,
+                         r_min=R_MIN_DEFAULT):
     """Diagonal KDN forward into caller-provided outputs, using the library's own
     fixed scratch array instead of a workspace, for callers that may not
     allocate device memory.  Problems needing more than
     KDN_NOALLOC_SCRATCH_BYTES of scratch are rejected.  Returns o."""
-    desc = _desc_from(0, q, v, g, chunk=0, mu=mu, scale=scale, out_dtype=o.dtype)
+    desc = _desc_from(0, q, v, g, chunk=0, mu=mu, scale=scale, out_dtype=o.dtype, gates=gates,
+                      r_min=r_min)
     st = lib().kdn_diag_fwd_noalloc(ctypes.byref(desc), _ptr(q), _ptr(k), _ptr(v), _ptr(g),
                                     _ptr(omega), _ptr(r), _ptr(S0), _ptr(p0), _ptr(o), _ptr(ST),
                                     _ptr(pT), _stream(stream))

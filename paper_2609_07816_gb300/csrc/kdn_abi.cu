@@ -33,6 +33,9 @@ kdn_status_t fill_sizes(const kdn_desc_t *d, int variant, bool decode, Args *a) 
   if (variant == 1 && d->decay_per_channel != 0 && d->decay_per_channel != 1)
     return KDN_ERR_INVALID_ARG;
   if (isnan(d->mu) || isinf(d->mu) || isinf(d->scale)) return KDN_ERR_INVALID_ARG;
+  if (d->gates != KDN_GATES_POST && d->gates != KDN_GATES_LOGITS) return KDN_ERR_INVALID_ARG;
+  if (d->gates == KDN_GATES_LOGITS && !(d->r_min >= 0.f && d->r_min < INFINITY))
+    return KDN_ERR_INVALID_ARG;
   const long long BH = (long long)d->B * d->H;
   const int T = decode ? 1 : d->T;
   if (BH > 65535LL * 1024 || T > (1 << 21)) return KDN_ERR_UNSUPPORTED;
@@ -52,6 +55,8 @@ kdn_status_t fill_sizes(const kdn_desc_t *d, int variant, bool decode, Args *a) 
   a->dtype = d->dtype;
   a->odt = d->out_dtype;
   a->chunk = d->chunk;
+  a->gates = d->gates;
+  a->rmin = d->gates == KDN_GATES_LOGITS ? d->r_min : 0.f;
   a->mu = d->mu > 0.f ? d->mu : (float)d->dk;
   a->tau = isnan(d->scale) ? 1.0f / sqrtf((float)d->dk) : d->scale;
   return KDN_OK;

@@ -57,10 +57,10 @@ __global__ void __launch_bounds__(32) k_gain_scan_diag(Args a) {
       g_[j] = 0.f; w_[j] = 0.f; k_[j] = 0.f; r_[j] = 1.f;
       if (t < a.T) {
         const size_t th = tok_index(a, b, t, h);
-        g_[j] = ld<DT>(a.g, th * dk + i);
-        w_[j] = ld<DT>(a.omega, th * dk + i);
+        g_[j] = gate_logalpha(a.gates, ld<DT>(a.g, th * dk + i));
+        w_[j] = gate_omega(a.gates, ld<DT>(a.omega, th * dk + i));
         k_[j] = ld<DT>(a.k, th * dk + i);
-        r_[j] = ld<DT>(a.r, th);
+        r_[j] = gate_r(a.gates, a.rmin, ld<DT>(a.r, th));
       }
     }
   };
@@ -101,11 +101,11 @@ __global__ void __launch_bounds__(32) k_gain_scan_iso(Args a) {
       for (int i = 0; i < dk; ++i) {
         const float kk = ld<DT>(a.k, th * dk + i);
         n2 += kk * kk;
-        if (a.pcd) sa += expf(2.f * ld<DT>(a.g, th * dk + i));
+        if (a.pcd) sa += expf(2.f * gate_logalpha(a.gates, ld<DT>(a.g, th * dk + i)));
       }
-      aa = a.pcd ? sa / dk : expf(2.f * ld<DT>(a.g, th));
-      w = ld<DT>(a.omega, th);
-      rr = ld<DT>(a.r, th);
+      aa = a.pcd ? sa / dk : expf(2.f * gate_logalpha(a.gates, ld<DT>(a.g, th)));
+      w = gate_omega(a.gates, ld<DT>(a.omega, th));
+      rr = gate_r(a.gates, a.rmin, ld<DT>(a.r, th));
       a.isotok[((size_t)bh * a.Tp + t) * 2 + 0] = aa;
       a.isotok[((size_t)bh * a.Tp + t) * 2 + 1] = n2;
     }
@@ -163,7 +163,7 @@ __device__ void prep_core(const Args &a, int c, int bh, float *sK, float *sQ, fl
   // gain emission from the pre-write predictive variance (eq. chunk-gain-emission)
   for (int t = warp; t < CC; t += NT / 32) {
     const int tt = c * CC + t;
-    const float rr = tt < a.T ? ld<DT>(a.r, tok_index(a, b, tt, h)) : 1.f;
+    const float rr = tt < a.T ? gate_r(a.gates, a.rmin, ld<DT>(a.r, tok_index(a, b, tt, h))) : 1.f;
     if (V == 0) {
       const float *ph = a.phat + ((size_t)bh * a.Tp + tt) * DK;
       float part = 0.f;
@@ -194,7 +194,7 @@ __device__ void prep_core(const Args &a, int c, int bh, float *sK, float *sQ, fl
       float gg = 0.f;
       if (tt < a.T) {
         const size_t th = tok_index(a, b, tt, h);
-        gg = a.pcd ? ld<DT>(a.g, th * DK + i) : ld<DT>(a.g, th);
+        gg = a.pcd ? gate_logalpha(a.gates, ld<DT>(a.g, th * DK + i)) : gate_logalpha(a.gates, ld<DT>(a.g, th));
       }
       G += gg;
       gam = expf(G);
@@ -694,7 +694,7 @@ __global__ void __launch_bounds__(NT) k_chunk_bwd(Args a) {
     const int tt = c * CC + t;
     const size_t row = (size_t)bh * a.Tp + tt;
     float rr = 1.f;
-    if (tt < a.T) rr = ld<DT>(a.r, tok_index(a, b, tt, h));
+    if (tt < a.T) rr = gate_r(a.gates, a.rmin, ld<DT>(a.r, tok_index(a, b, tt, h)));
     float kv[DK / 32];
 #pragma unroll
     for (int m = 0; m < DK / 32; ++m) {
@@ -766,8 +766,8 @@ __global__ void __launch_bounds__(32) k_gain_bwd_diag(Args a) {
         const size_t th = tok_index(a, b, t, h), row = hrow + t;
         ph_[j] = a.phat[row * dk + i];
         k_[j] = ld<DT>(a.k, th * dk + i);
-        r_[j] = ld<DT>(a.r, th);
-        g_[j] = ld<DT>(a.g, th * dk + i);
+        r_[j] = gate_r(a.gates, a.rmin, ld<DT>(a.r, th));
+        g_[j] = gate_logalpha(a.gates, ld<DT>(a.g, th * dk + i));
         dl_[j] = a.dphloc[row * dk + i];
         dk_[j] = a.dkpart[row * dk + i];
         dg_[j] = a.dgpart[row * dk + i];
@@ -807,8 +807,11 @@ __global__ void __launch_bounds__(32) k_gain_bwd_diag(Args a) {
         if (lane == 0) a.drw[row * 4 + blockIdx.y] = drp;
         const float pprev = j > 0 ? pt[j - 1] : pprev_block;
         const float al2 = expf(2.f * cg[j]);
-        sto(a.odt, a.domega, th * dk + i, dph);
-        sto(a.odt, a.dg, th * dk + i, cdg[j] + 2.f * al2 * pprev * dph);
+        // logit gates: d omega / dy = sigmoid(y), d log alpha / dx = 1 - alpha
+        const float fw = a.gates ? sigmoid_f(ld<DT>(a.omega, th * dk + i)) : 1.f;
+        const float fg = a.gates ? -expm1f(cg[j]) : 1.f;
+        sto(a.odt, a.domega, th * dk + i, dph * fw);
+        sto(a.odt, a.dg, th * dk + i, (cdg[j] + 2.f * al2 * pprev * dph) * fg);
         sto(a.odt, a.dk_, th * dk + i, dkk);
         dp = al2 * dph;
       }
@@ -832,7 +835,9 @@ __global__ void k_finalize_dr_diag(Args a) {
     const size_t row = (size_t)bh * a.Tp + t;
     float acc = a.drpart[row];
     for (int w = 0; w < nw; ++w) acc += a.drw[row * 4 + w];
-    sto(a.odt, a.dr, tok_index(a, bh / a.H, t, bh % a.H), acc);
+    const size_t th = tok_index(a, bh / a.H, t, bh % a.H);
+    if (a.gates) acc *= sigmoid_f(ld<DT>(a.r, th));  // d r / dz
+    sto(a.odt, a.dr, th, acc);
   }
 }
 
@@ -855,7 +860,7 @@ __global__ void __launch_bounds__(32) k_gain_bwd_iso(Args a) {
         ph = a.phat[row];
         aa = a.isotok[row * 2 + 0];
         n2 = a.isotok[row * 2 + 1];
-        rr = ld<DT>(a.r, tok_index(a, b, t, h));
+        rr = gate_r(a.gates, a.rmin, ld<DT>(a.r, tok_index(a, b, t, h)));
         if (j < 32) {
           s_dl[j] = a.dphloc[row];
           s_dr[j] = a.drpart[row];
@@ -897,7 +902,9 @@ __global__ void __launch_bounds__(32) k_gain_bwd_iso(Args a) {
         a.drpart[row] = s_dr[lane];
         a.isoadj[row * 2 + 0] = s_o1[lane];
         a.isoadj[row * 2 + 1] = s_o2[lane];
-        sto(a.odt, a.domega, tok_index(a, b, t, h), s_dw[lane]);
+        const size_t th = tok_index(a, b, t, h);
+        const float fw = a.gates ? sigmoid_f(ld<DT>(a.omega, th)) : 1.f;  // d omega / dy
+        sto(a.odt, a.domega, th, s_dw[lane] * fw);
       }
     }
     __syncwarp();
@@ -916,8 +923,10 @@ __global__ void __launch_bounds__(DK) k_finalize_iso(Args a) {
   const float kk = ld<DT>(a.k, th * DK + i);
   sto(a.odt, a.dk_, th * DK + i, a.dkpart[row * DK + i] + 2.f * kk * dn2);
   if (a.pcd) {
-    const float al2 = expf(2.f * ld<DT>(a.g, th * DK + i));
-    sto(a.odt, a.dg, th * DK + i, a.dgpart[row * DK + i] + 2.f * al2 * da / DK);
+    const float lal = gate_logalpha(a.gates, ld<DT>(a.g, th * DK + i));
+    const float al2 = expf(2.f * lal);
+    const float fg = a.gates ? -expm1f(lal) : 1.f;  // d log alpha / dx
+    sto(a.odt, a.dg, th * DK + i, (a.dgpart[row * DK + i] + 2.f * al2 * da / DK) * fg);
   } else {
     __shared__ float red[DK / 32];
     float part = warp_sum(a.dgpart[row * DK + i]);
@@ -926,11 +935,16 @@ __global__ void __launch_bounds__(DK) k_finalize_iso(Args a) {
     if (i == 0) {
       float tot = 0.f;
       for (int w = 0; w < DK / 32; ++w) tot += red[w];
-      const float al2 = expf(2.f * ld<DT>(a.g, th));
-      sto(a.odt, a.dg, th, tot + 2.f * al2 * da);
+      const float lal = gate_logalpha(a.gates, ld<DT>(a.g, th));
+      const float al2 = expf(2.f * lal);
+      const float fg = a.gates ? -expm1f(lal) : 1.f;  // d log alpha / dx
+      sto(a.odt, a.dg, th, (tot + 2.f * al2 * da) * fg);
     }
   }
-  if (i == 0) sto(a.odt, a.dr, th, a.drpart[row]);
+  if (i == 0) {
+    const float fr = a.gates ? sigmoid_f(ld<DT>(a.r, th)) : 1.f;  // d r / dz
+    sto(a.odt, a.dr, th, a.drpart[row] * fr);
+  }
 }
 
 // ---------------------------------------------------------------------------

@@ -36,7 +36,9 @@ __device__ __forceinline__ void vstore(float *p, const float *x) {
   *reinterpret_cast<typename Vec<CPL>::T *>(p) = v;
 }
 
-template <int V, typename DT, int DK, int DV>
+// G: the gate inputs are logits (compile-time, so that post-activation inputs
+// carry none of the activation code)
+template <int V, typename DT, int DK, int DV, int G>
 __global__ void __launch_bounds__(DNT) k_decode(Args a, float *S, float *P) {
   constexpr int RPW = DK / 8;   // rows per warp
   constexpr int CPL = DV / 32;  // columns per lane
@@ -58,9 +60,9 @@ __global__ void __launch_bounds__(DNT) k_decode(Args a, float *S, float *P) {
     kk = ld<DT>(a.k, th * DK + i);
     qq = ld<DT>(a.q, th * DK + i);
     const float gg = (V == 0 || a.pcd) ? ld<DT>(a.g, th * DK + i) : ld<DT>(a.g, th);
-    al = expf(gg);
+    al = G ? sigmoid_f(gg) : expf(gg);
     if (V == 0) {
-      ph = al * al * P[(size_t)bh * DK + i] + ld<DT>(a.omega, th * DK + i);
+      ph = al * al * P[(size_t)bh * DK + i] + gate_omega(G, ld<DT>(a.omega, th * DK + i));
       x0 = ph * kk * kk;  // -> sum phat k^2
       x1 = ph * kk * qq;  // -> sum phat k q
     } else {
@@ -79,7 +81,7 @@ __global__ void __launch_bounds__(DNT) k_decode(Args a, float *S, float *P) {
 #pragma unroll
     for (int w = 0; w < NWK; ++w) { t0 += s_part[w][0]; t1 += s_part[w][1]; t2 += s_part[w][2]; }
     const int i = tid;
-    const float rr = ld<DT>(a.r, th);
+    const float rr = gate_r(G, a.rmin, ld<DT>(a.r, th));
     float kap, kq;
     if (V == 0) {
       const float sden = rr + t0;
@@ -89,7 +91,7 @@ __global__ void __launch_bounds__(DNT) k_decode(Args a, float *S, float *P) {
       P[(size_t)bh * DK + i] = ph / (1.f + u * ph);
     } else {
       const float aa = a.pcd ? t0 / DK : al * al;
-      const float bhat = aa * P[bh] + ld<DT>(a.omega, th);
+      const float bhat = aa * P[bh] + gate_omega(G, ld<DT>(a.omega, th));
       const float beta = bhat / (rr + bhat * t1);
       kap = beta * kk;
       kq = beta * t2;
@@ -145,34 +147,41 @@ __global__ void __launch_bounds__(DNT) k_decode(Args a, float *S, float *P) {
   }
 }
 
-template <int V, typename DT, int DK>
+template <int V, typename DT, int DK, int G>
 kdn_status_t dec_dv(const Args &a, float *S, float *P, cudaStream_t s) {
   const int BH = a.B * a.H;
   switch (a.dv) {
-    case 32: k_decode<V, DT, DK, 32><<<BH, DNT, 0, s>>>(a, S, P); break;
-    case 64: k_decode<V, DT, DK, 64><<<BH, DNT, 0, s>>>(a, S, P); break;
-    case 128: k_decode<V, DT, DK, 128><<<BH, DNT, 0, s>>>(a, S, P); break;
+    case 32: k_decode<V, DT, DK, 32, G><<<BH, DNT, 0, s>>>(a, S, P); break;
+    case 64: k_decode<V, DT, DK, 64, G><<<BH, DNT, 0, s>>>(a, S, P); break;
+    case 128: k_decode<V, DT, DK, 128, G><<<BH, DNT, 0, s>>>(a, S, P); break;
     default: return KDN_ERR_UNSUPPORTED;
   }
   return cudaGetLastError() == cudaSuccess ? KDN_OK : KDN_ERR_CUDA;
 }
 
-template <int V, typename DT>
+template <int V, typename DT, int G>
 kdn_status_t dec_dk(const Args &a, float *S, float *P, cudaStream_t s) {
   switch (a.dk) {
-    case 32: return dec_dv<V, DT, 32>(a, S, P, s);
-    case 64: return dec_dv<V, DT, 64>(a, S, P, s);
-    case 128: return dec_dv<V, DT, 128>(a, S, P, s);
+    case 32: return dec_dv<V, DT, 32, G>(a, S, P, s);
+    case 64: return dec_dv<V, DT, 64, G>(a, S, P, s);
+    case 128: return dec_dv<V, DT, 128, G>(a, S, P, s);
   }
   return KDN_ERR_UNSUPPORTED;
+}
+
+template <int V, typename DT>
+kdn_status_t dec_gates(const Args &a, float *S, float *P, cudaStream_t s) {
+  return a.gates ? dec_dk<V, DT, 1>(a, S, P, s) : dec_dk<V, DT, 0>(a, S, P, s);
 }
 
 }  // namespace
 
 kdn_status_t launch_decode(const Args &a, float *S, float *P, cudaStream_t s) {
   if (a.variant == 0)
-    return a.dtype == KDN_BF16 ? dec_dk<0, __nv_bfloat16>(a, S, P, s) : dec_dk<0, float>(a, S, P, s);
-  return a.dtype == KDN_BF16 ? dec_dk<1, __nv_bfloat16>(a, S, P, s) : dec_dk<1, float>(a, S, P, s);
+    return a.dtype == KDN_BF16 ? dec_gates<0, __nv_bfloat16>(a, S, P, s)
+                               : dec_gates<0, float>(a, S, P, s);
+  return a.dtype == KDN_BF16 ? dec_gates<1, __nv_bfloat16>(a, S, P, s)
+                             : dec_gates<1, float>(a, S, P, s);
 }
 
 }  // namespace kdn

@@ -85,7 +85,7 @@ constexpr int O_DWT = O_G, O_DAT = O_G + 16 * KB, O_XT = O_G + 24 * KB, O_KQH2 =
 constexpr int O_QL2 = O_RDO, O_DRTL = O_RH;
 // small arrays
 constexpr int OFF_SM = BUF_END;
-constexpr int SMALL_FLOATS = 64 * 14 + 256 * 2 + 128 * 2 + 16;
+constexpr int SMALL_FLOATS = 64 * 15 + 256 * 2 + 128 * 2 + 16;
 constexpr int OFF_BAR = OFF_SM + SMALL_FLOATS * 4;
 constexpr int SMEM_BYTES = OFF_BAR + 64 + 1024;  // + alignment slack
 static_assert(SMEM_BYTES <= 232448, "shared memory");
@@ -163,7 +163,9 @@ __device__ __forceinline__ void st_grad(void *p, size_t i, float x) {
   else static_cast<float *>(p)[i] = x;
 }
 
-template <int V, int OBF>
+// G: the gate inputs are logits (KDN_GATES_LOGITS), a compile-time choice so
+// that the post-activation path carries none of the chain-rule code
+template <int V, int OBF, int G>
 __global__ void __launch_bounds__(BT, 1)
     k_fused_bwd(const __grid_constant__ CUtensorMap mq, const __grid_constant__ CUtensorMap mk,
                 const __grid_constant__ CUtensorMap mv, const __grid_constant__ CUtensorMap mdo,
@@ -182,8 +184,8 @@ __global__ void __launch_bounds__(BT, 1)
   float *s_dp = s_gC + 128;     // [128] uncertainty cotangent carried between chunks
   float *s_si = s_dp + 128;     // [64] 1 / s_t
   float *s_ds = s_si + 64;      // [64] ds_t (cotangent of s_t)
-  float *s_om = s_ds + 64;      // [64] omega_t (iso)
-  float *s_gs = s_om + 64;      // [64] scalar log-decay g_t (iso, one decay per head)
+  float *s_fw = s_ds + 64;      // [64] d omega_t / d y_t (iso; 1 unless the gates are logits)
+  float *s_gs = s_fw + 64;      // [64] scalar log-decay g_t (iso, one decay per head)
   float *s_n2 = s_gs + 64;      // [64] |k_t|^2 (iso)
   float *s_a = s_n2 + 64;       // [64] a_t = mean alpha^2 (iso)
   float *s_bh = s_a + 64;       // [64] bhat_t (iso)
@@ -192,6 +194,7 @@ __global__ void __launch_bounds__(BT, 1)
   float *s_dn2 = s_x + 64;      // [64] cotangent of |k_t|^2 (iso)
   float *s_da = s_dn2 + 64;     // [64] cotangent of a_t (iso)
   float *s_misc = s_da + 64;    // [0] lambda, [1..] scratch
+  float *s_fr = s_misc + 16;    // [64] d r_t / d z_t (1 unless the gates are logits)
   uint64_t *bars = reinterpret_cast<uint64_t *>(sm + OFF_BAR);
   uint64_t *bar_a = bars, *bar_b = bars + 1, *bar_mma = bars + 2;
   uint32_t *s_tbase = reinterpret_cast<uint32_t *>(bars + 4);
@@ -326,16 +329,22 @@ __global__ void __launch_bounds__(BT, 1)
 
   // per-token scalars of the next chunk (r; the scalar decay of the isotropic KDN),
   // prefetched into registers
-  float nr = 1.f, ng = 0.f;
+  // (and, with logit gates, the chain factors sigmoid(z_t), sigmoid(y_t) of r and omega)
+  float nr = 1.f, ng = 0.f, nfr = 1.f, nfw = 1.f;
   auto load_r = [&](int c) {
     nr = 1.f;
     ng = 0.f;
+    nfr = 1.f;
+    nfw = 1.f;
     if (tid < CM && c >= 0) {
       const int t = c * CM + tid;
       if (t < a.T) {
         const size_t th = tok_index(a, b, t, h);
-        nr = ld<__nv_bfloat16>(a.r, th);
-        if (V == 1 && !a.pcd) ng = ld<__nv_bfloat16>(a.g, th);
+        const float z = ld<__nv_bfloat16>(a.r, th);
+        nr = gate_r(G, a.rmin, z);
+        nfr = dgate_sig(G, z);
+        if (V == 1 && !a.pcd) ng = gate_logalpha(G, ld<__nv_bfloat16>(a.g, th));
+        if (V == 1 && G) nfw = sigmoid_f(ld<__nv_bfloat16>(a.omega, th));
       }
     }
   };
@@ -379,6 +388,8 @@ __global__ void __launch_bounds__(BT, 1)
       s_r[tid] = nr;
       s_ri[tid] = 1.f / nr;
       s_gs[tid] = ng;
+      s_fr[tid] = nfr;
+      s_fw[tid] = nfw;
     }
     const unsigned char *rec = a.fSin + ((size_t)bh * NC + c) * kCtxBytes;
     float e16[16], ph16[16], tk[5];
@@ -835,9 +846,12 @@ __global__ void __launch_bounds__(BT, 1)
             run += sdg[j * BT + tid];
             const float dgt = run + 2.f * a2v[u] * pprev * dph;
             if (j < nval) {
+              // logit gates: d omega / dy = sigmoid(y), d log alpha / dx = 1 - alpha
+              const float fw = G ? sigmoid_f(ld<__nv_bfloat16>(a.omega, obase + (size_t)j * ostride)) : 1.f;
+              const float fg = G ? 1.f - sqrtf(a2v[u]) : 1.f;
               out(a.dk_, j, dkt * invl);
-              out(a.domega, j, dph * invl);
-              out(a.dg, j, dgt * invl);
+              out(a.domega, j, dph * fw * invl);
+              out(a.dg, j, dgt * fg * invl);
             }
             dp = a2v[u] * dph;
           }
@@ -850,7 +864,7 @@ __global__ void __launch_bounds__(BT, 1)
           const int tt = c * CM + tid;
           if (tt < a.T) {
             const float dr = s_ds[tid] + ((s_red2[tid] + s_red2[64 + tid]) + (s_red2[128 + tid] + s_red2[192 + tid]));
-            st_grad<OBF>(a.dr, tok_index(a, b, tt, h), dr * invl);
+            st_grad<OBF>(a.dr, tok_index(a, b, tt, h), dr * (G ? s_fr[tid] : 1.f) * invl);
           }
         }
       }
@@ -940,8 +954,8 @@ __global__ void __launch_bounds__(BT, 1)
           s_da[t] = s_bp[t] * dbhat;
           if (tt < a.T) {
             const size_t th = tok_index(a, b, tt, h);
-            st_grad<OBF>(a.domega, th, dbhat * invl);
-            st_grad<OBF>(a.dr, th, (-__fdividef(dbeta * beta, dd) - du * u * ri) * invl);
+            st_grad<OBF>(a.domega, th, dbhat * (G ? s_fw[t] : 1.f) * invl);
+            st_grad<OBF>(a.dr, th, (-__fdividef(dbeta * beta, dd) - du * u * ri) * (G ? s_fr[t] : 1.f) * invl);
           }
           db = s_a[t] * dbhat;
         }
@@ -968,7 +982,8 @@ __global__ void __launch_bounds__(BT, 1)
           if (j < nval) out(a.dk_, j, (c2[j] + 2.f * k16[j] * s_dn2[t]) * invl);
           if (pcd) {
             const float al = __fdividef(ga[j], j > 0 ? ga[j - 1] : ga_prev);
-            if (j < nval) out(a.dg, j, (run + s_da[t] * 2.f * al * al * (1.f / D)) * invl);
+            const float fg = G ? 1.f - al : 1.f;  // d log alpha / dx
+            if (j < nval) out(a.dg, j, (run + s_da[t] * 2.f * al * al * (1.f / D)) * fg * invl);
           } else {
             dgp[j] = run;
           }
@@ -983,7 +998,8 @@ __global__ void __launch_bounds__(BT, 1)
               const float al = __expf(s_gs[tid]);
               const float dg = (s_red2[tid] + s_red2[64 + tid]) + (s_red2[128 + tid] + s_red2[192 + tid]) +
                                2.f * al * al * s_da[tid];
-              st_grad<OBF>(a.dg, tok_index(a, b, tt, h), dg * invl);
+              const float fg = G ? -expm1f(s_gs[tid]) : 1.f;  // d log alpha / dx
+              st_grad<OBF>(a.dg, tok_index(a, b, tt, h), dg * fg * invl);
             }
           }
         }
@@ -1046,8 +1062,13 @@ kdn_status_t launch_fused_bwd_sweep(const Args &a, cudaStream_t s) {
       !make_map(&mdo, a.dO, a))
     return KDN_ERR_CUDA;
   const bool obf = a.odt == KDN_BF16;
-  auto kern = a.variant == 0 ? (obf ? k_fused_bwd<0, 1> : k_fused_bwd<0, 0>)
-                             : (obf ? k_fused_bwd<1, 1> : k_fused_bwd<1, 0>);
+  decltype(&k_fused_bwd<0, 0, 0>) kern;
+  if (a.gates)
+    kern = a.variant == 0 ? (obf ? k_fused_bwd<0, 1, 1> : k_fused_bwd<0, 0, 1>)
+                          : (obf ? k_fused_bwd<1, 1, 1> : k_fused_bwd<1, 0, 1>);
+  else
+    kern = a.variant == 0 ? (obf ? k_fused_bwd<0, 1, 0> : k_fused_bwd<0, 0, 0>)
+                          : (obf ? k_fused_bwd<1, 1, 0> : k_fused_bwd<1, 0, 0>);
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES) !=
       cudaSuccess)
     return KDN_ERR_CUDA;

@@ -77,7 +77,9 @@ struct FusedParams {
   float *save_p;          // optional [BH][NC][128] uncertainty carry entering each chunk
 };
 
-template <int V>
+// G: the gate inputs are logits (KDN_GATES_LOGITS), a compile-time choice so
+// that the post-activation path carries none of the activation code
+template <int V, int G>
 __global__ void __launch_bounds__(FT, 1)
     k_fused_fwd(const __grid_constant__ CUtensorMap mq, const __grid_constant__ CUtensorMap mk,
                 const __grid_constant__ CUtensorMap mv, const __grid_constant__ CUtensorMap mg,
@@ -194,10 +196,10 @@ __global__ void __launch_bounds__(FT, 1)
       nr = 1.f; nom = 0.f; ng = 0.f;
       if (c < NC && t < a.T) {
         const size_t th = tok_index(a, b, t, h);
-        nr = ld<__nv_bfloat16>(a.r, th);
+        nr = gate_r(G, a.rmin, ld<__nv_bfloat16>(a.r, th));
         if (V == 1) {
-          nom = ld<__nv_bfloat16>(a.omega, th);
-          if (!a.pcd) ng = ld<__nv_bfloat16>(a.g, th);
+          nom = gate_omega(G, ld<__nv_bfloat16>(a.omega, th));
+          if (!a.pcd) ng = gate_logalpha(G, ld<__nv_bfloat16>(a.g, th));
         }
       }
     }
@@ -242,6 +244,15 @@ __global__ void __launch_bounds__(FT, 1)
     //          (eq. chunk-gain-carry), then every quarter runs its own 16 steps
     //          (eq. chunk-gain-local-prefix, -emission).  Results go to fp32
     //          scratch: phat to b3, gamma to fs (both free here).
+    // alpha and omega from the per-channel gate tiles (log alpha or logits); with
+    // logit gates the zero-filled tokens past T are kept identity updates
+    const int t_valid = a.T - c * CM;
+    auto tile_alpha = [&](float x, int t) {
+      return G ? (t < t_valid ? sigmoid_f(x) : 1.f) : __expf(x);
+    };
+    auto tile_omega = [&](float y, int t) {
+      return G ? (t < t_valid ? softplus_f(y) : 0.f) : y;
+    };
     float *Pb = reinterpret_cast<float *>(b3);  // [64][128] phat_t
     float *Eb = fs;                             // [64][128] gamma_t
     float *sQ = reinterpret_cast<float *>(a2);  // [4][128][5] per-quarter summaries (a2 is free)
@@ -253,8 +264,8 @@ __global__ void __launch_bounds__(FT, 1)
 #pragma unroll
         for (int j = 0; j < 16; ++j) {
           const float kk = bf(kq, 16384, t0 + j, i);
-          al[j] = __expf(bf(rg, 8192, t0 + j, i));
-          w[j] = bf(rw, 8192, t0 + j, i);
+          al[j] = tile_alpha(bf(rg, 8192, t0 + j, i), t0 + j);
+          w[j] = tile_omega(bf(rw, 8192, t0 + j, i), t0 + j);
           uk[j] = a.mu * kk * kk * s_ri[t0 + j];
         }
         float m00 = 1.f, m01 = 0.f, m10 = 0.f, m11 = 1.f, eq = 1.f;
@@ -307,7 +318,7 @@ __global__ void __launch_bounds__(FT, 1)
             unpack_bf8(sm16(rg, sl * 8192 + chunk_off(t, cc)), gv);
 #pragma unroll
             for (int j = 0; j < 8; ++j) {
-              const float al = __expf(gv[j]);
+              const float al = tile_alpha(gv[j], t);
               sa += al * al;
             }
           }
@@ -327,7 +338,7 @@ __global__ void __launch_bounds__(FT, 1)
         float el[16], eq = 1.f;
 #pragma unroll
         for (int j = 0; j < 16; ++j) {
-          eq *= __expf(pcd ? bf(rg, 8192, t0 + j, i) : s_gs[t0 + j]);
+          eq *= pcd ? tile_alpha(bf(rg, 8192, t0 + j, i), t0 + j) : __expf(s_gs[t0 + j]);
           el[j] = eq;
         }
         sQ[(qq * D + i) * 5 + 4] = eq;
@@ -751,17 +762,12 @@ kdn_status_t launch_fused_fwd(const Args &a, cudaStream_t s, unsigned char *save
   if (P.has_g_map && !make_map(&mg, a.g, a)) return KDN_ERR_CUDA;
   if (P.has_w_map && !make_map(&mw, a.omega, a)) return KDN_ERR_CUDA;
   const int BH = a.B * a.H;
-  if (a.variant == 0) {
-    if (cudaFuncSetAttribute(k_fused_fwd<0>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             SMEM_BYTES) != cudaSuccess)
-      return KDN_ERR_CUDA;
-    k_fused_fwd<0><<<BH, FT, SMEM_BYTES, s>>>(mq, mk, mv, mg, mw, mo, P);
-  } else {
-    if (cudaFuncSetAttribute(k_fused_fwd<1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             SMEM_BYTES) != cudaSuccess)
-      return KDN_ERR_CUDA;
-    k_fused_fwd<1><<<BH, FT, SMEM_BYTES, s>>>(mq, mk, mv, mg, mw, mo, P);
-  }
+  auto kern = a.variant == 0 ? (a.gates ? k_fused_fwd<0, 1> : k_fused_fwd<0, 0>)
+                             : (a.gates ? k_fused_fwd<1, 1> : k_fused_fwd<1, 0>);
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES) !=
+      cudaSuccess)
+    return KDN_ERR_CUDA;
+  kern<<<BH, FT, SMEM_BYTES, s>>>(mq, mk, mv, mg, mw, mo, P);
   return cudaGetLastError() == cudaSuccess ? KDN_OK : KDN_ERR_CUDA;
 }
 

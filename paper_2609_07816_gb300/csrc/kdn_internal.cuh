@@ -35,6 +35,29 @@ __device__ __forceinline__ void sto(int odt, void *p, size_t i, float x) {
   else static_cast<float *>(p)[i] = x;
 }
 
+// Gate activations of the layer's parameterisation for KDN_GATES_LOGITS
+// inputs: alpha = sigmoid(x), omega = softplus(y), r = r_min + softplus(z).
+__device__ __forceinline__ float softplus_f(float x) {
+  return fmaxf(x, 0.f) + log1pf(__expf(-fabsf(x)));
+}
+__device__ __forceinline__ float sigmoid_f(float x) { return 1.f / (1.f + __expf(-x)); }
+// log alpha from the gate input: g itself, or log sigmoid(x) = -softplus(-x)
+__device__ __forceinline__ float gate_logalpha(int gates, float g) {
+  return gates ? -softplus_f(-g) : g;
+}
+__device__ __forceinline__ float gate_omega(int gates, float w) {
+  return gates ? softplus_f(w) : w;
+}
+__device__ __forceinline__ float gate_r(int gates, float rmin, float r) {
+  return gates ? rmin + softplus_f(r) : r;
+}
+// Chain-rule factors from the post-activation gates back to the logits:
+// d log(alpha) / dx = 1 - alpha, d omega / dy = sigmoid(y), d r / dz = sigmoid(z).
+__device__ __forceinline__ float dgate_logalpha(int gates, float alpha) {
+  return gates ? 1.f - alpha : 1.f;
+}
+__device__ __forceinline__ float dgate_sig(int gates, float y) { return gates ? sigmoid_f(y) : 1.f; }
+
 __device__ __forceinline__ float warp_sum(float x) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
@@ -55,6 +78,8 @@ struct Args {
   int dtype;
   int odt;      // dtype of o and of the input gradients
   int chunk;    // chunk length requested in the descriptor (0, 32 or 64)
+  int gates;    // kdn_gates_t: post-activation gates or their logits
+  float rmin;   // observation-noise floor of the logit parameterisation
   float mu, tau;
   // forward inputs / outputs
   const void *q, *k, *v, *g, *omega, *r;

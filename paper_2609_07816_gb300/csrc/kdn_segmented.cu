@@ -44,6 +44,7 @@ __device__ __forceinline__ void renorm4(float &m00, float &m01, float &m10, floa
 // largest entry every 4 tokens (all entries are non-negative).  One warp per
 // chunk, four adjacent channels per lane (8-byte loads of a 256-byte row).
 constexpr int kCompWarps = 4;
+template <int G>  // G: logit gates (compile-time)
 __global__ void __launch_bounds__(32 * kCompWarps) k_seg_comp_diag(const Args a, float4 *comp) {
   const int lane = threadIdx.x & 31;
   const int c = blockIdx.x * kCompWarps + (threadIdx.x >> 5), bh = blockIdx.y;
@@ -64,7 +65,7 @@ __global__ void __launch_bounds__(32 * kCompWarps) k_seg_comp_diag(const Args a,
       kr[u] = *reinterpret_cast<const uint2 *>(kb + th * D + i0);
       gr[u] = *reinterpret_cast<const uint2 *>(gb + th * D + i0);
       wr[u] = *reinterpret_cast<const uint2 *>(wb + th * D + i0);
-      rr[u] = a.mu / ld<bf16>(a.r, th);
+      rr[u] = a.mu / gate_r(G, a.rmin, ld<bf16>(a.r, th));
     }
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
@@ -78,11 +79,19 @@ __global__ void __launch_bounds__(32 * kCompWarps) k_seg_comp_diag(const Args a,
       const float wv[4] = {w01.x, w01.y, w23.x, w23.y};
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
-        const float al2 = __expf(2.f * gv[q]);
+        float al2, w;
+        if (G) {
+          const float al = sigmoid_f(gv[q]);
+          al2 = al * al;
+          w = softplus_f(wv[q]);
+        } else {
+          al2 = __expf(2.f * gv[q]);
+          w = wv[q];
+        }
         const float uu = rr[u] * kv[q] * kv[q];
         // rows of M_t: [al2, w] and u * [al2, w] + [0, 1]
-        const float n00 = al2 * m[q][0] + wv[q] * m[q][2];
-        const float n01 = al2 * m[q][1] + wv[q] * m[q][3];
+        const float n00 = al2 * m[q][0] + w * m[q][2];
+        const float n01 = al2 * m[q][1] + w * m[q][3];
         m[q][2] = fmaf(uu, n00, m[q][2]);
         m[q][3] = fmaf(uu, n01, m[q][3]);
         m[q][0] = n00;
@@ -99,6 +108,7 @@ __global__ void __launch_bounds__(32 * kCompWarps) k_seg_comp_diag(const Args a,
 
 // Isotropic KDN: one thread per token forms M_t; the 64 matrices are multiplied
 // in order by a shuffle tree within each warp, then the two warp products.
+template <int G>  // G: logit gates (compile-time)
 __global__ void __launch_bounds__(CM) k_seg_comp_iso(const Args a, float4 *comp) {
   const int c = blockIdx.x, bh = blockIdx.y, b = bh / a.H, h = bh % a.H;
   const int tid = threadIdx.x, lane = tid & 31;
@@ -126,14 +136,26 @@ __global__ void __launch_bounds__(CM) k_seg_comp_iso(const Args a, float4 *comp)
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
         const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&wv[q]));
-        al2 += __expf(2.f * f.x) + __expf(2.f * f.y);
+        if (G) {
+          const float ax = sigmoid_f(f.x), ay = sigmoid_f(f.y);
+          al2 += ax * ax + ay * ay;
+        } else {
+          al2 += __expf(2.f * f.x) + __expf(2.f * f.y);
+        }
       }
     }
     al2 *= 1.f / D;
   } else {
-    al2 = __expf(2.f * ld<bf16>(a.g, th));
+    const float x = ld<bf16>(a.g, th);
+    if (G) {
+      const float al = sigmoid_f(x);
+      al2 = al * al;
+    } else {
+      al2 = __expf(2.f * x);
+    }
   }
-  const float w = ld<bf16>(a.omega, th), r = ld<bf16>(a.r, th);
+  const float w = gate_omega(G, ld<bf16>(a.omega, th));
+  const float r = gate_r(G, a.rmin, ld<bf16>(a.r, th));
   const float uu = a.mu * n2 / ((float)a.dk * r);
   float m00 = al2, m01 = w, m10 = uu * al2, m11 = fmaf(uu, w, 1.f);
   renorm4(m00, m01, m10, m11);
@@ -302,10 +324,11 @@ kdn_status_t launch_seg_fwd(const Args &a, int P, char *ws, cudaStream_t s) {
   // uncertainty entering every segment
   const dim3 gc((unsigned)NC, (unsigned)BH);
   if (a.variant == 0)
-    k_seg_comp_diag<<<dim3((unsigned)((NC + kCompWarps - 1) / kCompWarps), (unsigned)BH),
-                      32 * kCompWarps, 0, s>>>(a, comp);
+    (a.gates ? k_seg_comp_diag<1> : k_seg_comp_diag<0>)
+        <<<dim3((unsigned)((NC + kCompWarps - 1) / kCompWarps), (unsigned)BH), 32 * kCompWarps,
+           0, s>>>(a, comp);
   else
-    k_seg_comp_iso<<<gc, CM, 0, s>>>(a, comp);
+    (a.gates ? k_seg_comp_iso<1> : k_seg_comp_iso<0>)<<<gc, CM, 0, s>>>(a, comp);
   k_seg_scan<<<(unsigned)BH, D * kScanGroups, 0, s>>>(a, comp, (int)(NC / P), pseg);
   if (cudaGetLastError() != cudaSuccess) return KDN_ERR_CUDA;
 

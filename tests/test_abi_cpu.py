@@ -79,14 +79,23 @@ def test_rejects_bad_descriptors_before_launch(kdn):
         (dict(out_dtype=3), kdn.KDN_ERR_INVALID_ARG),
         (dict(mu=math.nan), kdn.KDN_ERR_INVALID_ARG),
         (dict(scale=math.inf), kdn.KDN_ERR_INVALID_ARG),
+        (dict(gates=2), kdn.KDN_ERR_INVALID_ARG),
+        (dict(gates=-1), kdn.KDN_ERR_INVALID_ARG),
+        (dict(gates=kdn.KDN_GATES_LOGITS, r_min=-0.01), kdn.KDN_ERR_INVALID_ARG),
+        (dict(gates=kdn.KDN_GATES_LOGITS, r_min=math.inf), kdn.KDN_ERR_INVALID_ARG),
+        (dict(gates=kdn.KDN_GATES_LOGITS, r_min=math.nan), kdn.KDN_ERR_INVALID_ARG),
     ]
     for over, want in cases:
         kw = dict(B=1, T=10, H=1, dk=32, dv=32, dtype=kdn.KDN_F32)
         kw.update(over)
         d = kdn.make_desc(kw["B"], kw["T"], kw["H"], kw["dk"], kw["dv"], kw["dtype"],
                           chunk=kw.get("chunk", 0), mu=kw.get("mu"), scale=kw.get("scale"),
-                          out_dtype=kw.get("out_dtype", 0))
+                          out_dtype=kw.get("out_dtype", 0), gates=kw.get("gates", 0),
+                          r_min=kw.get("r_min", 0.01))
         assert _fwd(kdn, d) == want, over
+    # r_min is not read with post-activation gates
+    d = kdn.make_desc(1, 10, 1, 32, 32, kdn.KDN_F32, r_min=math.nan)
+    assert kdn.workspace_bytes(d, 0) > 0
 
 
 def test_rejects_null_and_misaligned_pointers(kdn):

@@ -497,3 +497,58 @@ def test_p9_backward_matches_torch_autograd(variant, per_channel):
                   ("r", "dr"), ("S0", "dS0"), ("p0", "dp0")):
         np.testing.assert_allclose(an[gn], tt[n].grad.numpy(), rtol=1e-9, atol=1e-12,
                                    err_msg=n)
+
+
+# --------------------------------------------------------------------------
+# Gate parameterisation (eq. kla-box-parameterization): logits in, logit gradients out
+
+
+def _logit_inputs(variant, per_channel, seed):
+    """Logits whose activations look like the workload's gates: x ~ N(2, 1) for the
+    decay, y, z ~ N(0, 1) for the noises."""
+    ins = make_inputs(variant, 1, 9, 2, 3, 2, dtype="f32", seed=seed, s0_std=0.4,
+                      p0_range=(0.5, 2.0), per_channel_decay=per_channel, with_grad=True)
+    rng = np.random.default_rng(seed + 1)
+    ins["g"] = rng.normal(2.0, 1.0, ins["g"].shape)
+    ins["omega"] = rng.normal(0.0, 1.0, ins["omega"].shape)
+    ins["r"] = rng.normal(0.0, 1.0, ins["r"].shape)
+    return ins
+
+
+def test_gate_activations_special_values():
+    """sigmoid(0) = 1/2, softplus(0) = log 2, softplus(z) -> z for large z and
+    -> e^z for very negative z, r_min the floor of r; log alpha <= 0."""
+    x = np.array([0.0, 40.0, -40.0, 3.0])
+    g, w, r = oracle.gates_from_logits(x, x, x, 0.01)
+    assert np.allclose(np.exp(g), [0.5, 1.0, np.exp(-40.0), 1 / (1 + np.exp(-3.0))], rtol=1e-14,
+                       atol=0)
+    assert np.allclose(w, [np.log(2.0), 40.0, np.exp(-40.0), np.log1p(np.exp(3.0))], rtol=1e-14)
+    assert np.allclose(r - 0.01, w, rtol=1e-14) and np.all(r > 0.01) and np.all(g <= 0)
+
+
+@pytest.mark.parametrize("variant,per_channel", [("diag", True), ("iso", True), ("iso", False)])
+def test_gate_logits_backward_finite_differences(variant, per_channel):
+    """The logit gradients (the adjoint through sigmoid / softplus / r_min +
+    softplus) agree with central differences of the logit-mode forward."""
+    ins = _logit_inputs(variant, per_channel, 53)
+    rng = np.random.default_rng(9)
+    wS = rng.standard_normal(ins["S0"].shape)
+    wp = rng.standard_normal(ins["p0"].shape)
+
+    def f(d):
+        res = oracle.fwd(variant, d["q"], d["k"], d["v"], d["g"], d["omega"], d["r"], d["S0"],
+                         d["p0"], gates="logits", r_min=0.05)
+        return np.sum(ins["dO"] * res["o"]) + np.sum(wS * res["ST"]) + np.sum(wp * res["pT"])
+
+    an = oracle.bwd(variant, ins["q"], ins["k"], ins["v"], ins["g"], ins["omega"], ins["r"],
+                    ins["S0"], ins["p0"], ins["dO"], wS, wp, gates="logits", r_min=0.05)
+    h = 1e-6
+    for n, gn in (("g", "dg"), ("omega", "domega"), ("r", "dr"), ("k", "dk")):
+        x = ins[n]
+        fd = np.zeros_like(x)
+        for idx in np.ndindex(x.shape):
+            xp = dict(ins); xp[n] = x.copy(); xp[n][idx] += h
+            xm = dict(ins); xm[n] = x.copy(); xm[n][idx] -= h
+            fd[idx] = (f(xp) - f(xm)) / (2 * h)
+        err = np.max(np.abs(fd - an[gn])) / max(np.max(np.abs(fd)), 1e-30)
+        assert err < 1e-6, (n, err)
