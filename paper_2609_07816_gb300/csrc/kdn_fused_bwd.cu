@@ -716,7 +716,7 @@ __global__ void __launch_bounds__(BT, 1)
     // ---- [18] per channel (lane ci, tokens t0..t0+15): back through Gamma and the
     //           gain emission, then the uncertainty recursion backwards in time.
     //           Free TMEM columns hold per-(channel, token) intermediates between passes:
-    //           X2 <- dphat (gain part), X1 <- dk (memory + gain part), X0 <- alpha^2,
+    //           X2 <- dphat (gain part), X1 <- dk (memory + gain part), X0 <- alpha,
     //           X3 <- 1 / (1 + u phat).
     if (V == 0)
     {
@@ -805,7 +805,7 @@ __global__ void __launch_bounds__(BT, 1)
             const float aj = al2 * rd * rd;
             Bv = aj * Bv + al2 * dphl;
             A = aj * A;
-            a2v[u] = al2;
+            a2v[u] = al;  // alpha (the last pass squares it again)
             rdv[u] = rd;
             c1[u] = dphl;
           }
@@ -826,6 +826,14 @@ __global__ void __launch_bounds__(BT, 1)
         float run = dgC * s_gC[ci];  // dG_63 gains dgamma_C gamma_C; it lies in every suffix
         for (int q2 = qq + 1; q2 < 4; ++q2) run += s_tot[q2 * D + ci];
         float rd16[16], drp[16];
+        // logit gates: the quarter's omega logits, loaded together for the chain
+        // factor sigmoid(y) of domega
+        float ylog[16];
+        if (G) {
+#pragma unroll
+          for (int j = 0; j < 16; ++j)
+            ylog[j] = j < nval ? ld<__nv_bfloat16>(a.omega, obase + (size_t)j * ostride) : 0.f;
+        }
         tmem_ld16(X3 + lane_base + t0, rd16);
 #pragma unroll
         for (int h8 = 1; h8 >= 0; --h8) {
@@ -844,16 +852,17 @@ __global__ void __launch_bounds__(BT, 1)
             const float dkt = c2[u] + 2.f * ds * ph[j] * kk + du * 2.f * mu * kk * ri;
             drp[j] = -du * mu * kk * kk * ri * ri;
             run += sdg[j * BT + tid];
-            const float dgt = run + 2.f * a2v[u] * pprev * dph;
+            const float al2 = a2v[u] * a2v[u];
+            const float dgt = run + 2.f * al2 * pprev * dph;
             if (j < nval) {
               // logit gates: d omega / dy = sigmoid(y), d log alpha / dx = 1 - alpha
-              const float fw = G ? sigmoid_f(ld<__nv_bfloat16>(a.omega, obase + (size_t)j * ostride)) : 1.f;
-              const float fg = G ? 1.f - sqrtf(a2v[u]) : 1.f;
+              const float fw = G ? sigmoid_f(ylog[j]) : 1.f;
+              const float fg = G ? 1.f - a2v[u] : 1.f;
               out(a.dk_, j, dkt * invl);
               out(a.domega, j, dph * fw * invl);
               out(a.dg, j, dgt * fg * invl);
             }
-            dp = a2v[u] * dph;
+            dp = al2 * dph;
           }
         }
         const float rs2 = rs16(drp, lane);

@@ -37,10 +37,14 @@ __device__ __forceinline__ void sto(int odt, void *p, size_t i, float x) {
 
 // Gate activations of the layer's parameterisation for KDN_GATES_LOGITS
 // inputs: alpha = sigmoid(x), omega = softplus(y), r = r_min + softplus(z).
+// softplus(x) = max(x, 0) + log1p(u), u = exp(-|x|) in (0, 1]: the fast logarithm
+// of 1 + u, or for small u the series u - u^2/2 + u^3/3 (error below u^4 / 4)
 __device__ __forceinline__ float softplus_f(float x) {
-  return fmaxf(x, 0.f) + log1pf(__expf(-fabsf(x)));
+  const float u = __expf(-fabsf(x));
+  const float lp = u < 1e-3f ? u * (1.f - u * (0.5f - u * (1.f / 3.f))) : __logf(1.f + u);
+  return fmaxf(x, 0.f) + lp;
 }
-__device__ __forceinline__ float sigmoid_f(float x) { return 1.f / (1.f + __expf(-x)); }
+__device__ __forceinline__ float sigmoid_f(float x) { return __fdividef(1.f, 1.f + __expf(-x)); }
 // log alpha from the gate input: g itself, or log sigmoid(x) = -softplus(-x)
 __device__ __forceinline__ float gate_logalpha(int gates, float g) {
   return gates ? -softplus_f(-g) : g;
