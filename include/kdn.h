@@ -147,14 +147,18 @@ kdn_status_t kdn_iso_fwd(const kdn_desc_t *desc, const void *q, const void *k,
 
 /* Backward: gradients of <dO, o> + <dST, ST> + <dpT, pT> with respect to every
    forward input.  It recomputes the forward from the inputs (no saved
-   context).  dST / dpT NULL -> zero cotangent.  dS0 / dp0 NULL -> not written;
-   all other gradient pointers are required. */
+   context).  dST / dpT NULL -> zero cotangent.  dS0 / dp0 / dmu NULL -> not
+   written; all other gradient pointers are required.  dmu [B,H] float32: the
+   gradient with respect to the information scale mu of each sequence (mu
+   enters only through u of eq. diag-cov-update / Prop. 5); a mu shared by all
+   sequences has the sum.  The gradient of a learned initial uncertainty
+   c_{0,h} (p_0 = c_{0,h} in every channel) is the per-head sum of dp0. */
 kdn_status_t kdn_diag_bwd(const kdn_desc_t *desc, const void *q, const void *k,
                           const void *v, const void *g, const void *omega,
                           const void *r, const float *S0, const float *p0,
                           const void *dO, const float *dST, const float *dpT,
                           void *dq, void *dk, void *dv, void *dg, void *domega,
-                          void *dr, float *dS0, float *dp0, void *workspace,
+                          void *dr, float *dS0, float *dp0, float *dmu, void *workspace,
                           size_t workspace_bytes, void *stream);
 
 kdn_status_t kdn_iso_bwd(const kdn_desc_t *desc, const void *q, const void *k,
@@ -162,7 +166,7 @@ kdn_status_t kdn_iso_bwd(const kdn_desc_t *desc, const void *q, const void *k,
                          const void *r, const float *S0, const float *p0,
                          const void *dO, const float *dST, const float *dpT,
                          void *dq, void *dk, void *dv, void *dg, void *domega,
-                         void *dr, float *dS0, float *dp0, void *workspace,
+                         void *dr, float *dS0, float *dp0, float *dmu, void *workspace,
                          size_t workspace_bytes, void *stream);
 
 /* Training pair.  kdn_diag_fwd_save is kdn_diag_fwd that also keeps, in
@@ -198,7 +202,7 @@ kdn_status_t kdn_diag_bwd_saved(const kdn_desc_t *desc, const void *q,
                                 const void *dO, const float *dST,
                                 const float *dpT, void *dq, void *dk, void *dv,
                                 void *dg, void *domega, void *dr, float *dS0,
-                                float *dp0, void *workspace,
+                                float *dp0, float *dmu, void *workspace,
                                 size_t workspace_bytes, void *stream);
 
 kdn_status_t kdn_iso_fwd_save(const kdn_desc_t *desc, const void *q,
@@ -216,7 +220,7 @@ kdn_status_t kdn_iso_bwd_saved(const kdn_desc_t *desc, const void *q,
                                const void *dO, const float *dST,
                                const float *dpT, void *dq, void *dk, void *dv,
                                void *dg, void *domega, void *dr, float *dS0,
-                               float *dp0, void *workspace,
+                               float *dp0, float *dmu, void *workspace,
                                size_t workspace_bytes, void *stream);
 
 /* One decode token for all B*H heads (the update of Prop. 3), in place:

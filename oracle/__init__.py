@@ -53,7 +53,7 @@ def _load():
             D = ctypes.c_double
             lib.kdn_oracle_fwd.argtypes = [I, I, I, I, I, I, D, D, I] + [P] * 15 + [I]
             lib.kdn_oracle_fwd.restype = I
-            lib.kdn_oracle_bwd.argtypes = [I, I, I, I, I, I, D, D, I] + [P] * 20 + [I]
+            lib.kdn_oracle_bwd.argtypes = [I, I, I, I, I, I, D, D, I] + [P] * 21 + [I]
             lib.kdn_oracle_bwd.restype = I
             _lib = lib
     return _lib
@@ -146,7 +146,8 @@ def fwd(variant, q, k, v, g, omega, r, S0=None, p0=None, *, mu=None, scale=None,
 
 def bwd(variant, q, k, v, g, omega, r, S0, p0, dO, dST=None, dpT=None, *, mu=None,
         scale=None, bhat=None, threads=0, gates="post", r_min=0.01):
-    """Gradients of <dO, o> + <dST, ST> + <dpT, pT> with respect to every input.
+    """Gradients of <dO, o> + <dST, ST> + <dpT, pT> with respect to every input,
+    and ``dmu`` [B,H]: with respect to the information scale mu of each sequence.
 
     ``gates="logits"``: g, omega, r are logits, and dg, domega, dr are the
     gradients with respect to them (chain rule through ``gates_from_logits``:
@@ -173,13 +174,13 @@ def bwd(variant, q, k, v, g, omega, r, S0, p0, dO, dST=None, dpT=None, *, mu=Non
     out = dict(dq=np.zeros_like(q), dk=np.zeros_like(k), dv=np.zeros_like(v),
                dg=np.zeros_like(g), domega=np.zeros_like(omega), dr=np.zeros_like(r),
                dS0=np.zeros((B, H, dk, dv)),
-               dp0=np.zeros((B, H, dk) if vid == 0 else (B, H)))
+               dp0=np.zeros((B, H, dk) if vid == 0 else (B, H)), dmu=np.zeros((B, H)))
     n = lib.kdn_oracle_bwd(vid, B, T, H, dk, dv, mu, scale, per_channel,
                            _ptr(q), _ptr(k), _ptr(v), _ptr(g), _ptr(omega), _ptr(r),
                            _ptr(S0), _ptr(p0), _ptr(bhat), _ptr(dO), _ptr(dST), _ptr(dpT),
                            _ptr(out["dq"]), _ptr(out["dk"]), _ptr(out["dv"]),
                            _ptr(out["dg"]), _ptr(out["domega"]), _ptr(out["dr"]),
-                           _ptr(out["dS0"]), _ptr(out["dp0"]), int(threads))
+                           _ptr(out["dS0"]), _ptr(out["dp0"]), _ptr(out["dmu"]), int(threads))
     if n < 0:
         raise ValueError("oracle rejected the arguments")
     out["threads"] = n

@@ -66,6 +66,7 @@ typedef struct {
   /* backward */
   const double *dO, *dST, *dpT;
   double *dq, *dk_, *dv_, *dg, *domega, *dr, *dS0, *dp0;
+  double *dmu; /* [B,H] dL/dmu of each sequence (mu enters only through u), or NULL */
 } job_t;
 
 /* Per-token intermediates of one forward step, kept for the adjoint. */
@@ -244,6 +245,7 @@ static void bwd_step(const job_t *J, int b, int t, int h, const double *Sprev,
       /* u = mu k^2 / r */
       dkt[i] += du * 2.0 * J->mu * kt[i] / rt;
       dr += -du * st->u[i] / rt;
+      if (J->dmu) J->dmu[(size_t)b * J->H + h] += du * kt[i] * kt[i] / rt;
     }
   }
   double dbhat = 0.0, dn2 = 0.0;
@@ -255,6 +257,7 @@ static void bwd_step(const job_t *J, int b, int t, int h, const double *Sprev,
     /* u = mu n2 / (dk r) */
     dn2 += du * J->mu / (dk * rt);
     dr += -du * st->u[0] / rt;
+    if (J->dmu) J->dmu[(size_t)b * J->H + h] += du * st->n2 / (dk * rt);
   }
 
   /* residual write S_t = Shat + kappa delta^T, delta = v - Shat^T k */
@@ -369,6 +372,7 @@ static void bwd_one(const job_t *J, int b, int h) {
   }
 
   const size_t bh = (size_t)b * J->H + h;
+  if (J->dmu) J->dmu[bh] = 0.0;
   for (size_t e = 0; e < sz; ++e) dS[e] = J->dST ? J->dST[bh * sz + e] : 0.0;
   for (int i = 0; i < np; ++i) dp[i] = J->dpT ? J->dpT[bh * np + i] : 0.0;
 
@@ -472,7 +476,8 @@ int kdn_oracle_fwd(int variant, int B, int T, int H, int dk, int dv, double mu,
 }
 
 /* Backward (adjoint of the forward token loop).  dST / dpT may be NULL (zero
-   cotangent).  dS0 / dp0 may be NULL. */
+   cotangent).  dS0 / dp0 may be NULL.  dmu (may be NULL) [B,H] receives dL/dmu of each
+   sequence: mu enters only through u, so dmu = sum_t sum_i du_{t,i} u_{t,i} / mu. */
 int kdn_oracle_bwd(int variant, int B, int T, int H, int dk, int dv, double mu,
                    double tau, int per_channel_decay, const double *q,
                    const double *k, const double *v, const double *g,
@@ -480,7 +485,7 @@ int kdn_oracle_bwd(int variant, int B, int T, int H, int dk, int dv, double mu,
                    const double *p0, const double *bhat_in, const double *dO,
                    const double *dST, const double *dpT, double *dq, double *dk_,
                    double *dv_, double *dg, double *domega, double *dr,
-                   double *dS0, double *dp0, int nthreads) {
+                   double *dS0, double *dp0, double *dmu, int nthreads) {
   if (check(variant, B, T, H, dk, dv)) return -1;
   job_t J;
   memset(&J, 0, sizeof J);
@@ -490,6 +495,6 @@ int kdn_oracle_bwd(int variant, int B, int T, int H, int dk, int dv, double mu,
   J.bhat_in = variant == 1 ? bhat_in : NULL;
   J.dO = dO; J.dST = dST; J.dpT = dpT;
   J.dq = dq; J.dk_ = dk_; J.dv_ = dv_; J.dg = dg; J.domega = domega; J.dr = dr;
-  J.dS0 = dS0; J.dp0 = dp0;
+  J.dS0 = dS0; J.dp0 = dp0; J.dmu = dmu;
   return run(&J, 1, nthreads);
 }

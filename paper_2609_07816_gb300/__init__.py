@@ -58,19 +58,19 @@ _SIG = {
     "kdn_bwd_workspace_bytes": ([ctypes.POINTER(kdn_desc_t), ctypes.c_int], ctypes.c_size_t),
     "kdn_diag_fwd": ([ctypes.POINTER(kdn_desc_t)] + [_P] * 12 + [ctypes.c_size_t, _P], ctypes.c_int),
     "kdn_iso_fwd": ([ctypes.POINTER(kdn_desc_t)] + [_P] * 12 + [ctypes.c_size_t, _P], ctypes.c_int),
-    "kdn_diag_bwd": ([ctypes.POINTER(kdn_desc_t)] + [_P] * 20 + [ctypes.c_size_t, _P], ctypes.c_int),
-    "kdn_iso_bwd": ([ctypes.POINTER(kdn_desc_t)] + [_P] * 20 + [ctypes.c_size_t, _P], ctypes.c_int),
+    "kdn_diag_bwd": ([ctypes.POINTER(kdn_desc_t)] + [_P] * 21 + [ctypes.c_size_t, _P], ctypes.c_int),
+    "kdn_iso_bwd": ([ctypes.POINTER(kdn_desc_t)] + [_P] * 21 + [ctypes.c_size_t, _P], ctypes.c_int),
     "kdn_diag_decode_step": ([ctypes.POINTER(kdn_desc_t)] + [_P] * 10, ctypes.c_int),
     "kdn_iso_decode_step": ([ctypes.POINTER(kdn_desc_t)] + [_P] * 10, ctypes.c_int),
     "kdn_diag_fwd_noalloc": ([ctypes.POINTER(kdn_desc_t)] + [_P] * 12, ctypes.c_int),
     "kdn_saved_bytes": ([ctypes.POINTER(kdn_desc_t), ctypes.c_int], ctypes.c_size_t),
     "kdn_diag_fwd_save": ([ctypes.POINTER(kdn_desc_t)] + [_P] * 12 + [ctypes.c_size_t, _P,
                                                                    ctypes.c_size_t, _P], ctypes.c_int),
-    "kdn_diag_bwd_saved": ([ctypes.POINTER(kdn_desc_t)] + [_P] * 7 + [ctypes.c_size_t] + [_P] * 12
+    "kdn_diag_bwd_saved": ([ctypes.POINTER(kdn_desc_t)] + [_P] * 7 + [ctypes.c_size_t] + [_P] * 13
                            + [ctypes.c_size_t, _P], ctypes.c_int),
     "kdn_iso_fwd_save": ([ctypes.POINTER(kdn_desc_t)] + [_P] * 12 + [ctypes.c_size_t, _P,
                                                                   ctypes.c_size_t, _P], ctypes.c_int),
-    "kdn_iso_bwd_saved": ([ctypes.POINTER(kdn_desc_t)] + [_P] * 7 + [ctypes.c_size_t] + [_P] * 12
+    "kdn_iso_bwd_saved": ([ctypes.POINTER(kdn_desc_t)] + [_P] * 7 + [ctypes.c_size_t] + [_P] * 13
                           + [ctypes.c_size_t, _P], ctypes.c_int),
     "kdn_kernel_launches": ([ctypes.POINTER(kdn_desc_t), ctypes.c_int, ctypes.c_int], ctypes.c_int),
     "kdn_get_device_status": ([_P, _P], ctypes.c_int),
@@ -207,6 +207,7 @@ def _bwd(name, variant, q, k, v, g, omega, r, S0, p0, dO, dST, dpT, *, chunk, mu
             grads["dS0"] = torch.empty(B, H, dk, dv, dtype=torch.float32, device=dev)
             grads["dp0"] = torch.empty((B, H, dk) if variant == 0 else (B, H),
                                        dtype=torch.float32, device=dev)
+            grads["dmu"] = torch.empty(B, H, dtype=torch.float32, device=dev)
     if workspace is None:
         workspace = alloc_workspace(desc, variant, True, dev)
     G = grads
@@ -214,7 +215,8 @@ def _bwd(name, variant, q, k, v, g, omega, r, S0, p0, dO, dST, dpT, *, chunk, mu
                               _ptr(omega), _ptr(r), _ptr(S0), _ptr(p0), _ptr(dO), _ptr(dST),
                               _ptr(dpT), _ptr(G["dq"]), _ptr(G["dk"]), _ptr(G["dv"]),
                               _ptr(G["dg"]), _ptr(G["domega"]), _ptr(G["dr"]),
-                              _ptr(G.get("dS0")), _ptr(G.get("dp0")), _ptr(workspace),
+                              _ptr(G.get("dS0")), _ptr(G.get("dp0")), _ptr(G.get("dmu")),
+                              _ptr(workspace),
                               workspace.numel(), _stream(stream))
     _check(st, name)
     return grads
@@ -224,7 +226,8 @@ def kdn_diag_bwd(q, k, v, g, omega, r, S0, p0, dO, dST=None, dpT=None, *, chunk=
                  scale=None, grads=None, want_state_grads=True, workspace=None, stream=None,
                  out_dtype=torch.float32, gates=KDN_GATES_POST,
                  r_min=R_MIN_DEFAULT):
-    """Gradients of the Diagonal KDN forward.  Returns a dict dq, dk, dv, dg, domega, dr, dS0, dp0."""
+    """Gradients of the Diagonal KDN forward.  Returns a dict dq, dk, dv, dg, domega, dr,
+    and with want_state_grads dS0, dp0 and dmu [B,H] (the gradient with respect to mu)."""
     return _bwd("kdn_diag_bwd", 0, q, k, v, g, omega, r, S0, p0, dO, dST, dpT, chunk=chunk,
                 mu=mu, scale=scale, grads=grads, want_state_grads=want_state_grads,
                 workspace=workspace, stream=stream, out_dtype=out_dtype,
@@ -311,6 +314,7 @@ def _bwd_saved(name, variant, q, k, v, g, omega, r, saved, dO, dST, dpT, *, mu, 
             grads["dS0"] = torch.empty(B, H, dk, dv, dtype=torch.float32, device=dev)
             grads["dp0"] = torch.empty((B, H, dk) if variant == 0 else (B, H),
                                        dtype=torch.float32, device=dev)
+            grads["dmu"] = torch.empty(B, H, dtype=torch.float32, device=dev)
     if workspace is None:
         workspace = alloc_workspace(desc, variant, False, dev)
     G = grads
@@ -318,7 +322,8 @@ def _bwd_saved(name, variant, q, k, v, g, omega, r, saved, dO, dST, dpT, *, mu, 
                               _ptr(omega), _ptr(r), _ptr(saved), saved.numel(), _ptr(dO),
                               _ptr(dST), _ptr(dpT), _ptr(G["dq"]), _ptr(G["dk"]),
                               _ptr(G["dv"]), _ptr(G["dg"]), _ptr(G["domega"]), _ptr(G["dr"]),
-                              _ptr(G.get("dS0")), _ptr(G.get("dp0")), _ptr(workspace),
+                              _ptr(G.get("dS0")), _ptr(G.get("dp0")), _ptr(G.get("dmu")),
+                              _ptr(workspace),
                               workspace.numel(), _stream(stream))
     _check(st, name)
     return grads

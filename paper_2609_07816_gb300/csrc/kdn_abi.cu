@@ -103,6 +103,8 @@ kdn_status_t empty_fwd(const Args &a, cudaStream_t s) {
 
 kdn_status_t empty_bwd(const Args &a, cudaStream_t s) {
   const size_t ns = (size_t)a.B * a.H * a.dk * a.dv, np = (size_t)a.B * a.H * a.P;
+  if (a.dmu && cudaMemsetAsync(a.dmu, 0, (size_t)a.B * a.H * sizeof(float), s) != cudaSuccess)
+    return KDN_ERR_CUDA;
   if (a.dS0) {
     cudaError_t e = a.dST ? cudaMemcpyAsync(a.dS0, a.dST, ns * 4, cudaMemcpyDeviceToDevice, s)
                           : cudaMemsetAsync(a.dS0, 0, ns * 4, s);
@@ -148,28 +150,31 @@ kdn_status_t bwd_entry(int variant, const kdn_desc_t *d, const void *q, const vo
                        const void *v, const void *g, const void *omega, const void *r,
                        const float *S0, const float *p0, const void *dO, const float *dST,
                        const float *dpT, void *dq, void *dk, void *dv, void *dg, void *domega,
-                       void *dr, float *dS0, float *dp0, void *ws, size_t ws_bytes,
-                       void *stream) {
+                       void *dr, float *dS0, float *dp0, float *dmu, void *ws,
+                       size_t ws_bytes, void *stream) {
   Args a;
   kdn_status_t st = fill_sizes(d, variant, false, &a);
   if (st != KDN_OK) return st;
   const bool work = (size_t)a.B * a.H * a.T > 0;
   if (work && !ptrs_ok({q, k, v, g, omega, r, dO, dq, dk, dv, dg, domega, dr},
-                       {S0, p0, dST, dpT, dS0, dp0}))
+                       {S0, p0, dST, dpT, dS0, dp0, dmu}))
     return KDN_ERR_INVALID_ARG;
-  if (!work && !ptrs_ok({}, {S0, p0, dST, dpT, dS0, dp0})) return KDN_ERR_INVALID_ARG;
+  if (!work && !ptrs_ok({}, {S0, p0, dST, dpT, dS0, dp0, dmu})) return KDN_ERR_INVALID_ARG;
   const size_t need = workspace_layout(&a, nullptr, true);
   if (need > ws_bytes || (need && (!ws || ((uintptr_t)ws % kAlign)))) return KDN_ERR_WORKSPACE;
   workspace_layout(&a, static_cast<char *>(ws), true);
   a.q = q; a.k = k; a.v = v; a.g = g; a.omega = omega; a.r = r; a.S0 = S0; a.p0 = p0;
   a.dO = dO; a.dST = dST; a.dpT = dpT;
   a.dq = dq; a.dk_ = dk; a.dv_ = dv; a.dg = dg; a.domega = domega; a.dr = dr;
-  a.dS0 = dS0; a.dp0 = dp0;
+  a.dS0 = dS0; a.dp0 = dp0; a.dmu = dmu;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   if (cudaMemsetAsync(a.status, 0, sizeof(unsigned), s) != cudaSuccess) return KDN_ERR_CUDA;
   if ((size_t)a.B * a.H == 0) return KDN_OK;
   if (a.T == 0) return empty_bwd(a, s);
   if (use_fused_bwd(a)) return launch_fused_bwd(a, s);
+  // the general kernels accumulate dmu with atomics
+  if (a.dmu && cudaMemsetAsync(a.dmu, 0, (size_t)a.B * a.H * sizeof(float), s) != cudaSuccess)
+    return KDN_ERR_CUDA;
   return launch_chunked_bwd(a, s);
 }
 
@@ -206,17 +211,17 @@ kdn_status_t bwd_saved_entry(int variant, const kdn_desc_t *d, const void *q, co
                              const void *g, const void *omega, const void *r, const void *saved,
                              size_t saved_bytes, const void *dO, const float *dST,
                              const float *dpT, void *dq, void *dk, void *dv, void *dg,
-                             void *domega, void *dr, float *dS0, float *dp0, void *ws,
-                             size_t ws_bytes, void *stream) {
+                             void *domega, void *dr, float *dS0, float *dp0, float *dmu,
+                             void *ws, size_t ws_bytes, void *stream) {
   Args a;
   kdn_status_t st = fill_sizes(d, variant, false, &a);
   if (st != KDN_OK) return st;
   const bool work = (size_t)a.B * a.H * a.T > 0;
   if (work && !use_fused_bwd(a)) return KDN_ERR_UNSUPPORTED;
   if (work && !ptrs_ok({q, k, v, g, omega, r, saved, dO, dq, dk, dv, dg, domega, dr},
-                       {dST, dpT, dS0, dp0}))
+                       {dST, dpT, dS0, dp0, dmu}))
     return KDN_ERR_INVALID_ARG;
-  if (!work && !ptrs_ok({}, {dST, dpT, dS0, dp0})) return KDN_ERR_INVALID_ARG;
+  if (!work && !ptrs_ok({}, {dST, dpT, dS0, dp0, dmu})) return KDN_ERR_INVALID_ARG;
   if (work && (saved_bytes < fused_saved_bytes(a) || ((uintptr_t)saved % kAlign)))
     return KDN_ERR_WORKSPACE;
   const size_t need = workspace_layout(&a, nullptr, false);
@@ -225,7 +230,7 @@ kdn_status_t bwd_saved_entry(int variant, const kdn_desc_t *d, const void *q, co
   a.q = q; a.k = k; a.v = v; a.g = g; a.omega = omega; a.r = r;
   a.dO = dO; a.dST = dST; a.dpT = dpT;
   a.dq = dq; a.dk_ = dk; a.dv_ = dv; a.dg = dg; a.domega = domega; a.dr = dr;
-  a.dS0 = dS0; a.dp0 = dp0;
+  a.dS0 = dS0; a.dp0 = dp0; a.dmu = dmu;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   if (cudaMemsetAsync(a.status, 0, sizeof(unsigned), s) != cudaSuccess) return KDN_ERR_CUDA;
   if ((size_t)a.B * a.H == 0) return KDN_OK;
@@ -349,20 +354,20 @@ kdn_status_t kdn_diag_bwd(const kdn_desc_t *desc, const void *q, const void *k, 
                           const void *g, const void *omega, const void *r, const float *S0,
                           const float *p0, const void *dO, const float *dST, const float *dpT,
                           void *dq, void *dk, void *dv, void *dg, void *domega, void *dr,
-                          float *dS0, float *dp0, void *workspace, size_t workspace_bytes,
-                          void *stream) {
+                          float *dS0, float *dp0, float *dmu, void *workspace,
+                          size_t workspace_bytes, void *stream) {
   return bwd_entry(0, desc, q, k, v, g, omega, r, S0, p0, dO, dST, dpT, dq, dk, dv, dg, domega,
-                   dr, dS0, dp0, workspace, workspace_bytes, stream);
+                   dr, dS0, dp0, dmu, workspace, workspace_bytes, stream);
 }
 
 kdn_status_t kdn_iso_bwd(const kdn_desc_t *desc, const void *q, const void *k, const void *v,
                          const void *g, const void *omega, const void *r, const float *S0,
                          const float *p0, const void *dO, const float *dST, const float *dpT,
                          void *dq, void *dk, void *dv, void *dg, void *domega, void *dr,
-                         float *dS0, float *dp0, void *workspace, size_t workspace_bytes,
-                         void *stream) {
+                         float *dS0, float *dp0, float *dmu, void *workspace,
+                         size_t workspace_bytes, void *stream) {
   return bwd_entry(1, desc, q, k, v, g, omega, r, S0, p0, dO, dST, dpT, dq, dk, dv, dg, domega,
-                   dr, dS0, dp0, workspace, workspace_bytes, stream);
+                   dr, dS0, dp0, dmu, workspace, workspace_bytes, stream);
 }
 
 size_t kdn_saved_bytes(const kdn_desc_t *desc, int variant) {
@@ -385,9 +390,10 @@ kdn_status_t kdn_diag_bwd_saved(const kdn_desc_t *desc, const void *q, const voi
                                 const void *saved, size_t saved_bytes, const void *dO,
                                 const float *dST, const float *dpT, void *dq, void *dk, void *dv,
                                 void *dg, void *domega, void *dr, float *dS0, float *dp0,
-                                void *workspace, size_t workspace_bytes, void *stream) {
+                                float *dmu, void *workspace, size_t workspace_bytes,
+                                void *stream) {
   return bwd_saved_entry(0, desc, q, k, v, g, omega, r, saved, saved_bytes, dO, dST, dpT, dq, dk, dv,
-                         dg, domega, dr, dS0, dp0, workspace, workspace_bytes, stream);
+                         dg, domega, dr, dS0, dp0, dmu, workspace, workspace_bytes, stream);
 }
 
 kdn_status_t kdn_iso_fwd_save(const kdn_desc_t *desc, const void *q, const void *k,
@@ -404,9 +410,10 @@ kdn_status_t kdn_iso_bwd_saved(const kdn_desc_t *desc, const void *q, const void
                                const void *saved, size_t saved_bytes, const void *dO,
                                const float *dST, const float *dpT, void *dq, void *dk, void *dv,
                                void *dg, void *domega, void *dr, float *dS0, float *dp0,
-                               void *workspace, size_t workspace_bytes, void *stream) {
+                               float *dmu, void *workspace, size_t workspace_bytes,
+                               void *stream) {
   return bwd_saved_entry(1, desc, q, k, v, g, omega, r, saved, saved_bytes, dO, dST, dpT, dq, dk, dv,
-                         dg, domega, dr, dS0, dp0, workspace, workspace_bytes, stream);
+                         dg, domega, dr, dS0, dp0, dmu, workspace, workspace_bytes, stream);
 }
 
 kdn_status_t kdn_diag_decode_step(const kdn_desc_t *desc, const void *q, const void *k,

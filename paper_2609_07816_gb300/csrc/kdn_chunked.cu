@@ -751,6 +751,7 @@ __global__ void __launch_bounds__(32) k_gain_bwd_diag(Args a) {
   const int bh = blockIdx.x, b = bh / a.H, h = bh % a.H;
   const int lane = threadIdx.x, i = blockIdx.y * 32 + lane, dk = a.dk;
   float dp = a.dpT ? a.dpT[(size_t)bh * dk + i] : 0.f;
+  float dmu_acc = 0.f;  // this channel's part of dL/dmu
   const size_t hrow = (size_t)bh * a.Tp;
   const float p_init = a.p0 ? a.p0[(size_t)bh * dk + i] : 1.f;
   // per token: phat, k, r, g, local dphat, dk and dg partials; blocks of GU
@@ -802,6 +803,7 @@ __global__ void __launch_bounds__(32) k_gain_bwd_diag(Args a) {
         const float den = 1.f + u * cph[j];
         const float dph = dp / (den * den) + cdl[j];
         const float du = -dp * pt[j] * pt[j];
+        dmu_acc += du * ck[j] * ck[j] / cr[j];  // u = mu k^2 / r
         const float dkk = cdk[j] + du * 2.f * a.mu * ck[j] / cr[j];
         const float drp = warp_sum(-du * u / cr[j]);
         if (lane == 0) a.drw[row * 4 + blockIdx.y] = drp;
@@ -823,6 +825,10 @@ __global__ void __launch_bounds__(32) k_gain_bwd_diag(Args a) {
     }
   }
   if (a.dp0) a.dp0[(size_t)bh * dk + i] = dp;
+  if (a.dmu) {
+    dmu_acc = warp_sum(dmu_acc);
+    if (lane == 0) atomicAdd(a.dmu + bh, dmu_acc);
+  }
 }
 
 template <typename DT>
@@ -847,6 +853,7 @@ __global__ void __launch_bounds__(32) k_gain_bwd_iso(Args a) {
   const int lane = threadIdx.x;
   __shared__ float s_ph[33], s_a[33], s_n2[33], s_r[33], s_dl[32], s_dr[32], s_o1[32], s_o2[32], s_dw[32];
   float db = a.dpT ? a.dpT[bh] : 0.f;
+  float dmu_acc = 0.f;  // dL/dmu of this sequence (lane 0)
   const size_t hrow = (size_t)bh * a.Tp;
   const int nblk = (a.T + 31) / 32;
   for (int blk = nblk - 1; blk >= 0; --blk) {
@@ -879,6 +886,7 @@ __global__ void __launch_bounds__(32) k_gain_bwd_iso(Args a) {
         const float bt = bhat / den;
         const float dbh = db / (den * den) + s_dl[j];
         const float du = -db * bt * bt;
+        dmu_acc += du * s_n2[j] / (a.dk * rr);  // u = mu |k|^2 / (dk r)
         s_dr[j] += -du * u / rr;
         float bprev;
         if (j > 0 || t > 0) {
@@ -910,6 +918,7 @@ __global__ void __launch_bounds__(32) k_gain_bwd_iso(Args a) {
     __syncwarp();
   }
   if (lane == 0 && a.dp0) a.dp0[bh] = db;
+  if (lane == 0 && a.dmu) atomicAdd(a.dmu + bh, dmu_acc);
 }
 
 // per token: dk += 2 k d|k|^2, dg += d a_t * d a_t / d g, dr -> output dtype

@@ -85,7 +85,7 @@ constexpr int O_DWT = O_G, O_DAT = O_G + 16 * KB, O_XT = O_G + 24 * KB, O_KQH2 =
 constexpr int O_QL2 = O_RDO, O_DRTL = O_RH;
 // small arrays
 constexpr int OFF_SM = BUF_END;
-constexpr int SMALL_FLOATS = 64 * 15 + 256 * 2 + 128 * 2 + 16;
+constexpr int SMALL_FLOATS = 64 * 16 + 256 * 2 + 128 * 2 + 16;
 constexpr int OFF_BAR = OFF_SM + SMALL_FLOATS * 4;
 constexpr int SMEM_BYTES = OFF_BAR + 64 + 1024;  // + alignment slack
 static_assert(SMEM_BYTES <= 232448, "shared memory");
@@ -195,6 +195,8 @@ __global__ void __launch_bounds__(BT, 1)
   float *s_da = s_dn2 + 64;     // [64] cotangent of a_t (iso)
   float *s_misc = s_da + 64;    // [0] lambda, [1..] scratch
   float *s_fr = s_misc + 16;    // [64] d r_t / d z_t (1 unless the gates are logits)
+  float *s_dmu = s_fr + 64;     // [64] parts of dL/dmu (lambda-scaled), summed at the end:
+                                //      diag one per token slot, iso one per quarter
   uint64_t *bars = reinterpret_cast<uint64_t *>(sm + OFF_BAR);
   uint64_t *bar_a = bars, *bar_b = bars + 1, *bar_mma = bars + 2;
   uint32_t *s_tbase = reinterpret_cast<uint32_t *>(bars + 4);
@@ -380,6 +382,7 @@ __global__ void __launch_bounds__(BT, 1)
   auto raw_k = [&](int t) { return bf(rkq, 16384, t, ci); };
   auto raw_q = [&](int t) { return bf(rkq + 8192, 16384, t, ci); };
 
+  if (tid < CM) s_dmu[tid] = 0.f;  // ordered before use by the loop's barriers
   for (int it = 0; it < NC && ok; ++it) {
     const int c = NC - 1 - it;
     // ---- [1] per-token scalars; the chunk's gains from the context the forward saved
@@ -872,8 +875,12 @@ __global__ void __launch_bounds__(BT, 1)
         if (tid < CM) {
           const int tt = c * CM + tid;
           if (tt < a.T) {
-            const float dr = s_ds[tid] + ((s_red2[tid] + s_red2[64 + tid]) + (s_red2[128 + tid] + s_red2[192 + tid]));
+            // the part of dr_t through u = mu k^2 / r: -sum_i du mu k^2 / r^2
+            const float dru = (s_red2[tid] + s_red2[64 + tid]) + (s_red2[128 + tid] + s_red2[192 + tid]);
+            const float dr = s_ds[tid] + dru;
             st_grad<OBF>(a.dr, tok_index(a, b, tt, h), dr * (G ? s_fr[tid] : 1.f) * invl);
+            // dL/dmu gains sum_i du k^2 / r = -dru r / mu
+            if (a.dmu) s_dmu[tid] += -dru * s_r[tid] / mu;
           }
         }
       }
@@ -949,6 +956,7 @@ __global__ void __launch_bounds__(BT, 1)
       __syncthreads();
       float db = 0.f;
       if (ci == 0) {
+        float dmu = 0.f;
         db = s_dp[0];
         for (int q2 = 3; q2 > qq; --q2) db = s_aff[q2 * 2] * db + s_aff[q2 * 2 + 1];
         for (int j = 15; j >= 0; --j) {
@@ -959,6 +967,7 @@ __global__ void __launch_bounds__(BT, 1)
           const float dd = r + bhat * n2, dbeta = s_ds[t];
           const float dbhat = db * rden * rden + __fdividef(dbeta * r, dd * dd);
           const float du = -db * bt * bt;
+          dmu += du * n2 * ri * (1.f / D);  // u = mu |k|^2 / (dk r)
           s_dn2[t] = -dbeta * beta * beta + du * mu * ri * (1.f / D);
           s_da[t] = s_bp[t] * dbhat;
           if (tt < a.T) {
@@ -968,6 +977,7 @@ __global__ void __launch_bounds__(BT, 1)
           }
           db = s_a[t] * dbhat;
         }
+        s_dmu[qq] += dmu;
       }
       __syncthreads();
       if (tid == 0) s_dp[0] = db;
@@ -1035,6 +1045,11 @@ __global__ void __launch_bounds__(BT, 1)
     if (a.dp0 && tid < D) {
       if (V == 0) a.dp0[(size_t)bh * D + tid] = s_dp[tid] * invl;
       else if (tid == 0) a.dp0[bh] = s_dp[0] * invl;
+    }
+    if (a.dmu && tid == 0) {  // dL/dmu of this sequence: the warps' parts
+      float tot = 0.f;
+      for (int w = 0; w < CM; ++w) tot += s_dmu[w];
+      a.dmu[bh] = tot * invl;
     }
   } else {
     if (tid == 0) atomicExch(a.status, (unsigned)KDN_ERR_TIMEOUT);

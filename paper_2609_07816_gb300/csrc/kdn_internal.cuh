@@ -95,6 +95,7 @@ struct Args {
   const float *dST, *dpT;
   void *dq, *dk_, *dv_, *dg, *domega, *dr;
   float *dS0, *dp0;
+  float *dmu;  // [B,H] gradient with respect to mu (nullable)
   // workspace regions (float32 unless noted)
   unsigned *status;
   float *phat;    // [BH][Tp][P]   predictive variance phat_t (pre-write)

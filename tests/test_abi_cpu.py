@@ -124,8 +124,11 @@ def test_rejects_small_or_misaligned_workspace(kdn):
 def test_backward_and_decode_validate(kdn):
     L = kdn.lib()
     d = kdn.make_desc(1, 10, 1, 32, 32, kdn.KDN_BF16)
-    p = [FAKE] * 19
+    p = [FAKE] * 20
     p[15] = None  # domega is required
+    assert L.kdn_iso_bwd(ctypes.byref(d), *p, FAKE, 1 << 40, None) == kdn.KDN_ERR_INVALID_ARG
+    p = [FAKE] * 20
+    p[19] = MIS  # dmu is optional but must be aligned
     assert L.kdn_iso_bwd(ctypes.byref(d), *p, FAKE, 1 << 40, None) == kdn.KDN_ERR_INVALID_ARG
     q = [FAKE] * 9
     q[7] = None  # p (state) is required
@@ -232,7 +235,7 @@ def test_training_pair_validation(kdn):
 
     def bwd_saved(desc, saved=FAKE, saved_bytes=1 << 40):
         return L.kdn_diag_bwd_saved(ctypes.byref(desc), *([FAKE] * 6), saved, saved_bytes,
-                                    *([FAKE] * 11), FAKE, 1 << 40, None)
+                                    *([FAKE] * 12), FAKE, 1 << 40, None)
 
     for fn in (fwd_save, bwd_saved):
         assert fn(kdn.make_desc(B, T, H, 64, 128, kdn.KDN_BF16)) == kdn.KDN_ERR_UNSUPPORTED

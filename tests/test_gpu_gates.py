@@ -74,7 +74,7 @@ def test_logit_gates_forward_backward(kdn, case):
     check("o", o, ref["o"], dt)
     check("ST", ST, ref["ST"], dt)
     check("pT", pT, ref["pT"], dt)
-    for n in ("dq", "dk", "dv", "dg", "domega", "dr", "dS0", "dp0"):
+    for n in ("dq", "dk", "dv", "dg", "domega", "dr", "dS0", "dp0", "dmu"):
         check(n, grads[n], gref[n], dt)
 
 

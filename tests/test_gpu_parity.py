@@ -179,7 +179,7 @@ def test_backward_parity(kdn, case):
             torch.tensor(dST, dtype=torch.float32, device="cuda"),
             torch.tensor(dpT, dtype=torch.float32, device="cuda"))
     torch.cuda.synchronize()
-    for n in ("dq", "dk", "dv", "dg", "domega", "dr", "dS0", "dp0"):
+    for n in ("dq", "dk", "dv", "dg", "domega", "dr", "dS0", "dp0", "dmu"):
         check(n, gr[n], ref[n], dt)
 
 
@@ -381,7 +381,7 @@ def test_training_pair_matches_recompute_path(kdn):
     torch.cuda.synchronize()
     ref = oracle.bwd("diag", *[ins[n] for n in ("q", "k", "v", "g", "omega", "r")], ins["S0"],
                      ins["p0"], ins["dO"], ins["dST"], ins["dpT"])
-    for n in ("dq", "dk", "dv", "dg", "domega", "dr", "dS0", "dp0"):
+    for n in ("dq", "dk", "dv", "dg", "domega", "dr", "dS0", "dp0", "dmu"):
         assert torch.equal(g1[n], g2[n]), n
         check(n, g2[n], ref[n], "bf16")
 

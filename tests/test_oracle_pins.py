@@ -450,6 +450,10 @@ def test_p9_backward_finite_differences(variant, per_channel):
             fd[idx] = (f(xp) - f(xm)) / (2 * h)
         err = np.max(np.abs(fd - an[gn])) / max(np.max(np.abs(fd)), 1e-30)
         assert err < 1e-6, (n, err)
+    # the information scale mu (one value shared by all sequences): sum of dmu
+    fd_mu = (_loss_fn(variant, ins, ins["dO"], wS, wp, mu + h)(ins)
+             - _loss_fn(variant, ins, ins["dO"], wS, wp, mu - h)(ins)) / (2 * h)
+    assert abs(fd_mu - an["dmu"].sum()) <= 1e-6 * abs(fd_mu), (fd_mu, an["dmu"].sum())
 
 
 @pytest.mark.parametrize("variant,per_channel", [("diag", True), ("iso", True), ("iso", False)])
