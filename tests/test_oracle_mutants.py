@@ -37,17 +37,32 @@ MUTANTS = [
      "const double dshat = dS[(size_t)i * dv + j];"),
     ("dkt[i] += du * 2.0 * J->mu * kt[i] / rt;", "dkt[i] += du * J->mu * kt[i] / rt;"),
     ("dp[i] = st->alpha[i] * st->alpha[i] * dphat[i];", "dp[i] = st->alpha[i] * dphat[i];"),
+    # gradient with respect to mu
+    ("J->dmu[(size_t)b * J->H + h] += du * kt[i] * kt[i] / rt;",
+     "J->dmu[(size_t)b * J->H + h] += du * kt[i] / rt;"),
+    ("J->dmu[(size_t)b * J->H + h] += du * st->n2 / (dk * rt);",
+     "J->dmu[(size_t)b * J->H + h] += du * st->n2 / rt;"),
+    # logit gates (the Python side of the oracle)
+    ("__init__.py", 'out["dg"] = out["dg"] * _sigmoid(-x)', 'out["dg"] = out["dg"] * _sigmoid(x)'),
+    ("__init__.py", 'out["domega"] = out["domega"] * _sigmoid(y)', 'out["domega"] = out["domega"]'),
+    ("__init__.py", 'out["dr"] = out["dr"] * _sigmoid(z)', 'out["dr"] = out["dr"] * _sigmoid(-z)'),
+    ("__init__.py", "return -_softplus(-x), _softplus(y), r_min + _softplus(z)",
+     "return -_softplus(-x), _softplus(y), _softplus(z)"),
+    ("__init__.py", "return -_softplus(-x), _softplus(y), r_min + _softplus(z)",
+     "return -_softplus(x), _softplus(y), r_min + _softplus(z)"),
 ]
 
 
 @pytest.mark.parametrize("idx", range(len(MUTANTS)))
 def test_pins_catch_planted_mistake(idx, tmp_path):
-    src, mut = MUTANTS[idx]
-    text = open(os.path.join(ROOT, "oracle", "kdn_oracle.c")).read()
-    assert text.count(src) >= 1, "mutation site not found: " + src
+    fname, src, mut = MUTANTS[idx] if len(MUTANTS[idx]) == 3 else ("kdn_oracle.c",) + MUTANTS[idx]
     (tmp_path / "oracle").mkdir()
-    (tmp_path / "oracle" / "kdn_oracle.c").write_text(text.replace(src, mut, 1))
-    shutil.copy(os.path.join(ROOT, "oracle", "__init__.py"), tmp_path / "oracle")
+    for f in ("kdn_oracle.c", "__init__.py"):
+        text = open(os.path.join(ROOT, "oracle", f)).read()
+        if f == fname:
+            assert text.count(src) >= 1, "mutation site not found: " + src
+            text = text.replace(src, mut, 1)
+        (tmp_path / "oracle" / f).write_text(text)
     shutil.copy(os.path.join(ROOT, "kdn_inputs.py"), tmp_path)
     shutil.copytree(os.path.join(ROOT, "tests", "golden"), tmp_path / "tests" / "golden")
     for f in ("conftest.py", "test_oracle_pins.py"):
