@@ -568,6 +568,9 @@ __global__ void __launch_bounds__(FT, 1)
     tmem_st_wait();
     if (!(ok = mma_wait())) break;
     tc_fence_after();
+    // kq and rw are free: MMA-T and MMA-W have read them, the Qbar and K_tail
+    // conversions above have finished (the wait's barrier)
+    if (tid == 0 && c + 1 < NC) issue_raw_kqw(c + 1);
     if (tid == 0 && P.save_S) {  // A fp16 [t][s] into the backward context
       bulk_s2g(ctx + kCtxA, af, 8192);
       bulk_commit();
@@ -599,7 +602,6 @@ __global__ void __launch_bounds__(FT, 1)
     fence_proxy_async();
     tc_fence_before();
     __syncthreads();
-    if (tid == 0 && c + 1 < NC) issue_raw_kqw(c + 1);  // raw k, q, omega buffers are free
     if (tid == 0 && P.save_S) {  // S_in, -W and A_qk into the backward context
       bulk_s2g(ctx + kCtxS, b3, 32768);
       bulk_s2g(ctx + kCtxW, a1l, 8192);
