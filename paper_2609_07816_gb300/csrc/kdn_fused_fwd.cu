@@ -342,23 +342,55 @@ __global__ void __launch_bounds__(FT, 1)
           el[j] = eq;
         }
         sQ[(qq * D + i) * 5 + 4] = eq;
-        // scalar Moebius product of this quarter (Prop. 5, eq. iso-kla-box-mobius)
-        if (i == 0) {
-          float m00 = 1.f, m01 = 0.f, m10 = 0.f, m11 = 1.f;
-          for (int j = 0; j < 16; ++j) {
-            const int t = t0 + j;
+        // scalar uncertainty of the chunk (Prop. 5, eq. iso-kla-box-mobius) by an
+        // ordered scan of the token matrices M_t = [[a, w], [u a, 1 + u w]] in one
+        // warp: lane l holds tokens 2l, 2l + 1; after the scan it holds the product
+        // of tokens 0 .. 2l + 1 (later tokens on the left, renormalised by the
+        // largest entry), and the exclusive product gives b_{t-1} for its tokens
+        // from the carry b entering the chunk
+        if (warp == 0) {
+          const int ta = 2 * lane, tb = ta + 1;
+          auto tok_m = [&](int t, float &m00, float &m01, float &m10, float &m11) {
             const float at = s_a[t], wt = s_om[t], ut = a.mu * s_n2[t] * s_ri[t] * (1.f / D);
-            const float n00 = at * m00 + wt * m10, n01 = at * m01 + wt * m11;
-            const float n10 = ut * at * m00 + (1.f + ut * wt) * m10;
-            const float n11 = ut * at * m01 + (1.f + ut * wt) * m11;
-            m00 = n00; m01 = n01; m10 = n10; m11 = n11;
-            if ((j & 7) == 7) {
-              const float sc = __frcp_rn(fmaxf(fmaxf(fabsf(m00), fabsf(m01)), fmaxf(fabsf(m10), fabsf(m11))));
-              m00 *= sc; m01 *= sc; m10 *= sc; m11 *= sc;
+            m00 = at; m01 = wt; m10 = ut * at; m11 = fmaf(ut, wt, 1.f);
+          };
+          float a00, a01, a10, a11, b00, b01, b10, b11;
+          tok_m(ta, a00, a01, a10, a11);
+          tok_m(tb, b00, b01, b10, b11);
+          // pair product M_tb M_ta
+          float m00 = b00 * a00 + b01 * a10, m01 = b00 * a01 + b01 * a11;
+          float m10 = b10 * a00 + b11 * a10, m11 = b10 * a01 + b11 * a11;
+          renorm4(m00, m01, m10, m11);
+#pragma unroll
+          for (int off = 1; off < 32; off <<= 1) {
+            const float p00 = __shfl_up_sync(0xffffffffu, m00, off);
+            const float p01 = __shfl_up_sync(0xffffffffu, m01, off);
+            const float p10 = __shfl_up_sync(0xffffffffu, m10, off);
+            const float p11 = __shfl_up_sync(0xffffffffu, m11, off);
+            if (lane >= off) {
+              float n00 = m00 * p00 + m01 * p10, n01 = m00 * p01 + m01 * p11;
+              float n10 = m10 * p00 + m11 * p10, n11 = m10 * p01 + m11 * p11;
+              renorm4(n00, n01, n10, n11);
+              m00 = n00; m01 = n01; m10 = n10; m11 = n11;
             }
           }
-          float *mine = sQ + (qq * D) * 5;
-          mine[0] = m00; mine[1] = m01; mine[2] = m10; mine[3] = m11;
+          // exclusive product (tokens 0 .. ta - 1) applied to the carry [b, 1]
+          float e00 = __shfl_up_sync(0xffffffffu, m00, 1), e01 = __shfl_up_sync(0xffffffffu, m01, 1);
+          float e10 = __shfl_up_sync(0xffffffffu, m10, 1), e11 = __shfl_up_sync(0xffffffffu, m11, 1);
+          if (lane == 0) { e00 = 1.f; e01 = 0.f; e10 = 0.f; e11 = 1.f; }
+          const float bin = s_b[0];
+          float n = fmaf(e00, bin, e01), d = fmaf(e10, bin, e11);
+          const float bpa = __fdividef(n, d);                       // b_{ta - 1}
+          const float nn = fmaf(a00, n, a01 * d), dd = fmaf(a10, n, a11 * d);
+          const float bpb = __fdividef(nn, dd);                     // b_{ta}
+          const float bha = fmaf(s_a[ta], bpa, s_om[ta]);           // eq. iso-kla-box-cov-update
+          const float bhb = fmaf(s_a[tb], bpb, s_om[tb]);
+          s_bp[ta] = bpa; s_bh[ta] = bha;
+          s_bp[tb] = bpb; s_bh[tb] = bhb;
+          s_x[ta] = __fdividef(bha, s_r[ta] + bha * s_n2[ta]);     // beta_t, eq. iso-kla-box-gain
+          s_x[tb] = __fdividef(bhb, s_r[tb] + bhb * s_n2[tb]);
+          if (lane == 31)  // b_63 leaves the chunk
+            carry_out = __fdividef(bhb, 1.f + a.mu * s_n2[tb] * s_ri[tb] * (1.f / D) * bhb);
         }
         __syncthreads();
         float pre = 1.f;
@@ -366,34 +398,14 @@ __global__ void __launch_bounds__(FT, 1)
 #pragma unroll
         for (int j = 0; j < 16; ++j) Eb[(t0 + j) * D + i] = pre * el[j];
         gc_out = pre * eq;
-        if (i == 0) {
-          float n = s_b[0], d = 1.f;
-          for (int q2 = 0; q2 < qq; ++q2) {
-            const float *o = sQ + (q2 * D) * 5;
-            const float nn = o[0] * n + o[1] * d, dd = o[2] * n + o[3] * d;
-            const float sc = __frcp_rn(fmaxf(fabsf(nn), fabsf(dd)));
-            n = nn * sc;
-            d = dd * sc;
-          }
-          float bb = __fdividef(n, d);
-          for (int j = 0; j < 16; ++j) {
-            const int t = t0 + j;
-            const float bhat = s_a[t] * bb + s_om[t];          // eq. iso-kla-box-cov-update
-            s_bp[t] = bb;
-            s_bh[t] = bhat;
-            s_x[t] = __fdividef(bhat, s_r[t] + bhat * s_n2[t]);  // beta_t, eq. iso-kla-box-gain
-            bb = __fdividef(bhat, 1.f + a.mu * s_n2[t] * s_ri[t] * (1.f / D) * bhat);
-          }
-          carry_out = bb;
-        }
       }
       __syncthreads();
       if (qq == 3) {
         s_gC[i] = gc_out;
         check_gamma_range(gc_out, a.status);
         if (V == 0) s_p[i] = carry_out;
-        else if (i == 0) s_b[0] = carry_out;
       }
+      if (V == 1 && tid == 31) s_b[0] = carry_out;  // lane 31 of warp 0 formed b_63
     }
     fence_proxy_async();  // phat / gamma are read by the bulk copies below
     __syncthreads();

@@ -62,6 +62,15 @@ __device__ __forceinline__ float dgate_logalpha(int gates, float alpha) {
 }
 __device__ __forceinline__ float dgate_sig(int gates, float y) { return gates ? sigmoid_f(y) : 1.f; }
 
+// A 2x2 Moebius matrix (homogeneous coordinates of the uncertainty) divided by
+// its largest entry: the ratio it represents is unchanged, and long products stay
+// in range.
+__device__ __forceinline__ void renorm4(float &m00, float &m01, float &m10, float &m11) {
+  const float s = fmaxf(fmaxf(fabsf(m00), fabsf(m01)), fmaxf(fabsf(m10), fabsf(m11)));
+  const float inv = __fdividef(1.f, s);
+  m00 *= inv; m01 *= inv; m10 *= inv; m11 *= inv;
+}
+
 __device__ __forceinline__ float warp_sum(float x) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);

@@ -33,12 +33,6 @@ constexpr int kMinSegChunks = 8;
 
 using bf16 = __nv_bfloat16;
 
-__device__ __forceinline__ void renorm4(float &m00, float &m01, float &m10, float &m11) {
-  const float s = fmaxf(fmaxf(fabsf(m00), fabsf(m01)), fmaxf(fabsf(m10), fabsf(m11)));
-  const float inv = 1.f / s;
-  m00 *= inv; m01 *= inv; m10 *= inv; m11 *= inv;
-}
-
 // Diagonal KDN: per (chunk, batch*head) and channel, the ordered product of the
 // chunk's 64 token matrices (later tokens on the left), renormalised by its
 // largest entry every 4 tokens (all entries are non-negative).  One warp per
