@@ -196,7 +196,7 @@ __global__ void __launch_bounds__(BT, 1)
   float *s_misc = s_da + 64;    // [0] lambda, [1..] scratch
   float *s_fr = s_misc + 16;    // [64] d r_t / d z_t (1 unless the gates are logits)
   float *s_dmu = s_fr + 64;     // [64] parts of dL/dmu (lambda-scaled), summed at the end:
-                                //      diag one per token slot, iso one per quarter
+                                //      diag one per token slot, iso in [0]
   uint64_t *bars = reinterpret_cast<uint64_t *>(sm + OFF_BAR);
   uint64_t *bar_a = bars, *bar_b = bars + 1, *bar_mma = bars + 2;
   uint32_t *s_tbase = reinterpret_cast<uint32_t *>(bars + 4);
@@ -890,7 +890,6 @@ __global__ void __launch_bounds__(BT, 1)
       float *sdg = reinterpret_cast<float *>(sm + O_G);  // [16][512] dG_t
       float *s_tot = reinterpret_cast<float *>(sm + O_DT);  // [4][128] quarter sums of dG
       float *s_dgc = s_tot + 512;                           // [4][128] dgamma_C parts
-      float *s_aff = s_dgc + 512;                           // [4][2] affine summaries
       float ga[16], k16[16], q16[16];
       tmem_ld16(TGM + lane_base + t0, ga);
 #pragma unroll
@@ -938,49 +937,64 @@ __global__ void __launch_bounds__(BT, 1)
       __syncthreads();
       if (tid < CM) s_ds[tid] = (s_red[tid] + s_red[64 + tid]) + (s_red[128 + tid] + s_red[192 + tid]);
       __syncthreads();
-      // the scalar recursion: db_{t-1} = a_t (db_t / den_t^2 + dbeta_t r_t / dd_t^2), one
-      // thread per quarter composes its 16 maps, then runs its tokens
-      if (ci == 0) {
-        float A = 1.f, Bv = 0.f;
-        for (int j = 15; j >= 0; --j) {
-          const int t = t0 + j;
+      // the scalar recursion backwards over the chunk, db_{t-1} = A_t db_t + B_t with
+      // A_t = a_t / den_t^2 and B_t = a_t dbeta_t r_t / dd_t^2, as a suffix scan of
+      // these affine maps in one warp (lane l holds tokens 2l, 2l + 1); A_t <= 1
+      float db_in = 0.f;
+      if (warp == 0) {
+        const int ta = 2 * lane, tb = ta + 1;
+        auto coef = [&](int t, float &A_, float &B_, float &rden, float &dd) {
           const float bhat = s_bh[t], u = mu * s_n2[t] * s_ri[t] * (1.f / D);
-          const float rden = __fdividef(1.f, 1.f + u * bhat), dd = s_r[t] + bhat * s_n2[t];
-          const float aj = s_a[t] * rden * rden;
-          Bv = aj * Bv + s_a[t] * __fdividef(s_ds[t] * s_r[t], dd * dd);
-          A = aj * A;
+          rden = __fdividef(1.f, 1.f + u * bhat);
+          dd = s_r[t] + bhat * s_n2[t];
+          A_ = s_a[t] * rden * rden;
+          B_ = s_a[t] * __fdividef(s_ds[t] * s_r[t], dd * dd);
+        };
+        float Aa, Ba, rda, dda, Ab, Bb, rdb, ddb;
+        coef(ta, Aa, Ba, rda, dda);
+        coef(tb, Ab, Bb, rdb, ddb);
+        // this pair's map db_{tb} -> db_{ta - 1}, then composed with the later pairs'
+        float SA = Aa * Ab, SB = fmaf(Aa, Bb, Ba);
+#pragma unroll
+        for (int off = 1; off < 32; off <<= 1) {
+          const float pA = __shfl_down_sync(0xffffffffu, SA, off);
+          const float pB = __shfl_down_sync(0xffffffffu, SB, off);
+          if (lane + off < 32) {
+            SB = fmaf(SA, pB, SB);
+            SA = SA * pA;
+          }
         }
-        s_aff[qq * 2] = A;
-        s_aff[qq * 2 + 1] = Bv;
-      }
-      __syncthreads();
-      float db = 0.f;
-      if (ci == 0) {
+        // the later pairs' map applied to the cotangent entering from the next chunk
+        float EA = __shfl_down_sync(0xffffffffu, SA, 1), EB = __shfl_down_sync(0xffffffffu, SB, 1);
+        if (lane == 31) { EA = 1.f; EB = 0.f; }
+        const float dbb = fmaf(EA, s_dp[0], EB);  // db_{tb}
+        const float dba = fmaf(Ab, dbb, Bb);      // db_{ta}
         float dmu = 0.f;
-        db = s_dp[0];
-        for (int q2 = 3; q2 > qq; --q2) db = s_aff[q2 * 2] * db + s_aff[q2 * 2 + 1];
-        for (int j = 15; j >= 0; --j) {
-          const int t = t0 + j, tt = c * CM + t;
+        auto tok = [&](int t, float dbt, float rden, float dd) {
           const float bhat = s_bh[t], beta = s_x[t], n2 = s_n2[t], r = s_r[t], ri = s_ri[t];
-          const float u = mu * n2 * ri * (1.f / D);
-          const float rden = __fdividef(1.f, 1.f + u * bhat), bt = bhat * rden;
-          const float dd = r + bhat * n2, dbeta = s_ds[t];
-          const float dbhat = db * rden * rden + __fdividef(dbeta * r, dd * dd);
-          const float du = -db * bt * bt;
+          const float u = mu * n2 * ri * (1.f / D), bt = bhat * rden, dbeta = s_ds[t];
+          const float dbhat = dbt * rden * rden + __fdividef(dbeta * r, dd * dd);
+          const float du = -dbt * bt * bt;
           dmu += du * n2 * ri * (1.f / D);  // u = mu |k|^2 / (dk r)
           s_dn2[t] = -dbeta * beta * beta + du * mu * ri * (1.f / D);
           s_da[t] = s_bp[t] * dbhat;
+          const int tt = c * CM + t;
           if (tt < a.T) {
             const size_t th = tok_index(a, b, tt, h);
             st_grad<OBF>(a.domega, th, dbhat * (G ? s_fw[t] : 1.f) * invl);
             st_grad<OBF>(a.dr, th, (-__fdividef(dbeta * beta, dd) - du * u * ri) * (G ? s_fr[t] : 1.f) * invl);
           }
-          db = s_a[t] * dbhat;
+          return s_a[t] * dbhat;  // db_{t-1}
+        };
+        tok(tb, dbb, rdb, ddb);
+        db_in = tok(ta, dba, rda, dda);  // lane 0: the cotangent leaving the chunk
+        if (a.dmu) {
+          dmu = warp_sum(dmu);
+          if (lane == 0) s_dmu[0] += dmu;
         }
-        s_dmu[qq] += dmu;
       }
       __syncthreads();
-      if (tid == 0) s_dp[0] = db;
+      if (tid == 0) s_dp[0] = db_in;
       // per element: dk and dg
       {
         const float dgC = (s_dgc[ci] + s_dgc[D + ci]) + (s_dgc[2 * D + ci] + s_dgc[3 * D + ci]);
