@@ -268,21 +268,24 @@ __global__ void __launch_bounds__(FT, 1)
           w[j] = tile_omega(bf(rw, 8192, t0 + j, i), t0 + j);
           uk[j] = a.mu * kk * kk * s_ri[t0 + j];
         }
-        float m00 = 1.f, m01 = 0.f, m10 = 0.f, m11 = 1.f, eq = 1.f;
+        // a quarter's summary is read by the later quarters only: the last one skips it
+        if (qq < 3) {
+          float m00 = 1.f, m01 = 0.f, m10 = 0.f, m11 = 1.f, eq = 1.f;
 #pragma unroll
-        for (int j = 0; j < 16; ++j) {
-          const float a2_ = al[j] * al[j], ua2 = uk[j] * a2_, d1 = 1.f + uk[j] * w[j];
-          const float n00 = a2_ * m00 + w[j] * m10, n01 = a2_ * m01 + w[j] * m11;
-          const float n10 = ua2 * m00 + d1 * m10, n11 = ua2 * m01 + d1 * m11;
-          m00 = n00; m01 = n01; m10 = n10; m11 = n11;
-          eq *= al[j];
-          if ((j & 7) == 7) {  // renormalise by the largest magnitude (n/d is scale free)
-            const float sc = __frcp_rn(fmaxf(fmaxf(fabsf(m00), fabsf(m01)), fmaxf(fabsf(m10), fabsf(m11))));
-            m00 *= sc; m01 *= sc; m10 *= sc; m11 *= sc;
+          for (int j = 0; j < 16; ++j) {
+            const float a2_ = al[j] * al[j], ua2 = uk[j] * a2_, d1 = 1.f + uk[j] * w[j];
+            const float n00 = a2_ * m00 + w[j] * m10, n01 = a2_ * m01 + w[j] * m11;
+            const float n10 = ua2 * m00 + d1 * m10, n11 = ua2 * m01 + d1 * m11;
+            m00 = n00; m01 = n01; m10 = n10; m11 = n11;
+            eq *= al[j];
+            if ((j & 7) == 7) {  // renormalise by the largest magnitude (n/d is scale free)
+              const float sc = __frcp_rn(fmaxf(fmaxf(fabsf(m00), fabsf(m01)), fmaxf(fabsf(m10), fabsf(m11))));
+              m00 *= sc; m01 *= sc; m10 *= sc; m11 *= sc;
+            }
           }
+          float *mine = sQ + (qq * D + i) * 5;
+          mine[0] = m00; mine[1] = m01; mine[2] = m10; mine[3] = m11; mine[4] = eq;
         }
-        float *mine = sQ + (qq * D + i) * 5;
-        mine[0] = m00; mine[1] = m01; mine[2] = m10; mine[3] = m11; mine[4] = eq;
         __syncthreads();
         float n = s_p[i], d = 1.f, e = 1.f;
         for (int q2 = 0; q2 < qq; ++q2) {
