@@ -75,7 +75,7 @@ def decode_bytes(b, h, dk, dv, in_bytes=2, out_bytes=4):
 # DRAM bytes per launch of each kernel at the bench workload, from one ncu
 # capture (dram__bytes_read.sum + dram__bytes_write.sum) of the current build;
 # reported as `traffic` only for that workload.
-NCU_TRAFFIC = {"k_fused_fwd": None, "k_fused_bwd": 1883851520 + 1345211648}
+NCU_TRAFFIC = {"k_fused_fwd": 672318720 + 1442769920, "k_fused_bwd": 1884394752 + 1344989952}
 
 
 def chunk_flops(dk, dv, C=64):
