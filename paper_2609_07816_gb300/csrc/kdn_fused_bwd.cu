@@ -715,7 +715,12 @@ __global__ void __launch_bounds__(BT, 1)
     }
     if (!(ok = mma_wait())) break;
     tc_fence_after();
-    if (tid == 0 && c > 0) issue_a_ctx(c - 1);  // the context buffers are free
+    if (tid == 0 && c > 0) {
+      issue_a_ctx(c - 1);  // the context buffers are free
+      // phat, gamma and the token scalars of chunk c - 1 are read with plain loads at the
+      // top of its iteration: bring them into L2 now
+      bulk_prefetch_l2(rec - kCtxBytes + kCtxPh, kCtxBytes - kCtxPh);
+    }
     // ---- [18] per channel (lane ci, tokens t0..t0+15): back through Gamma and the
     //           gain emission, then the uncertainty recursion backwards in time.
     //           Free TMEM columns hold per-(channel, token) intermediates between passes:
