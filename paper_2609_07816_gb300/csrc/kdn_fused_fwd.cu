@@ -63,9 +63,19 @@ constexpr int OFF_B3 = OFF_A2 + 16384;    // S_in fp16 (MN-major)               
 constexpr int OFF_F = OFF_B3 + 32768;     // fp32 scratch: gamma [64][128] / T, A [64][LT] + X
 constexpr int F_BYTES = 2 * 64 * LT * 4 + 3 * 256 * 4;  // 37888 >= 32768
 constexpr int OFF_SM = OFF_F + F_BYTES;                  // small arrays
-constexpr int SMALL_FLOATS = 64 * 9 + 128 * 3;
+constexpr int SMALL_FLOATS = 64 * 11 + 128 * 3;
 constexpr int OFF_BAR = OFF_SM + SMALL_FLOATS * 4;
 constexpr int SMEM_BYTES = OFF_BAR + 64 + 1024;  // + alignment slack
+
+// n consecutive floats of 16-byte-aligned shared memory, by float4
+__device__ __forceinline__ void ld_f8(const float *p, float *x) {
+  const float4 a0 = reinterpret_cast<const float4 *>(p)[0], a1 = reinterpret_cast<const float4 *>(p)[1];
+  x[0] = a0.x; x[1] = a0.y; x[2] = a0.z; x[3] = a0.w; x[4] = a1.x; x[5] = a1.y; x[6] = a1.z; x[7] = a1.w;
+}
+__device__ __forceinline__ void ld_f16(const float *p, float *x) {
+  ld_f8(p, x);
+  ld_f8(p + 8, x + 8);
+}
 
 struct FusedParams {
   Args a;
@@ -78,8 +88,16 @@ struct FusedParams {
 };
 
 // G: the gate inputs are logits (KDN_GATES_LOGITS), a compile-time choice so
-// that the post-activation path carries none of the activation code
-template <int V, int G>
+// that the post-activation path carries none of the activation code.
+// SD: isotropic KDN with one decay per head (decay_per_channel = 0).  Gamma is
+// then a per-token scalar and factors out of every intra-chunk product:
+//   T_ts = beta_s (k_t . k_s) gamma_t / gamma_s,
+//   A_qk,ts = tau beta_s (q_t . k_s) gamma_t / gamma_s,
+//   W = (A diag(gamma)) K,
+// so MMA-T runs once per K step on the raw bf16 k and q tiles (exact products,
+// no hi/lo split) and the decay ratios and beta_s are applied in fp32 when T and
+// A_qk leave TMEM; no Gamma-scaled operand tile is formed.
+template <int V, int G, int SD>
 __global__ void __launch_bounds__(FT, 1)
     k_fused_fwd(const __grid_constant__ CUtensorMap mq, const __grid_constant__ CUtensorMap mk,
                 const __grid_constant__ CUtensorMap mv, const __grid_constant__ CUtensorMap mg,
@@ -106,6 +124,8 @@ __global__ void __launch_bounds__(FT, 1)
   float *s_gC = s_ri + 64;   // [128] gamma_C
   float *s_b = s_gC + 128;   // [1] isotropic carry b
   float *s_p = s_b + 128;    // [128] diagonal carry p (per channel)
+  float *s_gm = s_p + 128;   // [64] gamma_t (SD: one value per token)
+  float *s_kf = s_gm + 64;   // [64] beta_t / gamma_t (SD)
   uint64_t *bars = reinterpret_cast<uint64_t *>(sm + OFF_BAR);
   uint64_t *bar_raw = bars, *bar_v = bars + 1, *bar_mma = bars + 2;
   uint32_t *s_tbase = reinterpret_cast<uint32_t *>(bars + 4);
@@ -337,14 +357,16 @@ __global__ void __launch_bounds__(FT, 1)
           }
         }
         __syncthreads();
-        // cumulative decay of channel i within this quarter
+        // cumulative decay of channel i within this quarter (SD: per token, below)
         float el[16], eq = 1.f;
+        if (!SD) {
 #pragma unroll
-        for (int j = 0; j < 16; ++j) {
-          eq *= pcd ? tile_alpha(bf(rg, 8192, t0 + j, i), t0 + j) : __expf(s_gs[t0 + j]);
-          el[j] = eq;
+          for (int j = 0; j < 16; ++j) {
+            eq *= pcd ? tile_alpha(bf(rg, 8192, t0 + j, i), t0 + j) : __expf(s_gs[t0 + j]);
+            el[j] = eq;
+          }
+          sQ[(qq * D + i) * 5 + 4] = eq;
         }
-        sQ[(qq * D + i) * 5 + 4] = eq;
         // scalar uncertainty of the chunk (Prop. 5, eq. iso-kla-box-mobius) by an
         // ordered scan of the token matrices M_t = [[a, w], [u a, 1 + u w]] in one
         // warp: lane l holds tokens 2l, 2l + 1; after the scan it holds the product
@@ -390,17 +412,44 @@ __global__ void __launch_bounds__(FT, 1)
           const float bhb = fmaf(s_a[tb], bpb, s_om[tb]);
           s_bp[ta] = bpa; s_bh[ta] = bha;
           s_bp[tb] = bpb; s_bh[tb] = bhb;
-          s_x[ta] = __fdividef(bha, s_r[ta] + bha * s_n2[ta]);     // beta_t, eq. iso-kla-box-gain
-          s_x[tb] = __fdividef(bhb, s_r[tb] + bhb * s_n2[tb]);
+          const float xa = __fdividef(bha, s_r[ta] + bha * s_n2[ta]);  // beta_t, eq. iso-kla-box-gain
+          const float xb = __fdividef(bhb, s_r[tb] + bhb * s_n2[tb]);
+          s_x[ta] = xa;
+          s_x[tb] = xb;
           if (lane == 31)  // b_63 leaves the chunk
             carry_out = __fdividef(bhb, 1.f + a.mu * s_n2[tb] * s_ri[tb] * (1.f / D) * bhb);
+          if (SD) {
+            // gamma_t = prod_{s <= t} alpha_s by a product scan over the lanes' pairs
+            const float aa = __expf(s_gs[ta]), ab = __expf(s_gs[tb]);
+            float pr = aa * ab;
+#pragma unroll
+            for (int off = 1; off < 32; off <<= 1) {
+              const float pv = __shfl_up_sync(0xffffffffu, pr, off);
+              if (lane >= off) pr *= pv;
+            }
+            float ex = __shfl_up_sync(0xffffffffu, pr, 1);
+            if (lane == 0) ex = 1.f;
+            const float ga = ex * aa, gb = ga * ab;
+            s_gm[ta] = ga;
+            s_gm[tb] = gb;
+            s_kf[ta] = xa * __frcp_rn(ga);
+            s_kf[tb] = xb * __frcp_rn(gb);
+          }
         }
         __syncthreads();
-        float pre = 1.f;
-        for (int q2 = 0; q2 < qq; ++q2) pre *= sQ[(q2 * D + i) * 5 + 4];
+        if (SD) {  // gamma is the same in every channel; the [64][128] copy is for the context
+          if (P.save_S) {
 #pragma unroll
-        for (int j = 0; j < 16; ++j) Eb[(t0 + j) * D + i] = pre * el[j];
-        gc_out = pre * eq;
+            for (int j = 0; j < 16; ++j) Eb[(t0 + j) * D + i] = s_gm[t0 + j];
+          }
+          gc_out = s_gm[CM - 1];
+        } else {
+          float pre = 1.f;
+          for (int q2 = 0; q2 < qq; ++q2) pre *= sQ[(q2 * D + i) * 5 + 4];
+#pragma unroll
+          for (int j = 0; j < 16; ++j) Eb[(t0 + j) * D + i] = pre * el[j];
+          gc_out = pre * eq;
+        }
       }
       __syncthreads();
       if (qq == 3) {
@@ -421,8 +470,8 @@ __global__ void __launch_bounds__(FT, 1)
     // ---- [3] operand tiles, 16-byte chunks (t, 8 channels), one half-warp per token:
     //   Kk = phat k / (s_t gamma) (diag, s_t = r_t + sum phat k^2) or beta_t k / gamma (iso)
     //   Kbar = gamma k, Qbar = tau gamma q; each as a hi/lo bf16 pair, written over
-    //   the raw tiles (hi) and into the lo buffers
-    for (int m = 0; m < 2; ++m) {
+    //   the raw tiles (hi) and into the lo buffers.  SD: none (MMA-T reads the raw tiles)
+    for (int m = 0; m < (SD ? 0 : 2); ++m) {
       const int t = 32 * m + 2 * warp + (lane >> 4), c8 = lane & 15, sl = c8 >> 3, cc = c8 & 7;
       const uint32_t ok16 = sl * 16384 + chunk_off(t, cc), oq16 = ok16 + 8192;
       const uint32_t o8 = sl * 8192 + chunk_off(t, cc);
@@ -477,7 +526,11 @@ __global__ void __launch_bounds__(FT, 1)
     if (tid == 0) {
       tc_fence_after();
       const uint32_t AH = smem_u32(kq), AL = smem_u32(a1l), BH = smem_u32(rw), BL = smem_u32(b1l);
-      for (int kk = 0; kk < 8; ++kk) {
+      for (int kk = 0; SD && kk < 8; ++kk) {  // [K; Q] K^T on the raw tiles (B: rows 0..63)
+        const uint64_t ad = sw128_desc(AH + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024);
+        umma_bf16(TD1, ad, ad, id_T, kk > 0);
+      }
+      for (int kk = 0; !SD && kk < 8; ++kk) {
         const uint32_t ao = (kk >> 2) * 16384 + (kk & 3) * 32, bo = (kk >> 2) * 8192 + (kk & 3) * 32;
         const uint64_t ah = sw128_desc(AH + ao, 16, 1024), bh_ = sw128_desc(BH + bo, 16, 1024);
         umma_bf16(TD1, ah, bh_, id_T, kk > 0);
@@ -510,9 +563,12 @@ __global__ void __launch_bounds__(FT, 1)
       const int r = 32 * wq + lane, s0 = 16 * wg;
       float v[16];
       tmem_ld16(TD1 + lane_base + s0, v);
+      float kf[16];
+      if (SD) ld_f16(s_kf + s0, kf);
+      const float gr = SD ? s_gm[r] : 1.f;
 #pragma unroll
-      for (int u = 0; u < 16; ++u)
-        if (s0 + u >= r) v[u] = 0.f;
+      for (int u = 0; u < 16; ++u)  // SD: T_ts = beta_s gamma_t / gamma_s (k_t . k_s)
+        v[u] = (s0 + u >= r) ? 0.f : (SD ? v[u] * (gr * kf[u]) : v[u]);
 #pragma unroll
       for (int u = 0; u < 4; ++u)
         *reinterpret_cast<float4 *>(sT + r * LT + s0 + 4 * u) = make_float4(v[4 * u], v[4 * u + 1], v[4 * u + 2], v[4 * u + 3]);
@@ -528,7 +584,15 @@ __global__ void __launch_bounds__(FT, 1)
         const int sidx = 8 * cc + j;
         v[j] = (r < 64 && sidx <= r) ? sA[r * LT + sidx] : 0.f;
       }
-      sm16(a2, chunk_off(r, cc)) = pack_bf8(v);
+      if (SD) {  // W = (A diag(gamma)) K
+        float w[8], gm[8];
+        ld_f8(s_gm + 8 * cc, gm);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) w[j] = v[j] * gm[j];
+        sm16(a2, chunk_off(r, cc)) = pack_bf8(w);
+      } else {
+        sm16(a2, chunk_off(r, cc)) = pack_bf8(v);
+      }
       sm16(af, chunk_off(r, cc)) = pack_h8(v);  // [A; 0] fp16 for MMA-U (over the dead T tile)
     }
     fence_proxy_async();
@@ -569,6 +633,18 @@ __global__ void __launch_bounds__(FT, 1)
       const int t = 32 * m + 2 * warp + (lane >> 4), c8 = lane & 15, sl = c8 >> 3, cc = c8 & 7;
       const uint32_t oq16 = sl * 16384 + 8192 + chunk_off(t, cc), o8 = sl * 8192 + chunk_off(t, cc);
       float hv[8], lv[8];
+      if (SD) {  // Qbar = tau gamma_t q_t, K_tail = gamma_C beta_t k_t / gamma_t from the raw tiles
+        unpack_bf8(sm16(kq, oq16), hv);
+        const float fq = a.tau * s_gm[t], fk = s_kf[t];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) hv[j] *= fq;
+        sm16(a1l, oq16) = pack_h8(hv);
+        unpack_bf8(sm16(kq, oq16 - 8192), hv);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) hv[j] *= s_gC[8 * c8 + j] * fk;
+        sm16(b1l, o8) = pack_h8(hv);
+        continue;
+      }
       unpack_bf8(sm16(kq, oq16), hv);
       unpack_bf8(sm16(a1l, oq16), lv);
 #pragma unroll
@@ -608,9 +684,12 @@ __global__ void __launch_bounds__(FT, 1)
       const int r = 32 * wq + lane - 64, s0 = 16 * wg;
       float v[16];
       tmem_ld16(TD1 + lane_base + s0, v);
+      float kf[16];
+      if (SD) ld_f16(s_kf + s0, kf);
+      const float fq = SD ? a.tau * s_gm[r] : 1.f;
 #pragma unroll
-      for (int u = 0; u < 16; ++u)
-        if (s0 + u > r) v[u] = 0.f;
+      for (int u = 0; u < 16; ++u)  // SD: A_qk,ts = tau beta_s gamma_t / gamma_s (q_t . k_s)
+        v[u] = (s0 + u > r) ? 0.f : (SD ? v[u] * (fq * kf[u]) : v[u]);
       sm16(a2, chunk_off(64 + r, s0 >> 3)) = pack_h8(v);
       sm16(a2, chunk_off(64 + r, (s0 >> 3) + 1)) = pack_h8(v + 8);
     }
@@ -779,8 +858,9 @@ kdn_status_t launch_fused_fwd(const Args &a, cudaStream_t s, unsigned char *save
   if (P.has_g_map && !make_map(&mg, a.g, a)) return KDN_ERR_CUDA;
   if (P.has_w_map && !make_map(&mw, a.omega, a)) return KDN_ERR_CUDA;
   const int BH = a.B * a.H;
-  auto kern = a.variant == 0 ? (a.gates ? k_fused_fwd<0, 1> : k_fused_fwd<0, 0>)
-                             : (a.gates ? k_fused_fwd<1, 1> : k_fused_fwd<1, 0>);
+  auto kern = a.variant == 0 ? (a.gates ? k_fused_fwd<0, 1, 0> : k_fused_fwd<0, 0, 0>)
+               : a.pcd     ? (a.gates ? k_fused_fwd<1, 1, 0> : k_fused_fwd<1, 0, 0>)
+                           : (a.gates ? k_fused_fwd<1, 1, 1> : k_fused_fwd<1, 0, 1>);
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES) !=
       cudaSuccess)
     return KDN_ERR_CUDA;
