@@ -435,3 +435,35 @@ def test_isotropic_training_pair_matches_recompute_path(kdn):
     for n in ("dq", "dk", "dv", "dg", "domega", "dr", "dS0", "dp0"):
         assert torch.equal(g1[n], g2[n]), n
         check(n, g2[n], ref[n], "bf16")
+
+
+@pytest.mark.parametrize("variant,pc", [("diag", True), ("iso", False), ("iso", True)])
+def test_fused_strong_decay_inside_range(kdn, variant, pc):
+    """alpha = sigmoid(N(0, 1)): the cumulative decay reaches ~1e-20 within a chunk,
+    inside the fused kernels' range (no KDN_ERR_RANGE).  The decay ratios are then
+    far from 1: with one decay per head they are applied as fp32 factors around
+    exact products, otherwise through the hi/lo operand pairs; forward and backward
+    must keep the oracle's accuracy."""
+    B, T, H = 1, 200, 2
+    ins = make_inputs(variant, B, T, H, 128, 128, dtype="bf16", seed=61, s0_std=0.05,
+                      p0_range=(0.5, 2.0), per_channel_decay=pc, with_grad=True)
+    rng = np.random.default_rng(67)
+    x = rng.normal(0.0, 1.0, ins["g"].shape)
+    ins["g"] = round_to(-np.logaddexp(0.0, -x), "bf16")  # log sigmoid(x)
+    d = to_dev(ins)
+    xs = [d[n] for n in ("q", "k", "v", "g", "omega", "r")]
+    desc = kdn.make_desc(B, T, H, 128, 128, torch.bfloat16, decay_per_channel=int(pc))
+    ws = kdn.alloc_workspace(desc, 0 if variant == "diag" else 1, True)
+    fwd = kdn.kdn_diag_fwd if variant == "diag" else kdn.kdn_iso_fwd
+    bwd = kdn.kdn_diag_bwd if variant == "diag" else kdn.kdn_iso_bwd
+    o, ST, pT = fwd(*xs, d["S0"], d["p0"], workspace=ws)
+    assert kdn.kdn_get_device_status(ws) == kdn.KDN_OK
+    grads = bwd(*xs, d["S0"], d["p0"], d["dO"], workspace=ws)
+    assert kdn.kdn_get_device_status(ws) == kdn.KDN_OK
+    ref = _oracle_fwd(variant, ins)
+    gref = oracle.bwd(variant, *[ins[n] for n in ("q", "k", "v", "g", "omega", "r")],
+                      ins["S0"], ins["p0"], ins["dO"])
+    for n in ("o", "ST", "pT"):
+        check(n, {"o": o, "ST": ST, "pT": pT}[n], ref[n], "bf16")
+    for n in ("dq", "dk", "dv", "dg", "domega", "dr", "dS0", "dp0"):
+        check(n, grads[n], gref[n], "bf16")
