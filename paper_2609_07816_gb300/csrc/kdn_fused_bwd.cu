@@ -85,7 +85,7 @@ constexpr int O_DWT = O_G, O_DAT = O_G + 16 * KB, O_XT = O_G + 24 * KB, O_KQH2 =
 constexpr int O_QL2 = O_RDO, O_DRTL = O_RH;
 // small arrays
 constexpr int OFF_SM = BUF_END;
-constexpr int SMALL_FLOATS = 64 * 16 + 256 * 2 + 128 * 2 + 16;
+constexpr int SMALL_FLOATS = 64 * 18 + 256 * 2 + 128 * 2 + 16;
 constexpr int OFF_BAR = OFF_SM + SMALL_FLOATS * 4;
 constexpr int SMEM_BYTES = OFF_BAR + 64 + 1024;  // + alignment slack
 static_assert(SMEM_BYTES <= 232448, "shared memory");
@@ -156,16 +156,27 @@ __device__ __forceinline__ float rs16(const float *v, int lane) {
   return w1 + __shfl_xor_sync(0xffffffffu, w1, 1);
 }
 
-// Output store in the gradient dtype (OBF: bfloat16, else float32).
+// Output store in the gradient dtype (OBF: bfloat16, else float32).  float32
+// gradients are written with the streaming hint: they are not read again by this
+// kernel, and evicting them first keeps L2 for the context records it prefetches.
 template <int OBF>
 __device__ __forceinline__ void st_grad(void *p, size_t i, float x) {
   if (OBF) static_cast<__nv_bfloat16 *>(p)[i] = __float2bfloat16_rn(x);
-  else static_cast<float *>(p)[i] = x;
+  else __stcs(static_cast<float *>(p) + i, x);
 }
 
 // G: the gate inputs are logits (KDN_GATES_LOGITS), a compile-time choice so
-// that the post-activation path carries none of the chain-rule code
-template <int V, int OBF, int G>
+// that the post-activation path carries none of the chain-rule code.
+// SD: isotropic KDN with one decay per head.  Gamma is then a per-token scalar
+// and the products that meet Gamma-scaled operands take it, with beta and tau,
+// as fp32 factors on their 64 x 64 partner instead:
+//   B8b  (dA_qk Kk)^T   = K^T (dA_qk diag(beta / gamma))^T
+//   B9a  (dA_qk^T Qbar)^T = Q^T (diag(tau gamma) dA_qk)
+//   B9b  (dT^T Kbar)^T  = K^T (diag(gamma) dT)
+//   B10b (dT Kk)^T      = K^T (dT diag(beta / gamma))^T
+// with K, Q the raw bf16 tiles (exact operands); the Qbar and Kk tiles of the
+// second operand set are not formed.
+template <int V, int OBF, int G, int SD>
 __global__ void __launch_bounds__(BT, 1)
     k_fused_bwd(const __grid_constant__ CUtensorMap mq, const __grid_constant__ CUtensorMap mk,
                 const __grid_constant__ CUtensorMap mv, const __grid_constant__ CUtensorMap mdo,
@@ -197,6 +208,8 @@ __global__ void __launch_bounds__(BT, 1)
   float *s_fr = s_misc + 16;    // [64] d r_t / d z_t (1 unless the gates are logits)
   float *s_dmu = s_fr + 64;     // [64] parts of dL/dmu (lambda-scaled), summed at the end:
                                 //      diag one per token slot, iso in [0]
+  float *s_gm = s_dmu + 64;     // [64] gamma_t (SD)
+  float *s_kf = s_gm + 64;      // [64] beta_t / gamma_t (SD)
   uint64_t *bars = reinterpret_cast<uint64_t *>(sm + OFF_BAR);
   uint64_t *bar_a = bars, *bar_b = bars + 1, *bar_mma = bars + 2;
   uint32_t *s_tbase = reinterpret_cast<uint32_t *>(bars + 4);
@@ -426,6 +439,10 @@ __global__ void __launch_bounds__(BT, 1)
         s_gC[ci] = e16[15];
         check_gamma_range(e16[15], a.status);
       }
+      if (SD && ci == 0) {
+#pragma unroll
+        for (int j = 0; j < 16; ++j) s_gm[t0 + j] = e16[j];
+      }
       if (tid < CM) {
         if (V == 0) {
           s_s[tid] = tk[0];
@@ -444,6 +461,7 @@ __global__ void __launch_bounds__(BT, 1)
     // ---- [3] operands of the chunk adjoint from the context and the gains:
     //          A bf16 (from the saved fp16 A); dS -> fp16 [i][j] and dS <- gamma_C dS in
     //          TMEM; K_tail^T [i][s]; lambda dO and v to fp16 in place
+    if (SD && tid < CM) s_kf[tid] = s_x[tid] * __frcp_rn(s_gm[tid]);
     {
       const uint4 ah = sm16(sm + O_AH, tid * 16);  // 512 chunks of 8: the whole 8 KB tile
       float v[8];
@@ -530,6 +548,18 @@ __global__ void __launch_bounds__(BT, 1)
         for (int u = 0; u < 16; ++u)
           if (tc0 + u < j) v[u] = 0.f;
         uint4 lo0, lo1;
+        if (SD) {  // row s of dA_qk^T: diag(tau gamma) dA_qk -> O_AQ | O_DT (B9a)
+          float w[16];
+#pragma unroll
+          for (int u = 0; u < 16; ++u) w[u] = v[u] * (tau * s_gm[tc0 + u]);
+          sm16(sm + O_AQ, chunk_off(j, tc0 >> 3)) = split_bf8(w, &lo0);
+          sm16(sm + O_AQ, chunk_off(j, (tc0 >> 3) + 1)) = split_bf8(w + 8, &lo1);
+          sm16(sm + O_DT, chunk_off(j, tc0 >> 3)) = lo0;
+          sm16(sm + O_DT, chunk_off(j, (tc0 >> 3) + 1)) = lo1;
+          const float f = s_kf[j];  // dA_qk diag(beta / gamma) (B8b)
+#pragma unroll
+          for (int u = 0; u < 16; ++u) v[u] *= f;
+        }
         sm16(sm + O_DAQ, chunk_off(j, tc0 >> 3)) = split_bf8(v, &lo0);
         sm16(sm + O_DAQ, chunk_off(j, (tc0 >> 3) + 1)) = split_bf8(v + 8, &lo1);
         sm16(sm + O_DAQ + 8192, chunk_off(j, tc0 >> 3)) = lo0;
@@ -585,6 +615,10 @@ __global__ void __launch_bounds__(BT, 1)
 #pragma unroll
       for (int j = 0; j < 16; ++j) v[j] = ga[j] * raw_k(t0 + j);
       st_row16_bf(sm + O_KQH2, ci, qq, v);  // Kbar^T hi
+    }
+    if (!SD) {
+      float gf[16], ga[16], v[16];
+      load_gain(gf, ga);
 #pragma unroll
       for (int j = 0; j < 16; ++j) v[j] = tau * ga[j] * raw_q(t0 + j);
       st_row16_split(sm + O_KQH2 + 16384, sm + O_QL2, ci, qq, v);  // Qbar^T hi / lo
@@ -595,7 +629,19 @@ __global__ void __launch_bounds__(BT, 1)
     fence_proxy_async();
     tc_fence_before();
     __syncthreads();
-    if (tid == 0) {
+    if (SD && tid == 0) {  // raw K^T, Q^T (channel-major) against the scaled 64 x 64 partners
+      tc_fence_after();
+      const uint32_t id11 = idesc_bf16(128, 64, 1, 1), id10 = idesc_bf16(128, 64, 1, 0);
+      for (int kk = 0; kk < 4; ++kk) {
+        const uint64_t kt = mdesc(rkq + kk * 2048, 16384), qt = mdesc(rkq + 8192 + kk * 2048, 16384);
+        umma_bf16(X3, kt, mdesc(sm + O_DAQ + kk * 2048, 8192), id11, 1);
+        umma_bf16(X3, kt, mdesc(sm + O_DAQ + 8192 + kk * 2048, 8192), id11, 1);
+        umma_bf16(X0, qt, kdesc(sm + O_AQ + kk * 32), id10, 1);
+        umma_bf16(X0, qt, kdesc(sm + O_DT + kk * 32), id10, 1);
+      }
+      umma_commit(bar_mma);
+    }
+    if (!SD && tid == 0) {
       tc_fence_after();
       const uint32_t id01 = idesc_bf16(128, 64, 0, 1), id00 = idesc_bf16(128, 64, 0, 0);
       for (int kk = 0; kk < 4; ++kk) {
@@ -697,6 +743,16 @@ __global__ void __launch_bounds__(BT, 1)
       tmem_ld16(X1 + lane_base + tc0, v);
 #pragma unroll
       for (int u = 0; u < 16; ++u) v[u] = (tc0 + u < r) ? -v[u] : 0.f;
+      if (SD) {  // dT diag(beta / gamma) -> O_AQ (B10b); diag(gamma) dT below (B9b)
+        float w[16];
+#pragma unroll
+        for (int u = 0; u < 16; ++u) w[u] = v[u] * s_kf[tc0 + u];
+        sm16(sm + O_AQ, chunk_off(r, tc0 >> 3)) = pack_bf8(w);
+        sm16(sm + O_AQ, chunk_off(r, (tc0 >> 3) + 1)) = pack_bf8(w + 8);
+        const float f = s_gm[r];
+#pragma unroll
+        for (int u = 0; u < 16; ++u) v[u] *= f;
+      }
       sm16(sm + O_DT, chunk_off(r, tc0 >> 3)) = pack_bf8(v);
       sm16(sm + O_DT, chunk_off(r, (tc0 >> 3) + 1)) = pack_bf8(v + 8);
     }
@@ -707,9 +763,16 @@ __global__ void __launch_bounds__(BT, 1)
     if (tid == 0) {
       tc_fence_after();
       const uint32_t id01 = idesc_bf16(128, 64, 0, 1), id00 = idesc_bf16(128, 64, 0, 0);
+      const uint32_t id11 = idesc_bf16(128, 64, 1, 1), id10 = idesc_bf16(128, 64, 1, 0);
       for (int kk = 0; kk < 4; ++kk) {
-        umma_bf16(X0, kdesc(sm + O_KQH2 + kk * 32), mdesc(sm + O_DT + kk * 2048, 8192), id01, 1);
-        umma_bf16(X2, kdesc(sm + O_KKH2 + kk * 32), kdesc(sm + O_DT + kk * 32), id00, 1);
+        if (SD) {
+          const uint64_t kt = mdesc(rkq + kk * 2048, 16384);
+          umma_bf16(X0, kt, mdesc(sm + O_DT + kk * 2048, 8192), id11, 1);
+          umma_bf16(X2, kt, kdesc(sm + O_AQ + kk * 32), id10, 1);
+        } else {
+          umma_bf16(X0, kdesc(sm + O_KQH2 + kk * 32), mdesc(sm + O_DT + kk * 2048, 8192), id01, 1);
+          umma_bf16(X2, kdesc(sm + O_KKH2 + kk * 32), kdesc(sm + O_DT + kk * 32), id00, 1);
+        }
       }
       umma_commit(bar_mma);
     }
@@ -1105,13 +1168,16 @@ kdn_status_t launch_fused_bwd_sweep(const Args &a, cudaStream_t s) {
       !make_map(&mdo, a.dO, a))
     return KDN_ERR_CUDA;
   const bool obf = a.odt == KDN_BF16;
-  decltype(&k_fused_bwd<0, 0, 0>) kern;
-  if (a.gates)
-    kern = a.variant == 0 ? (obf ? k_fused_bwd<0, 1, 1> : k_fused_bwd<0, 0, 1>)
-                          : (obf ? k_fused_bwd<1, 1, 1> : k_fused_bwd<1, 0, 1>);
+  decltype(&k_fused_bwd<0, 0, 0, 0>) kern;
+  if (a.variant == 0)
+    kern = a.gates ? (obf ? k_fused_bwd<0, 1, 1, 0> : k_fused_bwd<0, 0, 1, 0>)
+                   : (obf ? k_fused_bwd<0, 1, 0, 0> : k_fused_bwd<0, 0, 0, 0>);
+  else if (a.pcd)
+    kern = a.gates ? (obf ? k_fused_bwd<1, 1, 1, 0> : k_fused_bwd<1, 0, 1, 0>)
+                   : (obf ? k_fused_bwd<1, 1, 0, 0> : k_fused_bwd<1, 0, 0, 0>);
   else
-    kern = a.variant == 0 ? (obf ? k_fused_bwd<0, 1, 0> : k_fused_bwd<0, 0, 0>)
-                          : (obf ? k_fused_bwd<1, 1, 0> : k_fused_bwd<1, 0, 0>);
+    kern = a.gates ? (obf ? k_fused_bwd<1, 1, 1, 1> : k_fused_bwd<1, 0, 1, 1>)
+                   : (obf ? k_fused_bwd<1, 1, 0, 1> : k_fused_bwd<1, 0, 0, 1>);
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES) !=
       cudaSuccess)
     return KDN_ERR_CUDA;
