@@ -432,7 +432,7 @@ int kdn_kernel_launches(const kdn_desc_t *desc, int variant, int op) {
   Args a;
   if (fill_sizes(desc, variant, op == 2, &a) != KDN_OK) return -1;
   switch (op) {
-    case 0: return seg_count(a) > 1 ? 6 : use_fused(a) ? 1 : chunked_fwd_launches(a);
+    case 0: return seg_count(a) > 1 ? 5 : use_fused(a) ? 1 : chunked_fwd_launches(a);
     case 1: return (a.T > 0 && use_fused_bwd(a)) ? 2 : chunked_bwd_launches(a);
     case 2: return 1;
     case 3:

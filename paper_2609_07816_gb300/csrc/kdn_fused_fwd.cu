@@ -82,7 +82,7 @@ struct FusedParams {
   int has_g_map;  // per-channel decay tile through TMA
   int has_w_map;  // per-channel omega tile through TMA (diag)
   int write_o;    // 0: the outputs o are not written (state-saving pass of the backward)
-  int s0_eye;     // 1: the initial memory is the identity (dk = dv); S0 is ignored
+  float *phi_T;   // PH: [BH][128][128] transition of the whole sequence (from S = I, v = 0)
   unsigned char *save_S;  // optional [BH][NC] context records of the backward (kCtxBytes each)
   float *save_p;          // optional [BH][NC][128] uncertainty carry entering each chunk
 };
@@ -97,7 +97,13 @@ struct FusedParams {
 // so MMA-T runs once per K step on the raw bf16 k and q tiles (exact products,
 // no hi/lo split) and the decay ratios and beta_s are applied in fp32 when T and
 // A_qk leave TMEM; no Gamma-scaled operand tile is formed.
-template <int V, int G, int SD>
+// PH: besides the memory S (from S_0, with v), carry the transition Phi of the
+// sequence, the memory the same recurrence reaches from S = I with v = 0
+// (dk = dv).  Both share every gain, T, A and W; Phi's state pass is
+// R_Phi = -W Phi_in, Phi_out = diag(gamma_C) Phi_in + K_tail^T R_Phi.  Nothing is
+// written per token (no o, no context): the sequence-parallel forward joins the
+// segments with these two end states.
+template <int V, int G, int SD, int PH>
 __global__ void __launch_bounds__(FT, 1)
     k_fused_fwd(const __grid_constant__ CUtensorMap mq, const __grid_constant__ CUtensorMap mk,
                 const __grid_constant__ CUtensorMap mv, const __grid_constant__ CUtensorMap mg,
@@ -157,7 +163,9 @@ __global__ void __launch_bounds__(FT, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tb = *s_tbase;
-  const uint32_t TS = tb, TD1 = tb + 128, TW = tb + 256, TU = tb + 384;
+  // PH: Phi takes the columns of MMA-T's output, which then shares TW's (T has been
+  // read before MMA-W writes W, and A_qk is not needed without o)
+  const uint32_t TS = tb, TPH = tb + 128, TD1 = PH ? tb + 256 : tb + 128, TW = tb + 256, TU = tb + 384;
   const uint32_t lane_base = (uint32_t)(32 * wq) << 16;
 
   // Raw tiles of chunk c arrive on bar_raw in two groups: the decay tile as
@@ -200,9 +208,14 @@ __global__ void __launch_bounds__(FT, 1)
         }
       } else {
 #pragma unroll
-        for (int u = 0; u < 16; ++u) v[u] = (P.s0_eye && i == j0 + u) ? 1.f : 0.f;
+        for (int u = 0; u < 16; ++u) v[u] = 0.f;
       }
       tmem_st16(TS + lane_base + j0, v);
+      if (PH) {  // Phi_0 = I
+#pragma unroll
+        for (int u = 0; u < 16; ++u) v[u] = (i == j0 + u) ? 1.f : 0.f;
+        tmem_st16(TPH + lane_base + j0, v);
+      }
     }
     tmem_st_wait();
   }
@@ -679,8 +692,9 @@ __global__ void __launch_bounds__(FT, 1)
         sm16(a1l, sl * 16384 + chunk_off(r, cc0)) = pack_h8(v);
         sm16(a1l, sl * 16384 + chunk_off(r, cc0 + 1)) = pack_h8(v + 8);
       }
-      for (int cc = 2 * wg; cc < 2 * wg + 2; ++cc) sm16(a2, chunk_off(r, cc)) = make_uint4(0, 0, 0, 0);
-    } else {
+      if (!PH)
+        for (int cc = 2 * wg; cc < 2 * wg + 2; ++cc) sm16(a2, chunk_off(r, cc)) = make_uint4(0, 0, 0, 0);
+    } else if (!PH) {
       const int r = 32 * wq + lane - 64, s0 = 16 * wg;
       float v[16];
       tmem_ld16(TD1 + lane_base + s0, v);
@@ -692,6 +706,22 @@ __global__ void __launch_bounds__(FT, 1)
         v[u] = (s0 + u > r) ? 0.f : (SD ? v[u] * (fq * kf[u]) : v[u]);
       sm16(a2, chunk_off(64 + r, s0 >> 3)) = pack_h8(v);
       sm16(a2, chunk_off(64 + r, (s0 >> 3) + 1)) = pack_h8(v + 8);
+    }
+    if (PH) {  // Phi_in -> fp16 in fs (laid out like S_in in b3); diag(gamma_C) Phi_in back to TMEM
+      unsigned char *b4 = reinterpret_cast<unsigned char *>(fs);
+      const int i = 32 * wq + lane;
+      const float gC = s_gC[i];
+      for (int c0 = 0; c0 < 32; c0 += 16) {
+        float v[16];
+        const int j0 = 32 * wg + c0, sl = j0 >> 6, cc0 = (j0 & 63) >> 3;
+        tmem_ld16(TPH + lane_base + j0, v);
+        sm16(b4, sl * 16384 + chunk_off(i, cc0)) = pack_h8(v);
+        sm16(b4, sl * 16384 + chunk_off(i, cc0 + 1)) = pack_h8(v + 8);
+#pragma unroll
+        for (int u = 0; u < 16; ++u) v[u] *= gC;
+        tmem_st16(TPH + lane_base + j0, v);
+      }
+      tmem_st_wait();
     }
     fence_proxy_async();
     tc_fence_before();
@@ -710,6 +740,12 @@ __global__ void __launch_bounds__(FT, 1)
       for (int kk = 0; kk < 8; ++kk)
         umma_bf16(TU, sw128_desc(A1 + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024),
                   sw128_desc(B3 + kk * 2048, 16384, 1024), ih_S1, 1);
+      if (PH) {  // [R_Phi; .] = [-W; Qbar] Phi_in  (U = 0: v = 0 for Phi)
+        const uint32_t B4 = smem_u32(fs);
+        for (int kk = 0; kk < 8; ++kk)
+          umma_bf16(TW, sw128_desc(A1 + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024),
+                    sw128_desc(B4 + kk * 2048, 16384, 1024), ih_S1, kk > 0);
+      }
       umma_commit(bar_mma);
     }
     if (!(ok = mma_wait())) break;
@@ -723,6 +759,11 @@ __global__ void __launch_bounds__(FT, 1)
         tmem_ld16(TU + lane_base + j0, v);
         sm16(vr, sl * 8192 + chunk_off(t, cc0)) = pack_h8(v);
         sm16(vr, sl * 8192 + chunk_off(t, cc0 + 1)) = pack_h8(v + 8);
+        if (PH) {  // R_Phi -> a2, the same layout
+          tmem_ld16(TW + lane_base + j0, v);
+          sm16(a2, sl * 8192 + chunk_off(t, cc0)) = pack_h8(v);
+          sm16(a2, sl * 8192 + chunk_off(t, cc0 + 1)) = pack_h8(v + 8);
+        }
       }
     }
     fence_proxy_async();
@@ -738,8 +779,11 @@ __global__ void __launch_bounds__(FT, 1)
       const uint32_t A2 = smem_u32(a2), B1 = smem_u32(b1l), VR = smem_u32(vr);
       for (int kk = 0; kk < 4; ++kk) {
         const uint64_t bd = sw128_desc(VR + kk * 2048, 8192, 1024);
-        umma_bf16(TU, sw128_desc(A2 + kk * 32, 16, 1024), bd, ih_S1, 1);
+        if (!PH) umma_bf16(TU, sw128_desc(A2 + kk * 32, 16, 1024), bd, ih_S1, 1);
         umma_bf16(TS, sw128_desc(B1 + kk * 2048, 8192, 1024), bd, ih_S2, 1);
+        if (PH)  // Phi += K_tail^T R_Phi
+          umma_bf16(TPH, sw128_desc(B1 + kk * 2048, 8192, 1024), sw128_desc(A2 + kk * 2048, 8192, 1024),
+                    ih_S2, 1);
       }
       umma_commit(bar_mma);
     }
@@ -798,6 +842,17 @@ __global__ void __launch_bounds__(FT, 1)
         for (int u = 0; u < 4; ++u) dst[u] = make_float4(v[4 * u], v[4 * u + 1], v[4 * u + 2], v[4 * u + 3]);
       }
     }
+    if (PH && P.phi_T) {
+      const int i = 32 * wq + lane;
+      for (int c0 = 0; c0 < 32; c0 += 16) {
+        float v[16];
+        const int j0 = 32 * wg + c0;
+        tmem_ld16(TPH + lane_base + j0, v);
+        float4 *dst = reinterpret_cast<float4 *>(P.phi_T + ((size_t)bh * D + i) * D + j0);
+#pragma unroll
+        for (int u = 0; u < 4; ++u) dst[u] = make_float4(v[4 * u], v[4 * u + 1], v[4 * u + 2], v[4 * u + 3]);
+      }
+    }
     if (a.pT) {
       if (V == 0 && tid < D) a.pT[(size_t)bh * D + tid] = s_p[tid];
       if (V == 1 && tid == 0) a.pT[bh] = s_b[0];
@@ -830,27 +885,20 @@ bool fused_fwd_supported(const Args &a) {
 int fused_fwd_smem_bytes() { return SMEM_BYTES; }
 
 kdn_status_t launch_fused_fwd(const Args &a, cudaStream_t s, unsigned char *save_S,
-                              float *save_p, bool write_o, bool s0_eye, const void *v_zero) {
+                              float *save_p, bool write_o, float *phi_T) {
+  // the transition pass writes nothing per token
+  if (phi_T && (save_S || save_p || write_o)) return KDN_ERR_INVALID_ARG;
   FusedParams P;
   P.a = a;
   P.has_g_map = (a.variant == 0 || a.pcd) ? 1 : 0;
   P.has_w_map = a.variant == 0 ? 1 : 0;
   P.write_o = write_o ? 1 : 0;
-  P.s0_eye = s0_eye ? 1 : 0;
+  P.phi_T = phi_T;
   P.save_S = save_S;
   P.save_p = save_p;
   CUtensorMap mq, mk, mv, mg, mw, mo;
-  if (!make_map(&mq, a.q, a) || !make_map(&mk, a.k, a)) return KDN_ERR_CUDA;
-  if (v_zero) {
-    // v = 0: a map over one zeroed 64-token block of a single sequence; every
-    // other chunk lies outside it and the TMA fills the tile with zeros.
-    Args az = a;
-    az.B = 1;
-    az.T = 64;
-    if (!make_map(&mv, v_zero, az)) return KDN_ERR_CUDA;
-  } else if (!make_map(&mv, a.v, a)) {
+  if (!make_map(&mq, a.q, a) || !make_map(&mk, a.k, a) || !make_map(&mv, a.v, a))
     return KDN_ERR_CUDA;
-  }
   if (P.write_o ? !make_map(&mo, a.o, a, a.odt != KDN_BF16) : !make_map(&mo, a.q, a))
     return KDN_ERR_CUDA;
   mg = mq;
@@ -858,9 +906,15 @@ kdn_status_t launch_fused_fwd(const Args &a, cudaStream_t s, unsigned char *save
   if (P.has_g_map && !make_map(&mg, a.g, a)) return KDN_ERR_CUDA;
   if (P.has_w_map && !make_map(&mw, a.omega, a)) return KDN_ERR_CUDA;
   const int BH = a.B * a.H;
-  auto kern = a.variant == 0 ? (a.gates ? k_fused_fwd<0, 1, 0> : k_fused_fwd<0, 0, 0>)
-               : a.pcd     ? (a.gates ? k_fused_fwd<1, 1, 0> : k_fused_fwd<1, 0, 0>)
-                           : (a.gates ? k_fused_fwd<1, 1, 1> : k_fused_fwd<1, 0, 1>);
+  const int sd = a.variant == 1 && !a.pcd;
+  using K = decltype(&k_fused_fwd<0, 0, 0, 0>);
+  // [variant][gates][scalar decay][transition]
+  static const K kerns[2][2][2][2] = {
+      {{{k_fused_fwd<0, 0, 0, 0>, k_fused_fwd<0, 0, 0, 1>}, {nullptr, nullptr}},
+       {{k_fused_fwd<0, 1, 0, 0>, k_fused_fwd<0, 1, 0, 1>}, {nullptr, nullptr}}},
+      {{{k_fused_fwd<1, 0, 0, 0>, k_fused_fwd<1, 0, 0, 1>}, {k_fused_fwd<1, 0, 1, 0>, k_fused_fwd<1, 0, 1, 1>}},
+       {{k_fused_fwd<1, 1, 0, 0>, k_fused_fwd<1, 1, 0, 1>}, {k_fused_fwd<1, 1, 1, 0>, k_fused_fwd<1, 1, 1, 1>}}}};
+  const K kern = kerns[a.variant][a.gates ? 1 : 0][sd][phi_T ? 1 : 0];
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES) !=
       cudaSuccess)
     return KDN_ERR_CUDA;

@@ -139,12 +139,12 @@ size_t workspace_layout(Args *a, char *base, bool bwd);
 // `save_S` / `save_p` it also stores the context of the fused backward: the
 // fp16 image of every chunk's entry memory (32 KB) and the uncertainty entering
 // every chunk (128 floats); `write_o` = false skips the outputs o.
-// `s0_eye` starts every sequence from S = I (dk = dv) instead of a.S0; `v_zero`
-// (a zeroed device buffer of 64 * H * 128 bf16) replaces v by zeros.
+// `phi_T` ([B*H][128][128]) selects the transition pass: besides the memory from
+// a.S0 with v (to a.ST), every sequence also carries the memory the recurrence
+// reaches from S = I with v = 0, written to phi_T; no o and no context then.
 bool fused_fwd_supported(const Args &a);
 kdn_status_t launch_fused_fwd(const Args &a, cudaStream_t s, unsigned char *save_S = nullptr,
-                              float *save_p = nullptr, bool write_o = true, bool s0_eye = false,
-                              const void *v_zero = nullptr);
+                              float *save_p = nullptr, bool write_o = true, float *phi_T = nullptr);
 // Fused tcgen05 backward (Diagonal KDN, bf16, dk = dv = 128, 64-token chunks):
 // one reverse sweep per (batch, head) from the saved context in a.fSin / a.fpin.
 // launch_fused_bwd first runs the context-saving forward (without o).

@@ -16,11 +16,14 @@
 //  * Memory.  With the gains fixed, the chunked recurrence (App. F) is linear in
 //    (S_in, v) jointly, so a segment's exit memory is Phi S_in + S_out|(S_in = 0),
 //    where the transition Phi (d_k x d_k) is the exit memory of a run from S = I
-//    with v = 0.  A short sequential pass over segments then gives every
-//    segment's exact entry memory, and a last run of all segments writes o.
+//    with v = 0.  One fused pass carries both memories (they share every gain
+//    and WY factor; only the state products are doubled).  A short sequential
+//    pass over segments then gives every segment's exact entry memory, and a last
+//    run of all segments writes o.
 //
-// Cost: three fused runs over T / P tokens instead of one over T, plus two light
-// passes over the gates; used when P >= 4 segments of >= 8 chunks fit.
+// Cost: two fused runs over T / P tokens instead of one over T (the first with
+// a second state pass), plus two light passes over the gates; used when P >= 4
+// segments of >= 8 chunks fit.
 #include "kdn_internal.cuh"
 
 namespace kdn {
@@ -292,8 +295,7 @@ int seg_count(const Args &a) {
 size_t seg_workspace_bytes(const Args &a, int P) {
   const size_t BH = (size_t)a.B * a.H, Pn = a.variant == 0 ? D : 1, NC = a.T / CM;
   auto r = [](size_t x) { return (x + 255) / 256 * 256; };
-  return r(BH * NC * Pn * 16) + r(BH * P * Pn * 4) * 2 + r(BH * P * D * D * 4) * 3 +
-         r((size_t)CM * a.H * D * 2);
+  return r(BH * NC * Pn * 16) + r(BH * P * Pn * 4) * 2 + r(BH * P * D * D * 4) * 3;
 }
 
 kdn_status_t launch_seg_fwd(const Args &a, int P, char *ws, cudaStream_t s) {
@@ -306,10 +308,8 @@ kdn_status_t launch_seg_fwd(const Args &a, int P, char *ws, cudaStream_t s) {
   float *pbuf = reinterpret_cast<float *>(p); p += r(BH * P * Pn * 4);
   float *S0seg = reinterpret_cast<float *>(p); p += r(BH * P * nS * 4);
   float *Sv = reinterpret_cast<float *>(p); p += r(BH * P * nS * 4);
-  float *Sphi = reinterpret_cast<float *>(p); p += r(BH * P * nS * 4);
-  void *vzero = p;
+  float *Sphi = reinterpret_cast<float *>(p);
 
-  if (cudaMemsetAsync(vzero, 0, (size_t)CM * a.H * D * 2, s) != cudaSuccess) return KDN_ERR_CUDA;
   if (cudaMemsetAsync(S0seg, 0, BH * P * nS * 4, s) != cudaSuccess) return KDN_ERR_CUDA;
   if (a.S0 && cudaMemcpy2DAsync(S0seg, (size_t)P * seqS * 4, a.S0, seqS * 4, seqS * 4, a.B,
                                 cudaMemcpyDeviceToDevice, s) != cudaSuccess)
@@ -335,20 +335,16 @@ kdn_status_t launch_seg_fwd(const Args &a, int P, char *ws, cudaStream_t s) {
   sa.p0 = pseg;
   sa.o = nullptr;
   sa.pT = nullptr;
-  // (1) from S_in = 0 (S_0 for the first segment) with v
+  // (1) one pass carries two memories through every segment: from S_in = 0 (S_0
+  // for the first segment) with v, and from S = I with v = 0 (the transition Phi)
   sa.S0 = S0seg;
   sa.ST = Sv;
-  kdn_status_t st = launch_fused_fwd(sa, s, nullptr, nullptr, false);
-  if (st != KDN_OK) return st;
-  // (2) from S = I with v = 0: the transition Phi of every segment
-  sa.S0 = nullptr;
-  sa.ST = Sphi;
-  st = launch_fused_fwd(sa, s, nullptr, nullptr, false, true, vzero);
+  kdn_status_t st = launch_fused_fwd(sa, s, nullptr, nullptr, false, Sphi);
   if (st != KDN_OK) return st;
   // exact entry memories
   k_seg_combine<<<dim3(D / 16, (unsigned)BH), 256, 0, s>>>(a, P, Sv, Sphi, S0seg);
   if (cudaGetLastError() != cudaSuccess) return KDN_ERR_CUDA;
-  // (3) every segment from its exact entry state: o, and the final state
+  // (2) every segment from its exact entry state: o, and the final state
   sa.S0 = S0seg;
   sa.o = a.o;
   sa.ST = a.ST ? Sphi : nullptr;

@@ -114,7 +114,7 @@ def test_logit_gates_sequence_parallel_forward(kdn, variant, pc):
     ins["g"] = round_to(rng.normal(6.0, 1.0, ins["g"].shape), "bf16")
     desc = kdn.make_desc(B, T, H, 128, 128, kdn.KDN_BF16, decay_per_channel=int(pc),
                          gates=kdn.KDN_GATES_LOGITS, r_min=R_MIN)
-    assert kdn.kdn_kernel_launches(desc, 0 if variant == "diag" else 1, 0) == 6
+    assert kdn.kdn_kernel_launches(desc, 0 if variant == "diag" else 1, 0) == 5
     fwd = kdn.kdn_diag_fwd if variant == "diag" else kdn.kdn_iso_fwd
     d = to_dev(ins)
     o, ST, pT = fwd(*[d[n] for n in NAMES], d["S0"], d["p0"], gates=kdn.KDN_GATES_LOGITS,
