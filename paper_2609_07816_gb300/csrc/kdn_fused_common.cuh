@@ -207,7 +207,9 @@ inline PFN_cuTensorMapEncodeTiled_v12000 encoder() {
 
 // [B, T, H, 128] tensor of 2- or 4-byte elements; box = 128 bytes of channels
 // x 1 head x 64 tokens x 1 batch, 128-byte swizzle.
-inline bool make_map(CUtensorMap *m, const void *ptr, const Args &a, bool fp32 = false) {
+// f16: fp16 elements (else bf16) when not fp32.
+inline bool make_map(CUtensorMap *m, const void *ptr, const Args &a, bool fp32 = false,
+                     bool f16 = false) {
   auto enc = encoder();
   if (!enc) return false;
   const cuuint64_t es_bytes = fp32 ? 4 : 2;
@@ -217,7 +219,10 @@ inline bool make_map(CUtensorMap *m, const void *ptr, const Args &a, bool fp32 =
                            (cuuint64_t)a.T * a.H * D * es_bytes};
   cuuint32_t box[4] = {fp32 ? 32u : 64u, 1, 64, 1};
   cuuint32_t es[4] = {1, 1, 1, 1};
-  return enc(m, fp32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4,
+  const CUtensorMapDataType dt = fp32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32
+                                 : f16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16
+                                       : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
+  return enc(m, dt, 4,
              const_cast<void *>(ptr), dims, strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
              CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;

@@ -100,15 +100,17 @@ struct FusedParams {
 // PH: besides the memory S (from S_0, with v), carry the transition Phi of the
 // sequence, the memory the same recurrence reaches from S = I with v = 0
 // (dk = dv).  Both share every gain, T, A and W; Phi's state pass is
-// R_Phi = -W Phi_in, Phi_out = diag(gamma_C) Phi_in + K_tail^T R_Phi.  Nothing is
-// written per token (no o, no context): the sequence-parallel forward joins the
-// segments with these two end states.
+// R_Phi = -W Phi_in, Phi_out = diag(gamma_C) Phi_in + K_tail^T R_Phi.  Per token
+// it writes o from the memory (float32, map mo) and o_Phi = tau Phi_t^T q_t, the
+// output the transition state would give (fp16, map mo2); the sequence-parallel
+// forward joins the segments with the two end states and then forms the exact
+// output o + S_in^T o_Phi.  No context is saved.
 template <int V, int G, int SD, int PH>
 __global__ void __launch_bounds__(FT, 1)
     k_fused_fwd(const __grid_constant__ CUtensorMap mq, const __grid_constant__ CUtensorMap mk,
                 const __grid_constant__ CUtensorMap mv, const __grid_constant__ CUtensorMap mg,
                 const __grid_constant__ CUtensorMap mw, const __grid_constant__ CUtensorMap mo,
-                const FusedParams P) {
+                const __grid_constant__ CUtensorMap mo2, const FusedParams P) {
   const Args &a = P.a;
   extern __shared__ unsigned char smraw[];
   unsigned char *sm =
@@ -585,6 +587,20 @@ __global__ void __launch_bounds__(FT, 1)
 #pragma unroll
       for (int u = 0; u < 4; ++u)
         *reinterpret_cast<float4 *>(sT + r * LT + s0 + 4 * u) = make_float4(v[4 * u], v[4 * u + 1], v[4 * u + 2], v[4 * u + 3]);
+    } else if (PH) {
+      // A_qk leaves TMEM now: MMA-W overwrites it (TD1 = TW).  fp16 into rows
+      // 64..127 of a2, which MMA-W reads only into accumulator rows nobody reads
+      const int r = 32 * wq + lane - 64, s0 = 16 * wg;
+      float v[16];
+      tmem_ld16(TD1 + lane_base + s0, v);
+      float kf[16];
+      if (SD) ld_f16(s_kf + s0, kf);
+      const float fq = SD ? a.tau * s_gm[r] : 1.f;
+#pragma unroll
+      for (int u = 0; u < 16; ++u)
+        v[u] = (s0 + u > r) ? 0.f : (SD ? v[u] * (fq * kf[u]) : v[u]);
+      sm16(a2, chunk_off(64 + r, s0 >> 3)) = pack_h8(v);
+      sm16(a2, chunk_off(64 + r, (s0 >> 3) + 1)) = pack_h8(v + 8);
     }
     __syncthreads();
     tri_inverse64(sT, sA, sX);
@@ -597,7 +613,9 @@ __global__ void __launch_bounds__(FT, 1)
         const int sidx = 8 * cc + j;
         v[j] = (r < 64 && sidx <= r) ? sA[r * LT + sidx] : 0.f;
       }
-      if (SD) {  // W = (A diag(gamma)) K
+      if (PH && r >= 64) {
+        // rows 64..127 of a2 hold A_qk (PH)
+      } else if (SD) {  // W = (A diag(gamma)) K
         float w[8], gm[8];
         ld_f8(s_gm + 8 * cc, gm);
 #pragma unroll
@@ -692,8 +710,7 @@ __global__ void __launch_bounds__(FT, 1)
         sm16(a1l, sl * 16384 + chunk_off(r, cc0)) = pack_h8(v);
         sm16(a1l, sl * 16384 + chunk_off(r, cc0 + 1)) = pack_h8(v + 8);
       }
-      if (!PH)
-        for (int cc = 2 * wg; cc < 2 * wg + 2; ++cc) sm16(a2, chunk_off(r, cc)) = make_uint4(0, 0, 0, 0);
+      for (int cc = 2 * wg; cc < 2 * wg + 2; ++cc) sm16(a2, chunk_off(r, cc)) = make_uint4(0, 0, 0, 0);
     } else if (!PH) {
       const int r = 32 * wq + lane - 64, s0 = 16 * wg;
       float v[16];
@@ -759,10 +776,11 @@ __global__ void __launch_bounds__(FT, 1)
         tmem_ld16(TU + lane_base + j0, v);
         sm16(vr, sl * 8192 + chunk_off(t, cc0)) = pack_h8(v);
         sm16(vr, sl * 8192 + chunk_off(t, cc0 + 1)) = pack_h8(v + 8);
-        if (PH) {  // R_Phi -> a2, the same layout
+        if (PH) {  // R_Phi -> fs (Phi_in has been read), the same layout
+          unsigned char *rp = reinterpret_cast<unsigned char *>(fs);
           tmem_ld16(TW + lane_base + j0, v);
-          sm16(a2, sl * 8192 + chunk_off(t, cc0)) = pack_h8(v);
-          sm16(a2, sl * 8192 + chunk_off(t, cc0 + 1)) = pack_h8(v + 8);
+          sm16(rp, sl * 8192 + chunk_off(t, cc0)) = pack_h8(v);
+          sm16(rp, sl * 8192 + chunk_off(t, cc0 + 1)) = pack_h8(v + 8);
         }
       }
     }
@@ -779,11 +797,13 @@ __global__ void __launch_bounds__(FT, 1)
       const uint32_t A2 = smem_u32(a2), B1 = smem_u32(b1l), VR = smem_u32(vr);
       for (int kk = 0; kk < 4; ++kk) {
         const uint64_t bd = sw128_desc(VR + kk * 2048, 8192, 1024);
-        if (!PH) umma_bf16(TU, sw128_desc(A2 + kk * 32, 16, 1024), bd, ih_S1, 1);
+        umma_bf16(TU, sw128_desc(A2 + kk * 32, 16, 1024), bd, ih_S1, 1);
         umma_bf16(TS, sw128_desc(B1 + kk * 2048, 8192, 1024), bd, ih_S2, 1);
-        if (PH)  // Phi += K_tail^T R_Phi
-          umma_bf16(TPH, sw128_desc(B1 + kk * 2048, 8192, 1024), sw128_desc(A2 + kk * 2048, 8192, 1024),
-                    ih_S2, 1);
+        if (PH) {  // O_Phi += A_qk R_Phi;  Phi += K_tail^T R_Phi
+          const uint64_t bp = sw128_desc(smem_u32(fs) + kk * 2048, 8192, 1024);
+          umma_bf16(TW, sw128_desc(A2 + kk * 32, 16, 1024), bp, ih_S1, 1);
+          umma_bf16(TPH, sw128_desc(B1 + kk * 2048, 8192, 1024), bp, ih_S2, 1);
+        }
       }
       umma_commit(bar_mma);
     }
@@ -814,6 +834,12 @@ __global__ void __launch_bounds__(FT, 1)
                 make_uint4(__float_as_uint(v[4 * m]), __float_as_uint(v[4 * m + 1]),
                            __float_as_uint(v[4 * m + 2]), __float_as_uint(v[4 * m + 3]));
         }
+        if (PH) {  // O_Phi (rows 64..127 of TW) -> fp16 staging in a2, boxes of 64 columns
+          tmem_ld16(TW + lane_base + j0, v);
+          const int bx = j0 >> 6, cc = (j0 & 63) >> 3;
+          sm16(a2, bx * 8192 + chunk_off(t, cc)) = pack_h8(v);
+          sm16(a2, bx * 8192 + chunk_off(t, cc + 1)) = pack_h8(v + 8);
+        }
       }
     }
     fence_proxy_async();
@@ -822,6 +848,8 @@ __global__ void __launch_bounds__(FT, 1)
       const unsigned char *stg = reinterpret_cast<const unsigned char *>(fs);
       const int nbox = a.odt == KDN_BF16 ? 2 : 4, bw = a.odt == KDN_BF16 ? 64 : 32;
       for (int bx = 0; bx < nbox; ++bx) tma_store_4d(&mo, stg + bx * 8192, bx * bw, h, c * CM, b);
+      if (PH)
+        for (int bx = 0; bx < 2; ++bx) tma_store_4d(&mo2, a2 + bx * 8192, bx * 64, h, c * CM, b);
       bulk_commit();
     }
     tc_fence_before();
@@ -885,9 +913,10 @@ bool fused_fwd_supported(const Args &a) {
 int fused_fwd_smem_bytes() { return SMEM_BYTES; }
 
 kdn_status_t launch_fused_fwd(const Args &a, cudaStream_t s, unsigned char *save_S,
-                              float *save_p, bool write_o, float *phi_T) {
-  // the transition pass writes nothing per token
-  if (phi_T && (save_S || save_p || write_o)) return KDN_ERR_INVALID_ARG;
+                              float *save_p, bool write_o, float *phi_T, void *o_phi) {
+  // the transition pass writes o (float32) and o_Phi, and no context
+  if (phi_T && (save_S || save_p || !write_o || !o_phi || a.odt != KDN_F32))
+    return KDN_ERR_INVALID_ARG;
   FusedParams P;
   P.a = a;
   P.has_g_map = (a.variant == 0 || a.pcd) ? 1 : 0;
@@ -896,11 +925,12 @@ kdn_status_t launch_fused_fwd(const Args &a, cudaStream_t s, unsigned char *save
   P.phi_T = phi_T;
   P.save_S = save_S;
   P.save_p = save_p;
-  CUtensorMap mq, mk, mv, mg, mw, mo;
+  CUtensorMap mq, mk, mv, mg, mw, mo, mo2;
   if (!make_map(&mq, a.q, a) || !make_map(&mk, a.k, a) || !make_map(&mv, a.v, a))
     return KDN_ERR_CUDA;
   if (P.write_o ? !make_map(&mo, a.o, a, a.odt != KDN_BF16) : !make_map(&mo, a.q, a))
     return KDN_ERR_CUDA;
+  if (phi_T ? !make_map(&mo2, o_phi, a, false, true) : !make_map(&mo2, a.q, a)) return KDN_ERR_CUDA;
   mg = mq;
   mw = mq;
   if (P.has_g_map && !make_map(&mg, a.g, a)) return KDN_ERR_CUDA;
@@ -918,7 +948,7 @@ kdn_status_t launch_fused_fwd(const Args &a, cudaStream_t s, unsigned char *save
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES) !=
       cudaSuccess)
     return KDN_ERR_CUDA;
-  kern<<<BH, FT, SMEM_BYTES, s>>>(mq, mk, mv, mg, mw, mo, P);
+  kern<<<BH, FT, SMEM_BYTES, s>>>(mq, mk, mv, mg, mw, mo, mo2, P);
   return cudaGetLastError() == cudaSuccess ? KDN_OK : KDN_ERR_CUDA;
 }
 

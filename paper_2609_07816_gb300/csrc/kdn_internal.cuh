@@ -140,11 +140,13 @@ size_t workspace_layout(Args *a, char *base, bool bwd);
 // fp16 image of every chunk's entry memory (32 KB) and the uncertainty entering
 // every chunk (128 floats); `write_o` = false skips the outputs o.
 // `phi_T` ([B*H][128][128]) selects the transition pass: besides the memory from
-// a.S0 with v (to a.ST), every sequence also carries the memory the recurrence
-// reaches from S = I with v = 0, written to phi_T; no o and no context then.
+// a.S0 with v (to a.ST, its output to a.o, float32), every sequence also carries
+// the memory the recurrence reaches from S = I with v = 0, written to phi_T, and
+// its output tau Phi_t^T q_t to `o_phi` (fp16, the layout of o); no context then.
 bool fused_fwd_supported(const Args &a);
 kdn_status_t launch_fused_fwd(const Args &a, cudaStream_t s, unsigned char *save_S = nullptr,
-                              float *save_p = nullptr, bool write_o = true, float *phi_T = nullptr);
+                              float *save_p = nullptr, bool write_o = true, float *phi_T = nullptr,
+                              void *o_phi = nullptr);
 // Fused tcgen05 backward (Diagonal KDN, bf16, dk = dv = 128, 64-token chunks):
 // one reverse sweep per (batch, head) from the saved context in a.fSin / a.fpin.
 // launch_fused_bwd first runs the context-saving forward (without o).

@@ -17,14 +17,18 @@
 //    (S_in, v) jointly, so a segment's exit memory is Phi S_in + S_out|(S_in = 0),
 //    where the transition Phi (d_k x d_k) is the exit memory of a run from S = I
 //    with v = 0.  One fused pass carries both memories (they share every gain
-//    and WY factor; only the state products are doubled).  A short sequential
-//    pass over segments then gives every segment's exact entry memory, and a last
-//    run of all segments writes o.
+//    and WY factor; only the state products are doubled) and writes both
+//    outputs per token.  A short sequential pass over segments then gives every
+//    segment's exact entry memory S_in(j).
+//  * Output.  By the same linearity o_t = o_v,t + S_in(j)^T o_Phi,t: one dense
+//    128 x 128 product per token on the tensor cores (k_seg_out).
 //
-// Cost: two fused runs over T / P tokens instead of one over T (the first with
-// a second state pass), plus two light passes over the gates; used when P >= 4
-// segments of >= 8 chunks fit.
+// Cost: one fused run over T / P tokens (with a second state pass) instead of
+// one over T, plus light passes over the gates and the outputs; used when
+// P >= 4 segments of >= 8 chunks fit.
 #include "kdn_internal.cuh"
+#include "kdn_sm103.cuh"
+#include "kdn_fused_common.cuh"
 
 namespace kdn {
 namespace {
@@ -230,13 +234,14 @@ __global__ void __launch_bounds__(D * kScanGroups) k_seg_scan(const Args a, floa
   }
 }
 
-// Entry memory of every segment j >= 1:  S_in(1) = Sv(0),
-// S_in(j + 1) = Phi(j) S_in(j) + Sv(j), with Sv(j) the exit memory of the run
-// from S_in = 0 (the true S_0 for j = 0) and Phi(j) the exit memory of the run
-// from S = I with v = 0.  Columns of the memory are independent: a CTA owns 16
-// of them for one (batch, head); thread (row, half) holds 8 entries.
+// Entry memory of every segment:  S_in(0) = S_0 (0 when absent), then
+// S_in(j + 1) = Phi(j) S_in(j) + Sv(j), with Sv(j) the exit memory of segment j
+// run from S_in = 0 with v and Phi(j) its exit memory from S = I with v = 0;
+// S_in(P) is the final memory S_T (written when ST is given).  Columns of the
+// memory are independent: a CTA owns 16 of them for one (batch, head); thread
+// (row, half) holds 8 entries.
 __global__ void __launch_bounds__(256) k_seg_combine(const Args a, int P, const float *Sv,
-                                                     const float *Sphi, float *S0seg) {
+                                                     const float *Sphi, float *S0seg, float *ST) {
   __shared__ __align__(16) float sS[D][16];
   const int bh = blockIdx.y, b = bh / a.H, h = bh % a.H;
   const int tid = threadIdx.x, row = tid >> 1, half = tid & 1;
@@ -244,16 +249,13 @@ __global__ void __launch_bounds__(256) k_seg_combine(const Args a, int P, const 
   auto ent = [&](int j) { return ((size_t)(b * P + j) * a.H + h) * D * D; };
   float acc[8];
   {
-    const float4 *src = reinterpret_cast<const float4 *>(Sv + ent(0) + (size_t)row * D + col);
+    const float4 *src = reinterpret_cast<const float4 *>(S0seg + ent(0) + (size_t)row * D + col);
     const float4 x0 = src[0], x1 = src[1];
     acc[0] = x0.x; acc[1] = x0.y; acc[2] = x0.z; acc[3] = x0.w;
     acc[4] = x1.x; acc[5] = x1.y; acc[6] = x1.z; acc[7] = x1.w;
   }
-  for (int j = 1; j < P; ++j) {
-    float4 *dst = reinterpret_cast<float4 *>(S0seg + ent(j) + (size_t)row * D + col);
-    dst[0] = make_float4(acc[0], acc[1], acc[2], acc[3]);
-    dst[1] = make_float4(acc[4], acc[5], acc[6], acc[7]);
-    if (j == P - 1) break;
+  for (int j = 0; j < P; ++j) {  // acc = S_in(j)
+    if (j == P - 1 && !ST) break;
 #pragma unroll
     for (int u = 0; u < 8; ++u) sS[row][half * 8 + u] = acc[u];
     __syncthreads();
@@ -277,7 +279,149 @@ __global__ void __launch_bounds__(256) k_seg_combine(const Args a, int P, const 
       }
     }
     __syncthreads();
+    float *base = j + 1 < P ? S0seg + ent(j + 1) : ST + (size_t)bh * D * D;
+    float4 *dst = reinterpret_cast<float4 *>(base + (size_t)row * D + col);
+    dst[0] = make_float4(acc[0], acc[1], acc[2], acc[3]);
+    dst[1] = make_float4(acc[4], acc[5], acc[6], acc[7]);
   }
+}
+
+// Exact output of every token:  o_t = o_v,t + S_in(j)^T o_Phi,t, with o_v the
+// output of the run from S_in = 0 with v, o_Phi,t = tau Phi_t^T q_t that of the
+// transition run, and S_in(j) the entry memory of the token's segment j (the
+// recurrence is linear in S_in).  One CTA per (128-token tile, head, batch):
+// TMA brings the o_Phi tile (fp16, K-major A) and the o_v tile (fp32); S_in(j)
+// is converted to the fp16 MN-major B operand (the layout of MMA-S1's S_in in
+// the fused forward); eight tcgen05 MMAs (M = N = 128, K = 16 each) form
+// o_Phi S_in in TMEM, the epilogue adds o_v and TMA stores the tile.  Segments
+// are whole 64-token chunks, so a tile whose second half starts a new segment
+// also forms o_Phi S_in(j + 1) (a second operand and accumulator) for that half.
+constexpr int kOutT = 128, kOutThreads = 128;
+constexpr int kOutSmem = 32768 + 2 * 32768 + 65536 + 64 + 1024;
+constexpr uint32_t kOutWait = 1u << 25;
+
+__global__ void __launch_bounds__(kOutThreads, 1)
+    k_seg_out(const __grid_constant__ CUtensorMap m_ophi, const __grid_constant__ CUtensorMap m_ov,
+              const __grid_constant__ CUtensorMap m_o, const Args a, int P, const float *S0seg) {
+  using namespace sm103;
+  using namespace fused;
+  extern __shared__ unsigned char smraw[];
+  unsigned char *sm =
+      reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(smraw) + 1023) & ~uintptr_t(1023));
+  unsigned char *sA = sm, *sB = sm + 32768, *sO = sm + 98304;
+  uint64_t *bars = reinterpret_cast<uint64_t *>(sm + 163840);
+  uint64_t *bar_a = bars, *bar_o = bars + 1, *bar_m = bars + 2;
+  uint32_t *s_tbase = reinterpret_cast<uint32_t *>(bars + 4);
+  const int tid = threadIdx.x, warp = tid >> 5;
+  const int t0 = blockIdx.x * kOutT, h = blockIdx.y, b = blockIdx.z;
+  // segments of the two 64-token halves (a last tile may hold only the first;
+  // the TMA fills and clips the tokens past T)
+  const int seg = t0 / (a.T / P), seg2 = t0 + 64 < a.T ? (t0 + 64) / (a.T / P) : seg;
+  const bool two = seg2 != seg;
+  if (tid == 0) {
+    mbar_init(bar_a, 1);
+    mbar_init(bar_o, 1);
+    mbar_init(bar_m, 1);
+    fence_mbar_init();
+    mbar_expect_tx(bar_a, 32768);
+    for (int sl = 0; sl < 2; ++sl)
+      for (int th = 0; th < 2; ++th)  // slab sl: rows 0..63 (th 0), 64..127 (th 1)
+        tma_load_4d(sA + sl * 16384 + th * 8192, &m_ophi, bar_a, 64 * sl, h, t0 + 64 * th, b);
+    mbar_expect_tx(bar_o, 65536);
+    for (int bx = 0; bx < 4; ++bx)
+      for (int th = 0; th < 2; ++th)
+        tma_load_4d(sO + (bx * 2 + th) * 8192, &m_ov, bar_o, 32 * bx, h, t0 + 64 * th, b);
+  }
+  if (warp == 0) {
+    tmem_alloc(s_tbase, 256);
+    tmem_relinquish();
+  }
+  // S_in(seg) row i -> fp16, MN-major: 64 value columns per 128-byte row, two slabs
+  for (int u = 0; u < (two ? 2 : 1); ++u) {
+    const int i = tid;
+    const float4 *src = reinterpret_cast<const float4 *>(
+        S0seg + (((size_t)(b * P + seg + u) * a.H + h) * D + i) * D);
+    unsigned char *dst = sB + u * 32768;
+#pragma unroll 4
+    for (int c8 = 0; c8 < 16; ++c8) {
+      const float4 x0 = src[2 * c8], x1 = src[2 * c8 + 1];
+      const float v[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
+      sm16(dst, (c8 >> 3) * 16384 + chunk_off(i, c8 & 7)) = pack_h8(v);
+    }
+  }
+  fence_proxy_async();
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tb = *s_tbase;
+  bool ok = true;
+  if (tid == 0) {
+    ok = mbar_wait(bar_a, 0, kOutWait);
+    if (ok) {
+      const uint32_t id = idesc_f16(128, 128, 0, 1), A = smem_u32(sA), B = smem_u32(sB);
+      for (int u = 0; u < (two ? 2 : 1); ++u)
+        for (int kk = 0; kk < 8; ++kk)
+          umma_bf16(tb + 128 * u, sw128_desc(A + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024),
+                    sw128_desc(B + u * 32768 + kk * 2048, 16384, 1024), id, kk > 0);
+      umma_commit(bar_m);
+      ok = mbar_wait(bar_m, 0, kOutWait) && mbar_wait(bar_o, 0, kOutWait);
+    }
+  }
+  ok = __syncthreads_and(ok);
+  if (ok) {
+    tc_fence_after();
+    // token t = tid: TMEM lane t; o_v row t % 64 of box (column group, t / 64)
+    const int t = tid, r = t & 63, th = t >> 6;
+    const bool obf = a.odt == KDN_BF16;
+    const uint32_t acc = tb + ((two && th) ? 128u : 0u);  // the second half's segment
+    for (int j0 = 0; j0 < D; j0 += 16) {
+      float v[16];
+      tmem_ld16(acc + ((uint32_t)(32 * warp) << 16) + j0, v);
+      const int bx = j0 >> 5, cc = (j0 & 31) >> 2;
+      unsigned char *box = sO + (bx * 2 + th) * 8192;
+#pragma unroll
+      for (int m = 0; m < 4; ++m) {
+        uint4 &u = sm16(box, chunk_off(r, cc + m));
+        v[4 * m] += __uint_as_float(u.x);
+        v[4 * m + 1] += __uint_as_float(u.y);
+        v[4 * m + 2] += __uint_as_float(u.z);
+        v[4 * m + 3] += __uint_as_float(u.w);
+        if (!obf)
+          u = make_uint4(__float_as_uint(v[4 * m]), __float_as_uint(v[4 * m + 1]),
+                         __float_as_uint(v[4 * m + 2]), __float_as_uint(v[4 * m + 3]));
+      }
+      if (obf) {  // bf16 o: boxes of 64 columns over the o_Phi tile (read by the MMAs)
+        const int bb = j0 >> 6, c2 = (j0 & 63) >> 3;
+        unsigned char *ob = sA + (bb * 2 + th) * 8192;
+        sm16(ob, chunk_off(r, c2)) = pack_bf8(v);
+        sm16(ob, chunk_off(r, c2 + 1)) = pack_bf8(v + 8);
+      }
+    }
+    fence_proxy_async();
+  }
+  __syncthreads();
+  if (tid == 0) {
+    if (ok) {
+      if (a.odt == KDN_BF16) {
+        for (int bb = 0; bb < 2; ++bb)
+          for (int th = 0; th < 2; ++th)
+            tma_store_4d(&m_o, sA + (bb * 2 + th) * 8192, 64 * bb, h, t0 + 64 * th, b);
+      } else {
+        for (int bx = 0; bx < 4; ++bx)
+          for (int th = 0; th < 2; ++th)
+            tma_store_4d(&m_o, sO + (bx * 2 + th) * 8192, 32 * bx, h, t0 + 64 * th, b);
+      }
+      bulk_commit();
+      bulk_wait_all();
+    } else {
+      atomicExch(a.status, (unsigned)KDN_ERR_TIMEOUT);
+      mbar_wait(bar_a, 0, kOutWait);  // copies in flight land before the CTA leaves
+      mbar_wait(bar_o, 0, kOutWait);
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) tmem_dealloc(tb, 256);
 }
 
 }  // namespace
@@ -295,7 +439,9 @@ int seg_count(const Args &a) {
 size_t seg_workspace_bytes(const Args &a, int P) {
   const size_t BH = (size_t)a.B * a.H, Pn = a.variant == 0 ? D : 1, NC = a.T / CM;
   auto r = [](size_t x) { return (x + 255) / 256 * 256; };
-  return r(BH * NC * Pn * 16) + r(BH * P * Pn * 4) * 2 + r(BH * P * D * D * 4) * 3;
+  const size_t ntok = (size_t)a.B * a.T * a.H * D;  // o_Phi (fp16); o_v (fp32) unless o is
+  return r(BH * NC * Pn * 16) + r(BH * P * Pn * 4) * 2 + r(BH * P * D * D * 4) * 3 +
+         r(ntok * 2) + (a.odt == KDN_BF16 ? r(ntok * 4) : 0);
 }
 
 kdn_status_t launch_seg_fwd(const Args &a, int P, char *ws, cudaStream_t s) {
@@ -308,7 +454,11 @@ kdn_status_t launch_seg_fwd(const Args &a, int P, char *ws, cudaStream_t s) {
   float *pbuf = reinterpret_cast<float *>(p); p += r(BH * P * Pn * 4);
   float *S0seg = reinterpret_cast<float *>(p); p += r(BH * P * nS * 4);
   float *Sv = reinterpret_cast<float *>(p); p += r(BH * P * nS * 4);
-  float *Sphi = reinterpret_cast<float *>(p);
+  float *Sphi = reinterpret_cast<float *>(p); p += r(BH * P * nS * 4);
+  const size_t ntok = (size_t)a.B * a.T * a.H * D;
+  void *ophi = p; p += r(ntok * 2);
+  // output of the run from S_in = 0: float32, in o itself unless o is bf16
+  float *ov = a.odt == KDN_BF16 ? reinterpret_cast<float *>(p) : static_cast<float *>(a.o);
 
   if (cudaMemsetAsync(S0seg, 0, BH * P * nS * 4, s) != cudaSuccess) return KDN_ERR_CUDA;
   if (a.S0 && cudaMemcpy2DAsync(S0seg, (size_t)P * seqS * 4, a.S0, seqS * 4, seqS * 4, a.B,
@@ -326,34 +476,36 @@ kdn_status_t launch_seg_fwd(const Args &a, int P, char *ws, cudaStream_t s) {
   k_seg_scan<<<(unsigned)BH, D * kScanGroups, 0, s>>>(a, comp, (int)(NC / P), pseg);
   if (cudaGetLastError() != cudaSuccess) return KDN_ERR_CUDA;
 
-  // the segments as B * P sequences of T / P tokens
+  // (1) the segments as B * P sequences of T / P tokens, in one pass that carries
+  // two memories: from S_in = 0 with v, and from S = I with v = 0 (the
+  // transition Phi), with both outputs per token
   Args sa = a;
   sa.B = a.B * P;
   sa.T = a.T / P;
   sa.NC = (sa.T + a.C - 1) / a.C;
   sa.Tp = sa.NC * a.C;
   sa.p0 = pseg;
-  sa.o = nullptr;
-  sa.pT = nullptr;
-  // (1) one pass carries two memories through every segment: from S_in = 0 (S_0
-  // for the first segment) with v, and from S = I with v = 0 (the transition Phi)
-  sa.S0 = S0seg;
+  sa.S0 = nullptr;  // every segment from S_in = 0; S_0 enters through the join
   sa.ST = Sv;
-  kdn_status_t st = launch_fused_fwd(sa, s, nullptr, nullptr, false, Sphi);
-  if (st != KDN_OK) return st;
-  // exact entry memories
-  k_seg_combine<<<dim3(D / 16, (unsigned)BH), 256, 0, s>>>(a, P, Sv, Sphi, S0seg);
-  if (cudaGetLastError() != cudaSuccess) return KDN_ERR_CUDA;
-  // (2) every segment from its exact entry state: o, and the final state
-  sa.S0 = S0seg;
-  sa.o = a.o;
-  sa.ST = a.ST ? Sphi : nullptr;
+  sa.o = ov;
+  sa.odt = KDN_F32;
   sa.pT = a.pT ? pbuf : nullptr;
-  st = launch_fused_fwd(sa, s);
+  kdn_status_t st = launch_fused_fwd(sa, s, nullptr, nullptr, true, Sphi, ophi);
   if (st != KDN_OK) return st;
-  if (a.ST && cudaMemcpy2DAsync(a.ST, seqS * 4, Sphi + (size_t)(P - 1) * seqS, (size_t)P * seqS * 4,
-                                seqS * 4, a.B, cudaMemcpyDeviceToDevice, s) != cudaSuccess)
+  // (2) exact entry memories (S_in(0) = S_0 is in place), and the final one
+  k_seg_combine<<<dim3(D / 16, (unsigned)BH), 256, 0, s>>>(a, P, Sv, Sphi, S0seg, a.ST);
+  if (cudaGetLastError() != cudaSuccess) return KDN_ERR_CUDA;
+  // (3) exact outputs o = o_v + S_in^T o_Phi
+  CUtensorMap m_ophi, m_ov, m_o;
+  if (!fused::make_map(&m_ophi, ophi, a, false, true) || !fused::make_map(&m_ov, ov, a, true) ||
+      !fused::make_map(&m_o, a.o, a, a.odt != KDN_BF16))
     return KDN_ERR_CUDA;
+  if (cudaFuncSetAttribute(k_seg_out, cudaFuncAttributeMaxDynamicSharedMemorySize, kOutSmem) !=
+      cudaSuccess)
+    return KDN_ERR_CUDA;
+  k_seg_out<<<dim3((unsigned)((a.T + kOutT - 1) / kOutT), (unsigned)a.H, (unsigned)a.B), kOutThreads, kOutSmem,
+              s>>>(m_ophi, m_ov, m_o, a, P, S0seg);
+  if (cudaGetLastError() != cudaSuccess) return KDN_ERR_CUDA;
   const size_t seqP = (size_t)a.H * Pn;
   if (a.pT && cudaMemcpy2DAsync(a.pT, seqP * 4, pbuf + (size_t)(P - 1) * seqP, (size_t)P * seqP * 4,
                                 seqP * 4, a.B, cudaMemcpyDeviceToDevice, s) != cudaSuccess)
