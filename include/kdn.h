@@ -122,7 +122,7 @@ const char *kdn_status_string(kdn_status_t status);
    sequence into P segments, joined exactly (uncertainty by a scan of per-chunk
    Moebius summaries, memory by the linearity of the chunk recurrence in
    (S_in, v)), and kdn_fwd_workspace_bytes includes its segment buffers
-   (3 x 64 KB per (batch, head, segment), 2 KB per (batch, head, chunk), and
+   (160 KB per (batch, head, segment), 2 KB per (batch, head, chunk), and
    2 bytes per element of o, 6 when out_dtype is KDN_BF16).
    A smaller workspace that still holds the single-pass layout (256 bytes)
    runs the single pass. */

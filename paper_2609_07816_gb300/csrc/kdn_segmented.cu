@@ -240,20 +240,29 @@ __global__ void __launch_bounds__(D * kScanGroups) k_seg_scan(const Args a, floa
 // S_in(P) is the final memory S_T (written when ST is given).  Columns of the
 // memory are independent: a CTA owns 16 of them for one (batch, head); thread
 // (row, half) holds 8 entries.
+// Every S_in(j) also goes to `img` as the fp16 B operand of the output pass
+// (32 KB per segment: two slabs of 64 value columns, rows = key channels,
+// 128-byte swizzle), so that pass fetches it with one bulk copy.
 __global__ void __launch_bounds__(256) k_seg_combine(const Args a, int P, const float *Sv,
-                                                     const float *Sphi, float *S0seg, float *ST) {
+                                                     const float *Sphi, float *ST,
+                                                     unsigned char *img) {
   __shared__ __align__(16) float sS[D][16];
   const int bh = blockIdx.y, b = bh / a.H, h = bh % a.H;
   const int tid = threadIdx.x, row = tid >> 1, half = tid & 1;
   const int col = blockIdx.x * 16 + half * 8;
   auto ent = [&](int j) { return ((size_t)(b * P + j) * a.H + h) * D * D; };
-  float acc[8];
-  {
-    const float4 *src = reinterpret_cast<const float4 *>(S0seg + ent(0) + (size_t)row * D + col);
+  auto put_img = [&](int j, const float *x) {
+    unsigned char *dst = img + ((size_t)(b * P + j) * a.H + h) * 32768;
+    fused::sm16(dst, (col >> 6) * 16384 + fused::chunk_off(row, (col & 63) >> 3)) = fused::pack_h8(x);
+  };
+  float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+  if (a.S0) {  // S_in(0) = S_0
+    const float4 *src = reinterpret_cast<const float4 *>(a.S0 + ((size_t)bh * D + row) * D + col);
     const float4 x0 = src[0], x1 = src[1];
     acc[0] = x0.x; acc[1] = x0.y; acc[2] = x0.z; acc[3] = x0.w;
     acc[4] = x1.x; acc[5] = x1.y; acc[6] = x1.z; acc[7] = x1.w;
   }
+  put_img(0, acc);
   for (int j = 0; j < P; ++j) {  // acc = S_in(j)
     if (j == P - 1 && !ST) break;
 #pragma unroll
@@ -279,10 +288,13 @@ __global__ void __launch_bounds__(256) k_seg_combine(const Args a, int P, const 
       }
     }
     __syncthreads();
-    float *base = j + 1 < P ? S0seg + ent(j + 1) : ST + (size_t)bh * D * D;
-    float4 *dst = reinterpret_cast<float4 *>(base + (size_t)row * D + col);
-    dst[0] = make_float4(acc[0], acc[1], acc[2], acc[3]);
-    dst[1] = make_float4(acc[4], acc[5], acc[6], acc[7]);
+    if (j + 1 < P) {
+      put_img(j + 1, acc);
+    } else {
+      float4 *dst = reinterpret_cast<float4 *>(ST + (size_t)bh * D * D + (size_t)row * D + col);
+      dst[0] = make_float4(acc[0], acc[1], acc[2], acc[3]);
+      dst[1] = make_float4(acc[4], acc[5], acc[6], acc[7]);
+    }
   }
 }
 
@@ -290,30 +302,35 @@ __global__ void __launch_bounds__(256) k_seg_combine(const Args a, int P, const 
 // output of the run from S_in = 0 with v, o_Phi,t = tau Phi_t^T q_t that of the
 // transition run, and S_in(j) the entry memory of the token's segment j (the
 // recurrence is linear in S_in).  One CTA per (128-token tile, head, batch):
-// TMA brings the o_Phi tile (fp16, K-major A) and the o_v tile (fp32); S_in(j)
-// is converted to the fp16 MN-major B operand (the layout of MMA-S1's S_in in
-// the fused forward); eight tcgen05 MMAs (M = N = 128, K = 16 each) form
-// o_Phi S_in in TMEM, the epilogue adds o_v and TMA stores the tile.  Segments
-// are whole 64-token chunks, so a tile whose second half starts a new segment
-// also forms o_Phi S_in(j + 1) (a second operand and accumulator) for that half.
+// TMA brings the o_Phi tile (fp16, K-major A) and a bulk copy the fp16 image of
+// S_in(j) (MN-major B, written by k_seg_combine); eight tcgen05 MMAs
+// (M = N = 128, K = 16 each) form o_Phi S_in in TMEM.  With float32 o (which
+// then already holds o_v) the epilogue stages the product and a TMA reduce-add
+// adds it to o; with bf16 o it loads o_v from the workspace, adds, rounds and
+// stores.  Segments are whole 64-token chunks, so a tile whose second half
+// starts a new segment also forms o_Phi S_in(j + 1) for that half.  96 KB of
+// shared memory and 256 TMEM columns: two CTAs per SM.
 constexpr int kOutT = 128, kOutThreads = 128;
-constexpr int kOutSmem = 32768 + 2 * 32768 + 65536 + 64 + 1024;
+constexpr int kOutSmem = 32768 + 65536 + 64 + 1024;
 constexpr uint32_t kOutWait = 1u << 25;
 
-__global__ void __launch_bounds__(kOutThreads, 1)
+__global__ void __launch_bounds__(kOutThreads, 2)
     k_seg_out(const __grid_constant__ CUtensorMap m_ophi, const __grid_constant__ CUtensorMap m_ov,
-              const __grid_constant__ CUtensorMap m_o, const Args a, int P, const float *S0seg) {
+              const __grid_constant__ CUtensorMap m_o, const Args a, int P,
+              const unsigned char *img) {
   using namespace sm103;
   using namespace fused;
   extern __shared__ unsigned char smraw[];
   unsigned char *sm =
       reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(smraw) + 1023) & ~uintptr_t(1023));
-  unsigned char *sA = sm, *sB = sm + 32768, *sO = sm + 98304;
-  uint64_t *bars = reinterpret_cast<uint64_t *>(sm + 163840);
+  unsigned char *sA = sm, *sB = sm + 32768;  // after the MMAs: [0, 64K) float32 staging,
+                                             // [64K, 96K) bf16 staging
+  uint64_t *bars = reinterpret_cast<uint64_t *>(sm + 98304);
   uint64_t *bar_a = bars, *bar_o = bars + 1, *bar_m = bars + 2;
   uint32_t *s_tbase = reinterpret_cast<uint32_t *>(bars + 4);
   const int tid = threadIdx.x, warp = tid >> 5;
   const int t0 = blockIdx.x * kOutT, h = blockIdx.y, b = blockIdx.z;
+  const bool obf = a.odt == KDN_BF16;
   // segments of the two 64-token halves (a last tile may hold only the first;
   // the TMA fills and clips the tokens past T)
   const int seg = t0 / (a.T / P), seg2 = t0 + 64 < a.T ? (t0 + 64) / (a.T / P) : seg;
@@ -323,38 +340,22 @@ __global__ void __launch_bounds__(kOutThreads, 1)
     mbar_init(bar_o, 1);
     mbar_init(bar_m, 1);
     fence_mbar_init();
-    mbar_expect_tx(bar_a, 32768);
+    mbar_expect_tx(bar_a, 32768u * (two ? 3 : 2));
     for (int sl = 0; sl < 2; ++sl)
       for (int th = 0; th < 2; ++th)  // slab sl: rows 0..63 (th 0), 64..127 (th 1)
         tma_load_4d(sA + sl * 16384 + th * 8192, &m_ophi, bar_a, 64 * sl, h, t0 + 64 * th, b);
-    mbar_expect_tx(bar_o, 65536);
-    for (int bx = 0; bx < 4; ++bx)
-      for (int th = 0; th < 2; ++th)
-        tma_load_4d(sO + (bx * 2 + th) * 8192, &m_ov, bar_o, 32 * bx, h, t0 + 64 * th, b);
+    for (int u = 0; u < (two ? 2 : 1); ++u)
+      bulk_g2s(sB + u * 32768, img + ((size_t)(b * P + seg + u) * a.H + h) * 32768, 32768, bar_a);
   }
   if (warp == 0) {
     tmem_alloc(s_tbase, 256);
     tmem_relinquish();
   }
-  // S_in(seg) row i -> fp16, MN-major: 64 value columns per 128-byte row, two slabs
-  for (int u = 0; u < (two ? 2 : 1); ++u) {
-    const int i = tid;
-    const float4 *src = reinterpret_cast<const float4 *>(
-        S0seg + (((size_t)(b * P + seg + u) * a.H + h) * D + i) * D);
-    unsigned char *dst = sB + u * 32768;
-#pragma unroll 4
-    for (int c8 = 0; c8 < 16; ++c8) {
-      const float4 x0 = src[2 * c8], x1 = src[2 * c8 + 1];
-      const float v[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
-      sm16(dst, (c8 >> 3) * 16384 + chunk_off(i, c8 & 7)) = pack_h8(v);
-    }
-  }
-  fence_proxy_async();
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tb = *s_tbase;
-  bool ok = true;
+  bool ok = true, o_issued = false;
   if (tid == 0) {
     ok = mbar_wait(bar_a, 0, kOutWait);
     if (ok) {
@@ -364,35 +365,44 @@ __global__ void __launch_bounds__(kOutThreads, 1)
           umma_bf16(tb + 128 * u, sw128_desc(A + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024),
                     sw128_desc(B + u * 32768 + kk * 2048, 16384, 1024), id, kk > 0);
       umma_commit(bar_m);
-      ok = mbar_wait(bar_m, 0, kOutWait) && mbar_wait(bar_o, 0, kOutWait);
+      ok = mbar_wait(bar_m, 0, kOutWait);
+      if (ok && obf) {  // o_v (float32, workspace) over the operands the MMAs have read
+        mbar_expect_tx(bar_o, 65536);
+        o_issued = true;
+        for (int bx = 0; bx < 4; ++bx)
+          for (int th = 0; th < 2; ++th)
+            tma_load_4d(sm + (bx * 2 + th) * 8192, &m_ov, bar_o, 32 * bx, h, t0 + 64 * th, b);
+        ok = mbar_wait(bar_o, 0, kOutWait);
+      }
     }
   }
   ok = __syncthreads_and(ok);
   if (ok) {
     tc_fence_after();
-    // token t = tid: TMEM lane t; o_v row t % 64 of box (column group, t / 64)
+    // token t = tid: TMEM lane t; float32 row t % 64 of box (column group, t / 64)
     const int t = tid, r = t & 63, th = t >> 6;
-    const bool obf = a.odt == KDN_BF16;
     const uint32_t acc = tb + ((two && th) ? 128u : 0u);  // the second half's segment
     for (int j0 = 0; j0 < D; j0 += 16) {
       float v[16];
       tmem_ld16(acc + ((uint32_t)(32 * warp) << 16) + j0, v);
       const int bx = j0 >> 5, cc = (j0 & 31) >> 2;
-      unsigned char *box = sO + (bx * 2 + th) * 8192;
+      unsigned char *box = sm + (bx * 2 + th) * 8192;
 #pragma unroll
       for (int m = 0; m < 4; ++m) {
         uint4 &u = sm16(box, chunk_off(r, cc + m));
-        v[4 * m] += __uint_as_float(u.x);
-        v[4 * m + 1] += __uint_as_float(u.y);
-        v[4 * m + 2] += __uint_as_float(u.z);
-        v[4 * m + 3] += __uint_as_float(u.w);
-        if (!obf)
+        if (obf) {
+          v[4 * m] += __uint_as_float(u.x);
+          v[4 * m + 1] += __uint_as_float(u.y);
+          v[4 * m + 2] += __uint_as_float(u.z);
+          v[4 * m + 3] += __uint_as_float(u.w);
+        } else {
           u = make_uint4(__float_as_uint(v[4 * m]), __float_as_uint(v[4 * m + 1]),
                          __float_as_uint(v[4 * m + 2]), __float_as_uint(v[4 * m + 3]));
+        }
       }
-      if (obf) {  // bf16 o: boxes of 64 columns over the o_Phi tile (read by the MMAs)
+      if (obf) {  // boxes of 64 bf16 columns
         const int bb = j0 >> 6, c2 = (j0 & 63) >> 3;
-        unsigned char *ob = sA + (bb * 2 + th) * 8192;
+        unsigned char *ob = sm + 65536 + (bb * 2 + th) * 8192;
         sm16(ob, chunk_off(r, c2)) = pack_bf8(v);
         sm16(ob, chunk_off(r, c2 + 1)) = pack_bf8(v + 8);
       }
@@ -402,21 +412,21 @@ __global__ void __launch_bounds__(kOutThreads, 1)
   __syncthreads();
   if (tid == 0) {
     if (ok) {
-      if (a.odt == KDN_BF16) {
+      if (obf) {
         for (int bb = 0; bb < 2; ++bb)
           for (int th = 0; th < 2; ++th)
-            tma_store_4d(&m_o, sA + (bb * 2 + th) * 8192, 64 * bb, h, t0 + 64 * th, b);
-      } else {
+            tma_store_4d(&m_o, sm + 65536 + (bb * 2 + th) * 8192, 64 * bb, h, t0 + 64 * th, b);
+      } else {  // o += o_Phi S_in
         for (int bx = 0; bx < 4; ++bx)
           for (int th = 0; th < 2; ++th)
-            tma_store_4d(&m_o, sO + (bx * 2 + th) * 8192, 32 * bx, h, t0 + 64 * th, b);
+            tma_add_4d(&m_o, sm + (bx * 2 + th) * 8192, 32 * bx, h, t0 + 64 * th, b);
       }
       bulk_commit();
       bulk_wait_all();
     } else {
       atomicExch(a.status, (unsigned)KDN_ERR_TIMEOUT);
       mbar_wait(bar_a, 0, kOutWait);  // copies in flight land before the CTA leaves
-      mbar_wait(bar_o, 0, kOutWait);
+      if (o_issued) mbar_wait(bar_o, 0, kOutWait);
     }
   }
   tc_fence_before();
@@ -440,30 +450,26 @@ size_t seg_workspace_bytes(const Args &a, int P) {
   const size_t BH = (size_t)a.B * a.H, Pn = a.variant == 0 ? D : 1, NC = a.T / CM;
   auto r = [](size_t x) { return (x + 255) / 256 * 256; };
   const size_t ntok = (size_t)a.B * a.T * a.H * D;  // o_Phi (fp16); o_v (fp32) unless o is
-  return r(BH * NC * Pn * 16) + r(BH * P * Pn * 4) * 2 + r(BH * P * D * D * 4) * 3 +
-         r(ntok * 2) + (a.odt == KDN_BF16 ? r(ntok * 4) : 0);
+  return r(BH * NC * Pn * 16) + r(BH * P * Pn * 4) * 2 + r(BH * P * D * D * 4) * 2 +
+         r(BH * P * 32768) + r(ntok * 2) + (a.odt == KDN_BF16 ? r(ntok * 4) : 0);
 }
 
 kdn_status_t launch_seg_fwd(const Args &a, int P, char *ws, cudaStream_t s) {
   const size_t BH = (size_t)a.B * a.H, Pn = a.variant == 0 ? D : 1, NC = a.T / CM;
-  const size_t nS = (size_t)D * D, seqS = (size_t)a.H * nS;
+  const size_t nS = (size_t)D * D;
   auto r = [](size_t x) { return (x + 255) / 256 * 256; };
   char *p = ws;
   float4 *comp = reinterpret_cast<float4 *>(p); p += r(BH * NC * Pn * 16);
   float *pseg = reinterpret_cast<float *>(p); p += r(BH * P * Pn * 4);
   float *pbuf = reinterpret_cast<float *>(p); p += r(BH * P * Pn * 4);
-  float *S0seg = reinterpret_cast<float *>(p); p += r(BH * P * nS * 4);
   float *Sv = reinterpret_cast<float *>(p); p += r(BH * P * nS * 4);
   float *Sphi = reinterpret_cast<float *>(p); p += r(BH * P * nS * 4);
+  unsigned char *img = reinterpret_cast<unsigned char *>(p); p += r(BH * P * 32768);
   const size_t ntok = (size_t)a.B * a.T * a.H * D;
   void *ophi = p; p += r(ntok * 2);
   // output of the run from S_in = 0: float32, in o itself unless o is bf16
   float *ov = a.odt == KDN_BF16 ? reinterpret_cast<float *>(p) : static_cast<float *>(a.o);
 
-  if (cudaMemsetAsync(S0seg, 0, BH * P * nS * 4, s) != cudaSuccess) return KDN_ERR_CUDA;
-  if (a.S0 && cudaMemcpy2DAsync(S0seg, (size_t)P * seqS * 4, a.S0, seqS * 4, seqS * 4, a.B,
-                                cudaMemcpyDeviceToDevice, s) != cudaSuccess)
-    return KDN_ERR_CUDA;
 
   // uncertainty entering every segment
   const dim3 gc((unsigned)NC, (unsigned)BH);
@@ -492,8 +498,8 @@ kdn_status_t launch_seg_fwd(const Args &a, int P, char *ws, cudaStream_t s) {
   sa.pT = a.pT ? pbuf : nullptr;
   kdn_status_t st = launch_fused_fwd(sa, s, nullptr, nullptr, true, Sphi, ophi);
   if (st != KDN_OK) return st;
-  // (2) exact entry memories (S_in(0) = S_0 is in place), and the final one
-  k_seg_combine<<<dim3(D / 16, (unsigned)BH), 256, 0, s>>>(a, P, Sv, Sphi, S0seg, a.ST);
+  // (2) exact entry memories (as fp16 operand images) from S_in(0) = S_0, and the final one
+  k_seg_combine<<<dim3(D / 16, (unsigned)BH), 256, 0, s>>>(a, P, Sv, Sphi, a.ST, img);
   if (cudaGetLastError() != cudaSuccess) return KDN_ERR_CUDA;
   // (3) exact outputs o = o_v + S_in^T o_Phi
   CUtensorMap m_ophi, m_ov, m_o;
@@ -504,7 +510,7 @@ kdn_status_t launch_seg_fwd(const Args &a, int P, char *ws, cudaStream_t s) {
       cudaSuccess)
     return KDN_ERR_CUDA;
   k_seg_out<<<dim3((unsigned)((a.T + kOutT - 1) / kOutT), (unsigned)a.H, (unsigned)a.B), kOutThreads, kOutSmem,
-              s>>>(m_ophi, m_ov, m_o, a, P, S0seg);
+              s>>>(m_ophi, m_ov, m_o, a, P, img);
   if (cudaGetLastError() != cudaSuccess) return KDN_ERR_CUDA;
   const size_t seqP = (size_t)a.H * Pn;
   if (a.pT && cudaMemcpy2DAsync(a.pT, seqP * 4, pbuf + (size_t)(P - 1) * seqP, (size_t)P * seqP * 4,

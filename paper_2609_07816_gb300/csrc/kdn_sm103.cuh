@@ -67,6 +67,16 @@ __device__ __forceinline__ void tma_store_4d(const CUtensorMap *map, const void 
       "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(smem_u32(src))
       : "memory");
 }
+// Bulk tensor reduction shared -> global: global += shared elementwise, in the
+// element type of the map; rows past the tensor's extent are not touched.
+__device__ __forceinline__ void tma_add_4d(const CUtensorMap *map, const void *src, int c0, int c1,
+                                           int c2, int c3) {
+  asm volatile(
+      "cp.reduce.async.bulk.tensor.4d.global.shared::cta.add.tile.bulk_group"
+      " [%0, {%1, %2, %3, %4}], [%5];" ::"l"(reinterpret_cast<uint64_t>(map)),
+      "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(smem_u32(src))
+      : "memory");
+}
 // Untiled bulk copies (16-byte aligned addresses, size a multiple of 16).
 __device__ __forceinline__ void bulk_g2s(void *dst, const void *src, uint32_t bytes, uint64_t *bar) {
   asm volatile(

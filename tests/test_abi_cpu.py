@@ -182,9 +182,11 @@ def _seg_bytes(B, T, H, P, variant):
     r = lambda x: (x + 255) // 256 * 256
     Pn = 128 if variant == 0 else 1
     BH, NC = B * H, T // 64
-    # + the fp16 output of the transition pass (o is float32 here, so it holds o_v)
-    return (r(BH * NC * Pn * 16) + 2 * r(BH * P * Pn * 4) + 3 * r(BH * P * 128 * 128 * 4)
-            + r(B * T * H * 128 * 2))
+    # summaries, 2 uncertainty buffers, the exit memories Sv and Phi, the fp16
+    # images of the entry memories and the fp16 output of the transition pass
+    # (o is float32 here, so it holds o_v)
+    return (r(BH * NC * Pn * 16) + 2 * r(BH * P * Pn * 4) + 2 * r(BH * P * 128 * 128 * 4)
+            + r(BH * P * 32768) + r(B * T * H * 128 * 2))
 
 
 @pytest.mark.parametrize("B,T,H,P", [

@@ -79,6 +79,7 @@ SEG_CASES = [
     ("iso", False, 1, 2048, 2, 0.02, (0.5, 2.0), 4, False),
     ("iso", False, 1, 2048, 2, 0.02, (0.5, 2.0), 4, True),
     ("iso", True, 2, 2560, 1, 0.1, (0.1, 2.0), 5, True),
+    ("iso", False, 1, 2880, 2, 0.05, (0.5, 2.0), 5, True),    # 45 chunks: half a last tile
 ]
 
 
@@ -86,8 +87,9 @@ SEG_CASES = [
                          ids=lambda c: "-".join(map(str, c[:5])) + ("-weak" if c[8] else ""))
 def test_sequence_parallel_forward_parity(kdn, case):
     """Few long sequences: the forward cut into segments (gain summaries and
-    scan, a run from S = 0, a run from S = I with v = 0, the state join, the
-    final run) matches the token-by-token oracle on o, S_T and p_T."""
+    scan, one run carrying the memory from S = 0 and the transition from S = I
+    with v = 0, the state join, the outputs o_v + S_in^T o_Phi) matches the
+    token-by-token oracle on o, S_T and p_T."""
     variant, pc, B, T, H, s0, p0r, nseg, weak = case
     ins = make_inputs(variant, B, T, H, 128, 128, dtype="bf16", seed=T + B, s0_std=s0,
                       p0_range=p0r, per_channel_decay=pc)
@@ -106,6 +108,26 @@ def test_sequence_parallel_forward_parity(kdn, case):
     for j in range(1, nseg):
         t = j * step
         check(f"o[t={t}]", o[:, t:t + 2], ref["o"][:, t:t + 2], "bf16")
+
+
+@pytest.mark.parametrize("variant,pc", [("diag", True), ("iso", False)])
+def test_sequence_parallel_forward_bf16_outputs(kdn, variant, pc):
+    """bf16 o from the segmented forward (o_v is then held in float32 in the
+    workspace and rounded once by the output pass), with 9-chunk segments whose
+    128-token output tiles straddle segment boundaries."""
+    B, T, H = 1, 2304, 2
+    ins = _weak_decay(make_inputs(variant, B, T, H, 128, 128, dtype="bf16", seed=71,
+                                  s0_std=0.05, p0_range=(0.5, 2.0), per_channel_decay=pc), 72)
+    d = kdn.make_desc(B, T, H, 128, 128, kdn.KDN_BF16, decay_per_channel=int(pc),
+                      out_dtype=kdn.KDN_BF16)
+    assert kdn.kdn_kernel_launches(d, 0 if variant == "diag" else 1, 0) == 5
+    ref = _oracle_fwd(variant, ins)
+    o, ST, pT = _gpu_fwd(kdn, variant, to_dev(ins), out_dtype=torch.bfloat16)
+    torch.cuda.synchronize()
+    assert o.dtype == torch.bfloat16
+    check_stored_bf16("o", o, ref["o"])
+    check("ST", ST, ref["ST"], "bf16")
+    check("pT", pT, ref["pT"], "bf16")
 
 
 def test_sequence_parallel_forward_without_state_outputs(kdn):
