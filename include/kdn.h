@@ -224,6 +224,24 @@ kdn_status_t kdn_iso_bwd_saved(const kdn_desc_t *desc, const void *q,
                                float *dp0, float *dmu, void *workspace,
                                size_t workspace_bytes, void *stream);
 
+/* Effective write strength of every token, beta_eff,t = k_t^T kappa_t (the
+   coefficient of the residual identity of eq. appendix-effective-write:
+   v_t - S_t^T k_t = (1 - beta_eff,t)(v_t - Shat_t^T k_t); 0 <= beta_eff < 1),
+   read from the per-token gain scalars a kdn_*_fwd_save call stored in `saved`
+   (same descriptor and variant).  Diagonal: 1 - r_t / s_t with
+   s_t = r_t + sum_i phat_i k_i^2; Isotropic: beta_t |k_t|^2.
+   r: the r input that call was given (logits when desc->gates says so).
+   beta_eff: float32 [B,T,H].  One small kernel, asynchronous on `stream`.
+   Returns KDN_ERR_UNSUPPORTED for descriptors kdn_*_fwd_save does not serve,
+   KDN_ERR_INVALID_ARG for a null or misaligned pointer, KDN_ERR_WORKSPACE when
+   saved_bytes < kdn_saved_bytes(desc, variant). */
+kdn_status_t kdn_diag_beta_eff(const kdn_desc_t *desc, const void *saved,
+                               size_t saved_bytes, const void *r, float *beta_eff,
+                               void *stream);
+kdn_status_t kdn_iso_beta_eff(const kdn_desc_t *desc, const void *saved,
+                              size_t saved_bytes, const void *r, float *beta_eff,
+                              void *stream);
+
 /* One decode token for all B*H heads (the update of Prop. 3), in place:
    S [B,H,dk,dv] and p [B,H,dk] are read and overwritten; o [B,H,dv] is
    written.  Per-step inputs drop the T axis: q, k [B,H,dk], v [B,H,dv],
@@ -266,7 +284,7 @@ kdn_status_t kdn_diag_fwd_noalloc(const kdn_desc_t *desc, const void *q,
 
 /* Number of CUDA kernels one call of an entry point launches for this
    descriptor when T > 0 (op 0 = kdn_*_fwd, 1 = kdn_*_bwd, 2 = kdn_*_decode_step,
-   3 = kdn_*_fwd_save, 4 = kdn_*_bwd_saved; variant 0 = diagonal,
+   3 = kdn_*_fwd_save, 4 = kdn_*_bwd_saved, 5 = kdn_*_beta_eff; variant 0 = diagonal,
    1 = isotropic).  -1 for an invalid descriptor or op, or an op the descriptor
    does not serve.
    Calls with T = 0 launch at most one small fill kernel. */

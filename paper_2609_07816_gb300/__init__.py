@@ -72,6 +72,8 @@ _SIG = {
                                                                   ctypes.c_size_t, _P], ctypes.c_int),
     "kdn_iso_bwd_saved": ([ctypes.POINTER(kdn_desc_t)] + [_P] * 7 + [ctypes.c_size_t] + [_P] * 13
                           + [ctypes.c_size_t, _P], ctypes.c_int),
+    "kdn_diag_beta_eff": ([ctypes.POINTER(kdn_desc_t), _P, ctypes.c_size_t, _P, _P, _P], ctypes.c_int),
+    "kdn_iso_beta_eff": ([ctypes.POINTER(kdn_desc_t), _P, ctypes.c_size_t, _P, _P, _P], ctypes.c_int),
     "kdn_kernel_launches": ([ctypes.POINTER(kdn_desc_t), ctypes.c_int, ctypes.c_int], ctypes.c_int),
     "kdn_get_device_status": ([_P, _P], ctypes.c_int),
 }
@@ -349,6 +351,33 @@ def kdn_iso_bwd_saved(q, k, v, g, omega, r, saved, dO, dST=None, dpT=None, *, mu
                       scale=scale, grads=grads, want_state_grads=want_state_grads,
                       workspace=workspace, stream=stream, out_dtype=out_dtype,
         gates=gates, r_min=r_min)
+
+
+def _beta_eff(name, variant, k, v, g, r, saved, *, out, stream, gates, r_min):
+    desc = _desc_from(variant, k, v, g, chunk=0, mu=None, scale=None, out_dtype=torch.float32,
+                      gates=gates, r_min=r_min)
+    B, T, H, _ = k.shape
+    if out is None:
+        out = torch.empty(B, T, H, dtype=torch.float32, device=k.device)
+    st = getattr(lib(), name)(ctypes.byref(desc), _ptr(saved), ctypes.c_size_t(saved.numel()),
+                              _ptr(r), _ptr(out), _stream(stream))
+    _check(st, name)
+    return out
+
+
+def kdn_diag_beta_eff(k, v, g, r, saved, *, out=None, stream=None, gates=KDN_GATES_POST,
+                      r_min=R_MIN_DEFAULT):
+    """beta_eff = k_t^T kappa_t [B,T,H] (float32) from the context kdn_diag_fwd_save kept;
+    k, v, g fix the descriptor, r is the forward's r."""
+    return _beta_eff("kdn_diag_beta_eff", 0, k, v, g, r, saved, out=out, stream=stream,
+                     gates=gates, r_min=r_min)
+
+
+def kdn_iso_beta_eff(k, v, g, r, saved, *, out=None, stream=None, gates=KDN_GATES_POST,
+                     r_min=R_MIN_DEFAULT):
+    """beta_eff = beta_t |k_t|^2 [B,T,H] (float32) from the context kdn_iso_fwd_save kept."""
+    return _beta_eff("kdn_iso_beta_eff", 1, k, v, g, r, saved, out=out, stream=stream,
+                     gates=gates, r_min=r_min)
 
 
 def _decode(name, variant, q, k, v, g, omega, r, S, p, *, mu, scale, o, stream, out_dtype,

@@ -253,6 +253,19 @@ kdn_status_t decode_entry(int variant, const kdn_desc_t *d, const void *q, const
   return launch_decode(a, S, p, static_cast<cudaStream_t>(stream));
 }
 
+kdn_status_t beta_eff_entry(int variant, const kdn_desc_t *d, const void *saved,
+                            size_t saved_bytes, const void *r, float *beta_eff, void *stream) {
+  Args a;
+  kdn_status_t st = fill_sizes(d, variant, false, &a);
+  if (st != KDN_OK) return st;
+  if ((size_t)a.B * a.H * a.T == 0) return KDN_OK;
+  if (!use_fused_bwd(a)) return KDN_ERR_UNSUPPORTED;
+  if (!ptrs_ok({saved, r, beta_eff}, {})) return KDN_ERR_INVALID_ARG;
+  if (saved_bytes < fused_saved_bytes(a)) return KDN_ERR_WORKSPACE;
+  a.r = r;
+  return launch_beta_eff(a, saved, beta_eff, static_cast<cudaStream_t>(stream));
+}
+
 }  // namespace
 
 size_t fwd_min_workspace_bytes(const kdn_desc_t *desc, int variant) {
@@ -436,9 +449,20 @@ int kdn_kernel_launches(const kdn_desc_t *desc, int variant, int op) {
     case 1: return (a.T > 0 && use_fused_bwd(a)) ? 2 : chunked_bwd_launches(a);
     case 2: return 1;
     case 3:
-    case 4: return fused_saved_bytes(a) > 0 ? 1 : -1;
+    case 4:
+    case 5: return fused_saved_bytes(a) > 0 ? 1 : -1;
   }
   return -1;
+}
+
+kdn_status_t kdn_diag_beta_eff(const kdn_desc_t *desc, const void *saved, size_t saved_bytes,
+                               const void *r, float *beta_eff, void *stream) {
+  return beta_eff_entry(0, desc, saved, saved_bytes, r, beta_eff, stream);
+}
+
+kdn_status_t kdn_iso_beta_eff(const kdn_desc_t *desc, const void *saved, size_t saved_bytes,
+                              const void *r, float *beta_eff, void *stream) {
+  return beta_eff_entry(1, desc, saved, saved_bytes, r, beta_eff, stream);
 }
 
 kdn_status_t kdn_get_device_status(void *workspace, void *stream) {

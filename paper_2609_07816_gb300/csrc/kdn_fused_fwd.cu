@@ -901,10 +901,37 @@ __global__ void __launch_bounds__(FT, 1)
   if (warp == 0) tmem_dealloc(tb, 512);
 }
 
+// Effective write strength beta_eff,t = k_t^T kappa_t of every token (eq.
+// appendix-effective-write: v - S_t^T k = (1 - beta_eff)(v - Shat_t^T k)), from
+// the per-token gain scalars a training forward saved: Diagonal KDN
+// kappa = phat k / s_t, so k^T kappa = (s_t - r_t) / s_t = 1 - r_t / s_t;
+// Isotropic KDN kappa = beta_t k, so k^T kappa = beta_t |k_t|^2.  One thread per
+// token, one CTA per (chunk, batch * head).
+__global__ void __launch_bounds__(CM) k_beta_eff(const Args a, const unsigned char *saved, float *out) {
+  const int c = blockIdx.x, bh = blockIdx.y, t = threadIdx.x;
+  const int b = bh / a.H, h = bh % a.H, NC = (a.T + CM - 1) / CM, tt = c * CM + t;
+  if (tt >= a.T) return;
+  const float *tok = reinterpret_cast<const float *>(saved + ((size_t)bh * NC + c) * kCtxBytes + kCtxTok);
+  const size_t th = tok_index(a, b, tt, h);
+  if (a.variant == 0) {
+    const float rr = gate_r(a.gates, a.rmin, ld<__nv_bfloat16>(a.r, th));
+    out[th] = 1.f - rr / tok[t];
+  } else {
+    out[th] = tok[t] * tok[CM + t];
+  }
+}
+
 // ---------------------------------------------------------------------------
 // host side
 
 }  // namespace
+
+kdn_status_t launch_beta_eff(const Args &a, const void *saved, float *out, cudaStream_t s) {
+  const int NC = (a.T + CM - 1) / CM;
+  k_beta_eff<<<dim3((unsigned)NC, (unsigned)(a.B * a.H)), CM, 0, s>>>(
+      a, static_cast<const unsigned char *>(saved), out);
+  return cudaGetLastError() == cudaSuccess ? KDN_OK : KDN_ERR_CUDA;
+}
 
 bool fused_fwd_supported(const Args &a) {
   return a.dtype == KDN_BF16 && a.dk == D && a.dv == D && a.T > 0;

@@ -147,6 +147,9 @@ bool fused_fwd_supported(const Args &a);
 kdn_status_t launch_fused_fwd(const Args &a, cudaStream_t s, unsigned char *save_S = nullptr,
                               float *save_p = nullptr, bool write_o = true, float *phi_T = nullptr,
                               void *o_phi = nullptr);
+// beta_eff [B,T,H] (float32) from the per-token gain scalars of a context saved by
+// the fused training forward (one launch).
+kdn_status_t launch_beta_eff(const Args &a, const void *saved, float *out, cudaStream_t s);
 // Fused tcgen05 backward (Diagonal KDN, bf16, dk = dv = 128, 64-token chunks):
 // one reverse sweep per (batch, head) from the saved context in a.fSin / a.fpin.
 // launch_fused_bwd first runs the context-saving forward (without o).

@@ -245,3 +245,26 @@ def test_training_pair_validation(kdn):
         assert fn(d, saved_bytes=n - 1) == kdn.KDN_ERR_WORKSPACE
         assert fn(d, saved=MIS) in (kdn.KDN_ERR_INVALID_ARG, kdn.KDN_ERR_WORKSPACE)
         assert fn(d, saved=None) == kdn.KDN_ERR_INVALID_ARG
+
+
+def test_beta_eff_validation(kdn):
+    """kdn_*_beta_eff reads a saved training context: served for the same
+    descriptors as the training pair, pointers and the saved size are checked
+    before anything runs, T = 0 is a no-op (no GPU needed for any of this)."""
+    L = kdn.lib()
+    B, T, H = 2, 130, 3
+    d = kdn.make_desc(B, T, H, 128, 128, kdn.KDN_BF16)
+    n = kdn.saved_bytes(d)
+    assert kdn.kdn_kernel_launches(d, 0, 5) == 1 and kdn.kdn_kernel_launches(d, 1, 5) == 1
+    assert kdn.kdn_kernel_launches(kdn.make_desc(B, T, H, 128, 128, kdn.KDN_F32), 0, 5) == -1
+    for fn in (L.kdn_diag_beta_eff, L.kdn_iso_beta_eff):
+        def call(desc, saved=FAKE, saved_bytes=1 << 40, r=FAKE, out=FAKE):
+            return fn(ctypes.byref(desc), saved, saved_bytes, r, out, None)
+        assert call(kdn.make_desc(B, T, H, 64, 128, kdn.KDN_BF16)) == kdn.KDN_ERR_UNSUPPORTED
+        assert call(kdn.make_desc(B, T, H, 128, 128, kdn.KDN_F32)) == kdn.KDN_ERR_UNSUPPORTED
+        assert call(d, saved=None) == kdn.KDN_ERR_INVALID_ARG
+        assert call(d, r=None) == kdn.KDN_ERR_INVALID_ARG
+        assert call(d, out=MIS) == kdn.KDN_ERR_INVALID_ARG
+        assert call(d, saved_bytes=n - 1) == kdn.KDN_ERR_WORKSPACE
+        assert call(kdn.make_desc(B, 0, H, 128, 128, kdn.KDN_BF16), saved=None) == kdn.KDN_OK
+        assert call(d, saved=MIS) == kdn.KDN_ERR_INVALID_ARG

@@ -489,3 +489,35 @@ def test_fused_strong_decay_inside_range(kdn, variant, pc):
         check(n, {"o": o, "ST": ST, "pT": pT}[n], ref[n], "bf16")
     for n in ("dq", "dk", "dv", "dg", "domega", "dr", "dS0", "dp0"):
         check(n, grads[n], gref[n], "bf16")
+
+
+@pytest.mark.parametrize("variant,pc,gates", [("diag", True, False), ("iso", False, False),
+                                              ("iso", True, False), ("diag", True, True)])
+def test_beta_eff_from_saved_context(kdn, variant, pc, gates):
+    """kdn_*_beta_eff against k_t^T kappa_t of the oracle's gains (its trace), on a
+    ragged T, every variant and decay mode, and logit gates; the values lie in
+    [0, 1) (the invariant of the effective write)."""
+    B, T, H = 2, 150, 2
+    ins = make_inputs(variant, B, T, H, 128, 128, dtype="bf16", seed=83, s0_std=0.05,
+                      p0_range=(0.5, 2.0), per_channel_decay=pc)
+    kw, okw = {}, {}
+    if gates:
+        rng = np.random.default_rng(89)
+        for n, m in (("g", 2.0), ("omega", 0.0), ("r", 0.0)):
+            ins[n] = round_to(rng.normal(m, 1.0, ins[n].shape), "bf16")
+        kw = dict(gates=kdn.KDN_GATES_LOGITS, r_min=0.01)
+        okw = dict(gates="logits", r_min=0.01)
+    d = to_dev(ins)
+    x = [d[n] for n in ("q", "k", "v", "g", "omega", "r")]
+    fsave = kdn.kdn_diag_fwd_save if variant == "diag" else kdn.kdn_iso_fwd_save
+    beff = kdn.kdn_diag_beta_eff if variant == "diag" else kdn.kdn_iso_beta_eff
+    _, _, _, saved = fsave(*x, d["S0"], d["p0"], **kw)
+    be = beff(d["k"], d["v"], d["g"], d["r"], saved, **kw)
+    torch.cuda.synchronize()
+    ref = oracle.fwd(variant, *[ins[n] for n in ("q", "k", "v", "g", "omega", "r")], ins["S0"],
+                     ins["p0"], trace=True, **okw)
+    ref_be = np.sum(ins["k"].astype(np.float64) * ref["kappa"], axis=-1)
+    got = to_np(be)
+    assert got.shape == (B, T, H)
+    assert np.all(got >= 0) and np.all(got < 1)
+    check("beta_eff", be, ref_be, "bf16")
