@@ -410,11 +410,12 @@ __global__ void __launch_bounds__(BT, 1)
     const unsigned char *rec = a.fSin + ((size_t)bh * NC + c) * kCtxBytes;
     float e16[16], ph16[16], tk[5];
     {
-      const float *cga = reinterpret_cast<const float *>(rec + kCtxGa) + t0 * D + ci;
+      // gamma [64][128] (SD: one value per token, [64])
+      const float *cga = reinterpret_cast<const float *>(rec + kCtxGa) + (SD ? t0 : t0 * D + ci);
       const float *cph = reinterpret_cast<const float *>(rec + kCtxPh) + t0 * D + ci;
       const float *tok = reinterpret_cast<const float *>(rec + kCtxTok);
 #pragma unroll
-      for (int j = 0; j < 16; ++j) e16[j] = cga[j * D];
+      for (int j = 0; j < 16; ++j) e16[j] = cga[SD ? j : j * D];
       if (V == 0) {
 #pragma unroll
         for (int j = 0; j < 16; ++j) ph16[j] = cph[j * D];

@@ -452,11 +452,7 @@ __global__ void __launch_bounds__(FT, 1)
           }
         }
         __syncthreads();
-        if (SD) {  // gamma is the same in every channel; the [64][128] copy is for the context
-          if (P.save_S) {
-#pragma unroll
-            for (int j = 0; j < 16; ++j) Eb[(t0 + j) * D + i] = s_gm[t0 + j];
-          }
+        if (SD) {  // gamma is the same in every channel: the context keeps the 64 values
           gc_out = s_gm[CM - 1];
         } else {
           float pre = 1.f;
@@ -479,7 +475,8 @@ __global__ void __launch_bounds__(FT, 1)
     if (tid == 0 && c + 1 < NC) issue_raw_g(c + 1);  // the decay tile is no longer read
     if (tid == 0 && P.save_S) {  // phat and gamma into the backward context
       if (V == 0) bulk_s2g(ctx + kCtxPh, Pb, 32768);
-      bulk_s2g(ctx + kCtxGa, Eb, 32768);
+      if (SD) bulk_s2g(ctx + kCtxGa, s_gm, CM * 4);  // one gamma per token
+      else bulk_s2g(ctx + kCtxGa, Eb, 32768);
       bulk_commit();
     }
     // ---- [3] operand tiles, 16-byte chunks (t, 8 channels), one half-warp per token:
