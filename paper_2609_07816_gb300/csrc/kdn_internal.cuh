@@ -164,8 +164,8 @@ size_t fused_ctx_record_bytes();
 
 // Sequence-parallel forward (kdn_segmented.cu): the number of segments P each
 // sequence is cut into (1: not used), the workspace it needs after the common
-// layout, and the launcher (gain summaries, scan, two fused runs per segment,
-// the state join and the final fused run).
+// layout, and the launcher (gain summaries, scan, one fused run per segment
+// carrying memory and transition, the state join, and the output pass).
 int seg_count(const Args &a);
 // Smallest forward workspace for a descriptor (the single-pass layout; 0 for an
 // invalid descriptor); kdn_fwd_workspace_bytes adds the segment buffers.
