@@ -180,7 +180,7 @@ template <int V, int OBF, int G, int SD>
 __global__ void __launch_bounds__(BT, 1)
     k_fused_bwd(const __grid_constant__ CUtensorMap mq, const __grid_constant__ CUtensorMap mk,
                 const __grid_constant__ CUtensorMap mv, const __grid_constant__ CUtensorMap mdo,
-                const BwdParams P) {
+                const __grid_constant__ CUtensorMap mw, const BwdParams P) {
   const Args &a = P.a;
   extern __shared__ unsigned char smraw[];
   unsigned char *sm =
@@ -212,6 +212,9 @@ __global__ void __launch_bounds__(BT, 1)
   float *s_kf = s_gm + 64;      // [64] beta_t / gamma_t (SD)
   uint64_t *bars = reinterpret_cast<uint64_t *>(sm + OFF_BAR);
   uint64_t *bar_a = bars, *bar_b = bars + 1, *bar_mma = bars + 2;
+  // diagonal KDN with logit gates: the chunk's omega logits (tile in O_KT, pass C)
+  uint64_t *bar_w = bars + 3;
+  constexpr bool WT = V == 0 && G;
   uint32_t *s_tbase = reinterpret_cast<uint32_t *>(bars + 4);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -226,11 +229,13 @@ __global__ void __launch_bounds__(BT, 1)
     mbar_init(bar_a, 1);
     mbar_init(bar_b, 1);
     mbar_init(bar_mma, 1);
+    if (WT) mbar_init(bar_w, 1);
     fence_mbar_init();
     prefetch_tmap(&mq);
     prefetch_tmap(&mk);
     prefetch_tmap(&mv);
     prefetch_tmap(&mdo);
+    if (WT) prefetch_tmap(&mw);
   }
   if (warp == 0) {
     tmem_alloc(s_tbase, 512);
@@ -785,6 +790,10 @@ __global__ void __launch_bounds__(BT, 1)
       // top of its iteration: bring them into L2 now
       bulk_prefetch_l2(rec - kCtxBytes + kCtxPh, kCtxBytes - kCtxPh);
     }
+    if (WT && tid == 0) {  // this chunk's omega logits for pass C (O_KT is free until [3])
+      mbar_expect_tx(bar_w, 16384);
+      for (int s = 0; s < 2; ++s) tma_load_4d(sm + O_KT + s * 8192, &mw, bar_w, 64 * s, h, c * CM, b);
+    }
     // ---- [18] per channel (lane ci, tokens t0..t0+15): back through Gamma and the
     //           gain emission, then the uncertainty recursion backwards in time.
     //           Free TMEM columns hold per-(channel, token) intermediates between passes:
@@ -889,7 +898,9 @@ __global__ void __launch_bounds__(BT, 1)
         s_aff[(qq * D + ci) * 2 + 1] = Bv;
       }
       tmem_st_wait();
-      __syncthreads();
+      // (logit gates: the omega-logit tile has landed)
+      ok = __syncthreads_and(!WT || tid != 0 || mbar_wait(bar_w, it & 1, kWaitIters));
+      if (!ok) break;
       // pass C: the recursion backwards through this quarter's tokens
       {
         float dp = s_dp[ci];
@@ -898,13 +909,12 @@ __global__ void __launch_bounds__(BT, 1)
         float run = dgC * s_gC[ci];  // dG_63 gains dgamma_C gamma_C; it lies in every suffix
         for (int q2 = qq + 1; q2 < 4; ++q2) run += s_tot[q2 * D + ci];
         float rd16[16], drp[16];
-        // logit gates: the quarter's omega logits, loaded together for the chain
-        // factor sigmoid(y) of domega
+        // logit gates: the quarter's omega logits (TMA tile in O_KT; zero past T) for the
+        // chain factor sigmoid(y) of domega
         float ylog[16];
         if (G) {
 #pragma unroll
-          for (int j = 0; j < 16; ++j)
-            ylog[j] = j < nval ? ld<__nv_bfloat16>(a.omega, obase + (size_t)j * ostride) : 0.f;
+          for (int j = 0; j < 16; ++j) ylog[j] = bf(sm + O_KT, 8192, t0 + j, ci);
         }
         tmem_ld16(X3 + lane_base + t0, rd16);
 #pragma unroll
@@ -1142,6 +1152,10 @@ __global__ void __launch_bounds__(BT, 1)
       mbar_wait(bar_a, 1, kWaitIters);
       mbar_wait(bar_b, 0, kWaitIters);
       mbar_wait(bar_b, 1, kWaitIters);
+      if (WT) {
+        mbar_wait(bar_w, 0, kWaitIters);
+        mbar_wait(bar_w, 1, kWaitIters);
+      }
     }
   }
   tc_fence_before();
@@ -1168,6 +1182,9 @@ kdn_status_t launch_fused_bwd_sweep(const Args &a, cudaStream_t s) {
   if (!make_map(&mq, a.q, a) || !make_map(&mk, a.k, a) || !make_map(&mv, a.v, a) ||
       !make_map(&mdo, a.dO, a))
     return KDN_ERR_CUDA;
+  CUtensorMap mw = mq;  // the omega logits (diagonal KDN, logit gates)
+  if (a.variant == 0 && a.gates && !make_map(&mw, a.omega, a))
+    return KDN_ERR_CUDA;
   const bool obf = a.odt == KDN_BF16;
   decltype(&k_fused_bwd<0, 0, 0, 0>) kern;
   if (a.variant == 0)
@@ -1182,7 +1199,7 @@ kdn_status_t launch_fused_bwd_sweep(const Args &a, cudaStream_t s) {
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES) !=
       cudaSuccess)
     return KDN_ERR_CUDA;
-  kern<<<a.B * a.H, BT, SMEM_BYTES, s>>>(mq, mk, mv, mdo, P);
+  kern<<<a.B * a.H, BT, SMEM_BYTES, s>>>(mq, mk, mv, mdo, mw, P);
   return cudaGetLastError() == cudaSuccess ? KDN_OK : KDN_ERR_CUDA;
 }
 
