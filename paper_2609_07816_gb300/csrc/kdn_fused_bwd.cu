@@ -704,6 +704,10 @@ __global__ void __launch_bounds__(BT, 1)
     if (!(ok = mma_wait())) break;
     tc_fence_after();
     if (tid == 0 && c > 0) issue_b_v(c - 1);  // v buffer is free
+    if (WT && tid == 0) {  // this chunk's omega logits for pass C (B6 has read dR^T in O_KT,
+      mbar_expect_tx(bar_w, 16384);  // which is free until [3] of the next chunk)
+      for (int s = 0; s < 2; ++s) tma_load_4d(sm + O_KT + s * 8192, &mw, bar_w, 64 * s, h, c * CM, b);
+    }
     // ---- [16] dT = strict_lower(-A^T dA A^T): X = A^T dA, Y = X A^T (fp16)
     if (wq < 2) {
       const int s = 32 * wq + lane, tc0 = 16 * wg;
@@ -789,10 +793,6 @@ __global__ void __launch_bounds__(BT, 1)
       // phat, gamma and the token scalars of chunk c - 1 are read with plain loads at the
       // top of its iteration: bring them into L2 now
       bulk_prefetch_l2(rec - kCtxBytes + kCtxPh, kCtxBytes - kCtxPh);
-    }
-    if (WT && tid == 0) {  // this chunk's omega logits for pass C (O_KT is free until [3])
-      mbar_expect_tx(bar_w, 16384);
-      for (int s = 0; s < 2; ++s) tma_load_4d(sm + O_KT + s * 8192, &mw, bar_w, 64 * s, h, c * CM, b);
     }
     // ---- [18] per channel (lane ci, tokens t0..t0+15): back through Gamma and the
     //           gain emission, then the uncertainty recursion backwards in time.
