@@ -898,9 +898,12 @@ __global__ void __launch_bounds__(BT, 1)
         s_aff[(qq * D + ci) * 2 + 1] = Bv;
       }
       tmem_st_wait();
-      // (logit gates: the omega-logit tile has landed)
-      ok = __syncthreads_and(!WT || tid != 0 || mbar_wait(bar_w, it & 1, kWaitIters));
-      if (!ok) break;
+      if (WT) {  // logit gates: the omega-logit tile has landed
+        ok = __syncthreads_and(tid != 0 || mbar_wait(bar_w, it & 1, kWaitIters));
+        if (!ok) break;
+      } else {
+        __syncthreads();
+      }
       // pass C: the recursion backwards through this quarter's tokens
       {
         float dp = s_dp[ci];
