@@ -75,7 +75,7 @@ def decode_bytes(b, h, dk, dv, in_bytes=2, out_bytes=4):
 # DRAM bytes per launch of each kernel at the bench workload, from one ncu
 # capture (dram__bytes_read.sum + dram__bytes_write.sum) of the current build;
 # reported as `traffic` only for that workload.
-NCU_TRAFFIC = {"k_fused_fwd": 672270592 + 1443449344, "k_fused_bwd": 1898262016 + 1315403264}
+NCU_TRAFFIC = {"k_fused_fwd": 672253952 + 1443657984, "k_fused_bwd": 1898199296 + 1315182080}
 
 
 def chunk_flops(dk, dv, C=64):
