@@ -32,6 +32,13 @@
 // fp32; with alpha = sigmoid(x) that needs an average alpha > 0.29 over a
 // 64-token chunk).  Every wait on an mbarrier is bounded; on timeout the
 // kernel records KDN_ERR_TIMEOUT in the workspace status word and returns.
+//
+// Instantiations (template <V, G, SD, PH>, described at the kernel): the
+// variant, logit gates, the isotropic KDN with one decay per head (exact
+// single-MMA intra-chunk products on the raw tiles), and the transition pass of
+// the sequence-parallel forward (a second memory from S = I with v = 0).  This
+// file also holds k_beta_eff, which reads the gain scalars a training forward
+// saved.
 #include "kdn_internal.cuh"
 #include "kdn_sm103.cuh"
 #include "kdn_fused_common.cuh"
