@@ -147,3 +147,31 @@ def test_logit_gates_decode(kdn, variant):
         check(f"o[{t}]", o, oref, "bf16")
     check("S", S, Sr, "bf16")
     check("p", p, pr, "bf16")
+
+
+@pytest.mark.parametrize("variant,pc", [("diag", True), ("iso", False), ("iso", True)])
+@pytest.mark.parametrize("logits", [False, True])
+def test_fused_backward_bf16_gradients_every_instantiation(kdn, variant, pc, logits):
+    """bf16-stored gradients from every fused backward instantiation: both
+    variants, one or per-channel isotropic decay, post-activation and logit
+    gates, on a ragged T; each gradient meets the bf16 rule plus its own
+    rounding."""
+    from kdn_gpu_util import check_stored_bf16
+    B, T, H = 1, 140, 2
+    ins = make_inputs(variant, B, T, H, 128, 128, dtype="bf16", seed=97, s0_std=0.05,
+                      p0_range=(0.5, 2.0), per_channel_decay=pc, with_grad=True)
+    kw, okw = {}, {}
+    if logits:
+        ins = _logits(ins, "bf16", 101)
+        kw = dict(gates=kdn.KDN_GATES_LOGITS, r_min=R_MIN)
+        okw = dict(gates="logits", r_min=R_MIN)
+    _, bwd, _, _ = _fns(kdn, variant)
+    d = to_dev(ins)
+    grads = bwd(*[d[n] for n in NAMES], d["S0"], d["p0"], d["dO"], out_dtype=torch.bfloat16, **kw)
+    torch.cuda.synchronize()
+    gref = oracle.bwd(variant, *[ins[n] for n in NAMES], ins["S0"], ins["p0"], ins["dO"], **okw)
+    for n in ("dq", "dk", "dv", "dg", "domega", "dr"):
+        assert grads[n].dtype == torch.bfloat16
+        check_stored_bf16(n, grads[n], gref[n])
+    for n in ("dS0", "dp0"):
+        check(n, grads[n], gref[n], "bf16")
