@@ -297,6 +297,17 @@ int kdn_kernel_launches(const kdn_desc_t *desc, int variant, int op);
    workspace gave up.  Each of those calls clears the word before it starts. */
 kdn_status_t kdn_get_device_status(void *workspace, void *stream);
 
+/* Self-test of the device-side failure reporting: clears the status word of
+   `workspace` (any workspace of at least 256 bytes, 256-byte aligned) and
+   launches one small kernel. Thread 0 waits, with the bounded wait every
+   kernel of this library uses, on an mbarrier phase that nothing completes.
+   After 4096 polls, well under a millisecond, the kernel records
+   KDN_ERR_TIMEOUT in the word and returns normally, so the CUDA context stays
+   usable.
+   kdn_get_device_status(workspace, stream) then returns KDN_ERR_TIMEOUT.
+   Returns KDN_ERR_INVALID_ARG for a null or misaligned workspace. */
+kdn_status_t kdn_selftest_wait_timeout(void *workspace, void *stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -76,6 +76,7 @@ _SIG = {
     "kdn_iso_beta_eff": ([ctypes.POINTER(kdn_desc_t), _P, ctypes.c_size_t, _P, _P, _P], ctypes.c_int),
     "kdn_kernel_launches": ([ctypes.POINTER(kdn_desc_t), ctypes.c_int, ctypes.c_int], ctypes.c_int),
     "kdn_get_device_status": ([_P, _P], ctypes.c_int),
+    "kdn_selftest_wait_timeout": ([_P, _P], ctypes.c_int),
 }
 EXPORTED = tuple(_SIG)
 
@@ -433,6 +434,12 @@ def kdn_diag_fwd_noalloc(q, k, v, g, omega, r, S0=None, p0=None, *, o, ST=None, 
 def kdn_kernel_launches(desc: kdn_desc_t, variant: int, op: int) -> int:
     """Kernels one call launches (op 0 fwd, 1 bwd, 2 decode step)."""
     return int(lib().kdn_kernel_launches(ctypes.byref(desc), int(variant), int(op)))
+
+
+def kdn_selftest_wait_timeout(workspace, stream=None) -> int:
+    """Runs the device self-test of the bounded waits on ``workspace`` (asynchronous);
+    kdn_get_device_status then reports KDN_ERR_TIMEOUT."""
+    return int(lib().kdn_selftest_wait_timeout(_ptr(workspace), _stream(stream)))
 
 
 def kdn_get_device_status(workspace, stream=None) -> int:

@@ -465,6 +465,14 @@ kdn_status_t kdn_iso_beta_eff(const kdn_desc_t *desc, const void *saved, size_t 
   return beta_eff_entry(1, desc, saved, saved_bytes, r, beta_eff, stream);
 }
 
+kdn_status_t kdn_selftest_wait_timeout(void *workspace, void *stream) {
+  if (!workspace || ((uintptr_t)workspace % kAlign)) return KDN_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  unsigned *status = static_cast<unsigned *>(workspace);
+  if (cudaMemsetAsync(status, 0, sizeof(unsigned), s) != cudaSuccess) return KDN_ERR_CUDA;
+  return launch_wait_selftest(status, s);
+}
+
 kdn_status_t kdn_get_device_status(void *workspace, void *stream) {
   if (!workspace || ((uintptr_t)workspace % kAlign)) return KDN_ERR_INVALID_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);

@@ -925,10 +925,30 @@ __global__ void __launch_bounds__(CM) k_beta_eff(const Args a, const unsigned ch
   }
 }
 
+// Self-test of the bounded waits: thread 0 waits on phase 0 of an mbarrier that
+// nothing ever arrives on, with the same helper and a short poll limit (4096
+// polls, well under a millisecond), and the CTA reports the timeout in the status
+// word exactly as the fused kernels do.  No fault, trap or unbounded loop.
+__global__ void __launch_bounds__(32) k_wait_selftest(unsigned *status) {
+  __shared__ uint64_t bar;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    fence_mbar_init();
+  }
+  __syncthreads();
+  const bool ok = threadIdx.x != 0 || mbar_wait(&bar, 0, 1u << 12);
+  if (!__syncthreads_and(ok) && threadIdx.x == 0) atomicExch(status, (unsigned)KDN_ERR_TIMEOUT);
+}
+
 // ---------------------------------------------------------------------------
 // host side
 
 }  // namespace
+
+kdn_status_t launch_wait_selftest(unsigned *status, cudaStream_t s) {
+  k_wait_selftest<<<1, 32, 0, s>>>(status);
+  return cudaGetLastError() == cudaSuccess ? KDN_OK : KDN_ERR_CUDA;
+}
 
 kdn_status_t launch_beta_eff(const Args &a, const void *saved, float *out, cudaStream_t s) {
   const int NC = (a.T + CM - 1) / CM;

@@ -150,6 +150,8 @@ kdn_status_t launch_fused_fwd(const Args &a, cudaStream_t s, unsigned char *save
 // beta_eff [B,T,H] (float32) from the per-token gain scalars of a context saved by
 // the fused training forward (one launch).
 kdn_status_t launch_beta_eff(const Args &a, const void *saved, float *out, cudaStream_t s);
+// One bounded wait that runs out (the self-test of kdn_selftest_wait_timeout).
+kdn_status_t launch_wait_selftest(unsigned *status, cudaStream_t s);
 // Fused tcgen05 backward (Diagonal KDN, bf16, dk = dv = 128, 64-token chunks):
 // one reverse sweep per (batch, head) from the saved context in a.fSin / a.fpin.
 // launch_fused_bwd first runs the context-saving forward (without o).

@@ -268,3 +268,11 @@ def test_beta_eff_validation(kdn):
         assert call(d, saved_bytes=n - 1) == kdn.KDN_ERR_WORKSPACE
         assert call(kdn.make_desc(B, 0, H, 128, 128, kdn.KDN_BF16), saved=None) == kdn.KDN_OK
         assert call(d, saved=MIS) == kdn.KDN_ERR_INVALID_ARG
+
+
+def test_wait_timeout_selftest_validates(kdn):
+    """The device self-test of the bounded waits rejects a null or misaligned
+    workspace before anything runs (no GPU needed)."""
+    L = kdn.lib()
+    assert L.kdn_selftest_wait_timeout(None, None) == kdn.KDN_ERR_INVALID_ARG
+    assert L.kdn_selftest_wait_timeout(MIS, None) == kdn.KDN_ERR_INVALID_ARG

@@ -521,3 +521,19 @@ def test_beta_eff_from_saved_context(kdn, variant, pc, gates):
     assert got.shape == (B, T, H)
     assert np.all(got >= 0) and np.all(got < 1)
     check("beta_eff", be, ref_be, "bf16")
+
+
+def test_bounded_wait_timeout_is_reported(kdn):
+    """Failure detection without a fault: a bounded device wait on an mbarrier
+    phase nothing completes gives up after its poll limit, the kernel records
+    KDN_ERR_TIMEOUT in the workspace status word and returns; the status query
+    reports and clears it, and the same context and workspace then run a
+    forward that matches the oracle."""
+    ws = torch.empty(4096, dtype=torch.uint8, device="cuda")
+    assert kdn.kdn_selftest_wait_timeout(ws) == kdn.KDN_OK
+    assert kdn.kdn_get_device_status(ws) == kdn.KDN_ERR_TIMEOUT
+    assert kdn.kdn_get_device_status(ws) == kdn.KDN_OK  # cleared by the query
+    ins = make_inputs("diag", 1, 100, 2, 128, 128, dtype="bf16", seed=107, s0_std=0.05)
+    o, _, _ = _gpu_fwd(kdn, "diag", to_dev(ins))
+    torch.cuda.synchronize()
+    check("o", o, _oracle_fwd("diag", ins)["o"], "bf16")
