@@ -2,15 +2,22 @@
 
 One step = one Diagonal-KDN training forward + backward (all steps of the
 chunked forward, its adjoint) over one synthetic batch shaped like a 1.3B-model
-layer: B=8, H=16, T=4096, d_k=d_v=128, bfloat16 activations, float32 state and
-outputs.  The forward is kdn_diag_fwd_save (o, S_T, p_T and the per-chunk
-context of the backward) and the backward kdn_diag_bwd_saved (every gradient
-from that context); each is one kernel.  `value` is layer tokens/s (B*T per
-step, summed over ranks).  The same JSON line also carries the decode step
+layer: B=8, H=16, T=4096, d_k=d_v=128, bfloat16 activations, float32 state.
+o and the input gradients are stored in bfloat16, the dtype of their inputs.
+The forward is kdn_diag_fwd_save (o, S_T, p_T and the per-chunk context of the
+backward) and the backward kdn_diag_bwd_saved (every gradient from that
+context); each is one kernel.  `value` is layer tokens/s (B*T per step, summed
+over ranks).  The same JSON line also carries the plain inference forward of
+the same shape (kdn_diag_fwd: o, S_T, p_T, no context), the decode step
 (B=256, H=16, d=128, 1024 consecutive tokens in one CUDA graph) in steps/s, the
 roofline of the dominant kernel (the backward sweep) and of the forward, an
 end-to-end number through host buffers, and the oracle's CPU throughput on a
 bounded sample.
+
+Algorithmic bytes count every input read once and every output written once
+at its stored dtype (bf16 activations in, bf16 o and gradients out) plus the
+state once per sequence: 1538 B per token-head for the diagonal forward and
+2820 B for its backward at d = 128.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
 
@@ -52,14 +59,14 @@ def peaks():
 # ---------------------------------------------------------------------------
 # algorithmic work (bytes that must cross HBM once; no intermediates)
 
-def fwd_bytes(b, t, h, dk, dv, in_bytes=2, out_bytes=4, with_state=True):
+def fwd_bytes(b, t, h, dk, dv, in_bytes=2, out_bytes=2, with_state=True):
     # per token-head: q, k, g, omega (dk each) + v (dv) + r read; o (dv) written
     per_tok = (4 * dk + dv + 1) * in_bytes + dv * out_bytes
     per_seq = (dk * dv * 4 + dk * 4) if with_state else 0   # S_T, p_T written
     return b * t * h * per_tok + b * h * per_seq
 
 
-def bwd_bytes(b, t, h, dk, dv, in_bytes=2, out_bytes=4):
+def bwd_bytes(b, t, h, dk, dv, in_bytes=2, out_bytes=2):
     reads = (2 * dk + dv + 2 * dk + 1 + dv) * in_bytes          # q k v g omega r dO
     writes = (2 * dk + dv + 2 * dk + 1) * out_bytes              # dq dk dv dg domega dr
     per_seq = dk * dv * 4 + dk * 4                               # dS0, dp0
@@ -74,8 +81,9 @@ def decode_bytes(b, h, dk, dv, in_bytes=2, out_bytes=4):
 
 # DRAM bytes per launch of each kernel at the bench workload, from one ncu
 # capture (dram__bytes_read.sum + dram__bytes_write.sum) of the current build;
-# reported as `traffic` only for that workload.
-NCU_TRAFFIC = {"k_fused_fwd": 672253952 + 1443657984, "k_fused_bwd": 1898199296 + 1315182080}
+# reported as `traffic` only for that workload.  None: not captured for the
+# current kernels.
+NCU_TRAFFIC = {"k_fused_fwd": None, "k_fused_bwd": None, "k_fused_fwd_plain": None}
 
 
 def chunk_flops(dk, dv, C=64):
@@ -231,14 +239,14 @@ def run_gpu(args):
     dt = torch.bfloat16
     ins = device_inputs("diag", B, T, H, DK, DV, seed=1000 + rank, dtype=dt)
     x = [ins[n] for n in NAMES]
-    desc = kdn.make_desc(B, T, H, DK, DV, dt)
+    desc = kdn.make_desc(B, T, H, DK, DV, dt, out_dtype=dt)
     ws_f = kdn.alloc_workspace(desc, 0, False)
     ws_b = kdn.alloc_workspace(desc, 0, False)
     saved = torch.empty(kdn.saved_bytes(desc), dtype=torch.uint8, device="cuda")
-    o = torch.empty(B, T, H, DV, dtype=torch.float32, device="cuda")
+    o = torch.empty(B, T, H, DV, dtype=dt, device="cuda")
     ST = torch.empty(B, H, DK, DV, dtype=torch.float32, device="cuda")
     pT = torch.empty(B, H, DK, dtype=torch.float32, device="cuda")
-    grads = {n: torch.empty(ins[m].shape, dtype=torch.float32, device="cuda") for n, m in
+    grads = {n: torch.empty(ins[m].shape, dtype=dt, device="cuda") for n, m in
              (("dq", "q"), ("dk", "k"), ("dv", "v"), ("dg", "g"), ("domega", "omega"),
               ("dr", "r"))}
     grads["dS0"] = torch.empty(B, H, DK, DV, dtype=torch.float32, device="cuda")
@@ -248,11 +256,11 @@ def run_gpu(args):
     def step(ev=None):
         if ev is not None:
             ev[0].record(stream)
-        kdn.kdn_diag_fwd_save(*x, o=o, ST=ST, pT=pT, saved=saved, workspace=ws_f)
+        kdn.kdn_diag_fwd_save(*x, o=o, ST=ST, pT=pT, saved=saved, workspace=ws_f, out_dtype=dt)
         if ev is not None:
             ev[1].record(stream)
         if not args.fwd_only:
-            kdn.kdn_diag_bwd_saved(*x, saved, ins["dO"], grads=grads, workspace=ws_b)
+            kdn.kdn_diag_bwd_saved(*x, saved, ins["dO"], grads=grads, workspace=ws_b, out_dtype=dt)
         if ev is not None:
             ev[2].record(stream)
 
@@ -293,8 +301,10 @@ def run_gpu(args):
         roof, other = fwd_roof, None
     else:
         roof, other = (bwd_roof, fwd_roof) if bwd_ms >= fwd_ms else (fwd_roof, bwd_roof)
-    # the paper-style roofline: max(FLOPs / 2.25 PF, bytes / 8 TB/s)
-    spec_time = max(B * T * H * chunk_flops(DK, DV) * 3.5 / 2.25e15, (fb + bb) / 8e12)
+    # the roofline of the step against the spec peaks, max(FLOPs / 2.25 PF, bytes / 8 TB/s):
+    # the bytes term binds (the forward's FLOPs take 42 us at the bench size, its bytes 102 us)
+    spec_time = (fb + bb) / 8e12
+    plain = run_forward_plain(kdn, torch, args, x, hbm, peak_kind) if rank == 0 else None
 
     dec = (run_decode(kdn, torch, hbm, args.decode_steps)
            if rank == 0 and not args.no_decode else None)
@@ -309,12 +319,13 @@ def run_gpu(args):
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
         "data": "synthetic",
         "config": {"workload": "Diagonal KDN fwd+bwd, 1.3B-layer shape", "B": B, "T": T, "H": H,
-                   "dk": DK, "dv": DV, "activations": "bf16", "outputs": "f32",
+                   "dk": DK, "dv": DV, "activations": "bf16", "outputs": "bf16",
                    "state": "f32", "parallelism": f"replicas x{world}",
                    "l2": "inputs larger than L2 (each activation tensor 134 MB)"},
         "fwd_ms": fwd_ms, "bwd_ms": bwd_ms,
         "roofline": roof, "roofline_other_kernel": other,
         "spec_roofline_frac": spec_time / (ms_step / 1e3) if ms_step > 0 else None,
+        "forward_plain": plain,
         "gpu_launches": launches_per_step * args.steps,
         "clocks": clk.summary(),
         "decode": dec, "iso_step": iso, "e2e": e2e, "long_context": lng, "logit_gates": lgt,
@@ -328,6 +339,49 @@ def run_gpu(args):
         dist.destroy_process_group()
 
 
+def run_forward_plain(kdn, torch, args, x, hbm, peak_kind):
+    """The inference forward of the bench shape (B=8, H=16, T=4096, d=128):
+    kdn_diag_fwd writing o (bf16), S_T and p_T, without the backward context;
+    tokens/s and its roofline, against the spec peak (bytes / 8 TB/s, the
+    target's formula) and against the measured copy rate."""
+    dt = torch.bfloat16
+    desc = kdn.make_desc(B, T, H, DK, DV, dt, out_dtype=dt)
+    ws = kdn.alloc_workspace(desc, 0, False)
+    o = torch.empty(B, T, H, DV, dtype=dt, device="cuda")
+    ST = torch.empty(B, H, DK, DV, dtype=torch.float32, device="cuda")
+    pT = torch.empty(B, H, DK, dtype=torch.float32, device="cuda")
+
+    def fwd():
+        kdn.kdn_diag_fwd(*x, o=o, ST=ST, pT=pT, workspace=ws, out_dtype=dt)
+
+    for _ in range(args.warmup):
+        fwd()
+    torch.cuda.synchronize()
+    stream = torch.cuda.current_stream()
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in range(args.steps)]
+    for e0, e1 in evs:
+        e0.record(stream)
+        fwd()
+        e1.record(stream)
+    torch.cuda.synchronize()
+    ms = statistics.mean(e0.elapsed_time(e1) for e0, e1 in evs)
+    nb = fwd_bytes(B, T, H, DK, DV)
+    flops = B * T * H * chunk_flops(DK, DV)
+    spec_s = max(nb / 8e12, flops / 2.25e15)
+    return {"workload": f"Diagonal KDN forward, B={B} H={H} T={T} d=128, bf16 in / bf16 o, "
+                        "f32 state (kdn_diag_fwd)",
+            "value": B * T / (ms / 1e3), "unit": "tokens/s", "ms": ms,
+            "gpu_launches": kdn.kdn_kernel_launches(desc, 0, 0) * args.steps,
+            "spec_roofline_frac": spec_s / (ms / 1e3),
+            "spec_roofline_us": spec_s * 1e6,
+            "roofline": {"bound": "hbm", "kernel": "k_fused_fwd (kdn_diag_fwd)",
+                         "achieved": nb / (ms / 1e3) / 1e9, "peak": hbm, "unit": "GB/s",
+                         "peak_kind": peak_kind, "frac": nb / (ms / 1e3) / 1e9 / hbm,
+                         "algorithmic_bytes": nb,
+                         "traffic": NCU_TRAFFIC["k_fused_fwd_plain"] if B == 8 else None}}
+
+
 def run_iso_step(kdn, torch, args, hbm):
     """The Isotropic KDN on its 750M-layer shape (B=8, H=12, T=2048, d=128, one
     decay per head): the training step kdn_iso_fwd_save + kdn_iso_bwd_saved, and
@@ -336,13 +390,15 @@ def run_iso_step(kdn, torch, args, hbm):
     b, t, h = 8, 2048, 12
     ins = device_inputs("iso", b, t, h, DK, DV, seed=7, dtype=torch.bfloat16, per_channel=False)
     x = [ins[n] for n in NAMES]
-    desc = kdn.make_desc(b, t, h, DK, DV, torch.bfloat16, decay_per_channel=0)
+    bf = torch.bfloat16
+    desc = kdn.make_desc(b, t, h, DK, DV, bf, decay_per_channel=0, out_dtype=bf)
     saved = torch.empty(kdn.saved_bytes(desc, 1), dtype=torch.uint8, device="cuda")
     ws = kdn.alloc_workspace(desc, 1, False)
 
     def step():
-        kdn.kdn_iso_fwd_save(*x, saved=saved, want_state=False, workspace=ws)
-        kdn.kdn_iso_bwd_saved(*x, saved, ins["dO"], want_state_grads=False, workspace=ws)
+        kdn.kdn_iso_fwd_save(*x, saved=saved, want_state=False, workspace=ws, out_dtype=bf)
+        kdn.kdn_iso_bwd_saved(*x, saved, ins["dO"], want_state_grads=False, workspace=ws,
+                              out_dtype=bf)
 
     for _ in range(args.warmup):
         step()
@@ -355,12 +411,12 @@ def run_iso_step(kdn, torch, args, hbm):
     torch.cuda.synchronize()
     ms = e0.elapsed_time(e1) / args.steps
     # the inference forward alone (o, S_T, b_T) through kdn_iso_fwd
-    o = torch.empty(b, t, h, DV, dtype=torch.float32, device="cuda")
+    o = torch.empty(b, t, h, DV, dtype=bf, device="cuda")
     ST = torch.empty(b, h, DK, DV, dtype=torch.float32, device="cuda")
     bT = torch.empty(b, h, dtype=torch.float32, device="cuda")
 
     def fwd():
-        kdn.kdn_iso_fwd(*x, o=o, ST=ST, pT=bT, workspace=ws)
+        kdn.kdn_iso_fwd(*x, o=o, ST=ST, pT=bT, workspace=ws, out_dtype=bf)
 
     for _ in range(args.warmup):
         fwd()
@@ -375,15 +431,16 @@ def run_iso_step(kdn, torch, args, hbm):
     # the paper's layer: one decay per channel (alpha_t in R^dk), same shape, both calls
     pins = device_inputs("iso", b, t, h, DK, DV, seed=8, dtype=torch.bfloat16, per_channel=True)
     px = [pins[n] for n in NAMES]
-    pdesc = kdn.make_desc(b, t, h, DK, DV, torch.bfloat16, decay_per_channel=1)
+    pdesc = kdn.make_desc(b, t, h, DK, DV, bf, decay_per_channel=1, out_dtype=bf)
     psaved = torch.empty(kdn.saved_bytes(pdesc, 1), dtype=torch.uint8, device="cuda")
 
     def pstep():
-        kdn.kdn_iso_fwd_save(*px, saved=psaved, want_state=False, workspace=ws)
-        kdn.kdn_iso_bwd_saved(*px, psaved, pins["dO"], want_state_grads=False, workspace=ws)
+        kdn.kdn_iso_fwd_save(*px, saved=psaved, want_state=False, workspace=ws, out_dtype=bf)
+        kdn.kdn_iso_bwd_saved(*px, psaved, pins["dO"], want_state_grads=False, workspace=ws,
+                              out_dtype=bf)
 
     def pfwd():
-        kdn.kdn_iso_fwd(*px, o=o, ST=ST, pT=bT, workspace=ws)
+        kdn.kdn_iso_fwd(*px, o=o, ST=ST, pT=bT, workspace=ws, out_dtype=bf)
 
     res_pc = {}
     for name, fn in (("step", pstep), ("forward", pfwd)):
@@ -423,7 +480,7 @@ def run_logit_step(kdn, torch, args, x, o, saved, grads, ws_f, ws_b, dO):
     lg = [t for t in x]
     for idx, mean in ((3, 2.0), (4, 0.0), (5, 0.0)):
         lg[idx] = (torch.randn(x[idx].shape, device="cuda", generator=gen) + mean).to(x[idx].dtype)
-    kw = dict(gates=kdn.KDN_GATES_LOGITS, r_min=0.01)
+    kw = dict(gates=kdn.KDN_GATES_LOGITS, r_min=0.01, out_dtype=o.dtype)
 
     def step():
         kdn.kdn_diag_fwd_save(*lg, o=o, want_state=False, saved=saved, workspace=ws_f, **kw)
@@ -462,16 +519,17 @@ def run_long_context(kdn, torch, args, hbm):
         S0 = 0.02 * torch.randn(b, h, DK, DV, device="cuda", generator=gen)
         pshape = (b, h, DK) if pc else (b, h)
         p0 = 0.5 + 1.5 * torch.rand(pshape, device="cuda", generator=gen)
-        desc = kdn.make_desc(b, t, h, DK, DV, torch.bfloat16, decay_per_channel=int(pc))
+        desc = kdn.make_desc(b, t, h, DK, DV, torch.bfloat16, decay_per_channel=int(pc),
+                             out_dtype=torch.bfloat16)
         vi = 0 if pc else 1
         ws = kdn.alloc_workspace(desc, vi)
-        o = torch.empty(b, t, h, DV, dtype=torch.float32, device="cuda")
+        o = torch.empty(b, t, h, DV, dtype=torch.bfloat16, device="cuda")
         ST = torch.empty(b, h, DK, DV, dtype=torch.float32, device="cuda")
         pT = torch.empty(pshape, dtype=torch.float32, device="cuda")
         fn = kdn.kdn_diag_fwd if pc else kdn.kdn_iso_fwd
 
         def call():
-            fn(*x, S0, p0, o=o, ST=ST, pT=pT, workspace=ws)
+            fn(*x, S0, p0, o=o, ST=ST, pT=pT, workspace=ws, out_dtype=torch.bfloat16)
 
         for _ in range(max(3, args.warmup)):
             call()
@@ -489,7 +547,7 @@ def run_long_context(kdn, torch, args, hbm):
             nb -= b * t * h * 2 * DK * 2 - b * t * h * 2 * 2
         res[variant] = {
             "workload": f"{'Diagonal' if pc else 'Isotropic'} KDN forward, B={b} H={h} T={t} "
-                        f"d=128, bf16 in, f32 o / state",
+                        f"d=128, bf16 in / bf16 o, f32 state",
             "value": b * t / (ms / 1e3), "unit": "tokens/s", "ms": ms,
             "sequence_parallel": kdn.kdn_kernel_launches(desc, vi, 0) == 5,
             "gpu_launches": kdn.kdn_kernel_launches(desc, vi, 0),
@@ -568,11 +626,12 @@ def run_e2e(kdn, torch, x, ins, args):
     bufs = [{n: torch.empty_like(ins[n]) for n in names} for _ in range(2)]
     comp = torch.cuda.current_stream()
     copy = torch.cuda.Stream()
-    desc = kdn.make_desc(B, T, H, DK, DV, torch.bfloat16)
+    bf = torch.bfloat16
+    desc = kdn.make_desc(B, T, H, DK, DV, bf, out_dtype=bf)
     saved = torch.empty(kdn.saved_bytes(desc), dtype=torch.uint8, device="cuda")
     ws = kdn.alloc_workspace(desc, 0, False)
-    o = torch.empty(B, T, H, DV, dtype=torch.float32, device="cuda")
-    grads = {n: torch.empty(ins[m].shape, dtype=torch.float32, device="cuda") for n, m in
+    o = torch.empty(B, T, H, DV, dtype=bf, device="cuda")
+    grads = {n: torch.empty(ins[m].shape, dtype=bf, device="cuda") for n, m in
              (("dq", "q"), ("dk", "k"), ("dv", "v"), ("dg", "g"), ("domega", "omega"),
               ("dr", "r"))}
     nmax = args.warmup + args.steps
@@ -592,10 +651,10 @@ def run_e2e(kdn, torch, x, ins, args):
         b = i % 2
         comp.wait_event(copied[b])
         xx = [bufs[b][n] for n in NAMES]
-        kdn.kdn_diag_fwd_save(*xx, o=o, want_state=False, saved=saved, workspace=ws)
+        kdn.kdn_diag_fwd_save(*xx, o=o, want_state=False, saved=saved, workspace=ws, out_dtype=bf)
         kdn.kdn_diag_bwd_saved(*xx, saved, bufs[b]["dO"], grads=grads, want_state_grads=False,
-                               workspace=ws)
-        loss = torch.sum(o.view(-1) * bufs[b]["dO"].view(-1), dtype=torch.float32)
+                               workspace=ws, out_dtype=bf)
+        loss = torch.sum(o.view(-1).float() * bufs[b]["dO"].view(-1).float(), dtype=torch.float32)
         freed[b].record(comp)
         loss_host[i].copy_(loss, non_blocking=True)
 

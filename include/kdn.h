@@ -268,19 +268,32 @@ kdn_status_t kdn_iso_decode_step(const kdn_desc_t *desc, const void *q,
    a framework that forbids allocation outside its own allocator).  Arguments
    and results are those of kdn_diag_fwd without the workspace pair.
    Scratch is a fixed array of KDN_NOALLOC_SCRATCH_BYTES in the library's
-   device memory, held by every GPU that loads the library until exit; a
-   problem whose single-pass workspace exceeds it is rejected with
-   KDN_ERR_WORKSPACE before anything runs (the sequence-parallel forward is
-   used when its larger workspace fits the array, else the single pass).  The first call on a device looks
-   up the array's device address (cudaGetSymbolAddress, with that device
-   current); make it before any stream capture.  All calls on a device share
-   the array, so calls that overlap on the GPU race and must be serialised by
-   the caller. */
+   device memory, held by a GPU from the first use of the library on it (CUDA
+   loads the module lazily) until the process exits; a problem whose
+   single-pass workspace (kdn_fwd_workspace_bytes without the segment buffers
+   of the sequence-parallel forward) exceeds it is rejected with
+   KDN_ERR_WORKSPACE before anything runs.  The sequence-parallel forward is
+   used when its larger workspace fits the array, else the single pass.  The
+   first call on a device looks up the array's device address
+   (cudaGetSymbolAddress, with that device current) and caches it with the
+   device's CUDA context; a later call under another context (after a device
+   reset) looks it up again.  Make the first call before any stream capture.
+   All calls on a device share the array, so calls that overlap on the GPU
+   race and must be serialised by the caller. */
 kdn_status_t kdn_diag_fwd_noalloc(const kdn_desc_t *desc, const void *q,
                                   const void *k, const void *v, const void *g,
                                   const void *omega, const void *r,
                                   const float *S0, const float *p0, void *o,
                                   float *ST, float *pT, void *stream);
+
+/* Device status word of the most recent kdn_diag_fwd_noalloc call on the
+   current device (kept in the library's scratch array, which the caller cannot
+   address): synchronises `stream`, then returns and clears it, as
+   kdn_get_device_status does for a workspace (KDN_OK, KDN_ERR_RANGE or
+   KDN_ERR_TIMEOUT).  The paper has no counterpart.  Allocates nothing; the
+   first call on a device performs the same address look-up as
+   kdn_diag_fwd_noalloc. */
+kdn_status_t kdn_noalloc_device_status(void *stream);
 
 /* Number of CUDA kernels one call of an entry point launches for this
    descriptor when T > 0 (op 0 = kdn_*_fwd, 1 = kdn_*_bwd, 2 = kdn_*_decode_step,

@@ -76,6 +76,7 @@ _SIG = {
     "kdn_iso_beta_eff": ([ctypes.POINTER(kdn_desc_t), _P, ctypes.c_size_t, _P, _P, _P], ctypes.c_int),
     "kdn_kernel_launches": ([ctypes.POINTER(kdn_desc_t), ctypes.c_int, ctypes.c_int], ctypes.c_int),
     "kdn_get_device_status": ([_P, _P], ctypes.c_int),
+    "kdn_noalloc_device_status": ([_P], ctypes.c_int),
     "kdn_selftest_wait_timeout": ([_P, _P], ctypes.c_int),
 }
 EXPORTED = tuple(_SIG)
@@ -444,3 +445,8 @@ def kdn_selftest_wait_timeout(workspace, stream=None) -> int:
 
 def kdn_get_device_status(workspace, stream=None) -> int:
     return int(lib().kdn_get_device_status(_ptr(workspace), _stream(stream)))
+
+
+def kdn_noalloc_device_status(stream=None) -> int:
+    """Reads and clears the status word of the last kdn_diag_fwd_noalloc call."""
+    return int(lib().kdn_noalloc_device_status(_stream(stream)))
