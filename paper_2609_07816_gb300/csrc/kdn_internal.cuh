@@ -147,6 +147,14 @@ bool fused_fwd_supported(const Args &a);
 kdn_status_t launch_fused_fwd(const Args &a, cudaStream_t s, unsigned char *save_S = nullptr,
                               float *save_p = nullptr, bool write_o = true, float *phi_T = nullptr,
                               void *o_phi = nullptr);
+// Chunked forward of the Diagonal KDN in compact-WY form with tf32 intra-chunk
+// products (kdn_wy_fwd.cu): bf16 activations, post-activation gates, dk = dv =
+// 128, 64-token chunks; writes o, S_T, p_T where their pointers are non-null,
+// and with save_S / save_p the fused backward's context (the layout of
+// launch_fused_fwd's saving mode).
+bool wy_fwd_supported(const Args &a);
+kdn_status_t launch_wy_fwd(const Args &a, cudaStream_t s, unsigned char *save_S = nullptr,
+                           float *save_p = nullptr);
 // beta_eff [B,T,H] (float32) from the per-token gain scalars of a context saved by
 // the fused training forward (one launch).
 kdn_status_t launch_beta_eff(const Args &a, const void *saved, float *out, cudaStream_t s);

@@ -1,0 +1,917 @@
+// kdn_wy_fwd.cu -- chunked forward of the Diagonal KDN in compact-WY form
+// (App. F.2, eq. chunk-memory-wy / chunk-memory-output-state) for bfloat16
+// activations, d_k = d_v = 128 and chunks of C = 64 tokens, on the tcgen05
+// tensor cores of sm_103a.
+//
+// One CTA (16 warps) owns one (batch, head) and walks its chunks in order; the
+// 128 x 128 float32 memory S stays in tensor memory for the whole sequence,
+// every activation tile is read once by TMA and o is written once.  Per chunk,
+// with G_t = sum_{u<=t} g_u the cumulative log-decay inside the chunk (per
+// channel) and gamma_t = exp(G_t):
+//
+//   gain     warps 0-3, one thread per key channel, run the uncertainty
+//            recursion of Prop. 3 over the 64 tokens (eq. diag-cov-update,
+//            eq. prefix-diag-uncertainty).  Each thread writes
+//              Kk'_t = phat_t k_t exp(c - G_t)          (tf32, MMA-T operand)
+//              K'_t  = phat_t k_t exp(G_C - G_t)        (fp16, tensor memory)
+//            where c = G_C / 2 is a per-channel reference in the middle of
+//            the chunk's decay range.
+//   prepare  warps 4-11, one thread per (4 channels, 8 tokens), form
+//              Kbar_t = k_t exp(G_t - c), Qbar_t = tau q_t exp(G_t - c)  (tf32)
+//              Kbar_t = gamma_t k_t, Qbar_t = tau gamma_t q_t           (fp16)
+//   MMA-T    [Kbar; Qbar] Kk'^T (tf32) = [T'; A'_qk].  The ratios
+//            exp(G_t - G_s) of App. F.2 are exact products of the two
+//            referenced factors, each within exp(+-|G_C| / 2).
+//            s_t = r_t + sum_i phat_t,i k_t,i^2 (the denominator of the gain,
+//            eq. kla-box-gain) is r_t plus the diagonal of T'.
+//   solve    with L = diag(s) + strict_lower(T'), A = (I + T)^-1 = diag(s) L^-1
+//            (T = strict_lower(T') diag(1/s)) on CUDA cores in fp32.
+//   MMA-W/U  W = A Kbar, U = A V (fp16)
+//   MMA-S1   [U; 0] + [-W; Qbar] S_in = [R; Qbar S_in]          (fp16)
+//   MMA-O    O = Qbar S_in + A'_qk R'          with R' = diag(1/s) R
+//   MMA-S2   S_out = diag(gamma_C) S_in + K'^T R'   (K' in tensor memory)
+// so that A'_qk R' = A_qk R and K'^T R' = K_tail^T R of eq.
+// chunk-memory-output-state, with A_qk = lower(A'_qk) diag(1/s).  Every MMA
+// accumulates in float32 in tensor memory.
+//
+// Shared-memory instructions are the scarce resource of this kernel: every
+// per-element pass reads and writes 8 or 16 bytes per instruction wherever the
+// layout allows (the gain's per-channel recursion is the exception).
+//
+// Range: the referenced factors stay finite while the chunk's cumulative
+// log-decay G_C >= -160 in every channel (average alpha >= 0.082 over 64
+// tokens).  A chunk below that records KDN_ERR_RANGE in the status word.
+//
+// Every wait on an mbarrier is bounded; on timeout the kernel records
+// KDN_ERR_TIMEOUT in the status word, waits (bounded) for its copies in flight,
+// frees its tensor memory and returns.
+#include "kdn_internal.cuh"
+#include "kdn_sm103.cuh"
+#include "kdn_fused_common.cuh"
+
+namespace kdn {
+namespace {
+
+using namespace sm103;
+using namespace fused;
+
+constexpr int WT = 512;  // threads
+constexpr int CM = 64;   // chunk length
+constexpr int D = 128;   // d_k = d_v
+constexpr uint32_t kWait = 1u << 25;
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kMinHalfG = -80.f;  // c = G_C / 2 below this: out of range
+constexpr int kPrepThreads = 256;   // warps 4-11
+constexpr int kNamed = 128 + kPrepThreads;  // gain + prepare threads at named barrier 1
+
+// shared-memory map (bytes from the 1024-aligned base)
+constexpr int LT = 68;          // row stride (floats) of the fp32 T and A tiles
+constexpr int O_RK = 0;        // raw k  [64 t][128 i] bf16, two 64-channel slabs   16 KB
+constexpr int O_RG = 16384;    // raw g                                          16 KB
+constexpr int O_RW = 32768;    // raw omega                                      16 KB
+constexpr int O_V = 49152;     // q (TMA, the preparing pass), then V (TMA bf16 -> fp16),
+                               // then R' fp16 [64 s][128 j]                       16 KB
+constexpr int O_TA = 65536;    // tf32 [Kbar; Qbar] [128][128], four 32-channel slabs 64 KB
+constexpr int O_TB = 133120;   // tf32 Kk' [64][128], four slabs                   32 KB
+constexpr int O_KB = 165888;   // fp16 Kbar [64 s][128 i], two slabs (MMA-W B)     16 KB
+constexpr int O_AS1 = 182272;  // fp16 [-W; Qbar] [128][128], two slabs (MMA-S1 A) 32 KB
+constexpr int O_SMALL = 215040;
+// after MMA-T has read the tf32 tiles (T and A run 2 KB past the tf32 tile)
+constexpr int O_S16 = O_TA;                      // fp16 S_in [128 i][128 j], two slabs (MMA-S1 B)
+constexpr int O_SWT = O_TA + 32768;              // fp32 T' [64][LT]
+constexpr int O_SWA = O_SWT + 64 * LT * 4;       // fp32 L^-1 [64][LT]
+static_assert(O_SWA + 64 * LT * 4 <= O_TB, "T and A tiles overlap the Kk' tile");
+constexpr int O_AWU = O_TB;            // fp16 [A; 0] [128][64] (MMA-W/U A)
+constexpr int O_AO = O_TB + 16384;     // fp16 [0; A'_qk] [128][64] (MMA-O A)
+// inverse scratch in rows 0..63 of the first slab of [-W; Qbar] (written after it)
+constexpr int O_SX = O_AS1;            // 2 x 256 floats
+constexpr int O_SY = O_AS1 + 2048;     // 32 x 32 floats
+// small arrays (floats)
+constexpr int SM_R = 0, SM_MUR = 64, SM_S = 128, SM_IS = 192, SM_C = 256, SM_GC = 384,
+              SM_PART = 512, SM_FLOATS = 512 + 8 * 128;
+constexpr int O_BAR = O_SMALL + SM_FLOATS * 4;
+constexpr int SMEM_BYTES = O_BAR + 64 + 1024;
+
+// tensor-memory columns (512 allocated)
+constexpr uint32_t TC_S = 0, TC_D1 = 128, TC_KT = 192, TC_W = 256, TC_U = 384;
+
+__device__ __forceinline__ float ex2f(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+__device__ __forceinline__ float rcpf(float x) {
+  float y;
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+// round to tf32 (nearest, ties away): the tensor core reads the top 19 bits
+__device__ __forceinline__ float tf32r(float x) {
+  uint32_t u;
+  asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(u) : "f"(x));
+  return __uint_as_float(u);
+}
+// byte offset of fp32 element (row, col) of a 128-byte-swizzled tile with 32
+// elements per row
+__device__ __forceinline__ uint32_t sw32_off(uint32_t row, uint32_t col) {
+  return row * 128u + ((((col >> 2) ^ (row & 7u)) << 4) | ((col & 3u) << 2));
+}
+__device__ __forceinline__ void bar_arrive(int id, int n) {
+  asm volatile("bar.arrive %0, %1;" ::"r"(id), "r"(n) : "memory");
+}
+__device__ __forceinline__ void bar_sync(int id, int n) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory");
+}
+__host__ __device__ constexpr uint32_t idesc_tf32(int M, int N) {
+  return (1u << 4) | (2u << 7) | (2u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+__device__ __forceinline__ void umma_tf32(uint32_t d, uint64_t a, uint64_t b, uint32_t idesc,
+                                          uint32_t acc) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::tf32 [%0], %1, %2, %3, p;\n}\n" ::"r"(d),
+      "l"(a), "l"(b), "r"(idesc), "r"(acc)
+      : "memory");
+}
+// A operand in tensor memory: lane = row, 32-bit column c holds the 16-bit
+// elements 2c (low half) and 2c + 1 of that row
+__device__ __forceinline__ void umma_f16_tA(uint32_t d, uint32_t a_tmem, uint64_t b, uint32_t idesc,
+                                            uint32_t acc) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n}\n" ::"r"(d),
+      "r"(a_tmem), "l"(b), "r"(idesc), "r"(acc)
+      : "memory");
+}
+__device__ __forceinline__ void tmem_st4u(uint32_t taddr, const uint32_t *v) {
+  asm volatile("tcgen05.st.sync.aligned.32x32b.x4.b32 [%0], {%1, %2, %3, %4};" ::"r"(taddr),
+               "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3])
+               : "memory");
+}
+// four bf16 (8 bytes) -> floats
+__device__ __forceinline__ void unpack_bf4(uint2 u, float *v) {
+  v[0] = __uint_as_float(u.x << 16);
+  v[1] = __uint_as_float(u.x & 0xffff0000u);
+  v[2] = __uint_as_float(u.y << 16);
+  v[3] = __uint_as_float(u.y & 0xffff0000u);
+}
+__device__ __forceinline__ uint2 pack_h4(float a0, float a1, float a2, float a3) {
+  uint2 u;
+  __half2 h0 = __floats2half2_rn(a0, a1), h1 = __floats2half2_rn(a2, a3);
+  u.x = *reinterpret_cast<uint32_t *>(&h0);
+  u.y = *reinterpret_cast<uint32_t *>(&h1);
+  return u;
+}
+// byte offset of the 4 bf16 / fp16 channels i0..i0+3 (i0 % 4 == 0) of row t
+// in a 128-byte-swizzled [t][64] slab
+__device__ __forceinline__ uint32_t sw128_off4(uint32_t t, uint32_t i0) {
+  return t * 128u + (((((i0 & 63u) >> 3) ^ (t & 7u)) << 4) | ((i0 & 7u) << 1));
+}
+
+// X = L^-1 for the lower triangular 64 x 64 fp32 L = diag(s) + strict_lower(T')
+// held in sT (row stride LT; only the lower triangle is read), with
+// s_t = r_t + T'_tt, into sA (its strict upper triangle zero), by 16 x 16
+// blocks: the diagonal blocks D_I = L_II^-1 by forward substitution (one thread
+// per column), then the 32 x 32 halves
+//   X_10 = -D_1 L_10 D_0,  X_32 = -D_3 L_32 D_2,
+// and the lower-left quarter X_21 = -X22 L21 X11 (X11, X22 the 32 x 32
+// diagonal halves), each output thread forming four adjacent columns from
+// 16-byte loads.  s_t and 1 / s_t go to s_s, s_is.  Every thread of the CTA
+// calls it (block barriers inside).
+__device__ __forceinline__ void wy_inverse(const float *sT, float *sA, float *sX, float *sY,
+                                           const float *s_r, float *s_s, float *s_is) {
+  const int tid = threadIdx.x;
+  if (tid < 64) {
+    // column c of D_I: x_r = (delta_rc - sum_{m<r} L_rm x_m) / L_rr, rows read 16 bytes at a time
+    const int o = 16 * (tid >> 4), c = tid & 15;
+    const float *tb = sT + o * (LT + 1);
+    float x[16];
+#pragma unroll
+    for (int r = 0; r < 16; ++r) {
+      float lr[16];
+#pragma unroll
+      for (int j = 0; 4 * j <= r; ++j) {
+        const float4 t4 = *reinterpret_cast<const float4 *>(tb + r * LT + 4 * j);
+        lr[4 * j] = t4.x; lr[4 * j + 1] = t4.y; lr[4 * j + 2] = t4.z; lr[4 * j + 3] = t4.w;
+      }
+      const float lrr = s_r[o + r] + lr[r];  // s_t = r_t + sum_i phat k^2 (eq. kla-box-gain)
+      const float inv = rcpf(lrr);
+      if (r == c) {
+        s_s[o + r] = lrr;
+        s_is[o + r] = inv;
+      }
+      float acc0 = (r == c) ? 1.f : 0.f, acc1 = 0.f;
+#pragma unroll
+      for (int m = 0; m < r; ++m) {
+        if (m & 1) acc1 = fmaf(-lr[m], x[m], acc1);
+        else acc0 = fmaf(-lr[m], x[m], acc0);
+      }
+      x[r] = (acc0 + acc1) * inv;  // x[r] = 0 for r < c
+    }
+    float *ab = sA + o * (LT + 1) + c;
+#pragma unroll
+    for (int r = 0; r < 16; ++r) ab[r * LT] = x[r];
+  } else if (tid < 64 + 384) {
+    // zero the strictly upper 16 x 16 blocks (I < J): 6 blocks x 16 rows x 4 float4
+    const int e = tid - 64, blk = e >> 6, rr = (e >> 2) & 15, q4 = e & 3;
+    const int I = blk < 3 ? 0 : (blk < 5 ? 1 : 2);
+    const int J = blk < 3 ? blk + 1 : (blk < 5 ? blk - 1 : 3);
+    *reinterpret_cast<float4 *>(sA + (16 * I + rr) * LT + 16 * J + 4 * q4) = make_float4(0.f, 0.f, 0.f, 0.f);
+  }
+  __syncthreads();
+  // X_10, X_32: one thread per (block, row, 4 columns)
+  const int blk = tid >> 6, r2 = (tid >> 2) & 15, cq2 = 4 * (tid & 3);
+  const int C0 = 32 * blk, R0 = C0 + 16;
+  if (tid < 128) {
+    const float *tp = sT + (R0 + r2) * LT + C0;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const float4 t4 = *reinterpret_cast<const float4 *>(tp + 4 * j);
+      const float tv[4] = {t4.x, t4.y, t4.z, t4.w};
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const float4 a4 = *reinterpret_cast<const float4 *>(sA + (C0 + 4 * j + u) * LT + C0 + cq2);
+        acc.x = fmaf(tv[u], a4.x, acc.x);
+        acc.y = fmaf(tv[u], a4.y, acc.y);
+        acc.z = fmaf(tv[u], a4.z, acc.z);
+        acc.w = fmaf(tv[u], a4.w, acc.w);
+      }
+    }
+    *reinterpret_cast<float4 *>(sX + blk * 256 + r2 * 16 + cq2) = acc;
+  }
+  __syncthreads();
+  if (tid < 128) {
+    const float *dp = sA + (R0 + r2) * LT + R0;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const float4 d4 = *reinterpret_cast<const float4 *>(dp + 4 * j);
+      const float dv[4] = {d4.x, d4.y, d4.z, d4.w};
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const float4 x4 = *reinterpret_cast<const float4 *>(sX + blk * 256 + (4 * j + u) * 16 + cq2);
+        acc.x = fmaf(dv[u], x4.x, acc.x);
+        acc.y = fmaf(dv[u], x4.y, acc.y);
+        acc.z = fmaf(dv[u], x4.z, acc.z);
+        acc.w = fmaf(dv[u], x4.w, acc.w);
+      }
+    }
+    *reinterpret_cast<float4 *>(sA + (R0 + r2) * LT + C0 + cq2) = make_float4(-acc.x, -acc.y, -acc.z, -acc.w);
+  }
+  __syncthreads();
+  // Y = L21 X11, then X_21 = -X22 Y (32 x 32 x 32 each): one thread per (row, 4 columns)
+  const int r3 = tid >> 3, cq3 = 4 * (tid & 7);
+  if (tid < 256) {
+    const float *tp = sT + (32 + r3) * LT;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const float4 t4 = *reinterpret_cast<const float4 *>(tp + 4 * j);
+      const float tv[4] = {t4.x, t4.y, t4.z, t4.w};
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const float4 a4 = *reinterpret_cast<const float4 *>(sA + (4 * j + u) * LT + cq3);
+        acc.x = fmaf(tv[u], a4.x, acc.x);
+        acc.y = fmaf(tv[u], a4.y, acc.y);
+        acc.z = fmaf(tv[u], a4.z, acc.z);
+        acc.w = fmaf(tv[u], a4.w, acc.w);
+      }
+    }
+    *reinterpret_cast<float4 *>(sY + r3 * 32 + cq3) = acc;
+  }
+  __syncthreads();
+  if (tid < 256) {
+    const float *dp = sA + (32 + r3) * LT + 32;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const float4 d4 = *reinterpret_cast<const float4 *>(dp + 4 * j);
+      const float dv[4] = {d4.x, d4.y, d4.z, d4.w};
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const float4 y4 = *reinterpret_cast<const float4 *>(sY + (4 * j + u) * 32 + cq3);
+        acc.x = fmaf(dv[u], y4.x, acc.x);
+        acc.y = fmaf(dv[u], y4.y, acc.y);
+        acc.z = fmaf(dv[u], y4.z, acc.z);
+        acc.w = fmaf(dv[u], y4.w, acc.w);
+      }
+    }
+    *reinterpret_cast<float4 *>(sA + (32 + r3) * LT + cq3) = make_float4(-acc.x, -acc.y, -acc.z, -acc.w);
+  }
+  __syncthreads();
+}
+
+struct WyParams {
+  Args a;
+  unsigned char *save_S;  // SV: [BH][NC] context records of the backward (kCtxBytes each)
+  float *save_p;          // SV: [BH][NC][128] uncertainty carry entering each chunk
+};
+
+// SV: besides o, S_T and p_T (each written when its pointer is non-null), keep
+// the chunked backward's context: per chunk the fp16 tiles S_in, R, -W, A_qk
+// and A = (I + T)^-1 in the 128-byte-swizzled layout of the fused backward,
+// phat and gamma in float32 [64 t][128 i], s_t per token, and the uncertainty
+// entering the chunk.  The arithmetic is the same with and without it.
+
+template <int SV>
+__global__ void __launch_bounds__(WT, 1)
+    k_wy_fwd(const __grid_constant__ CUtensorMap mk, const __grid_constant__ CUtensorMap mg,
+             const __grid_constant__ CUtensorMap mw, const __grid_constant__ CUtensorMap mv,
+             const __grid_constant__ CUtensorMap mq, const WyParams P) {
+  const Args &a = P.a;
+  extern __shared__ unsigned char smraw[];
+  unsigned char *sm =
+      reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(smraw) + 1023) & ~uintptr_t(1023));
+  unsigned char *rk = sm + O_RK, *rg = sm + O_RG, *rw = sm + O_RW, *vr = sm + O_V;
+  unsigned char *ta = sm + O_TA, *tb = sm + O_TB, *kb = sm + O_KB, *as1 = sm + O_AS1;
+  unsigned char *s16 = sm + O_S16, *awu = sm + O_AWU, *ao = sm + O_AO;
+  float *sT = reinterpret_cast<float *>(sm + O_SWT), *sA = reinterpret_cast<float *>(sm + O_SWA);
+  float *sX = reinterpret_cast<float *>(sm + O_SX), *sY = reinterpret_cast<float *>(sm + O_SY);
+  float *sf = reinterpret_cast<float *>(sm + O_SMALL);
+  float *s_r = sf + SM_R, *s_mur = sf + SM_MUR, *s_s = sf + SM_S, *s_is = sf + SM_IS;
+  float *s_c = sf + SM_C, *s_gC = sf + SM_GC, *s_part = sf + SM_PART;
+  uint64_t *bars = reinterpret_cast<uint64_t *>(sm + O_BAR);
+  uint64_t *bar_raw = bars, *bar_v = bars + 1, *bar_mma = bars + 2, *bar_q = bars + 3;
+  uint32_t *s_tbase = reinterpret_cast<uint32_t *>(bars + 4);
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int wq = warp & 3, wg = warp >> 2;  // TMEM lane quarter, column group
+  const int bh = blockIdx.x, b = bh / a.H, h = bh % a.H;
+  const int NC = (a.T + CM - 1) / CM;
+  const bool issuer = tid == 128;
+  const uint32_t lane_base = (uint32_t)(32 * wq) << 16;
+
+  if (issuer) {
+    mbar_init(bar_raw, 1);
+    mbar_init(bar_v, 1);
+    mbar_init(bar_mma, 1);
+    mbar_init(bar_q, 1);
+    fence_mbar_init();
+    prefetch_tmap(&mk);
+    prefetch_tmap(&mg);
+    prefetch_tmap(&mw);
+    prefetch_tmap(&mv);
+    prefetch_tmap(&mq);
+  }
+  if (warp == 0) {
+    tmem_alloc(s_tbase, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tbase = *s_tbase;
+  const uint32_t TS = tbase + TC_S, TD1 = tbase + TC_D1, TKT = tbase + TC_KT, TW = tbase + TC_W,
+                 TU = tbase + TC_U;
+
+  // k, g, omega of chunk c (the gain and the preparing pass), q of chunk c (the
+  // preparing pass, in the V buffer), V of chunk c (after the preparing pass)
+  auto issue_raw = [&](int c) {
+    mbar_expect_tx(bar_raw, 49152);
+    for (int s = 0; s < 2; ++s) {
+      tma_load_4d(rk + s * 8192, &mk, bar_raw, 64 * s, h, c * CM, b);
+      tma_load_4d(rg + s * 8192, &mg, bar_raw, 64 * s, h, c * CM, b);
+      tma_load_4d(rw + s * 8192, &mw, bar_raw, 64 * s, h, c * CM, b);
+    }
+  };
+  auto issue_q = [&](int c) {
+    mbar_expect_tx(bar_q, 16384);
+    for (int s = 0; s < 2; ++s) tma_load_4d(vr + s * 8192, &mq, bar_q, 64 * s, h, c * CM, b);
+  };
+  auto issue_v = [&](int c) {
+    mbar_expect_tx(bar_v, 16384);
+    for (int s = 0; s < 2; ++s) tma_load_4d(vr + s * 8192, &mv, bar_v, 64 * s, h, c * CM, b);
+  };
+  if (issuer && NC > 0) {
+    issue_raw(0);
+    issue_q(0);
+    for (int s = 0; s < 2; ++s) tma_prefetch_4d(&mv, 64 * s, h, 0, b);
+  }
+
+  // initial memory S_0 -> TMEM (row = key channel i, column = value j)
+  {
+    const int i = 32 * wq + lane;
+    for (int c0 = 0; c0 < 32; c0 += 16) {
+      float v[16];
+      const int j0 = 32 * wg + c0;
+      if (a.S0) {
+        const float4 *src = reinterpret_cast<const float4 *>(a.S0 + ((size_t)bh * D + i) * D + j0);
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const float4 x = src[u];
+          v[4 * u] = x.x; v[4 * u + 1] = x.y; v[4 * u + 2] = x.z; v[4 * u + 3] = x.w;
+        }
+      } else {
+#pragma unroll
+        for (int u = 0; u < 16; ++u) v[u] = 0.f;
+      }
+      tmem_st16(TS + lane_base + j0, v);
+    }
+    tmem_st_wait();
+  }
+
+  // roles in the first phase of a chunk
+  const bool gain = tid < 128;
+  const bool prep = tid >= 128 && tid < 128 + kPrepThreads;
+  const int pi = tid - 128;  // preparing thread: channels 4 (pi % 32) .. +3, tokens 8 (pi / 32) .. +7
+  float p = 1.f;             // gain threads: uncertainty carry of channel tid
+  if (gain && a.p0) p = a.p0[(size_t)bh * D + tid];
+  float nr = 1.f;            // preparing threads pi < 64: r of token pi of the next chunk
+  auto load_r = [&](int c) {
+    if (pi >= 0 && pi < CM) {
+      nr = 1.f;
+      if (c < NC && c * CM + pi < a.T) nr = ld<__nv_bfloat16>(a.r, tok_index(a, b, c * CM + pi, h));
+    }
+  };
+  load_r(0);
+
+  uint32_t mph = 0;  // MMA-completion phases observed
+  bool ok = true;
+  auto mma_wait_all = [&]() -> bool {
+    const bool r = mbar_wait(bar_mma, mph & 1, kWait);
+    ++mph;
+    return r;
+  };
+  const uint32_t id_T = idesc_tf32(128, 64);
+  const uint32_t id_16 = idesc_f16(128, 128, 0, 1);  // A K-major, B MN-major
+
+  for (int c = 0; c < NC && ok; ++c) {
+    const uint32_t tkt = TKT + (uint32_t)((c & 1) * 32);
+    unsigned char *ctx = SV ? P.save_S + ((size_t)bh * NC + c) * kCtxBytes : nullptr;
+    if (SV && issuer) bulk_wait_read();  // the previous chunk's context tiles have left shared memory
+    // ---- [0] per-token scalars; the previous chunk's MMA-O / MMA-S2 must be done
+    //          before q is brought into its R' buffer
+    if (pi >= 0 && pi < CM) {
+      s_r[pi] = nr;
+      s_mur[pi] = a.mu / nr;
+    }
+    bool w_ok = mbar_wait(bar_raw, c & 1, kWait);
+    if (issuer && c > 0) {
+      w_ok = w_ok && mma_wait_all();  // MMA-O / MMA-S2 of chunk c - 1
+      if (w_ok) issue_q(c);
+    } else if (c > 0) {
+      ++mph;
+    }
+    ok = __syncthreads_and(w_ok);
+    if (!ok) break;
+
+    // ---- [1] gain (warps 0-3), operand preparation (warps 4-11) and the
+    //          previous chunk's output (warps 14, 15)
+    bool p_ok = true;
+    if (gain) {
+      const int i = tid;
+      const unsigned char *pg = rg + (i >> 6) * 8192, *pw = rw + (i >> 6) * 8192, *pk = rk + (i >> 6) * 8192;
+      const int cl = i & 63;
+      // element (t, i) of a raw slab: row t, 128-byte swizzle
+      auto raw = [&](const unsigned char *base, int t) {
+        return __bfloat162float(*reinterpret_cast<const __nv_bfloat16 *>(base + sw128_off(t, cl)));
+      };
+      float g0 = 0.f, g1 = 0.f, g2 = 0.f, g3 = 0.f;
+#pragma unroll
+      for (int t = 0; t < CM; t += 4) {
+        g0 += raw(pg, t);
+        g1 += raw(pg, t + 1);
+        g2 += raw(pg, t + 2);
+        g3 += raw(pg, t + 3);
+      }
+      const float GC = (g0 + g1) + (g2 + g3), cref = 0.5f * GC;
+      s_c[i] = cref;
+      if (cref < kMinHalfG) atomicCAS(a.status, 0u, (unsigned)KDN_ERR_RANGE);
+      bar_arrive(1, kNamed);
+      if (SV) P.save_p[((size_t)bh * NC + c) * D + i] = p;
+      float *cph = SV ? reinterpret_cast<float *>(ctx + kCtxPh) + i : nullptr;
+      float f = ex2f(cref * kLog2e);                // exp(c - G_t), G_{-1} = 0
+      const float E2 = ex2f((GC - cref) * kLog2e);  // exp(G_C - c)
+      unsigned char *pb = tb + (i >> 5) * 8192;
+      const int cb = i & 31;
+      // the chunk in blocks of 8 tokens; the next block's inputs are loaded
+      // before the current block's outputs are stored
+      float gb[8], wb[8], kb8[8], mb[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        gb[j] = raw(pg, j);
+        wb[j] = raw(pw, j);
+        kb8[j] = raw(pk, j);
+      }
+      {
+        const float4 m0 = *reinterpret_cast<const float4 *>(s_mur), m1 = *reinterpret_cast<const float4 *>(s_mur + 4);
+        mb[0] = m0.x; mb[1] = m0.y; mb[2] = m0.z; mb[3] = m0.w; mb[4] = m1.x; mb[5] = m1.y; mb[6] = m1.z; mb[7] = m1.w;
+      }
+#pragma unroll
+      for (int blk = 0; blk < 8; ++blk) {
+        float gn[8], wn[8], kn[8], mn[8];
+        if (blk < 7) {
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const int t = 8 * (blk + 1) + j;
+            gn[j] = raw(pg, t);
+            wn[j] = raw(pw, t);
+            kn[j] = raw(pk, t);
+          }
+          const float4 m0 = *reinterpret_cast<const float4 *>(s_mur + 8 * (blk + 1));
+          const float4 m1 = *reinterpret_cast<const float4 *>(s_mur + 8 * (blk + 1) + 4);
+          mn[0] = m0.x; mn[1] = m0.y; mn[2] = m0.z; mn[3] = m0.w; mn[4] = m1.x; mn[5] = m1.y; mn[6] = m1.z; mn[7] = m1.w;
+        }
+        uint32_t kt[4];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const int t = 8 * blk + j;
+          const float al = ex2f(gb[j] * kLog2e), a2 = al * al;
+          const float ph = fmaf(a2, p, wb[j]);               // eq. diag-covariance-prediction
+          const float u = kb8[j] * kb8[j] * mb[j];
+          const float den = fmaf(u, ph, 1.f);
+          const float x = rcpf(al * den);
+          p = ph * (x * al);                                  // eq. prefix-diag-uncertainty
+          f *= x * den;                                       // / alpha_t
+          const float pkv = ph * kb8[j];
+          if (SV) cph[t * D] = ph;
+          *reinterpret_cast<float *>(pb + sw32_off(t, cb)) = tf32r(pkv * f);
+          const uint32_t hb = (uint32_t)__half_as_ushort(__float2half_rn(pkv * (f * E2)));
+          if ((j & 1) == 0) kt[j >> 1] = hb;
+          else kt[j >> 1] |= hb << 16;
+        }
+        tmem_st4u(tkt + lane_base + (uint32_t)(4 * blk), kt);
+        if (blk < 7) {
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            gb[j] = gn[j];
+            wb[j] = wn[j];
+            kb8[j] = kn[j];
+            mb[j] = mn[j];
+          }
+        }
+      }
+      tmem_st_wait();
+    } else if (prep) {
+      const int i0 = 4 * (pi & 31), seg = pi >> 5, t0 = 8 * seg;
+      const uint32_t sl8 = (uint32_t)(i0 >> 6) * 8192u;  // 64-channel slab of a [t][64] 16-bit tile
+      // the chunk's g for this thread's 8 tokens and 4 channels (8 bytes a token)
+      uint2 gq[8];
+      float ps[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        gq[j] = *reinterpret_cast<const uint2 *>(rg + sl8 + sw128_off4(t0 + j, i0));
+        float gv[4];
+        unpack_bf4(gq[j], gv);
+#pragma unroll
+        for (int u = 0; u < 4; ++u) ps[u] += gv[u];
+      }
+      *reinterpret_cast<float4 *>(s_part + seg * D + i0) = make_float4(ps[0], ps[1], ps[2], ps[3]);
+      bar_sync(1, kNamed);
+      float cr[4], G[4] = {0.f, 0.f, 0.f, 0.f}, Ec[4], gm[4];
+      {
+        const float4 c4 = *reinterpret_cast<const float4 *>(s_c + i0);
+        cr[0] = c4.x; cr[1] = c4.y; cr[2] = c4.z; cr[3] = c4.w;
+      }
+      for (int s2 = 0; s2 < seg; ++s2) {
+        const float4 p4 = *reinterpret_cast<const float4 *>(s_part + s2 * D + i0);
+        G[0] += p4.x; G[1] += p4.y; G[2] += p4.z; G[3] += p4.w;
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) Ec[u] = ex2f(cr[u] * kLog2e);
+      p_ok = mbar_wait(bar_q, c & 1, kWait);
+      unsigned char *pa = ta + (i0 >> 5) * 16384, *pkb = kb + sl8, *pqh = as1 + (i0 >> 6) * 16384;
+      const int cc = i0 & 31;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const int t = t0 + j;
+        float gv[4], kv[4], qv[4], e[4];
+        unpack_bf4(gq[j], gv);
+        unpack_bf4(*reinterpret_cast<const uint2 *>(rk + sl8 + sw128_off4(t, i0)), kv);
+        unpack_bf4(*reinterpret_cast<const uint2 *>(vr + sl8 + sw128_off4(t, i0)), qv);
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          G[u] += gv[u];
+          e[u] = ex2f((G[u] - cr[u]) * kLog2e);
+          gm[u] = e[u] * Ec[u];
+          qv[u] *= a.tau;
+        }
+        *reinterpret_cast<float4 *>(pa + sw32_off(t, cc)) =
+            make_float4(tf32r(e[0] * kv[0]), tf32r(e[1] * kv[1]), tf32r(e[2] * kv[2]), tf32r(e[3] * kv[3]));
+        *reinterpret_cast<float4 *>(pa + sw32_off(64 + t, cc)) =
+            make_float4(tf32r(e[0] * qv[0]), tf32r(e[1] * qv[1]), tf32r(e[2] * qv[2]), tf32r(e[3] * qv[3]));
+        *reinterpret_cast<uint2 *>(pkb + sw128_off4(t, i0)) =
+            pack_h4(gm[0] * kv[0], gm[1] * kv[1], gm[2] * kv[2], gm[3] * kv[3]);
+        *reinterpret_cast<uint2 *>(pqh + sw128_off4(64 + t, i0)) =
+            pack_h4(gm[0] * qv[0], gm[1] * qv[1], gm[2] * qv[2], gm[3] * qv[3]);
+        if (SV)
+          *reinterpret_cast<float4 *>(reinterpret_cast<float *>(ctx + kCtxGa) + t * D + i0) =
+              make_float4(gm[0], gm[1], gm[2], gm[3]);
+      }
+      if (seg == 7) {
+        *reinterpret_cast<float4 *>(s_gC + i0) = make_float4(gm[0], gm[1], gm[2], gm[3]);
+        // the fused backward divides by the saved gamma: it needs gamma_C >= 1e-36
+        if (SV)
+          for (int u = 0; u < 4; ++u) check_gamma_range(gm[u], a.status);
+      }
+      load_r(c + 1);
+    } else if (wq >= 2 && c > 0 && a.o) {  // warps 14, 15: O of chunk c - 1 (rows 64..127 of TU)
+      const int t = 32 * (wq - 2) + lane, tt = (c - 1) * CM + t;
+      for (int j0 = 0; j0 < D; j0 += 16) {
+        float v[16];
+        tmem_ld16(TU + lane_base + j0, v);
+        if (tt < a.T) {
+          const size_t base = tok_index(a, b, tt, h) * D + j0;
+          if (a.odt == KDN_BF16) {
+            uint4 *dst = reinterpret_cast<uint4 *>(static_cast<__nv_bfloat16 *>(a.o) + base);
+            dst[0] = pack_bf8(v);
+            dst[1] = pack_bf8(v + 8);
+          } else {
+            float4 *dst = reinterpret_cast<float4 *>(static_cast<float *>(a.o) + base);
+#pragma unroll
+            for (int u = 0; u < 4; ++u) dst[u] = make_float4(v[4 * u], v[4 * u + 1], v[4 * u + 2], v[4 * u + 3]);
+          }
+        }
+      }
+    }
+    fence_proxy_async();
+    tc_fence_before();
+    ok = __syncthreads_and(p_ok);
+    if (!ok) break;
+
+    // ---- [2] MMA-T; the next chunk's k, g, omega; this chunk's V over q
+    if (issuer) {
+      tc_fence_after();
+      const uint32_t A0 = smem_u32(ta), B0 = smem_u32(tb);
+      for (int kk = 0; kk < 16; ++kk)
+        umma_tf32(TD1, sw128_desc(A0 + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024),
+                  sw128_desc(B0 + (kk >> 2) * 8192 + (kk & 3) * 32, 16, 1024), id_T, kk > 0);
+      umma_commit(bar_mma);
+      issue_v(c);
+      if (c + 1 < NC) {
+        issue_raw(c + 1);
+        for (int s = 0; s < 2; ++s) {
+          tma_prefetch_4d(&mq, 64 * s, h, (c + 1) * CM, b);
+          tma_prefetch_4d(&mv, 64 * s, h, (c + 1) * CM, b);
+        }
+      }
+    }
+    ok = __syncthreads_and(mma_wait_all());
+    if (!ok) break;
+    tc_fence_after();
+
+    // ---- [3] T' (with its diagonal) and A'_qk out of TMEM; S_in -> fp16; V -> fp16
+    {
+      const int s0 = 16 * wg;
+      float v[16];
+      tmem_ld16(TD1 + lane_base + s0, v);
+      if (wq < 2) {  // T' rows 0..63, lower triangle with the diagonal -> fp32 tile
+        const int t = 32 * wq + lane;
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          float4 o;
+          o.x = (s0 + 4 * u + 0 <= t) ? v[4 * u + 0] : 0.f;
+          o.y = (s0 + 4 * u + 1 <= t) ? v[4 * u + 1] : 0.f;
+          o.z = (s0 + 4 * u + 2 <= t) ? v[4 * u + 2] : 0.f;
+          o.w = (s0 + 4 * u + 3 <= t) ? v[4 * u + 3] : 0.f;
+          *reinterpret_cast<float4 *>(sT + t * LT + s0 + 4 * u) = o;
+        }
+      } else {  // A'_qk rows 64..127 (lower triangle) -> fp16
+        const int t = 32 * (wq - 2) + lane;
+#pragma unroll
+        for (int u = 0; u < 16; ++u) v[u] = (s0 + u <= t) ? v[u] : 0.f;
+        sm16(ao, chunk_off(64 + t, s0 >> 3)) = pack_h8(v);
+        sm16(ao, chunk_off(64 + t, (s0 >> 3) + 1)) = pack_h8(v + 8);
+      }
+    }
+    // zero rows 0..63 of [0; A'_qk] and rows 64..127 of [A; 0]
+    for (int e = tid; e < 1024; e += WT) {
+      unsigned char *base = e < 512 ? ao : awu + 8192;
+      const int ee = e & 511;
+      sm16(base, (uint32_t)(ee >> 3) * 128u + (uint32_t)((ee & 7) << 4)) = make_uint4(0, 0, 0, 0);
+    }
+    {  // S_in -> fp16 (MN-major B of MMA-S1); diag(gamma_C) S_in back to TMEM
+      const int i = 32 * wq + lane;
+      const float gC = s_gC[i];
+      for (int c0 = 0; c0 < 32; c0 += 16) {
+        float v[16];
+        const int j0 = 32 * wg + c0, sl = j0 >> 6, cc0 = (j0 & 63) >> 3;
+        tmem_ld16(TS + lane_base + j0, v);
+        sm16(s16, sl * 16384 + chunk_off(i, cc0)) = pack_h8(v);
+        sm16(s16, sl * 16384 + chunk_off(i, cc0 + 1)) = pack_h8(v + 8);
+#pragma unroll
+        for (int u = 0; u < 16; ++u) v[u] *= gC;
+        tmem_st16(TS + lane_base + j0, v);
+      }
+    }
+    bool v_ok = mbar_wait(bar_v, c & 1, kWait);
+    if (v_ok) {  // V -> fp16 in place (two 16-byte chunks per thread)
+      for (int e = tid; e < 1024; e += WT) {
+        const uint32_t off = (e >> 9) * 8192 + chunk_off((e >> 3) & 63, e & 7);
+        float v[8];
+        unpack_bf8(sm16(vr, off), v);
+        sm16(vr, off) = pack_h8(v);
+      }
+    }
+    tmem_st_wait();
+    fence_proxy_async();
+    ok = __syncthreads_and(v_ok);
+    if (!ok) break;
+    if (SV && issuer) {
+      bulk_s2g(ctx + kCtxS, s16, 32768);
+      bulk_commit();
+    }
+
+    // ---- [4] A = (I + T)^-1 = diag(s) L^-1 with L = diag(s) + strict_lower(T')
+    //          (T = strict_lower(T') diag(1/s)), then [A; 0] fp16
+    wy_inverse(sT, sA, sX, sY, s_r, s_s, s_is);
+    {
+      const int r = tid >> 3, cc = tid & 7;
+      const float sr = s_s[r];
+      const float4 a0 = *reinterpret_cast<const float4 *>(sA + r * LT + 8 * cc);
+      const float4 a1 = *reinterpret_cast<const float4 *>(sA + r * LT + 8 * cc + 4);
+      const float av[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
+      float v[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) v[j] = (8 * cc + j <= r) ? sr * av[j] : 0.f;
+      sm16(awu, chunk_off(r, cc)) = pack_h8(v);
+      if (SV) {  // A_qk = lower(A'_qk) diag(1/s) and s_t into the context
+        float q8[8];
+        unpack_h8(sm16(ao, chunk_off(64 + r, cc)), q8);
+        const float4 i0v = *reinterpret_cast<const float4 *>(s_is + 8 * cc);
+        const float4 i1v = *reinterpret_cast<const float4 *>(s_is + 8 * cc + 4);
+        const float is8[8] = {i0v.x, i0v.y, i0v.z, i0v.w, i1v.x, i1v.y, i1v.z, i1v.w};
+#pragma unroll
+        for (int j = 0; j < 8; ++j) q8[j] *= is8[j];
+        *reinterpret_cast<uint4 *>(ctx + kCtxAqk + chunk_off(r, cc)) = pack_h8(q8);
+        if (tid < CM) reinterpret_cast<float *>(ctx + kCtxTok)[tid] = s_s[tid];
+      }
+    }
+    fence_proxy_async();
+    tc_fence_before();
+    __syncthreads();
+
+    // ---- [5] MMA-W = A Kbar, MMA-U = A V (fp16)
+    if (issuer) {
+      if (SV) {
+        bulk_s2g(ctx + kCtxA, awu, 8192);
+        bulk_commit();
+      }
+      tc_fence_after();
+      const uint32_t AW = smem_u32(awu), KB = smem_u32(kb), VR = smem_u32(vr);
+      for (int kk = 0; kk < 4; ++kk) {
+        const uint64_t ad = sw128_desc(AW + kk * 32, 16, 1024);
+        umma_bf16(TW, ad, sw128_desc(KB + kk * 2048, 8192, 1024), id_16, kk > 0);
+        umma_bf16(TU, ad, sw128_desc(VR + kk * 2048, 8192, 1024), id_16, kk > 0);
+      }
+      umma_commit(bar_mma);
+    }
+    ok = __syncthreads_and(mma_wait_all());
+    if (!ok) break;
+    tc_fence_after();
+
+    // ---- [6] -W -> fp16 rows 0..63 of [-W; Qbar]
+    if (wq < 2) {
+      const int t = 32 * wq + lane;
+      for (int c0 = 0; c0 < 32; c0 += 16) {
+        float v[16];
+        const int j0 = 32 * wg + c0, sl = j0 >> 6, cc0 = (j0 & 63) >> 3;
+        tmem_ld16(TW + lane_base + j0, v);
+#pragma unroll
+        for (int u = 0; u < 16; ++u) v[u] = -v[u];
+        sm16(as1, sl * 16384 + chunk_off(t, cc0)) = pack_h8(v);
+        sm16(as1, sl * 16384 + chunk_off(t, cc0 + 1)) = pack_h8(v + 8);
+      }
+    }
+    fence_proxy_async();
+    tc_fence_before();
+    __syncthreads();
+
+    // ---- [7] MMA-S1: [U; 0] += [-W; Qbar] S_in  (fp16)
+    if (issuer) {
+      if (SV) {
+        bulk_s2g(ctx + kCtxW, as1, 8192);
+        bulk_s2g(ctx + kCtxW + 8192, as1 + 16384, 8192);
+        bulk_commit();
+      }
+      tc_fence_after();
+      const uint32_t A1 = smem_u32(as1), B1 = smem_u32(s16);
+      for (int kk = 0; kk < 8; ++kk)
+        umma_bf16(TU, sw128_desc(A1 + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024),
+                  sw128_desc(B1 + kk * 2048, 16384, 1024), id_16, 1);
+      umma_commit(bar_mma);
+    }
+    ok = __syncthreads_and(mma_wait_all());
+    if (!ok) break;
+    tc_fence_after();
+
+    // ---- [8] R' = diag(1/s) R -> fp16 [t][j] (MN-major B), over V
+    if (wq < 2) {
+      const int t = 32 * wq + lane;
+      const float ist = s_is[t];
+      for (int c0 = 0; c0 < 32; c0 += 16) {
+        float v[16];
+        const int j0 = 32 * wg + c0, sl = j0 >> 6, cc0 = (j0 & 63) >> 3;
+        tmem_ld16(TU + lane_base + j0, v);
+        if (SV) {
+          *reinterpret_cast<uint4 *>(ctx + kCtxR + sl * 8192 + chunk_off(t, cc0)) = pack_h8(v);
+          *reinterpret_cast<uint4 *>(ctx + kCtxR + sl * 8192 + chunk_off(t, cc0 + 1)) = pack_h8(v + 8);
+        }
+#pragma unroll
+        for (int u = 0; u < 16; ++u) v[u] *= ist;
+        sm16(vr, sl * 8192 + chunk_off(t, cc0)) = pack_h8(v);
+        sm16(vr, sl * 8192 + chunk_off(t, cc0 + 1)) = pack_h8(v + 8);
+      }
+    }
+    fence_proxy_async();
+    tc_fence_before();
+    __syncthreads();
+
+    // ---- [9] MMA-O (rows 64..127 of TU += A'_qk R') and MMA-S2 (S += K'^T R')
+    if (issuer) {
+      tc_fence_after();
+      const uint32_t AO = smem_u32(ao), VR = smem_u32(vr);
+      for (int kk = 0; kk < 4; ++kk) {
+        const uint64_t bd = sw128_desc(VR + kk * 2048, 8192, 1024);
+        umma_bf16(TU, sw128_desc(AO + kk * 32, 16, 1024), bd, id_16, 1);
+        umma_f16_tA(TS, tkt + (uint32_t)(kk * 8), bd, id_16, 1);
+      }
+      umma_commit(bar_mma);
+    }
+  }
+
+  if (ok && NC > 0) {
+    ok = mma_wait_all();  // MMA-O / MMA-S2 of the last chunk
+    ok = __syncthreads_and(ok);
+    tc_fence_after();
+  }
+  if (ok) {
+    if (wq >= 2 && NC > 0 && a.o) {  // O of the last chunk
+      const int c = NC - 1, t = 32 * (wq - 2) + lane, tt = c * CM + t;
+      for (int c0 = 0; c0 < 32; c0 += 16) {
+        float v[16];
+        const int j0 = 32 * wg + c0;
+        tmem_ld16(TU + lane_base + j0, v);
+        if (tt < a.T) {
+          const size_t base = tok_index(a, b, tt, h) * D + j0;
+          if (a.odt == KDN_BF16) {
+            uint4 *dst = reinterpret_cast<uint4 *>(static_cast<__nv_bfloat16 *>(a.o) + base);
+            dst[0] = pack_bf8(v);
+            dst[1] = pack_bf8(v + 8);
+          } else {
+            float4 *dst = reinterpret_cast<float4 *>(static_cast<float *>(a.o) + base);
+#pragma unroll
+            for (int u = 0; u < 4; ++u) dst[u] = make_float4(v[4 * u], v[4 * u + 1], v[4 * u + 2], v[4 * u + 3]);
+          }
+        }
+      }
+    }
+    if (a.ST) {
+      const int i = 32 * wq + lane;
+      for (int c0 = 0; c0 < 32; c0 += 16) {
+        float v[16];
+        const int j0 = 32 * wg + c0;
+        tmem_ld16(TS + lane_base + j0, v);
+        float4 *dst = reinterpret_cast<float4 *>(a.ST + ((size_t)bh * D + i) * D + j0);
+#pragma unroll
+        for (int u = 0; u < 4; ++u) dst[u] = make_float4(v[4 * u], v[4 * u + 1], v[4 * u + 2], v[4 * u + 3]);
+      }
+    }
+    if (a.pT && gain) a.pT[(size_t)bh * D + tid] = p;
+  } else {
+    if (tid == 0) atomicExch(a.status, (unsigned)KDN_ERR_TIMEOUT);
+    // copies and MMAs in flight land before the CTA's memory goes away
+    if (issuer) {
+      mbar_wait(bar_raw, 0, kWait);
+      mbar_wait(bar_raw, 1, kWait);
+      mbar_wait(bar_v, 0, kWait);
+      mbar_wait(bar_v, 1, kWait);
+      mbar_wait(bar_q, 0, kWait);
+      mbar_wait(bar_q, 1, kWait);
+      mbar_wait(bar_mma, 0, kWait);
+      mbar_wait(bar_mma, 1, kWait);
+    }
+  }
+  if (SV && issuer) bulk_wait_all();
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) tmem_dealloc(tbase, 512);
+}
+
+}  // namespace
+
+bool wy_fwd_supported(const Args &a) {
+  return a.variant == 0 && a.gates == KDN_GATES_POST && a.dtype == KDN_BF16 && a.dk == D &&
+         a.dv == D && a.T > 0 && a.chunk != 32;
+}
+
+kdn_status_t launch_wy_fwd(const Args &a, cudaStream_t s, unsigned char *save_S, float *save_p) {
+  if (!wy_fwd_supported(a) || (!save_S) != (!save_p)) return KDN_ERR_UNSUPPORTED;
+  WyParams P;
+  P.a = a;
+  P.save_S = save_S;
+  P.save_p = save_p;
+  CUtensorMap mk, mg, mw, mv, mq;
+  if (!make_map(&mk, a.k, a) || !make_map(&mg, a.g, a) || !make_map(&mw, a.omega, a) ||
+      !make_map(&mv, a.v, a) || !make_map(&mq, a.q, a))
+    return KDN_ERR_CUDA;
+  const auto kern = save_S ? k_wy_fwd<1> : k_wy_fwd<0>;
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES) !=
+      cudaSuccess)
+    return KDN_ERR_CUDA;
+  kern<<<a.B * a.H, WT, SMEM_BYTES, s>>>(mk, mg, mw, mv, mq, P);
+  return cudaGetLastError() == cudaSuccess ? KDN_OK : KDN_ERR_CUDA;
+}
+
+}  // namespace kdn

@@ -410,9 +410,14 @@ def test_training_pair_matches_recompute_path(kdn):
 
 @pytest.mark.parametrize("variant", ["diag", "iso"])
 def test_fused_decay_range_is_reported(kdn, variant):
-    """alpha = e^-2 for 64 tokens puts exp(G_C) at e^-128, below the fused kernels'
-    range: the call records KDN_ERR_RANGE in the workspace status word (no fault);
-    the general kernels (32-token chunks, exp(G_C) >= e^-64) match the oracle."""
+    """A decay outside a fused kernel's range is reported in the workspace status
+    word (no fault), and the general kernels (32-token chunks) still match the
+    oracle.  alpha = e^-2 for 64 tokens puts exp(G_C) at e^-128: below the range
+    of the fused backward (and of the isotropic forward), which divide by
+    gamma, but inside that of the Diagonal forward, whose decay factors are
+    referenced at the middle of the chunk's range (exp(+-64)): there it must
+    match the oracle with KDN_OK.  alpha = e^-3 (exp(G_C) = e^-192) leaves the
+    Diagonal forward's range too."""
     ins = make_inputs(variant, 1, 100, 2, 128, 128, dtype="bf16", seed=3, with_grad=True)
     ins["g"][...] = -2.0
     d = to_dev(ins)
@@ -421,9 +426,16 @@ def test_fused_decay_range_is_reported(kdn, variant):
     desc = kdn.make_desc(1, 100, 2, 128, 128, torch.bfloat16,
                          decay_per_channel=int(d["g"].dim() == 4))
     ws = kdn.alloc_workspace(desc, 0 if variant == "diag" else 1, True)
-    fwd(*x, workspace=ws)
+    ref = _oracle_fwd(variant, ins)
+    o, _, _ = fwd(*x, workspace=ws)
+    if variant == "diag":
+        assert kdn.kdn_get_device_status(ws) == kdn.KDN_OK
+        check("o", o, ref["o"], "bf16")
+        x3 = [t.clone() for t in x]
+        x3[3].fill_(-3.0)
+        fwd(*x3, workspace=ws)
     assert kdn.kdn_get_device_status(ws) == kdn.KDN_ERR_RANGE
-    fwd(*x, workspace=ws)  # the word is cleared by the query and set again by the call
+    fwd(*(x3 if variant == "diag" else x), workspace=ws)  # cleared by the query, set again
     assert kdn.kdn_get_device_status(ws) == kdn.KDN_ERR_RANGE
     bwd = kdn.kdn_diag_bwd if variant == "diag" else kdn.kdn_iso_bwd
     bwd(*x, None, None, d["dO"], workspace=ws)
@@ -434,7 +446,6 @@ def test_fused_decay_range_is_reported(kdn, variant):
     o, ST, pT = fwd(*x, chunk=32, workspace=ws32)
     torch.cuda.synchronize()
     assert kdn.kdn_get_device_status(ws32) == kdn.KDN_OK
-    ref = _oracle_fwd(variant, ins)
     check("o", o, ref["o"], "bf16")
 
 
