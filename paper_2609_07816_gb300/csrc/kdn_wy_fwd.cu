@@ -61,8 +61,9 @@ constexpr int D = 128;   // d_k = d_v
 constexpr uint32_t kWait = 1u << 25;
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kMinHalfG = -80.f;  // c = G_C / 2 below this: out of range
-constexpr int kPrepThreads = 256;   // warps 4-11
-constexpr int kNamed = 128 + kPrepThreads;  // gain + prepare threads at named barrier 1
+constexpr int kPrepThreads = 256;   // warps 4-11: the preparing pass
+constexpr int kMain = 384;          // warps 4-15: everything but the gain
+constexpr int kBarPrep = 1, kBarMain = 2, kBarGain = 3;  // named barriers (0 = __syncthreads)
 
 // shared-memory map (bytes from the 1024-aligned base)
 constexpr int LT = 68;          // row stride (floats) of the fp32 T and A tiles
@@ -81,14 +82,13 @@ constexpr int O_S16 = O_TA;                      // fp16 S_in [128 i][128 j], tw
 constexpr int O_SWT = O_TA + 32768;              // fp32 T' [64][LT]
 constexpr int O_SWA = O_SWT + 64 * LT * 4;       // fp32 L^-1 [64][LT]
 static_assert(O_SWA + 64 * LT * 4 <= O_TB, "T and A tiles overlap the Kk' tile");
-constexpr int O_AWU = O_TB;            // fp16 [A; 0] [128][64] (MMA-W/U A)
-constexpr int O_AO = O_TB + 16384;     // fp16 [0; A'_qk] [128][64] (MMA-O A)
+constexpr int O_AWU = O_SWT;           // fp16 [A; 0] [128][64] (MMA-W/U A), over T' after the solve
 // inverse scratch in rows 0..63 of the first slab of [-W; Qbar] (written after it)
 constexpr int O_SX = O_AS1;            // 2 x 256 floats
 constexpr int O_SY = O_AS1 + 2048;     // 32 x 32 floats
-// small arrays (floats)
-constexpr int SM_R = 0, SM_MUR = 64, SM_S = 128, SM_IS = 192, SM_C = 256, SM_GC = 384,
-              SM_PART = 512, SM_FLOATS = 512 + 8 * 128;
+// small arrays (floats); r and mu / r per token for two chunks (the gain works one chunk ahead)
+constexpr int SM_R = 0, SM_MUR = 128, SM_S = 256, SM_IS = 320, SM_C = 384, SM_GC = 512,
+              SM_PART = 640, SM_FLOATS = 640 + 8 * 128;
 constexpr int O_BAR = O_SMALL + SM_FLOATS * 4;
 constexpr int SMEM_BYTES = O_BAR + 64 + 1024;
 
@@ -115,9 +115,6 @@ __device__ __forceinline__ float tf32r(float x) {
 // elements per row
 __device__ __forceinline__ uint32_t sw32_off(uint32_t row, uint32_t col) {
   return row * 128u + ((((col >> 2) ^ (row & 7u)) << 4) | ((col & 3u) << 2));
-}
-__device__ __forceinline__ void bar_arrive(int id, int n) {
-  asm volatile("bar.arrive %0, %1;" ::"r"(id), "r"(n) : "memory");
 }
 __device__ __forceinline__ void bar_sync(int id, int n) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory");
@@ -176,11 +173,10 @@ __device__ __forceinline__ uint32_t sw128_off4(uint32_t t, uint32_t i0) {
 //   X_10 = -D_1 L_10 D_0,  X_32 = -D_3 L_32 D_2,
 // and the lower-left quarter X_21 = -X22 L21 X11 (X11, X22 the 32 x 32
 // diagonal halves), each output thread forming four adjacent columns from
-// 16-byte loads.  s_t and 1 / s_t go to s_s, s_is.  Every thread of the CTA
-// calls it (block barriers inside).
-__device__ __forceinline__ void wy_inverse(const float *sT, float *sA, float *sX, float *sY,
+// 16-byte loads.  s_t and 1 / s_t go to s_s, s_is.  Called by the kMain
+// threads tid = 0 .. kMain - 1 of warps 4-15 (named-barrier synchronisation).
+__device__ __forceinline__ void wy_inverse(int tid, const float *sT, float *sA, float *sX, float *sY,
                                            const float *s_r, float *s_s, float *s_is) {
-  const int tid = threadIdx.x;
   if (tid < 64) {
     // column c of D_I: x_r = (delta_rc - sum_{m<r} L_rm x_m) / L_rr, rows read 16 bytes at a time
     const int o = 16 * (tid >> 4), c = tid & 15;
@@ -211,14 +207,16 @@ __device__ __forceinline__ void wy_inverse(const float *sT, float *sA, float *sX
     float *ab = sA + o * (LT + 1) + c;
 #pragma unroll
     for (int r = 0; r < 16; ++r) ab[r * LT] = x[r];
-  } else if (tid < 64 + 384) {
+  } else {
     // zero the strictly upper 16 x 16 blocks (I < J): 6 blocks x 16 rows x 4 float4
-    const int e = tid - 64, blk = e >> 6, rr = (e >> 2) & 15, q4 = e & 3;
-    const int I = blk < 3 ? 0 : (blk < 5 ? 1 : 2);
-    const int J = blk < 3 ? blk + 1 : (blk < 5 ? blk - 1 : 3);
-    *reinterpret_cast<float4 *>(sA + (16 * I + rr) * LT + 16 * J + 4 * q4) = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int e = tid - 64; e < 384; e += kMain - 64) {
+      const int blk = e >> 6, rr = (e >> 2) & 15, q4 = e & 3;
+      const int I = blk < 3 ? 0 : (blk < 5 ? 1 : 2);
+      const int J = blk < 3 ? blk + 1 : (blk < 5 ? blk - 1 : 3);
+      *reinterpret_cast<float4 *>(sA + (16 * I + rr) * LT + 16 * J + 4 * q4) = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
   }
-  __syncthreads();
+  bar_sync(kBarMain, kMain);
   // X_10, X_32: one thread per (block, row, 4 columns)
   const int blk = tid >> 6, r2 = (tid >> 2) & 15, cq2 = 4 * (tid & 3);
   const int C0 = 32 * blk, R0 = C0 + 16;
@@ -240,7 +238,7 @@ __device__ __forceinline__ void wy_inverse(const float *sT, float *sA, float *sX
     }
     *reinterpret_cast<float4 *>(sX + blk * 256 + r2 * 16 + cq2) = acc;
   }
-  __syncthreads();
+  bar_sync(kBarMain, kMain);
   if (tid < 128) {
     const float *dp = sA + (R0 + r2) * LT + R0;
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
@@ -259,7 +257,7 @@ __device__ __forceinline__ void wy_inverse(const float *sT, float *sA, float *sX
     }
     *reinterpret_cast<float4 *>(sA + (R0 + r2) * LT + C0 + cq2) = make_float4(-acc.x, -acc.y, -acc.z, -acc.w);
   }
-  __syncthreads();
+  bar_sync(kBarMain, kMain);
   // Y = L21 X11, then X_21 = -X22 Y (32 x 32 x 32 each): one thread per (row, 4 columns)
   const int r3 = tid >> 3, cq3 = 4 * (tid & 7);
   if (tid < 256) {
@@ -280,7 +278,7 @@ __device__ __forceinline__ void wy_inverse(const float *sT, float *sA, float *sX
     }
     *reinterpret_cast<float4 *>(sY + r3 * 32 + cq3) = acc;
   }
-  __syncthreads();
+  bar_sync(kBarMain, kMain);
   if (tid < 256) {
     const float *dp = sA + (32 + r3) * LT + 32;
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
@@ -299,7 +297,7 @@ __device__ __forceinline__ void wy_inverse(const float *sT, float *sA, float *sX
     }
     *reinterpret_cast<float4 *>(sA + (32 + r3) * LT + cq3) = make_float4(-acc.x, -acc.y, -acc.z, -acc.w);
   }
-  __syncthreads();
+  bar_sync(kBarMain, kMain);
 }
 
 struct WyParams {
@@ -325,7 +323,7 @@ __global__ void __launch_bounds__(WT, 1)
       reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(smraw) + 1023) & ~uintptr_t(1023));
   unsigned char *rk = sm + O_RK, *rg = sm + O_RG, *rw = sm + O_RW, *vr = sm + O_V;
   unsigned char *ta = sm + O_TA, *tb = sm + O_TB, *kb = sm + O_KB, *as1 = sm + O_AS1;
-  unsigned char *s16 = sm + O_S16, *awu = sm + O_AWU, *ao = sm + O_AO;
+  unsigned char *s16 = sm + O_S16, *awu = sm + O_AWU;
   float *sT = reinterpret_cast<float *>(sm + O_SWT), *sA = reinterpret_cast<float *>(sm + O_SWA);
   float *sX = reinterpret_cast<float *>(sm + O_SX), *sY = reinterpret_cast<float *>(sm + O_SY);
   float *sf = reinterpret_cast<float *>(sm + O_SMALL);
@@ -333,7 +331,8 @@ __global__ void __launch_bounds__(WT, 1)
   float *s_c = sf + SM_C, *s_gC = sf + SM_GC, *s_part = sf + SM_PART;
   uint64_t *bars = reinterpret_cast<uint64_t *>(sm + O_BAR);
   uint64_t *bar_raw = bars, *bar_v = bars + 1, *bar_mma = bars + 2, *bar_q = bars + 3;
-  uint32_t *s_tbase = reinterpret_cast<uint32_t *>(bars + 4);
+  uint64_t *bar_t = bars + 4;  // MMA-T completions (one a chunk)
+  uint32_t *s_tbase = reinterpret_cast<uint32_t *>(bars + 5);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int wq = warp & 3, wg = warp >> 2;  // TMEM lane quarter, column group
@@ -347,6 +346,7 @@ __global__ void __launch_bounds__(WT, 1)
     mbar_init(bar_v, 1);
     mbar_init(bar_mma, 1);
     mbar_init(bar_q, 1);
+    mbar_init(bar_t, 1);
     fence_mbar_init();
     prefetch_tmap(&mk);
     prefetch_tmap(&mg);
@@ -411,24 +411,26 @@ __global__ void __launch_bounds__(WT, 1)
     tmem_st_wait();
   }
 
-  // roles in the first phase of a chunk
+  // roles: warps 0-3 run the gain one chunk ahead; warps 4-15 (the main warps)
+  // prepare the operands (warps 4-11), store o (warps 14, 15), and run every
+  // tensor-core and solve stage, synchronised among themselves by named barriers
   const bool gain = tid < 128;
   const bool prep = tid >= 128 && tid < 128 + kPrepThreads;
-  const int pi = tid - 128;  // preparing thread: channels 4 (pi % 32) .. +3, tokens 8 (pi / 32) .. +7
-  float p = 1.f;             // gain threads: uncertainty carry of channel tid
+  const int mt = tid - 128;           // main thread 0 .. kMain - 1
+  const int wgm = (warp >> 2) - 1;    // main warps: 0, 1, 2 within a lane quarter
+  float p = 1.f;                      // gain threads: uncertainty carry of channel tid
   if (gain && a.p0) p = a.p0[(size_t)bh * D + tid];
-  float nr = 1.f;            // preparing threads pi < 64: r of token pi of the next chunk
+  float rnext = 1.f;                  // gain threads tid < 64: r of the next chunk's token tid
   auto load_r = [&](int c) {
-    if (pi >= 0 && pi < CM) {
-      nr = 1.f;
-      if (c < NC && c * CM + pi < a.T) nr = ld<__nv_bfloat16>(a.r, tok_index(a, b, c * CM + pi, h));
+    if (tid < CM) {
+      rnext = 1.f;
+      if (c < NC && c * CM + tid < a.T) rnext = ld<__nv_bfloat16>(a.r, tok_index(a, b, c * CM + tid, h));
     }
   };
   load_r(0);
 
-  uint32_t mph = 0;  // MMA-completion phases observed
-  bool ok = true;
-  auto mma_wait_all = [&]() -> bool {
+  uint32_t mph = 0;  // main threads: completions of bar_mma observed (three per chunk)
+  auto mma_wait_main = [&]() -> bool {
     const bool r = mbar_wait(bar_mma, mph & 1, kWait);
     ++mph;
     return r;
@@ -436,114 +438,135 @@ __global__ void __launch_bounds__(WT, 1)
   const uint32_t id_T = idesc_tf32(128, 64);
   const uint32_t id_16 = idesc_f16(128, 128, 0, 1);  // A K-major, B MN-major
 
-  for (int c = 0; c < NC && ok; ++c) {
+  // ---- the gain of chunk c (warps 0-3): r and mu / r of its tokens into buffer
+  //      c & 1, the recursion over its 64 tokens.  Its Kk' tile may be written
+  //      once MMA-T of chunk c - 1 has read the previous one.
+  auto gain_chunk = [&](int c) -> bool {
+    const int i = tid, sb = c & 1;
+    float *sr = s_r + 64 * sb, *smur = s_mur + 64 * sb;
+    if (tid < CM) {
+      sr[tid] = rnext;
+      smur[tid] = a.mu / rnext;
+    }
+    load_r(c + 1);
+    bar_sync(kBarGain, 128);
+    bool g_ok = mbar_wait(bar_raw, c & 1, kWait);
+    const unsigned char *pg = rg + (i >> 6) * 8192, *pw = rw + (i >> 6) * 8192, *pk = rk + (i >> 6) * 8192;
+    const int cl = i & 63;
+    // element (t, i) of a raw slab: row t, 128-byte swizzle
+    auto raw = [&](const unsigned char *base, int t) {
+      return __bfloat162float(*reinterpret_cast<const __nv_bfloat16 *>(base + sw128_off(t, cl)));
+    };
+    float g0 = 0.f, g1 = 0.f, g2 = 0.f, g3 = 0.f;
+#pragma unroll
+    for (int t = 0; t < CM; t += 4) {
+      g0 += raw(pg, t);
+      g1 += raw(pg, t + 1);
+      g2 += raw(pg, t + 2);
+      g3 += raw(pg, t + 3);
+    }
+    const float GC = (g0 + g1) + (g2 + g3), cref = 0.5f * GC;
+    s_c[i] = cref;
+    if (cref < kMinHalfG) atomicCAS(a.status, 0u, (unsigned)KDN_ERR_RANGE);
+    unsigned char *gctx = SV ? P.save_S + ((size_t)bh * NC + c) * kCtxBytes : nullptr;
+    if (SV) P.save_p[((size_t)bh * NC + c) * D + i] = p;
+    float *cph = SV ? reinterpret_cast<float *>(gctx + kCtxPh) + i : nullptr;
+    float f = ex2f(cref * kLog2e);                // exp(c - G_t), G_{-1} = 0
+    const float E2 = ex2f((GC - cref) * kLog2e);  // exp(G_C - c)
+    unsigned char *pb = tb + (i >> 5) * 8192;
+    const int cb = i & 31;
+    const uint32_t tkt = TKT + (uint32_t)((c & 1) * 32);
+    float gb[8], wb[8], kb8[8], mb[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      gb[j] = raw(pg, j);
+      wb[j] = raw(pw, j);
+      kb8[j] = raw(pk, j);
+    }
+    {
+      const float4 m0 = *reinterpret_cast<const float4 *>(smur), m1 = *reinterpret_cast<const float4 *>(smur + 4);
+      mb[0] = m0.x; mb[1] = m0.y; mb[2] = m0.z; mb[3] = m0.w; mb[4] = m1.x; mb[5] = m1.y; mb[6] = m1.z; mb[7] = m1.w;
+    }
+    if (c > 0) g_ok = mbar_wait(bar_t, (c - 1) & 1, kWait) && g_ok;  // Kk' of chunk c - 1 has been read
+    // the chunk in blocks of 8 tokens; the next block's inputs are loaded
+    // before the current block's outputs are stored
+#pragma unroll
+    for (int blk = 0; blk < 8; ++blk) {
+      float gn[8], wn[8], kn[8], mn[8];
+      if (blk < 7) {
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const int t = 8 * (blk + 1) + j;
+          gn[j] = raw(pg, t);
+          wn[j] = raw(pw, t);
+          kn[j] = raw(pk, t);
+        }
+        const float4 m0 = *reinterpret_cast<const float4 *>(smur + 8 * (blk + 1));
+        const float4 m1 = *reinterpret_cast<const float4 *>(smur + 8 * (blk + 1) + 4);
+        mn[0] = m0.x; mn[1] = m0.y; mn[2] = m0.z; mn[3] = m0.w; mn[4] = m1.x; mn[5] = m1.y; mn[6] = m1.z; mn[7] = m1.w;
+      }
+      uint32_t kt[4];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const int t = 8 * blk + j;
+        const float al = ex2f(gb[j] * kLog2e), a2 = al * al;
+        const float ph = fmaf(a2, p, wb[j]);               // eq. diag-covariance-prediction
+        const float u = kb8[j] * kb8[j] * mb[j];
+        const float den = fmaf(u, ph, 1.f);
+        const float x = rcpf(al * den);
+        p = ph * (x * al);                                  // eq. prefix-diag-uncertainty
+        f *= x * den;                                       // / alpha_t
+        const float pkv = ph * kb8[j];
+        if (SV) cph[t * D] = ph;
+        *reinterpret_cast<float *>(pb + sw32_off(t, cb)) = tf32r(pkv * f);
+        const uint32_t hb = (uint32_t)__half_as_ushort(__float2half_rn(pkv * (f * E2)));
+        if ((j & 1) == 0) kt[j >> 1] = hb;
+        else kt[j >> 1] |= hb << 16;
+      }
+      tmem_st4u(tkt + lane_base + (uint32_t)(4 * blk), kt);
+      if (blk < 7) {
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          gb[j] = gn[j];
+          wb[j] = wn[j];
+          kb8[j] = kn[j];
+          mb[j] = mn[j];
+        }
+      }
+    }
+    tmem_st_wait();
+    fence_proxy_async();
+    return g_ok;
+  };
+
+  bool mine = true;    // this thread's waits so far; combined at the CTA-wide barriers
+  bool failed = false;
+  if (gain && NC > 0) mine = gain_chunk(0);
+
+  for (int c = 0; c < NC; ++c) {
     const uint32_t tkt = TKT + (uint32_t)((c & 1) * 32);
     unsigned char *ctx = SV ? P.save_S + ((size_t)bh * NC + c) * kCtxBytes : nullptr;
     if (SV && issuer) bulk_wait_read();  // the previous chunk's context tiles have left shared memory
-    // ---- [0] per-token scalars; the previous chunk's MMA-O / MMA-S2 must be done
-    //          before q is brought into its R' buffer
-    if (pi >= 0 && pi < CM) {
-      s_r[pi] = nr;
-      s_mur[pi] = a.mu / nr;
-    }
-    bool w_ok = mbar_wait(bar_raw, c & 1, kWait);
+    // ---- [0] the previous chunk's MMA-O / MMA-S2 must be done before q is brought
+    //          into its R' buffer; the gain of this chunk is done (its warps arrive here)
+    if (!gain) mine = mbar_wait(bar_raw, c & 1, kWait) && mine;
     if (issuer && c > 0) {
-      w_ok = w_ok && mma_wait_all();  // MMA-O / MMA-S2 of chunk c - 1
-      if (w_ok) issue_q(c);
-    } else if (c > 0) {
+      mine = mma_wait_main() && mine;  // MMA-O / MMA-S2 of chunk c - 1
+      if (mine) issue_q(c);
+    } else if (!gain && c > 0) {
       ++mph;
     }
-    ok = __syncthreads_and(w_ok);
-    if (!ok) break;
+    tc_fence_before();
+    if (!__syncthreads_and(mine)) {
+      failed = true;
+      break;
+    }
+    tc_fence_after();
 
-    // ---- [1] gain (warps 0-3), operand preparation (warps 4-11) and the
-    //          previous chunk's output (warps 14, 15)
-    bool p_ok = true;
-    if (gain) {
-      const int i = tid;
-      const unsigned char *pg = rg + (i >> 6) * 8192, *pw = rw + (i >> 6) * 8192, *pk = rk + (i >> 6) * 8192;
-      const int cl = i & 63;
-      // element (t, i) of a raw slab: row t, 128-byte swizzle
-      auto raw = [&](const unsigned char *base, int t) {
-        return __bfloat162float(*reinterpret_cast<const __nv_bfloat16 *>(base + sw128_off(t, cl)));
-      };
-      float g0 = 0.f, g1 = 0.f, g2 = 0.f, g3 = 0.f;
-#pragma unroll
-      for (int t = 0; t < CM; t += 4) {
-        g0 += raw(pg, t);
-        g1 += raw(pg, t + 1);
-        g2 += raw(pg, t + 2);
-        g3 += raw(pg, t + 3);
-      }
-      const float GC = (g0 + g1) + (g2 + g3), cref = 0.5f * GC;
-      s_c[i] = cref;
-      if (cref < kMinHalfG) atomicCAS(a.status, 0u, (unsigned)KDN_ERR_RANGE);
-      bar_arrive(1, kNamed);
-      if (SV) P.save_p[((size_t)bh * NC + c) * D + i] = p;
-      float *cph = SV ? reinterpret_cast<float *>(ctx + kCtxPh) + i : nullptr;
-      float f = ex2f(cref * kLog2e);                // exp(c - G_t), G_{-1} = 0
-      const float E2 = ex2f((GC - cref) * kLog2e);  // exp(G_C - c)
-      unsigned char *pb = tb + (i >> 5) * 8192;
-      const int cb = i & 31;
-      // the chunk in blocks of 8 tokens; the next block's inputs are loaded
-      // before the current block's outputs are stored
-      float gb[8], wb[8], kb8[8], mb[8];
-#pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        gb[j] = raw(pg, j);
-        wb[j] = raw(pw, j);
-        kb8[j] = raw(pk, j);
-      }
-      {
-        const float4 m0 = *reinterpret_cast<const float4 *>(s_mur), m1 = *reinterpret_cast<const float4 *>(s_mur + 4);
-        mb[0] = m0.x; mb[1] = m0.y; mb[2] = m0.z; mb[3] = m0.w; mb[4] = m1.x; mb[5] = m1.y; mb[6] = m1.z; mb[7] = m1.w;
-      }
-#pragma unroll
-      for (int blk = 0; blk < 8; ++blk) {
-        float gn[8], wn[8], kn[8], mn[8];
-        if (blk < 7) {
-#pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            const int t = 8 * (blk + 1) + j;
-            gn[j] = raw(pg, t);
-            wn[j] = raw(pw, t);
-            kn[j] = raw(pk, t);
-          }
-          const float4 m0 = *reinterpret_cast<const float4 *>(s_mur + 8 * (blk + 1));
-          const float4 m1 = *reinterpret_cast<const float4 *>(s_mur + 8 * (blk + 1) + 4);
-          mn[0] = m0.x; mn[1] = m0.y; mn[2] = m0.z; mn[3] = m0.w; mn[4] = m1.x; mn[5] = m1.y; mn[6] = m1.z; mn[7] = m1.w;
-        }
-        uint32_t kt[4];
-#pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          const int t = 8 * blk + j;
-          const float al = ex2f(gb[j] * kLog2e), a2 = al * al;
-          const float ph = fmaf(a2, p, wb[j]);               // eq. diag-covariance-prediction
-          const float u = kb8[j] * kb8[j] * mb[j];
-          const float den = fmaf(u, ph, 1.f);
-          const float x = rcpf(al * den);
-          p = ph * (x * al);                                  // eq. prefix-diag-uncertainty
-          f *= x * den;                                       // / alpha_t
-          const float pkv = ph * kb8[j];
-          if (SV) cph[t * D] = ph;
-          *reinterpret_cast<float *>(pb + sw32_off(t, cb)) = tf32r(pkv * f);
-          const uint32_t hb = (uint32_t)__half_as_ushort(__float2half_rn(pkv * (f * E2)));
-          if ((j & 1) == 0) kt[j >> 1] = hb;
-          else kt[j >> 1] |= hb << 16;
-        }
-        tmem_st4u(tkt + lane_base + (uint32_t)(4 * blk), kt);
-        if (blk < 7) {
-#pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            gb[j] = gn[j];
-            wb[j] = wn[j];
-            kb8[j] = kn[j];
-            mb[j] = mn[j];
-          }
-        }
-      }
-      tmem_st_wait();
-    } else if (prep) {
+    // ---- [1] operand preparation (warps 4-11) and the previous chunk's output
+    //          (warps 14, 15); the gain of this chunk is already done
+    if (prep) {
+      const int pi = mt;
       const int i0 = 4 * (pi & 31), seg = pi >> 5, t0 = 8 * seg;
       const uint32_t sl8 = (uint32_t)(i0 >> 6) * 8192u;  // 64-channel slab of a [t][64] 16-bit tile
       // the chunk's g for this thread's 8 tokens and 4 channels (8 bytes a token)
@@ -558,7 +581,7 @@ __global__ void __launch_bounds__(WT, 1)
         for (int u = 0; u < 4; ++u) ps[u] += gv[u];
       }
       *reinterpret_cast<float4 *>(s_part + seg * D + i0) = make_float4(ps[0], ps[1], ps[2], ps[3]);
-      bar_sync(1, kNamed);
+      bar_sync(kBarPrep, kPrepThreads);
       float cr[4], G[4] = {0.f, 0.f, 0.f, 0.f}, Ec[4], gm[4];
       {
         const float4 c4 = *reinterpret_cast<const float4 *>(s_c + i0);
@@ -570,7 +593,7 @@ __global__ void __launch_bounds__(WT, 1)
       }
 #pragma unroll
       for (int u = 0; u < 4; ++u) Ec[u] = ex2f(cr[u] * kLog2e);
-      p_ok = mbar_wait(bar_q, c & 1, kWait);
+      mine = mbar_wait(bar_q, c & 1, kWait) && mine;
       unsigned char *pa = ta + (i0 >> 5) * 16384, *pkb = kb + sl8, *pqh = as1 + (i0 >> 6) * 16384;
       const int cc = i0 & 31;
 #pragma unroll
@@ -605,8 +628,7 @@ __global__ void __launch_bounds__(WT, 1)
         if (SV)
           for (int u = 0; u < 4; ++u) check_gamma_range(gm[u], a.status);
       }
-      load_r(c + 1);
-    } else if (wq >= 2 && c > 0 && a.o) {  // warps 14, 15: O of chunk c - 1 (rows 64..127 of TU)
+    } else if (!gain && wq >= 2 && wgm == 2 && c > 0 && a.o) {  // warps 14, 15: O of chunk c - 1
       const int t = 32 * (wq - 2) + lane, tt = (c - 1) * CM + t;
       for (int j0 = 0; j0 < D; j0 += 16) {
         float v[16];
@@ -627,8 +649,10 @@ __global__ void __launch_bounds__(WT, 1)
     }
     fence_proxy_async();
     tc_fence_before();
-    ok = __syncthreads_and(p_ok);
-    if (!ok) break;
+    if (!__syncthreads_and(mine)) {
+      failed = true;
+      break;
+    }
 
     // ---- [2] MMA-T; the next chunk's k, g, omega; this chunk's V over q
     if (issuer) {
@@ -637,7 +661,7 @@ __global__ void __launch_bounds__(WT, 1)
       for (int kk = 0; kk < 16; ++kk)
         umma_tf32(TD1, sw128_desc(A0 + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024),
                   sw128_desc(B0 + (kk >> 2) * 8192 + (kk & 3) * 32, 16, 1024), id_T, kk > 0);
-      umma_commit(bar_mma);
+      umma_commit(bar_t);
       issue_v(c);
       if (c + 1 < NC) {
         issue_raw(c + 1);
@@ -647,17 +671,22 @@ __global__ void __launch_bounds__(WT, 1)
         }
       }
     }
-    ok = __syncthreads_and(mma_wait_all());
-    if (!ok) break;
+    if (gain) {
+      // the next chunk's gain, overlapping this chunk's remaining stages
+      if (c + 1 < NC) mine = gain_chunk(c + 1) && mine;
+      continue;
+    }
+    mine = mbar_wait(bar_t, c & 1, kWait) && mine;
     tc_fence_after();
 
-    // ---- [3] T' (with its diagonal) and A'_qk out of TMEM; S_in -> fp16; V -> fp16
-    {
-      const int s0 = 16 * wg;
-      float v[16];
-      tmem_ld16(TD1 + lane_base + s0, v);
-      if (wq < 2) {  // T' rows 0..63, lower triangle with the diagonal -> fp32 tile
-        const int t = 32 * wq + lane;
+    // ---- [3] T' (with its diagonal) out of TMEM; A'_qk -> fp16 pairs in place (the
+    //          A operand of MMA-O); S_in -> fp16; V -> fp16
+    if (wq < 2) {  // T' rows 0..63, lower triangle with the diagonal -> fp32 tile
+      const int t = 32 * wq + lane;
+      for (int g = wgm; g < 4; g += 3) {
+        const int s0 = 16 * g;
+        float v[16];
+        tmem_ld16(TD1 + lane_base + s0, v);
 #pragma unroll
         for (int u = 0; u < 4; ++u) {
           float4 o;
@@ -667,26 +696,29 @@ __global__ void __launch_bounds__(WT, 1)
           o.w = (s0 + 4 * u + 3 <= t) ? v[4 * u + 3] : 0.f;
           *reinterpret_cast<float4 *>(sT + t * LT + s0 + 4 * u) = o;
         }
-      } else {  // A'_qk rows 64..127 (lower triangle) -> fp16
-        const int t = 32 * (wq - 2) + lane;
-#pragma unroll
-        for (int u = 0; u < 16; ++u) v[u] = (s0 + u <= t) ? v[u] : 0.f;
-        sm16(ao, chunk_off(64 + t, s0 >> 3)) = pack_h8(v);
-        sm16(ao, chunk_off(64 + t, (s0 >> 3) + 1)) = pack_h8(v + 8);
       }
-    }
-    // zero rows 0..63 of [0; A'_qk] and rows 64..127 of [A; 0]
-    for (int e = tid; e < 1024; e += WT) {
-      unsigned char *base = e < 512 ? ao : awu + 8192;
-      const int ee = e & 511;
-      sm16(base, (uint32_t)(ee >> 3) * 128u + (uint32_t)((ee & 7) << 4)) = make_uint4(0, 0, 0, 0);
+    } else if (wgm == 0) {
+      // A'_qk rows 64..127, lower triangle: columns 16g .. 16g + 15 -> fp16 pairs in
+      // columns 8g .. 8g + 7 (each column is read before it is overwritten)
+      const int t = 32 * (wq - 2) + lane;
+      for (int g = 0; g < 4; ++g) {
+        float v[16], hv[8];
+        tmem_ld16(TD1 + lane_base + 16 * g, v);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const __half2 h2 = __floats2half2_rn((16 * g + 2 * j <= t) ? v[2 * j] : 0.f,
+                                               (16 * g + 2 * j + 1 <= t) ? v[2 * j + 1] : 0.f);
+          hv[j] = __uint_as_float(*reinterpret_cast<const uint32_t *>(&h2));
+        }
+        tmem_st8(TD1 + lane_base + 8 * g, hv);
+      }
     }
     {  // S_in -> fp16 (MN-major B of MMA-S1); diag(gamma_C) S_in back to TMEM
       const int i = 32 * wq + lane;
       const float gC = s_gC[i];
-      for (int c0 = 0; c0 < 32; c0 += 16) {
+      for (int g = wgm; g < 8; g += 3) {
         float v[16];
-        const int j0 = 32 * wg + c0, sl = j0 >> 6, cc0 = (j0 & 63) >> 3;
+        const int j0 = 16 * g, sl = j0 >> 6, cc0 = (j0 & 63) >> 3;
         tmem_ld16(TS + lane_base + j0, v);
         sm16(s16, sl * 16384 + chunk_off(i, cc0)) = pack_h8(v);
         sm16(s16, sl * 16384 + chunk_off(i, cc0 + 1)) = pack_h8(v + 8);
@@ -695,9 +727,10 @@ __global__ void __launch_bounds__(WT, 1)
         tmem_st16(TS + lane_base + j0, v);
       }
     }
-    bool v_ok = mbar_wait(bar_v, c & 1, kWait);
-    if (v_ok) {  // V -> fp16 in place (two 16-byte chunks per thread)
-      for (int e = tid; e < 1024; e += WT) {
+    {
+      const bool v_ok = mbar_wait(bar_v, c & 1, kWait);
+      mine = v_ok && mine;
+      for (int e = mt; v_ok && e < 1024; e += kMain) {  // V -> fp16 in place
         const uint32_t off = (e >> 9) * 8192 + chunk_off((e >> 3) & 63, e & 7);
         float v[8];
         unpack_bf8(sm16(vr, off), v);
@@ -706,41 +739,59 @@ __global__ void __launch_bounds__(WT, 1)
     }
     tmem_st_wait();
     fence_proxy_async();
-    ok = __syncthreads_and(v_ok);
-    if (!ok) break;
+    tc_fence_before();
+    bar_sync(kBarMain, kMain);
+    tc_fence_after();
     if (SV && issuer) {
       bulk_s2g(ctx + kCtxS, s16, 32768);
       bulk_commit();
     }
 
     // ---- [4] A = (I + T)^-1 = diag(s) L^-1 with L = diag(s) + strict_lower(T')
-    //          (T = strict_lower(T') diag(1/s)), then [A; 0] fp16
-    wy_inverse(sT, sA, sX, sY, s_r, s_s, s_is);
-    {
-      const int r = tid >> 3, cc = tid & 7;
-      const float sr = s_s[r];
-      const float4 a0 = *reinterpret_cast<const float4 *>(sA + r * LT + 8 * cc);
-      const float4 a1 = *reinterpret_cast<const float4 *>(sA + r * LT + 8 * cc + 4);
-      const float av[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
+    //          (T = strict_lower(T') diag(1/s)), then [A; 0] fp16 over T'
+    wy_inverse(mt, sT, sA, sX, sY, s_r + 64 * (c & 1), s_s, s_is);
+    for (int e = mt; e < 1024; e += kMain) {
+      const int r = e >> 3, cc = e & 7;
       float v[8];
+      if (r < 64) {
+        const float sr = s_s[r];
+        const float4 a0 = *reinterpret_cast<const float4 *>(sA + r * LT + 8 * cc);
+        const float4 a1 = *reinterpret_cast<const float4 *>(sA + r * LT + 8 * cc + 4);
+        const float av[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
 #pragma unroll
-      for (int j = 0; j < 8; ++j) v[j] = (8 * cc + j <= r) ? sr * av[j] : 0.f;
-      sm16(awu, chunk_off(r, cc)) = pack_h8(v);
-      if (SV) {  // A_qk = lower(A'_qk) diag(1/s) and s_t into the context
-        float q8[8];
-        unpack_h8(sm16(ao, chunk_off(64 + r, cc)), q8);
-        const float4 i0v = *reinterpret_cast<const float4 *>(s_is + 8 * cc);
-        const float4 i1v = *reinterpret_cast<const float4 *>(s_is + 8 * cc + 4);
-        const float is8[8] = {i0v.x, i0v.y, i0v.z, i0v.w, i1v.x, i1v.y, i1v.z, i1v.w};
+        for (int j = 0; j < 8; ++j) v[j] = (8 * cc + j <= r) ? sr * av[j] : 0.f;
+      } else {
 #pragma unroll
-        for (int j = 0; j < 8; ++j) q8[j] *= is8[j];
-        *reinterpret_cast<uint4 *>(ctx + kCtxAqk + chunk_off(r, cc)) = pack_h8(q8);
-        if (tid < CM) reinterpret_cast<float *>(ctx + kCtxTok)[tid] = s_s[tid];
+        for (int j = 0; j < 8; ++j) v[j] = 0.f;
       }
+      sm16(awu, chunk_off(r, cc)) = pack_h8(v);
+    }
+    if (SV) {
+      if (wq >= 2 && wgm == 0) {  // A_qk = lower(A'_qk) diag(1/s) into the context
+        const int t = 32 * (wq - 2) + lane;
+        for (int h2 = 0; h2 < 2; ++h2) {
+          float pv[16];
+          tmem_ld16(TD1 + lane_base + 16 * h2, pv);  // 32 fp16 of columns 32 h2 ..
+#pragma unroll
+          for (int q4 = 0; q4 < 4; ++q4) {
+            const int cc = 4 * h2 + q4;
+            float v8[8];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+              const uint32_t bits = __float_as_uint(pv[4 * q4 + j]);
+              const float2 f2 = __half22float2(*reinterpret_cast<const __half2 *>(&bits));
+              v8[2 * j] = f2.x * s_is[8 * cc + 2 * j];
+              v8[2 * j + 1] = f2.y * s_is[8 * cc + 2 * j + 1];
+            }
+            *reinterpret_cast<uint4 *>(ctx + kCtxAqk + chunk_off(t, cc)) = pack_h8(v8);
+          }
+        }
+      }
+      if (mt < CM) reinterpret_cast<float *>(ctx + kCtxTok)[mt] = s_s[mt];
     }
     fence_proxy_async();
     tc_fence_before();
-    __syncthreads();
+    bar_sync(kBarMain, kMain);
 
     // ---- [5] MMA-W = A Kbar, MMA-U = A V (fp16)
     if (issuer) {
@@ -757,16 +808,15 @@ __global__ void __launch_bounds__(WT, 1)
       }
       umma_commit(bar_mma);
     }
-    ok = __syncthreads_and(mma_wait_all());
-    if (!ok) break;
+    mine = mma_wait_main() && mine;
     tc_fence_after();
 
     // ---- [6] -W -> fp16 rows 0..63 of [-W; Qbar]
     if (wq < 2) {
       const int t = 32 * wq + lane;
-      for (int c0 = 0; c0 < 32; c0 += 16) {
+      for (int g = wgm; g < 8; g += 3) {
         float v[16];
-        const int j0 = 32 * wg + c0, sl = j0 >> 6, cc0 = (j0 & 63) >> 3;
+        const int j0 = 16 * g, sl = j0 >> 6, cc0 = (j0 & 63) >> 3;
         tmem_ld16(TW + lane_base + j0, v);
 #pragma unroll
         for (int u = 0; u < 16; ++u) v[u] = -v[u];
@@ -776,7 +826,7 @@ __global__ void __launch_bounds__(WT, 1)
     }
     fence_proxy_async();
     tc_fence_before();
-    __syncthreads();
+    bar_sync(kBarMain, kMain);
 
     // ---- [7] MMA-S1: [U; 0] += [-W; Qbar] S_in  (fp16)
     if (issuer) {
@@ -792,17 +842,16 @@ __global__ void __launch_bounds__(WT, 1)
                   sw128_desc(B1 + kk * 2048, 16384, 1024), id_16, 1);
       umma_commit(bar_mma);
     }
-    ok = __syncthreads_and(mma_wait_all());
-    if (!ok) break;
+    mine = mma_wait_main() && mine;
     tc_fence_after();
 
     // ---- [8] R' = diag(1/s) R -> fp16 [t][j] (MN-major B), over V
     if (wq < 2) {
       const int t = 32 * wq + lane;
       const float ist = s_is[t];
-      for (int c0 = 0; c0 < 32; c0 += 16) {
+      for (int g = wgm; g < 8; g += 3) {
         float v[16];
-        const int j0 = 32 * wg + c0, sl = j0 >> 6, cc0 = (j0 & 63) >> 3;
+        const int j0 = 16 * g, sl = j0 >> 6, cc0 = (j0 & 63) >> 3;
         tmem_ld16(TU + lane_base + j0, v);
         if (SV) {
           *reinterpret_cast<uint4 *>(ctx + kCtxR + sl * 8192 + chunk_off(t, cc0)) = pack_h8(v);
@@ -816,32 +865,34 @@ __global__ void __launch_bounds__(WT, 1)
     }
     fence_proxy_async();
     tc_fence_before();
-    __syncthreads();
+    bar_sync(kBarMain, kMain);
 
-    // ---- [9] MMA-O (rows 64..127 of TU += A'_qk R') and MMA-S2 (S += K'^T R')
+    // ---- [9] MMA-O (rows 64..127 of TU += A'_qk R', A'_qk in TMEM) and
+    //          MMA-S2 (S += K'^T R', K' in TMEM)
     if (issuer) {
       tc_fence_after();
-      const uint32_t AO = smem_u32(ao), VR = smem_u32(vr);
+      const uint32_t VR = smem_u32(vr);
       for (int kk = 0; kk < 4; ++kk) {
         const uint64_t bd = sw128_desc(VR + kk * 2048, 8192, 1024);
-        umma_bf16(TU, sw128_desc(AO + kk * 32, 16, 1024), bd, id_16, 1);
+        umma_f16_tA(TU, TD1 + (uint32_t)(kk * 8), bd, id_16, 1);
         umma_f16_tA(TS, tkt + (uint32_t)(kk * 8), bd, id_16, 1);
       }
       umma_commit(bar_mma);
     }
   }
 
-  if (ok && NC > 0) {
-    ok = mma_wait_all();  // MMA-O / MMA-S2 of the last chunk
-    ok = __syncthreads_and(ok);
+  if (!failed && NC > 0) {
+    if (!gain) mine = mma_wait_main() && mine;  // MMA-O / MMA-S2 of the last chunk
+    tc_fence_before();
+    failed = !__syncthreads_and(mine);
     tc_fence_after();
   }
-  if (ok) {
-    if (wq >= 2 && NC > 0 && a.o) {  // O of the last chunk
-      const int c = NC - 1, t = 32 * (wq - 2) + lane, tt = c * CM + t;
-      for (int c0 = 0; c0 < 32; c0 += 16) {
+  if (!failed) {
+    if (!gain && wq >= 2 && NC > 0 && a.o) {  // O of the last chunk
+      const int t = 32 * (wq - 2) + lane, tt = (NC - 1) * CM + t;
+      for (int g = wgm; g < 8; g += 3) {
         float v[16];
-        const int j0 = 32 * wg + c0;
+        const int j0 = 16 * g;
         tmem_ld16(TU + lane_base + j0, v);
         if (tt < a.T) {
           const size_t base = tok_index(a, b, tt, h) * D + j0;
@@ -857,11 +908,11 @@ __global__ void __launch_bounds__(WT, 1)
         }
       }
     }
-    if (a.ST) {
+    if (!gain && a.ST) {
       const int i = 32 * wq + lane;
-      for (int c0 = 0; c0 < 32; c0 += 16) {
+      for (int g = wgm; g < 8; g += 3) {
         float v[16];
-        const int j0 = 32 * wg + c0;
+        const int j0 = 16 * g;
         tmem_ld16(TS + lane_base + j0, v);
         float4 *dst = reinterpret_cast<float4 *>(a.ST + ((size_t)bh * D + i) * D + j0);
 #pragma unroll
@@ -879,6 +930,8 @@ __global__ void __launch_bounds__(WT, 1)
       mbar_wait(bar_v, 1, kWait);
       mbar_wait(bar_q, 0, kWait);
       mbar_wait(bar_q, 1, kWait);
+      mbar_wait(bar_t, 0, kWait);
+      mbar_wait(bar_t, 1, kWait);
       mbar_wait(bar_mma, 0, kWait);
       mbar_wait(bar_mma, 1, kWait);
     }
