@@ -83,7 +83,7 @@ def decode_bytes(b, h, dk, dv, in_bytes=2, out_bytes=4):
 # capture (dram__bytes_read.sum + dram__bytes_write.sum) of the current build;
 # reported as `traffic` only for that workload.  None: not captured for the
 # current kernels.
-NCU_TRAFFIC = {"k_fused_fwd": None, "k_fused_bwd": None, "k_fused_fwd_plain": None}
+NCU_TRAFFIC = {"k_wy_fwd<1>": None, "k_fused_bwd": None, "k_wy_fwd<0>": None}
 
 
 def chunk_flops(dk, dv, C=64):
@@ -286,11 +286,11 @@ def run_gpu(args):
 
     fb = fwd_bytes(B, T, H, DK, DV)
     bb = bwd_bytes(B, T, H, DK, DV)
-    # one kernel per call: k_fused_fwd<0,0,0,0> (forward + context), k_fused_bwd<0,0,0,0> (backward sweep)
-    fwd_roof = {"bound": "hbm", "kernel": "k_fused_fwd<0,0,0,0> (kdn_diag_fwd_save)",
+    # one kernel per call: k_wy_fwd<1> (forward + context), k_fused_bwd<0,0,0,0> (backward sweep)
+    fwd_roof = {"bound": "hbm", "kernel": "k_wy_fwd<1> (kdn_diag_fwd_save)",
                 "achieved": fb / (fwd_ms / 1e3) / 1e9, "peak": hbm, "unit": "GB/s",
                 "peak_kind": peak_kind, "algorithmic_bytes": fb, "ms": fwd_ms,
-                "traffic": NCU_TRAFFIC["k_fused_fwd"] if B == 8 else None}
+                "traffic": NCU_TRAFFIC["k_wy_fwd<1>"] if B == 8 else None}
     fwd_roof["frac"] = fwd_roof["achieved"] / hbm
     bwd_roof = {"bound": "hbm", "kernel": "k_fused_bwd<0,0,0,0> (kdn_diag_bwd_saved)",
                 "achieved": bb / (bwd_ms / 1e3) / 1e9, "peak": hbm, "unit": "GB/s",
@@ -375,11 +375,11 @@ def run_forward_plain(kdn, torch, args, x, hbm, peak_kind):
             "gpu_launches": kdn.kdn_kernel_launches(desc, 0, 0) * args.steps,
             "spec_roofline_frac": spec_s / (ms / 1e3),
             "spec_roofline_us": spec_s * 1e6,
-            "roofline": {"bound": "hbm", "kernel": "k_fused_fwd (kdn_diag_fwd)",
+            "roofline": {"bound": "hbm", "kernel": "k_wy_fwd<0> (kdn_diag_fwd)",
                          "achieved": nb / (ms / 1e3) / 1e9, "peak": hbm, "unit": "GB/s",
                          "peak_kind": peak_kind, "frac": nb / (ms / 1e3) / 1e9 / hbm,
                          "algorithmic_bytes": nb,
-                         "traffic": NCU_TRAFFIC["k_fused_fwd_plain"] if B == 8 else None}}
+                         "traffic": NCU_TRAFFIC["k_wy_fwd<0>"] if B == 8 else None}}
 
 
 def run_iso_step(kdn, torch, args, hbm):

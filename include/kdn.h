@@ -49,9 +49,12 @@
  *              S0, ST, dST, dS0 (float32)   [B, H, dk, dv]
  *              p0, pT, dpT, dp0 (float32)   diag [B, H, dk];  iso [B, H]
  *              Gradients have the layout of the input they belong to.
- *   Dtypes     q, k, v, g, omega, r, o, dO and the input gradients share
- *              desc->dtype (float32 or bfloat16).  State is always float32;
- *              all arithmetic is float32.
+ *   Dtypes     q, k, v, g, omega, r and dO have desc->dtype (float32 or
+ *              bfloat16); o and the input gradients have desc->out_dtype.
+ *              State is always float32.  Accumulation is float32; the
+ *              bf16 d = 128 forward runs its intra-chunk products on the
+ *              tensor cores with tf32 and fp16 operands (Sec. 4.2 products,
+ *              float32 accumulators).
  *   Sizes      dk, dv in {32, 64, 128}; T >= 0 (any length; a ragged last
  *              chunk is padded with identity tokens); B, H >= 0.
  */
@@ -71,10 +74,13 @@ typedef enum {
   KDN_ERR_WORKSPACE = 3,   /* workspace missing or smaller than required */
   KDN_ERR_CUDA = 4,        /* a CUDA launch or runtime call failed */
   KDN_ERR_TIMEOUT = 5,     /* a bounded device-side wait gave up */
-  KDN_ERR_RANGE = 6        /* device status only: a 64-token chunk's cumulative decay
-                              exp(G_C) fell below 1e-36 in some channel, outside the fused
-                              kernels' range (results of that call are invalid); the
-                              general kernels (desc->chunk = 32) halve the exposure */
+  KDN_ERR_RANGE = 6        /* device status only: a 64-token chunk's cumulative log-decay
+                              G_C left a fused kernel's range in some channel (results of
+                              that call are invalid).  The plain bf16 d = 128 diagonal
+                              forward takes G_C >= -160; the calls that write or read the
+                              backward context (the *_fwd_save / *_bwd_saved pairs, the
+                              other fused forwards) take exp(G_C) >= 1e-36, G_C >= -82.8.
+                              desc->chunk = 32 halves the exposure. */
 } kdn_status_t;
 
 typedef enum { KDN_F32 = 0, KDN_BF16 = 1 } kdn_dtype_t;

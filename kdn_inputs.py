@@ -110,19 +110,32 @@ def make_decode_inputs(variant: str, B: int, H: int, dk: int, dv: int, steps: in
     S = rng.normal(0.0, s_std, size=(B, H, dk, dv))
     pshape = (B, H, dk) if variant == "diag" else (B, H)
     p = rng.uniform(p_range[0], p_range[1], size=pshape)
-    gshape = (B, H, dk) if per_channel_decay else (B, H)
-    wshape = (B, H, dk) if variant == "diag" else (B, H)
     cols = {n: [] for n in ("q", "k", "v", "g", "omega", "r")}
     for _ in range(steps):
-        cols["q"].append(_l2n(rng.standard_normal((B, H, dk))))
-        cols["k"].append(_l2n(rng.standard_normal((B, H, dk))))
-        cols["v"].append(rng.standard_normal((B, H, dv)))
-        cols["g"].append(_log_sigmoid(rng.normal(2.0, 1.0, size=gshape)))
-        cols["omega"].append(_softplus(rng.standard_normal(wshape)))
-        cols["r"].append(_softplus(rng.standard_normal((B, H))))
+        one = draw_decode_step(rng, variant, B, H, dk, dv, per_channel_decay=per_channel_decay)
+        for n in cols:
+            cols[n].append(one[n])
     out = dict(variant=variant, dtype=dtype, B=B, H=H, dk=dk, dv=dv, steps=steps,
                per_channel_decay=bool(per_channel_decay),
                S=round_to(S, "f32"), p=round_to(p, "f32"))
     for n, lst in cols.items():
         out[n] = round_to(np.stack(lst), dtype)
     return out
+
+
+def draw_decode_step(rng, variant: str, B: int, H: int, dk: int, dv: int, *,
+                     per_channel_decay: bool, dtype: str | None = None) -> dict:
+    """One decode token's inputs, drawn from ``rng`` in the order q, k, v,
+    x_decay, x_omega, x_r; rounded to ``dtype`` when one is given.  Long decode
+    runs draw step by step so that no [steps, B, H, d] float64 array is held."""
+    gshape = (B, H, dk) if per_channel_decay else (B, H)
+    wshape = (B, H, dk) if variant == "diag" else (B, H)
+    one = {"q": _l2n(rng.standard_normal((B, H, dk))),
+           "k": _l2n(rng.standard_normal((B, H, dk))),
+           "v": rng.standard_normal((B, H, dv)),
+           "g": _log_sigmoid(rng.normal(2.0, 1.0, size=gshape)),
+           "omega": _softplus(rng.standard_normal(wshape)),
+           "r": _softplus(rng.standard_normal((B, H)))}
+    if dtype is not None:
+        one = {n: round_to(x, dtype) for n, x in one.items()}
+    return one

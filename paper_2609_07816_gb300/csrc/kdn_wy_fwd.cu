@@ -18,16 +18,18 @@
 //            the chunk's decay range.
 //   prepare  warps 4-11, one thread per (4 channels, 8 tokens), form
 //              Kbar_t = k_t exp(G_t - c), Qbar_t = tau q_t exp(G_t - c)  (tf32)
-//              Kbar_t = gamma_t k_t, Qbar_t = tau gamma_t q_t           (fp16)
+//              -Kbar_t = -gamma_t k_t, Qbar_t = tau gamma_t q_t        (fp16)
 //   MMA-T    [Kbar; Qbar] Kk'^T (tf32) = [T'; A'_qk].  The ratios
 //            exp(G_t - G_s) of App. F.2 are exact products of the two
 //            referenced factors, each within exp(+-|G_C| / 2).
 //            s_t = r_t + sum_i phat_t,i k_t,i^2 (the denominator of the gain,
 //            eq. kla-box-gain) is r_t plus the diagonal of T'.
+//   MMA-KS   [-Kbar; Qbar] S_in = [-Kbar S_in; Qbar S_in]  (fp16), on the tensor
+//            cores while the CUDA cores solve
 //   solve    with L = diag(s) + strict_lower(T'), A = (I + T)^-1 = diag(s) L^-1
 //            (T = strict_lower(T') diag(1/s)) on CUDA cores in fp32.
-//   MMA-W/U  W = A Kbar, U = A V (fp16)
-//   MMA-S1   [U; 0] + [-W; Qbar] S_in = [R; Qbar S_in]          (fp16)
+//   MMA-R    R = U - W S_in = A (V - Kbar S_in)  (fp16; W = A Kbar, U = A V of
+//            eq. chunk-memory-wy are only formed for the backward's context)
 //   MMA-O    O = Qbar S_in + A'_qk R'          with R' = diag(1/s) R
 //   MMA-S2   S_out = diag(gamma_C) S_in + K'^T R'   (K' in tensor memory)
 // so that A'_qk R' = A_qk R and K'^T R' = K_tail^T R of eq.
@@ -59,6 +61,7 @@ constexpr int WT = 512;  // threads
 constexpr int CM = 64;   // chunk length
 constexpr int D = 128;   // d_k = d_v
 constexpr uint32_t kWait = 1u << 25;
+constexpr uint32_t kDrain = 1u << 14;  // bounded waits of the failure path
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kMinHalfG = -80.f;  // c = G_C / 2 below this: out of range
 constexpr int kPrepThreads = 256;   // warps 4-11: the preparing pass
@@ -74,18 +77,17 @@ constexpr int O_V = 49152;     // q (TMA, the preparing pass), then V (TMA bf16 
                                // then R' fp16 [64 s][128 j]                       16 KB
 constexpr int O_TA = 65536;    // tf32 [Kbar; Qbar] [128][128], four 32-channel slabs 64 KB
 constexpr int O_TB = 133120;   // tf32 Kk' [64][128], four slabs                   32 KB
-constexpr int O_KB = 165888;   // fp16 Kbar [64 s][128 i], two slabs (MMA-W B)     16 KB
-constexpr int O_AS1 = 182272;  // fp16 [-W; Qbar] [128][128], two slabs (MMA-S1 A) 32 KB
+constexpr int O_SCR = 165888;  // scratch of the solve (sX, sY)                    16 KB
+constexpr int O_AS1 = 182272;  // fp16 [-Kbar; Qbar] [128][128], two slabs (MMA-KS A) 32 KB
 constexpr int O_SMALL = 215040;
 // after MMA-T has read the tf32 tiles (T and A run 2 KB past the tf32 tile)
-constexpr int O_S16 = O_TA;                      // fp16 S_in [128 i][128 j], two slabs (MMA-S1 B)
+constexpr int O_S16 = O_TA;                      // fp16 S_in [128 i][128 j], two slabs (MMA-KS B)
 constexpr int O_SWT = O_TA + 32768;              // fp32 T' [64][LT]
 constexpr int O_SWA = O_SWT + 64 * LT * 4;       // fp32 L^-1 [64][LT]
 static_assert(O_SWA + 64 * LT * 4 <= O_TB, "T and A tiles overlap the Kk' tile");
-constexpr int O_AWU = O_SWT;           // fp16 [A; 0] [128][64] (MMA-W/U A), over T' after the solve
-// inverse scratch in rows 0..63 of the first slab of [-W; Qbar] (written after it)
-constexpr int O_SX = O_AS1;            // 2 x 256 floats
-constexpr int O_SY = O_AS1 + 2048;     // 32 x 32 floats
+constexpr int O_AWU = O_SWT;           // fp16 [A; 0] [128][64] (MMA-R A), over T' after the solve
+constexpr int O_SX = O_SCR;            // 2 x 256 floats
+constexpr int O_SY = O_SCR + 2048;     // 32 x 32 floats
 // small arrays (floats); r and mu / r per token for two chunks (the gain works one chunk ahead)
 constexpr int SM_R = 0, SM_MUR = 128, SM_S = 256, SM_IS = 320, SM_C = 384, SM_GC = 512,
               SM_PART = 640, SM_FLOATS = 640 + 8 * 128;
@@ -322,7 +324,7 @@ __global__ void __launch_bounds__(WT, 1)
   unsigned char *sm =
       reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(smraw) + 1023) & ~uintptr_t(1023));
   unsigned char *rk = sm + O_RK, *rg = sm + O_RG, *rw = sm + O_RW, *vr = sm + O_V;
-  unsigned char *ta = sm + O_TA, *tb = sm + O_TB, *kb = sm + O_KB, *as1 = sm + O_AS1;
+  unsigned char *ta = sm + O_TA, *tb = sm + O_TB, *as1 = sm + O_AS1;
   unsigned char *s16 = sm + O_S16, *awu = sm + O_AWU;
   float *sT = reinterpret_cast<float *>(sm + O_SWT), *sA = reinterpret_cast<float *>(sm + O_SWA);
   float *sX = reinterpret_cast<float *>(sm + O_SX), *sY = reinterpret_cast<float *>(sm + O_SY);
@@ -332,7 +334,8 @@ __global__ void __launch_bounds__(WT, 1)
   uint64_t *bars = reinterpret_cast<uint64_t *>(sm + O_BAR);
   uint64_t *bar_raw = bars, *bar_v = bars + 1, *bar_mma = bars + 2, *bar_q = bars + 3;
   uint64_t *bar_t = bars + 4;  // MMA-T completions (one a chunk)
-  uint32_t *s_tbase = reinterpret_cast<uint32_t *>(bars + 5);
+  uint64_t *bar_w = bars + 5;  // MMA-W completions (context mode only, one a chunk)
+  uint32_t *s_tbase = reinterpret_cast<uint32_t *>(bars + 6);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int wq = warp & 3, wg = warp >> 2;  // TMEM lane quarter, column group
@@ -347,6 +350,7 @@ __global__ void __launch_bounds__(WT, 1)
     mbar_init(bar_mma, 1);
     mbar_init(bar_q, 1);
     mbar_init(bar_t, 1);
+    mbar_init(bar_w, 1);
     fence_mbar_init();
     prefetch_tmap(&mk);
     prefetch_tmap(&mg);
@@ -429,7 +433,8 @@ __global__ void __launch_bounds__(WT, 1)
   };
   load_r(0);
 
-  uint32_t mph = 0;  // main threads: completions of bar_mma observed (three per chunk)
+  uint32_t mph = 0;  // main threads: completions of bar_mma observed (three per chunk:
+                     // MMA-KS, MMA-R, MMA-O / MMA-S2)
   auto mma_wait_main = [&]() -> bool {
     const bool r = mbar_wait(bar_mma, mph & 1, kWait);
     ++mph;
@@ -594,7 +599,7 @@ __global__ void __launch_bounds__(WT, 1)
 #pragma unroll
       for (int u = 0; u < 4; ++u) Ec[u] = ex2f(cr[u] * kLog2e);
       mine = mbar_wait(bar_q, c & 1, kWait) && mine;
-      unsigned char *pa = ta + (i0 >> 5) * 16384, *pkb = kb + sl8, *pqh = as1 + (i0 >> 6) * 16384;
+      unsigned char *pa = ta + (i0 >> 5) * 16384, *pqh = as1 + (i0 >> 6) * 16384;
       const int cc = i0 & 31;
 #pragma unroll
       for (int j = 0; j < 8; ++j) {
@@ -614,8 +619,8 @@ __global__ void __launch_bounds__(WT, 1)
             make_float4(tf32r(e[0] * kv[0]), tf32r(e[1] * kv[1]), tf32r(e[2] * kv[2]), tf32r(e[3] * kv[3]));
         *reinterpret_cast<float4 *>(pa + sw32_off(64 + t, cc)) =
             make_float4(tf32r(e[0] * qv[0]), tf32r(e[1] * qv[1]), tf32r(e[2] * qv[2]), tf32r(e[3] * qv[3]));
-        *reinterpret_cast<uint2 *>(pkb + sw128_off4(t, i0)) =
-            pack_h4(gm[0] * kv[0], gm[1] * kv[1], gm[2] * kv[2], gm[3] * kv[3]);
+        *reinterpret_cast<uint2 *>(pqh + sw128_off4(t, i0)) =
+            pack_h4(-gm[0] * kv[0], -gm[1] * kv[1], -gm[2] * kv[2], -gm[3] * kv[3]);
         *reinterpret_cast<uint2 *>(pqh + sw128_off4(64 + t, i0)) =
             pack_h4(gm[0] * qv[0], gm[1] * qv[1], gm[2] * qv[2], gm[3] * qv[3]);
         if (SV)
@@ -713,7 +718,7 @@ __global__ void __launch_bounds__(WT, 1)
         tmem_st8(TD1 + lane_base + 8 * g, hv);
       }
     }
-    {  // S_in -> fp16 (MN-major B of MMA-S1); diag(gamma_C) S_in back to TMEM
+    {  // S_in -> fp16 (MN-major B of MMA-KS); diag(gamma_C) S_in back to TMEM
       const int i = 32 * wq + lane;
       const float gC = s_gC[i];
       for (int g = wgm; g < 8; g += 3) {
@@ -727,24 +732,22 @@ __global__ void __launch_bounds__(WT, 1)
         tmem_st16(TS + lane_base + j0, v);
       }
     }
-    {
-      const bool v_ok = mbar_wait(bar_v, c & 1, kWait);
-      mine = v_ok && mine;
-      for (int e = mt; v_ok && e < 1024; e += kMain) {  // V -> fp16 in place
-        const uint32_t off = (e >> 9) * 8192 + chunk_off((e >> 3) & 63, e & 7);
-        float v[8];
-        unpack_bf8(sm16(vr, off), v);
-        sm16(vr, off) = pack_h8(v);
-      }
-    }
     tmem_st_wait();
     fence_proxy_async();
     tc_fence_before();
     bar_sync(kBarMain, kMain);
     tc_fence_after();
-    if (SV && issuer) {
-      bulk_s2g(ctx + kCtxS, s16, 32768);
-      bulk_commit();
+    // MMA-KS: TU = [-Kbar; Qbar] S_in (fp16), while the CUDA cores solve
+    if (issuer) {
+      const uint32_t A1 = smem_u32(as1), B1 = smem_u32(s16);
+      for (int kk = 0; kk < 8; ++kk)
+        umma_bf16(TU, sw128_desc(A1 + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024),
+                  sw128_desc(B1 + kk * 2048, 16384, 1024), id_16, kk > 0);
+      umma_commit(bar_mma);
+      if (SV) {
+        bulk_s2g(ctx + kCtxS, s16, 32768);
+        bulk_commit();
+      }
     }
 
     // ---- [4] A = (I + T)^-1 = diag(s) L^-1 with L = diag(s) + strict_lower(T')
@@ -793,66 +796,79 @@ __global__ void __launch_bounds__(WT, 1)
     tc_fence_before();
     bar_sync(kBarMain, kMain);
 
-    // ---- [5] MMA-W = A Kbar, MMA-U = A V (fp16)
-    if (issuer) {
-      if (SV) {
+    // ---- [5] (context only) -W = A (-Kbar) into TW, then to the context
+    if (SV) {
+      if (issuer) {
         bulk_s2g(ctx + kCtxA, awu, 8192);
         bulk_commit();
+        tc_fence_after();
+        const uint32_t AW = smem_u32(awu), KN = smem_u32(as1);
+        for (int kk = 0; kk < 4; ++kk)  // B = rows 0..63 of [-Kbar; Qbar], MN-major
+          umma_bf16(TW, sw128_desc(AW + kk * 32, 16, 1024), sw128_desc(KN + kk * 2048, 16384, 1024),
+                    id_16, kk > 0);
+        umma_commit(bar_w);  // its own barrier: MMA-KS may not have been observed yet
       }
-      tc_fence_after();
-      const uint32_t AW = smem_u32(awu), KB = smem_u32(kb), VR = smem_u32(vr);
-      for (int kk = 0; kk < 4; ++kk) {
-        const uint64_t ad = sw128_desc(AW + kk * 32, 16, 1024);
-        umma_bf16(TW, ad, sw128_desc(KB + kk * 2048, 8192, 1024), id_16, kk > 0);
-        umma_bf16(TU, ad, sw128_desc(VR + kk * 2048, 8192, 1024), id_16, kk > 0);
-      }
-      umma_commit(bar_mma);
     }
-    mine = mma_wait_main() && mine;
-    tc_fence_after();
-
-    // ---- [6] -W -> fp16 rows 0..63 of [-W; Qbar]
-    if (wq < 2) {
-      const int t = 32 * wq + lane;
-      for (int g = wgm; g < 8; g += 3) {
-        float v[16];
-        const int j0 = 16 * g, sl = j0 >> 6, cc0 = (j0 & 63) >> 3;
-        tmem_ld16(TW + lane_base + j0, v);
+    // ---- [6] Y = V - Kbar S_in (rows 0..63 of TU plus V) -> fp16 in place over V
+    {
+      const bool ks_ok = mma_wait_main();  // MMA-KS
+      const bool v_ok = mbar_wait(bar_v, c & 1, kWait);
+      mine = ks_ok && v_ok && mine;
+      tc_fence_after();
+      if (wq < 2) {
+        const int t = 32 * wq + lane;
+        for (int g = wgm; g < 8; g += 3) {
+          float v[16], vv[16];
+          const int j0 = 16 * g, sl = j0 >> 6, cc0 = (j0 & 63) >> 3;
+          tmem_ld16(TU + lane_base + j0, v);
+          const uint32_t o0 = sl * 8192 + chunk_off(t, cc0), o1 = sl * 8192 + chunk_off(t, cc0 + 1);
+          unpack_bf8(sm16(vr, o0), vv);
+          unpack_bf8(sm16(vr, o1), vv + 8);
 #pragma unroll
-        for (int u = 0; u < 16; ++u) v[u] = -v[u];
-        sm16(as1, sl * 16384 + chunk_off(t, cc0)) = pack_h8(v);
-        sm16(as1, sl * 16384 + chunk_off(t, cc0 + 1)) = pack_h8(v + 8);
+          for (int u = 0; u < 16; ++u) v[u] += vv[u];
+          sm16(vr, o0) = pack_h8(v);
+          sm16(vr, o1) = pack_h8(v + 8);
+        }
+      }
+    }
+    if (SV) {  // -W of the context (rows 0..63 of TW), once MMA-W has completed
+      mine = mbar_wait(bar_w, c & 1, kWait) && mine;
+      tc_fence_after();
+      if (wq < 2) {
+        const int t = 32 * wq + lane;
+        for (int g = wgm; g < 8; g += 3) {
+          float v[16];
+          const int j0 = 16 * g, sl = j0 >> 6, cc0 = (j0 & 63) >> 3;
+          tmem_ld16(TW + lane_base + j0, v);
+          *reinterpret_cast<uint4 *>(ctx + kCtxW + sl * 8192 + chunk_off(t, cc0)) = pack_h8(v);
+          *reinterpret_cast<uint4 *>(ctx + kCtxW + sl * 8192 + chunk_off(t, cc0 + 1)) = pack_h8(v + 8);
+        }
       }
     }
     fence_proxy_async();
     tc_fence_before();
     bar_sync(kBarMain, kMain);
 
-    // ---- [7] MMA-S1: [U; 0] += [-W; Qbar] S_in  (fp16)
+    // ---- [7] MMA-R: TW = [A; 0] Y = [R; 0]  (fp16)
     if (issuer) {
-      if (SV) {
-        bulk_s2g(ctx + kCtxW, as1, 8192);
-        bulk_s2g(ctx + kCtxW + 8192, as1 + 16384, 8192);
-        bulk_commit();
-      }
       tc_fence_after();
-      const uint32_t A1 = smem_u32(as1), B1 = smem_u32(s16);
-      for (int kk = 0; kk < 8; ++kk)
-        umma_bf16(TU, sw128_desc(A1 + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024),
-                  sw128_desc(B1 + kk * 2048, 16384, 1024), id_16, 1);
+      const uint32_t AW = smem_u32(awu), VR = smem_u32(vr);
+      for (int kk = 0; kk < 4; ++kk)
+        umma_bf16(TW, sw128_desc(AW + kk * 32, 16, 1024), sw128_desc(VR + kk * 2048, 8192, 1024), id_16,
+                  kk > 0);
       umma_commit(bar_mma);
     }
     mine = mma_wait_main() && mine;
     tc_fence_after();
 
-    // ---- [8] R' = diag(1/s) R -> fp16 [t][j] (MN-major B), over V
+    // ---- [8] R' = diag(1/s) R -> fp16 [t][j] (MN-major B), over Y
     if (wq < 2) {
       const int t = 32 * wq + lane;
       const float ist = s_is[t];
       for (int g = wgm; g < 8; g += 3) {
         float v[16];
         const int j0 = 16 * g, sl = j0 >> 6, cc0 = (j0 & 63) >> 3;
-        tmem_ld16(TU + lane_base + j0, v);
+        tmem_ld16(TW + lane_base + j0, v);
         if (SV) {
           *reinterpret_cast<uint4 *>(ctx + kCtxR + sl * 8192 + chunk_off(t, cc0)) = pack_h8(v);
           *reinterpret_cast<uint4 *>(ctx + kCtxR + sl * 8192 + chunk_off(t, cc0 + 1)) = pack_h8(v + 8);
@@ -923,17 +939,13 @@ __global__ void __launch_bounds__(WT, 1)
   } else {
     if (tid == 0) atomicExch(a.status, (unsigned)KDN_ERR_TIMEOUT);
     // copies and MMAs in flight land before the CTA's memory goes away
+    // (short bounds: a copy or MMA that was issued lands within microseconds,
+    // and a phase that was never armed must not hold the call for long)
     if (issuer) {
-      mbar_wait(bar_raw, 0, kWait);
-      mbar_wait(bar_raw, 1, kWait);
-      mbar_wait(bar_v, 0, kWait);
-      mbar_wait(bar_v, 1, kWait);
-      mbar_wait(bar_q, 0, kWait);
-      mbar_wait(bar_q, 1, kWait);
-      mbar_wait(bar_t, 0, kWait);
-      mbar_wait(bar_t, 1, kWait);
-      mbar_wait(bar_mma, 0, kWait);
-      mbar_wait(bar_mma, 1, kWait);
+      for (int k = 0; k < 6; ++k) {
+        mbar_wait(bars + k, 0, kDrain);
+        mbar_wait(bars + k, 1, kDrain);
+      }
     }
   }
   if (SV && issuer) bulk_wait_all();

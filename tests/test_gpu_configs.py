@@ -8,8 +8,8 @@ import pytest
 import torch
 
 import oracle
-from kdn_inputs import make_decode_inputs, make_inputs
-from kdn_gpu_util import check, head_slice, to_dev
+from kdn_inputs import draw_decode_step, make_decode_inputs, make_inputs
+from kdn_gpu_util import check, check_stored_bf16, head_slice, to_dev
 
 pytestmark = pytest.mark.gpu
 NAMES = ("q", "k", "v", "g", "omega", "r")
@@ -82,6 +82,39 @@ def test_diag_1p3b_layer_shape_backward(kdn):
         check(f"dp0[{b},{h}]", gr["dp0"][b:b + 1, h:h + 1], ref["dp0"], "bf16")
 
 
+def test_diag_1p3b_layer_shape_bench_launch(kdn):
+    """B=8 H=16 T=4096 d=128 in the launch configuration the benchmark times:
+    bf16 o and gradients, the training pair kdn_diag_fwd_save + kdn_diag_bwd_saved
+    with a preallocated context and workspaces, and the plain inference forward.
+    Stored bf16 values are checked under the bf16 rule plus one final rounding."""
+    B, T, H = 8, 4096, 16
+    bf = torch.bfloat16
+    ins = make_inputs("diag", B, T, H, 128, 128, dtype="bf16", seed=3, with_grad=True)
+    d = to_dev(ins)
+    x = [d[n] for n in NAMES]
+    desc = kdn.make_desc(B, T, H, 128, 128, bf, out_dtype=bf)
+    ws_f = kdn.alloc_workspace(desc, 0, False)
+    ws_b = kdn.alloc_workspace(desc, 0, False)
+    saved = torch.empty(kdn.saved_bytes(desc), dtype=torch.uint8, device="cuda")
+    o, ST, pT, _ = kdn.kdn_diag_fwd_save(*x, saved=saved, workspace=ws_f, out_dtype=bf)
+    gr = kdn.kdn_diag_bwd_saved(*x, saved, d["dO"], workspace=ws_b, out_dtype=bf)
+    o_plain, ST_plain, pT_plain = kdn.kdn_diag_fwd(*x, workspace=ws_f, out_dtype=bf)
+    torch.cuda.synchronize()
+    assert kdn.kdn_get_device_status(ws_f) == 0 and kdn.kdn_get_device_status(ws_b) == 0
+    for b, h in [(0, 0), (4, 10)]:
+        sl = head_slice(ins, b, h)
+        ref = oracle.fwd("diag", *[sl[n] for n in NAMES], None, None)
+        for tag, oo, SS, pp in (("save", o, ST, pT), ("plain", o_plain, ST_plain, pT_plain)):
+            check_stored_bf16(f"o[{b},{h}] {tag}", oo[b:b + 1, :, h:h + 1], ref["o"])
+            check(f"ST[{b},{h}] {tag}", SS[b:b + 1, h:h + 1], ref["ST"], "bf16")
+            check(f"pT[{b},{h}] {tag}", pp[b:b + 1, h:h + 1], ref["pT"], "bf16")
+        rg = oracle.bwd("diag", *[sl[n] for n in NAMES], None, None, sl["dO"])
+        for n in ("dq", "dk", "dv", "dg", "domega", "dr"):
+            check_stored_bf16(f"{n}[{b},{h}]", gr[n][b:b + 1, :, h:h + 1], rg[n])
+        check(f"dS0[{b},{h}]", gr["dS0"][b:b + 1, h:h + 1], rg["dS0"], "bf16")
+        check(f"dp0[{b},{h}]", gr["dp0"][b:b + 1, h:h + 1], rg["dp0"], "bf16")
+
+
 @pytest.mark.parametrize("variant", ["diag", "iso"])
 def test_long_context_shape(kdn, variant):
     """B=1 H=16 T=65536 d=128, S_0 ~ N(0, 0.02^2), p_0 ~ U(0.5, 2)."""
@@ -111,3 +144,60 @@ def test_decode_batch_shape(kdn, variant):
             check(f"o[{s}][{b},{h}]", outs[s][b:b + 1, h:h + 1], o_ref, "bf16")
         check(f"S[{b},{h}]", S[b:b + 1, h:h + 1], Sr, "bf16")
         check(f"p[{b},{h}]", p[b:b + 1, h:h + 1], pr, "bf16")
+
+
+@pytest.mark.parametrize("variant", ["diag", "iso"])
+def test_decode_long_horizon(kdn, variant):
+    """256 consecutive decode tokens at B=256 H=16 d=128 replayed from one CUDA
+    graph, as the decode benchmark runs them: every token's output and the final
+    state of sampled heads against the oracle's step-by-step recurrence (Eq. 8),
+    so that drift of the float32 state over a long run shows."""
+    B, H, D, steps = 256, 16, 128, 256
+    heads = [(0, 0), (77, 9), (255, 15)]
+    rng = np.random.Generator(np.random.PCG64(2024))
+    S0 = round_to_f32(rng.normal(0.0, 0.02, size=(B, H, D, D)))
+    p0 = round_to_f32(rng.uniform(0.1, 2.0, size=(B, H, D) if variant == "diag" else (B, H)))
+    bf = torch.bfloat16
+    dev = {n: [] for n in NAMES}
+    host = []
+    for _ in range(steps):
+        one = draw_decode_step(rng, variant, B, H, D, D, per_channel_decay=variant == "diag",
+                               dtype="bf16")
+        for n in NAMES:
+            dev[n].append(torch.tensor(one[n], dtype=bf))
+        host.append({n: np.stack([one[n][b, h] for b, h in heads]) for n in NAMES})
+    x = {n: torch.stack(dev[n]).to("cuda") for n in NAMES}
+    S = torch.tensor(S0, dtype=torch.float32, device="cuda")
+    p = torch.tensor(p0, dtype=torch.float32, device="cuda")
+    o = torch.empty(steps, B, H, D, dtype=torch.float32, device="cuda")
+    fn = kdn.kdn_diag_decode_step if variant == "diag" else kdn.kdn_iso_decode_step
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        # one untimed call outside the graph loads the module; state is restored below
+        fn(*[x[n][0] for n in NAMES], S.clone(), p.clone(), o=o[0], stream=side)
+    torch.cuda.current_stream().wait_stream(side)
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        st = torch.cuda.current_stream()
+        for i in range(steps):
+            fn(*[x[n][i] for n in NAMES], S, p, o=o[i], stream=st)
+    graph.replay()
+    torch.cuda.synchronize()
+    o_h = o.cpu()
+    for j, (b, h) in enumerate(heads):
+        Sr, pr = S0[b:b + 1, h:h + 1], p0[b:b + 1, h:h + 1]
+        ref_o = []
+        for i in range(steps):
+            o_ref, Sr, pr = oracle.decode_step(
+                variant, *[host[i][n][j][None, None] for n in NAMES], Sr, pr)
+            ref_o.append(o_ref[0, 0])
+        check(f"o[0:{steps}][{b},{h}]", o_h[:, b, h], np.stack(ref_o), "bf16")
+        check(f"o[{steps - 1}][{b},{h}]", o_h[steps - 1, b, h], ref_o[-1], "bf16")
+        check(f"S[{b},{h}]", S[b:b + 1, h:h + 1], Sr, "bf16")
+        check(f"p[{b},{h}]", p[b:b + 1, h:h + 1], pr, "bf16")
+
+
+def round_to_f32(x):
+    return np.asarray(x, dtype=np.float32).astype(np.float64)
