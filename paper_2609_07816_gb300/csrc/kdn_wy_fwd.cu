@@ -73,11 +73,10 @@ constexpr int LT = 68;          // row stride (floats) of the fp32 T and A tiles
 constexpr int O_RK = 0;        // raw k  [64 t][128 i] bf16, two 64-channel slabs   16 KB
 constexpr int O_RG = 16384;    // raw g                                          16 KB
 constexpr int O_RW = 32768;    // raw omega                                      16 KB
-constexpr int O_V = 49152;     // q (TMA, the preparing pass), then V (TMA bf16 -> fp16),
-                               // then R' fp16 [64 s][128 j]                       16 KB
+constexpr int O_V = 49152;     // V (TMA bf16), then Y fp16, then R' fp16 [64 s][128 j]  16 KB
 constexpr int O_TA = 65536;    // tf32 [Kbar; Qbar] [128][128], four 32-channel slabs 64 KB
 constexpr int O_TB = 133120;   // tf32 Kk' [64][128], four slabs                   32 KB
-constexpr int O_SCR = 165888;  // scratch of the solve (sX, sY)                    16 KB
+constexpr int O_Q = 165888;    // q (TMA, one chunk ahead; the preparing pass)    16 KB
 constexpr int O_AS1 = 182272;  // fp16 [-Kbar; Qbar] [128][128], two slabs (MMA-KS A) 32 KB
 constexpr int O_SMALL = 215040;
 // after MMA-T has read the tf32 tiles (T and A run 2 KB past the tf32 tile)
@@ -86,13 +85,14 @@ constexpr int O_SWT = O_TA + 32768;              // fp32 T' [64][LT]
 constexpr int O_SWA = O_SWT + 64 * LT * 4;       // fp32 L^-1 [64][LT]
 static_assert(O_SWA + 64 * LT * 4 <= O_TB, "T and A tiles overlap the Kk' tile");
 constexpr int O_AWU = O_SWT;           // fp16 [A; 0] [128][64] (MMA-R A), over T' after the solve
-constexpr int O_SX = O_SCR;            // 2 x 256 floats
-constexpr int O_SY = O_SCR + 2048;     // 32 x 32 floats
 // small arrays (floats); r and mu / r per token for two chunks (the gain works one chunk ahead)
 constexpr int SM_R = 0, SM_MUR = 128, SM_S = 256, SM_IS = 320, SM_C = 384, SM_GC = 512,
               SM_PART = 640, SM_FLOATS = 640 + 8 * 128;
 constexpr int O_BAR = O_SMALL + SM_FLOATS * 4;
-constexpr int SMEM_BYTES = O_BAR + 64 + 1024;
+constexpr int O_SX = O_BAR + 64;       // scratch of the solve: 2 x 256 floats
+constexpr int O_SY = O_SX + 2048;      //                       32 x 32 floats
+constexpr int SMEM_BYTES = O_SY + 4096 + 1024;
+static_assert(SMEM_BYTES <= 232448, "shared memory per CTA");
 
 // tensor-memory columns (512 allocated)
 constexpr uint32_t TC_S = 0, TC_D1 = 128, TC_KT = 192, TC_W = 256, TC_U = 384;
@@ -177,8 +177,11 @@ __device__ __forceinline__ uint32_t sw128_off4(uint32_t t, uint32_t i0) {
 // diagonal halves), each output thread forming four adjacent columns from
 // 16-byte loads.  s_t and 1 / s_t go to s_s, s_is.  Called by the kMain
 // threads tid = 0 .. kMain - 1 of warps 4-15 (named-barrier synchronisation).
+template <class Side>
 __device__ __forceinline__ void wy_inverse(int tid, const float *sT, float *sA, float *sX, float *sY,
-                                           const float *s_r, float *s_s, float *s_is) {
+                                           const float *s_r, float *s_s, float *s_is,
+                                           unsigned char *awu, Side side) {
+  const int w = tid >> 5;  // main warp 0 .. 11 (lane quarter w & 3)
   if (tid < 64) {
     // column c of D_I: x_r = (delta_rc - sum_{m<r} L_rm x_m) / L_rr, rows read 16 bytes at a time
     const int o = 16 * (tid >> 4), c = tid & 15;
@@ -209,9 +212,12 @@ __device__ __forceinline__ void wy_inverse(int tid, const float *sT, float *sA, 
     float *ab = sA + o * (LT + 1) + c;
 #pragma unroll
     for (int r = 0; r < 16; ++r) ab[r * LT] = x[r];
+  } else if ((w & 3) < 2) {
+    side();  // warps 4, 5, 8, 9 of the main group (lane quarters 0, 1)
   } else {
     // zero the strictly upper 16 x 16 blocks (I < J): 6 blocks x 16 rows x 4 float4
-    for (int e = tid - 64; e < 384; e += kMain - 64) {
+    const int z = 64 * (w >> 2) + 32 * ((w & 3) - 2) + (tid & 31);  // 0 .. 191
+    for (int e = z; e < 384; e += 192) {
       const int blk = e >> 6, rr = (e >> 2) & 15, q4 = e & 3;
       const int I = blk < 3 ? 0 : (blk < 5 ? 1 : 2);
       const int J = blk < 3 ? blk + 1 : (blk < 5 ? blk - 1 : 3);
@@ -260,7 +266,7 @@ __device__ __forceinline__ void wy_inverse(int tid, const float *sT, float *sA, 
     *reinterpret_cast<float4 *>(sA + (R0 + r2) * LT + C0 + cq2) = make_float4(-acc.x, -acc.y, -acc.z, -acc.w);
   }
   bar_sync(kBarMain, kMain);
-  // Y = L21 X11, then X_21 = -X22 Y (32 x 32 x 32 each): one thread per (row, 4 columns)
+  // Y = L21 X11 (32 x 32 x 32): one thread per (row, 4 columns)
   const int r3 = tid >> 3, cq3 = 4 * (tid & 7);
   if (tid < 256) {
     const float *tp = sT + (32 + r3) * LT;
@@ -281,6 +287,8 @@ __device__ __forceinline__ void wy_inverse(int tid, const float *sT, float *sA, 
     *reinterpret_cast<float4 *>(sY + r3 * 32 + cq3) = acc;
   }
   bar_sync(kBarMain, kMain);
+  // T' is dead from here on: [A; 0] fp16 [128 t][64 s] (A = diag(s) L^-1) is written over it.
+  // X_21 = -X22 Y by threads 0..255, straight to fp16; threads 256..383 convert the rest.
   if (tid < 256) {
     const float *dp = sA + (32 + r3) * LT + 32;
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
@@ -297,9 +305,39 @@ __device__ __forceinline__ void wy_inverse(int tid, const float *sT, float *sA, 
         acc.w = fmaf(dv[u], y4.w, acc.w);
       }
     }
-    *reinterpret_cast<float4 *>(sA + (32 + r3) * LT + cq3) = make_float4(-acc.x, -acc.y, -acc.z, -acc.w);
+    const int r = 32 + r3;
+    const float sr = -s_s[r];
+    *reinterpret_cast<uint2 *>(awu + chunk_off(r, cq3 >> 3) + 2 * (cq3 & 4)) =
+        pack_h4(sr * acc.x, sr * acc.y, sr * acc.z, sr * acc.w);
+  } else {
+    // rows 0..31 (8 column chunks), rows 32..63 columns 32..63 (4 chunks), rows 64..127 zero
+    for (int e = tid - 256; e < 896; e += 128) {
+      int r, cc;
+      if (e < 256) {
+        r = e >> 3;
+        cc = e & 7;
+      } else if (e < 384) {
+        r = 32 + ((e - 256) >> 2);
+        cc = 4 + (e & 3);
+      } else {
+        r = 64 + ((e - 384) >> 3);
+        cc = e & 7;
+      }
+      float v[8];
+      if (r < 64) {
+        const float sr = s_s[r];
+        const float4 a0 = *reinterpret_cast<const float4 *>(sA + r * LT + 8 * cc);
+        const float4 a1 = *reinterpret_cast<const float4 *>(sA + r * LT + 8 * cc + 4);
+        const float av[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
+#pragma unroll
+        for (int j = 0; j < 8; ++j) v[j] = (8 * cc + j <= r) ? sr * av[j] : 0.f;
+      } else {
+#pragma unroll
+        for (int j = 0; j < 8; ++j) v[j] = 0.f;
+      }
+      sm16(awu, chunk_off(r, cc)) = pack_h8(v);
+    }
   }
-  bar_sync(kBarMain, kMain);
 }
 
 struct WyParams {
@@ -323,7 +361,7 @@ __global__ void __launch_bounds__(WT, 1)
   extern __shared__ unsigned char smraw[];
   unsigned char *sm =
       reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(smraw) + 1023) & ~uintptr_t(1023));
-  unsigned char *rk = sm + O_RK, *rg = sm + O_RG, *rw = sm + O_RW, *vr = sm + O_V;
+  unsigned char *rk = sm + O_RK, *rg = sm + O_RG, *rw = sm + O_RW, *vr = sm + O_V, *rq = sm + O_Q;
   unsigned char *ta = sm + O_TA, *tb = sm + O_TB, *as1 = sm + O_AS1;
   unsigned char *s16 = sm + O_S16, *awu = sm + O_AWU;
   float *sT = reinterpret_cast<float *>(sm + O_SWT), *sA = reinterpret_cast<float *>(sm + O_SWA);
@@ -370,7 +408,7 @@ __global__ void __launch_bounds__(WT, 1)
                  TU = tbase + TC_U;
 
   // k, g, omega of chunk c (the gain and the preparing pass), q of chunk c (the
-  // preparing pass, in the V buffer), V of chunk c (after the preparing pass)
+  // preparing pass), V of chunk c (once MMA-O / MMA-S2 of chunk c - 1 has read R')
   auto issue_raw = [&](int c) {
     mbar_expect_tx(bar_raw, 49152);
     for (int s = 0; s < 2; ++s) {
@@ -381,7 +419,7 @@ __global__ void __launch_bounds__(WT, 1)
   };
   auto issue_q = [&](int c) {
     mbar_expect_tx(bar_q, 16384);
-    for (int s = 0; s < 2; ++s) tma_load_4d(vr + s * 8192, &mq, bar_q, 64 * s, h, c * CM, b);
+    for (int s = 0; s < 2; ++s) tma_load_4d(rq + s * 8192, &mq, bar_q, 64 * s, h, c * CM, b);
   };
   auto issue_v = [&](int c) {
     mbar_expect_tx(bar_v, 16384);
@@ -390,7 +428,15 @@ __global__ void __launch_bounds__(WT, 1)
   if (issuer && NC > 0) {
     issue_raw(0);
     issue_q(0);
-    for (int s = 0; s < 2; ++s) tma_prefetch_4d(&mv, 64 * s, h, 0, b);
+    issue_v(0);
+    if (NC > 1) {
+      for (int s = 0; s < 2; ++s) {
+        tma_prefetch_4d(&mk, 64 * s, h, CM, b);
+        tma_prefetch_4d(&mg, 64 * s, h, CM, b);
+        tma_prefetch_4d(&mw, 64 * s, h, CM, b);
+        tma_prefetch_4d(&mq, 64 * s, h, CM, b);
+      }
+    }
   }
 
   // initial memory S_0 -> TMEM (row = key channel i, column = value j)
@@ -552,12 +598,12 @@ __global__ void __launch_bounds__(WT, 1)
     const uint32_t tkt = TKT + (uint32_t)((c & 1) * 32);
     unsigned char *ctx = SV ? P.save_S + ((size_t)bh * NC + c) * kCtxBytes : nullptr;
     if (SV && issuer) bulk_wait_read();  // the previous chunk's context tiles have left shared memory
-    // ---- [0] the previous chunk's MMA-O / MMA-S2 must be done before q is brought
+    // ---- [0] the previous chunk's MMA-O / MMA-S2 must be done before V is brought
     //          into its R' buffer; the gain of this chunk is done (its warps arrive here)
     if (!gain) mine = mbar_wait(bar_raw, c & 1, kWait) && mine;
     if (issuer && c > 0) {
       mine = mma_wait_main() && mine;  // MMA-O / MMA-S2 of chunk c - 1
-      if (mine) issue_q(c);
+      if (mine) issue_v(c);
     } else if (!gain && c > 0) {
       ++mph;
     }
@@ -607,7 +653,7 @@ __global__ void __launch_bounds__(WT, 1)
         float gv[4], kv[4], qv[4], e[4];
         unpack_bf4(gq[j], gv);
         unpack_bf4(*reinterpret_cast<const uint2 *>(rk + sl8 + sw128_off4(t, i0)), kv);
-        unpack_bf4(*reinterpret_cast<const uint2 *>(vr + sl8 + sw128_off4(t, i0)), qv);
+        unpack_bf4(*reinterpret_cast<const uint2 *>(rq + sl8 + sw128_off4(t, i0)), qv);
 #pragma unroll
         for (int u = 0; u < 4; ++u) {
           G[u] += gv[u];
@@ -659,7 +705,7 @@ __global__ void __launch_bounds__(WT, 1)
       break;
     }
 
-    // ---- [2] MMA-T; the next chunk's k, g, omega; this chunk's V over q
+    // ---- [2] MMA-T; the next chunk's k, g, omega and q
     if (issuer) {
       tc_fence_after();
       const uint32_t A0 = smem_u32(ta), B0 = smem_u32(tb);
@@ -667,12 +713,17 @@ __global__ void __launch_bounds__(WT, 1)
         umma_tf32(TD1, sw128_desc(A0 + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024),
                   sw128_desc(B0 + (kk >> 2) * 8192 + (kk & 3) * 32, 16, 1024), id_T, kk > 0);
       umma_commit(bar_t);
-      issue_v(c);
       if (c + 1 < NC) {
         issue_raw(c + 1);
+        issue_q(c + 1);
+        for (int s = 0; s < 2; ++s) tma_prefetch_4d(&mv, 64 * s, h, (c + 1) * CM, b);
+      }
+      if (c + 2 < NC) {  // chunk c + 2 into L2: its tiles are loaded during chunk c + 1
         for (int s = 0; s < 2; ++s) {
-          tma_prefetch_4d(&mq, 64 * s, h, (c + 1) * CM, b);
-          tma_prefetch_4d(&mv, 64 * s, h, (c + 1) * CM, b);
+          tma_prefetch_4d(&mk, 64 * s, h, (c + 2) * CM, b);
+          tma_prefetch_4d(&mg, 64 * s, h, (c + 2) * CM, b);
+          tma_prefetch_4d(&mw, 64 * s, h, (c + 2) * CM, b);
+          tma_prefetch_4d(&mq, 64 * s, h, (c + 2) * CM, b);
         }
       }
     }
@@ -751,23 +802,31 @@ __global__ void __launch_bounds__(WT, 1)
     }
 
     // ---- [4] A = (I + T)^-1 = diag(s) L^-1 with L = diag(s) + strict_lower(T')
-    //          (T = strict_lower(T') diag(1/s)), then [A; 0] fp16 over T'
-    wy_inverse(mt, sT, sA, sX, sY, s_r + 64 * (c & 1), s_s, s_is);
-    for (int e = mt; e < 1024; e += kMain) {
-      const int r = e >> 3, cc = e & 7;
-      float v[8];
-      if (r < 64) {
-        const float sr = s_s[r];
-        const float4 a0 = *reinterpret_cast<const float4 *>(sA + r * LT + 8 * cc);
-        const float4 a1 = *reinterpret_cast<const float4 *>(sA + r * LT + 8 * cc + 4);
-        const float av[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
+    //          (T = strict_lower(T') diag(1/s)), then [A; 0] fp16 over T';
+    //          Y = V - Kbar S_in (rows 0..63 of TU plus V) -> fp16 in place over V, by warps
+    //          8, 9, 12, 13 while warps 4, 5 solve the diagonal blocks
+    {
+      auto y_side = [&]() {
+        const bool ks_ok = mma_wait_main();  // MMA-KS
+        const bool v_ok = mbar_wait(bar_v, c & 1, kWait);
+        mine = ks_ok && v_ok && mine;
+        tc_fence_after();
+        const int t = 32 * wq + lane;
+        for (int g = wgm - 1; g < 8; g += 2) {
+          float v[16], vv[16];
+          const int j0 = 16 * g, sl = j0 >> 6, cc0 = (j0 & 63) >> 3;
+          tmem_ld16(TU + lane_base + j0, v);
+          const uint32_t o0 = sl * 8192 + chunk_off(t, cc0), o1 = sl * 8192 + chunk_off(t, cc0 + 1);
+          unpack_bf8(sm16(vr, o0), vv);
+          unpack_bf8(sm16(vr, o1), vv + 8);
 #pragma unroll
-        for (int j = 0; j < 8; ++j) v[j] = (8 * cc + j <= r) ? sr * av[j] : 0.f;
-      } else {
-#pragma unroll
-        for (int j = 0; j < 8; ++j) v[j] = 0.f;
-      }
-      sm16(awu, chunk_off(r, cc)) = pack_h8(v);
+          for (int u = 0; u < 16; ++u) v[u] += vv[u];
+          sm16(vr, o0) = pack_h8(v);
+          sm16(vr, o1) = pack_h8(v + 8);
+        }
+      };
+      wy_inverse(mt, sT, sA, sX, sY, s_r + 64 * (c & 1), s_s, s_is, awu, y_side);
+      if (!(wq < 2 && wgm >= 1)) ++mph;  // MMA-KS, observed by the Y warps
     }
     if (SV) {
       if (wq >= 2 && wgm == 0) {  // A_qk = lower(A'_qk) diag(1/s) into the context
@@ -809,28 +868,7 @@ __global__ void __launch_bounds__(WT, 1)
         umma_commit(bar_w);  // its own barrier: MMA-KS may not have been observed yet
       }
     }
-    // ---- [6] Y = V - Kbar S_in (rows 0..63 of TU plus V) -> fp16 in place over V
-    {
-      const bool ks_ok = mma_wait_main();  // MMA-KS
-      const bool v_ok = mbar_wait(bar_v, c & 1, kWait);
-      mine = ks_ok && v_ok && mine;
-      tc_fence_after();
-      if (wq < 2) {
-        const int t = 32 * wq + lane;
-        for (int g = wgm; g < 8; g += 3) {
-          float v[16], vv[16];
-          const int j0 = 16 * g, sl = j0 >> 6, cc0 = (j0 & 63) >> 3;
-          tmem_ld16(TU + lane_base + j0, v);
-          const uint32_t o0 = sl * 8192 + chunk_off(t, cc0), o1 = sl * 8192 + chunk_off(t, cc0 + 1);
-          unpack_bf8(sm16(vr, o0), vv);
-          unpack_bf8(sm16(vr, o1), vv + 8);
-#pragma unroll
-          for (int u = 0; u < 16; ++u) v[u] += vv[u];
-          sm16(vr, o0) = pack_h8(v);
-          sm16(vr, o1) = pack_h8(v + 8);
-        }
-      }
-    }
+    // ---- [6] (context only) -W out of TMEM
     if (SV) {  // -W of the context (rows 0..63 of TW), once MMA-W has completed
       mine = mbar_wait(bar_w, c & 1, kWait) && mine;
       tc_fence_after();
@@ -844,10 +882,9 @@ __global__ void __launch_bounds__(WT, 1)
           *reinterpret_cast<uint4 *>(ctx + kCtxW + sl * 8192 + chunk_off(t, cc0 + 1)) = pack_h8(v + 8);
         }
       }
+      tc_fence_before();
+      bar_sync(kBarMain, kMain);  // TW is free for MMA-R
     }
-    fence_proxy_async();
-    tc_fence_before();
-    bar_sync(kBarMain, kMain);
 
     // ---- [7] MMA-R: TW = [A; 0] Y = [R; 0]  (fp16)
     if (issuer) {
