@@ -76,11 +76,13 @@ typedef enum {
   KDN_ERR_TIMEOUT = 5,     /* a bounded device-side wait gave up */
   KDN_ERR_RANGE = 6        /* device status only: a 64-token chunk's cumulative log-decay
                               G_C left a fused kernel's range in some channel (results of
-                              that call are invalid).  The plain bf16 d = 128 diagonal
-                              forward takes G_C >= -160; the calls that write or read the
-                              backward context (the *_fwd_save / *_bwd_saved pairs, the
-                              other fused forwards) take exp(G_C) >= 1e-36, G_C >= -82.8.
-                              desc->chunk = 32 halves the exposure. */
+                              that call are invalid).  The single-pass bf16 d = 128
+                              diagonal forward (kdn_diag_fwd) takes any decay.  The calls
+                              that write or read the backward context (the *_fwd_save /
+                              *_bwd_saved pairs, the fused backwards), the isotropic fused
+                              forward and the sequence-parallel forward take
+                              exp(G_C) >= 1e-36, G_C >= -82.8.  desc->chunk = 32 halves
+                              the exposure. */
 } kdn_status_t;
 
 typedef enum { KDN_F32 = 0, KDN_BF16 = 1 } kdn_dtype_t;

@@ -42,11 +42,23 @@
 //
 // Range: the referenced factors stay finite while the chunk's cumulative
 // log-decay G_C >= -160 in every channel (average alpha >= 0.082 over 64
-// tokens).  A chunk below that records KDN_ERR_RANGE in the status word.
+// tokens).  A chunk below that (flagged by the gain warps, for every channel
+// at once) runs in range mode: the main warps form T' and A'_qk on the CUDA
+// cores from exp(G_t - G_s), s <= t, which never exceeds 1, in place of MMA-T;
+// gamma_t and K' are then formed from G_t directly.  The context-saving
+// instantiation keeps the referenced form (the fused backward it feeds divides
+// by gamma and reports exp(G_C) < 1e-36 as KDN_ERR_RANGE).
+//
+// Logit gates (LG): g, omega, r hold the logits x, y, z of the layer's
+// parameterisation (Sec. 5): log alpha = -softplus(-x), omega = softplus(y),
+// r = r_min + softplus(z), formed in float32 where each is read; the tokens
+// past T are identity updates.
 //
 // Every wait on an mbarrier is bounded; on timeout the kernel records
 // KDN_ERR_TIMEOUT in the status word, waits (bounded) for its copies in flight,
 // frees its tensor memory and returns.
+#include <type_traits>
+
 #include "kdn_internal.cuh"
 #include "kdn_sm103.cuh"
 #include "kdn_fused_common.cuh"
@@ -87,7 +99,7 @@ static_assert(O_SWA + 64 * LT * 4 <= O_TB, "T and A tiles overlap the Kk' tile")
 constexpr int O_AWU = O_SWT;           // fp16 [A; 0] [128][64] (MMA-R A), over T' after the solve
 // small arrays (floats); r and mu / r per token for two chunks (the gain works one chunk ahead)
 constexpr int SM_R = 0, SM_MUR = 128, SM_S = 256, SM_IS = 320, SM_C = 384, SM_GC = 512,
-              SM_PART = 640, SM_FLOATS = 640 + 8 * 128;
+              SM_PART = 640, SM_OOR = 640 + 8 * 128, SM_FLOATS = SM_OOR + 16;
 constexpr int O_BAR = O_SMALL + SM_FLOATS * 4;
 constexpr int O_SX = O_BAR + 64;       // scratch of the solve: 2 x 256 floats
 constexpr int O_SY = O_SX + 2048;      //                       32 x 32 floats
@@ -120,6 +132,17 @@ __device__ __forceinline__ uint32_t sw32_off(uint32_t row, uint32_t col) {
 }
 __device__ __forceinline__ void bar_sync(int id, int n) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory");
+}
+// named barrier that also returns the OR of a predicate over its n threads
+__device__ __forceinline__ bool bar_or(int id, int n, bool p) {
+  uint32_t r;
+  asm volatile(
+      "{\n .reg .pred pi, po;\n setp.ne.u32 pi, %1, 0;\n barrier.cta.red.or.pred po, %2, %3, pi;\n"
+      " selp.u32 %0, 1, 0, po;\n}"
+      : "=r"(r)
+      : "r"((uint32_t)p), "r"(id), "r"(n)
+      : "memory");
+  return r != 0;
 }
 __host__ __device__ constexpr uint32_t idesc_tf32(int M, int N) {
   return (1u << 4) | (2u << 7) | (2u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
@@ -340,6 +363,67 @@ __device__ __forceinline__ void wy_inverse(int tid, const float *sT, float *sA, 
   }
 }
 
+// fp32 G_t of the range mode: [64 t][128 i], 512-byte rows, 16-byte groups of four
+// channels XOR-swizzled by the row
+__device__ __forceinline__ uint32_t g_off(int t, int i4) {
+  return (uint32_t)t * 512u + ((uint32_t)(i4 ^ (t & 31)) << 4);
+}
+
+// Range mode: a chunk whose cumulative log-decay leaves the range of the
+// referenced factors (G_C < -160 in some channel) forms
+//   T'_ts   = sum_i k_t,i phat_s,i k_s,i exp(G_t,i - G_s,i)
+//   A'qk_ts = tau sum_i q_t,i phat_s,i k_s,i exp(G_t,i - G_s,i)      (s <= t)
+// from the cumulative log-decay differences themselves (App. F.2): every ratio
+// exp(G_t - G_s), s <= t, lies in (0, 1].  Inputs: raw k, q (bf16 tiles), G (fp32,
+// g_off layout) and phat k (fp32 in the layout of the Kk' tile).  Outputs: T' into
+// sT and A'_qk into sA (fp32 [64][LT]), zero above the diagonal.  One thread per
+// (row t, group of four columns); rows t and 63 - t together have 17 groups.
+__device__ __noinline__ void direct_products(int tid, const unsigned char *rk, const unsigned char *rq,
+                                                const unsigned char *gbuf, const unsigned char *tb,
+                                                float tau, float *sT, float *sA) {
+  for (int e = tid; e < 32 * 17; e += kMain) {
+    const int pr = e / 17, j = e - 17 * pr, n0 = (pr >> 2) + 1;
+    const int t = j < n0 ? pr : 63 - pr;
+    const int s0 = 4 * (j < n0 ? j : j - n0);
+    float aT[4] = {0.f, 0.f, 0.f, 0.f}, aQ[4] = {0.f, 0.f, 0.f, 0.f};
+    for (int i4 = 0; i4 < 32; ++i4) {
+      const int i0 = 4 * i4;
+      const uint32_t sl8 = (uint32_t)(i0 >> 6) * 8192u;
+      float kv[4], qv[4];
+      unpack_bf4(*reinterpret_cast<const uint2 *>(rk + sl8 + sw128_off4(t, i0)), kv);
+      unpack_bf4(*reinterpret_cast<const uint2 *>(rq + sl8 + sw128_off4(t, i0)), qv);
+      const float4 gt = *reinterpret_cast<const float4 *>(gbuf + g_off(t, i4));
+      const unsigned char *pkb = tb + (i0 >> 5) * 8192;
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int sidx = s0 + u;
+        const float4 gs = *reinterpret_cast<const float4 *>(gbuf + g_off(sidx, i4));
+        const float4 pk = *reinterpret_cast<const float4 *>(pkb + sw32_off(sidx, i0 & 31));
+        // columns above the diagonal are clamped to finite values and masked below
+        const float e0 = ex2f(fminf(gt.x - gs.x, 0.f) * kLog2e) * pk.x;
+        const float e1 = ex2f(fminf(gt.y - gs.y, 0.f) * kLog2e) * pk.y;
+        const float e2 = ex2f(fminf(gt.z - gs.z, 0.f) * kLog2e) * pk.z;
+        const float e3 = ex2f(fminf(gt.w - gs.w, 0.f) * kLog2e) * pk.w;
+        aT[u] = fmaf(kv[0], e0, fmaf(kv[1], e1, fmaf(kv[2], e2, fmaf(kv[3], e3, aT[u]))));
+        aQ[u] = fmaf(qv[0], e0, fmaf(qv[1], e1, fmaf(qv[2], e2, fmaf(qv[3], e3, aQ[u]))));
+      }
+    }
+    *reinterpret_cast<float4 *>(sT + t * LT + s0) =
+        make_float4(s0 <= t ? aT[0] : 0.f, s0 + 1 <= t ? aT[1] : 0.f, s0 + 2 <= t ? aT[2] : 0.f,
+                    s0 + 3 <= t ? aT[3] : 0.f);
+    *reinterpret_cast<float4 *>(sA + t * LT + s0) =
+        make_float4(s0 <= t ? tau * aQ[0] : 0.f, s0 + 1 <= t ? tau * aQ[1] : 0.f,
+                    s0 + 2 <= t ? tau * aQ[2] : 0.f, s0 + 3 <= t ? tau * aQ[3] : 0.f);
+  }
+  for (int e = tid; e < 64 * 16; e += kMain) {
+    const int t = e >> 4, s0 = 4 * (e & 15);
+    if (s0 > t) {
+      *reinterpret_cast<float4 *>(sT + t * LT + s0) = make_float4(0.f, 0.f, 0.f, 0.f);
+      *reinterpret_cast<float4 *>(sA + t * LT + s0) = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+  }
+}
+
 struct WyParams {
   Args a;
   unsigned char *save_S;  // SV: [BH][NC] context records of the backward (kCtxBytes each)
@@ -352,7 +436,7 @@ struct WyParams {
 // phat and gamma in float32 [64 t][128 i], s_t per token, and the uncertainty
 // entering the chunk.  The arithmetic is the same with and without it.
 
-template <int SV>
+template <int SV, int LG>  // LG: g, omega, r hold the logits x, y, z of the gates
 __global__ void __launch_bounds__(WT, 1)
     k_wy_fwd(const __grid_constant__ CUtensorMap mk, const __grid_constant__ CUtensorMap mg,
              const __grid_constant__ CUtensorMap mw, const __grid_constant__ CUtensorMap mv,
@@ -369,6 +453,8 @@ __global__ void __launch_bounds__(WT, 1)
   float *sf = reinterpret_cast<float *>(sm + O_SMALL);
   float *s_r = sf + SM_R, *s_mur = sf + SM_MUR, *s_s = sf + SM_S, *s_is = sf + SM_IS;
   float *s_c = sf + SM_C, *s_gC = sf + SM_GC, *s_part = sf + SM_PART;
+  // per chunk (slot c & 1): some channel's decay left the range of the referenced factors
+  int *s_oor = reinterpret_cast<int *>(sf + SM_OOR);
   uint64_t *bars = reinterpret_cast<uint64_t *>(sm + O_BAR);
   uint64_t *bar_raw = bars, *bar_v = bars + 1, *bar_mma = bars + 2, *bar_q = bars + 3;
   uint64_t *bar_t = bars + 4;  // MMA-T completions (one a chunk)
@@ -474,7 +560,10 @@ __global__ void __launch_bounds__(WT, 1)
   auto load_r = [&](int c) {
     if (tid < CM) {
       rnext = 1.f;
-      if (c < NC && c * CM + tid < a.T) rnext = ld<__nv_bfloat16>(a.r, tok_index(a, b, c * CM + tid, h));
+      if (c < NC && c * CM + tid < a.T) {
+        const float z = ld<__nv_bfloat16>(a.r, tok_index(a, b, c * CM + tid, h));
+        rnext = LG ? a.rmin + softplus_f(z) : z;  // r = r_min + softplus(z) (Sec. 5)
+      }
     }
   };
   load_r(0);
@@ -508,17 +597,27 @@ __global__ void __launch_bounds__(WT, 1)
     auto raw = [&](const unsigned char *base, int t) {
       return __bfloat162float(*reinterpret_cast<const __nv_bfloat16 *>(base + sw128_off(t, cl)));
     };
+    // log alpha and omega of token t (logit gates: the tokens past T are identity updates)
+    const int tv = a.T - c * CM;
+    auto lga = [&](float x, int t) { return LG ? (t < tv ? -softplus_f(-x) : 0.f) : x; };
+    auto omg = [&](float y, int t) { return LG ? (t < tv ? softplus_f(y) : 0.f) : y; };
     float g0 = 0.f, g1 = 0.f, g2 = 0.f, g3 = 0.f;
 #pragma unroll
     for (int t = 0; t < CM; t += 4) {
-      g0 += raw(pg, t);
-      g1 += raw(pg, t + 1);
-      g2 += raw(pg, t + 2);
-      g3 += raw(pg, t + 3);
+      g0 += lga(raw(pg, t), t);
+      g1 += lga(raw(pg, t + 1), t + 1);
+      g2 += lga(raw(pg, t + 2), t + 2);
+      g3 += lga(raw(pg, t + 3), t + 3);
     }
     const float GC = (g0 + g1) + (g2 + g3), cref = 0.5f * GC;
     s_c[i] = cref;
-    if (cref < kMinHalfG) atomicCAS(a.status, 0u, (unsigned)KDN_ERR_RANGE);
+    // out of the referenced factors' range in some channel: this chunk forms T' and A'_qk
+    // from exp(G_t - G_s) directly
+    // (the training forward keeps the referenced form: its context feeds a backward
+    // that needs exp(G_C) >= 1e-36, and such chunks are reported instead)
+    const bool oor = !SV && bar_or(kBarGain, 128, cref < kMinHalfG);
+    if (tid == 0) s_oor[sb] = oor ? 1 : 0;
+    float Gt = 0.f;  // G_t of this channel (range mode)
     unsigned char *gctx = SV ? P.save_S + ((size_t)bh * NC + c) * kCtxBytes : nullptr;
     if (SV) P.save_p[((size_t)bh * NC + c) * D + i] = p;
     float *cph = SV ? reinterpret_cast<float *>(gctx + kCtxPh) + i : nullptr;
@@ -530,8 +629,8 @@ __global__ void __launch_bounds__(WT, 1)
     float gb[8], wb[8], kb8[8], mb[8];
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
-      gb[j] = raw(pg, j);
-      wb[j] = raw(pw, j);
+      gb[j] = lga(raw(pg, j), j);
+      wb[j] = omg(raw(pw, j), j);
       kb8[j] = raw(pk, j);
     }
     {
@@ -541,47 +640,74 @@ __global__ void __launch_bounds__(WT, 1)
     if (c > 0) g_ok = mbar_wait(bar_t, (c - 1) & 1, kWait) && g_ok;  // Kk' of chunk c - 1 has been read
     // the chunk in blocks of 8 tokens; the next block's inputs are loaded
     // before the current block's outputs are stored
-#pragma unroll
-    for (int blk = 0; blk < 8; ++blk) {
-      float gn[8], wn[8], kn[8], mn[8];
-      if (blk < 7) {
+    if (oor) {
+      // range mode (rare): Kk' is replaced by phat k itself, and K' is formed from G_t
+      // directly; a compact loop without the prefetching of the referenced mode
+#pragma unroll 1
+      for (int blk = 0; blk < 8; ++blk) {
+        uint32_t kt[4];
 #pragma unroll
         for (int j = 0; j < 8; ++j) {
-          const int t = 8 * (blk + 1) + j;
-          gn[j] = raw(pg, t);
-          wn[j] = raw(pw, t);
-          kn[j] = raw(pk, t);
+          const int t = 8 * blk + j;
+          const float lg = lga(raw(pg, t), t), kk = raw(pk, t);
+          const float al = ex2f(lg * kLog2e);
+          const float ph = fmaf(al * al, p, omg(raw(pw, t), t));
+          const float den = fmaf(kk * kk * smur[t], ph, 1.f);
+          p = ph * rcpf(den);
+          Gt += lg;
+          const float pkv = ph * kk;
+          if (SV) cph[t * D] = ph;
+          *reinterpret_cast<float *>(pb + sw32_off(t, cb)) = pkv;
+          const uint32_t hb =
+              (uint32_t)__half_as_ushort(__float2half_rn(pkv * ex2f((GC - Gt) * kLog2e)));
+          if ((j & 1) == 0) kt[j >> 1] = hb;
+          else kt[j >> 1] |= hb << 16;
         }
-        const float4 m0 = *reinterpret_cast<const float4 *>(smur + 8 * (blk + 1));
-        const float4 m1 = *reinterpret_cast<const float4 *>(smur + 8 * (blk + 1) + 4);
-        mn[0] = m0.x; mn[1] = m0.y; mn[2] = m0.z; mn[3] = m0.w; mn[4] = m1.x; mn[5] = m1.y; mn[6] = m1.z; mn[7] = m1.w;
+        tmem_st4u(tkt + lane_base + (uint32_t)(4 * blk), kt);
       }
-      uint32_t kt[4];
+    } else {
 #pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        const int t = 8 * blk + j;
-        const float al = ex2f(gb[j] * kLog2e), a2 = al * al;
-        const float ph = fmaf(a2, p, wb[j]);               // eq. diag-covariance-prediction
-        const float u = kb8[j] * kb8[j] * mb[j];
-        const float den = fmaf(u, ph, 1.f);
-        const float x = rcpf(al * den);
-        p = ph * (x * al);                                  // eq. prefix-diag-uncertainty
-        f *= x * den;                                       // / alpha_t
-        const float pkv = ph * kb8[j];
-        if (SV) cph[t * D] = ph;
-        *reinterpret_cast<float *>(pb + sw32_off(t, cb)) = tf32r(pkv * f);
-        const uint32_t hb = (uint32_t)__half_as_ushort(__float2half_rn(pkv * (f * E2)));
-        if ((j & 1) == 0) kt[j >> 1] = hb;
-        else kt[j >> 1] |= hb << 16;
-      }
-      tmem_st4u(tkt + lane_base + (uint32_t)(4 * blk), kt);
-      if (blk < 7) {
+      for (int blk = 0; blk < 8; ++blk) {
+        float gn[8], wn[8], kn[8], mn[8];
+        if (blk < 7) {
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const int t = 8 * (blk + 1) + j;
+            gn[j] = lga(raw(pg, t), t);
+            wn[j] = omg(raw(pw, t), t);
+            kn[j] = raw(pk, t);
+          }
+          const float4 m0 = *reinterpret_cast<const float4 *>(smur + 8 * (blk + 1));
+          const float4 m1 = *reinterpret_cast<const float4 *>(smur + 8 * (blk + 1) + 4);
+          mn[0] = m0.x; mn[1] = m0.y; mn[2] = m0.z; mn[3] = m0.w; mn[4] = m1.x; mn[5] = m1.y; mn[6] = m1.z; mn[7] = m1.w;
+        }
+        uint32_t kt[4];
 #pragma unroll
         for (int j = 0; j < 8; ++j) {
-          gb[j] = gn[j];
-          wb[j] = wn[j];
-          kb8[j] = kn[j];
-          mb[j] = mn[j];
+          const int t = 8 * blk + j;
+          const float al = ex2f(gb[j] * kLog2e), a2 = al * al;
+          const float ph = fmaf(a2, p, wb[j]);               // eq. diag-covariance-prediction
+          const float u = kb8[j] * kb8[j] * mb[j];
+          const float den = fmaf(u, ph, 1.f);
+          const float x = rcpf(al * den);
+          p = ph * (x * al);                                  // eq. prefix-diag-uncertainty
+          f *= x * den;                                       // / alpha_t
+          const float pkv = ph * kb8[j];
+          if (SV) cph[t * D] = ph;
+          *reinterpret_cast<float *>(pb + sw32_off(t, cb)) = tf32r(pkv * f);
+          const uint32_t hb = (uint32_t)__half_as_ushort(__float2half_rn(pkv * (f * E2)));
+          if ((j & 1) == 0) kt[j >> 1] = hb;
+          else kt[j >> 1] |= hb << 16;
+        }
+        tmem_st4u(tkt + lane_base + (uint32_t)(4 * blk), kt);
+        if (blk < 7) {
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            gb[j] = gn[j];
+            wb[j] = wn[j];
+            kb8[j] = kn[j];
+            mb[j] = mn[j];
+          }
         }
       }
     }
@@ -623,11 +749,20 @@ __global__ void __launch_bounds__(WT, 1)
       // the chunk's g for this thread's 8 tokens and 4 channels (8 bytes a token)
       uint2 gq[8];
       float ps[4] = {0.f, 0.f, 0.f, 0.f};
+      const int tv = a.T - c * CM;  // logit gates: tokens past T are identity updates
+      const bool oor = !SV && s_oor[c & 1] != 0;
+      auto unpack_lga = [&](uint2 u, int t, float *gv) {
+        unpack_bf4(u, gv);
+        if (LG) {
+#pragma unroll
+          for (int w = 0; w < 4; ++w) gv[w] = t < tv ? -softplus_f(-gv[w]) : 0.f;
+        }
+      };
 #pragma unroll
       for (int j = 0; j < 8; ++j) {
         gq[j] = *reinterpret_cast<const uint2 *>(rg + sl8 + sw128_off4(t0 + j, i0));
         float gv[4];
-        unpack_bf4(gq[j], gv);
+        unpack_lga(gq[j], t0 + j, gv);
 #pragma unroll
         for (int u = 0; u < 4; ++u) ps[u] += gv[u];
       }
@@ -647,32 +782,47 @@ __global__ void __launch_bounds__(WT, 1)
       mine = mbar_wait(bar_q, c & 1, kWait) && mine;
       unsigned char *pa = ta + (i0 >> 5) * 16384, *pqh = as1 + (i0 >> 6) * 16384;
       const int cc = i0 & 31;
+      auto prep_loop = [&](auto range_mode) {
+        constexpr bool RM = decltype(range_mode)::value;
 #pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        const int t = t0 + j;
-        float gv[4], kv[4], qv[4], e[4];
-        unpack_bf4(gq[j], gv);
-        unpack_bf4(*reinterpret_cast<const uint2 *>(rk + sl8 + sw128_off4(t, i0)), kv);
-        unpack_bf4(*reinterpret_cast<const uint2 *>(rq + sl8 + sw128_off4(t, i0)), qv);
+        for (int j = 0; j < 8; ++j) {
+          const int t = t0 + j;
+          float gv[4], kv[4], qv[4], e[4];
+          unpack_lga(gq[j], t, gv);
+          unpack_bf4(*reinterpret_cast<const uint2 *>(rk + sl8 + sw128_off4(t, i0)), kv);
+          unpack_bf4(*reinterpret_cast<const uint2 *>(rq + sl8 + sw128_off4(t, i0)), qv);
+          if constexpr (RM) {  // G_t itself for the direct products; gamma_t = exp(G_t) (may underflow)
 #pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          G[u] += gv[u];
-          e[u] = ex2f((G[u] - cr[u]) * kLog2e);
-          gm[u] = e[u] * Ec[u];
-          qv[u] *= a.tau;
+            for (int u = 0; u < 4; ++u) {
+              G[u] += gv[u];
+              gm[u] = ex2f(G[u] * kLog2e);
+              qv[u] *= a.tau;
+            }
+            *reinterpret_cast<float4 *>(ta + g_off(t, i0 >> 2)) = make_float4(G[0], G[1], G[2], G[3]);
+          } else {
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+              G[u] += gv[u];
+              e[u] = ex2f((G[u] - cr[u]) * kLog2e);
+              gm[u] = e[u] * Ec[u];
+              qv[u] *= a.tau;
+            }
+            *reinterpret_cast<float4 *>(pa + sw32_off(t, cc)) =
+                make_float4(tf32r(e[0] * kv[0]), tf32r(e[1] * kv[1]), tf32r(e[2] * kv[2]), tf32r(e[3] * kv[3]));
+            *reinterpret_cast<float4 *>(pa + sw32_off(64 + t, cc)) =
+                make_float4(tf32r(e[0] * qv[0]), tf32r(e[1] * qv[1]), tf32r(e[2] * qv[2]), tf32r(e[3] * qv[3]));
+          }
+          *reinterpret_cast<uint2 *>(pqh + sw128_off4(t, i0)) =
+              pack_h4(-gm[0] * kv[0], -gm[1] * kv[1], -gm[2] * kv[2], -gm[3] * kv[3]);
+          *reinterpret_cast<uint2 *>(pqh + sw128_off4(64 + t, i0)) =
+              pack_h4(gm[0] * qv[0], gm[1] * qv[1], gm[2] * qv[2], gm[3] * qv[3]);
+          if (SV)
+            *reinterpret_cast<float4 *>(reinterpret_cast<float *>(ctx + kCtxGa) + t * D + i0) =
+                make_float4(gm[0], gm[1], gm[2], gm[3]);
         }
-        *reinterpret_cast<float4 *>(pa + sw32_off(t, cc)) =
-            make_float4(tf32r(e[0] * kv[0]), tf32r(e[1] * kv[1]), tf32r(e[2] * kv[2]), tf32r(e[3] * kv[3]));
-        *reinterpret_cast<float4 *>(pa + sw32_off(64 + t, cc)) =
-            make_float4(tf32r(e[0] * qv[0]), tf32r(e[1] * qv[1]), tf32r(e[2] * qv[2]), tf32r(e[3] * qv[3]));
-        *reinterpret_cast<uint2 *>(pqh + sw128_off4(t, i0)) =
-            pack_h4(-gm[0] * kv[0], -gm[1] * kv[1], -gm[2] * kv[2], -gm[3] * kv[3]);
-        *reinterpret_cast<uint2 *>(pqh + sw128_off4(64 + t, i0)) =
-            pack_h4(gm[0] * qv[0], gm[1] * qv[1], gm[2] * qv[2], gm[3] * qv[3]);
-        if (SV)
-          *reinterpret_cast<float4 *>(reinterpret_cast<float *>(ctx + kCtxGa) + t * D + i0) =
-              make_float4(gm[0], gm[1], gm[2], gm[3]);
-      }
+      };
+      if (oor) prep_loop(std::true_type{});
+      else prep_loop(std::false_type{});
       if (seg == 7) {
         *reinterpret_cast<float4 *>(s_gC + i0) = make_float4(gm[0], gm[1], gm[2], gm[3]);
         // the fused backward divides by the saved gamma: it needs gamma_C >= 1e-36
@@ -705,14 +855,11 @@ __global__ void __launch_bounds__(WT, 1)
       break;
     }
 
-    // ---- [2] MMA-T; the next chunk's k, g, omega and q
-    if (issuer) {
-      tc_fence_after();
-      const uint32_t A0 = smem_u32(ta), B0 = smem_u32(tb);
-      for (int kk = 0; kk < 16; ++kk)
-        umma_tf32(TD1, sw128_desc(A0 + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024),
-                  sw128_desc(B0 + (kk >> 2) * 8192 + (kk & 3) * 32, 16, 1024), id_T, kk > 0);
-      umma_commit(bar_t);
+    // ---- [2] MMA-T; the next chunk's k, g, omega and q.  In range mode the main
+    //          warps form T' and A'_qk on the CUDA cores instead, and the issuer
+    //          completes the MMA-T barrier's phase by hand once they are done.
+    const bool oor = !SV && s_oor[c & 1] != 0;
+    auto issue_next = [&]() {
       if (c + 1 < NC) {
         issue_raw(c + 1);
         issue_q(c + 1);
@@ -726,18 +873,35 @@ __global__ void __launch_bounds__(WT, 1)
           tma_prefetch_4d(&mq, 64 * s, h, (c + 2) * CM, b);
         }
       }
+    };
+    if (issuer && !oor) {
+      tc_fence_after();
+      const uint32_t A0 = smem_u32(ta), B0 = smem_u32(tb);
+      for (int kk = 0; kk < 16; ++kk)
+        umma_tf32(TD1, sw128_desc(A0 + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024),
+                  sw128_desc(B0 + (kk >> 2) * 8192 + (kk & 3) * 32, 16, 1024), id_T, kk > 0);
+      umma_commit(bar_t);
+      issue_next();
     }
     if (gain) {
       // the next chunk's gain, overlapping this chunk's remaining stages
       if (c + 1 < NC) mine = gain_chunk(c + 1) && mine;
       continue;
     }
+    if (oor) {
+      direct_products(mt, rk, rq, ta, tb, a.tau, sT, sA);
+      bar_sync(kBarMain, kMain);
+      if (issuer) {  // the raw tiles and phat k have been read
+        mbar_arrive(bar_t);
+        issue_next();
+      }
+    }
     mine = mbar_wait(bar_t, c & 1, kWait) && mine;
     tc_fence_after();
 
     // ---- [3] T' (with its diagonal) out of TMEM; A'_qk -> fp16 pairs in place (the
     //          A operand of MMA-O); S_in -> fp16; V -> fp16
-    if (wq < 2) {  // T' rows 0..63, lower triangle with the diagonal -> fp32 tile
+    if (wq < 2 && !oor) {  // T' rows 0..63, lower triangle with the diagonal -> fp32 tile
       const int t = 32 * wq + lane;
       for (int g = wgm; g < 4; g += 3) {
         const int s0 = 16 * g;
@@ -759,7 +923,15 @@ __global__ void __launch_bounds__(WT, 1)
       const int t = 32 * (wq - 2) + lane;
       for (int g = 0; g < 4; ++g) {
         float v[16], hv[8];
-        tmem_ld16(TD1 + lane_base + 16 * g, v);
+        if (oor) {
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            const float4 x4 = *reinterpret_cast<const float4 *>(sA + t * LT + 16 * g + 4 * u);
+            v[4 * u] = x4.x; v[4 * u + 1] = x4.y; v[4 * u + 2] = x4.z; v[4 * u + 3] = x4.w;
+          }
+        } else {
+          tmem_ld16(TD1 + lane_base + 16 * g, v);
+        }
 #pragma unroll
         for (int j = 0; j < 8; ++j) {
           const __half2 h2 = __floats2half2_rn((16 * g + 2 * j <= t) ? v[2 * j] : 0.f,
@@ -994,8 +1166,8 @@ __global__ void __launch_bounds__(WT, 1)
 }  // namespace
 
 bool wy_fwd_supported(const Args &a) {
-  return a.variant == 0 && a.gates == KDN_GATES_POST && a.dtype == KDN_BF16 && a.dk == D &&
-         a.dv == D && a.T > 0 && a.chunk != 32;
+  return a.variant == 0 && (a.gates == KDN_GATES_POST || a.gates == KDN_GATES_LOGITS) &&
+         a.dtype == KDN_BF16 && a.dk == D && a.dv == D && a.T > 0 && a.chunk != 32;
 }
 
 kdn_status_t launch_wy_fwd(const Args &a, cudaStream_t s, unsigned char *save_S, float *save_p) {
@@ -1008,7 +1180,8 @@ kdn_status_t launch_wy_fwd(const Args &a, cudaStream_t s, unsigned char *save_S,
   if (!make_map(&mk, a.k, a) || !make_map(&mg, a.g, a) || !make_map(&mw, a.omega, a) ||
       !make_map(&mv, a.v, a) || !make_map(&mq, a.q, a))
     return KDN_ERR_CUDA;
-  const auto kern = save_S ? k_wy_fwd<1> : k_wy_fwd<0>;
+  const bool lg = a.gates == KDN_GATES_LOGITS;
+  const auto kern = save_S ? (lg ? k_wy_fwd<1, 1> : k_wy_fwd<1, 0>) : (lg ? k_wy_fwd<0, 1> : k_wy_fwd<0, 0>);
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES) !=
       cudaSuccess)
     return KDN_ERR_CUDA;

@@ -413,33 +413,25 @@ def test_fused_decay_range_is_reported(kdn, variant):
     """A decay outside a fused kernel's range is reported in the workspace status
     word (no fault), and the general kernels (32-token chunks) still match the
     oracle.  alpha = e^-2 for 64 tokens puts exp(G_C) at e^-128: below the range
-    of the fused backward (and of the isotropic forward), which divide by
-    gamma, but inside that of the Diagonal forward, whose decay factors are
-    referenced at the middle of the chunk's range (exp(+-64)): there it must
-    match the oracle with KDN_OK.  alpha = e^-3 (exp(G_C) = e^-192) leaves the
-    Diagonal forward's range too."""
+    of the fused backward and of the isotropic forward, which divide by gamma.
+    (The Diagonal forward takes any decay: test_diag_forward_any_decay.)"""
     ins = make_inputs(variant, 1, 100, 2, 128, 128, dtype="bf16", seed=3, with_grad=True)
     ins["g"][...] = -2.0
     d = to_dev(ins)
     x = [d[n] for n in ("q", "k", "v", "g", "omega", "r")]
-    fwd = kdn.kdn_diag_fwd if variant == "diag" else kdn.kdn_iso_fwd
     desc = kdn.make_desc(1, 100, 2, 128, 128, torch.bfloat16,
                          decay_per_channel=int(d["g"].dim() == 4))
     ws = kdn.alloc_workspace(desc, 0 if variant == "diag" else 1, True)
     ref = _oracle_fwd(variant, ins)
-    o, _, _ = fwd(*x, workspace=ws)
-    if variant == "diag":
-        assert kdn.kdn_get_device_status(ws) == kdn.KDN_OK
-        check("o", o, ref["o"], "bf16")
-        x3 = [t.clone() for t in x]
-        x3[3].fill_(-3.0)
-        fwd(*x3, workspace=ws)
-    assert kdn.kdn_get_device_status(ws) == kdn.KDN_ERR_RANGE
-    fwd(*(x3 if variant == "diag" else x), workspace=ws)  # cleared by the query, set again
-    assert kdn.kdn_get_device_status(ws) == kdn.KDN_ERR_RANGE
+    if variant == "iso":
+        kdn.kdn_iso_fwd(*x, workspace=ws)
+        assert kdn.kdn_get_device_status(ws) == kdn.KDN_ERR_RANGE
+        kdn.kdn_iso_fwd(*x, workspace=ws)  # cleared by the query, set again
+        assert kdn.kdn_get_device_status(ws) == kdn.KDN_ERR_RANGE
     bwd = kdn.kdn_diag_bwd if variant == "diag" else kdn.kdn_iso_bwd
     bwd(*x, None, None, d["dO"], workspace=ws)
     assert kdn.kdn_get_device_status(ws) == kdn.KDN_ERR_RANGE
+    fwd = kdn.kdn_diag_fwd if variant == "diag" else kdn.kdn_iso_fwd
     desc32 = kdn.make_desc(1, 100, 2, 128, 128, torch.bfloat16, chunk=32,
                            decay_per_channel=int(d["g"].dim() == 4))
     ws32 = kdn.alloc_workspace(desc32, 0 if variant == "diag" else 1, False)
@@ -447,6 +439,65 @@ def test_fused_decay_range_is_reported(kdn, variant):
     torch.cuda.synchronize()
     assert kdn.kdn_get_device_status(ws32) == kdn.KDN_OK
     check("o", o, ref["o"], "bf16")
+
+
+def _strong_decay(ins, kind, seed):
+    """Decays of the range test: 'e-2' (alpha = e^-2, G_C = -128 per 64-token chunk),
+    'e-3' (alpha = e^-3, G_C = -192 in every chunk and channel), 'mixed' (the
+    configs' decay, with alpha = e^-3.5 in a random half of the channels of every
+    other chunk), 'logits' (logit gates x ~ N(-3, 1), y, z ~ N(0, 1))."""
+    ins = dict(ins)
+    rng = np.random.default_rng(seed)
+    if kind == "e-2":
+        ins["g"] = np.full_like(ins["g"], -2.0)
+    elif kind == "e-3":
+        ins["g"] = np.full_like(ins["g"], -3.0)
+    elif kind == "mixed":
+        g = ins["g"].copy()
+        T = g.shape[1]
+        for c0 in range(0, T, 128):
+            ch = rng.permutation(g.shape[-1])[: g.shape[-1] // 2]
+            g[:, c0:c0 + 64, :, ch] = -3.5
+        ins["g"] = g
+    else:
+        ins["g"] = round_to(rng.normal(-3.0, 1.0, ins["g"].shape), "bf16")
+        ins["omega"] = round_to(rng.normal(0.0, 1.0, ins["omega"].shape), "bf16")
+        ins["r"] = round_to(rng.normal(0.0, 1.0, ins["r"].shape), "bf16")
+    return ins
+
+
+@pytest.mark.parametrize("kind", ["e-2", "e-3", "mixed", "logits"])
+def test_diag_forward_any_decay(kdn, kind):
+    """The Diagonal forward matches the oracle with KDN_OK at any decay.  Its
+    T' / A'_qk factors are referenced at the middle of each chunk's decay range
+    (each within exp(+-|G_C| / 2)); a chunk with G_C < -160 in some channel forms
+    them from exp(G_t - G_s) directly (App. F.2, cumulative log-decay
+    differences).  The training forward keeps the referenced form (its context
+    feeds the fused backward, which divides by gamma) and reports KDN_ERR_RANGE
+    once exp(G_C) < 1e-36; where its factors stay in range (alpha = e^-2) its
+    outputs equal the plain forward's bit for bit."""
+    T = 300
+    ins = _strong_decay(make_inputs("diag", 1, T, 2, 128, 128, dtype="bf16", seed=7,
+                                    s0_std=0.05, p0_range=(0.5, 2.0)), kind, 5)
+    logits = kind == "logits"
+    kw = dict(gates=kdn.KDN_GATES_LOGITS, r_min=0.01) if logits else {}
+    okw = dict(gates="logits", r_min=0.01) if logits else {}
+    d = to_dev(ins)
+    x = [d[n] for n in ("q", "k", "v", "g", "omega", "r")]
+    desc = kdn.make_desc(1, T, 2, 128, 128, torch.bfloat16, **kw)
+    ws = kdn.alloc_workspace(desc, 0, False)
+    o, ST, pT = kdn.kdn_diag_fwd(*x, d["S0"], d["p0"], workspace=ws, **kw)
+    torch.cuda.synchronize()
+    assert kdn.kdn_get_device_status(ws) == kdn.KDN_OK
+    ref = _oracle_fwd("diag", ins, **okw)
+    check("o", o, ref["o"], "bf16")
+    check("ST", ST, ref["ST"], "bf16")
+    check("pT", pT, ref["pT"], "bf16")
+    o2, ST2, pT2, _ = kdn.kdn_diag_fwd_save(*x, d["S0"], d["p0"], workspace=ws, **kw)
+    st = kdn.kdn_get_device_status(ws)
+    assert st == kdn.KDN_ERR_RANGE  # exp(G_C) < 1e-36 in every case here
+    if kind == "e-2":  # referenced form in both: the same arithmetic
+        assert torch.equal(o, o2) and torch.equal(ST, ST2) and torch.equal(pT, pT2)
 
 
 def test_isotropic_training_pair_matches_recompute_path(kdn):

@@ -81,13 +81,15 @@ def test_noalloc_same_problem_twice_after_a_larger_one(kdn):
 
 
 def test_noalloc_status_word_is_readable(kdn):
-    """A chunk whose cumulative decay leaves the fused kernel's range is reported
+    """A chunk whose cumulative decay leaves a fused kernel's range is reported
     in the status word kept in the library's array, through
-    kdn_noalloc_device_status, which then clears it."""
-    ins = make_inputs("diag", 1, 100, 2, 128, 128, dtype="bf16", seed=3)
-    ins["g"][...] = -3.0  # exp(G_C) = e^-192 over a 64-token chunk
+    kdn_noalloc_device_status, which then clears it.  The problem (B=1, H=2,
+    T=2048) is served by the sequence-parallel forward, whose segment passes
+    take exp(G_C) >= 1e-36; alpha = e^-3 gives exp(G_C) = e^-192."""
+    ins = make_inputs("diag", 1, 2048, 2, 128, 128, dtype="bf16", seed=3)
+    ins["g"][...] = -3.0
     d = to_dev(ins)
-    o = torch.empty(1, 100, 2, 128, dtype=torch.float32, device="cuda")
+    o = torch.empty(1, 2048, 2, 128, dtype=torch.float32, device="cuda")
     assert _noalloc(kdn, d, o, None, None) == kdn.KDN_OK
     assert kdn.kdn_noalloc_device_status() == kdn.KDN_ERR_RANGE
     assert kdn.kdn_noalloc_device_status() == kdn.KDN_OK
