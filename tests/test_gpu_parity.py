@@ -500,6 +500,57 @@ def test_diag_forward_any_decay(kdn, kind):
         assert torch.equal(o, o2) and torch.equal(ST, ST2) and torch.equal(pT, pT2)
 
 
+WY_CASES = [
+    # T, B, H, range-mode chunk (or None), logit gates
+    (1, 3, 5, None, False),
+    (63, 2, 3, None, True),
+    (64, 1, 2, 0, False),
+    (65, 2, 2, 0, False),
+    (191, 1, 3, 1, True),
+    (257, 3, 5, 2, False),
+]
+
+
+@pytest.mark.parametrize("case", WY_CASES, ids=lambda c: "-".join(map(str, c)))
+def test_diag_forward_chunk_edges(kdn, case):
+    """The compact-WY Diagonal forward (bf16, d = 128) at chunk edges (T = 1, 63, 64,
+    65, 191, 257), odd head counts, a random S_0 and p_0, optionally one chunk in
+    range mode (alpha = e^-3 in some channels of that chunk only) and logit gates;
+    o, S_T and p_T against the oracle, and the training forward's o, S_T, p_T bit for
+    bit where no chunk is in range mode."""
+    T, B, H, rm_chunk, logits = case
+    ins = make_inputs("diag", B, T, H, 128, 128, dtype="bf16", seed=T * 7 + H, s0_std=0.05,
+                      p0_range=(0.3, 2.0))
+    rng = np.random.default_rng(T)
+    if logits:
+        ins["g"] = round_to(rng.normal(2.0, 1.0, ins["g"].shape), "bf16")
+        ins["omega"] = round_to(rng.normal(0.0, 1.0, ins["omega"].shape), "bf16")
+        ins["r"] = round_to(rng.normal(0.0, 1.0, ins["r"].shape), "bf16")
+    if rm_chunk is not None:
+        g = ins["g"].copy()
+        ch = rng.permutation(128)[:40]
+        t0, t1 = 64 * rm_chunk, min(T, 64 * rm_chunk + 64)
+        g[:, t0:t1, :, ch] = -3.0  # log alpha = -3, or the logit -3 (log alpha ~ -3.05)
+        ins["g"] = g
+    kw = dict(gates=kdn.KDN_GATES_LOGITS, r_min=0.01) if logits else {}
+    okw = dict(gates="logits", r_min=0.01) if logits else {}
+    d = to_dev(ins)
+    x = [d[n] for n in ("q", "k", "v", "g", "omega", "r")]
+    desc = kdn.make_desc(B, T, H, 128, 128, torch.bfloat16, **kw)
+    ws = kdn.alloc_workspace(desc, 0, False)
+    o, ST, pT = kdn.kdn_diag_fwd(*x, d["S0"], d["p0"], workspace=ws, **kw)
+    torch.cuda.synchronize()
+    assert kdn.kdn_get_device_status(ws) == kdn.KDN_OK
+    ref = _oracle_fwd("diag", ins, **okw)
+    check("o", o, ref["o"], "bf16")
+    check("ST", ST, ref["ST"], "bf16")
+    check("pT", pT, ref["pT"], "bf16")
+    if rm_chunk is None:
+        o2, ST2, pT2, _ = kdn.kdn_diag_fwd_save(*x, d["S0"], d["p0"], workspace=ws, **kw)
+        torch.cuda.synchronize()
+        assert torch.equal(o, o2) and torch.equal(ST, ST2) and torch.equal(pT, pT2)
+
+
 def test_isotropic_training_pair_matches_recompute_path(kdn):
     """kdn_iso_fwd_save / kdn_iso_bwd_saved (scalar decay per head) against
     kdn_iso_fwd / kdn_iso_bwd bit for bit, and against the oracle."""
