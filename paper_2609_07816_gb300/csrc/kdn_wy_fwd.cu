@@ -881,9 +881,13 @@ __global__ void __launch_bounds__(WT, 1)
         umma_tf32(TD1, sw128_desc(A0 + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024),
                   sw128_desc(B0 + (kk >> 2) * 8192 + (kk & 3) * 32, 16, 1024), id_T, kk > 0);
       umma_commit(bar_t);
-      issue_next();
+      // the next chunk's tiles (the raw tiles are free: the preparing pass is done).
+      // The context-saving instantiation, whose main warps are the longer path, leaves
+      // them to a gain thread; the plain one, whose gain warps are, issues them here.
+      if (!SV) issue_next();
     }
     if (gain) {
+      if (SV && tid == 0) issue_next();
       // the next chunk's gain, overlapping this chunk's remaining stages
       if (c + 1 < NC) mine = gain_chunk(c + 1) && mine;
       continue;
