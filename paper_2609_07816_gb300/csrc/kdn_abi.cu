@@ -142,7 +142,7 @@ kdn_status_t fwd_entry(int variant, const kdn_desc_t *d, const void *q, const vo
   if ((size_t)a.B * a.H == 0) return KDN_OK;
   if (a.T == 0) return empty_fwd(a, s);
   if (nseg > 1) return launch_seg_fwd(a, nseg, static_cast<char *>(ws) + base, s);
-  if (use_fused(a) && wy_fwd_supported(a)) return launch_wy_fwd(a, s);
+  if (use_fused(a) && wy_fwd_supported(a, false)) return launch_wy_fwd(a, s);
   if (use_fused(a)) return launch_fused_fwd(a, s);
   return launch_chunked_fwd(a, s, false);
 }
@@ -204,7 +204,7 @@ kdn_status_t fwd_save_entry(int variant, const kdn_desc_t *d, const void *q, con
   if ((size_t)a.B * a.H == 0) return KDN_OK;
   if (a.T == 0) return empty_fwd(a, s);
   const size_t nsv = (size_t)a.B * a.H * ((a.T + 63) / 64) * fused_ctx_record_bytes();
-  if (wy_fwd_supported(a))
+  if (wy_fwd_supported(a, true))
     return launch_wy_fwd(a, s, static_cast<unsigned char *>(saved),
                          reinterpret_cast<float *>(static_cast<char *>(saved) + nsv));
   return launch_fused_fwd(a, s, static_cast<unsigned char *>(saved),

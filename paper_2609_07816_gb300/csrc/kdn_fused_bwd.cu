@@ -1212,7 +1212,7 @@ kdn_status_t launch_fused_bwd(const Args &a, cudaStream_t s) {
   f.o = nullptr;
   f.ST = nullptr;
   f.pT = nullptr;
-  kdn_status_t st = wy_fwd_supported(f) ? launch_wy_fwd(f, s, a.fSin, a.fpin)
+  kdn_status_t st = wy_fwd_supported(f, true) ? launch_wy_fwd(f, s, a.fSin, a.fpin)
                                          : launch_fused_fwd(f, s, a.fSin, a.fpin, false);
   if (st != KDN_OK) return st;
   return launch_fused_bwd_sweep(a, s);

@@ -37,12 +37,13 @@ __device__ __forceinline__ void sto(int odt, void *p, size_t i, float x) {
 
 // Gate activations of the layer's parameterisation for KDN_GATES_LOGITS
 // inputs: alpha = sigmoid(x), omega = softplus(y), r = r_min + softplus(z).
-// softplus(x) = max(x, 0) + log1p(u), u = exp(-|x|) in (0, 1]: the fast logarithm
-// of 1 + u, or for small u the series u - u^2/2 + u^3/3 (error below u^4 / 4)
+// softplus(x) = max(x, 0) + log1p(u), u = exp(-|x|) in (0, 1], with log1p(u) taken
+// as the fast logarithm of 1 + u: no branch inside the unrolled per-token loops.
+// For u below ~1e-4 the rounding of 1 + u costs relative precision in the small
+// term log1p(u) ~ u, never more than 6e-8 in absolute terms.
 __device__ __forceinline__ float softplus_f(float x) {
   const float u = __expf(-fabsf(x));
-  const float lp = u < 1e-3f ? u * (1.f - u * (0.5f - u * (1.f / 3.f))) : __logf(1.f + u);
-  return fmaxf(x, 0.f) + lp;
+  return fmaxf(x, 0.f) + __logf(1.f + u);
 }
 __device__ __forceinline__ float sigmoid_f(float x) { return __fdividef(1.f, 1.f + __expf(-x)); }
 // log alpha from the gate input: g itself, or log sigmoid(x) = -softplus(-x)
@@ -152,7 +153,7 @@ kdn_status_t launch_fused_fwd(const Args &a, cudaStream_t s, unsigned char *save
 // 128, 64-token chunks; writes o, S_T, p_T where their pointers are non-null,
 // and with save_S / save_p the fused backward's context (the layout of
 // launch_fused_fwd's saving mode).
-bool wy_fwd_supported(const Args &a);
+bool wy_fwd_supported(const Args &a, bool save);  // save: the context-saving instantiation
 kdn_status_t launch_wy_fwd(const Args &a, cudaStream_t s, unsigned char *save_S = nullptr,
                            float *save_p = nullptr);
 // beta_eff [B,T,H] (float32) from the per-token gain scalars of a context saved by

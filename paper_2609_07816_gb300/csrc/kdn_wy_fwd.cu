@@ -601,13 +601,27 @@ __global__ void __launch_bounds__(WT, 1)
     const int tv = a.T - c * CM;
     auto lga = [&](float x, int t) { return LG ? (t < tv ? -softplus_f(-x) : 0.f) : x; };
     auto omg = [&](float y, int t) { return LG ? (t < tv ? softplus_f(y) : 0.f) : y; };
+    unsigned char *pb = tb + (i >> 5) * 8192;
+    const int cb = i & 31;
+    // logit gates: log alpha is formed once per element here and kept (fp32) in this
+    // channel's column of the Kk' tile, which the loop below overwrites token by token
+    // after reading it; the tile is free once MMA-T of chunk c - 1 has read it
+    if (LG && c > 0) g_ok = mbar_wait(bar_t, (c - 1) & 1, kWait) && g_ok;
+    auto lga_keep = [&](int t) {
+      const float la = lga(raw(pg, t), t);
+      if (LG) *reinterpret_cast<float *>(pb + sw32_off(t, cb)) = la;
+      return la;
+    };
+    auto lga_t = [&](int t) {  // log alpha of token t in the loop
+      return LG ? *reinterpret_cast<const float *>(pb + sw32_off(t, cb)) : lga(raw(pg, t), t);
+    };
     float g0 = 0.f, g1 = 0.f, g2 = 0.f, g3 = 0.f;
 #pragma unroll
     for (int t = 0; t < CM; t += 4) {
-      g0 += lga(raw(pg, t), t);
-      g1 += lga(raw(pg, t + 1), t + 1);
-      g2 += lga(raw(pg, t + 2), t + 2);
-      g3 += lga(raw(pg, t + 3), t + 3);
+      g0 += lga_keep(t);
+      g1 += lga_keep(t + 1);
+      g2 += lga_keep(t + 2);
+      g3 += lga_keep(t + 3);
     }
     const float GC = (g0 + g1) + (g2 + g3), cref = 0.5f * GC;
     s_c[i] = cref;
@@ -623,13 +637,11 @@ __global__ void __launch_bounds__(WT, 1)
     float *cph = SV ? reinterpret_cast<float *>(gctx + kCtxPh) + i : nullptr;
     float f = ex2f(cref * kLog2e);                // exp(c - G_t), G_{-1} = 0
     const float E2 = ex2f((GC - cref) * kLog2e);  // exp(G_C - c)
-    unsigned char *pb = tb + (i >> 5) * 8192;
-    const int cb = i & 31;
     const uint32_t tkt = TKT + (uint32_t)((c & 1) * 32);
     float gb[8], wb[8], kb8[8], mb[8];
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
-      gb[j] = lga(raw(pg, j), j);
+      gb[j] = lga_t(j);
       wb[j] = omg(raw(pw, j), j);
       kb8[j] = raw(pk, j);
     }
@@ -637,7 +649,7 @@ __global__ void __launch_bounds__(WT, 1)
       const float4 m0 = *reinterpret_cast<const float4 *>(smur), m1 = *reinterpret_cast<const float4 *>(smur + 4);
       mb[0] = m0.x; mb[1] = m0.y; mb[2] = m0.z; mb[3] = m0.w; mb[4] = m1.x; mb[5] = m1.y; mb[6] = m1.z; mb[7] = m1.w;
     }
-    if (c > 0) g_ok = mbar_wait(bar_t, (c - 1) & 1, kWait) && g_ok;  // Kk' of chunk c - 1 has been read
+    if (!LG && c > 0) g_ok = mbar_wait(bar_t, (c - 1) & 1, kWait) && g_ok;  // Kk' of chunk c - 1 has been read
     // the chunk in blocks of 8 tokens; the next block's inputs are loaded
     // before the current block's outputs are stored
     if (oor) {
@@ -649,7 +661,7 @@ __global__ void __launch_bounds__(WT, 1)
 #pragma unroll
         for (int j = 0; j < 8; ++j) {
           const int t = 8 * blk + j;
-          const float lg = lga(raw(pg, t), t), kk = raw(pk, t);
+          const float lg = lga_t(t), kk = raw(pk, t);
           const float al = ex2f(lg * kLog2e);
           const float ph = fmaf(al * al, p, omg(raw(pw, t), t));
           const float den = fmaf(kk * kk * smur[t], ph, 1.f);
@@ -673,7 +685,7 @@ __global__ void __launch_bounds__(WT, 1)
 #pragma unroll
           for (int j = 0; j < 8; ++j) {
             const int t = 8 * (blk + 1) + j;
-            gn[j] = lga(raw(pg, t), t);
+            gn[j] = lga_t(t);
             wn[j] = omg(raw(pw, t), t);
             kn[j] = raw(pk, t);
           }
@@ -1169,13 +1181,16 @@ __global__ void __launch_bounds__(WT, 1)
 
 }  // namespace
 
-bool wy_fwd_supported(const Args &a) {
-  return a.variant == 0 && (a.gates == KDN_GATES_POST || a.gates == KDN_GATES_LOGITS) &&
+bool wy_fwd_supported(const Args &a, bool save) {
+  // The context-saving forward with logit gates stays on the first fused kernel: its
+  // gate conversions cost less there, and the backward it feeds has that kernel's
+  // decay range either way.
+  return a.variant == 0 && (a.gates == KDN_GATES_POST || (a.gates == KDN_GATES_LOGITS && !save)) &&
          a.dtype == KDN_BF16 && a.dk == D && a.dv == D && a.T > 0 && a.chunk != 32;
 }
 
 kdn_status_t launch_wy_fwd(const Args &a, cudaStream_t s, unsigned char *save_S, float *save_p) {
-  if (!wy_fwd_supported(a) || (!save_S) != (!save_p)) return KDN_ERR_UNSUPPORTED;
+  if (!wy_fwd_supported(a, save_S != nullptr) || (!save_S) != (!save_p)) return KDN_ERR_UNSUPPORTED;
   WyParams P;
   P.a = a;
   P.save_S = save_S;
@@ -1185,7 +1200,7 @@ kdn_status_t launch_wy_fwd(const Args &a, cudaStream_t s, unsigned char *save_S,
       !make_map(&mv, a.v, a) || !make_map(&mq, a.q, a))
     return KDN_ERR_CUDA;
   const bool lg = a.gates == KDN_GATES_LOGITS;
-  const auto kern = save_S ? (lg ? k_wy_fwd<1, 1> : k_wy_fwd<1, 0>) : (lg ? k_wy_fwd<0, 1> : k_wy_fwd<0, 0>);
+  const auto kern = save_S ? k_wy_fwd<1, 0> : (lg ? k_wy_fwd<0, 1> : k_wy_fwd<0, 0>);
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES) !=
       cudaSuccess)
     return KDN_ERR_CUDA;
