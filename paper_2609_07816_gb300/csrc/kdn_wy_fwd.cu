@@ -79,6 +79,7 @@ constexpr float kMinHalfG = -80.f;  // c = G_C / 2 below this: out of range
 constexpr int kPrepThreads = 256;   // warps 4-11: the preparing pass
 constexpr int kMain = 384;          // warps 4-15: everything but the gain
 constexpr int kBarPrep = 1, kBarMain = 2, kBarGain = 3;  // named barriers (0 = __syncthreads)
+constexpr int kTmaThread = 224;  // warp 7, lane 0: issues each chunk's next-chunk TMA operations
 
 // shared-memory map (bytes from the 1024-aligned base)
 constexpr int LT = 68;          // row stride (floats) of the fp32 T and A tiles
@@ -893,13 +894,12 @@ __global__ void __launch_bounds__(WT, 1)
         umma_tf32(TD1, sw128_desc(A0 + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024),
                   sw128_desc(B0 + (kk >> 2) * 8192 + (kk & 3) * 32, 16, 1024), id_T, kk > 0);
       umma_commit(bar_t);
-      // the next chunk's tiles (the raw tiles are free: the preparing pass is done).
-      // The context-saving instantiation, whose main warps are the longer path, leaves
-      // them to a gain thread; the plain one, whose gain warps are, issues them here.
-      if (!SV) issue_next();
     }
+    // the next chunk's tiles (the raw tiles are free: the preparing pass is done), from a
+    // main thread outside the MMA issuer's warp: its ~20 TMA operations then overlap
+    // MMA-T, for which every main warp waits anyway
+    if (tid == kTmaThread && !oor) issue_next();
     if (gain) {
-      if (SV && tid == 0) issue_next();
       // the next chunk's gain, overlapping this chunk's remaining stages
       if (c + 1 < NC) mine = gain_chunk(c + 1) && mine;
       continue;
