@@ -36,9 +36,13 @@
 // chunk-memory-output-state, with A_qk = lower(A'_qk) diag(1/s).  Every MMA
 // accumulates in float32 in tensor memory.
 //
-// Shared-memory instructions are the scarce resource of this kernel: every
-// per-element pass reads and writes 8 or 16 bytes per instruction wherever the
-// layout allows (the gain's per-channel recursion is the exception).
+// The chunk is a chain of dependent stages inside one CTA, and the gain (run one
+// chunk ahead on its own warps) is as long as the rest: the kernel is bound by
+// that latency, not by HBM or shared-memory throughput.  Every per-element pass
+// still reads and writes 8 or 16 bytes per shared-memory instruction wherever the
+// layout allows (the gain's per-channel recursion is the exception), and the
+// next chunk's TMA operations are issued from a thread outside the MMA issuer's
+// warp while every main warp waits for MMA-T.
 //
 // Range: the referenced factors stay finite while the chunk's cumulative
 // log-decay G_C >= -160 in every channel (average alpha >= 0.082 over 64
@@ -51,8 +55,10 @@
 //
 // Logit gates (LG): g, omega, r hold the logits x, y, z of the layer's
 // parameterisation (Sec. 5): log alpha = -softplus(-x), omega = softplus(y),
-// r = r_min + softplus(z), formed in float32 where each is read; the tokens
-// past T are identity updates.
+// r = r_min + softplus(z), formed in float32.  The gain forms log alpha once per
+// element and keeps it in its column of the Kk' tile until the recursion
+// overwrites it; the prepare pass forms its own; the tokens past T are identity
+// updates.  (The context-saving forward with logit gates runs k_fused_fwd.)
 //
 // Every wait on an mbarrier is bounded; on timeout the kernel records
 // KDN_ERR_TIMEOUT in the status word, waits (bounded) for its copies in flight,
