@@ -44,6 +44,35 @@ def test_iso_750m_layer_shape(kdn):
     _sampled_fwd_check(kdn, "iso", ins, [(0, 0), (3, 7), (7, 11)])
 
 
+def test_iso_750m_layer_shape_bench_launch(kdn):
+    """Isotropic KDN, B=8 H=12 T=2048 d=128, one decay per head, in the launch
+    configuration the benchmark times: bf16 o and gradients, the training pair
+    kdn_iso_fwd_save + kdn_iso_bwd_saved with a preallocated context, without state
+    outputs or state gradients.  Stored bf16 values are checked under the bf16 rule
+    plus one final rounding."""
+    B, T, H = 8, 2048, 12
+    bf = torch.bfloat16
+    ins = make_inputs("iso", B, T, H, 128, 128, dtype="bf16", seed=11, per_channel_decay=False,
+                      with_grad=True)
+    d = to_dev(ins)
+    x = [d[n] for n in NAMES]
+    desc = kdn.make_desc(B, T, H, 128, 128, bf, decay_per_channel=0, out_dtype=bf)
+    ws = kdn.alloc_workspace(desc, 1, False)
+    saved = torch.empty(kdn.saved_bytes(desc, 1), dtype=torch.uint8, device="cuda")
+    o, _, _, _ = kdn.kdn_iso_fwd_save(*x, saved=saved, want_state=False, workspace=ws, out_dtype=bf)
+    gr = kdn.kdn_iso_bwd_saved(*x, saved, d["dO"], want_state_grads=False, workspace=ws,
+                               out_dtype=bf)
+    torch.cuda.synchronize()
+    assert kdn.kdn_get_device_status(ws) == 0
+    for b, h in [(1, 2), (6, 9)]:
+        sl = head_slice(ins, b, h)
+        ref = oracle.fwd("iso", *[sl[n] for n in NAMES], None, None)
+        check_stored_bf16(f"o[{b},{h}]", o[b:b + 1, :, h:h + 1], ref["o"])
+        rg = oracle.bwd("iso", *[sl[n] for n in NAMES], None, None, sl["dO"])
+        for n in ("dq", "dk", "dv", "dg", "domega", "dr"):
+            check_stored_bf16(f"{n}[{b},{h}]", gr[n][b:b + 1, :, h:h + 1], rg[n])
+
+
 def test_iso_750m_layer_shape_backward(kdn):
     """Isotropic KDN backward, B=8 H=12 T=2048 d=128, scalar decay, dO ~ N(0,1)."""
     ins = make_inputs("iso", 8, 2048, 12, 128, 128, dtype="bf16", seed=0,
