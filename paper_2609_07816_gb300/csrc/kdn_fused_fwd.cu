@@ -150,6 +150,9 @@ __global__ void __launch_bounds__(FT, 1)
   const int bh = blockIdx.x, b = bh / a.H, h = bh % a.H;
   const int NC = (a.T + CM - 1) / CM;
   const bool pcd = (V == 0) || a.pcd;
+  // the copies (TMA loads, context and output stores) are issued by lane 0 of warp 15,
+  // not by the MMA issuer: each TMA operation holds the issuing warp for tens of cycles
+  const bool io = tid == 480;
   const uint32_t raw_bytes = 8192u * (4 + (P.has_g_map ? 2 : 0) + (P.has_w_map ? 2 : 0));
 
   if (tid == 0) {
@@ -196,7 +199,7 @@ __global__ void __launch_bounds__(FT, 1)
     mbar_expect_tx(bar_v, 16384);
     for (int s = 0; s < 2; ++s) tma_load_4d(vr + s * 8192, &mv, bar_v, 64 * s, h, c * CM, b);
   };
-  if (tid == 0 && NC > 0) {
+  if (io && NC > 0) {
     issue_raw_g(0);
     issue_raw_kqw(0);
     issue_v(0);
@@ -271,7 +274,7 @@ __global__ void __launch_bounds__(FT, 1)
       s_om[tid] = nom;
       s_gs[tid] = ng;
     }
-    if (tid == 0) bulk_wait_read();  // O staging and the saved S image have been read
+    if (io) bulk_wait_read();  // O staging and the saved S image have been read
     if (P.save_p && tid < D)
       P.save_p[((size_t)bh * NC + c) * D + tid] = (V == 0) ? s_p[tid] : s_b[0];
     unsigned char *ctx = P.save_S ? P.save_S + ((size_t)bh * NC + c) * kCtxBytes : nullptr;
@@ -479,8 +482,8 @@ __global__ void __launch_bounds__(FT, 1)
     }
     fence_proxy_async();  // phat / gamma are read by the bulk copies below
     __syncthreads();
-    if (tid == 0 && c + 1 < NC) issue_raw_g(c + 1);  // the decay tile is no longer read
-    if (tid == 0 && P.save_S) {  // phat and gamma into the backward context
+    if (io && c + 1 < NC) issue_raw_g(c + 1);  // the decay tile is no longer read
+    if (io && P.save_S) {  // phat and gamma into the backward context
       if (V == 0) bulk_s2g(ctx + kCtxPh, Pb, 32768);
       if (SD) bulk_s2g(ctx + kCtxGa, s_gm, CM * 4);  // one gamma per token
       else bulk_s2g(ctx + kCtxGa, Eb, 32768);
@@ -537,7 +540,7 @@ __global__ void __launch_bounds__(FT, 1)
     fence_proxy_async();
     tc_fence_before();
     __syncthreads();
-    if (tid == 0 && P.save_S) {  // per-token scalars of the gain into the backward context
+    if (io && P.save_S) {  // per-token scalars of the gain into the backward context
       bulk_s2g(ctx + kCtxTok, s_x, 5 * 64 * 4);
       bulk_commit();
     }
@@ -569,7 +572,7 @@ __global__ void __launch_bounds__(FT, 1)
         sm16(vr, off) = pack_h8(v);
       }
     }
-    if (tid == 0 && P.save_S) bulk_wait_read();  // phat / gamma have left b3 / fs
+    if (io && P.save_S) bulk_wait_read();  // phat / gamma have left b3 / fs
     ok = mma_wait() && v_ok;
     if (!ok) break;
     tc_fence_after();
@@ -696,8 +699,8 @@ __global__ void __launch_bounds__(FT, 1)
     tc_fence_after();
     // kq and rw are free: MMA-T and MMA-W have read them, the Qbar and K_tail
     // conversions above have finished (the wait's barrier)
-    if (tid == 0 && c + 1 < NC) issue_raw_kqw(c + 1);
-    if (tid == 0 && P.save_S) {  // A fp16 [t][s] into the backward context
+    if (io && c + 1 < NC) issue_raw_kqw(c + 1);
+    if (io && P.save_S) {  // A fp16 [t][s] into the backward context
       bulk_s2g(ctx + kCtxA, af, 8192);
       bulk_commit();
     }
@@ -747,7 +750,7 @@ __global__ void __launch_bounds__(FT, 1)
     fence_proxy_async();
     tc_fence_before();
     __syncthreads();
-    if (tid == 0 && P.save_S) {  // S_in, -W and A_qk into the backward context
+    if (io && P.save_S) {  // S_in, -W and A_qk into the backward context
       bulk_s2g(ctx + kCtxS, b3, 32768);
       bulk_s2g(ctx + kCtxW, a1l, 8192);
       bulk_s2g(ctx + kCtxW + 8192, a1l + 16384, 8192);
@@ -791,7 +794,7 @@ __global__ void __launch_bounds__(FT, 1)
     fence_proxy_async();
     tc_fence_before();
     __syncthreads();
-    if (tid == 0 && P.save_S) {  // R into the backward context
+    if (io && P.save_S) {  // R into the backward context
       bulk_s2g(ctx + kCtxR, vr, 16384);
       bulk_commit();
     }
@@ -811,10 +814,10 @@ __global__ void __launch_bounds__(FT, 1)
       }
       umma_commit(bar_mma);
     }
-    if (tid == 0 && P.save_S) bulk_wait_read();  // the saved R and A have left vr and fs
+    if (io && P.save_S) bulk_wait_read();  // the saved R and A have left vr and fs
     if (!(ok = mma_wait())) break;
     tc_fence_after();
-    if (tid == 0 && c + 1 < NC) issue_v(c + 1);  // R in vr has been consumed
+    if (io && c + 1 < NC) issue_v(c + 1);  // R in vr has been consumed
     // ---- [11] O (rows 64..127 of TU) -> 128-byte-swizzled staging tiles in fs
     //           -> TMA bulk tensor stores (rows past T are not written)
     if (wq >= 2 && P.write_o) {
@@ -848,7 +851,7 @@ __global__ void __launch_bounds__(FT, 1)
     }
     fence_proxy_async();
     __syncthreads();
-    if (tid == 0 && P.write_o) {
+    if (io && P.write_o) {
       const unsigned char *stg = reinterpret_cast<const unsigned char *>(fs);
       const int nbox = a.odt == KDN_BF16 ? 2 : 4, bw = a.odt == KDN_BF16 ? 64 : 32;
       for (int bx = 0; bx < nbox; ++bx) tma_store_4d(&mo, stg + bx * 8192, bx * bw, h, c * CM, b);
@@ -899,7 +902,7 @@ __global__ void __launch_bounds__(FT, 1)
       mbar_wait(bar_v, 1, kWaitIters);
     }
   }
-  if (tid == 0) bulk_wait_all();
+  if (io) bulk_wait_all();
   tc_fence_before();
   __syncthreads();
   if (warp == 0) tmem_dealloc(tb, 512);
