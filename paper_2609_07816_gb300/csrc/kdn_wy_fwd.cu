@@ -84,7 +84,7 @@ constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kMinHalfG = -80.f;  // c = G_C / 2 below this: out of range
 constexpr int kPrepThreads = 256;   // warps 4-11: the preparing pass
 constexpr int kMain = 384;          // warps 4-15: everything but the gain
-constexpr int kBarPrep = 1, kBarMain = 2, kBarGain = 3;  // named barriers (0 = __syncthreads)
+constexpr int kBarMain = 2, kBarGain = 3;  // named barriers (0 = __syncthreads)
 constexpr int kTmaThread = 224;  // warp 7, lane 0: issues each chunk's next-chunk TMA operations
 
 // shared-memory map (bytes from the 1024-aligned base)
@@ -622,15 +622,18 @@ __global__ void __launch_bounds__(WT, 1)
     auto lga_t = [&](int t) {  // log alpha of token t in the loop
       return LG ? *reinterpret_cast<const float *>(pb + sw32_off(t, cb)) : lga(raw(pg, t), t);
     };
-    float g0 = 0.f, g1 = 0.f, g2 = 0.f, g3 = 0.f;
+    // G_C, and the sums of the chunk's eight 8-token segments for the preparing pass
+    // (which reads them at the next chunk boundary; it is done with the previous chunk's)
+    float GC = 0.f;
 #pragma unroll
-    for (int t = 0; t < CM; t += 4) {
-      g0 += lga_keep(t);
-      g1 += lga_keep(t + 1);
-      g2 += lga_keep(t + 2);
-      g3 += lga_keep(t + 3);
+    for (int sg = 0; sg < 8; ++sg) {
+      const int t = 8 * sg;
+      const float ss = ((lga_keep(t) + lga_keep(t + 1)) + (lga_keep(t + 2) + lga_keep(t + 3))) +
+                       ((lga_keep(t + 4) + lga_keep(t + 5)) + (lga_keep(t + 6) + lga_keep(t + 7)));
+      s_part[sg * D + i] = ss;
+      GC += ss;
     }
-    const float GC = (g0 + g1) + (g2 + g3), cref = 0.5f * GC;
+    const float cref = 0.5f * GC;
     s_c[i] = cref;
     // out of the referenced factors' range in some channel: this chunk forms T' and A'_qk
     // from exp(G_t - G_s) directly
@@ -767,7 +770,6 @@ __global__ void __launch_bounds__(WT, 1)
       const uint32_t sl8 = (uint32_t)(i0 >> 6) * 8192u;  // 64-channel slab of a [t][64] 16-bit tile
       // the chunk's g for this thread's 8 tokens and 4 channels (8 bytes a token)
       uint2 gq[8];
-      float ps[4] = {0.f, 0.f, 0.f, 0.f};
       const int tv = a.T - c * CM;  // logit gates: tokens past T are identity updates
       const bool oor = !SV && s_oor[c & 1] != 0;
       auto unpack_lga = [&](uint2 u, int t, float *gv) {
@@ -778,15 +780,8 @@ __global__ void __launch_bounds__(WT, 1)
         }
       };
 #pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        gq[j] = *reinterpret_cast<const uint2 *>(rg + sl8 + sw128_off4(t0 + j, i0));
-        float gv[4];
-        unpack_lga(gq[j], t0 + j, gv);
-#pragma unroll
-        for (int u = 0; u < 4; ++u) ps[u] += gv[u];
-      }
-      *reinterpret_cast<float4 *>(s_part + seg * D + i0) = make_float4(ps[0], ps[1], ps[2], ps[3]);
-      bar_sync(kBarPrep, kPrepThreads);
+      for (int j = 0; j < 8; ++j) gq[j] = *reinterpret_cast<const uint2 *>(rg + sl8 + sw128_off4(t0 + j, i0));
+      // G at the start of this thread's segment from the segment sums the gain formed
       float cr[4], G[4] = {0.f, 0.f, 0.f, 0.f}, Ec[4], gm[4];
       {
         const float4 c4 = *reinterpret_cast<const float4 *>(s_c + i0);
