@@ -57,8 +57,9 @@
 // parameterisation (Sec. 5): log alpha = -softplus(-x), omega = softplus(y),
 // r = r_min + softplus(z), formed in float32.  The gain forms log alpha once per
 // element and keeps it in its column of the Kk' tile until the recursion
-// overwrites it; the prepare pass forms its own; the tokens past T are identity
-// updates.  (The context-saving forward with logit gates runs k_fused_fwd.)
+// overwrites it; the prepare pass forms its own.  The tokens past T are identity
+// updates: their rows of the g and omega tiles are set to logits whose
+// activations are exactly alpha = 1 and omega = 0, so no pass masks elements.
 //
 // Every wait on an mbarrier is bounded; on timeout the kernel records
 // KDN_ERR_TIMEOUT in the status word, waits (bounded) for its copies in flight,
@@ -81,6 +82,7 @@ constexpr int D = 128;   // d_k = d_v
 constexpr uint32_t kWait = 1u << 25;
 constexpr uint32_t kDrain = 1u << 14;  // bounded waits of the failure path
 constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kLn2 = 0.6931471805599453f;
 constexpr float kMinHalfG = -80.f;  // c = G_C / 2 below this: out of range
 constexpr int kPrepThreads = 256;   // warps 4-11: the preparing pass
 constexpr int kMain = 384;          // warps 4-15: everything but the gain
@@ -125,6 +127,16 @@ __device__ __forceinline__ float rcpf(float x) {
   float y;
   asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
+}
+__device__ __forceinline__ float lg2f(float x) {
+  float y;
+  asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+// softplus(x) = max(x, 0) + log(1 + exp(-|x|)), from the two approximate base-2
+// operations with subnormals flushed (exactly 0 below x = -88)
+__device__ __forceinline__ float softplus_w(float x) {
+  return fmaxf(x, 0.f) + kLn2 * lg2f(1.f + ex2f(-fabsf(x) * kLog2e));
 }
 // round to tf32 (nearest, ties away): the tensor core reads the top 19 bits
 __device__ __forceinline__ float tf32r(float x) {
@@ -569,7 +581,7 @@ __global__ void __launch_bounds__(WT, 1)
       rnext = 1.f;
       if (c < NC && c * CM + tid < a.T) {
         const float z = ld<__nv_bfloat16>(a.r, tok_index(a, b, c * CM + tid, h));
-        rnext = LG ? a.rmin + softplus_f(z) : z;  // r = r_min + softplus(z) (Sec. 5)
+        rnext = LG ? a.rmin + softplus_w(z) : z;  // r = r_min + softplus(z) (Sec. 5)
       }
     }
   };
@@ -604,34 +616,59 @@ __global__ void __launch_bounds__(WT, 1)
     auto raw = [&](const unsigned char *base, int t) {
       return __bfloat162float(*reinterpret_cast<const __nv_bfloat16 *>(base + sw128_off(t, cl)));
     };
-    // log alpha and omega of token t (logit gates: the tokens past T are identity updates)
-    const int tv = a.T - c * CM;
-    auto lga = [&](float x, int t) { return LG ? (t < tv ? -softplus_f(-x) : 0.f) : x; };
-    auto omg = [&](float y, int t) { return LG ? (t < tv ? softplus_f(y) : 0.f) : y; };
+    // log alpha and omega from the tile's values
+    auto lga = [&](float x) { return LG ? -softplus_w(-x) : x; };
+    auto omg = [&](float y) { return LG ? softplus_w(y) : y; };
+    // logit gates: the tokens past T must be identity updates (alpha = 1, omega = 0).
+    // Their rows of the g and omega tiles, zero-filled by TMA, get the logits +-1e30,
+    // whose activations are exactly those (softplus(-1e30) = 0), so that no pass
+    // masks its elements; the preparing pass reads the same rows
+    if (LG && a.T - c * CM < CM) {
+      const __nv_bfloat16 big = __float2bfloat16_rn(1e30f), nbig = __float2bfloat16_rn(-1e30f);
+      for (int t = a.T - c * CM; t < CM; ++t) {
+        *reinterpret_cast<__nv_bfloat16 *>(rg + (i >> 6) * 8192 + sw128_off(t, cl)) = big;
+        *reinterpret_cast<__nv_bfloat16 *>(rw + (i >> 6) * 8192 + sw128_off(t, cl)) = nbig;
+      }
+    }
     unsigned char *pb = tb + (i >> 5) * 8192;
     const int cb = i & 31;
     // logit gates: log alpha is formed once per element here and kept (fp32) in this
     // channel's column of the Kk' tile, which the loop below overwrites token by token
     // after reading it; the tile is free once MMA-T of chunk c - 1 has read it
     if (LG && c > 0) g_ok = mbar_wait(bar_t, (c - 1) & 1, kWait) && g_ok;
-    auto lga_keep = [&](int t) {
-      const float la = lga(raw(pg, t), t);
-      if (LG) *reinterpret_cast<float *>(pb + sw32_off(t, cb)) = la;
-      return la;
-    };
     auto lga_t = [&](int t) {  // log alpha of token t in the loop
-      return LG ? *reinterpret_cast<const float *>(pb + sw32_off(t, cb)) : lga(raw(pg, t), t);
+      return LG ? *reinterpret_cast<const float *>(pb + sw32_off(t, cb)) : lga(raw(pg, t));
     };
     // G_C, and the sums of the chunk's eight 8-token segments for the preparing pass
     // (which reads them at the next chunk boundary; it is done with the previous chunk's)
+    // (logit gates: 16 tokens at a time, their loads ahead of the stores of log alpha,
+    // which the compiler must otherwise keep in order with the next loads)
     float GC = 0.f;
+    if constexpr (!LG) {
 #pragma unroll
-    for (int sg = 0; sg < 8; ++sg) {
-      const int t = 8 * sg;
-      const float ss = ((lga_keep(t) + lga_keep(t + 1)) + (lga_keep(t + 2) + lga_keep(t + 3))) +
-                       ((lga_keep(t + 4) + lga_keep(t + 5)) + (lga_keep(t + 6) + lga_keep(t + 7)));
-      s_part[sg * D + i] = ss;
-      GC += ss;
+      for (int sg = 0; sg < 8; ++sg) {
+        const int t = 8 * sg;
+        const float ss = ((raw(pg, t) + raw(pg, t + 1)) + (raw(pg, t + 2) + raw(pg, t + 3))) +
+                         ((raw(pg, t + 4) + raw(pg, t + 5)) + (raw(pg, t + 6) + raw(pg, t + 7)));
+        s_part[sg * D + i] = ss;
+        GC += ss;
+      }
+    } else {
+#pragma unroll
+    for (int s2 = 0; s2 < 4; ++s2) {
+      float x[16];
+#pragma unroll
+      for (int j = 0; j < 16; ++j) x[j] = lga(raw(pg, 16 * s2 + j));
+#pragma unroll
+      for (int h2 = 0; h2 < 2; ++h2) {
+        const float *y = x + 8 * h2;
+        const float ss = ((y[0] + y[1]) + (y[2] + y[3])) + ((y[4] + y[5]) + (y[6] + y[7]));
+        s_part[(2 * s2 + h2) * D + i] = ss;
+        GC += ss;
+      }
+#pragma unroll
+      for (int j = 0; j < 16; ++j) *reinterpret_cast<float *>(pb + sw32_off(16 * s2 + j, cb)) = x[j];
+    }
     }
     const float cref = 0.5f * GC;
     s_c[i] = cref;
@@ -652,7 +689,7 @@ __global__ void __launch_bounds__(WT, 1)
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
       gb[j] = lga_t(j);
-      wb[j] = omg(raw(pw, j), j);
+      wb[j] = omg(raw(pw, j));
       kb8[j] = raw(pk, j);
     }
     {
@@ -673,7 +710,7 @@ __global__ void __launch_bounds__(WT, 1)
           const int t = 8 * blk + j;
           const float lg = lga_t(t), kk = raw(pk, t);
           const float al = ex2f(lg * kLog2e);
-          const float ph = fmaf(al * al, p, omg(raw(pw, t), t));
+          const float ph = fmaf(al * al, p, omg(raw(pw, t)));
           const float den = fmaf(kk * kk * smur[t], ph, 1.f);
           p = ph * rcpf(den);
           Gt += lg;
@@ -696,7 +733,7 @@ __global__ void __launch_bounds__(WT, 1)
           for (int j = 0; j < 8; ++j) {
             const int t = 8 * (blk + 1) + j;
             gn[j] = lga_t(t);
-            wn[j] = omg(raw(pw, t), t);
+            wn[j] = omg(raw(pw, t));
             kn[j] = raw(pk, t);
           }
           const float4 m0 = *reinterpret_cast<const float4 *>(smur + 8 * (blk + 1));
@@ -770,13 +807,13 @@ __global__ void __launch_bounds__(WT, 1)
       const uint32_t sl8 = (uint32_t)(i0 >> 6) * 8192u;  // 64-channel slab of a [t][64] 16-bit tile
       // the chunk's g for this thread's 8 tokens and 4 channels (8 bytes a token)
       uint2 gq[8];
-      const int tv = a.T - c * CM;  // logit gates: tokens past T are identity updates
       const bool oor = !SV && s_oor[c & 1] != 0;
-      auto unpack_lga = [&](uint2 u, int t, float *gv) {
+      // (logit gates: the rows past T hold logits whose log alpha is exactly 0)
+      auto unpack_lga = [&](uint2 u, float *gv) {
         unpack_bf4(u, gv);
         if (LG) {
 #pragma unroll
-          for (int w = 0; w < 4; ++w) gv[w] = t < tv ? -softplus_f(-gv[w]) : 0.f;
+          for (int w = 0; w < 4; ++w) gv[w] = -softplus_w(-gv[w]);
         }
       };
 #pragma unroll
@@ -802,7 +839,7 @@ __global__ void __launch_bounds__(WT, 1)
         for (int j = 0; j < 8; ++j) {
           const int t = t0 + j;
           float gv[4], kv[4], qv[4], e[4];
-          unpack_lga(gq[j], t, gv);
+          unpack_lga(gq[j], gv);
           unpack_bf4(*reinterpret_cast<const uint2 *>(rk + sl8 + sw128_off4(t, i0)), kv);
           unpack_bf4(*reinterpret_cast<const uint2 *>(rq + sl8 + sw128_off4(t, i0)), qv);
           if constexpr (RM) {  // G_t itself for the direct products; gamma_t = exp(G_t) (may underflow)
@@ -1183,10 +1220,8 @@ __global__ void __launch_bounds__(WT, 1)
 }  // namespace
 
 bool wy_fwd_supported(const Args &a, bool save) {
-  // The context-saving forward with logit gates stays on the first fused kernel: its
-  // gate conversions cost less there, and the backward it feeds has that kernel's
-  // decay range either way.
-  return a.variant == 0 && (a.gates == KDN_GATES_POST || (a.gates == KDN_GATES_LOGITS && !save)) &&
+  (void)save;
+  return a.variant == 0 && (a.gates == KDN_GATES_POST || a.gates == KDN_GATES_LOGITS) &&
          a.dtype == KDN_BF16 && a.dk == D && a.dv == D && a.T > 0 && a.chunk != 32;
 }
 
@@ -1201,7 +1236,7 @@ kdn_status_t launch_wy_fwd(const Args &a, cudaStream_t s, unsigned char *save_S,
       !make_map(&mv, a.v, a) || !make_map(&mq, a.q, a))
     return KDN_ERR_CUDA;
   const bool lg = a.gates == KDN_GATES_LOGITS;
-  const auto kern = save_S ? k_wy_fwd<1, 0> : (lg ? k_wy_fwd<0, 1> : k_wy_fwd<0, 0>);
+  const auto kern = save_S ? (lg ? k_wy_fwd<1, 1> : k_wy_fwd<1, 0>) : (lg ? k_wy_fwd<0, 1> : k_wy_fwd<0, 0>);
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES) !=
       cudaSuccess)
     return KDN_ERR_CUDA;
