@@ -190,6 +190,8 @@ kdn_status_t fwd_save_entry(int variant, const kdn_desc_t *d, const void *q, con
   if (st != KDN_OK) return st;
   const bool work = (size_t)a.B * a.H * a.T > 0;
   if (work && !use_fused_bwd(a)) return KDN_ERR_UNSUPPORTED;
+  // (the diagonal backward reads Y = V - Kbar S_in from the context, which the WY forward writes)
+  if (work && variant == 0 && !wy_fwd_supported(a, true)) return KDN_ERR_UNSUPPORTED;
   if (work && !ptrs_ok({q, k, v, g, omega, r, o, saved}, {S0, p0, ST, pT})) return KDN_ERR_INVALID_ARG;
   if (!work && !ptrs_ok({}, {S0, p0, ST, pT})) return KDN_ERR_INVALID_ARG;
   if (work && (saved_bytes < fused_saved_bytes(a) || ((uintptr_t)saved % kAlign)))

@@ -65,7 +65,7 @@ constexpr int KB = 1024;
 // across the stages of a chunk; the comments give the sequence of tenants.
 constexpr int O_RKQ = 0;         // raw k | q, interleaved per 64-channel slab (whole chunk)
 constexpr int O_SIN = 32 * KB;   // S_in fp16 [i][j] (context)  -> Kbar^T hi | Qbar^T hi (second set)
-constexpr int O_RV = 64 * KB;    // raw v  -> v fp16
+constexpr int O_RV = 64 * KB;    // raw v  -> v fp16 (isotropic); Y (context) -> dW^T bf16 (diagonal)
 constexpr int O_RDO = 80 * KB;   // raw dO -> lambda dO fp16 -> Qbar^T lo
 constexpr int O_AH = 96 * KB;    // A fp16 [t][s] (context)
 constexpr int O_AB = 104 * KB;   // A bf16 [t][s] (from the saved fp16 A)
@@ -83,6 +83,8 @@ constexpr int O_DRT = O_KT, O_KKH2 = O_WN;
 constexpr int O_DSH = O_G, O_DAQ = O_G, O_QH = O_G + 16 * KB, O_KKL2 = O_G + 16 * KB;
 constexpr int O_DWT = O_G, O_DAT = O_G + 16 * KB, O_XT = O_G + 24 * KB, O_KQH2 = O_SIN;
 constexpr int O_QL2 = O_RDO, O_DRTL = O_RH;
+// Diagonal KDN: Y (context) in the v buffer, then dW^T; dA^T over A_qk
+constexpr int O_DWY = O_RV, O_DAY = O_AQ;
 // small arrays
 constexpr int OFF_SM = BUF_END;
 constexpr int SMALL_FLOATS = 64 * 18 + 256 * 2 + 128 * 2 + 16;
@@ -251,8 +253,9 @@ __global__ void __launch_bounds__(BT, 1)
 
   // loads of chunk c on bar_a: the context record (S_in, R, -W, A_qk, A; issued as
   // soon as their buffers free up) and the raw k, q, g, omega tiles (issued once the
-  // previous chunk is done; the one expect_tx covers both groups); bar_b <- dO, v
-  const uint32_t kBytesA = 81920u + 16384u * 2;
+  // previous chunk is done; the one expect_tx covers both groups); bar_b <- dO (isotropic: and v)
+  // (diagonal KDN: the context's Y in place of v)
+  const uint32_t kBytesA = 81920u + 16384u * 2 + (V == 0 ? 16384u : 0u);
   auto issue_a_ctx = [&](int c) {
     const unsigned char *rec = a.fSin + ((size_t)bh * NC + c) * kCtxBytes;
     mbar_expect_tx(bar_a, kBytesA);
@@ -261,6 +264,7 @@ __global__ void __launch_bounds__(BT, 1)
     bulk_g2s(sm + O_WN, rec + kCtxW, 16384, bar_a);
     bulk_g2s(sm + O_AQ, rec + kCtxAqk, 8192, bar_a);
     bulk_g2s(sm + O_AH, rec + kCtxA, 8192, bar_a);
+    if (V == 0) bulk_g2s(rv, rec + kCtxY, 16384, bar_a);
   };
   auto issue_a_raw = [&](int c) {
     for (int s = 0; s < 2; ++s) {
@@ -269,7 +273,7 @@ __global__ void __launch_bounds__(BT, 1)
     }
   };
   auto issue_b_do = [&](int c) {
-    mbar_expect_tx(bar_b, 32768);
+    mbar_expect_tx(bar_b, V == 0 ? 16384 : 32768);  // (isotropic: and v)
     for (int s = 0; s < 2; ++s) tma_load_4d(rdo + s * 8192, &mdo, bar_b, 64 * s, h, c * CM, b);
   };
   auto issue_b_v = [&](int c) {
@@ -279,7 +283,7 @@ __global__ void __launch_bounds__(BT, 1)
     issue_a_ctx(NC - 1);
     issue_a_raw(NC - 1);
     issue_b_do(NC - 1);
-    issue_b_v(NC - 1);
+    if (V != 0) issue_b_v(NC - 1);
   }
 
   // ---- cotangent scale lambda = 2^-e with max(|dO|, |dS_T|) * lambda in [1, 2)
@@ -512,8 +516,10 @@ __global__ void __launch_bounds__(BT, 1)
 #pragma unroll
       for (int j = 0; j < 8; ++j) v[j] *= lam;
       sm16(rdo, off) = pack_h8(v);
-      unpack_bf8(sm16(rv, off), v);
-      sm16(rv, off) = pack_h8(v);
+      if (V != 0) {
+        unpack_bf8(sm16(rv, off), v);
+        sm16(rv, off) = pack_h8(v);
+      }
     }
     tmem_st_wait();
     fence_proxy_async();
@@ -591,200 +597,349 @@ __global__ void __launch_bounds__(BT, 1)
     fence_proxy_async();
     tc_fence_before();
     __syncthreads();
-    // ---- [12] B2: TS += Qbar^T dO - W^T dR;  B5: X1 = -dW^T;  B7: X2 = dV^T (dR as hi + lo fp16);
-    //           B8a: X3 = (dO S_in^T)^T
-    if (tid == 0) {
-      tc_fence_after();
-      const uint32_t idS01 = idesc_f16(128, 128, 0, 1), idS10 = idesc_f16(128, 128, 1, 0);
-      const uint32_t id01 = idesc_f16(128, 64, 0, 1), id00 = idesc_f16(128, 64, 0, 0);
-      for (int kk = 0; kk < 4; ++kk) {
-        umma_bf16(TS, kdesc(sm + O_QH + kk * 32), mdesc(rdo + kk * 2048, 8192), idS01, 1);
-        umma_bf16(TS, mdesc(sm + O_WN + kk * 2048, 8192), kdesc(sm + O_DRT + kk * 32), idS10, 1);
-        const uint64_t ah = mdesc(sm + O_AH + kk * 2048, 8192);
-        umma_bf16(X2, kdesc(sm + O_DRT + kk * 32), ah, id01, kk > 0);
-        umma_bf16(X2, kdesc(sm + O_DRTL + kk * 32), ah, id01, 1);
+    if constexpr (V == 0) {
+      // Diagonal KDN: five tensor-core rounds.  With Y = V - Kbar S_in (the tile the
+      // forward formed R = A Y from, in the context), dA = dR V^T + dW Kbar^T =
+      // dR Y^T, since dW = -dR S_in^T: it comes out of the round that forms dR's
+      // other products, and X = A^T dA one round later.
+      // ---- [12] B2: TS += Qbar^T dO - W^T dR;  B5: X1 = -dW^T;  B6: X2 = dA^T = (dR Y^T)^T;
+      //           B8a: X3 = (dO S_in^T)^T
+      if (tid == 0) {
+        tc_fence_after();
+        const uint32_t idS01 = idesc_f16(128, 128, 0, 1), idS10 = idesc_f16(128, 128, 1, 0);
+        const uint32_t id01 = idesc_f16(128, 64, 0, 1), id00 = idesc_f16(128, 64, 0, 0);
+        for (int kk = 0; kk < 4; ++kk) {
+          umma_bf16(TS, kdesc(sm + O_QH + kk * 32), mdesc(rdo + kk * 2048, 8192), idS01, 1);
+          umma_bf16(TS, mdesc(sm + O_WN + kk * 2048, 8192), kdesc(sm + O_DRT + kk * 32), idS10, 1);
+        }
+        for (int kk = 0; kk < 8; ++kk) {
+          const uint64_t as = kdesc(sin + (kk >> 2) * 16384 + (kk & 3) * 32);
+          const uint64_t drt = mdesc(sm + O_DRT + kk * 2048, 8192);
+          umma_bf16(X1, as, drt, id01, kk > 0);
+          umma_bf16(X3, as, kdesc(rdo + (kk >> 2) * 8192 + (kk & 3) * 32), id00, kk > 0);
+          umma_bf16(X2, kdesc(rv + (kk >> 2) * 8192 + (kk & 3) * 32), drt, id01, kk > 0);
+        }
+        umma_commit(bar_mma);
       }
-      for (int kk = 0; kk < 8; ++kk) {
-        const uint64_t as = kdesc(sin + (kk >> 2) * 16384 + (kk & 3) * 32);
-        umma_bf16(X1, as, mdesc(sm + O_DRT + kk * 2048, 8192), id01, kk > 0);
-        umma_bf16(X3, as, kdesc(rdo + (kk >> 2) * 8192 + (kk & 3) * 32), id00, kk > 0);
-      }
-      umma_commit(bar_mma);
-    }
-    if (!(ok = mma_wait())) break;
-    tc_fence_after();
-    // ---- [13] second operand set: [Kbar; Qbar] hi (interleaved), Qbar lo, Kk hi / lo;
-    //           B8b: X3 += (dA_qk Kk)^T;  B9a: X0 += (dA_qk^T Qbar)^T
-    {
-      float gf[16], ga[16], v[16];
-      load_gain(gf, ga);
-#pragma unroll
-      for (int j = 0; j < 16; ++j) v[j] = ga[j] * raw_k(t0 + j);
-      st_row16_bf(sm + O_KQH2, ci, qq, v);  // Kbar^T hi
-    }
-    if (!SD) {
-      float gf[16], ga[16], v[16];
-      load_gain(gf, ga);
-#pragma unroll
-      for (int j = 0; j < 16; ++j) v[j] = tau * ga[j] * raw_q(t0 + j);
-      st_row16_split(sm + O_KQH2 + 16384, sm + O_QL2, ci, qq, v);  // Qbar^T hi / lo
-#pragma unroll
-      for (int j = 0; j < 16; ++j) v[j] = __fdividef(gf[j] * raw_k(t0 + j), ga[j]);
-      st_row16_split(sm + O_KKH2, sm + O_KKL2, ci, qq, v);  // Kk^T hi / lo
-    }
-    fence_proxy_async();
-    tc_fence_before();
-    __syncthreads();
-    if (SD && tid == 0) {  // raw K^T, Q^T (channel-major) against the scaled 64 x 64 partners
+      if (!(ok = mma_wait())) break;
       tc_fence_after();
-      const uint32_t id11 = idesc_bf16(128, 64, 1, 1), id10 = idesc_bf16(128, 64, 1, 0);
-      for (int kk = 0; kk < 4; ++kk) {
-        const uint64_t kt = mdesc(rkq + kk * 2048, 16384), qt = mdesc(rkq + 8192 + kk * 2048, 16384);
-        umma_bf16(X3, kt, mdesc(sm + O_DAQ + kk * 2048, 8192), id11, 1);
-        umma_bf16(X3, kt, mdesc(sm + O_DAQ + 8192 + kk * 2048, 8192), id11, 1);
-        umma_bf16(X0, qt, kdesc(sm + O_AQ + kk * 32), id10, 1);
-        umma_bf16(X0, qt, kdesc(sm + O_DT + kk * 32), id10, 1);
-      }
-      umma_commit(bar_mma);
-    }
-    if (!SD && tid == 0) {
-      tc_fence_after();
-      const uint32_t id01 = idesc_bf16(128, 64, 0, 1), id00 = idesc_bf16(128, 64, 0, 0);
-      for (int kk = 0; kk < 4; ++kk) {
-        const uint64_t kh = kdesc(sm + O_KKH2 + kk * 32), kl = kdesc(sm + O_KKL2 + kk * 32);
-        const uint64_t dh = mdesc(sm + O_DAQ + kk * 2048, 8192), dl = mdesc(sm + O_DAQ + 8192 + kk * 2048, 8192);
-        umma_bf16(X3, kh, dh, id01, 1);
-        umma_bf16(X3, kl, dh, id01, 1);
-        umma_bf16(X3, kh, dl, id01, 1);
-        const uint64_t qh = kdesc(sm + O_KQH2 + 16384 + kk * 32), ql = kdesc(sm + O_QL2 + kk * 32);
-        const uint64_t eh = kdesc(sm + O_DAQ + kk * 32), el = kdesc(sm + O_DAQ + 8192 + kk * 32);
-        umma_bf16(X0, qh, eh, id00, 1);
-        umma_bf16(X0, ql, eh, id00, 1);
-        umma_bf16(X0, qh, el, id00, 1);
-      }
-      umma_commit(bar_mma);
-    }
-    if (!(ok = mma_wait())) break;
-    tc_fence_after();
-    if (tid == 0 && c > 0) issue_b_do(c - 1);  // dO / Qbar lo buffer is free
-    // ---- [14] dW^T -> bf16 [i][t];  dV^T -> dv
-    {
-      const int j = 32 * wq + lane, tc0 = 16 * wg;
-      float v[16];
-      tmem_ld16(X1 + lane_base + tc0, v);
+      // ---- [13] dW^T -> bf16 [i][t] (over Y);  dA^T -> fp16 [s][t] (over A_qk);
+      //           second operand set: [Kbar; Qbar] hi (interleaved), Qbar lo, Kk hi / lo
+      {
+        const int j = 32 * wq + lane, tc0 = 16 * wg;
+        float v[16];
+        tmem_ld16(X1 + lane_base + tc0, v);
 #pragma unroll
-      for (int u = 0; u < 16; ++u) v[u] = -v[u];
-      sm16(sm + O_DWT, chunk_off(j, tc0 >> 3)) = pack_bf8(v);
-      sm16(sm + O_DWT, chunk_off(j, (tc0 >> 3) + 1)) = pack_bf8(v + 8);
-      tmem_ld16(X2 + lane_base + tc0, v);
-#pragma unroll
-      for (int u = 0; u < 16; ++u) {
-        const int t = c * CM + tc0 + u;
-        if (t < a.T) st_grad<OBF>(a.dv_, tok_index(a, b, t, h) * D + j, v[u] * invl);
+        for (int u = 0; u < 16; ++u) v[u] = -v[u];
+        sm16(sm + O_DWY, chunk_off(j, tc0 >> 3)) = pack_bf8(v);
+        sm16(sm + O_DWY, chunk_off(j, (tc0 >> 3) + 1)) = pack_bf8(v + 8);
+        if (wq < 2) {
+          tmem_ld16(X2 + lane_base + tc0, v);
+          sm16(sm + O_DAY, chunk_off(j, tc0 >> 3)) = pack_h8(v);
+          sm16(sm + O_DAY, chunk_off(j, (tc0 >> 3) + 1)) = pack_h8(v + 8);
+        }
       }
-    }
-    fence_proxy_async();
-    tc_fence_before();
-    __syncthreads();
-    // ---- [15] B6: X1 = dA^T = (dR V^T + dW Kbar^T)^T;  B10a: X2 = (A^T dW)^T
-    if (tid == 0) {
-      tc_fence_after();
-      const uint32_t ih01 = idesc_f16(128, 64, 0, 1), ib01 = idesc_bf16(128, 64, 0, 1);
-      const uint32_t ib11 = idesc_bf16(128, 64, 1, 1);
-      for (int kk = 0; kk < 8; ++kk) {
-        umma_bf16(X1, kdesc(rv + (kk >> 2) * 8192 + (kk & 3) * 32), mdesc(sm + O_DRT + kk * 2048, 8192),
-                  ih01, kk > 0);
-        umma_bf16(X1, mdesc(sm + O_KQH2 + kk * 2048, 16384), mdesc(sm + O_DWT + kk * 2048, 8192), ib11,
-                  1);
+      {
+        float gf[16], ga[16], v[16];
+        load_gain(gf, ga);
+#pragma unroll
+        for (int j = 0; j < 16; ++j) v[j] = ga[j] * raw_k(t0 + j);
+        st_row16_bf(sm + O_KQH2, ci, qq, v);  // Kbar^T hi
       }
-      for (int kk = 0; kk < 4; ++kk)
-        umma_bf16(X2, kdesc(sm + O_DWT + kk * 32), mdesc(sm + O_AB + kk * 2048, 8192), ib01, kk > 0);
-      umma_commit(bar_mma);
-    }
-    if (!(ok = mma_wait())) break;
-    tc_fence_after();
-    if (tid == 0 && c > 0) issue_b_v(c - 1);  // v buffer is free
-    if (WT && tid == 0) {  // this chunk's omega logits for pass C (B6 has read dR^T in O_KT,
-      mbar_expect_tx(bar_w, 16384);  // which is free until [3] of the next chunk)
-      for (int s = 0; s < 2; ++s) tma_load_4d(sm + O_KT + s * 8192, &mw, bar_w, 64 * s, h, c * CM, b);
-    }
-    // ---- [16] dT = strict_lower(-A^T dA A^T): X = A^T dA, Y = X A^T (fp16)
-    if (wq < 2) {
-      const int s = 32 * wq + lane, tc0 = 16 * wg;
-      float v[16];
-      tmem_ld16(X1 + lane_base + tc0, v);
-      sm16(sm + O_DAT, chunk_off(s, tc0 >> 3)) = pack_h8(v);
-      sm16(sm + O_DAT, chunk_off(s, (tc0 >> 3) + 1)) = pack_h8(v + 8);
-    }
-    fence_proxy_async();
-    tc_fence_before();
-    __syncthreads();
-    if (tid == 0) {
-      tc_fence_after();
-      const uint32_t id = idesc_f16(128, 64, 1, 0);
-      for (int kk = 0; kk < 4; ++kk)
-        umma_bf16(X1, mdesc(sm + O_AH + kk * 2048, 8192), kdesc(sm + O_DAT + kk * 32), id, kk > 0);
-      umma_commit(bar_mma);
-    }
-    if (!(ok = mma_wait())) break;
-    tc_fence_after();
-    if (wq < 2) {
-      const int r = 32 * wq + lane, tc0 = 16 * wg;
-      float v[16];
-      tmem_ld16(X1 + lane_base + tc0, v);
-      sm16(sm + O_XT, chunk_off(r, tc0 >> 3)) = pack_h8(v);
-      sm16(sm + O_XT, chunk_off(r, (tc0 >> 3) + 1)) = pack_h8(v + 8);
-    }
-    fence_proxy_async();
-    tc_fence_before();
-    __syncthreads();
-    if (tid == 0) {
-      tc_fence_after();
-      const uint32_t id = idesc_f16(128, 64, 0, 0);
-      for (int kk = 0; kk < 4; ++kk)
-        umma_bf16(X1, kdesc(sm + O_XT + kk * 32), kdesc(sm + O_AH + kk * 32), id, kk > 0);
-      umma_commit(bar_mma);
-    }
-    if (!(ok = mma_wait())) break;
-    tc_fence_after();
-    if (wq < 2) {
-      const int r = 32 * wq + lane, tc0 = 16 * wg;
-      float v[16];
-      tmem_ld16(X1 + lane_base + tc0, v);
+      {
+        float gf[16], ga[16], v[16];
+        load_gain(gf, ga);
 #pragma unroll
-      for (int u = 0; u < 16; ++u) v[u] = (tc0 + u < r) ? -v[u] : 0.f;
-      if (SD) {  // dT diag(beta / gamma) -> O_AQ (B10b); diag(gamma) dT below (B9b)
-        float w[16];
+        for (int j = 0; j < 16; ++j) v[j] = tau * ga[j] * raw_q(t0 + j);
+        st_row16_split(sm + O_KQH2 + 16384, sm + O_QL2, ci, qq, v);  // Qbar^T hi / lo
 #pragma unroll
-        for (int u = 0; u < 16; ++u) w[u] = v[u] * s_kf[tc0 + u];
-        sm16(sm + O_AQ, chunk_off(r, tc0 >> 3)) = pack_bf8(w);
-        sm16(sm + O_AQ, chunk_off(r, (tc0 >> 3) + 1)) = pack_bf8(w + 8);
-        const float f = s_gm[r];
-#pragma unroll
-        for (int u = 0; u < 16; ++u) v[u] *= f;
+        for (int j = 0; j < 16; ++j) v[j] = __fdividef(gf[j] * raw_k(t0 + j), ga[j]);
+        st_row16_split(sm + O_KKH2, sm + O_KKL2, ci, qq, v);  // Kk^T hi / lo
       }
-      sm16(sm + O_DT, chunk_off(r, tc0 >> 3)) = pack_bf8(v);
-      sm16(sm + O_DT, chunk_off(r, (tc0 >> 3) + 1)) = pack_bf8(v + 8);
-    }
-    fence_proxy_async();
-    tc_fence_before();
-    __syncthreads();
-    // ---- [17] B9b: X0 += (dT^T Kbar)^T;  B10b: X2 += (dT Kk)^T
-    if (tid == 0) {
+      fence_proxy_async();
+      tc_fence_before();
+      __syncthreads();
+      // ---- [14] B8b: X3 += (dA_qk Kk)^T;  B9a: X0 += (dA_qk^T Qbar)^T (hi/lo bf16 pairs);
+      //           B7: X2 = dV^T = (A^T dR)^T (dR as hi + lo fp16);  X1 = A^T dA (fp16)
+      if (tid == 0) {
+        tc_fence_after();
+        const uint32_t id01 = idesc_bf16(128, 64, 0, 1), id00 = idesc_bf16(128, 64, 0, 0);
+        const uint32_t ih01 = idesc_f16(128, 64, 0, 1), ih10 = idesc_f16(128, 64, 1, 0);
+        for (int kk = 0; kk < 4; ++kk) {
+          const uint64_t kh = kdesc(sm + O_KKH2 + kk * 32), kl = kdesc(sm + O_KKL2 + kk * 32);
+          const uint64_t dh = mdesc(sm + O_DAQ + kk * 2048, 8192), dl = mdesc(sm + O_DAQ + 8192 + kk * 2048, 8192);
+          umma_bf16(X3, kh, dh, id01, 1);
+          umma_bf16(X3, kl, dh, id01, 1);
+          umma_bf16(X3, kh, dl, id01, 1);
+          const uint64_t qh = kdesc(sm + O_KQH2 + 16384 + kk * 32), ql = kdesc(sm + O_QL2 + kk * 32);
+          const uint64_t eh = kdesc(sm + O_DAQ + kk * 32), el = kdesc(sm + O_DAQ + 8192 + kk * 32);
+          umma_bf16(X0, qh, eh, id00, 1);
+          umma_bf16(X0, ql, eh, id00, 1);
+          umma_bf16(X0, qh, el, id00, 1);
+          const uint64_t ah = mdesc(sm + O_AH + kk * 2048, 8192);
+          umma_bf16(X2, kdesc(sm + O_DRT + kk * 32), ah, ih01, kk > 0);
+          umma_bf16(X2, kdesc(sm + O_DRTL + kk * 32), ah, ih01, 1);
+          umma_bf16(X1, ah, kdesc(sm + O_DAY + kk * 32), ih10, kk > 0);
+        }
+        umma_commit(bar_mma);
+      }
+      if (!(ok = mma_wait())) break;
       tc_fence_after();
-      const uint32_t id01 = idesc_bf16(128, 64, 0, 1), id00 = idesc_bf16(128, 64, 0, 0);
-      const uint32_t id11 = idesc_bf16(128, 64, 1, 1), id10 = idesc_bf16(128, 64, 1, 0);
-      for (int kk = 0; kk < 4; ++kk) {
-        if (SD) {
-          const uint64_t kt = mdesc(rkq + kk * 2048, 16384);
-          umma_bf16(X0, kt, mdesc(sm + O_DT + kk * 2048, 8192), id11, 1);
-          umma_bf16(X2, kt, kdesc(sm + O_AQ + kk * 32), id10, 1);
-        } else {
+      if (tid == 0 && c > 0) issue_b_do(c - 1);  // the dO / Qbar lo buffer is free
+      if (WT && tid == 0) {  // this chunk's omega logits for pass C, into the dR^T buffer (free
+        mbar_expect_tx(bar_w, 16384);  // until [3] of the next chunk)
+        for (int s = 0; s < 2; ++s) tma_load_4d(sm + O_KT + s * 8192, &mw, bar_w, 64 * s, h, c * CM, b);
+      }
+      // ---- [15] dV^T -> dv;  X = A^T dA -> fp16 [r][s]
+      {
+        const int j = 32 * wq + lane, tc0 = 16 * wg;
+        float v[16];
+        tmem_ld16(X2 + lane_base + tc0, v);
+#pragma unroll
+        for (int u = 0; u < 16; ++u) {
+          const int t = c * CM + tc0 + u;
+          if (t < a.T) st_grad<OBF>(a.dv_, tok_index(a, b, t, h) * D + j, v[u] * invl);
+        }
+        if (wq < 2) {
+          tmem_ld16(X1 + lane_base + tc0, v);
+          sm16(sm + O_XT, chunk_off(j, tc0 >> 3)) = pack_h8(v);
+          sm16(sm + O_XT, chunk_off(j, (tc0 >> 3) + 1)) = pack_h8(v + 8);
+        }
+      }
+      fence_proxy_async();
+      tc_fence_before();
+      __syncthreads();
+      // ---- [16] X1 = X A^T (fp16), so that dT = strict_lower(-A^T dA A^T);  B10a: X2 = (A^T dW)^T
+      if (tid == 0) {
+        tc_fence_after();
+        const uint32_t ih00 = idesc_f16(128, 64, 0, 0), ib01 = idesc_bf16(128, 64, 0, 1);
+        for (int kk = 0; kk < 4; ++kk) {
+          umma_bf16(X1, kdesc(sm + O_XT + kk * 32), kdesc(sm + O_AH + kk * 32), ih00, kk > 0);
+          umma_bf16(X2, kdesc(sm + O_DWY + kk * 32), mdesc(sm + O_AB + kk * 2048, 8192), ib01, kk > 0);
+        }
+        umma_commit(bar_mma);
+      }
+      if (!(ok = mma_wait())) break;
+      tc_fence_after();
+      if (wq < 2) {  // dT -> bf16
+        const int r = 32 * wq + lane, tc0 = 16 * wg;
+        float v[16];
+        tmem_ld16(X1 + lane_base + tc0, v);
+#pragma unroll
+        for (int u = 0; u < 16; ++u) v[u] = (tc0 + u < r) ? -v[u] : 0.f;
+        sm16(sm + O_DT, chunk_off(r, tc0 >> 3)) = pack_bf8(v);
+        sm16(sm + O_DT, chunk_off(r, (tc0 >> 3) + 1)) = pack_bf8(v + 8);
+      }
+      fence_proxy_async();
+      tc_fence_before();
+      __syncthreads();
+      // ---- [17] B9b: X0 += (dT^T Kbar)^T;  B10b: X2 += (dT Kk)^T
+      if (tid == 0) {
+        tc_fence_after();
+        const uint32_t id01 = idesc_bf16(128, 64, 0, 1), id00 = idesc_bf16(128, 64, 0, 0);
+        for (int kk = 0; kk < 4; ++kk) {
           umma_bf16(X0, kdesc(sm + O_KQH2 + kk * 32), mdesc(sm + O_DT + kk * 2048, 8192), id01, 1);
           umma_bf16(X2, kdesc(sm + O_KKH2 + kk * 32), kdesc(sm + O_DT + kk * 32), id00, 1);
         }
+        umma_commit(bar_mma);
       }
-      umma_commit(bar_mma);
+    } else {
+      // Isotropic KDN: seven rounds (its context keeps no Y; B6 forms dA from V and dW)
+      // ---- [12] B2: TS += Qbar^T dO - W^T dR;  B5: X1 = -dW^T;  B7: X2 = dV^T (dR as hi + lo fp16);
+      //           B8a: X3 = (dO S_in^T)^T
+      if (tid == 0) {
+        tc_fence_after();
+        const uint32_t idS01 = idesc_f16(128, 128, 0, 1), idS10 = idesc_f16(128, 128, 1, 0);
+        const uint32_t id01 = idesc_f16(128, 64, 0, 1), id00 = idesc_f16(128, 64, 0, 0);
+        for (int kk = 0; kk < 4; ++kk) {
+          umma_bf16(TS, kdesc(sm + O_QH + kk * 32), mdesc(rdo + kk * 2048, 8192), idS01, 1);
+          umma_bf16(TS, mdesc(sm + O_WN + kk * 2048, 8192), kdesc(sm + O_DRT + kk * 32), idS10, 1);
+          const uint64_t ah = mdesc(sm + O_AH + kk * 2048, 8192);
+          umma_bf16(X2, kdesc(sm + O_DRT + kk * 32), ah, id01, kk > 0);
+          umma_bf16(X2, kdesc(sm + O_DRTL + kk * 32), ah, id01, 1);
+        }
+        for (int kk = 0; kk < 8; ++kk) {
+          const uint64_t as = kdesc(sin + (kk >> 2) * 16384 + (kk & 3) * 32);
+          umma_bf16(X1, as, mdesc(sm + O_DRT + kk * 2048, 8192), id01, kk > 0);
+          umma_bf16(X3, as, kdesc(rdo + (kk >> 2) * 8192 + (kk & 3) * 32), id00, kk > 0);
+        }
+        umma_commit(bar_mma);
+      }
+      if (!(ok = mma_wait())) break;
+      tc_fence_after();
+      // ---- [13] second operand set: [Kbar; Qbar] hi (interleaved), Qbar lo, Kk hi / lo;
+      //           B8b: X3 += (dA_qk Kk)^T;  B9a: X0 += (dA_qk^T Qbar)^T
+      {
+        float gf[16], ga[16], v[16];
+        load_gain(gf, ga);
+  #pragma unroll
+        for (int j = 0; j < 16; ++j) v[j] = ga[j] * raw_k(t0 + j);
+        st_row16_bf(sm + O_KQH2, ci, qq, v);  // Kbar^T hi
+      }
+      if (!SD) {
+        float gf[16], ga[16], v[16];
+        load_gain(gf, ga);
+  #pragma unroll
+        for (int j = 0; j < 16; ++j) v[j] = tau * ga[j] * raw_q(t0 + j);
+        st_row16_split(sm + O_KQH2 + 16384, sm + O_QL2, ci, qq, v);  // Qbar^T hi / lo
+  #pragma unroll
+        for (int j = 0; j < 16; ++j) v[j] = __fdividef(gf[j] * raw_k(t0 + j), ga[j]);
+        st_row16_split(sm + O_KKH2, sm + O_KKL2, ci, qq, v);  // Kk^T hi / lo
+      }
+      fence_proxy_async();
+      tc_fence_before();
+      __syncthreads();
+      if (SD && tid == 0) {  // raw K^T, Q^T (channel-major) against the scaled 64 x 64 partners
+        tc_fence_after();
+        const uint32_t id11 = idesc_bf16(128, 64, 1, 1), id10 = idesc_bf16(128, 64, 1, 0);
+        for (int kk = 0; kk < 4; ++kk) {
+          const uint64_t kt = mdesc(rkq + kk * 2048, 16384), qt = mdesc(rkq + 8192 + kk * 2048, 16384);
+          umma_bf16(X3, kt, mdesc(sm + O_DAQ + kk * 2048, 8192), id11, 1);
+          umma_bf16(X3, kt, mdesc(sm + O_DAQ + 8192 + kk * 2048, 8192), id11, 1);
+          umma_bf16(X0, qt, kdesc(sm + O_AQ + kk * 32), id10, 1);
+          umma_bf16(X0, qt, kdesc(sm + O_DT + kk * 32), id10, 1);
+        }
+        umma_commit(bar_mma);
+      }
+      if (!SD && tid == 0) {
+        tc_fence_after();
+        const uint32_t id01 = idesc_bf16(128, 64, 0, 1), id00 = idesc_bf16(128, 64, 0, 0);
+        for (int kk = 0; kk < 4; ++kk) {
+          const uint64_t kh = kdesc(sm + O_KKH2 + kk * 32), kl = kdesc(sm + O_KKL2 + kk * 32);
+          const uint64_t dh = mdesc(sm + O_DAQ + kk * 2048, 8192), dl = mdesc(sm + O_DAQ + 8192 + kk * 2048, 8192);
+          umma_bf16(X3, kh, dh, id01, 1);
+          umma_bf16(X3, kl, dh, id01, 1);
+          umma_bf16(X3, kh, dl, id01, 1);
+          const uint64_t qh = kdesc(sm + O_KQH2 + 16384 + kk * 32), ql = kdesc(sm + O_QL2 + kk * 32);
+          const uint64_t eh = kdesc(sm + O_DAQ + kk * 32), el = kdesc(sm + O_DAQ + 8192 + kk * 32);
+          umma_bf16(X0, qh, eh, id00, 1);
+          umma_bf16(X0, ql, eh, id00, 1);
+          umma_bf16(X0, qh, el, id00, 1);
+        }
+        umma_commit(bar_mma);
+      }
+      if (!(ok = mma_wait())) break;
+      tc_fence_after();
+      if (tid == 0 && c > 0) issue_b_do(c - 1);  // dO / Qbar lo buffer is free
+      // ---- [14] dW^T -> bf16 [i][t];  dV^T -> dv
+      {
+        const int j = 32 * wq + lane, tc0 = 16 * wg;
+        float v[16];
+        tmem_ld16(X1 + lane_base + tc0, v);
+  #pragma unroll
+        for (int u = 0; u < 16; ++u) v[u] = -v[u];
+        sm16(sm + O_DWT, chunk_off(j, tc0 >> 3)) = pack_bf8(v);
+        sm16(sm + O_DWT, chunk_off(j, (tc0 >> 3) + 1)) = pack_bf8(v + 8);
+        tmem_ld16(X2 + lane_base + tc0, v);
+  #pragma unroll
+        for (int u = 0; u < 16; ++u) {
+          const int t = c * CM + tc0 + u;
+          if (t < a.T) st_grad<OBF>(a.dv_, tok_index(a, b, t, h) * D + j, v[u] * invl);
+        }
+      }
+      fence_proxy_async();
+      tc_fence_before();
+      __syncthreads();
+      // ---- [15] B6: X1 = dA^T = (dR V^T + dW Kbar^T)^T;  B10a: X2 = (A^T dW)^T
+      if (tid == 0) {
+        tc_fence_after();
+        const uint32_t ih01 = idesc_f16(128, 64, 0, 1), ib01 = idesc_bf16(128, 64, 0, 1);
+        const uint32_t ib11 = idesc_bf16(128, 64, 1, 1);
+        for (int kk = 0; kk < 8; ++kk) {
+          umma_bf16(X1, kdesc(rv + (kk >> 2) * 8192 + (kk & 3) * 32), mdesc(sm + O_DRT + kk * 2048, 8192),
+                    ih01, kk > 0);
+          umma_bf16(X1, mdesc(sm + O_KQH2 + kk * 2048, 16384), mdesc(sm + O_DWT + kk * 2048, 8192), ib11,
+                    1);
+        }
+        for (int kk = 0; kk < 4; ++kk)
+          umma_bf16(X2, kdesc(sm + O_DWT + kk * 32), mdesc(sm + O_AB + kk * 2048, 8192), ib01, kk > 0);
+        umma_commit(bar_mma);
+      }
+      if (!(ok = mma_wait())) break;
+      tc_fence_after();
+      if (tid == 0 && c > 0) issue_b_v(c - 1);  // v buffer is free
+      if (WT && tid == 0) {  // this chunk's omega logits for pass C (B6 has read dR^T in O_KT,
+        mbar_expect_tx(bar_w, 16384);  // which is free until [3] of the next chunk)
+        for (int s = 0; s < 2; ++s) tma_load_4d(sm + O_KT + s * 8192, &mw, bar_w, 64 * s, h, c * CM, b);
+      }
+      // ---- [16] dT = strict_lower(-A^T dA A^T): X = A^T dA, Y = X A^T (fp16)
+      if (wq < 2) {
+        const int s = 32 * wq + lane, tc0 = 16 * wg;
+        float v[16];
+        tmem_ld16(X1 + lane_base + tc0, v);
+        sm16(sm + O_DAT, chunk_off(s, tc0 >> 3)) = pack_h8(v);
+        sm16(sm + O_DAT, chunk_off(s, (tc0 >> 3) + 1)) = pack_h8(v + 8);
+      }
+      fence_proxy_async();
+      tc_fence_before();
+      __syncthreads();
+      if (tid == 0) {
+        tc_fence_after();
+        const uint32_t id = idesc_f16(128, 64, 1, 0);
+        for (int kk = 0; kk < 4; ++kk)
+          umma_bf16(X1, mdesc(sm + O_AH + kk * 2048, 8192), kdesc(sm + O_DAT + kk * 32), id, kk > 0);
+        umma_commit(bar_mma);
+      }
+      if (!(ok = mma_wait())) break;
+      tc_fence_after();
+      if (wq < 2) {
+        const int r = 32 * wq + lane, tc0 = 16 * wg;
+        float v[16];
+        tmem_ld16(X1 + lane_base + tc0, v);
+        sm16(sm + O_XT, chunk_off(r, tc0 >> 3)) = pack_h8(v);
+        sm16(sm + O_XT, chunk_off(r, (tc0 >> 3) + 1)) = pack_h8(v + 8);
+      }
+      fence_proxy_async();
+      tc_fence_before();
+      __syncthreads();
+      if (tid == 0) {
+        tc_fence_after();
+        const uint32_t id = idesc_f16(128, 64, 0, 0);
+        for (int kk = 0; kk < 4; ++kk)
+          umma_bf16(X1, kdesc(sm + O_XT + kk * 32), kdesc(sm + O_AH + kk * 32), id, kk > 0);
+        umma_commit(bar_mma);
+      }
+      if (!(ok = mma_wait())) break;
+      tc_fence_after();
+      if (wq < 2) {
+        const int r = 32 * wq + lane, tc0 = 16 * wg;
+        float v[16];
+        tmem_ld16(X1 + lane_base + tc0, v);
+  #pragma unroll
+        for (int u = 0; u < 16; ++u) v[u] = (tc0 + u < r) ? -v[u] : 0.f;
+        if (SD) {  // dT diag(beta / gamma) -> O_AQ (B10b); diag(gamma) dT below (B9b)
+          float w[16];
+  #pragma unroll
+          for (int u = 0; u < 16; ++u) w[u] = v[u] * s_kf[tc0 + u];
+          sm16(sm + O_AQ, chunk_off(r, tc0 >> 3)) = pack_bf8(w);
+          sm16(sm + O_AQ, chunk_off(r, (tc0 >> 3) + 1)) = pack_bf8(w + 8);
+          const float f = s_gm[r];
+  #pragma unroll
+          for (int u = 0; u < 16; ++u) v[u] *= f;
+        }
+        sm16(sm + O_DT, chunk_off(r, tc0 >> 3)) = pack_bf8(v);
+        sm16(sm + O_DT, chunk_off(r, (tc0 >> 3) + 1)) = pack_bf8(v + 8);
+      }
+      fence_proxy_async();
+      tc_fence_before();
+      __syncthreads();
+      // ---- [17] B9b: X0 += (dT^T Kbar)^T;  B10b: X2 += (dT Kk)^T
+      if (tid == 0) {
+        tc_fence_after();
+        const uint32_t id01 = idesc_bf16(128, 64, 0, 1), id00 = idesc_bf16(128, 64, 0, 0);
+        const uint32_t id11 = idesc_bf16(128, 64, 1, 1), id10 = idesc_bf16(128, 64, 1, 0);
+        for (int kk = 0; kk < 4; ++kk) {
+          if (SD) {
+            const uint64_t kt = mdesc(rkq + kk * 2048, 16384);
+            umma_bf16(X0, kt, mdesc(sm + O_DT + kk * 2048, 8192), id11, 1);
+            umma_bf16(X2, kt, kdesc(sm + O_AQ + kk * 32), id10, 1);
+          } else {
+            umma_bf16(X0, kdesc(sm + O_KQH2 + kk * 32), mdesc(sm + O_DT + kk * 2048, 8192), id01, 1);
+            umma_bf16(X2, kdesc(sm + O_KKH2 + kk * 32), kdesc(sm + O_DT + kk * 32), id00, 1);
+          }
+        }
+        umma_commit(bar_mma);
+      }
     }
     if (!(ok = mma_wait())) break;
     tc_fence_after();
@@ -1212,6 +1367,8 @@ kdn_status_t launch_fused_bwd(const Args &a, cudaStream_t s) {
   f.o = nullptr;
   f.ST = nullptr;
   f.pT = nullptr;
+  // (the diagonal sweep reads Y = V - Kbar S_in from the context, which the WY forward writes)
+  if (a.variant == 0 && !wy_fwd_supported(f, true)) return KDN_ERR_UNSUPPORTED;
   kdn_status_t st = wy_fwd_supported(f, true) ? launch_wy_fwd(f, s, a.fSin, a.fpin)
                                          : launch_fused_fwd(f, s, a.fSin, a.fpin, false);
   if (st != KDN_OK) return st;

@@ -84,9 +84,11 @@ __device__ __forceinline__ void unpack_h8(uint4 u, float *v) {
 //   gamma fp32 [64 t][128 i] (cumulative decay in the chunk)   32 KB
 //   per-token fp32 [5][64]: s_t (diag) or beta_t, then |k_t|^2, a_t, bhat_t,
 //         b_{t-1} (iso)                                          2 KB
+//   Y = V - Kbar S_in  fp16 [64 t][128 j] as two slabs (diag; the
+//         tile R = A Y was formed from)                          16 KB
 constexpr int kCtxS = 0, kCtxR = 32768, kCtxW = 49152, kCtxAqk = 65536, kCtxA = 73728;
-constexpr int kCtxPh = 81920, kCtxGa = 114688, kCtxTok = 147456;
-constexpr int kCtxBytes = 149504;
+constexpr int kCtxPh = 81920, kCtxGa = 114688, kCtxTok = 147456, kCtxY = 149504;
+constexpr int kCtxBytes = 165888;
 
 // Smallest cumulative decay gamma_C = exp(G_C) of a chunk the fused kernels
 // accept: they divide by gamma (Kk = kappa / gamma), which must stay a normal

@@ -450,8 +450,9 @@ struct WyParams {
 };
 
 // SV: besides o, S_T and p_T (each written when its pointer is non-null), keep
-// the chunked backward's context: per chunk the fp16 tiles S_in, R, -W, A_qk
-// and A = (I + T)^-1 in the 128-byte-swizzled layout of the fused backward,
+// the chunked backward's context: per chunk the fp16 tiles S_in, R, -W, A_qk,
+// A = (I + T)^-1 and Y = V - Kbar S_in in the 128-byte-swizzled layout of the
+// fused backward,
 // phat and gamma in float32 [64 t][128 i], s_t per token, and the uncertainty
 // entering the chunk.  The arithmetic is the same with and without it.
 
@@ -1085,6 +1086,7 @@ __global__ void __launch_bounds__(WT, 1)
     if (SV) {
       if (issuer) {
         bulk_s2g(ctx + kCtxA, awu, 8192);
+        bulk_s2g(ctx + kCtxY, vr, 16384);  // Y, before R' is written over it
         bulk_commit();
         tc_fence_after();
         const uint32_t AW = smem_u32(awu), KN = smem_u32(as1);
@@ -1114,6 +1116,9 @@ __global__ void __launch_bounds__(WT, 1)
 
     // ---- [7] MMA-R: TW = [A; 0] Y = [R; 0]  (fp16)
     if (issuer) {
+      // (context: the copy of Y has left shared memory before MMA-R completes, after
+      // which R' is written over Y)
+      if (SV) bulk_wait_read();
       tc_fence_after();
       const uint32_t AW = smem_u32(awu), VR = smem_u32(vr);
       for (int kk = 0; kk < 4; ++kk)

@@ -162,14 +162,15 @@ def test_kernel_launch_query(kdn):
 def test_fused_path_launches_and_workspace(kdn):
     """bf16, dk = dv = 128: the fused forward is one launch; the fused backward
     (both variants) is two (context-saving forward + reverse sweep) and its
-    workspace holds an 80 KB context record (S_in, R, -W, A_qk, A as 16-bit
-    tiles) and 128 floats of uncertainty per chunk."""
+    workspace holds a 162 KB context record per chunk (S_in, R, -W, A_qk, A and
+    Y as 16-bit tiles, phat and gamma in fp32, per-token scalars) and 128 floats
+    of uncertainty per chunk."""
     B, T, H = 2, 130, 3
     d = kdn.make_desc(B, T, H, 128, 128, kdn.KDN_BF16)
     assert kdn.kdn_kernel_launches(d, 0, 0) == 1
     assert kdn.kdn_kernel_launches(d, 0, 1) == 2
     NC = (T + 63) // 64
-    need = 256 + B * H * NC * 149504 + B * H * NC * 128 * 4
+    need = 256 + B * H * NC * 165888 + B * H * NC * 128 * 4
     assert kdn.workspace_bytes(d, 0, True) == need
     # the isotropic backward is fused too; the 32-token chunk keeps the general kernels
     assert kdn.kdn_kernel_launches(d, 1, 1) == 2
@@ -224,7 +225,7 @@ def test_training_pair_validation(kdn):
     B, T, H = 2, 130, 3
     d = kdn.make_desc(B, T, H, 128, 128, kdn.KDN_BF16)
     n = kdn.saved_bytes(d)
-    assert n == B * H * 3 * (149504 + 512)
+    assert n == B * H * 3 * (165888 + 512)
     assert kdn.saved_bytes(d, 1) == n
     assert kdn.saved_bytes(kdn.make_desc(B, T, H, 64, 128, kdn.KDN_BF16)) == 0
     assert kdn.saved_bytes(kdn.make_desc(B, T, H, 128, 128, kdn.KDN_F32)) == 0
