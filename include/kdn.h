@@ -180,9 +180,11 @@ kdn_status_t kdn_iso_bwd(const kdn_desc_t *desc, const void *q, const void *k,
 
 /* Training pair.  kdn_diag_fwd_save is kdn_diag_fwd that also keeps, in
    `saved`, the context the chunked backward needs (App. F): for every 64-token
-   chunk the memory S entering it, its R = U - W S_in, -W, A_qk and
-   A = (I + T)^-1 as fp16 tiles (80 KB) and the float32 uncertainty p entering
-   it.  kdn_diag_bwd_saved is kdn_diag_bwd that starts from that
+   chunk the memory S entering it, its R = U - W S_in, -W, A_qk,
+   A = (I + T)^-1 and (Diagonal KDN) Y = V - Kbar S_in as fp16 tiles (96 KB),
+   the pre-write variance phat and the cumulative decay gamma of every
+   (token, channel) in float32 (64 KB), per-token scalars (2 KB), and the
+   float32 uncertainty p entering it.  kdn_diag_bwd_saved is kdn_diag_bwd that starts from that
    context instead of recomputing the forward (same gradients, one kernel).
    kdn_iso_fwd_save / kdn_iso_bwd_saved are the same for the Isotropic KDN.
    Served for bfloat16 activations, dk = dv = 128 and the default chunk; for
