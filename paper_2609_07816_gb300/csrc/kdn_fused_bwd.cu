@@ -384,6 +384,14 @@ __global__ void __launch_bounds__(BT, 1)
     ++mma_phase;
     return __syncthreads_and(r);
   };
+  // Diagonal KDN: every thread polls the MMA-completion barrier itself (no CTA barrier
+  // between the completion and the TMEM reads); the outcome is combined at the stage's
+  // closing barrier, so that every thread leaves the loop at the same point
+  auto mma_poll = [&]() -> bool {
+    const bool r = mbar_wait(bar_mma, mma_phase & 1, kWaitIters);
+    ++mma_phase;
+    return r;
+  };
   // the thread's tokens t0..t0+15: phat, gamma from TMEM, k from the raw tile
   auto load_ph_ga = [&](float *ph, float *ga) {
     tmem_ld16(TPH + lane_base + t0, ph);
@@ -438,10 +446,33 @@ __global__ void __launch_bounds__(BT, 1)
     if (!ok) break;
     load_r(c - 1);
 
-    // ---- [2] the chunk's gains from the context the forward saved: phat (diag) and
-    //          gamma -> TMEM (lane = channel), per-token s_t (diag) or beta_t, |k_t|^2,
-    //          a_t, bhat_t, b_{t-1} (iso)
+    // ---- [2] dS -> fp16 [i][j] (the B1 / B4 operand) and its dgamma_C part, and A bf16
+    //          (from the saved fp16 A), while the gains' global loads are in flight; then
+    //          the gains: phat (diag) and gamma -> TMEM (lane = channel), per-token s_t
+    //          (diag) or beta_t, |k_t|^2, a_t, bhat_t, b_{t-1} (iso).  (dS <- gamma_C dS
+    //          follows in [11]: B1 and B4 read the fp16 copy, B2 accumulates into TS.)
     float dgc = 0.f;  // this thread's part of dgamma_C for channel ci
+    {
+      const int i = 32 * wq + lane;
+      for (int c0 = 0; c0 < 32; c0 += 16) {
+        float v[16], sv[16];
+        const int j0 = 32 * wg + c0, sl = j0 >> 6, cc0 = (j0 & 63) >> 3;
+        const uint32_t o0 = sl * 16384 + chunk_off(i, cc0), o1 = sl * 16384 + chunk_off(i, cc0 + 1);
+        tmem_ld16(TS + lane_base + j0, v);
+        sm16(sm + O_DSH, o0) = pack_h8(v);
+        sm16(sm + O_DSH, o1) = pack_h8(v + 8);
+        unpack_h8(sm16(sin, o0), sv);
+        unpack_h8(sm16(sin, o1), sv + 8);
+#pragma unroll
+        for (int u = 0; u < 16; ++u) dgc += v[u] * sv[u];
+      }
+    }
+    {
+      const uint4 ah = sm16(sm + O_AH, tid * 16);  // 512 chunks of 8: the whole 8 KB tile
+      float v[8];
+      unpack_h8(ah, v);
+      sm16(sm + O_AB, tid * 16) = pack_bf8(v);
+    }
     {
       if (V == 0) tmem_st16(TPH + lane_base + t0, ph16);
       tmem_st16(TGM + lane_base + t0, e16);
@@ -469,35 +500,8 @@ __global__ void __launch_bounds__(BT, 1)
       __syncthreads();
     }
     // ---- [3] operands of the chunk adjoint from the context and the gains:
-    //          A bf16 (from the saved fp16 A); dS -> fp16 [i][j] and dS <- gamma_C dS in
-    //          TMEM; K_tail^T [i][s]; lambda dO and v to fp16 in place
+    //          K_tail^T [i][s]; lambda dO and v to fp16 in place
     if (SD && tid < CM) s_kf[tid] = s_x[tid] * __frcp_rn(s_gm[tid]);
-    {
-      const uint4 ah = sm16(sm + O_AH, tid * 16);  // 512 chunks of 8: the whole 8 KB tile
-      float v[8];
-      unpack_h8(ah, v);
-      sm16(sm + O_AB, tid * 16) = pack_bf8(v);
-    }
-    {
-      const int i = 32 * wq + lane;
-      const float gC = s_gC[i];
-      for (int c0 = 0; c0 < 32; c0 += 16) {
-        float v[16], sv[16];
-        const int j0 = 32 * wg + c0, sl = j0 >> 6, cc0 = (j0 & 63) >> 3;
-        const uint32_t o0 = sl * 16384 + chunk_off(i, cc0), o1 = sl * 16384 + chunk_off(i, cc0 + 1);
-        tmem_ld16(TS + lane_base + j0, v);
-        sm16(sm + O_DSH, o0) = pack_h8(v);
-        sm16(sm + O_DSH, o1) = pack_h8(v + 8);
-        unpack_h8(sm16(sin, o0), sv);
-        unpack_h8(sm16(sin, o1), sv + 8);
-#pragma unroll
-        for (int u = 0; u < 16; ++u) {
-          dgc += v[u] * sv[u];
-          v[u] *= gC;
-        }
-        tmem_st16(TS + lane_base + j0, v);
-      }
-    }
     {
       float gf[16], ga[16];
       load_gain(gf, ga);
@@ -541,7 +545,12 @@ __global__ void __launch_bounds__(BT, 1)
       }
       umma_commit(bar_mma);
     }
-    if (!(ok = mma_wait())) break;
+    bool mm_ok = true;
+    if constexpr (V == 0) {
+      mm_ok = mma_poll();
+    } else {
+      if (!(ok = mma_wait())) break;
+    }
     tc_fence_after();
     // ---- [11] dR^T -> fp16 [j][t] (and its fp16 remainder); dA_qk^T (masked to s <= t) -> hi/lo bf16 [s][t];
     //           X0 <- gamma_C dK_tail^T (start of dKk^T) and its dgamma_C part; Qbar fp16
@@ -593,10 +602,25 @@ __global__ void __launch_bounds__(BT, 1)
       tmem_st16(X0 + lane_base + t0, x);
       st_row16_h(sm + O_QH, ci, qq, gf);  // Qbar^T [i][t]
     }
+    {  // dS <- gamma_C dS in TMEM, before B2 accumulates into it
+      const int i = 32 * wq + lane;
+      const float gC = s_gC[i];
+      for (int c0 = 0; c0 < 32; c0 += 16) {
+        float v[16];
+        const int j0 = 32 * wg + c0;
+        tmem_ld16(TS + lane_base + j0, v);
+#pragma unroll
+        for (int u = 0; u < 16; ++u) v[u] *= gC;
+        tmem_st16(TS + lane_base + j0, v);
+      }
+    }
     tmem_st_wait();
     fence_proxy_async();
     tc_fence_before();
-    __syncthreads();
+    if (!__syncthreads_and(mm_ok)) {
+      ok = false;
+      break;
+    }
     if constexpr (V == 0) {
       // Diagonal KDN: five tensor-core rounds.  With Y = V - Kbar S_in (the tile the
       // forward formed R = A Y from, in the context), dA = dR V^T + dW Kbar^T =
@@ -621,7 +645,7 @@ __global__ void __launch_bounds__(BT, 1)
         }
         umma_commit(bar_mma);
       }
-      if (!(ok = mma_wait())) break;
+      mm_ok = mma_poll();
       tc_fence_after();
       // ---- [13] dW^T -> bf16 [i][t] (over Y);  dA^T -> fp16 [s][t] (over A_qk);
       //           second operand set: [Kbar; Qbar] hi (interleaved), Qbar lo, Kk hi / lo
@@ -658,7 +682,10 @@ __global__ void __launch_bounds__(BT, 1)
       }
       fence_proxy_async();
       tc_fence_before();
-      __syncthreads();
+      if (!__syncthreads_and(mm_ok)) {
+        ok = false;
+        break;
+      }
       // ---- [14] B8b: X3 += (dA_qk Kk)^T;  B9a: X0 += (dA_qk^T Qbar)^T (hi/lo bf16 pairs);
       //           B7: X2 = dV^T = (A^T dR)^T (dR as hi + lo fp16);  X1 = A^T dA (fp16)
       if (tid == 0) {
@@ -683,7 +710,7 @@ __global__ void __launch_bounds__(BT, 1)
         }
         umma_commit(bar_mma);
       }
-      if (!(ok = mma_wait())) break;
+      mm_ok = mma_poll();
       tc_fence_after();
       if (tid == 0 && c > 0) issue_b_do(c - 1);  // the dO / Qbar lo buffer is free
       if (WT && tid == 0) {  // this chunk's omega logits for pass C, into the dR^T buffer (free
@@ -708,7 +735,10 @@ __global__ void __launch_bounds__(BT, 1)
       }
       fence_proxy_async();
       tc_fence_before();
-      __syncthreads();
+      if (!__syncthreads_and(mm_ok)) {
+        ok = false;
+        break;
+      }
       // ---- [16] X1 = X A^T (fp16), so that dT = strict_lower(-A^T dA A^T);  B10a: X2 = (A^T dW)^T
       if (tid == 0) {
         tc_fence_after();
@@ -719,7 +749,7 @@ __global__ void __launch_bounds__(BT, 1)
         }
         umma_commit(bar_mma);
       }
-      if (!(ok = mma_wait())) break;
+      mm_ok = mma_poll();
       tc_fence_after();
       if (wq < 2) {  // dT -> bf16
         const int r = 32 * wq + lane, tc0 = 16 * wg;
@@ -732,7 +762,10 @@ __global__ void __launch_bounds__(BT, 1)
       }
       fence_proxy_async();
       tc_fence_before();
-      __syncthreads();
+      if (!__syncthreads_and(mm_ok)) {
+        ok = false;
+        break;
+      }
       // ---- [17] B9b: X0 += (dT^T Kbar)^T;  B10b: X2 += (dT Kk)^T
       if (tid == 0) {
         tc_fence_after();
@@ -941,7 +974,11 @@ __global__ void __launch_bounds__(BT, 1)
         umma_commit(bar_mma);
       }
     }
-    if (!(ok = mma_wait())) break;
+    if constexpr (V == 0) {
+      mm_ok = mma_poll();
+    } else {
+      if (!(ok = mma_wait())) break;
+    }
     tc_fence_after();
     if (tid == 0 && c > 0) {
       issue_a_ctx(c - 1);  // the context buffers are free
@@ -969,7 +1006,11 @@ __global__ void __launch_bounds__(BT, 1)
       }
       const float kprev = qq > 0 ? raw_k(t0 - 1) : 0.f;
       fence_proxy_async();
-      __syncthreads();  // raw k, q are in registers: the next chunk's tiles may land
+      // raw k, q are in registers: the next chunk's tiles may land
+      if (!__syncthreads_and(mm_ok)) {
+        ok = false;
+        break;
+      }
       if (tid == 0 && c > 0) issue_a_raw(c - 1);
       // outputs of token t0 + j live at obase + j * ostride; nval tokens of the quarter are real
       const size_t ostride = (size_t)a.H * D;
