@@ -85,6 +85,11 @@ constexpr int O_DWT = O_G, O_DAT = O_G + 16 * KB, O_XT = O_G + 24 * KB, O_KQH2 =
 constexpr int O_QL2 = O_RDO, O_DRTL = O_RH;
 // Diagonal KDN: Y (context) in the v buffer, then dW^T; dA^T over A_qk
 constexpr int O_DWY = O_RV, O_DAY = O_AQ;
+// Diagonal KDN: the next chunk's phat and gamma (fp32 [64 t][128 i]) arrive by bulk copies
+// into buffers idle from the end of a chunk's last pass to stage [3] of the next: phat over
+// the dS tile, gamma's tokens 0..31 over the A bf16 and dT tiles, tokens 32..63 over K_tail
+constexpr int O_PHB = O_G, O_GA0 = O_AB, O_GA1 = O_KT;
+static_assert(O_AB + 8 * KB == O_DT, "gamma's first half spans the A bf16 and dT tiles");
 // small arrays
 constexpr int OFF_SM = BUF_END;
 constexpr int SMALL_FLOATS = 64 * 18 + 256 * 2 + 128 * 2 + 16;
@@ -218,6 +223,7 @@ __global__ void __launch_bounds__(BT, 1)
   uint64_t *bar_w = bars + 3;
   constexpr bool WT = V == 0 && G;
   uint32_t *s_tbase = reinterpret_cast<uint32_t *>(bars + 4);
+  uint64_t *bar_g = bars + 5;  // diagonal KDN: phat and gamma of the chunk
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int wq = warp & 3, wg = warp >> 2;  // TMEM lane quarter, column group
@@ -232,6 +238,7 @@ __global__ void __launch_bounds__(BT, 1)
     mbar_init(bar_b, 1);
     mbar_init(bar_mma, 1);
     if (WT) mbar_init(bar_w, 1);
+    if (V == 0) mbar_init(bar_g, 1);
     fence_mbar_init();
     prefetch_tmap(&mq);
     prefetch_tmap(&mk);
@@ -279,11 +286,19 @@ __global__ void __launch_bounds__(BT, 1)
   auto issue_b_v = [&](int c) {
     for (int s = 0; s < 2; ++s) tma_load_4d(rv + s * 8192, &mv, bar_b, 64 * s, h, c * CM, b);
   };
+  auto issue_g = [&](int c) {
+    const unsigned char *rec = a.fSin + ((size_t)bh * NC + c) * kCtxBytes;
+    mbar_expect_tx(bar_g, 65536);
+    bulk_g2s(sm + O_PHB, rec + kCtxPh, 32768, bar_g);
+    bulk_g2s(sm + O_GA0, rec + kCtxGa, 16384, bar_g);
+    bulk_g2s(sm + O_GA1, rec + kCtxGa + 16384, 16384, bar_g);
+  };
   if (tid == 0) {
     issue_a_ctx(NC - 1);
     issue_a_raw(NC - 1);
     issue_b_do(NC - 1);
     if (V != 0) issue_b_v(NC - 1);
+    if (V == 0) issue_g(NC - 1);
   }
 
   // ---- cotangent scale lambda = 2^-e with max(|dO|, |dS_T|) * lambda in [1, 2)
@@ -416,7 +431,8 @@ __global__ void __launch_bounds__(BT, 1)
   for (int it = 0; it < NC && ok; ++it) {
     const int c = NC - 1 - it;
     // ---- [1] per-token scalars; the chunk's gains from the context the forward saved
-    //          (global loads issued before the wait for the tiles); raw tiles
+    //          (diagonal KDN: bulk copies issued at the end of the previous chunk, on
+    //          bar_g; isotropic: global loads issued before the wait for the tiles); raw tiles
     if (tid < CM) {
       s_r[tid] = nr;
       s_ri[tid] = 1.f / nr;
@@ -427,54 +443,38 @@ __global__ void __launch_bounds__(BT, 1)
     const unsigned char *rec = a.fSin + ((size_t)bh * NC + c) * kCtxBytes;
     float e16[16], ph16[16], tk[5];
     {
-      // gamma [64][128] (SD: one value per token, [64])
+      // gamma [64][128] (SD: one value per token, [64]) of the isotropic KDN
       const float *cga = reinterpret_cast<const float *>(rec + kCtxGa) + (SD ? t0 : t0 * D + ci);
-      const float *cph = reinterpret_cast<const float *>(rec + kCtxPh) + t0 * D + ci;
       const float *tok = reinterpret_cast<const float *>(rec + kCtxTok);
+      if (V != 0) {  // (the diagonal KDN's arrive in shared memory on bar_g)
 #pragma unroll
-      for (int j = 0; j < 16; ++j) e16[j] = cga[SD ? j : j * D];
-      if (V == 0) {
-#pragma unroll
-        for (int j = 0; j < 16; ++j) ph16[j] = cph[j * D];
+        for (int j = 0; j < 16; ++j) e16[j] = cga[SD ? j : j * D];
       }
       if (tid < CM) {
 #pragma unroll
         for (int m = 0; m < (V == 0 ? 1 : 5); ++m) tk[m] = tok[64 * m + tid];
       }
     }
-    ok = __syncthreads_and(mbar_wait(bar_a, it & 1, kWaitIters));
+    ok = __syncthreads_and(mbar_wait(bar_a, it & 1, kWaitIters) &&
+                           (V != 0 || mbar_wait(bar_g, it & 1, kWaitIters)));
     if (!ok) break;
     load_r(c - 1);
 
-    // ---- [2] dS -> fp16 [i][j] (the B1 / B4 operand) and its dgamma_C part, and A bf16
-    //          (from the saved fp16 A), while the gains' global loads are in flight; then
-    //          the gains: phat (diag) and gamma -> TMEM (lane = channel), per-token s_t
-    //          (diag) or beta_t, |k_t|^2, a_t, bhat_t, b_{t-1} (iso).  (dS <- gamma_C dS
-    //          follows in [11]: B1 and B4 read the fp16 copy, B2 accumulates into TS.)
+    // ---- [2] the chunk's gains from the context the forward saved: phat (diag) and
+    //          gamma -> TMEM (lane = channel), per-token s_t (diag) or beta_t, |k_t|^2,
+    //          a_t, bhat_t, b_{t-1} (iso)
     float dgc = 0.f;  // this thread's part of dgamma_C for channel ci
     {
-      const int i = 32 * wq + lane;
-      for (int c0 = 0; c0 < 32; c0 += 16) {
-        float v[16], sv[16];
-        const int j0 = 32 * wg + c0, sl = j0 >> 6, cc0 = (j0 & 63) >> 3;
-        const uint32_t o0 = sl * 16384 + chunk_off(i, cc0), o1 = sl * 16384 + chunk_off(i, cc0 + 1);
-        tmem_ld16(TS + lane_base + j0, v);
-        sm16(sm + O_DSH, o0) = pack_h8(v);
-        sm16(sm + O_DSH, o1) = pack_h8(v + 8);
-        unpack_h8(sm16(sin, o0), sv);
-        unpack_h8(sm16(sin, o1), sv + 8);
+      if constexpr (V == 0) {
+        const float *gs = reinterpret_cast<const float *>(sm + (qq < 2 ? O_GA0 : O_GA1)) + (t0 & 31) * D + ci;
+        const float *ps = reinterpret_cast<const float *>(sm + O_PHB) + t0 * D + ci;
 #pragma unroll
-        for (int u = 0; u < 16; ++u) dgc += v[u] * sv[u];
+        for (int j = 0; j < 16; ++j) {
+          e16[j] = gs[j * D];
+          ph16[j] = ps[j * D];
+        }
+        tmem_st16(TPH + lane_base + t0, ph16);
       }
-    }
-    {
-      const uint4 ah = sm16(sm + O_AH, tid * 16);  // 512 chunks of 8: the whole 8 KB tile
-      float v[8];
-      unpack_h8(ah, v);
-      sm16(sm + O_AB, tid * 16) = pack_bf8(v);
-    }
-    {
-      if (V == 0) tmem_st16(TPH + lane_base + t0, ph16);
       tmem_st16(TGM + lane_base + t0, e16);
       if (qq == 3) {
         s_gC[ci] = e16[15];
@@ -500,7 +500,30 @@ __global__ void __launch_bounds__(BT, 1)
       __syncthreads();
     }
     // ---- [3] operands of the chunk adjoint from the context and the gains:
-    //          K_tail^T [i][s]; lambda dO and v to fp16 in place
+    //          A bf16 (from the saved fp16 A); dS -> fp16 [i][j] (the B1 / B4 operand; dS <-
+    //          gamma_C dS follows in [11], before B2 accumulates into it); K_tail^T [i][s];
+    //          lambda dO and v to fp16 in place
+    {
+      const uint4 ah = sm16(sm + O_AH, tid * 16);  // 512 chunks of 8: the whole 8 KB tile
+      float v[8];
+      unpack_h8(ah, v);
+      sm16(sm + O_AB, tid * 16) = pack_bf8(v);
+    }
+    {
+      const int i = 32 * wq + lane;
+      for (int c0 = 0; c0 < 32; c0 += 16) {
+        float v[16], sv[16];
+        const int j0 = 32 * wg + c0, sl = j0 >> 6, cc0 = (j0 & 63) >> 3;
+        const uint32_t o0 = sl * 16384 + chunk_off(i, cc0), o1 = sl * 16384 + chunk_off(i, cc0 + 1);
+        tmem_ld16(TS + lane_base + j0, v);
+        sm16(sm + O_DSH, o0) = pack_h8(v);
+        sm16(sm + O_DSH, o1) = pack_h8(v + 8);
+        unpack_h8(sm16(sin, o0), sv);
+        unpack_h8(sm16(sin, o1), sv + 8);
+#pragma unroll
+        for (int u = 0; u < 16; ++u) dgc += v[u] * sv[u];
+      }
+    }
     if (SD && tid < CM) s_kf[tid] = s_x[tid] * __frcp_rn(s_gm[tid]);
     {
       float gf[16], ga[16];
@@ -1148,7 +1171,11 @@ __global__ void __launch_bounds__(BT, 1)
         }
         const float rs2 = rs16(drp, lane);
         if ((lane & 1) == 0) s_red2[wq * 64 + t0 + (lane >> 1)] = rs2;
+        fence_proxy_async();
         __syncthreads();
+        // every read of the dG scratch, the pass summaries and the omega logits is done:
+        // the next chunk's phat and gamma may land over them
+        if (tid == 0 && c > 0) issue_g(c - 1);
         if (qq == 0) s_dp[ci] = dp;
         if (tid < CM) {
           const int tt = c * CM + tid;
@@ -1354,6 +1381,10 @@ __global__ void __launch_bounds__(BT, 1)
       if (WT) {
         mbar_wait(bar_w, 0, kWaitIters);
         mbar_wait(bar_w, 1, kWaitIters);
+      }
+      if (V == 0) {
+        mbar_wait(bar_g, 0, kWaitIters);
+        mbar_wait(bar_g, 1, kWaitIters);
       }
     }
   }
