@@ -84,7 +84,7 @@ constexpr int O_DSH = O_G, O_DAQ = O_G, O_QH = O_G + 16 * KB, O_KKL2 = O_G + 16 
 constexpr int O_DWT = O_G, O_DAT = O_G + 16 * KB, O_XT = O_G + 24 * KB, O_KQH2 = O_SIN;
 constexpr int O_QL2 = O_RDO, O_DRTL = O_RH;
 // Diagonal KDN: Y (context) in the v buffer, then dW^T; dA^T over A_qk
-constexpr int O_DWY = O_RV, O_DAY = O_AQ;
+constexpr int O_DWY = O_RV, O_DAY = O_AQ, O_DVS = O_RH;
 // Diagonal KDN: the next chunk's phat and gamma (fp32 [64 t][128 i]) arrive by bulk copies
 // into buffers idle from the end of a chunk's last pass to stage [3] of the next: phat over
 // the dS tile, gamma's tokens 0..31 over the A bf16 and dT tiles, tokens 32..63 over K_tail
@@ -187,7 +187,8 @@ template <int V, int OBF, int G, int SD>
 __global__ void __launch_bounds__(BT, 1)
     k_fused_bwd(const __grid_constant__ CUtensorMap mq, const __grid_constant__ CUtensorMap mk,
                 const __grid_constant__ CUtensorMap mv, const __grid_constant__ CUtensorMap mdo,
-                const __grid_constant__ CUtensorMap mw, const BwdParams P) {
+                const __grid_constant__ CUtensorMap mw, const __grid_constant__ CUtensorMap mdv,
+                const BwdParams P) {
   const Args &a = P.a;
   extern __shared__ unsigned char smraw[];
   unsigned char *sm =
@@ -222,6 +223,8 @@ __global__ void __launch_bounds__(BT, 1)
   // diagonal KDN with logit gates: the chunk's omega logits (tile in O_KT, pass C)
   uint64_t *bar_w = bars + 3;
   constexpr bool WT = V == 0 && G;
+  // diagonal KDN with bf16 gradients: dv leaves by TMA stores of a shared-memory tile
+  constexpr bool DVT = V == 0 && OBF;
   uint32_t *s_tbase = reinterpret_cast<uint32_t *>(bars + 4);
   uint64_t *bar_g = bars + 5;  // diagonal KDN: phat and gamma of the chunk
 
@@ -245,6 +248,7 @@ __global__ void __launch_bounds__(BT, 1)
     prefetch_tmap(&mv);
     prefetch_tmap(&mdo);
     if (WT) prefetch_tmap(&mw);
+    if (DVT) prefetch_tmap(&mdv);
   }
   if (warp == 0) {
     tmem_alloc(s_tbase, 512);
@@ -740,15 +744,25 @@ __global__ void __launch_bounds__(BT, 1)
         mbar_expect_tx(bar_w, 16384);  // until [3] of the next chunk)
         for (int s = 0; s < 2; ++s) tma_load_4d(sm + O_KT + s * 8192, &mw, bar_w, 64 * s, h, c * CM, b);
       }
-      // ---- [15] dV^T -> dv;  X = A^T dA -> fp16 [r][s]
+      // ---- [15] dV^T -> dv (bf16: into the dR^T lo tile, free since B7, in the layout of
+      //           the TMA box, then two TMA stores; rows past T are clipped by the map);
+      //           X = A^T dA -> fp16 [r][s]
       {
         const int j = 32 * wq + lane, tc0 = 16 * wg;
         float v[16];
         tmem_ld16(X2 + lane_base + tc0, v);
+        if constexpr (DVT) {
+          unsigned char *slab = sm + O_DVS + (j >> 6) * 8192;
 #pragma unroll
-        for (int u = 0; u < 16; ++u) {
-          const int t = c * CM + tc0 + u;
-          if (t < a.T) st_grad<OBF>(a.dv_, tok_index(a, b, t, h) * D + j, v[u] * invl);
+          for (int u = 0; u < 16; ++u)
+            *reinterpret_cast<__nv_bfloat16 *>(slab + chunk_off(tc0 + u, (j & 63) >> 3) + 2 * (j & 7)) =
+                __float2bfloat16_rn(v[u] * invl);
+        } else {
+#pragma unroll
+          for (int u = 0; u < 16; ++u) {
+            const int t = c * CM + tc0 + u;
+            if (t < a.T) st_grad<OBF>(a.dv_, tok_index(a, b, t, h) * D + j, v[u] * invl);
+          }
         }
         if (wq < 2) {
           tmem_ld16(X1 + lane_base + tc0, v);
@@ -761,6 +775,11 @@ __global__ void __launch_bounds__(BT, 1)
       if (!__syncthreads_and(mm_ok)) {
         ok = false;
         break;
+      }
+      if (DVT && tid == 0) {
+        tma_store_4d(&mdv, sm + O_DVS, 0, h, c * CM, b);
+        tma_store_4d(&mdv, sm + O_DVS + 8192, 64, h, c * CM, b);
+        bulk_commit();
       }
       // ---- [16] X1 = X A^T (fp16), so that dT = strict_lower(-A^T dA A^T);  B10a: X2 = (A^T dW)^T
       if (tid == 0) {
@@ -1004,6 +1023,7 @@ __global__ void __launch_bounds__(BT, 1)
     }
     tc_fence_after();
     if (tid == 0 && c > 0) {
+      if (DVT) bulk_wait_read();  // the dv tile has left the R buffer
       issue_a_ctx(c - 1);  // the context buffers are free
       // phat, gamma and the token scalars of chunk c - 1 are read with plain loads at the
       // top of its iteration: bring them into L2 now
@@ -1370,8 +1390,10 @@ __global__ void __launch_bounds__(BT, 1)
       for (int w = 0; w < CM; ++w) tot += s_dmu[w];
       a.dmu[bh] = tot * invl;
     }
+    if (DVT && tid == 0) bulk_wait_all();  // the last chunk's dv stores
   } else {
     if (tid == 0) atomicExch(a.status, (unsigned)KDN_ERR_TIMEOUT);
+    if (DVT && tid == 0) bulk_wait_all();
     // let copies already in flight land before the CTA's shared memory goes away
     if (tid == 0) {
       mbar_wait(bar_a, 0, kWaitIters);
@@ -1416,6 +1438,9 @@ kdn_status_t launch_fused_bwd_sweep(const Args &a, cudaStream_t s) {
   if (a.variant == 0 && a.gates && !make_map(&mw, a.omega, a))
     return KDN_ERR_CUDA;
   const bool obf = a.odt == KDN_BF16;
+  CUtensorMap mdv = mq;  // dv (diagonal KDN, bf16 gradients: TMA stores)
+  if (a.variant == 0 && obf && !make_map(&mdv, a.dv_, a))
+    return KDN_ERR_CUDA;
   decltype(&k_fused_bwd<0, 0, 0, 0>) kern;
   if (a.variant == 0)
     kern = a.gates ? (obf ? k_fused_bwd<0, 1, 1, 0> : k_fused_bwd<0, 0, 1, 0>)
@@ -1429,7 +1454,7 @@ kdn_status_t launch_fused_bwd_sweep(const Args &a, cudaStream_t s) {
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES) !=
       cudaSuccess)
     return KDN_ERR_CUDA;
-  kern<<<a.B * a.H, BT, SMEM_BYTES, s>>>(mq, mk, mv, mdo, mw, P);
+  kern<<<a.B * a.H, BT, SMEM_BYTES, s>>>(mq, mk, mv, mdo, mw, mdv, P);
   return cudaGetLastError() == cudaSuccess ? KDN_OK : KDN_ERR_CUDA;
 }
 
