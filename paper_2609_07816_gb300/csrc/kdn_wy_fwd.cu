@@ -452,7 +452,7 @@ struct WyParams {
 // SV: besides o, S_T and p_T (each written when its pointer is non-null), keep
 // the chunked backward's context: per chunk the fp16 tiles S_in, R, -W, A_qk,
 // A = (I + T)^-1 and Y = V - Kbar S_in in the 128-byte-swizzled layout of the
-// fused backward,
+// fused backward (all but A_qk staged in shared memory and bulk-copied),
 // phat and gamma in float32 [64 t][128 i], s_t per token, and the uncertainty
 // entering the chunk.  The arithmetic is the same with and without it.
 
@@ -469,6 +469,7 @@ __global__ void __launch_bounds__(WT, 1)
   unsigned char *ta = sm + O_TA, *tb = sm + O_TB, *as1 = sm + O_AS1;
   unsigned char *s16 = sm + O_S16, *awu = sm + O_AWU;
   float *sT = reinterpret_cast<float *>(sm + O_SWT), *sA = reinterpret_cast<float *>(sm + O_SWA);
+  unsigned char *wst = sm + O_SWA;  // context: -W fp16 staged over L^-1 after the solve
   float *sX = reinterpret_cast<float *>(sm + O_SX), *sY = reinterpret_cast<float *>(sm + O_SY);
   float *sf = reinterpret_cast<float *>(sm + O_SMALL);
   float *s_r = sf + SM_R, *s_mur = sf + SM_MUR, *s_s = sf + SM_S, *s_is = sf + SM_IS;
@@ -1100,25 +1101,30 @@ __global__ void __launch_bounds__(WT, 1)
     if (SV) {  // -W of the context (rows 0..63 of TW), once MMA-W has completed
       mine = mbar_wait(bar_w, c & 1, kWait) && mine;
       tc_fence_after();
-      if (wq < 2) {
+      if (wq < 2) {  // into the fp32 L^-1 tile, dead since the solve, for one bulk copy
         const int t = 32 * wq + lane;
         for (int g = wgm; g < 8; g += 3) {
           float v[16];
           const int j0 = 16 * g, sl = j0 >> 6, cc0 = (j0 & 63) >> 3;
           tmem_ld16(TW + lane_base + j0, v);
-          *reinterpret_cast<uint4 *>(ctx + kCtxW + sl * 8192 + chunk_off(t, cc0)) = pack_h8(v);
-          *reinterpret_cast<uint4 *>(ctx + kCtxW + sl * 8192 + chunk_off(t, cc0 + 1)) = pack_h8(v + 8);
+          sm16(wst, sl * 8192 + chunk_off(t, cc0)) = pack_h8(v);
+          sm16(wst, sl * 8192 + chunk_off(t, cc0 + 1)) = pack_h8(v + 8);
         }
       }
+      fence_proxy_async();
       tc_fence_before();
       bar_sync(kBarMain, kMain);  // TW is free for MMA-R
+      if (issuer) {
+        bulk_s2g(ctx + kCtxW, wst, 16384);
+        bulk_commit();
+      }
     }
 
     // ---- [7] MMA-R: TW = [A; 0] Y = [R; 0]  (fp16)
     if (issuer) {
       // (context: the copy of Y has left shared memory before MMA-R completes, after
-      // which R' is written over Y)
-      if (SV) bulk_wait_read();
+      // which R' is written over Y; the copy of -W, committed after it, may still run)
+      if (SV) bulk_wait_read_but1();
       tc_fence_after();
       const uint32_t AW = smem_u32(awu), VR = smem_u32(vr);
       for (int kk = 0; kk < 4; ++kk)
@@ -1137,9 +1143,9 @@ __global__ void __launch_bounds__(WT, 1)
         float v[16];
         const int j0 = 16 * g, sl = j0 >> 6, cc0 = (j0 & 63) >> 3;
         tmem_ld16(TW + lane_base + j0, v);
-        if (SV) {
-          *reinterpret_cast<uint4 *>(ctx + kCtxR + sl * 8192 + chunk_off(t, cc0)) = pack_h8(v);
-          *reinterpret_cast<uint4 *>(ctx + kCtxR + sl * 8192 + chunk_off(t, cc0 + 1)) = pack_h8(v + 8);
+        if (SV) {  // R for the context, staged over [A; 0] (MMA-R has read it) for one bulk copy
+          sm16(awu, sl * 8192 + chunk_off(t, cc0)) = pack_h8(v);
+          sm16(awu, sl * 8192 + chunk_off(t, cc0 + 1)) = pack_h8(v + 8);
         }
 #pragma unroll
         for (int u = 0; u < 16; ++u) v[u] *= ist;
@@ -1154,6 +1160,10 @@ __global__ void __launch_bounds__(WT, 1)
     // ---- [9] MMA-O (rows 64..127 of TU += A'_qk R', A'_qk in TMEM) and
     //          MMA-S2 (S += K'^T R', K' in TMEM)
     if (issuer) {
+      if (SV) {
+        bulk_s2g(ctx + kCtxR, awu, 16384);
+        bulk_commit();
+      }
       tc_fence_after();
       const uint32_t VR = smem_u32(vr);
       for (int kk = 0; kk < 4; ++kk) {
