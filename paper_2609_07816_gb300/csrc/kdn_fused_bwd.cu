@@ -223,8 +223,8 @@ __global__ void __launch_bounds__(BT, 1)
   // diagonal KDN with logit gates: the chunk's omega logits (tile in O_KT, pass C)
   uint64_t *bar_w = bars + 3;
   constexpr bool WT = V == 0 && G;
-  // diagonal KDN with bf16 gradients: dv leaves by TMA stores of a shared-memory tile
-  constexpr bool DVT = V == 0 && OBF;
+  // bf16 gradients: dv leaves by TMA stores of a shared-memory tile
+  constexpr bool DVT = OBF;
   uint32_t *s_tbase = reinterpret_cast<uint32_t *>(bars + 4);
   uint64_t *bar_g = bars + 5;  // diagonal KDN: phat and gamma of the chunk
 
@@ -906,15 +906,28 @@ __global__ void __launch_bounds__(BT, 1)
         sm16(sm + O_DWT, chunk_off(j, tc0 >> 3)) = pack_bf8(v);
         sm16(sm + O_DWT, chunk_off(j, (tc0 >> 3) + 1)) = pack_bf8(v + 8);
         tmem_ld16(X2 + lane_base + tc0, v);
+        if constexpr (DVT) {  // into the dR^T lo tile (free since B7) for two TMA stores
+          unsigned char *slab = sm + O_DVS + (j >> 6) * 8192;
   #pragma unroll
-        for (int u = 0; u < 16; ++u) {
-          const int t = c * CM + tc0 + u;
-          if (t < a.T) st_grad<OBF>(a.dv_, tok_index(a, b, t, h) * D + j, v[u] * invl);
+          for (int u = 0; u < 16; ++u)
+            *reinterpret_cast<__nv_bfloat16 *>(slab + chunk_off(tc0 + u, (j & 63) >> 3) + 2 * (j & 7)) =
+                __float2bfloat16_rn(v[u] * invl);
+        } else {
+  #pragma unroll
+          for (int u = 0; u < 16; ++u) {
+            const int t = c * CM + tc0 + u;
+            if (t < a.T) st_grad<OBF>(a.dv_, tok_index(a, b, t, h) * D + j, v[u] * invl);
+          }
         }
       }
       fence_proxy_async();
       tc_fence_before();
       __syncthreads();
+      if (DVT && tid == 0) {
+        tma_store_4d(&mdv, sm + O_DVS, 0, h, c * CM, b);
+        tma_store_4d(&mdv, sm + O_DVS + 8192, 64, h, c * CM, b);
+        bulk_commit();
+      }
       // ---- [15] B6: X1 = dA^T = (dR V^T + dW Kbar^T)^T;  B10a: X2 = (A^T dW)^T
       if (tid == 0) {
         tc_fence_after();
@@ -1438,8 +1451,8 @@ kdn_status_t launch_fused_bwd_sweep(const Args &a, cudaStream_t s) {
   if (a.variant == 0 && a.gates && !make_map(&mw, a.omega, a))
     return KDN_ERR_CUDA;
   const bool obf = a.odt == KDN_BF16;
-  CUtensorMap mdv = mq;  // dv (diagonal KDN, bf16 gradients: TMA stores)
-  if (a.variant == 0 && obf && !make_map(&mdv, a.dv_, a))
+  CUtensorMap mdv = mq;  // dv (bf16 gradients: TMA stores)
+  if (obf && !make_map(&mdv, a.dv_, a))
     return KDN_ERR_CUDA;
   decltype(&k_fused_bwd<0, 0, 0, 0>) kern;
   if (a.variant == 0)
