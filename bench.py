@@ -84,7 +84,7 @@ def decode_bytes(b, h, dk, dv, in_bytes=2, out_bytes=4):
 # B=2 (the capture-size rule), scaled by the 4x (batch, head) sequences, which
 # every byte of these one-CTA-per-sequence kernels scales with; reported as
 # `traffic` only for that workload.  None: not captured for the current kernel.
-NCU_TRAFFIC = {"k_wy_fwd<1>": 4 * (168511232 + 317167360), "k_fused_bwd": 4 * (469570304 + 145853952),
+NCU_TRAFFIC = {"k_wy_fwd<1>": 4 * (168267008 + 316675584), "k_fused_bwd": 4 * (469453824 + 145414400),
                "k_wy_fwd<0>": None}
 
 
