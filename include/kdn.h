@@ -92,7 +92,8 @@ typedef struct {
   int dk, dv;            /* key and value head dimensions */
   int chunk;             /* memory-chunk length C_m of App. F.2: 0 (= 64), 32 or 64;
                             a tuning choice, results agree to rounding */
-  int dtype;             /* kdn_dtype_t of activations and their gradients */
+  int dtype;             /* kdn_dtype_t of q, k, v, g, omega, r and dO (the
+                            stored dtype of o and the gradients is out_dtype) */
   float mu;              /* information scale of eq. diag-cov-update; <= 0 -> dk */
   float scale;           /* query scale tau of App. F.2; NaN -> 1/sqrt(dk) */
   int decay_per_channel; /* isotropic only: 1 -> g is [B,T,H,dk], 0 -> [B,T,H].

@@ -6,21 +6,22 @@ on a device synchronisation, or a framework that forbids allocations outside
 its own allocator).  Its scratch is a fixed array inside the library, so this
 test checks, through the C ABI, that consecutive calls (each reusing the array
 the previous one left behind) give the same results as the regular workspace
-entry point, within the float32 parity tolerance, that the status word kept
-in the array is readable through kdn_noalloc_device_status, and that a
-problem too large for the array is refused.
+entry point, within the float32 parity tolerance, and match the fp64 oracle
+within the tolerance of their input dtype; that the status word kept in the
+array is readable through kdn_noalloc_device_status; and that a problem too
+large for the array is refused.
 
 This file is collected last on purpose: if it fails, a run that stops at the
 first failure has already run every other test.
 """
 import ctypes
 
-import numpy as np
 import pytest
 import torch
 
+import oracle
 from kdn_inputs import make_inputs
-from kdn_gpu_util import err_ratio, to_dev
+from kdn_gpu_util import check, err_ratio, to_dev
 
 pytestmark = pytest.mark.gpu
 
@@ -61,6 +62,9 @@ def _check_against_workspace_call(kdn, shape, dtype):
     torch.cuda.synchronize()
     for got, ref in ((o, o_ref), (ST, ST_ref), (pT, pT_ref)):
         assert err_ratio(got, ref.double().cpu().numpy()) <= 1e-4
+    exact = oracle.fwd("diag", *[ins[n] for n in NAMES], ins["S0"], ins["p0"])
+    for name, got in (("o", o), ("ST", ST), ("pT", pT)):
+        check(name, got, exact[name], dtype)
 
 
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
