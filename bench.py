@@ -73,9 +73,13 @@ def bwd_bytes(b, t, h, dk, dv, in_bytes=2, out_bytes=2):
     return b * t * h * (reads + writes) + b * h * per_seq
 
 
-def decode_bytes(b, h, dk, dv, in_bytes=2, out_bytes=4):
-    state = 2 * (dk * dv * 4 + dk * 4)
-    ins = (2 * dk + dv + 2 * dk + 1) * in_bytes
+def decode_bytes(b, h, dk, dv, in_bytes=2, out_bytes=2, variant="diag"):
+    # per head-step: S and p read and written (float32); q, k, v, g, omega, r read;
+    # o written, counted at the activations' dtype whatever dtype stores it.  The
+    # isotropic decode of the bench has one decay, one noise and one uncertainty per head.
+    per_ch = dk if variant == "diag" else 1
+    state = 2 * (dk * dv * 4 + per_ch * 4)
+    ins = (2 * dk + dv + 2 * per_ch + 1) * in_bytes
     return b * h * (state + ins + dv * out_bytes)
 
 
@@ -607,7 +611,7 @@ def run_decode(kdn, torch, hbm, steps=DEC_STEPS):
         torch.cuda.synchronize()
         ms = e0.elapsed_time(e1)
         per = ms / DEC_STEPS
-        by = decode_bytes(DEC_B, DEC_H, DK, DV)
+        by = decode_bytes(DEC_B, DEC_H, DK, DV, variant=variant)
         res[variant] = {"steps_per_s": DEC_STEPS / (ms / 1e3), "us_per_step": per * 1e3,
                         "achieved_GBs": by / (per / 1e3) / 1e9, "frac_hbm": by / (per / 1e3) / 1e9 / hbm,
                         "gpu_launches": DEC_STEPS}

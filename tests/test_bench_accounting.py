@@ -57,10 +57,14 @@ def test_decode_bytes_per_head_step(bench):
     d = 128
     state = 2 * (d * d * 4 + d * 4)               # S and p read and written, fp32
     ins = (4 * d + d + 1) * 2                     # q, k, g, omega, v, r in bf16
-    out = d * 4                                   # o in fp32
-    assert state + ins + out == 133890
-    assert bench.decode_bytes(1, 1, d, d) == 133890
-    assert bench.decode_bytes(256, 16, d, d) == 256 * 16 * 133890
+    out = d * 2                                   # o at the activations' dtype
+    assert state + ins + out == 133634            # ~133.6 KB
+    assert bench.decode_bytes(1, 1, d, d) == 133634
+    assert bench.decode_bytes(256, 16, d, d) == 256 * 16 * 133634
+    # isotropic, one decay per head: g, omega and b are one value per head
+    iso = 2 * (d * d * 4 + 4) + (3 * d + 3) * 2 + d * 2
+    assert iso == 132110                          # ~132.1 KB
+    assert bench.decode_bytes(1, 1, d, d, variant="iso") == 132110
 
 
 def test_chunked_flops(bench):
