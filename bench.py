@@ -201,6 +201,15 @@ def reduce_max(x, world, device="cuda"):
     return float(t.item())
 
 
+def step_config(world):
+    """The workload both arms report: the Diagonal KDN training step on the
+    1.3B-layer shape."""
+    return {"workload": "Diagonal KDN fwd+bwd, 1.3B-layer shape", "B": B, "T": T, "H": H,
+            "dk": DK, "dv": DV, "activations": "bf16", "outputs": "bf16", "state": "f32",
+            "parallelism": f"replicas x{world}",
+            "l2": "inputs larger than L2 (each activation tensor 134 MB)"}
+
+
 def job_throughput(tokens_per_rank, world, ms_per_step):
     """Whole-job tokens/s: every rank's tokens over the max-over-ranks step time."""
     return tokens_per_rank * world / (ms_per_step / 1e3)
@@ -324,10 +333,7 @@ def run_gpu(args):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
         "data": "synthetic",
-        "config": {"workload": "Diagonal KDN fwd+bwd, 1.3B-layer shape", "B": B, "T": T, "H": H,
-                   "dk": DK, "dv": DV, "activations": "bf16", "outputs": "bf16",
-                   "state": "f32", "parallelism": f"replicas x{world}",
-                   "l2": "inputs larger than L2 (each activation tensor 134 MB)"},
+        "config": step_config(world),
         "fwd_ms": fwd_ms, "bwd_ms": bwd_ms,
         "roofline": roof, "roofline_other_kernel": other,
         "spec_roofline_frac": spec_time / (ms_step / 1e3) if ms_step > 0 else None,
@@ -731,9 +737,7 @@ def run_reference(args):
            "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
            "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-           "config": {"workload": "Diagonal KDN fwd+bwd, 1.3B-layer shape", "B": B, "T": T,
-                      "H": H, "dk": DK, "dv": DV, "activations": "bf16",
-                      "sample": samples[0]["sample"]},
+           "config": dict(step_config(world), sample=samples[0]["sample"]),
            "cpu_baseline": {"value": val, "unit": "tokens/s", "cores": samples[0]["cores"],
                             "kind": "oracle", "sample": samples[0]["sample"]},
            "e2e": {"value": val, "unit": "tokens/s", "h2d_bytes_per_step": 0,

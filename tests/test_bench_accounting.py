@@ -91,3 +91,10 @@ def test_outputs_counted_at_the_input_dtype(bench):
 def test_job_throughput_sums_ranks(bench):
     # tokens of every rank over the slowest rank's time
     assert bench.job_throughput(1000, 4, 2.0) == pytest.approx(4 * 1000 / 2e-3)
+
+
+def test_both_arms_report_one_workload(bench):
+    cfg = bench.step_config(1)
+    assert (cfg["B"], cfg["T"], cfg["H"], cfg["dk"], cfg["dv"]) == (8, 4096, 16, 128, 128)
+    assert cfg["activations"] == "bf16" and cfg["outputs"] == "bf16" and cfg["state"] == "f32"
+    assert bench.step_config(4)["parallelism"] == "replicas x4"
