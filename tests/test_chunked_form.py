@@ -18,6 +18,10 @@ parity tests only measure rounding:
     strict_lower(T'); R = A (V - Kbar S_in); outputs and state from
     R' = diag(1/s) R and the unnormalised A'_qk and K'.
 
+The last test does the same for the backward: the chunk adjoint of the fused
+backward (its stages B1-B10 and the scalings by Gamma), then the gain adjoint
+token by token, against the oracle's gradients.
+
 Nothing here runs on, or is shared with, the CUDA path.
 """
 import numpy as np
@@ -256,3 +260,161 @@ def test_solve_form_is_the_paper_inverse():
     A_kernel = np.diag(s) @ np.linalg.inv(np.diag(s) + np.tril(Tp, -1))
     A_paper = np.linalg.inv(np.eye(C) + np.tril(Tp, -1) @ np.diag(1.0 / s))
     assert np.max(np.abs(A_kernel - A_paper)) <= 1e-10 * np.max(np.abs(A_paper))
+
+
+# ---------------------------------------------------------------------------
+# the chunk adjoint the fused backward forms (the paper gives no backward)
+
+def gain_forward(variant, k, g, omega, r, p0, mu):
+    """Per-token quantities of the gain recursion (Prop. 3 / Prop. 5), token by
+    token: the pre-write variance phat, the uncertainty before and after each
+    token, kappa and the scalars the adjoint needs."""
+    T, dk = k.shape
+    alpha = np.exp(g)
+    n2 = np.sum(k * k, axis=1)
+    if variant == "diag":
+        a, u, w = alpha * alpha, mu * k * k / r[:, None], omega
+    else:
+        a2 = alpha * alpha
+        a = (np.mean(a2, axis=1) if g.ndim == 2 else a2)[:, None]
+        u, w = (mu * n2 / (dk * r))[:, None], omega[:, None]
+    p = np.broadcast_to(p0, (a.shape[1],)).astype(np.float64)
+    prev, phat, post = np.empty_like(a), np.empty_like(a), np.empty_like(a)
+    for t in range(T):
+        prev[t] = p
+        phat[t] = a[t] * p + w[t]
+        p = phat[t] / (1.0 + u[t] * phat[t])
+        post[t] = p
+    if variant == "diag":
+        s = r + np.sum(phat * k * k, axis=1)
+        kappa = phat * k / s[:, None]
+    else:
+        s = r + phat[:, 0] * n2                       # beta = bhat / s
+        kappa = (phat[:, 0] / s)[:, None] * k
+    return dict(alpha=alpha, a=a, u=u, prev=prev, phat=phat, post=post, s=s, n2=n2,
+                kappa=kappa)
+
+
+def chunk_backward(variant, x, dO, dST, dpT, mu, tau, Cm):
+    """Gradients of <dO, o> + <dS_T, S_T> + <dp_T, p_T> for one sequence: the
+    memory adjoint chunk by chunk in reverse (the stages of the fused backward,
+    B1-B10), then the gain adjoint token by token in reverse."""
+    q, k, v, g, r = x["q"], x["k"], x["v"], x["g"], x["r"]
+    T, dk = k.shape
+    G = g if g.ndim == 2 else np.repeat(g[:, None], dk, axis=1)
+    gn = gain_forward(variant, k, g, x["omega"], r, x["p0"], mu)
+    kappa = gn["kappa"]
+    starts = list(range(0, T, Cm))
+    S_in, S = [], x["S0"].copy()
+    for c0 in starts:                                   # forward: the memory entering each chunk
+        S_in.append(S)
+        _, S = memory_chunked(q[c0:c0 + Cm], k[c0:c0 + Cm], v[c0:c0 + Cm], G[c0:c0 + Cm],
+                              kappa[c0:c0 + Cm], S, tau, Cm)
+    dq, dk_, dv = np.zeros_like(q), np.zeros_like(k), np.zeros_like(v)
+    dG, dkap = np.zeros_like(G), np.zeros_like(kappa)
+    dS = dST.copy()
+    for c0, Sin in zip(reversed(starts), reversed(S_in)):
+        sl = slice(c0, min(c0 + Cm, T))
+        C = sl.stop - sl.start
+        gam = np.exp(np.cumsum(G[sl], axis=0))
+        K, Kk, Q, V, dOc = k[sl], kappa[sl], q[sl], v[sl], dO[sl]
+        Kbar, Kkbar, Qbar = gam * K, Kk / gam, tau * gam * Q
+        A = np.linalg.inv(np.eye(C) + np.tril(Kbar @ Kkbar.T, -1))
+        W = A @ Kbar
+        R = A @ V - W @ Sin
+        Ktail, Aqk = gam[-1] * Kkbar, np.tril(Qbar @ Kkbar.T)
+        dR = Aqk.T @ dOc + Ktail @ dS                                   # B1
+        dSin = gam[-1][:, None] * dS + Qbar.T @ dOc - W.T @ dR          # B2
+        dAqk = np.tril(dOc @ R.T)                                       # B3
+        dKtail = R @ dS.T                                               # B4
+        dW = -dR @ Sin.T                                                # B5
+        dv[sl] = A.T @ dR                                               # B7 (U = A V)
+        dQbar = dOc @ Sin.T + dAqk @ Kkbar                              # B8
+        dA = dR @ V.T + dW @ Kbar.T                                     # B6
+        dT = np.tril(-A.T @ dA @ A.T, -1)                               # A = (I + T)^-1
+        dKkbar = dAqk.T @ Qbar + gam[-1] * dKtail + dT.T @ Kbar         # B9
+        dKbar = A.T @ dW + dT @ Kkbar                                   # B10
+        dgamC = np.sum(dKtail * Kkbar, axis=0) + np.sum(dS * Sin, axis=1)
+        # the scalings by Gamma, then gamma = exp(cumsum g) within the chunk
+        dk_[sl] += gam * dKbar
+        dkap[sl] += dKkbar / gam
+        dq[sl] += tau * gam * dQbar
+        dgam = K * dKbar - Kkbar * dKkbar / gam + tau * Q * dQbar
+        dgam[-1] += dgamC
+        dG[sl] += np.cumsum((gam * dgam)[::-1], axis=0)[::-1]
+        dS = dSin
+    # gain adjoint, tokens in reverse (eqs. kla-box-gain, diag-cov-update / Prop. 5)
+    a, u, prev, phat, post, s = gn["a"], gn["u"], gn["prev"], gn["phat"], gn["post"], gn["s"]
+    alpha, n2 = gn["alpha"], gn["n2"]
+    domega = np.zeros_like(x["omega"])
+    dr = np.zeros_like(r)
+    dgate = np.zeros_like(G)            # d/dalpha terms of the uncertainty, as d/dg
+    dp = np.broadcast_to(dpT, (a.shape[1],)).astype(np.float64)
+    for t in range(T - 1, -1, -1):
+        dphat = dp / (1.0 + u[t] * phat[t]) ** 2       # p = phat / (1 + u phat)
+        du = -dp * post[t] ** 2
+        if variant == "diag":
+            dk_[t] += du * 2.0 * mu * k[t] / r[t]
+            dr[t] -= np.sum(du * u[t]) / r[t]
+            c = np.sum(dkap[t] * kappa[t])
+            ds = -c / s[t]
+            dphat += dkap[t] * k[t] / s[t] + ds * k[t] ** 2
+            dk_[t] += dkap[t] * phat[t] / s[t] + 2.0 * ds * phat[t] * k[t]
+            dr[t] += ds
+            domega[t] = dphat
+            dgate[t] += 2.0 * alpha[t] ** 2 * prev[t] * dphat
+        else:
+            dn2 = du[0] * mu / (dk * r[t])
+            dr[t] -= du[0] * u[t, 0] / r[t]
+            beta = phat[t, 0] / s[t]
+            dbeta = np.dot(dkap[t], k[t])
+            dk_[t] += beta * dkap[t]
+            dphat = dphat + dbeta * r[t] / s[t] ** 2
+            dr[t] -= dbeta * beta / s[t]
+            dn2 -= dbeta * beta ** 2
+            dk_[t] += 2.0 * k[t] * dn2
+            domega[t] = dphat[0]
+            da = prev[t, 0] * dphat[0]                  # a = mean alpha^2 (or alpha^2)
+            if g.ndim == 2:
+                dgate[t] += da * 2.0 * alpha[t] ** 2 / dk
+            else:
+                dgate[t] += da * 2.0 * alpha[t] ** 2
+        dp = a[t] * dphat
+    if g.ndim == 2:
+        dg = dG + dgate
+    else:  # one decay per head: every channel's log-decay is g_t
+        dg = np.sum(dG, axis=1) + dgate[:, 0]
+    return dict(dq=dq, dk=dk_, dv=dv, dg=dg, domega=domega, dr=dr, dS0=dS, dp0=dp)
+
+
+BWD_CASES = [
+    # variant, per-channel decay, T, dk, dv, C_m
+    ("diag", True, 150, 16, 24, 64),
+    ("diag", True, 97, 32, 16, 32),
+    ("iso", True, 130, 16, 16, 64),
+    ("iso", False, 100, 32, 16, 32),
+]
+
+
+@pytest.mark.parametrize("case", BWD_CASES, ids=lambda c: "-".join(map(str, c)))
+def test_chunk_adjoint_equals_token_loop_adjoint(case):
+    """The chunk adjoint of the fused backward (B1-B10 and the scalings by
+    Gamma), followed by the gain adjoint, gives the oracle's gradients (which
+    are pinned to finite differences) with nonzero dS_T and dp_T."""
+    variant, pc, T, dk, dv, Cm = case
+    ins = make_inputs(variant, 1, T, 2, dk, dv, dtype="f32", seed=21, per_channel_decay=pc,
+                      s0_std=0.3, p0_range=(0.5, 2.0), with_grad=True)
+    rng = np.random.default_rng(4)
+    P = dk if variant == "diag" else 1
+    dST = rng.standard_normal((1, 2, dk, dv))
+    dpT = rng.standard_normal((1, 2, P) if variant == "diag" else (1, 2))
+    mu, tau = 0.7 * dk, dk ** -0.5
+    ref = oracle.bwd(variant, *[ins[n] for n in ("q", "k", "v", "g", "omega", "r")],
+                     ins["S0"], ins["p0"], ins["dO"], dST, dpT, mu=mu, scale=tau)
+    for h in range(2):
+        x = _seq(ins, 0, h)
+        got = chunk_backward(variant, x, ins["dO"][0, :, h], dST[0, h],
+                             np.atleast_1d(dpT[0, h]), mu, tau, Cm)
+        for n in ("dq", "dk", "dv", "dg", "domega", "dr", "dS0", "dp0"):
+            want = ref[n][0, :, h] if ref[n].ndim >= 3 and n not in ("dS0", "dp0") else ref[n][0, h]
+            assert _rel(got[n].reshape(np.shape(want)), np.asarray(want)) <= TOL, n
