@@ -1,0 +1,143 @@
+"""A rounding model of the Diagonal forward kernel's arithmetic, on the CPU.
+
+The kernel computes the chunked form in mixed precision.  This model follows
+its order of operations (mid-chunk referenced decay ratios, the solve as
+diag(s) L^-1, R = A (V - Kbar S_in), R' = diag(1/s) R) and rounds every
+tensor-core operand to the type the kernel stores it in:
+
+  * MMA-T: Kbar', Qbar', Kk' in tf32, rounded to nearest with ties away
+    (cvt.rna), float32 accumulation;
+  * the state products MMA-KS, MMA-R, MMA-O, MMA-S2: -Kbar, Qbar, S_in, Y, A,
+    R', A'_qk and K' in fp16, float32 accumulation;
+  * the gain, the decay sums, the solve and the memory in float32.
+
+Against the fp64 oracle at the workload's input distribution, the modelled
+error shows the margin of these choices under the bf16-input rule
+(max |err| <= 2e-2 RMS), and what single bf16 operands of MMA-T would give
+instead.  Nothing here runs on, or is shared with, the CUDA path.
+"""
+import numpy as np
+import pytest
+
+import oracle
+from kdn_inputs import make_inputs, round_to
+
+F32 = np.float32
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    oracle.build()
+
+
+def tf32_rna(x):
+    """Round float32 values to tf32 (10 explicit mantissa bits), ties away from zero."""
+    u = np.asarray(x, dtype=F32).view(np.uint32)
+    u = (u + np.uint32(0x1000)) & np.uint32(0xFFFFE000)
+    return u.view(F32)
+
+
+def f16(x):
+    return np.asarray(x, dtype=F32).astype(np.float16).astype(F32)
+
+
+def bf16(x):
+    return round_to(np.asarray(x, dtype=F32), "bf16").astype(F32)
+
+
+def mm(a, b):
+    """Product of rounded operands with a float32 accumulator."""
+    return np.matmul(a.astype(F32), b.astype(F32), dtype=F32)
+
+
+def kernel_model(q, k, v, g, omega, r, S0, p0, tau, C=64, mmat=tf32_rna):
+    """o, S_T, p_T of one sequence in the kernel's arithmetic; ``mmat`` rounds
+    the operands of MMA-T."""
+    q, k, v, g, omega, r = (np.asarray(x, dtype=F32) for x in (q, k, v, g, omega, r))
+    T, dk = k.shape
+    tau = F32(tau)
+    S = np.asarray(S0, dtype=F32).copy()
+    p = np.asarray(p0, dtype=F32).copy()
+    o = np.empty((T, v.shape[1]), dtype=F32)
+    for c0 in range(0, T, C):
+        sl = slice(c0, min(c0 + C, T))
+        K, Q, V, Gt = k[sl], q[sl], v[sl], g[sl]
+        # gain, float32, token by token (Prop. 3): phat from the pre-write state
+        alpha2 = np.exp(F32(2) * Gt)
+        phat = np.empty_like(K)
+        for t in range(K.shape[0]):
+            phat[t] = alpha2[t] * p + omega[sl][t]
+            u = F32(dk) * K[t] * K[t] / r[sl][t]   # mu = d_k
+            p = phat[t] / (F32(1) + u * phat[t])
+        Gc = np.cumsum(Gt, axis=0, dtype=F32)
+        GC = Gc[-1]
+        c = GC * F32(0.5)
+        Kb1 = mmat(K * np.exp(Gc - c))
+        Qb1 = mmat(tau * Q * np.exp(Gc - c))
+        Kk1 = mmat(phat * K * np.exp(c - Gc))
+        Tp, Ap = mm(Kb1, Kk1.T), mm(Qb1, Kk1.T)
+        s = r[sl] + np.diag(Tp)
+        L = np.diag(s) + np.tril(Tp, -1)
+        A = (np.diag(s) @ np.linalg.inv(L)).astype(F32)
+        gam = np.exp(Gc)
+        S16 = f16(S)
+        KS, QS = mm(f16(gam * K), S16), mm(f16(tau * gam * Q), S16)
+        Y = f16(V - KS)
+        R = mm(f16(A), Y)
+        Rp = f16(R / s[:, None])
+        o[sl] = QS + mm(f16(np.tril(Ap)), Rp)
+        S = np.exp(GC)[:, None] * S + mm(f16(phat * K * np.exp(GC - Gc)).T, Rp)
+    return o, S, p
+
+
+def _errors(mmat, T=512, H=3, seed=5):
+    d = 128
+    ins = make_inputs("diag", 1, T, H, d, d, dtype="bf16", seed=seed, s0_std=0.02,
+                      p0_range=(0.5, 2.0))
+    tau = d ** -0.5
+    ref = oracle.fwd("diag", *[ins[n] for n in ("q", "k", "v", "g", "omega", "r")],
+                     ins["S0"], ins["p0"], scale=tau)
+    worst = {"o": 0.0, "ST": 0.0, "pT": 0.0, "o_bf16": 0.0}
+    for h in range(H):
+        x = {n: ins[n][0, :, h] for n in ("q", "k", "v", "g", "omega", "r")}
+        o, ST, pT = kernel_model(x["q"], x["k"], x["v"], x["g"], x["omega"], x["r"],
+                                 ins["S0"][0, h], ins["p0"][0, h], tau, mmat=mmat)
+        for name, got, want in (("o", o, ref["o"][0, :, h]), ("ST", ST, ref["ST"][0, h]),
+                                ("pT", pT, ref["pT"][0, h])):
+            e = float(np.max(np.abs(got - want)) / np.sqrt(np.mean(want * want)))
+            worst[name] = max(worst[name], e)
+        # o stored in bf16: the rule plus that one rounding, |err| - 2^-8 |ref|
+        want = ref["o"][0, :, h]
+        excess = np.abs(bf16(o) - want) - 2.0 ** -8 * np.abs(want)
+        e = float(np.max(excess) / np.sqrt(np.mean(want * want)))
+        worst["o_bf16"] = max(worst["o_bf16"], e)
+    return worst
+
+
+def test_rounding_helpers():
+    x = np.array([1.0 + 2.0 ** -11, 1.0 + 3 * 2.0 ** -11, -1.0 - 2.0 ** -11], dtype=F32)
+    # halfway cases of the 10-bit mantissa round away from zero
+    assert np.array_equal(tf32_rna(x), np.array([1.0 + 2.0 ** -10, 1.0 + 2.0 ** -9,
+                                                 -1.0 - 2.0 ** -10], dtype=F32))
+    assert f16(np.array([65504.0], dtype=F32))[0] == 65504.0
+    assert bf16(np.array([1.0 + 2.0 ** -8], dtype=F32))[0] == 1.0   # tie to even
+
+
+def test_kernel_precision_meets_the_bf16_rule_with_margin():
+    """The kernel's precision choices, modelled: o and S_T within a quarter of the
+    2e-2 RMS rule (the GPU measures 2.6e-3 - 3.9e-3 at these distributions), p_T
+    at float32 level; o rounded to bf16 for storage stays within the rule plus
+    that one rounding."""
+    err = _errors(tf32_rna)
+    assert err["o"] <= 5e-3 and err["ST"] <= 5e-3, err
+    assert err["pT"] <= 1e-5, err
+    assert err["o_bf16"] <= 2e-2, err
+
+
+def test_single_bf16_mmat_operands_lose_the_margin():
+    """With MMA-T's referenced operands in single bf16 (8 mantissa bits) instead of
+    tf32, the modelled error of o is over four times larger and reaches the 2e-2
+    rule (2.2e-2 on this case): the reason the kernel runs MMA-T as kind::tf32."""
+    tf = _errors(tf32_rna)
+    b = _errors(bf16)
+    assert b["o"] > 4.0 * tf["o"] and b["o"] > 1.5e-2 and b["ST"] > tf["ST"], (tf, b)
