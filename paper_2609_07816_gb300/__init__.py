@@ -121,6 +121,74 @@ def _code(dtype):
     return _DTYPES[dtype] if isinstance(dtype, torch.dtype) else int(dtype)
 
 
+_TORCH = {KDN_F32: torch.float32, KDN_BF16: torch.bfloat16}
+
+
+def _torch_dtype(dtype):
+    return dtype if isinstance(dtype, torch.dtype) else _TORCH[int(dtype)]
+
+
+def _arg(t, name, dtype=None, numel=None, required=True):
+    """A tensor handed to the C ABI as a raw pointer: it must be device memory (a
+    CUDA tensor), dense in the ABI's row-major layout (contiguous), of the dtype
+    the library reads or writes there and of the element count the descriptor
+    implies.  Anything else would make the kernels read or write the wrong
+    memory, so it is refused here, before any launch."""
+    if t is None:
+        if required:
+            raise ValueError(f"{name} is required")
+        return
+    if not isinstance(t, torch.Tensor):
+        raise TypeError(f"{name}: expected a torch.Tensor, got {type(t).__name__}")
+    if not t.is_cuda:
+        raise ValueError(f"{name}: must be a CUDA tensor (the kernels read device memory), "
+                         f"got one on {t.device}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name}: must be contiguous (the C ABI's row-major layout)")
+    if dtype is not None and t.dtype != dtype:
+        raise TypeError(f"{name}: dtype {t.dtype}, expected {dtype}")
+    if numel is not None and t.numel() != numel:
+        raise ValueError(f"{name}: {t.numel()} elements, expected {numel}")
+
+
+def _check_inputs(variant, q, k, v, g, omega, r, dO=None, tokens=True):
+    """The per-token inputs (and dO): one activation dtype, the ABI's layouts.
+    ``tokens`` = False for the decode step, whose inputs drop the T axis."""
+    _arg(q, "q")
+    if q.dtype not in _DTYPES:
+        raise TypeError(f"q: dtype {q.dtype}, expected torch.float32 or torch.bfloat16")
+    if q.dim() != (4 if tokens else 3):
+        raise ValueError(f"q: {q.dim()} dimensions, expected {4 if tokens else 3}")
+    dk = q.shape[-1]
+    n = q.numel() // dk if dk else 0
+    _arg(v, "v", q.dtype)
+    _arg(g, "g", q.dtype)
+    dv = v.shape[-1]
+    per_channel = variant == 0 or g.dim() == q.dim()
+    for t, name, m in ((k, "k", dk), (v, "v", dv), (g, "g", dk if per_channel else 1),
+                       (omega, "omega", dk if variant == 0 else 1), (r, "r", 1)):
+        _arg(t, name, q.dtype, n * m)
+    if dO is not None:
+        _arg(dO, "dO", q.dtype, n * dv)
+
+
+def _state_sizes(variant, q, v, tokens=True):
+    B, H = q.shape[0], q.shape[2 if tokens else 1]
+    dk, dv = q.shape[-1], v.shape[-1]
+    return B * H * dk * dv, B * H * (dk if variant == 0 else 1)
+
+
+def _check_grads(G, q, k, v, g, omega, r, out_dtype, ns, np_):
+    """Gradient buffers: one per input, its element count, the output dtype;
+    dS0, dp0 and dmu (optional) in float32."""
+    od = _torch_dtype(out_dtype)
+    for n, x in (("dq", q), ("dk", k), ("dv", v), ("dg", g), ("domega", omega), ("dr", r)):
+        _arg(G.get(n), n, od, x.numel())
+    _arg(G.get("dS0"), "dS0", torch.float32, ns, required=False)
+    _arg(G.get("dp0"), "dp0", torch.float32, np_, required=False)
+    _arg(G.get("dmu"), "dmu", torch.float32, q.shape[0] * q.shape[2], required=False)
+
+
 def make_desc(B, T, H, dk, dv, dtype, *, chunk=0, mu=None, scale=None,
               decay_per_channel=1, out_dtype=KDN_F32, gates=KDN_GATES_POST,
               r_min=R_MIN_DEFAULT) -> kdn_desc_t:
@@ -154,11 +222,15 @@ def alloc_workspace(desc, variant, backward=False, device=None):
 def _fwd(name, variant, q, k, v, g, omega, r, S0, p0, *, chunk, mu, scale, o, ST, pT,
          want_state, workspace, stream, out_dtype,
          gates=KDN_GATES_POST, r_min=R_MIN_DEFAULT):
+    _check_inputs(variant, q, k, v, g, omega, r)
     desc = _desc_from(variant, q, v, g, chunk=chunk, mu=mu, scale=scale, out_dtype=out_dtype,
                       gates=gates, r_min=r_min)
     B, T, H, dk = q.shape
     dv = v.shape[-1]
     dev = q.device
+    ns, np_ = _state_sizes(variant, q, v)
+    _arg(S0, "S0", torch.float32, ns, required=False)
+    _arg(p0, "p0", torch.float32, np_, required=False)
     if o is None:
         o = torch.empty(B, T, H, dv, dtype=out_dtype, device=dev)
     if want_state and ST is None:
@@ -167,6 +239,10 @@ def _fwd(name, variant, q, k, v, g, omega, r, S0, p0, *, chunk, mu, scale, o, ST
         pT = torch.empty((B, H, dk) if variant == 0 else (B, H), dtype=torch.float32, device=dev)
     if workspace is None:
         workspace = alloc_workspace(desc, variant, False, dev)
+    _arg(o, "o", _torch_dtype(out_dtype), B * T * H * dv)
+    _arg(ST, "ST", torch.float32, ns, required=False)
+    _arg(pT, "pT", torch.float32, np_, required=False)
+    _arg(workspace, "workspace", torch.uint8)
     st = getattr(lib(), name)(ctypes.byref(desc), _ptr(q), _ptr(k), _ptr(v), _ptr(g),
                               _ptr(omega), _ptr(r), _ptr(S0), _ptr(p0), _ptr(o), _ptr(ST),
                               _ptr(pT), _ptr(workspace), workspace.numel(), _stream(stream))
@@ -199,11 +275,15 @@ def kdn_iso_fwd(q, k, v, g, omega, r, S0=None, p0=None, *, chunk=0, mu=None, sca
 def _bwd(name, variant, q, k, v, g, omega, r, S0, p0, dO, dST, dpT, *, chunk, mu, scale,
          grads, want_state_grads, workspace, stream, out_dtype,
          gates=KDN_GATES_POST, r_min=R_MIN_DEFAULT):
+    _check_inputs(variant, q, k, v, g, omega, r, dO)
     desc = _desc_from(variant, q, v, g, chunk=chunk, mu=mu, scale=scale, out_dtype=out_dtype,
                       gates=gates, r_min=r_min)
     B, T, H, dk = q.shape
     dv = v.shape[-1]
     dev = q.device
+    ns, np_ = _state_sizes(variant, q, v)
+    for t, n, m in ((S0, "S0", ns), (p0, "p0", np_), (dST, "dST", ns), (dpT, "dpT", np_)):
+        _arg(t, n, torch.float32, m, required=False)
     if grads is None:
         grads = {n: torch.empty(x.shape, dtype=out_dtype, device=dev) for n, x in
                  (("dq", q), ("dk", k), ("dv", v), ("dg", g), ("domega", omega), ("dr", r))}
@@ -215,6 +295,8 @@ def _bwd(name, variant, q, k, v, g, omega, r, S0, p0, dO, dST, dpT, *, chunk, mu
     if workspace is None:
         workspace = alloc_workspace(desc, variant, True, dev)
     G = grads
+    _check_grads(G, q, k, v, g, omega, r, out_dtype, ns, np_)
+    _arg(workspace, "workspace", torch.uint8)
     st = getattr(lib(), name)(ctypes.byref(desc), _ptr(q), _ptr(k), _ptr(v), _ptr(g),
                               _ptr(omega), _ptr(r), _ptr(S0), _ptr(p0), _ptr(dO), _ptr(dST),
                               _ptr(dpT), _ptr(G["dq"]), _ptr(G["dk"]), _ptr(G["dv"]),
@@ -257,11 +339,15 @@ def saved_bytes(desc: kdn_desc_t, variant: int = 0) -> int:
 def _fwd_save(name, variant, q, k, v, g, omega, r, S0, p0, *, mu, scale, o, ST, pT, saved,
               want_state, workspace, stream, out_dtype,
               gates=KDN_GATES_POST, r_min=R_MIN_DEFAULT):
+    _check_inputs(variant, q, k, v, g, omega, r)
     desc = _desc_from(variant, q, v, g, chunk=0, mu=mu, scale=scale, out_dtype=out_dtype,
                       gates=gates, r_min=r_min)
     B, T, H, dk = q.shape
     dv = v.shape[-1]
     dev = q.device
+    ns, np_ = _state_sizes(variant, q, v)
+    _arg(S0, "S0", torch.float32, ns, required=False)
+    _arg(p0, "p0", torch.float32, np_, required=False)
     if o is None:
         o = torch.empty(B, T, H, dv, dtype=out_dtype, device=dev)
     if want_state and ST is None:
@@ -272,6 +358,11 @@ def _fwd_save(name, variant, q, k, v, g, omega, r, S0, p0, *, mu, scale, o, ST, 
         saved = torch.empty(max(saved_bytes(desc, variant), 256), dtype=torch.uint8, device=dev)
     if workspace is None:
         workspace = alloc_workspace(desc, variant, False, dev)
+    _arg(o, "o", _torch_dtype(out_dtype), B * T * H * dv)
+    _arg(ST, "ST", torch.float32, ns, required=False)
+    _arg(pT, "pT", torch.float32, np_, required=False)
+    _arg(saved, "saved", torch.uint8)
+    _arg(workspace, "workspace", torch.uint8)
     st = getattr(lib(), name)(ctypes.byref(desc), _ptr(q), _ptr(k), _ptr(v), _ptr(g),
                               _ptr(omega), _ptr(r), _ptr(S0), _ptr(p0), _ptr(o), _ptr(ST),
                               _ptr(pT), _ptr(saved), saved.numel(), _ptr(workspace),
@@ -306,11 +397,16 @@ def kdn_iso_fwd_save(q, k, v, g, omega, r, S0=None, p0=None, *, mu=None, scale=N
 def _bwd_saved(name, variant, q, k, v, g, omega, r, saved, dO, dST, dpT, *, mu, scale, grads,
                want_state_grads, workspace, stream, out_dtype,
                gates=KDN_GATES_POST, r_min=R_MIN_DEFAULT):
+    _check_inputs(variant, q, k, v, g, omega, r, dO)
     desc = _desc_from(variant, q, v, g, chunk=0, mu=mu, scale=scale, out_dtype=out_dtype,
                       gates=gates, r_min=r_min)
     B, T, H, dk = q.shape
     dv = v.shape[-1]
     dev = q.device
+    ns, np_ = _state_sizes(variant, q, v)
+    _arg(saved, "saved", torch.uint8)
+    _arg(dST, "dST", torch.float32, ns, required=False)
+    _arg(dpT, "dpT", torch.float32, np_, required=False)
     if grads is None:
         grads = {n: torch.empty(x.shape, dtype=out_dtype, device=dev) for n, x in
                  (("dq", q), ("dk", k), ("dv", v), ("dg", g), ("domega", omega), ("dr", r))}
@@ -322,6 +418,8 @@ def _bwd_saved(name, variant, q, k, v, g, omega, r, saved, dO, dST, dpT, *, mu, 
     if workspace is None:
         workspace = alloc_workspace(desc, variant, False, dev)
     G = grads
+    _check_grads(G, q, k, v, g, omega, r, out_dtype, ns, np_)
+    _arg(workspace, "workspace", torch.uint8)
     st = getattr(lib(), name)(ctypes.byref(desc), _ptr(q), _ptr(k), _ptr(v), _ptr(g),
                               _ptr(omega), _ptr(r), _ptr(saved), saved.numel(), _ptr(dO),
                               _ptr(dST), _ptr(dpT), _ptr(G["dq"]), _ptr(G["dk"]),
@@ -359,8 +457,12 @@ def _beta_eff(name, variant, k, v, g, r, saved, *, out, stream, gates, r_min):
     desc = _desc_from(variant, k, v, g, chunk=0, mu=None, scale=None, out_dtype=torch.float32,
                       gates=gates, r_min=r_min)
     B, T, H, _ = k.shape
+    _arg(k, "k")
+    _arg(saved, "saved", torch.uint8)
+    _arg(r, "r", k.dtype, B * T * H)
     if out is None:
         out = torch.empty(B, T, H, dtype=torch.float32, device=k.device)
+    _arg(out, "out", torch.float32, B * T * H)
     st = getattr(lib(), name)(ctypes.byref(desc), _ptr(saved), ctypes.c_size_t(saved.numel()),
                               _ptr(r), _ptr(out), _stream(stream))
     _check(st, name)
@@ -384,14 +486,19 @@ def kdn_iso_beta_eff(k, v, g, r, saved, *, out=None, stream=None, gates=KDN_GATE
 
 def _decode(name, variant, q, k, v, g, omega, r, S, p, *, mu, scale, o, stream, out_dtype,
             gates=KDN_GATES_POST, r_min=R_MIN_DEFAULT):
+    _check_inputs(variant, q, k, v, g, omega, r, tokens=False)
     B, H, dk = q.shape
     dv = v.shape[-1]
     pcd = 1 if variant == 0 else int(g.dim() == 3)
     desc = make_desc(B, 1, H, dk, dv, q.dtype, mu=mu, scale=scale, decay_per_channel=pcd,
                      out_dtype=out_dtype,
         gates=gates, r_min=r_min)
+    ns, np_ = _state_sizes(variant, q, v, tokens=False)
+    _arg(S, "S", torch.float32, ns)
+    _arg(p, "p", torch.float32, np_)
     if o is None:
         o = torch.empty(B, H, dv, dtype=out_dtype, device=q.device)
+    _arg(o, "o", _torch_dtype(out_dtype), B * H * dv)
     st = getattr(lib(), name)(ctypes.byref(desc), _ptr(q), _ptr(k), _ptr(v), _ptr(g),
                               _ptr(omega), _ptr(r), _ptr(S), _ptr(p), _ptr(o), _stream(stream))
     _check(st, name)
@@ -423,8 +530,15 @@ def kdn_diag_fwd_noalloc(q, k, v, g, omega, r, S0=None, p0=None, *, o, ST=None, 
     fixed scratch array instead of a workspace, for callers that may not
     allocate device memory.  Problems needing more than
     KDN_NOALLOC_SCRATCH_BYTES of scratch are rejected.  Returns o."""
+    _check_inputs(0, q, k, v, g, omega, r)
+    _arg(o, "o")
     desc = _desc_from(0, q, v, g, chunk=0, mu=mu, scale=scale, out_dtype=o.dtype, gates=gates,
                       r_min=r_min)
+    B, T, H, dk = q.shape
+    ns, np_ = _state_sizes(0, q, v)
+    _arg(o, "o", None, B * T * H * v.shape[-1])
+    for t, n, m in ((S0, "S0", ns), (p0, "p0", np_), (ST, "ST", ns), (pT, "pT", np_)):
+        _arg(t, n, torch.float32, m, required=False)
     st = lib().kdn_diag_fwd_noalloc(ctypes.byref(desc), _ptr(q), _ptr(k), _ptr(v), _ptr(g),
                                     _ptr(omega), _ptr(r), _ptr(S0), _ptr(p0), _ptr(o), _ptr(ST),
                                     _ptr(pT), _stream(stream))
@@ -440,10 +554,12 @@ def kdn_kernel_launches(desc: kdn_desc_t, variant: int, op: int) -> int:
 def kdn_selftest_wait_timeout(workspace, stream=None) -> int:
     """Runs the device self-test of the bounded waits on ``workspace`` (asynchronous);
     kdn_get_device_status then reports KDN_ERR_TIMEOUT."""
+    _arg(workspace, "workspace")
     return int(lib().kdn_selftest_wait_timeout(_ptr(workspace), _stream(stream)))
 
 
 def kdn_get_device_status(workspace, stream=None) -> int:
+    _arg(workspace, "workspace")
     return int(lib().kdn_get_device_status(_ptr(workspace), _stream(stream)))
 
 

@@ -34,7 +34,7 @@ def _worker(rank, world, port, out):
 
 def test_two_ranks_max_time_and_job_throughput():
     world, port = 2, _free_port()
-    out = mp.Manager().dict()
+    out = mp.get_context("spawn").Manager().dict()  # no fork of a threaded process
     mp.spawn(_worker, args=(world, port, out), nprocs=world, join=True)
     for rank in range(world):
         m, v = out[rank]
