@@ -2,9 +2,11 @@
 
 Thin Python binding of ``libkdn.so`` (C ABI in ``include/kdn.h``).  The
 functions below carry the C entry points' names and only marshal arguments:
-they allocate outputs and the scratch workspace with PyTorch (device memory is
-PyTorch's job here), pass raw pointers and the current CUDA stream, and raise
-on any non-OK status.  Every step of the computation runs in the library's
+they check that every tensor is what the C ABI reads through its pointer (a
+contiguous CUDA tensor of the expected dtype and element count), allocate
+outputs and the scratch workspace with PyTorch (device memory is PyTorch's job
+here), pass raw pointers and the current CUDA stream, and raise on any non-OK
+status.  Every step of the computation runs in the library's
 CUDA kernels; there is no CPU or PyTorch fallback, and importing a function
 whose library is missing raises.
 
