@@ -56,7 +56,10 @@
  *              tensor cores with tf32 and fp16 operands (Sec. 4.2 products,
  *              float32 accumulators).
  *   Sizes      dk, dv in {32, 64, 128}; T >= 0 (any length; a ragged last
- *              chunk is padded with identity tokens); B, H >= 0.
+ *              chunk is padded with identity tokens); B, H >= 0.  At most
+ *              T = 2^21 tokens, B*H = 65535*1024 sequences and B*T*H =
+ *              2^31 - 1 token-heads per call; larger problems return
+ *              KDN_ERR_UNSUPPORTED (split them over calls).
  */
 #ifndef KDN_H
 #define KDN_H

@@ -98,6 +98,21 @@ def test_rejects_bad_descriptors_before_launch(kdn):
     assert kdn.workspace_bytes(d, 0) > 0
 
 
+def test_size_limits(kdn):
+    """The largest problems a call takes (T = 2^21, B*T*H = 2^31 - 1 token-heads)
+    get a workspace size; one token or sequence more is refused as unsupported,
+    before any CUDA call.  No call here launches anything."""
+    ok = [(1, 1 << 21, 1), (1023, 1 << 21, 1), (2, 1 << 20, 1023)]
+    over = [(1, (1 << 21) + 1, 1), (1024, 1 << 21, 1), (1 << 16, 1, 1 << 10)]
+    for B, T, H in ok:
+        assert B * T * H <= (1 << 31) - 1
+        assert kdn.workspace_bytes(kdn.make_desc(B, T, H, 32, 32, kdn.KDN_F32), 0) > 0
+    for B, T, H in over:
+        d = kdn.make_desc(B, T, H, 32, 32, kdn.KDN_F32)
+        assert kdn.workspace_bytes(d, 0) == 0
+        assert _fwd(kdn, d) == kdn.KDN_ERR_UNSUPPORTED
+
+
 def test_rejects_null_and_misaligned_pointers(kdn):
     d = kdn.make_desc(1, 10, 1, 32, 32, kdn.KDN_F32)
     for i in range(7):  # q, k, v, g, omega, r are required; S0, p0 optional; o required
