@@ -14,7 +14,10 @@ tensor-core operand to the type the kernel stores it in:
 Against the fp64 oracle at the workload's input distribution, the modelled
 error shows the margin of these choices under the bf16-input rule
 (max |err| <= 2e-2 RMS), and what single bf16 operands of MMA-T would give
-instead.  Nothing here runs on, or is shared with, the CUDA path.
+instead.  The same is done for the first fused forward (the Isotropic KDN with
+per-channel decay and the sequence-parallel segments), whose MMA-T runs on
+hi + lo bf16 pairs referenced at the chunk start.  Nothing here runs on, or is
+shared with, the CUDA path.
 """
 import numpy as np
 import pytest
