@@ -28,9 +28,10 @@
 // error reaches ~3% of RMS(o); with this split it stays below ~0.5%.
 //
 // Limits of this kernel: bf16 inputs, dk = dv = 128, per-chunk cumulative
-// log-decay above about -80 in every channel (exp(-G) must stay finite in
-// fp32; with alpha = sigmoid(x) that needs an average alpha > 0.29 over a
-// 64-token chunk).  Every wait on an mbarrier is bounded; on timeout the
+// decay exp(G_C) >= 1e-36 (G_C >= -82.8) in every channel, so that 1/gamma
+// stays a normal fp32 number; that is an average alpha above 0.27 over a
+// 64-token chunk.  A chunk below it is recorded as KDN_ERR_RANGE in the
+// workspace status word.  Every wait on an mbarrier is bounded; on timeout the
 // kernel records KDN_ERR_TIMEOUT in the workspace status word and returns.
 //
 // Instantiations (template <V, G, SD, PH>, described at the kernel): the
