@@ -3,9 +3,11 @@
 // on the tcgen05 tensor cores of sm_103a.
 //
 // Two launches:
-//  1. the fused forward in its state-saving mode stores, per chunk, the fp16
-//     image of the entry memory S_in (the tile MMA-S1 consumes) and the
-//     uncertainty p entering the chunk;
+//  1. a fused forward in its context-saving mode (the training forward, or the
+//     first pass of kdn_*_bwd) stores, per chunk, the 16-bit tiles it formed
+//     and multiplied with -- S_in, R, -W, A_qk, A and, for the Diagonal KDN,
+//     Y = V - Kbar S_in -- with phat and gamma in fp32, the per-token gain
+//     scalars and the uncertainty p entering the chunk;
 //  2. k_fused_bwd: one CTA per (batch, head) walks the chunks backwards.  The
 //     memory cotangent dS (128 x 128 fp32) stays in tensor memory for the whole
 //     sweep; the uncertainty cotangent dp (one value per channel) is carried in
@@ -20,6 +22,8 @@
 //   dW     = -dR S_in^T,     dV = A^T dR                (B5, B7)
 //   dQbar  = dO S_in^T + dA_qk Kk                       (B8)
 //   dA     = dR V^T + dW Kbar^T,  dT = strict_lower(-A^T dA A^T)   (B6, X, Y)
+//            (the Diagonal KDN forms dA = dR Y^T, the same matrix since
+//            dW = -dR S_in^T and Y = V - Kbar S_in)
 //   dKk    = dA_qk^T Qbar + gamma_C.dK_tail + dT^T Kbar (B9)
 //   dKbar  = A^T dW + dT Kk                             (B10)
 //   dgamma_C = colsum(dK_tail.Kk) + rowsum(dS.S_in)
