@@ -18,9 +18,12 @@ parity tests only measure rounding:
     strict_lower(T'); R = A (V - Kbar S_in); outputs and state from
     R' = diag(1/s) R and the unnormalised A'_qk and K'.
 
-The last test does the same for the backward: the chunk adjoint of the fused
-backward (its stages B1-B10 and the scalings by Gamma), then the gain adjoint
-token by token, against the oracle's gradients.
+The same is done for the backward (the chunk adjoint of the fused backward,
+its stages B1-B10 and the scalings by Gamma, then the gain adjoint token by
+token, against the oracle's gradients) and for the join of the
+sequence-parallel forward (a two-level scan of Moebius summaries for the
+uncertainty entering each segment; per segment the memory from 0 and the
+transition Phi; S_in(j+1) = Phi_j S_in(j) + Sv_j).
 
 Nothing here runs on, or is shared with, the CUDA path.
 """
@@ -418,3 +421,106 @@ def test_chunk_adjoint_equals_token_loop_adjoint(case):
         for n in ("dq", "dk", "dv", "dg", "domega", "dr", "dS0", "dp0"):
             want = ref[n][0, :, h] if ref[n].ndim >= 3 and n not in ("dS0", "dp0") else ref[n][0, h]
             assert _rel(got[n].reshape(np.shape(want)), np.asarray(want)) <= TOL, n
+
+
+# ---------------------------------------------------------------------------
+# the sequence-parallel forward: segments joined exactly
+
+def token_matrices(variant, k, g, omega, r, mu):
+    """The Moebius matrices M_t [T, P, 2, 2] of the uncertainty update."""
+    T, dk = k.shape
+    if variant == "diag":
+        a, u, w = np.exp(2.0 * g), mu * k * k / r[:, None], omega
+    else:
+        a = (np.mean(np.exp(2.0 * g), axis=1) if g.ndim == 2 else np.exp(2.0 * g))[:, None]
+        u, w = (mu * np.sum(k * k, axis=1) / (dk * r))[:, None], omega[:, None]
+    M = np.empty((T,) + a.shape[1:] + (2, 2))
+    M[..., 0, 0], M[..., 0, 1], M[..., 1, 0], M[..., 1, 1] = a, w, u * a, 1.0 + u * w
+    return M
+
+
+def segmented_forward(variant, x, mu, tau, P, C=64, join=True):
+    """o, S_T, p_T of one sequence cut into P segments of whole chunks, as the
+    sequence-parallel forward joins them:
+      * level 1: each chunk's Moebius summary, and each segment's product of its
+        chunk summaries (neither depends on p_0);
+      * level 2: the exclusive scan of the segment products from z_0 = [p_0, 1]
+        gives the uncertainty entering each segment, from which every segment
+        replays its gains;
+      * per segment, with the gains fixed: the memory from S_in = 0 with v (exit
+        Sv_j, outputs o_v) and the transition Phi_j from S_in = I with v = 0
+        (outputs o_Phi = tau Phi_t^T q_t);
+      * the join S_in(j+1) = Phi_j S_in(j) + Sv_j, o_t = o_v,t + S_in(j)^T o_Phi,t.
+    ``join`` = False runs every segment on its own from S = 0 and p = 1."""
+    q, k, v, g, omega, r = (x[n] for n in ("q", "k", "v", "g", "omega", "r"))
+    T, dk = k.shape
+    nc = -(-T // C)
+    assert nc % P == 0
+    seg = (nc // P) * C
+    segs = [slice(j * seg, min((j + 1) * seg, T)) for j in range(P)]
+    G = g if g.ndim == 2 else np.repeat(g[:, None], dk, axis=1)
+    M = token_matrices(variant, k, g, omega, r, mu)
+    Pn = M.shape[1]
+    # level 1: chunk summaries, then segment products (later chunks on the left)
+    seg_prod = []
+    for sl in segs:
+        prod = np.broadcast_to(np.eye(2), (Pn, 2, 2)).copy()
+        for c0 in range(sl.start, sl.stop, C):
+            summ = np.broadcast_to(np.eye(2), (Pn, 2, 2)).copy()
+            for t in range(c0, min(c0 + C, T)):
+                summ = _renorm(np.einsum("pij,pjk->pik", M[t], summ))
+            prod = _renorm(np.einsum("pij,pjk->pik", summ, prod))
+        seg_prod.append(prod)
+    # level 2: exclusive scan of the segment products from z_0
+    p0 = x["p0"] if join else np.ones_like(x["p0"])
+    z = np.stack([np.broadcast_to(p0, (Pn,)), np.ones(Pn)], axis=1)
+    p_in = []
+    for prod in seg_prod:
+        p_in.append(z[:, 0] / z[:, 1] if join else np.ones(Pn))
+        z = _renorm(np.einsum("pij,pj->pi", prod, z))
+    p_T = z[:, 0] / z[:, 1]
+    kappa = np.empty_like(k)
+    for sl, pj in zip(segs, p_in):
+        kappa[sl], _, _ = gain_chunked(variant, k[sl], g[sl], omega[sl], r[sl], pj, mu, C)
+    # per segment: the memory from 0 and the transition from I
+    o_v, o_phi, Sv, Phi = np.empty((T, v.shape[1])), np.empty((T, dk)), [], []
+    for sl in segs:
+        S, F = np.zeros((dk, v.shape[1])), np.eye(dk)
+        for t in range(sl.start, sl.stop):
+            a = np.exp(G[t])
+            Sh, Fh = a[:, None] * S, a[:, None] * F
+            S = Sh + np.outer(kappa[t], v[t] - Sh.T @ k[t])
+            F = Fh - np.outer(kappa[t], Fh.T @ k[t])
+            o_v[t], o_phi[t] = tau * S.T @ q[t], tau * F.T @ q[t]
+        Sv.append(S)
+        Phi.append(F)
+    if not join:
+        return o_v, None, None
+    S_in = x["S0"]
+    o = np.empty_like(o_v)
+    for sl, Sj, Fj in zip(segs, Sv, Phi):
+        o[sl] = o_v[sl] + o_phi[sl] @ S_in
+        S_in = Fj @ S_in + Sj
+    return o, S_in, p_T
+
+
+@pytest.mark.parametrize("variant,pc", [("diag", True), ("iso", False), ("iso", True)])
+def test_sequence_parallel_join_equals_token_loop(variant, pc):
+    """The join of the sequence-parallel forward is exact: with decays near 1, so
+    that memory and uncertainty carry across whole segments, the joined result
+    equals the token loop to 1e-9 in fp64, and differs from the segments run on
+    their own by far more than rounding."""
+    T, dk, dv, P = 512, 16, 8, 4
+    ins = make_inputs(variant, 1, T, 1, dk, dv, dtype="f32", seed=17, per_channel_decay=pc,
+                      s0_std=0.5, p0_range=(0.5, 2.0))
+    ins["g"] = ins["g"] * 0.02          # alpha ~ 0.997: long memory
+    mu, tau = float(dk), dk ** -0.5
+    ref = oracle.fwd(variant, *[ins[n] for n in ("q", "k", "v", "g", "omega", "r")],
+                     ins["S0"], ins["p0"], mu=mu, scale=tau)
+    x = _seq(ins, 0, 0)
+    o, ST, pT = segmented_forward(variant, x, mu, tau, P)
+    assert _rel(o, ref["o"][0, :, 0]) <= TOL
+    assert _rel(ST, ref["ST"][0, 0]) <= TOL
+    assert _rel(pT, np.atleast_1d(ref["pT"][0, 0])) <= TOL
+    alone, _, _ = segmented_forward(variant, x, mu, tau, P, join=False)
+    assert _rel(alone, ref["o"][0, :, 0]) > 1e-2
